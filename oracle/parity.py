@@ -1,0 +1,77 @@
+"""Comparison helpers for GPU-vs-oracle parity (test infrastructure only).
+
+Tolerances (applied by the tests, stated here once):
+  * pooled scores: ||s_gpu - s||_inf / ||s||_inf <= 1e-3, and elementwise
+    relative error <= 1e-3 on the oracle's top-2t scores;
+  * anchor sets: identical, except that positions whose oracle score lies
+    within ``band`` (relative to the oracle's t-th largest score) of that
+    threshold may be exchanged for one another (a tie band);
+  * assignment (an argmax whose exact ties are frequent): where the oracle's
+    best and second-best similarities differ by more than ``tau`` the GPU
+    must agree; elsewhere the GPU's choice must be within ``tau`` of the best;
+  * C_k, C_v, held-out outputs: relative Frobenius error <= 2e-3;
+  * beta: relative l2 error <= 2e-3 over entries whose oracle w* exceeds
+    1e-6 max w*; on the remaining entries the GPU's beta must also sit at a
+    near-zero weight (beta <= log(1e-5 max w*)).
+"""
+from __future__ import annotations
+
+import numpy as np
+
+
+def rel_inf(a, b) -> float:
+    return float(np.max(np.abs(a - b)) / np.max(np.abs(b)))
+
+
+def rel_fro(a, b) -> float:
+    nb = float(np.linalg.norm(b))
+    return float(np.linalg.norm(a - b) / (nb if nb > 0 else 1.0))
+
+
+def score_errors(s_gpu: np.ndarray, s: np.ndarray, t: int):
+    """(inf-norm relative error, max elementwise relative error on the top-2t)."""
+    top = np.argsort(-s, kind="stable")[: min(len(s), 2 * t)]
+    return rel_inf(s_gpu, s), float(np.max(np.abs(s_gpu[top] - s[top]) / np.abs(s[top])))
+
+
+def anchors_match(S_gpu: np.ndarray, S: np.ndarray, s: np.ndarray, t: int, band: float):
+    """True if the anchor sets agree up to exchanges inside the tie band.
+    Returns (ok, number of exchanged positions, widest relative gap seen)."""
+    thr = np.sort(s)[::-1][t - 1]
+    a, b = set(map(int, S_gpu)), set(map(int, S))
+    diff = sorted(a ^ b)
+    if len(a) != len(b) or len(S_gpu) != t:
+        return False, len(diff), float("inf")
+    if not diff:
+        return True, 0, 0.0
+    gaps = [abs(s[j] - thr) / thr for j in diff]
+    return bool(max(gaps) <= band), len(diff), float(max(gaps))
+
+
+def assignment_valid(kappa_gpu: np.ndarray, sim: np.ndarray, S: np.ndarray, tau: float):
+    """Check a GPU assignment against the oracle's similarity table sim [T, t].
+    Returns (ok, n_decided_mismatch, n_tied_differences, worst shortfall)."""
+    T = sim.shape[0]
+    best = sim.max(axis=1)
+    srt = np.sort(sim, axis=1)
+    gap = srt[:, -1] - (srt[:, -2] if sim.shape[1] > 1 else -np.inf)
+    is_anchor = np.zeros(T, bool)
+    is_anchor[S] = True
+    got = sim[np.arange(T), kappa_gpu]
+    short = best - got
+    dec = (~is_anchor) & (gap > tau)
+    kappa_ref = np.argmax(sim, axis=1)
+    n_dec_mis = int(np.sum(dec & (kappa_gpu != kappa_ref)))
+    anchors_ok = bool(np.all(kappa_gpu[S] == np.arange(len(S))))
+    worst = float(np.max(np.where(is_anchor, 0.0, short)))
+    n_tie = int(np.sum((~is_anchor) & (~dec) & (kappa_gpu != kappa_ref)))
+    return (n_dec_mis == 0 and anchors_ok and worst <= tau), n_dec_mis, n_tie, worst
+
+
+def beta_errors(beta_gpu: np.ndarray, beta: np.ndarray, w_star: np.ndarray):
+    """(relative l2 error on the supported entries, ok flag for the rest)."""
+    wmax = float(np.max(w_star))
+    sup = w_star > 1e-6 * wmax
+    e = rel_fro(beta_gpu[sup], beta[sup]) if np.any(sup) else 0.0
+    rest_ok = bool(np.all(beta_gpu[~sup] <= np.log(max(1e-5 * wmax, 1e-300)) + 1e-6))
+    return e, rest_ok

@@ -1,0 +1,424 @@
+"""Pins of the fp64 oracle against what the paper and the mathematics fix.
+
+Each test checks the oracle against something other than itself: a number
+the paper prints, a closed form on constructed inputs, an invariant the
+paper states, or an independent textbook route (Householder QR least
+squares, explicit loops on tiny inputs).  No GPU is needed.
+"""
+from pathlib import Path
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+GOLDEN = Path(__file__).resolve().parent / "golden"
+SC = 1.0 / np.sqrt(128.0)
+
+
+def small_pair(T=48, n_pos=24, seed_head=0, d_x=64, zero_value_path=False):
+    w = synth.Workload("pin", 99, 1, 1, T, n_pos, max(1, T // 4), shape=synth.IndexerShape(d_x=d_x))
+    p = synth.make_pair(w, 0, seed_head)
+    X = synth.make_layer_activations(w, 0)
+    W = {k: synth.bf16_to_f64(v) for k, v in synth.make_indexer(w, 0, seed_head, zero_value_path).items()}
+    K, V, Q = (synth.bf16_to_f64(p[k]) for k in "KVQ")
+    return w, K, V, Q, np.repeat(synth.bf16_to_f64(X), w.G, axis=0), W
+
+
+# ---------------------------------------------------------------- indexer
+
+def test_indexer_param_count_matches_table7():
+    """Table 7 (App. C.2) prints the total indexer size per model."""
+    rows = [l.split() for l in (GOLDEN / "indexer_size_table7.txt").read_text().splitlines()
+            if l.strip() and not l.startswith("#")]
+    assert len(rows) == 3
+    for _, pairs, d, d_x, total in rows:
+        n = oracle.indexer_param_count(int(d), int(d_x)) * int(pairs)
+        assert round(n / 1e6) == int(total), (n, total)
+    assert oracle.indexer_param_count(128, 4096) == 606216
+
+
+def test_rms_normalize_closed_form():
+    z = np.zeros((3, 128))
+    z[0, 0] = np.sqrt(128.0) * 2.0      # ||z||^2 / d_I = 4
+    z[1, :] = 1.0                        # ||z||^2 / d_I = 1
+    out = oracle.rms_normalize(z, 128)
+    assert out[0, 0] == pytest.approx(np.sqrt(128.0) * 2.0 / np.sqrt(4.0 + 1e-6), rel=1e-15)
+    assert np.allclose(out[1], 1.0 / np.sqrt(1.0 + 1e-6), rtol=1e-15)
+    assert np.all(out[2] == 0.0)
+
+
+def test_value_context_uniform_and_one_hot():
+    rng = np.random.default_rng(0)
+    T, d = 7, 128
+    K, V, Q = rng.normal(size=(T, d)), rng.normal(size=(T, d)), rng.normal(size=(3, d))
+    Uv = rng.normal(size=(128, d))
+    # U_k = 0: every logit is 0, A^V is uniform, c_i = mean_j U_v v_j
+    A, c = oracle.value_context(Q, K, V, rng.normal(size=(128, d)), np.zeros((128, d)), Uv)
+    assert np.allclose(A, 1.0 / T, rtol=1e-14)
+    assert np.allclose(c, np.mean(V @ Uv.T, axis=0)[None, :], rtol=1e-12, atol=1e-12)
+    # identity projections and a key far along the query: A^V picks that key
+    Q1 = np.zeros((1, d)); Q1[0, 0] = 1.0
+    K1 = np.zeros((T, d)); K1[3, 0] = 1000.0
+    A, c = oracle.value_context(Q1, K1, V, np.eye(d), np.eye(d), np.eye(d))
+    assert A[0, 3] == pytest.approx(1.0, abs=1e-12)
+    assert np.allclose(c[0], V[3], atol=1e-9)
+
+
+def test_index_logit_closed_form_leaky_relu_and_scale():
+    """Eq. pairwise_index_score with L_q = L_k = I, no value path, w = b_x = 1:
+    I_ij = LeakyReLU_0.1(N(q).N(k)/sqrt(d_I)).  For q = k = +-sqrt(d_I) e_1 the
+    product is +-d_I/(1+1e-6), so I = sqrt(d_I)/(1+1e-6) or -0.1 of it."""
+    d, dI = 128, 128
+    W = {"U_q": np.zeros((128, d)), "U_k": np.zeros((128, d)), "U_v": np.zeros((128, d)),
+         "L_q": np.eye(dI, d), "L_k": np.eye(dI, d), "L_c": np.zeros((dI, 128)), "L_v": np.zeros((dI, d)),
+         "L_x": np.zeros((1, 16)), "b_x": np.ones(1)}
+    e = np.zeros(d); e[0] = np.sqrt(dI)
+    Q = np.stack([e, -e]); K = np.stack([e, -e, 2 * e])
+    V = np.zeros_like(K)
+    I = oracle.indexer_logits(Q, np.zeros((2, 16)), K, V, W, H_I=1, d_I=dI)
+    pos = np.sqrt(dI) / (1.0 + 1e-6)
+    # N(2 sqrt(d_I) e_1) = 2 sqrt(d_I) e_1 / sqrt(4 + 1e-6)
+    pos2 = 2.0 * dI / np.sqrt(1.0 + 1e-6) / np.sqrt(4.0 + 1e-6) / np.sqrt(dI)
+    expect = np.array([[pos, -0.1 * pos, pos2], [-0.1 * pos, pos, -0.1 * pos2]])
+    assert np.allclose(I, expect, rtol=1e-13)
+
+
+def test_index_weights_use_activation_of_the_rows_position():
+    """w_{i,a} = (L_x x_r + b_x)_a: with L_x = 0 the weights are b_x, so
+    scaling b_x scales I linearly."""
+    w, K, V, Q, Xr, W = small_pair()
+    W0 = dict(W, L_x=np.zeros_like(W["L_x"]))
+    W2 = dict(W0, b_x=3.0 * W0["b_x"])
+    I1 = oracle.indexer_logits(Q, Xr, K, V, W0)
+    I2 = oracle.indexer_logits(Q, Xr, K, V, W2)
+    assert np.allclose(I2, 3.0 * I1, rtol=1e-12, atol=1e-14)
+
+
+def test_indexer_is_value_independent_with_zero_value_path():
+    """App. A.1: with L_c = L_v = 0 the logits reproduce a query-key-only scorer."""
+    w, K, V, Q, Xr, W = small_pair(zero_value_path=True)
+    I1 = oracle.indexer_logits(Q, Xr, K, V, W)
+    I2 = oracle.indexer_logits(Q, Xr, K, np.random.default_rng(1).normal(size=V.shape), W)
+    assert np.array_equal(I1, I2)
+    w, K, V, Q, Xr, W = small_pair(zero_value_path=False)
+    I3 = oracle.indexer_logits(Q, Xr, K, V, W)
+    I4 = oracle.indexer_logits(Q, Xr, K, V + 1.0, W)
+    assert not np.allclose(I3, I4)
+
+
+def test_indexer_logits_explicit_loops_tiny():
+    """Eqs. value_context, indexer_projection, pairwise_index_score evaluated
+    element by element with Python loops on a tiny case."""
+    rng = np.random.default_rng(3)
+    T, n, d, HI, dI, dA, dx = 5, 3, 6, 2, 4, 3, 5
+    K, V, Q, X = rng.normal(size=(T, d)), rng.normal(size=(T, d)), rng.normal(size=(n, d)), rng.normal(size=(n, dx))
+    W = {"U_q": rng.normal(size=(dA, d)), "U_k": rng.normal(size=(dA, d)), "U_v": rng.normal(size=(dA, d)),
+         "L_q": rng.normal(size=(HI * dI, d)), "L_k": rng.normal(size=(HI * dI, d)),
+         "L_c": rng.normal(size=(HI * dI, dA)), "L_v": rng.normal(size=(HI * dI, d)),
+         "L_x": rng.normal(size=(HI, dx)), "b_x": rng.normal(size=HI)}
+    I = oracle.indexer_logits(Q, X, K, V, W, H_I=HI, d_I=dI)
+
+    def mv(M, x):
+        return [sum(M[r][c] * x[c] for c in range(len(x))) for r in range(len(M))]
+
+    for i in range(n):
+        vq = mv(W["U_q"], Q[i])
+        lg = [sum(a * b for a, b in zip(vq, mv(W["U_k"], K[j]))) for j in range(T)]
+        mx = max(lg)
+        ex = [np.exp(x - mx) for x in lg]
+        A = [e / sum(ex) for e in ex]
+        c = [sum(A[j] * mv(W["U_v"], V[j])[q] for j in range(T)) for q in range(dA)]
+        qz = [a + b for a, b in zip(mv(W["L_q"], Q[i]), mv(W["L_c"], c))]
+        wv = [x + b for x, b in zip(mv(W["L_x"], X[i]), W["b_x"])]
+        for j in range(T):
+            kz = [a + b for a, b in zip(mv(W["L_k"], K[j]), mv(W["L_v"], V[j]))]
+            tot = 0.0
+            for a in range(HI):
+                qa, ka = qz[a * dI:(a + 1) * dI], kz[a * dI:(a + 1) * dI]
+                nq = np.sqrt(sum(x * x for x in qa) / dI + 1e-6)
+                nk = np.sqrt(sum(x * x for x in ka) / dI + 1e-6)
+                x = sum((p / nq) * (q / nk) for p, q in zip(qa, ka)) / np.sqrt(dI)
+                tot += wv[a] * (x if x >= 0 else 0.1 * x)
+            assert I[i, j] == pytest.approx(tot, rel=1e-10, abs=1e-12)
+
+
+def test_pooling_invariants_and_closed_forms():
+    rng = np.random.default_rng(2)
+    I = rng.normal(size=(6, 40)) * 3
+    pi, s = oracle.indexer_pool(I)
+    assert np.allclose(pi.sum(axis=1), 1.0, rtol=1e-14)
+    assert np.all((s >= 0) & (s <= 1))
+    tot = np.sum(s ** 2)
+    assert 1.0 / 40 - 1e-15 <= tot <= 1.0 + 1e-15
+    # invariance to a per-row shift of the logits (softmax normalises rows)
+    _, s2 = oracle.indexer_pool(I + rng.normal(size=(6, 1)) * 50)
+    assert np.allclose(s2, s, rtol=1e-12)
+    # uniform logits -> s_j = 1/T; a single row -> s = pi
+    _, su = oracle.indexer_pool(np.zeros((4, 10)))
+    assert np.allclose(su, 0.1, rtol=1e-15)
+    p1, s1 = oracle.indexer_pool(I[:1])
+    assert np.allclose(s1, p1[0], rtol=1e-14)
+    # RMS, not mean: a position important to one query only keeps a large score
+    I2 = np.zeros((4, 10)); I2[0, 3] = 20.0
+    _, s3 = oracle.indexer_pool(I2)
+    assert np.argmax(s3) == 3 and s3[3] == pytest.approx(np.sqrt((1 / (1 + 9 * np.exp(-20))) ** 2 / 4 + 3 * 0.01 / 4),
+                                                         rel=1e-12)
+
+
+def test_top_t_brute_force_and_ties():
+    rng = np.random.default_rng(4)
+    for _ in range(20):
+        s = rng.integers(0, 5, size=30).astype(float)  # many exact ties
+        t = int(rng.integers(1, 31))
+        S = oracle.top_t(s, t)
+        # brute force: rank by (-score, position), take t, sort ascending
+        ranked = sorted(range(30), key=lambda j: (-s[j], j))
+        assert list(S) == sorted(ranked[:t])
+    assert list(oracle.top_t(np.array([1.0, 3.0, 3.0, 2.0]), 2)) == [1, 2]
+    assert list(oracle.top_t(np.array([1.0, 3.0, 3.0, 3.0]), 2)) == [1, 2]
+
+
+# ------------------------------------------------------- attention / merge
+
+def test_full_attention_two_keys_closed_form():
+    q = np.zeros((1, 128)); q[0, 0] = 2.0
+    K = np.zeros((2, 128)); K[0, 0] = 3.0; K[1, 0] = -1.0
+    V = np.zeros((2, 128)); V[0, 1] = 1.0; V[1, 1] = -1.0
+    P, O = oracle.full_attention(q, K, V, SC)
+    p0 = 1.0 / (1.0 + np.exp(SC * (-2.0 - 6.0)))
+    assert P[0, 0] == pytest.approx(p0, rel=1e-15)
+    assert O[0, 1] == pytest.approx(2 * p0 - 1, rel=1e-14)
+
+
+def test_response_profiles_unit_and_equal_to_literal_form():
+    rng = np.random.default_rng(5)
+    l = rng.normal(size=(8, 12)) * 10
+    u, M = oracle.response_profiles(l)
+    assert np.allclose(np.linalg.norm(u, axis=0), 1.0, rtol=1e-14)
+    assert np.array_equal(M, l.max(axis=0))
+    # on a logit range fp64 can represent, the per-column evaluation equals the
+    # printed global-shift form of Eq. (response_profile)
+    assert np.allclose(u, oracle.response_profiles_literal(l), rtol=1e-12, atol=1e-300)
+    lp = oracle.log_mass_weights(l)
+    assert np.allclose(np.exp(lp - l.max()), oracle.mass_weights_literal(l), rtol=1e-12)
+    # beyond fp64's range the literal form breaks down, the evaluated one does not
+    l2 = l.copy(); l2[:, 0] -= 2000.0
+    u2, _ = oracle.response_profiles(l2)
+    assert np.all(np.isfinite(u2)) and np.allclose(u2[:, 0], u[:, 0], rtol=1e-12)
+    assert np.all(np.isfinite(oracle.log_mass_weights(l2)))
+
+
+def test_assignment_closed_form_two_queries():
+    """Two queries along e_1, e_2 with scale 1: u_j is the normalised
+    (e^{k_j1}, e^{k_j2}) direction, so the most similar anchor is the one whose
+    difference k_1 - k_2 is closest (cosine is monotone in the angle)."""
+    Q = np.zeros((2, 128)); Q[0, 0] = 1.0; Q[1, 1] = 1.0
+    diffs = np.array([-3.0, -1.0, 0.0, 0.4, 2.0, 5.0, -0.9])
+    K = np.zeros((7, 128)); K[:, 0] = diffs
+    S = np.array([0, 2, 5])
+    u, _ = oracle.response_profiles(oracle.attention_logits(Q, K, 1.0))
+    kappa = oracle.assign_to_anchors(u, S)
+    ang = np.arctan2(1.0, np.exp(diffs))
+    want = [int(np.argmin(np.abs(ang[j] - ang[S]))) for j in range(7)]
+    assert list(kappa) == want
+    assert list(kappa[S]) == [0, 1, 2]
+
+
+def test_assignment_brute_force_cosine_table_and_ties():
+    w, K, V, Q, Xr, W = small_pair(T=40, n_pos=10)
+    l = oracle.attention_logits(Q, K, SC)
+    S = np.array([1, 5, 9, 20, 33])
+    kappa = oracle.assign_to_anchors(oracle.response_profiles(l)[0], S)
+    E = np.exp(l - l.max(axis=0, keepdims=True))  # per-column shift: same directions
+    for j in range(40):
+        if j in S:
+            assert kappa[j] == list(S).index(j)
+            continue
+        cos = [E[:, j] @ E[:, s] / np.linalg.norm(E[:, j]) / np.linalg.norm(E[:, s]) for s in S]
+        best = max(cos)
+        near = [r for r, c in enumerate(cos) if c >= best - 1e-12]
+        # rounding decides only among candidates equal to 1e-12; otherwise exact
+        assert kappa[j] in near
+        if len(near) == 1:
+            assert kappa[j] == near[0]
+    # exact tie (two anchors with identical keys): the smaller r wins
+    K2 = K.copy(); K2[9] = K2[5]
+    kappa2 = oracle.assign_to_anchors(oracle.response_profiles(oracle.attention_logits(Q, K2, SC))[0], S)
+    assert not np.any(kappa2[np.setdiff1d(np.arange(40), S)] == 2)
+
+
+def test_mass_centroid_closed_form_one_query():
+    """n = 1: phi_j proportional to e^{scale q.k_j}; the centroid of a two-key
+    group is the softmax-weighted mean of the two keys."""
+    q = np.zeros((1, 128)); q[0, 0] = 1.0
+    K = np.zeros((3, 128)); K[0, 0] = 2.0; K[1, 0] = 0.5; K[1, 1] = 3.0; K[2, 2] = 1.0
+    l = oracle.attention_logits(q, K, 1.0)
+    logphi = oracle.log_mass_weights(l)
+    assert np.allclose(logphi, l[0], rtol=1e-15)
+    kappa = np.array([0, 0, 1])
+    C, mu = oracle.merge_keys(K, kappa, logphi, np.array([0, 2]), lambda_m=1.0)
+    a, b = np.exp(2.0), np.exp(0.5)
+    assert np.allclose(mu[0], (a * K[0] + b * K[1]) / (a + b), rtol=1e-14)
+    assert np.allclose(mu[1], K[2])
+
+
+def test_merge_endpoints_identity_and_convex_hull():
+    w, K, V, Q, Xr, W = small_pair(T=48, n_pos=12)
+    l = oracle.attention_logits(Q, K, SC)
+    u, _ = oracle.response_profiles(l)
+    logphi = oracle.log_mass_weights(l)
+    S = oracle.top_t(np.random.default_rng(6).random(48), 9)
+    kappa = oracle.assign_to_anchors(u, S)
+    C0, _ = oracle.merge_keys(K, kappa, logphi, S, 0.0)
+    assert np.array_equal(C0, K[S])                        # lambda_m = 0 -> K_S
+    C1, mu = oracle.merge_keys(K, kappa, logphi, S, 1.0)
+    assert np.allclose(C1, mu, rtol=1e-15)                 # lambda_m = 1 -> mu
+    assert np.all(np.bincount(kappa, minlength=9) >= 1)    # groups are nonempty
+    lam = 0.37
+    C, _ = oracle.merge_keys(K, kappa, logphi, S, lam)
+    rng = np.random.default_rng(7)
+    qs = rng.normal(size=(50, 128)) * 3
+    for r in range(9):
+        G = np.flatnonzero(kappa == r)
+        pg = np.exp(logphi[G] - logphi[G].max())   # phi restricted to G_r, common factor removed
+        alpha = lam * pg / pg.sum() + (1 - lam) * (G == S[r])
+        assert np.all(alpha >= 0) and alpha.sum() == pytest.approx(1.0, rel=1e-14)
+        assert np.allclose(alpha @ K[G], C[r], rtol=1e-12, atol=1e-12)
+        lg = qs @ K[G].T
+        lc = qs @ C[r]
+        assert np.all(lc <= lg.max(axis=1) + 1e-9) and np.all(lc >= lg.min(axis=1) - 1e-9)
+    # identity: t = T makes every group a singleton, C_k = K for any lambda_m
+    St = np.arange(48)
+    kt = oracle.assign_to_anchors(u, St)
+    for lm in (0.0, 0.25, 0.5, 0.75, 1.0):
+        Ct, _ = oracle.merge_keys(K, kt, logphi, St, lm)
+        assert np.array_equal(Ct, K)
+
+
+# ------------------------------------------------------------------- fits
+
+def _stacked_qr_solve(A, b, lam):
+    """Textbook ridge least squares by Householder QR of [A; sqrt(lam) I]."""
+    t = A.shape[1]
+    M = np.vstack([A, np.sqrt(lam) * np.eye(t)])
+    rhs = np.concatenate([b, np.zeros((t,) + b.shape[1:])])
+    Qm, R = np.linalg.qr(M)
+    return np.linalg.solve(R, Qm.T @ rhs)
+
+
+def test_fit_beta_duplicate_keys_gives_log_multiplicity():
+    """Three copies of one key and one distinct key; anchors = one copy and
+    the distinct key.  Z_K = 3 e^{l_a} + e^{l_b} is matched exactly by w = (3, 1),
+    so beta = (log 3, 0) (ridge 0, n >= t)."""
+    rng = np.random.default_rng(8)
+    k = rng.normal(size=128); k2 = rng.normal(size=128)
+    K = np.stack([k, k, k, k2])
+    Q = rng.normal(size=(6, 128))
+    cfg = oracle.OracleConfig(t=2, ridge_w=0.0)
+    fb = oracle.fit_beta(Q, K, K[[0, 3]], cfg, SC)
+    assert np.allclose(fb["w_tilde"], [3.0, 1.0], rtol=1e-10)
+    assert np.allclose(fb["beta"], [np.log(3.0), 0.0], atol=1e-10)
+
+
+def test_fit_beta_identity_optimality_and_qr():
+    w, K, V, Q, Xr, W = small_pair(T=24, n_pos=12)       # n = 48 >= T
+    cfg = oracle.OracleConfig(t=24, ridge_w=0.0)
+    # a small logit scale keeps Phi_C well conditioned for the unregularised solve
+    fb = oracle.fit_beta(Q, K, K.copy(), cfg, 0.02)
+    assert np.allclose(fb["w_tilde"], 1.0, rtol=1e-6)      # t = T, C_k = K: w = 1, beta = 0
+    assert np.allclose(fb["beta"], 0.0, atol=1e-6)
+    S = np.array([0, 3, 7, 11, 19])
+    cfg = oracle.OracleConfig(t=5, ridge_w=1e-3)
+    fb = oracle.fit_beta(Q, K, K[S] * 0.9, cfg, SC)
+    A, m, wt = fb["Phi_C"], fb["m"], fb["w_tilde"]
+    G = A.T @ A
+    lam = 1e-3 * np.trace(G) / 5
+    grad = A.T @ (A @ wt - m) + lam * wt                     # normal-equation optimality
+    assert np.linalg.norm(grad) <= 1e-10 * np.linalg.norm(A.T @ m)
+    assert np.allclose(wt, _stacked_qr_solve(A, m, lam), rtol=1e-8, atol=1e-12)
+    # Phi_C entries are <= 1 when every compact key is a convex combination
+    assert np.all(A <= 1.0 + 1e-12)
+
+
+def test_fit_beta_projection_and_clip():
+    """w* = max(w~, 0) and beta = clip(log max(w*, eps_w)): a negative or
+    zero weight lands exactly on b_min when eps_w = e^{b_min}."""
+    w, K, V, Q, Xr, W = small_pair(T=30, n_pos=8)
+    cfg = oracle.OracleConfig(t=12, ridge_w=1e-6)
+    S = np.arange(0, 30, 30 // 12)[:12]
+    fb = oracle.fit_beta(Q, K, K[S], cfg, SC)
+    neg = fb["w_tilde"] <= 0
+    assert np.all(fb["w_star"][neg] == 0.0) and np.all(fb["beta"][neg] == -20.0)
+    pos = fb["w_tilde"] > np.exp(-20)
+    assert np.allclose(fb["beta"][pos], np.clip(np.log(fb["w_tilde"][pos]), -20, 20), rtol=1e-15)
+
+
+def test_fit_values_single_anchor_closed_form():
+    """t = 1: P^ is the all-ones column, so C_v = sum_i Y_i / (n + lam) with
+    lam = ridge * tr(P^T P)/t = ridge * n."""
+    w, K, V, Q, Xr, W = small_pair(T=20, n_pos=5)
+    cfg = oracle.OracleConfig(t=1, ridge_v=0.1)
+    fv = oracle.fit_values(Q, K, V, K[[4]], np.zeros(1), cfg, SC)
+    _, Y = oracle.full_attention(Q, K, V, SC)
+    assert np.allclose(fv["C_v"][0], Y.mean(axis=0) / 1.1, rtol=1e-12)
+
+
+def test_fit_values_identity_optimality_and_qr():
+    w, K, V, Q, Xr, W = small_pair(T=16, n_pos=12)
+    cfg = oracle.OracleConfig(t=16, ridge_v=0.0)
+    fv = oracle.fit_values(Q, K, V, K.copy(), np.zeros(16), cfg, 0.02)
+    assert np.allclose(fv["C_v"], V, rtol=1e-5, atol=1e-5)  # t = T: C_v = V
+    S = np.array([1, 4, 6, 10, 15])
+    cfg = oracle.OracleConfig(t=5, ridge_v=1e-2)
+    beta = np.array([0.3, -0.2, 1.0, 0.0, 0.5])
+    fv = oracle.fit_values(Q, K, V, K[S], beta, cfg, SC)
+    P, Y, C = fv["P_hat"], fv["Y"], fv["C_v"]
+    lam = 1e-2 * np.trace(P.T @ P) / 5
+    grad = P.T @ (P @ C - Y) + lam * C
+    assert np.linalg.norm(grad) <= 1e-10 * np.linalg.norm(P.T @ Y)
+    assert np.allclose(C, _stacked_qr_solve(P, Y, lam), rtol=1e-8, atol=1e-10)
+    assert np.allclose(P.sum(axis=1), 1.0, rtol=1e-14)
+
+
+def test_compact_attention_reduces_to_full_and_hard_subset():
+    w, K, V, Q, Xr, W = small_pair(T=32, n_pos=6)
+    _, O = oracle.full_attention(Q, K, V, SC)
+    assert np.allclose(oracle.compact_attention(Q, K, np.zeros(32), V, SC), O, rtol=1e-13)
+    S = np.array([2, 3, 17])
+    assert np.allclose(oracle.compact_attention(Q, K[S], np.zeros(3), V[S], SC),
+                       oracle.hard_subset_attention(Q, K, V, S, SC), rtol=1e-14)
+    # beta = log(multiplicity) makes one copy of a duplicated key act like all copies
+    K2 = np.vstack([K[:1], K[:1], K[1:]])
+    V2 = np.vstack([V[:1], V[:1], V[1:]])
+    _, O2 = oracle.full_attention(Q, K2, V2, SC)
+    b = np.zeros(32); b[0] = np.log(2.0)
+    assert np.allclose(oracle.compact_attention(Q, K, b, V, SC), O2, rtol=1e-12)
+
+
+def test_diagnostics():
+    y = np.array([[3.0, 4.0]])
+    assert oracle.output_loss(y * 1.1, y) == pytest.approx(0.01, rel=1e-12)
+    assert oracle.mass_error(np.eye(2), np.array([1.0, 2.0]), np.array([1.0, 2.0])) == 0.0
+
+
+def test_pipeline_identity_budget_reproduces_cache():
+    """t = T (every key is an anchor, all groups singletons): C_k = K exactly
+    for any lambda_m, and with ridge 0 and n >= T, beta = 0 and C_v = V."""
+    w, K, V, Q, Xr, W = small_pair(T=20, n_pos=12)
+    out = oracle.compact_pair(K, V, Q, Xr, W, oracle.OracleConfig(t=20, lambda_m=0.75, ridge_w=0.0, ridge_v=0.0,
+                                                                  scale=0.02))
+    assert list(out["anchors"]) == list(range(20))
+    assert np.array_equal(out["C_k"], K)
+    assert np.allclose(out["beta"], 0.0, atol=1e-6)
+    assert np.allclose(out["C_v"], V, rtol=1e-4, atol=1e-4)
+
+
+def test_pipeline_anchors_in_matches_scored_pipeline():
+    w, K, V, Q, Xr, W = small_pair(T=40, n_pos=10)
+    cfg = oracle.OracleConfig(t=8)
+    a = oracle.compact_pair(K, V, Q, Xr, W, cfg)
+    b = oracle.compact_pair(K, V, Q, Xr, W, cfg, anchors_in=a["anchors"])
+    for k in ("C_k", "beta", "C_v", "assign"):
+        assert np.array_equal(a[k], b[k])
