@@ -1,0 +1,421 @@
+#!/usr/bin/env python3
+"""Benchmark of ARC-KV per-context KV-cache compaction on GB300.
+
+A step is one pass of the whole compaction path over one synthetic context:
+every (layer, KV head) pair of a Llama-3.1-8B-shaped cache (32 layers x 8 KV
+heads, head dim 128, T = 8192 bf16 tokens, n_q = 1024 reference queries per
+KV head, t = 819 anchors = 10% retention), compacted layer by layer through
+arckv_compact.  The metric is context tokens per second (T / seconds per
+context); seconds per context are reported alongside.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gpu|reference]
+For N > 1 launch under torchrun; every rank compacts its own context
+(weak scaling) and rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import threading
+import time
+from pathlib import Path
+
+ROOT = Path(__file__).resolve().parent
+if str(ROOT) not in sys.path:
+    sys.path.insert(0, str(ROOT))
+
+METRIC = "compaction s/context and context tokens/s at Llama-3.1-8B shape; % roofline"
+UNIT = "context tokens/s"
+DEFAULT_WORKLOAD = "llama8b_T8192_r10"
+SM_COUNT, FP32_LANES_PER_SM = 152, 128
+PROFILE_SUMMARY = ROOT / "profiles" / "index_logits_llama8b_layer_T8192.md"
+DOMINANT_SOURCE = ROOT / "paper_2609_36835_gb300" / "csrc" / "indexer.cu"
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=("gpu", "reference"), default="gpu")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--cpu-pairs", type=int, default=4, help="(layer, head) pairs the oracle baseline times")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile-layer", action="store_true",
+                    help="compact layer 0 twice and exit (a small case for ncu captures)")
+    return ap.parse_args(argv)
+
+
+# ------------------------------------------------------------ distributed
+
+class Dist:
+    """Rank bookkeeping; a real process group only when WORLD_SIZE > 1."""
+
+    def __init__(self):
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+        self.pg = None
+
+    def init(self, backend: str):
+        if self.world > 1:
+            import torch.distributed as dist
+            os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+            dist.init_process_group(backend=backend)
+            self.pg = dist
+
+    def barrier(self):
+        if self.pg is not None:
+            self.pg.barrier()
+
+    def max(self, x: float, device="cpu") -> float:
+        if self.pg is None:
+            return x
+        import torch
+        t = torch.tensor([x], dtype=torch.float64, device=device)
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.pg is not None:
+            self.pg.destroy_process_group()
+
+
+def context_layers(layers: int, rank: int):
+    """Layer seeds of the context a rank compacts (weak scaling: each rank owns
+    one whole, distinct context of ``layers`` layers)."""
+    return [rank * layers + l for l in range(layers)]
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling in the background (-lms 200)."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.lines = []
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.Q,
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+            return
+        self.th = threading.Thread(target=self._read, daemon=True)
+        self.th.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.th.join(timeout=5)
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for l in self.lines:
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------- helpers
+
+def blas_threads() -> int:
+    """Threads the oracle's BLAS uses (OpenBLAS query when available)."""
+    try:
+        maps = Path("/proc/self/maps").read_text()
+        libs = sorted({l.split()[-1] for l in maps.splitlines() if "openblas" in l.lower() and ".so" in l})
+        for path in libs:
+            lib = ctypes.CDLL(path)
+            for sym in ("scipy_openblas_get_num_threads64_", "openblas_get_num_threads64_",
+                        "openblas_get_num_threads"):
+                fn = getattr(lib, sym, None)
+                if fn is not None:
+                    fn.restype = ctypes.c_int
+                    return int(fn())
+    except OSError:
+        pass
+    return len(os.sched_getaffinity(0))
+
+
+def oracle_pair_seconds(w, pairs):
+    """Time the fp64 oracle (as it stands) on (layer, head) pairs at full size."""
+    import numpy as np
+    import oracle
+    import synth
+    f64 = synth.bf16_to_f64
+    times = []
+    for (layer, head) in pairs:
+        p = synth.make_pair(w, layer, head)
+        X = synth.make_layer_activations(w, layer)
+        W = {k: f64(v) for k, v in synth.make_indexer(w, layer, head).items()}
+        K, V, Q = f64(p["K"]), f64(p["V"]), f64(p["Q"])
+        Xr = np.repeat(f64(X), w.G, axis=0)
+        t0 = time.perf_counter()
+        oracle.compact_pair(K, V, Q, Xr, W, oracle.OracleConfig(t=w.t))
+        times.append(time.perf_counter() - t0)
+    return times
+
+
+def profiled_traffic():
+    """dram bytes per launch of the dominant kernel from the committed ncu
+    summary, if it was taken on the current source of that kernel."""
+    if not PROFILE_SUMMARY.exists():
+        return None
+    text = PROFILE_SUMMARY.read_text()
+    m = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    h = re.search(r"source_sha256:\s*([0-9a-f]{64})", text)
+    if not m or not h:
+        return None
+    cur = hashlib.sha256(DOMINANT_SOURCE.read_bytes()).hexdigest()
+    return float(m.group(1)) if h.group(1) == cur else None
+
+
+# ------------------------------------------------------------ reference arm
+
+def run_reference(args, dist: Dist):
+    if dist.rank != 0:
+        return 0
+    import synth
+    w = synth.WORKLOADS[args.workload]
+    pairs = [(l, h) for l in range(w.layers) for h in range(w.H_kv)]
+    pick = [pairs[(i * 37) % len(pairs)] for i in range(args.warmup + args.steps)]
+    oracle_pair_seconds(w, pick[:args.warmup])
+    times = oracle_pair_seconds(w, pick[args.warmup:])
+    per_pair = statistics.mean(times)
+    s_ctx = per_pair * len(pairs)
+    value = w.T / s_ctx
+    cores = blas_threads()
+    sample = ("fp64 oracle on %d (layer, KV head) pairs of %s at full size, one pair per step; "
+              "seconds per context extrapolated x%d pairs" % (len(times), w.name, len(pairs)))
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_pair * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": workload_config(w, "none (CPU)"), "s_per_context": s_ctx,
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config(w, l2: str):
+    return {"workload": "%s: %d layers x %d KV heads (GQA %d), head_dim 128, T=%d bf16, n_q=%d per KV head, "
+                        "t=%d (%.0f%% retention), H_I=8, d_I=d_A=128, d_x=%d" %
+                        (w.name, w.layers, w.H_kv, w.G, w.T, w.n, w.t, 100.0 * w.t / w.T, w.shape.d_x),
+            "layers": w.layers, "kv_heads": w.H_kv, "T": w.T, "n_q": w.n, "t": w.t, "head_dim": 128,
+            "l2": l2}
+
+
+# ------------------------------------------------------------------ GPU arm
+
+def run_gpu(args, dist: Dist):
+    import numpy as np
+    import torch
+    import synth
+    import paper_2609_36835_gb300 as pk
+    from paper_2609_36835_gb300 import workload
+
+    dist.init("nccl")
+    dev = torch.device("cuda", dist.local_rank)
+    torch.cuda.set_device(dev)
+    pk.load_library()
+    w = synth.WORKLOADS[args.workload]
+    layers = context_layers(w.layers, dist.rank)
+    if args.profile_layer:
+        layers = layers[:1]
+    cfg = workload.layer_config(w, w.H_kv, flags=pk.FLAG_NONBLOCKING)
+    cfg_block = workload.layer_config(w, w.H_kv)
+
+    host = [workload.layer_inputs_np(w, l, list(range(w.H_kv))) for l in layers]
+    dev_in = [workload.to_device(a, dev) for a in host]
+    ws = torch.empty(pk.workspace_bytes(cfg), dtype=torch.uint8, device=dev)
+    f32 = dict(dtype=torch.float32, device=dev)
+    outs = [{"C_k": torch.empty(w.H_kv, w.t, 128, **f32), "beta": torch.empty(w.H_kv, w.t, **f32),
+             "C_v": torch.empty(w.H_kv, w.t, 128, **f32)} for _ in layers]
+    stream = torch.cuda.current_stream(dev)
+
+    def compact(i, events=None, c=cfg, ins=None, out=None):
+        t = ins if ins is not None else dev_in[i]
+        o = out if out is not None else outs[i]
+        st, nl = pk.arckv_compact(c, t["K"], t["V"], t["Q"], t["X"], workload.indexer_dict(t), o["C_k"],
+                                  o["beta"], o["C_v"], ws, ws.numel(), stream=stream, stage_events=events)
+        if st != 0:
+            raise pk.ArckvError(st, "arckv_compact")
+        return nl
+
+    if args.profile_layer:
+        compact(0, c=cfg_block)
+        compact(0, c=cfg_block)
+        torch.cuda.synchronize()
+        print("profile-layer done", flush=True)
+        return 0
+
+    # correctness of every layer once (blocking status read per call)
+    for i in range(len(layers)):
+        compact(i, c=cfg_block)
+
+    def new_events(k):
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(k)]
+        for e in evs:
+            e.record(stream)
+        return evs
+
+    for _ in range(args.warmup):
+        for i in range(len(layers)):
+            compact(i)
+    torch.cuda.synchronize()
+
+    n_ev = pk.NUM_STAGES + 1
+    ev_sets = [[new_events(n_ev) for _ in layers] for _ in range(args.steps)]
+    handles = [[[e.cuda_event for e in evs] for evs in step] for step in ev_sets]
+    t_start, t_end = new_events(2)
+    launches = 0
+    clocks = ClockSampler(dist.local_rank)
+    clocks.start()
+    time.sleep(0.3)
+    dist.barrier()
+    torch.cuda.synchronize()
+    t_start.record(stream)
+    for s in range(args.steps):
+        for i in range(len(layers)):
+            launches += compact(i, handles[s][i])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    dist.barrier()
+    clk = clocks.stop()
+    ms_total = t_start.elapsed_time(t_end)
+    ms_total = dist.max(ms_total, dev)
+    ms_step = ms_total / args.steps
+    # status of the timed calls: one blocking read
+    st = pk.arckv_query_status(ws, stream)
+    if st != 0:
+        raise pk.ArckvError(st, "timed region")
+
+    stage_ms = [[0.0] * pk.NUM_STAGES for _ in range(1)][0]
+    logits_ms = []
+    for s in range(args.steps):
+        for evs in ev_sets[s]:
+            for k in range(pk.NUM_STAGES):
+                stage_ms[k] += evs[k].elapsed_time(evs[k + 1])
+            logits_ms.append(evs[1].elapsed_time(evs[2]))
+    stage_ms = [x / args.steps for x in stage_ms]
+
+    # roofline of the dominant kernel (index logits, one launch per layer)
+    flops = 2.0 * w.H_kv * w.n * w.T * w.shape.H_I * w.shape.d_I
+    avg_s = statistics.mean(logits_ms) / 1e3
+    sm_max = 2070.0
+    peak_fp32 = SM_COUNT * FP32_LANES_PER_SM * 2 * sm_max * 1e6 / 1e12
+    achieved = flops / avg_s / 1e12
+    traffic = profiled_traffic()
+    roofline = {"kernel": "index_logits_kernel", "bound": "alu", "achieved": achieved, "peak": peak_fp32,
+                "unit": "TFLOP/s", "frac": achieved / peak_fp32, "traffic": traffic,
+                "flops_per_launch": flops, "launch_ms": avg_s * 1e3,
+                "peak_note": "fp32 FMA: 152 SMs x 128 lanes x 2 flop x 2070 MHz (derived, not measured)"}
+
+    # end to end: pinned host inputs -> device -> compaction -> host outputs, every step
+    pinned = [workload.to_device(a, pin=True) for a in host]
+    host_out = [{k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in o.items()} for o in outs]
+    h2d = sum(t.numel() * t.element_size() for p in pinned for t in p.values())
+    d2h = sum(t.numel() * t.element_size() for o in host_out for t in o.values())
+
+    def e2e_step():
+        for i in range(len(layers)):
+            for k, t in pinned[i].items():
+                dev_in[i][k].copy_(t, non_blocking=True)
+            compact(i)
+            for k, t in outs[i].items():
+                host_out[i][k].copy_(t, non_blocking=True)
+
+    e2e_step()
+    torch.cuda.synchronize()
+    e0, e1 = new_events(2)
+    dist.barrier()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = dist.max(e0.elapsed_time(e1), dev) / args.e2e_steps
+    if pk.arckv_query_status(ws, stream) != 0:
+        raise RuntimeError("e2e status")
+
+    value = dist.world * w.T / (ms_step / 1e3)
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded Llama-3.1-8B-shaped caches)",
+        "config": workload_config(w, "inputs larger than L2 (%.2f GB per context)" %
+                                  (h2d / 1e9)),
+        "s_per_context": ms_step / 1e3,
+        "stage_ms_per_step": dict(zip(pk.STAGE_NAMES, stage_ms)),
+        "gpu_launches": launches,
+        "roofline": roofline,
+        "e2e": {"value": dist.world * w.T / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "clocks": clk,
+    }
+    if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
+        spread = [(0, 0), (w.layers - 1, w.H_kv - 1), (w.layers // 2, 3 % w.H_kv), (w.layers // 4, 5 % w.H_kv)]
+        pairs = spread[:max(1, min(len(spread), args.cpu_pairs))]
+        times = oracle_pair_seconds(w, pairs)
+        per_pair = statistics.mean(times)
+        n_pairs = w.layers * w.H_kv
+        line["cpu_baseline"] = {
+            "value": w.T / (per_pair * n_pairs), "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+            "sample": "fp64 oracle on %d (layer, KV head) pairs at full size (%.1f s each), seconds per "
+                      "context extrapolated x%d pairs" % (len(times), per_pair, n_pairs)}
+    if dist.rank == 0:
+        print(json.dumps(line), flush=True)
+    dist.close()
+    return 0
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    if args.warmup < 3 and not args.profile_layer:
+        sys.stderr.write("note: fewer than 3 warm-up steps\n")
+    dist = Dist()
+    if args.impl == "reference":
+        return run_reference(args, dist)
+    return run_gpu(args, dist)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

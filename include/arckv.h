@@ -1,0 +1,187 @@
+/*
+ * arckv.h -- C ABI of the GB300 (sm_103a) ARC-KV per-context KV-cache
+ * compaction library (libarckv.so).
+ *
+ * ARC-KV (arXiv 2609.36835) compacts, for every (layer, KV head) pair, a full
+ * cache K, V in R^{T x d} into t entries (C_k, beta, C_v) such that the
+ * compact operator
+ *        O^(Q) = softmax(Q C_k^T + 1 beta^T) C_v           (Sec. 3.1, Eq. compact_attention)
+ * approximates full attention softmax(Q K^T) V.  One call of arckv_compact
+ * runs the four context-specific stages of Sec. 3.2 for all H_kv heads of one
+ * layer:
+ *   1. value-aware indexer scoring and top-t anchor selection
+ *        (Sec. 3.3; App. A.1 Eqs. value_context, indexer_projection,
+ *         pairwise_index_score; Sec. 3.3 Eq. indexer_pooling;
+ *         App. A.6 Eq. persistent_support),
+ *   2. response-profile assignment and convex-hull key merge
+ *        (Sec. 3.4 Eqs. response_profile, anchor_assignment, mass_centroid,
+ *         key_merge),
+ *   3. attention-mass fit of beta (App. A.9 Eq. mass_fit),
+ *   4. ridge fit of C_v (App. A.9 Eq. value_lstsq).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Pointers named in the signatures are DEVICE pointers on the current CUDA
+ *   device, owned by the caller; the library allocates no device or host
+ *   memory.  Scratch space is the caller's workspace `ws` of at least the
+ *   size returned by the matching *_workspace_bytes function, aligned to
+ *   256 bytes.
+ * - Arguments are checked on the host before anything is enqueued; a bad
+ *   argument returns ARCKV_ERR_INVALID_ARG / ARCKV_ERR_SHAPE /
+ *   ARCKV_ERR_WORKSPACE / ARCKV_ERR_UNSUPPORTED and enqueues nothing.
+ * - All kernels are enqueued on `stream` in order.  Errors found on the
+ *   device (a non-positive Cholesky pivot, a non-finite output) are recorded
+ *   in a status word inside the workspace.  Without ARCKV_FLAG_NONBLOCKING
+ *   the call synchronises `stream` and returns that status; with it the call
+ *   returns ARCKV_OK after enqueueing and the status is read later with
+ *   arckv_query_status (the call then performs no host synchronisation).
+ * - Calls are reentrant as long as concurrent calls use distinct workspaces.
+ * - bf16 means IEEE bfloat16 bit patterns (uint16); fp32 is IEEE binary32.
+ * - All tensors are dense row-major with the listed shapes.
+ */
+#ifndef ARCKV_H_
+#define ARCKV_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  ARCKV_OK = 0,
+  ARCKV_ERR_INVALID_ARG = 1, /* null pointer, bad flag, bad scalar      */
+  ARCKV_ERR_SHAPE = 2,       /* sizes out of range (e.g. t > T)         */
+  ARCKV_ERR_WORKSPACE = 3,   /* workspace null, too small or misaligned */
+  ARCKV_ERR_NOT_SPD = 4,     /* a fit's normal matrix lost definiteness */
+  ARCKV_ERR_NONFINITE = 5,   /* NaN / Inf produced (or present in input)*/
+  ARCKV_ERR_TIMEOUT = 6,     /* a bounded device wait gave up           */
+  ARCKV_ERR_CUDA = 7,        /* a CUDA runtime call failed              */
+  ARCKV_ERR_UNSUPPORTED = 8  /* valid but not implemented configuration */
+} arckv_status;
+
+/* Flags (arckv_config.flags). */
+#define ARCKV_FLAG_NONBLOCKING 0x1u /* do not synchronise; see arckv_query_status */
+
+/*
+ * Problem description for one layer.  Sizes:
+ *   H_kv  KV heads in the layer (>= 1)
+ *   G     query heads per KV head (GQA group size, >= 1)
+ *   T     cache length (>= 1)
+ *   d     head dim (must be 128)
+ *   n_pos reference positions; each KV head gets n = n_pos * G reference rows
+ *   d_x   reference-activation width (multiple of 8)
+ *   H_I   index heads (1..16), d_I index-head width (must be 128),
+ *   d_A   value-attention width (must be 128)                       (App. A.1)
+ *   t     anchors per head, 1 <= t <= T                             (Sec. 3.1)
+ *   chunk_len  0 = global top-t (the only mode implemented)          (App. A.3)
+ * Scalars:
+ *   lambda_m  key-merging coefficient in [0, 1]                      (Eq. key_merge)
+ *   logit_scale  factor on every model-attention logit q.k; the paper writes
+ *             logits without the usual 1/sqrt(d) (Sec. 3.1), which callers
+ *             pass here (0 selects 1/sqrt(d))
+ *   ridge_w, ridge_v  >= 0: the beta and C_v normal matrices are solved as
+ *             (Gram + lam I) with lam = ridge * trace(Gram) / t
+ *   eps_w > 0, b_min <= b_max: the guards of Eq. mass_fit
+ */
+typedef struct {
+  int32_t H_kv, G, T, d, n_pos, d_x, H_I, d_I, d_A, t, chunk_len;
+  float lambda_m, logit_scale, ridge_w, ridge_v, eps_w, b_min, b_max;
+  uint32_t flags;
+} arckv_config;
+
+/*
+ * Frozen indexer parameters of the H_kv heads of one layer, bf16, stacked
+ * over heads (App. A.1 Eqs. indexer_parameters, value_indexer_parameters):
+ *   L_q, L_k, L_v [H_kv][H_I*d_I][d]     L_c [H_kv][H_I*d_I][d_A]
+ *   L_x [H_kv][H_I][d_x]                 b_x [H_kv][H_I]
+ *   U_q, U_k, U_v [H_kv][d_A][d]
+ */
+typedef struct {
+  const void *L_q, *L_k, *L_x, *b_x, *U_q, *U_k, *U_v, *L_c, *L_v;
+} arckv_indexer;
+
+/* Number of timed stages reported through arckv_aux.stage_events. */
+#define ARCKV_NUM_STAGES 6
+/* Stage order: 0 indexer features (k_bar, value context, q_bar, w),
+ * 1 index logits (one kernel), 2 row log-sum-exp, RMS pooling and top-t,
+ * 3 reference attention and assignment, 4 merge, 5 beta and C_v fits.
+ * With anchors_in, stages 0-2 are empty. */
+
+/*
+ * Optional inputs / outputs of arckv_compact (the pointer itself may be NULL;
+ * every field may be NULL).
+ *   scores     out fp32 [H_kv][T]  pooled indexer scores s (Eq. indexer_pooling)
+ *   anchors    out int32 [H_kv][t] anchor positions S, ascending
+ *   assign     out int32 [H_kv][T] group index kappa(j) in [0, t)
+ *   anchors_in in  int32 [H_kv][t] strictly ascending positions in [0, T):
+ *              replaces indexer scoring and selection (the hard branch of
+ *              Sec. 3.5 and stage-isolated testing); `scores` is then not written
+ *   assign_in  in  int32 [H_kv][T] replaces the computed assignment; requires
+ *              anchors_in and must satisfy assign_in[s_r] = r
+ *   stage_events  cudaEvent_t[ARCKV_NUM_STAGES + 1] created by the caller; when
+ *              non-NULL, event s is recorded on `stream` before stage s and the
+ *              last one after the final stage
+ *   launches   out: number of kernels this call enqueued
+ */
+typedef struct {
+  float* scores;
+  int32_t* anchors;
+  int32_t* assign;
+  const int32_t* anchors_in;
+  const int32_t* assign_in;
+  void* const* stage_events;
+  int32_t* launches;
+} arckv_aux;
+
+/* Workspace bytes arckv_compact needs for `cfg` (0 if cfg is invalid).
+ * Host-only; no CUDA call. */
+size_t arckv_workspace_bytes(const arckv_config* cfg);
+
+/*
+ * Compact one layer (all H_kv heads).
+ *   K, V    bf16 [H_kv][T][d]         post-RoPE keys / values       (Sec. 3.1)
+ *   Q_ref   bf16 [H_kv][n_pos][G][d]  reference queries; row i = r*G + g of a
+ *                                     head pairs position r with query head g
+ *   X_ref   bf16 [n_pos][d_x]         pre-query-projection activations, shared
+ *                                     by the G rows of a position and by all
+ *                                     heads of the layer           (App. A.1, A.5)
+ *   idx     indexer weights (above)
+ *   C_k     out fp32 [H_kv][t][d]     compact keys (row r <-> r-th anchor)
+ *   beta    out fp32 [H_kv][t]        attention-mass bias
+ *   C_v     out fp32 [H_kv][t][d]     compact values
+ *   aux     optional (above)
+ *   ws, ws_bytes  workspace
+ *   stream  cudaStream_t (NULL = legacy default stream)
+ */
+arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V,
+                           const void* Q_ref, const void* X_ref, const arckv_indexer* idx,
+                           float* C_k, float* beta, float* C_v, const arckv_aux* aux,
+                           void* ws, size_t ws_bytes, void* stream);
+
+/* Workspace bytes of arckv_attend (0 if the sizes are invalid). Host-only. */
+size_t arckv_attend_workspace_bytes(int32_t H_kv, int32_t n, int32_t t, int32_t d);
+
+/*
+ * Attention against a compact cache (Sec. 3.1 Eq. compact_attention):
+ *   O[h] = softmax(logit_scale * Q[h] C_k[h]^T + 1 beta[h]^T) C_v[h]
+ *   Q bf16 [H_kv][n][d]; C_k, C_v fp32 [H_kv][t][d]; beta fp32 [H_kv][t];
+ *   O out fp32 [H_kv][n][d].  n >= 1, 1 <= t, d == 128.
+ * `flags` takes ARCKV_FLAG_NONBLOCKING.
+ */
+arckv_status arckv_attend(int32_t H_kv, int32_t n, int32_t t, int32_t d, float logit_scale,
+                          const void* Q, const float* C_k, const float* beta, const float* C_v,
+                          float* O, void* ws, size_t ws_bytes, uint32_t flags, void* stream);
+
+/* Read (and clear) the device status word of a workspace after a
+ * non-blocking call; synchronises `stream`. */
+arckv_status arckv_query_status(void* ws, void* stream);
+
+/* Static description of a status code (never NULL). Host-only. */
+const char* arckv_status_string(arckv_status s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ARCKV_H_ */

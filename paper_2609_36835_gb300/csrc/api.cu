@@ -1,0 +1,258 @@
+// C ABI of libarckv: argument validation, workspace layout and the launch
+// sequence of one layer's compaction.  Declarations and contracts are in
+// include/arckv.h.
+#include <string.h>
+
+#include "kernels.h"
+
+using namespace arckv;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+
+inline size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+struct Layout {
+  size_t status, kbar, Uk, Uv, vq, cctx, qbar, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
+      US, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, split, total;
+};
+
+Dims dims_of(const arckv_config& c) {
+  Dims D;
+  D.H = c.H_kv; D.G = c.G; D.T = c.T; D.d = c.d; D.n_pos = c.n_pos; D.n = c.n_pos * c.G; D.d_x = c.d_x;
+  D.H_I = c.H_I; D.d_I = c.d_I; D.d_A = c.d_A; D.t = c.t; D.HD = c.H_I * c.d_I;
+  return D;
+}
+
+arckv_status validate(const arckv_config* c) {
+  if (!c) return ARCKV_ERR_INVALID_ARG;
+  if (c->flags & ~ARCKV_FLAG_NONBLOCKING) return ARCKV_ERR_INVALID_ARG;
+  if (c->H_kv < 1 || c->G < 1 || c->T < 1 || c->n_pos < 1 || c->t < 1 || c->t > c->T) return ARCKV_ERR_SHAPE;
+  if (c->H_I < 1 || c->H_I > 16 || c->d_x < 8 || (c->d_x % 8) != 0) return ARCKV_ERR_SHAPE;
+  if (c->d != 128 || c->d_I != 128 || c->d_A != 128) return ARCKV_ERR_UNSUPPORTED;
+  if (c->chunk_len != 0) return ARCKV_ERR_UNSUPPORTED;
+  // per-head element counts index with 32-bit ints inside the kernels
+  const long long n = (long long)c->n_pos * c->G;
+  if (n > (1 << 24) || (long long)c->T > (1 << 26) || n * c->T >= (1LL << 31) ||
+      (long long)c->t * c->t >= (1LL << 31) || (long long)c->T * c->H_I * 128 >= (1LL << 31) ||
+      (long long)c->H_kv * kSplitK > 65535)
+    return ARCKV_ERR_SHAPE;
+  if (!(c->lambda_m >= 0.f && c->lambda_m <= 1.f)) return ARCKV_ERR_INVALID_ARG;
+  if (!(c->logit_scale >= 0.f) || !isfinite(c->logit_scale)) return ARCKV_ERR_INVALID_ARG;
+  if (!(c->ridge_w >= 0.f) || !(c->ridge_v >= 0.f) || !isfinite(c->ridge_w) || !isfinite(c->ridge_v))
+    return ARCKV_ERR_INVALID_ARG;
+  if (!(c->eps_w > 0.f) || !(c->b_min <= c->b_max) || !isfinite(c->b_min) || !isfinite(c->b_max))
+    return ARCKV_ERR_INVALID_ARG;
+  return ARCKV_OK;
+}
+
+Layout plan(const arckv_config& c) {
+  const Dims D = dims_of(c);
+  const size_t H = D.H, T = D.T, n = D.n, t = D.t, HD = D.HD, f = 4;
+  const size_t nblk = (t + kCholNB - 1) / kCholNB, ntile = (T + 127) / 128;
+  Layout L;
+  size_t o = 0;
+  auto take = [&](size_t bytes) { size_t r = o; o += up(bytes); return r; };
+  L.status = take(sizeof(DevStatus));
+  L.kbar = take(H * T * HD * f);
+  L.Uk = take(H * T * 128 * f);
+  L.Uv = take(H * T * 128 * f);
+  L.vq = take(H * n * 128 * f);
+  L.cctx = take(H * n * 128 * f);
+  L.qbar = take(H * n * HD * f);
+  L.wts = take(H * (size_t)D.n_pos * D.H_I * f);
+  L.NT = take(H * n * T * f);
+  L.rA = take(H * n * f);
+  L.rB = take(H * n * f);
+  L.part = take(H * n * ntile * 8);
+  L.lse = take(H * n * f);
+  L.s = take(H * T * f);
+  L.anchors = take(H * t * 4);
+  L.z = take(H * n * f);
+  L.m = take(H * n * f);
+  L.invm = take(H * n * f);
+  L.Y = take(H * n * 128 * f);
+  L.logphi = take(H * T * f);
+  L.US = take(H * n * t * f);
+  L.best = take(H * T * 8);
+  L.kappa = take(H * T * 4);
+  L.perm = take(H * T * 4);
+  L.goff = take(H * (t + 1) * 4);
+  L.cursor = take(H * t * 4);
+  L.LC = take(H * n * t * f);
+  L.Phi = take(H * n * t * f);
+  L.Gram = take(H * t * t * f);
+  L.Linv = take(H * nblk * kCholNB * kCholNB * f);
+  L.rhs = take(H * t * f);
+  L.split = take((size_t)kSplitK * H * (n > t ? n : t) * 128 * f);
+  L.total = o;
+  return L;
+}
+
+struct Launcher {
+  int count = 0;
+  cudaStream_t st;
+};
+
+arckv_status read_status(void* ws, cudaStream_t st) {
+  unsigned int code = 0;
+  if (cudaMemcpyAsync(&code, ws, sizeof(code), cudaMemcpyDeviceToHost, st) != cudaSuccess) return ARCKV_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return ARCKV_ERR_CUDA;
+  return (arckv_status)code;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t arckv_workspace_bytes(const arckv_config* cfg) {
+  if (validate(cfg) != ARCKV_OK) return 0;
+  return plan(*cfg).total;
+}
+
+const char* arckv_status_string(arckv_status s) {
+  switch (s) {
+    case ARCKV_OK: return "ok";
+    case ARCKV_ERR_INVALID_ARG: return "invalid argument";
+    case ARCKV_ERR_SHAPE: return "shape out of range";
+    case ARCKV_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
+    case ARCKV_ERR_NOT_SPD: return "normal matrix of a fit is not positive definite";
+    case ARCKV_ERR_NONFINITE: return "non-finite value in inputs or results";
+    case ARCKV_ERR_TIMEOUT: return "bounded device wait timed out";
+    case ARCKV_ERR_CUDA: return "CUDA runtime error";
+    case ARCKV_ERR_UNSUPPORTED: return "configuration not supported";
+  }
+  return "unknown status";
+}
+
+arckv_status arckv_query_status(void* ws, void* stream) {
+  if (!ws) return ARCKV_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)stream;
+  arckv_status s = read_status(ws, st);
+  if (s == ARCKV_ERR_CUDA) return s;
+  if (cudaMemsetAsync(ws, 0, sizeof(unsigned int), st) != cudaSuccess) return ARCKV_ERR_CUDA;
+  return s;
+}
+
+arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V, const void* Q_ref,
+                           const void* X_ref, const arckv_indexer* idx, float* C_k, float* beta, float* C_v,
+                           const arckv_aux* aux, void* ws, size_t ws_bytes, void* stream) {
+  arckv_status vs = validate(cfg);
+  if (vs != ARCKV_OK) return vs;
+  if (!K || !V || !Q_ref || !X_ref || !idx || !C_k || !beta || !C_v) return ARCKV_ERR_INVALID_ARG;
+  const bool given_anchors = aux && aux->anchors_in;
+  const bool given_assign = aux && aux->assign_in;
+  if (given_assign && !given_anchors) return ARCKV_ERR_INVALID_ARG;
+  if (!given_anchors && (!idx->L_q || !idx->L_k || !idx->L_x || !idx->b_x || !idx->U_q || !idx->U_k ||
+                         !idx->U_v || !idx->L_c || !idx->L_v))
+    return ARCKV_ERR_INVALID_ARG;
+  const Layout L = plan(*cfg);
+  if (!ws || ws_bytes < L.total || ((uintptr_t)ws % kAlign) != 0) return ARCKV_ERR_WORKSPACE;
+
+  const Dims D = dims_of(*cfg);
+  cudaStream_t st = (cudaStream_t)stream;
+  char* w = (char*)ws;
+  auto F = [&](size_t off) { return (float*)(w + off); };
+  auto I32 = [&](size_t off) { return (int*)(w + off); };
+  DevStatus* stt = (DevStatus*)(w + L.status);
+  const float scale = cfg->logit_scale > 0.f ? cfg->logit_scale : 1.0f / sqrtf((float)D.d);
+  const bf16* Kb = (const bf16*)K;
+  const bf16* Vb = (const bf16*)V;
+  const bf16* Qb = (const bf16*)Q_ref;
+  cudaEvent_t const* ev = (aux && aux->stage_events) ? (cudaEvent_t const*)aux->stage_events : nullptr;
+  auto mark = [&](int s) {
+    if (ev) cudaEventRecord(ev[s], st);
+  };
+  int nl = 0;
+
+  cudaGetLastError();  // clear a stale error from earlier, unrelated work
+  if (cudaMemsetAsync(stt, 0, sizeof(DevStatus), st) != cudaSuccess) return ARCKV_ERR_CUDA;
+  int* anchors = I32(L.anchors);
+  mark(0);
+  if (!given_anchors) {
+    nl += launch_key_features(D, Kb, Vb, (const bf16*)idx->L_k, (const bf16*)idx->L_v, (const bf16*)idx->U_k,
+                              (const bf16*)idx->U_v, F(L.kbar), F(L.Uk), F(L.Uv), st);
+    nl += launch_query_features(D, Qb, (const bf16*)X_ref, (const bf16*)idx->U_q, (const bf16*)idx->L_q,
+                                (const bf16*)idx->L_c, (const bf16*)idx->L_x, (const bf16*)idx->b_x, F(L.Uk),
+                                F(L.Uv), F(L.vq), F(L.NT), F(L.rA), F(L.rB), F(L.split), F(L.cctx), F(L.qbar),
+                                F(L.wts), st);
+    mark(1);
+    nl += launch_index_logits(D, F(L.qbar), F(L.kbar), F(L.wts), F(L.NT), (float2*)(w + L.part), st);
+    mark(2);
+    nl += launch_index_pool(D, F(L.NT), (const float2*)(w + L.part), F(L.lse), F(L.s), st);
+    nl += launch_top_t(D, F(L.s), anchors, stt, st);
+  } else {
+    mark(1);
+    mark(2);
+    cudaMemcpyAsync(anchors, aux->anchors_in, sizeof(int) * (size_t)D.H * D.t, cudaMemcpyDeviceToDevice, st);
+    nl += launch_check_anchors(D, anchors, stt, st);
+  }
+  mark(3);
+  nl += launch_reference_attention(D, scale, Qb, Kb, Vb, F(L.NT), F(L.z), F(L.m), F(L.invm), F(L.split), F(L.Y),
+                                   F(L.logphi), st);
+  int* kappa = I32(L.kappa);
+  if (!given_assign) {
+    nl += launch_assign(D, F(L.NT), anchors, F(L.US), (unsigned long long*)(w + L.best), kappa, st);
+  } else {
+    cudaMemcpyAsync(kappa, aux->assign_in, sizeof(int) * (size_t)D.H * D.T, cudaMemcpyDeviceToDevice, st);
+    nl += launch_check_assign(D, kappa, anchors, stt, st);
+  }
+  mark(4);
+  nl += launch_merge(D, cfg->lambda_m, Kb, anchors, kappa, F(L.logphi), I32(L.perm), I32(L.goff), I32(L.cursor),
+                     C_k, st);
+  mark(5);
+  FitBufs B{F(L.LC), F(L.Phi), F(L.Gram), F(L.Linv), F(L.rhs), F(L.split)};
+  nl += launch_fits(D, scale, cfg->ridge_w, cfg->ridge_v, cfg->eps_w, cfg->b_min, cfg->b_max, Qb, C_k, F(L.z),
+                    F(L.m), F(L.Y), B, beta, C_v, stt, st);
+  nl += launch_check_finite(C_k, (long long)D.H * D.t * D.d, stt, st);
+  nl += launch_check_finite(beta, (long long)D.H * D.t, stt, st);
+  nl += launch_check_finite(C_v, (long long)D.H * D.t * D.d, stt, st);
+  mark(ARCKV_NUM_STAGES);
+  if (aux) {
+    if (aux->scores && !given_anchors)
+      cudaMemcpyAsync(aux->scores, F(L.s), sizeof(float) * (size_t)D.H * D.T, cudaMemcpyDeviceToDevice, st);
+    if (aux->anchors)
+      cudaMemcpyAsync(aux->anchors, anchors, sizeof(int) * (size_t)D.H * D.t, cudaMemcpyDeviceToDevice, st);
+    if (aux->assign)
+      cudaMemcpyAsync(aux->assign, kappa, sizeof(int) * (size_t)D.H * D.T, cudaMemcpyDeviceToDevice, st);
+    if (aux->launches) *aux->launches = nl;
+  }
+  if (cudaGetLastError() != cudaSuccess) return ARCKV_ERR_CUDA;
+  if (cfg->flags & ARCKV_FLAG_NONBLOCKING) return ARCKV_OK;
+  return read_status(ws, st);
+}
+
+size_t arckv_attend_workspace_bytes(int32_t H_kv, int32_t n, int32_t t, int32_t d) {
+  if (H_kv < 1 || n < 1 || t < 1 || d != 128) return 0;
+  if ((long long)n * t >= (1LL << 31) || (long long)H_kv * kSplitK > 65535) return 0;
+  const size_t H = H_kv;
+  return up(sizeof(DevStatus)) + up(H * n * t * 4) + up((size_t)kSplitK * H * n * 128 * 4);
+}
+
+arckv_status arckv_attend(int32_t H_kv, int32_t n, int32_t t, int32_t d, float logit_scale, const void* Q,
+                          const float* C_k, const float* beta, const float* C_v, float* O, void* ws,
+                          size_t ws_bytes, uint32_t flags, void* stream) {
+  if (flags & ~ARCKV_FLAG_NONBLOCKING) return ARCKV_ERR_INVALID_ARG;
+  if (d != 128) return ARCKV_ERR_UNSUPPORTED;
+  const size_t need = arckv_attend_workspace_bytes(H_kv, n, t, d);
+  if (need == 0) return ARCKV_ERR_SHAPE;
+  if (!Q || !C_k || !beta || !C_v || !O) return ARCKV_ERR_INVALID_ARG;
+  if (!(logit_scale >= 0.f) || !isfinite(logit_scale)) return ARCKV_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < need || ((uintptr_t)ws % kAlign) != 0) return ARCKV_ERR_WORKSPACE;
+  cudaStream_t st = (cudaStream_t)stream;
+  char* w = (char*)ws;
+  DevStatus* stt = (DevStatus*)w;
+  float* LC = (float*)(w + up(sizeof(DevStatus)));
+  float* split = (float*)(w + up(sizeof(DevStatus)) + up((size_t)H_kv * n * t * 4));
+  const float scale = logit_scale > 0.f ? logit_scale : 1.0f / sqrtf((float)d);
+  cudaGetLastError();
+  if (cudaMemsetAsync(stt, 0, sizeof(DevStatus), st) != cudaSuccess) return ARCKV_ERR_CUDA;
+  launch_attend(H_kv, n, t, scale, (const bf16*)Q, C_k, beta, C_v, O, LC, split, st);
+  launch_check_finite(O, (long long)H_kv * n * d, stt, st);
+  if (cudaGetLastError() != cudaSuccess) return ARCKV_ERR_CUDA;
+  if (flags & ARCKV_FLAG_NONBLOCKING) return ARCKV_OK;
+  return read_status(ws, st);
+}
+
+}  // extern "C"

@@ -1,0 +1,57 @@
+// Shared device helpers of the ARC-KV CUDA library (sm_103a).
+#pragma once
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+#include <math.h>
+
+#include "arckv.h"
+
+namespace arckv {
+
+typedef __nv_bfloat16 bf16;
+
+// Device status word layout (first 256 bytes of every workspace).
+struct DevStatus {
+  unsigned int code;       // first arckv_status recorded on the device (0 = OK)
+  unsigned int pad[63];
+};
+
+__device__ __forceinline__ void set_status(DevStatus* st, unsigned int code) {
+  atomicCAS(&st->code, 0u, code);
+}
+
+__device__ __forceinline__ float to_f32(float x) { return x; }
+__device__ __forceinline__ float to_f32(bf16 x) { return __bfloat162float(x); }
+
+// Monotone map of fp32 onto uint32 (total order of finite values).
+__device__ __forceinline__ unsigned int f32_ordered(float f) {
+  unsigned int u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float f32_from_ordered(unsigned int u) {
+  return __uint_as_float((u & 0x80000000u) ? (u & 0x7fffffffu) : ~u);
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// Combine two (max, sum of exp(x - max)) pairs.
+__device__ __forceinline__ void lse_combine(float& m, float& s, float m2, float s2) {
+  if (m2 == -INFINITY) return;
+  if (m == -INFINITY) { m = m2; s = s2; return; }
+  if (m2 > m) { s = s * expf(m - m2) + s2; m = m2; }
+  else        { s = s + s2 * expf(m2 - m); }
+}
+
+inline int cdiv(long long a, long long b) { return (int)((a + b - 1) / b); }
+
+}  // namespace arckv

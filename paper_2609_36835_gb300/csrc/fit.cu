@@ -1,0 +1,391 @@
+// Closed-form attention-mass and compact-value fits (App. A.9) and the
+// compact attention operator (Sec. 3.1 Eq. compact_attention).
+//
+// beta:  Phi_C = exp(scale Q C_k^T - z), z_i = max_j scale q_i.k_j;
+//        (Phi_C^T Phi_C + lam_w I) w = Phi_C^T (Phi_K 1);  w* = max(w, 0);
+//        beta = clip(log max(w*, eps_w), b_min, b_max)          (Eq. mass_fit)
+// C_v:   P^ = softmax(scale Q C_k^T + 1 beta^T);
+//        (P^T P^ + lam_v I) C_v = P^T Y, Y = softmax(scale Q K^T) V   (Eq. value_lstsq)
+// with lam = ridge * trace(Gram) / t.  Both systems are solved by a blocked
+// right-looking Cholesky factorisation (64 x 64 blocks; each diagonal block
+// is factored and inverted in shared memory) followed by blocked forward and
+// backward substitution.
+#include "gemm.cuh"
+#include "kernels.h"
+
+namespace arckv {
+
+constexpr int NB = kCholNB;
+
+__global__ void phi_kernel(const float* LC, const float* z, float* Phi, int n, int t, long long count) {
+  for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < count;
+       k += (long long)gridDim.x * blockDim.x) {
+    const long long row = k / t;  // = b * n + i
+    Phi[k] = expf(LC[k] - z[row]);
+  }
+}
+
+// rhs[b][r] = sum_i Phi[b][i][r] m[b][i]   (Phi_C^T Phi_K 1)
+__global__ void mass_rhs_kernel(const float* Phi, const float* m, float* rhs, int n, int t) {
+  const int b = blockIdx.y, r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= t) return;
+  const float* P = Phi + (long long)b * n * t + r;
+  const float* mb = m + (long long)b * n;
+  float a = 0.f;
+  for (int i = 0; i < n; ++i) a = fmaf(P[(long long)i * t], mb[i], a);
+  rhs[(long long)b * t + r] = a;
+}
+
+// Gram += ridge * trace(Gram) / t * I, one CTA per head.
+__global__ void ridge_kernel(float* Gram, int t, float ridge, DevStatus* stt) {
+  const int b = blockIdx.x;
+  float* G = Gram + (long long)b * t * t;
+  __shared__ float red[32];
+  float a = 0.f;
+  for (int r = threadIdx.x; r < t; r += blockDim.x) a += G[(long long)r * t + r];
+  a = warp_sum(a);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = a;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    float v = (threadIdx.x < (blockDim.x >> 5)) ? red[threadIdx.x] : 0.f;
+    v = warp_sum(v);
+    if (threadIdx.x == 0) red[0] = v;
+  }
+  __syncthreads();
+  const float tr = red[0];
+  if (!isfinite(tr)) set_status(stt, ARCKV_ERR_NONFINITE);
+  const float lam = ridge * tr / (float)t;
+  for (int r = threadIdx.x; r < t; r += blockDim.x) G[(long long)r * t + r] += lam;
+}
+
+// Factor the (already updated) diagonal block k in shared memory, write L_kk
+// into A and its inverse into Linv[b][k] (64 x 64, identity beyond the matrix).
+__global__ void __launch_bounds__(256) potrf_diag_kernel(float* A, int t, int k, float* Linv, int nblk,
+                                                         DevStatus* stt) {
+  const int b = blockIdx.x, tid = threadIdx.x;
+  float* Ab = A + (long long)b * t * t;
+  const int k0 = k * NB, kb = min(NB, t - k0);
+  __shared__ float L[NB][NB + 1];
+  __shared__ float Li[NB][NB + 1];
+  __shared__ int bad;
+  for (int e = tid; e < NB * NB; e += 256) {
+    const int r = e / NB, c = e % NB;
+    L[r][c] = (r < kb && c <= r) ? Ab[(long long)(k0 + r) * t + k0 + c] : (r == c ? 1.f : 0.f);
+  }
+  if (tid == 0) bad = 0;
+  __syncthreads();
+  for (int c = 0; c < NB; ++c) {
+    if (tid == 0) {
+      float p = L[c][c];
+      if (!(p > 0.f) || !isfinite(p)) { bad = 1; p = 1.f; }
+      L[c][c] = sqrtf(p);
+    }
+    __syncthreads();
+    const float dinv = 1.0f / L[c][c];
+    for (int r = c + 1 + tid; r < NB; r += 256) L[r][c] *= dinv;
+    __syncthreads();
+    const int w = NB - c - 1;
+    for (int e = tid; e < w * w; e += 256) {
+      const int rr = c + 1 + e / w, cc = c + 1 + e % w;
+      if (cc <= rr) L[rr][cc] = fmaf(-L[rr][c], L[cc][c], L[rr][cc]);
+    }
+    __syncthreads();
+  }
+  if (tid == 0 && bad) set_status(stt, ARCKV_ERR_NOT_SPD);
+  if (tid < NB) {
+    const int j = tid;
+    for (int i = 0; i < NB; ++i) {
+      if (i < j) { Li[i][j] = 0.f; continue; }
+      float s = (i == j) ? 1.f : 0.f;
+      for (int l = j; l < i; ++l) s = fmaf(-L[i][l], Li[l][j], s);
+      Li[i][j] = s / L[i][i];
+    }
+  }
+  __syncthreads();
+  float* Lo = Linv + ((long long)b * nblk + k) * NB * NB;
+  for (int e = tid; e < NB * NB; e += 256) {
+    const int r = e / NB, c = e % NB;
+    Lo[e] = Li[r][c];
+    if (r < kb && c <= r) Ab[(long long)(k0 + r) * t + k0 + c] = L[r][c];
+  }
+}
+
+// L_ik = A_ik Linv_kk^T for the block rows below k.
+__global__ void __launch_bounds__(256) trsm_kernel(float* A, int t, int k, const float* Linv, int nblk) {
+  const int b = blockIdx.y, tid = threadIdx.x;
+  const int i = k + 1 + blockIdx.x, i0 = i * NB, rb = min(NB, t - i0), k0 = k * NB;
+  float* Ab = A + (long long)b * t * t;
+  __shared__ float Aik[NB][NB + 1];
+  __shared__ float Li[NB][NB + 1];
+  const float* Lk = Linv + ((long long)b * nblk + k) * NB * NB;
+  for (int e = tid; e < NB * NB; e += 256) {
+    const int r = e / NB, c = e % NB;
+    Aik[r][c] = (r < rb) ? Ab[(long long)(i0 + r) * t + k0 + c] : 0.f;
+    Li[r][c] = Lk[e];
+  }
+  __syncthreads();
+  const int r = tid >> 2;
+  float out[16];
+#pragma unroll
+  for (int q = 0; q < 16; ++q) out[q] = 0.f;
+  for (int l = 0; l < NB; ++l) {
+    const float a = Aik[r][l];
+#pragma unroll
+    for (int q = 0; q < 16; ++q) out[q] = fmaf(a, Li[(tid & 3) + 4 * q][l], out[q]);
+  }
+  if (r < rb) {
+#pragma unroll
+    for (int q = 0; q < 16; ++q) Ab[(long long)(i0 + r) * t + k0 + (tid & 3) + 4 * q] = out[q];
+  }
+}
+
+// A_ij -= L_ik L_jk^T for the lower blocks k < j <= i of the trailing matrix.
+__global__ void __launch_bounds__(256) syrk_kernel(float* A, int t, int k) {
+  const int b = blockIdx.y, tid = threadIdx.x;
+  const int x = blockIdx.x;
+  int ii = (int)((sqrtf(8.f * x + 1.f) - 1.f) * 0.5f);
+  while (ii * (ii + 1) / 2 > x) --ii;
+  while ((ii + 1) * (ii + 2) / 2 <= x) ++ii;
+  const int jj = x - ii * (ii + 1) / 2;
+  const int i0 = (k + 1 + ii) * NB, j0 = (k + 1 + jj) * NB, k0 = k * NB;
+  const int rb = min(NB, t - i0), cb = min(NB, t - j0);
+  float* Ab = A + (long long)b * t * t;
+  __shared__ float Li[NB][NB + 1];
+  __shared__ float Lj[NB][NB + 1];
+  for (int e = tid; e < NB * NB; e += 256) {
+    const int r = e / NB, c = e % NB;
+    Li[r][c] = (r < rb) ? Ab[(long long)(i0 + r) * t + k0 + c] : 0.f;
+    Lj[r][c] = (r < cb) ? Ab[(long long)(j0 + r) * t + k0 + c] : 0.f;
+  }
+  __syncthreads();
+  const int ry = (tid >> 4) * 4, cx = (tid & 15) * 4;
+  float acc[4][4];
+#pragma unroll
+  for (int p = 0; p < 4; ++p)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
+  for (int l = 0; l < NB; ++l) {
+    float a[4], c[4];
+#pragma unroll
+    for (int p = 0; p < 4; ++p) { a[p] = Li[ry + p][l]; c[p] = Lj[cx + p][l]; }
+#pragma unroll
+    for (int p = 0; p < 4; ++p)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) acc[p][q] = fmaf(a[p], c[q], acc[p][q]);
+  }
+#pragma unroll
+  for (int p = 0; p < 4; ++p)
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      if (ry + p < rb && cx + q < cb) Ab[(long long)(i0 + ry + p) * t + j0 + cx + q] -= acc[p][q];
+}
+
+// Solve L L^T X = B in place (X holds B), columns [32 blockIdx.x, +32) of an
+// nrhs-column right-hand side with row stride ldx; one CTA per (column tile, head).
+__global__ void __launch_bounds__(256) chol_solve_kernel(const float* A, const float* Linv, float* X, int t,
+                                                         int ldx, int nrhs, long long xbs, int nblk) {
+  const int b = blockIdx.y, tid = threadIdx.x;
+  const int c0 = blockIdx.x * 32, nc = min(32, nrhs - c0);
+  const float* Ab = A + (long long)b * t * t;
+  const float* Lb = Linv + (long long)b * nblk * NB * NB;
+  float* Xb = X + (long long)b * xbs;
+  __shared__ float Lt[NB][NB + 1];
+  __shared__ float Yt[NB][33];
+  const int r = tid >> 2, cc = (tid & 3) * 8;
+  float acc[8];
+  // forward: Y_k = Linv_kk (B_k - sum_{j<k} L_kj Y_j)
+  for (int k = 0; k < nblk; ++k) {
+    const int k0 = k * NB, kb = min(NB, t - k0);
+#pragma unroll
+    for (int q = 0; q < 8; ++q)
+      acc[q] = (r < kb && cc + q < nc) ? Xb[(long long)(k0 + r) * ldx + c0 + cc + q] : 0.f;
+    for (int j = 0; j < k; ++j) {
+      const int j0 = j * NB;
+      __syncthreads();
+      for (int e = tid; e < NB * NB; e += 256) {
+        const int rr = e / NB, l = e % NB;
+        Lt[rr][l] = (rr < kb) ? Ab[(long long)(k0 + rr) * t + j0 + l] : 0.f;
+      }
+      for (int e = tid; e < NB * 32; e += 256) {
+        const int l = e >> 5, c = e & 31;
+        Yt[l][c] = (c < nc) ? Xb[(long long)(j0 + l) * ldx + c0 + c] : 0.f;
+      }
+      __syncthreads();
+      for (int l = 0; l < NB; ++l) {
+        const float a = Lt[r][l];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc[q] = fmaf(-a, Yt[l][cc + q], acc[q]);
+      }
+    }
+    __syncthreads();
+    const float* Lk = Lb + (long long)k * NB * NB;
+    for (int e = tid; e < NB * NB; e += 256) Lt[e / NB][e % NB] = Lk[e];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) Yt[r][cc + q] = acc[q];
+    __syncthreads();
+#pragma unroll
+    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+    for (int l = 0; l <= r; ++l) {
+      const float a = Lt[r][l];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) acc[q] = fmaf(a, Yt[l][cc + q], acc[q]);
+    }
+#pragma unroll
+    for (int q = 0; q < 8; ++q)
+      if (r < kb && cc + q < nc) Xb[(long long)(k0 + r) * ldx + c0 + cc + q] = acc[q];
+    __syncthreads();
+  }
+  // backward: X_k = Linv_kk^T (Y_k - sum_{j>k} L_jk^T X_j)
+  for (int k = nblk - 1; k >= 0; --k) {
+    const int k0 = k * NB, kb = min(NB, t - k0);
+#pragma unroll
+    for (int q = 0; q < 8; ++q)
+      acc[q] = (r < kb && cc + q < nc) ? Xb[(long long)(k0 + r) * ldx + c0 + cc + q] : 0.f;
+    for (int j = k + 1; j < nblk; ++j) {
+      const int j0 = j * NB, jb = min(NB, t - j0);
+      __syncthreads();
+      for (int e = tid; e < NB * NB; e += 256) {
+        const int l = e / NB, rr = e % NB;
+        Lt[l][rr] = (l < jb) ? Ab[(long long)(j0 + l) * t + k0 + rr] : 0.f;
+      }
+      for (int e = tid; e < NB * 32; e += 256) {
+        const int l = e >> 5, c = e & 31;
+        Yt[l][c] = (l < jb && c < nc) ? Xb[(long long)(j0 + l) * ldx + c0 + c] : 0.f;
+      }
+      __syncthreads();
+      for (int l = 0; l < NB; ++l) {
+        const float a = Lt[l][r];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc[q] = fmaf(-a, Yt[l][cc + q], acc[q]);
+      }
+    }
+    __syncthreads();
+    const float* Lk = Lb + (long long)k * NB * NB;
+    for (int e = tid; e < NB * NB; e += 256) Lt[e / NB][e % NB] = Lk[e];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) Yt[r][cc + q] = acc[q];
+    __syncthreads();
+#pragma unroll
+    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+    for (int l = r; l < NB; ++l) {
+      const float a = Lt[l][r];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) acc[q] = fmaf(a, Yt[l][cc + q], acc[q]);
+    }
+#pragma unroll
+    for (int q = 0; q < 8; ++q)
+      if (r < kb && cc + q < nc) Xb[(long long)(k0 + r) * ldx + c0 + cc + q] = acc[q];
+    __syncthreads();
+  }
+}
+
+static int cholesky_solve(int H, int t, float* Gram, float* Linv, float* X, int ldx, int nrhs, long long xbs,
+                          float ridge, DevStatus* stt, cudaStream_t st) {
+  int nl = 0;
+  ridge_kernel<<<H, 256, 0, st>>>(Gram, t, ridge, stt);
+  ++nl;
+  const int nblk = cdiv(t, NB);
+  for (int k = 0; k < nblk; ++k) {
+    potrf_diag_kernel<<<H, 256, 0, st>>>(Gram, t, k, Linv, nblk, stt);
+    ++nl;
+    const int m = nblk - k - 1;
+    if (m > 0) {
+      trsm_kernel<<<dim3(m, H), 256, 0, st>>>(Gram, t, k, Linv, nblk);
+      syrk_kernel<<<dim3(m * (m + 1) / 2, H), 256, 0, st>>>(Gram, t, k);
+      nl += 2;
+    }
+  }
+  chol_solve_kernel<<<dim3(cdiv(nrhs, 32), H), 256, 0, st>>>(Gram, Linv, X, t, ldx, nrhs, xbs, nblk);
+  return nl + 1;
+}
+
+__global__ void beta_kernel(const float* w, float* beta, long long count, float eps_w, float b_min, float b_max) {
+  for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < count;
+       k += (long long)gridDim.x * blockDim.x) {
+    const float ws = fmaxf(w[k], 0.f);
+    beta[k] = fminf(fmaxf(logf(fmaxf(ws, eps_w)), b_min), b_max);
+  }
+}
+
+// P[row] = softmax(LC[row] + beta), one warp per row (rows = H * n).
+__global__ void softmax_bias_kernel(const float* LC, const float* beta, float* P, int n, int t) {
+  const int b = blockIdx.y, row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= n) return;
+  const float* x = LC + ((long long)b * n + row) * t;
+  const float* be = beta + (long long)b * t;
+  float* o = P + ((long long)b * n + row) * t;
+  float mx = -INFINITY;
+  for (int c = lane; c < t; c += 32) mx = fmaxf(mx, x[c] + be[c]);
+  mx = warp_max(mx);
+  float sm = 0.f;
+  for (int c = lane; c < t; c += 32) sm += expf(x[c] + be[c] - mx);
+  sm = warp_sum(sm);
+  const float inv = 1.0f / sm;
+  for (int c = lane; c < t; c += 32) o[c] = expf(x[c] + be[c] - mx) * inv;
+}
+
+int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float eps_w, float b_min,
+                float b_max, const bf16* Q, const float* C_k, const float* z, const float* m,
+                const float* Y, const FitBufs& B, float* beta, float* C_v, DevStatus* stt, cudaStream_t st) {
+  int nl = 0;
+  const long long nd = (long long)D.n * D.d, nt = (long long)D.n * D.t, tt = (long long)D.t * D.t;
+  // logits of the compact keys: scale Q C_k^T
+  launch_gemm(RowK<bf16>{Q, nd, D.d}, RowK<float>{C_k, (long long)D.t * D.d, D.d},
+              EpiStore{B.LC, nt, 0, D.t, scale, false}, D.H, D.n, D.t, D.d, 1, st);
+  ++nl;
+  const long long cnt = (long long)D.H * nt;
+  phi_kernel<<<min(cdiv(cnt, 256), 152 * 16), 256, 0, st>>>(B.LC, z, B.Phi, D.n, D.t, cnt);
+  ++nl;
+  // beta system
+  launch_gemm<true>(ColK<float>{B.Phi, nt, D.t}, ColK<float>{B.Phi, nt, D.t}, EpiStore{B.Gram, tt, 0, D.t, 1.f, true},
+                    D.H, D.t, D.t, D.n, 1, st);
+  ++nl;
+  mass_rhs_kernel<<<dim3(cdiv(D.t, 128), D.H), 128, 0, st>>>(B.Phi, m, B.rhs, D.n, D.t);
+  ++nl;
+  nl += cholesky_solve(D.H, D.t, B.Gram, B.Linv, B.rhs, 1, 1, D.t, ridge_w, stt, st);
+  const long long ht = (long long)D.H * D.t;
+  beta_kernel<<<cdiv(ht, 256), 256, 0, st>>>(B.rhs, beta, ht, eps_w, b_min, b_max);
+  ++nl;
+  // value system: P^ over the compact keys with the fitted bias
+  softmax_bias_kernel<<<dim3(cdiv(D.n, 8), D.H), 256, 0, st>>>(B.LC, beta, B.Phi, D.n, D.t);
+  ++nl;
+  launch_gemm<true>(ColK<float>{B.Phi, nt, D.t}, ColK<float>{B.Phi, nt, D.t}, EpiStore{B.Gram, tt, 0, D.t, 1.f, true},
+                    D.H, D.t, D.t, D.n, 1, st);
+  ++nl;
+  const long long td = (long long)D.t * D.d;
+  launch_gemm(ColK<float>{B.Phi, nt, D.t}, ColK<float>{Y, nd, D.d},
+              EpiStore{B.split, td, (long long)D.H * td, D.d, 1.f, false}, D.H, D.t, D.d, D.n, kSplitK, st);
+  ++nl;
+  nl += launch_split_reduce(D.H, D.t, D.d, kSplitK, B.split, C_v, st);
+  nl += cholesky_solve(D.H, D.t, B.Gram, B.Linv, C_v, D.d, D.d, td, ridge_v, stt, st);
+  return nl;
+}
+
+__global__ void check_finite_kernel(const float* x, long long count, DevStatus* stt) {
+  bool bad = false;
+  for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < count;
+       k += (long long)gridDim.x * blockDim.x)
+    bad |= !isfinite(x[k]);
+  if (__any_sync(0xffffffffu, bad) && (threadIdx.x & 31) == 0) set_status(stt, ARCKV_ERR_NONFINITE);
+}
+
+int launch_check_finite(const float* x, long long count, DevStatus* stt, cudaStream_t st) {
+  check_finite_kernel<<<min(cdiv(count, 256), 152 * 8), 256, 0, st>>>(x, count, stt);
+  return 1;
+}
+
+int launch_attend(int H, int n, int t, float scale, const bf16* Q, const float* C_k, const float* beta,
+                  const float* C_v, float* O, float* LC, float* split, cudaStream_t st) {
+  const int d = 128;
+  const long long nd = (long long)n * d, nt = (long long)n * t, td = (long long)t * d;
+  launch_gemm(RowK<bf16>{Q, nd, d}, RowK<float>{C_k, td, d}, EpiStore{LC, nt, 0, t, scale, false}, H, n, t, d, 1,
+              st);
+  softmax_bias_kernel<<<dim3(cdiv(n, 8), H), 256, 0, st>>>(LC, beta, LC, n, t);
+  const int splits = max(1, min(kSplitK, cdiv(t, 128)));
+  launch_gemm(RowK<float>{LC, nt, t}, ColK<float>{C_v, td, d}, EpiStore{split, nd, (long long)H * nd, d, 1.f, false},
+              H, n, d, t, splits, st);
+  launch_split_reduce(H, n, d, splits, split, O, st);
+  return 4;
+}
+
+}  // namespace arckv

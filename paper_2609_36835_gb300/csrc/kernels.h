@@ -1,0 +1,64 @@
+// Internal launchers of the ARC-KV stage kernels (host side).  Every launcher
+// enqueues on `st` and returns the number of kernels it launched.
+#pragma once
+#include "common.cuh"
+
+namespace arckv {
+
+struct Dims {
+  int H, G, T, d, n_pos, n, d_x, H_I, d_I, d_A, t, HD;
+};
+
+constexpr int kSplitK = 8;   // K slices of the skinny (N = 128) long-K products
+constexpr int kCholNB = 64;  // Cholesky block size
+
+// ---- indexer (Sec. 3.3, App. A.1) --------------------------------------
+// k_bar = N(L_k k + L_v v) per d_I block; Uk = U_k k; Uv = U_v v.
+int launch_key_features(const Dims& D, const bf16* K, const bf16* V, const bf16* L_k, const bf16* L_v,
+                        const bf16* U_k, const bf16* U_v, float* kbar, float* Uk, float* Uv, cudaStream_t st);
+// value context c (Eq. value_context), q_bar (Eq. indexer_projection), w.
+int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf16* U_q, const bf16* L_q,
+                          const bf16* L_c, const bf16* L_x, const bf16* b_x, const float* Uk,
+                          const float* Uv, float* vq, float* logits, float* rshift, float* rmul,
+                          float* split, float* cctx, float* qbar, float* wts, cudaStream_t st);
+// I (Eq. pairwise_index_score) and per-(row, column tile) softmax partials.
+int launch_index_logits(const Dims& D, const float* qbar, const float* kbar, const float* wts, float* I,
+                        float2* part, cudaStream_t st);
+// row log-sum-exp and pooled s (Eq. indexer_pooling).
+int launch_index_pool(const Dims& D, const float* I, const float2* part, float* lse, float* s, cudaStream_t st);
+
+// ---- selection (Eq. persistent_support) ----------------------------------
+int launch_top_t(const Dims& D, const float* s, int* anchors, DevStatus* stt, cudaStream_t st);
+int launch_check_anchors(const Dims& D, int* anchors, DevStatus* stt, cudaStream_t st);
+
+// ---- reference attention, assignment, merge (Sec. 3.4) ------------------
+// l = scale Q K^T into `L`; z, m (row max / mass); Y = softmax(l) V;
+// column statistics log phi and the normalised profiles U written over `L`.
+int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const bf16* K, const bf16* V,
+                               float* L, float* z, float* m, float* invm, float* split, float* Y,
+                               float* logphi, cudaStream_t st);
+int launch_assign(const Dims& D, const float* U, const int* anchors, float* US, unsigned long long* best,
+                  int* kappa, cudaStream_t st);
+int launch_check_assign(const Dims& D, int* kappa, const int* anchors, DevStatus* stt, cudaStream_t st);
+int launch_merge(const Dims& D, float lambda_m, const bf16* K, const int* anchors, const int* kappa,
+                 const float* logphi, int* perm, int* goff, int* cursor, float* C_k, cudaStream_t st);
+
+// ---- fits (App. A.9) -----------------------------------------------------
+struct FitBufs {
+  float *LC, *Phi, *Gram, *Linv, *rhs, *split;
+};
+int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float eps_w, float b_min,
+                float b_max, const bf16* Q, const float* C_k, const float* z, const float* m,
+                const float* Y, const FitBufs& B, float* beta, float* C_v, DevStatus* stt, cudaStream_t st);
+int launch_check_finite(const float* x, long long count, DevStatus* stt, cudaStream_t st);
+
+// ---- compact attention (Eq. compact_attention) ----------------------------
+int launch_attend(int H, int n, int t, float scale, const bf16* Q, const float* C_k, const float* beta,
+                  const float* C_v, float* O, float* LC, float* split, cudaStream_t st);
+
+// Shared small kernels.
+int launch_row_stats(int H, int rows, int cols, const float* X, float* shift, float* mul, float* sum,
+                     cudaStream_t st);
+int launch_split_reduce(int H, int M, int N, int splits, const float* part, float* out, cudaStream_t st);
+
+}  // namespace arckv

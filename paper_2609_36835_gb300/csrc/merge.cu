@@ -1,0 +1,257 @@
+// Full-cache reference attention, response-profile assignment and the
+// convex-hull key merge (Sec. 3.4).
+//
+// The paper's profiles u_j and mass weights phi_j use one global shift
+// z_merge = max_ij l_ij (Eq. response_profile, Eq. mass_centroid).  Both u_j
+// (a normalised column) and the ratios phi_j / sum_{G_r} phi_j are invariant to
+// any per-column shift, so the kernels shift column j by its own maximum M_j,
+// which keeps every column representable in fp32 when the logit range
+// exceeds the fp32 exponent range.
+#include "gemm.cuh"
+#include "kernels.h"
+
+namespace arckv {
+
+// One thread per column j: M_j = max_i l_ij, s1 = sum_i e^{l_ij - M_j},
+// s2 = sum_i e^{2(l_ij - M_j)}; log phi_j = M_j + log s1 - log n; then
+// U_ij = e^{l_ij - M_j} / sqrt(s2) is written over l.
+__global__ void __launch_bounds__(128) col_stats_kernel(float* L, float* logphi, int n, int T) {
+  const int b = blockIdx.y, j = blockIdx.x * 128 + threadIdx.x;
+  if (j >= T) return;
+  float* Lb = L + (long long)b * n * T + j;
+  float mx = -INFINITY, s1 = 0.f, s2 = 0.f;
+#pragma unroll 4
+  for (int i = 0; i < n; ++i) {
+    const float v = Lb[(long long)i * T];
+    if (v > mx) {
+      const float r = (mx == -INFINITY) ? 0.f : expf(mx - v);
+      s1 = fmaf(s1, r, 1.f);
+      s2 = fmaf(s2, r * r, 1.f);
+      mx = v;
+    } else {
+      const float e = expf(v - mx);
+      s1 += e;
+      s2 = fmaf(e, e, s2);
+    }
+  }
+  logphi[(long long)b * T + j] = mx + logf(s1) - logf((float)n);
+  const float inv = 1.0f / sqrtf(s2);
+#pragma unroll 4
+  for (int i = 0; i < n; ++i) {
+    float* p = Lb + (long long)i * T;
+    *p = expf(*p - mx) * inv;
+  }
+}
+
+int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const bf16* K, const bf16* V,
+                               float* L, float* z, float* m, float* invm, float* split, float* Y,
+                               float* logphi, cudaStream_t st) {
+  const long long nd = (long long)D.n * D.d, Td = (long long)D.T * D.d, nT = (long long)D.n * D.T;
+  // l = scale * Q K^T
+  launch_gemm(RowK<bf16>{Q, nd, D.d}, RowK<bf16>{K, Td, D.d}, EpiStore{L, nT, 0, D.T, scale, false}, D.H, D.n,
+              D.T, D.d, 1, st);
+  // z_i = max_j l_ij (z^fit of Eq. mass_fit), m_i = sum_j e^{l_ij - z_i} = (Phi_K 1)_i
+  launch_row_stats(D.H, D.n, D.T, L, z, invm, m, st);
+  // Y = softmax(l) V
+  RowKExp P{{L, nT, D.T}, z, invm, D.n, 1.f};
+  launch_gemm(P, ColK<bf16>{V, Td, D.d}, EpiStore{split, nd, (long long)D.H * nd, D.d, 1.f, false}, D.H, D.n,
+              D.d, D.T, kSplitK, st);
+  launch_split_reduce(D.H, D.n, D.d, kSplitK, split, Y, st);
+  col_stats_kernel<<<dim3(cdiv(D.T, 128), D.H), 128, 0, st>>>(L, logphi, D.n, D.T);
+  return 5;
+}
+
+// US[b][i][r] = U[b][i][S_r]
+__global__ void gather_anchor_cols_kernel(const float* U, const int* anchors, float* US, int n, int T, int t) {
+  const int b = blockIdx.y, i = blockIdx.x;
+  const float* u = U + ((long long)b * n + i) * T;
+  const int* S = anchors + (long long)b * t;
+  float* o = US + ((long long)b * n + i) * t;
+  for (int r = threadIdx.x; r < t; r += blockDim.x) o[r] = u[S[r]];
+}
+
+__global__ void decode_assign_kernel(const unsigned long long* best, int* kappa, long long count) {
+  for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < count;
+       k += (long long)gridDim.x * blockDim.x) {
+    const unsigned long long v = best[k];
+    kappa[k] = v ? (int)(0xffffffffu - (unsigned int)(v & 0xffffffffull)) : 0;
+  }
+}
+
+// kappa(s_r) = r (Eq. anchor_assignment)
+__global__ void anchor_self_assign_kernel(const int* anchors, int* kappa, int T, int t, int H) {
+  const long long total = (long long)H * t;
+  for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < total;
+       k += (long long)gridDim.x * blockDim.x) {
+    const long long b = k / t;
+    kappa[b * T + anchors[k]] = (int)(k - b * t);
+  }
+}
+
+int launch_assign(const Dims& D, const float* U, const int* anchors, float* US, unsigned long long* best,
+                  int* kappa, cudaStream_t st) {
+  gather_anchor_cols_kernel<<<dim3(D.n, D.H), 256, 0, st>>>(U, anchors, US, D.n, D.T, D.t);
+  cudaMemsetAsync(best, 0, sizeof(unsigned long long) * (size_t)D.H * D.T, st);
+  // sim(j, r) = u_j . u_{s_r}: A(j, i) = U[i][j], B(r, i) = US[i][r]
+  launch_gemm(ColK<float>{U, (long long)D.n * D.T, D.T}, ColK<float>{US, (long long)D.n * D.t, D.t},
+              EpiArgmax{best, D.T}, D.H, D.T, D.t, D.n, 1, st);
+  const long long cnt = (long long)D.H * D.T;
+  decode_assign_kernel<<<min(cdiv(cnt, 256), 152 * 8), 256, 0, st>>>(best, kappa, cnt);
+  anchor_self_assign_kernel<<<cdiv((long long)D.H * D.t, 256), 256, 0, st>>>(anchors, kappa, D.T, D.t, D.H);
+  return 4;
+}
+
+// Caller-supplied assignment (copied into the workspace): values in [0, t)
+// and kappa(s_r) = r.  A violation is recorded as ARCKV_ERR_INVALID_ARG and
+// out-of-range entries are clamped to [0, t).  Runs after the anchors check,
+// so anchors are already inside [0, T).
+__global__ void check_assign_kernel(int* kappa, const int* anchors, int T, int t, int H, DevStatus* stt) {
+  const long long total = (long long)H * T;
+  for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < total;
+       k += (long long)gridDim.x * blockDim.x) {
+    const int v = kappa[k];
+    if (v < 0 || v >= t) {
+      set_status(stt, ARCKV_ERR_INVALID_ARG);
+      kappa[k] = min(max(v, 0), t - 1);
+    }
+  }
+  const long long ta = (long long)H * t;
+  for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < ta;
+       k += (long long)gridDim.x * blockDim.x) {
+    const long long b = k / t;
+    const int a = anchors[k];
+    const int v = kappa[b * T + a];
+    if (v != (int)(k - b * t) && (v >= 0 && v < t)) set_status(stt, ARCKV_ERR_INVALID_ARG);
+  }
+}
+
+int launch_check_assign(const Dims& D, int* kappa, const int* anchors, DevStatus* stt, cudaStream_t st) {
+  check_assign_kernel<<<min(cdiv((long long)D.H * D.T, 256), 152 * 8), 256, 0, st>>>(kappa, anchors, D.T, D.t,
+                                                                                      D.H, stt);
+  return 1;
+}
+
+__device__ __forceinline__ int block_excl_scan_1024_m(int v, int* sc, int& total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) sc[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = sc[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    sc[lane] = w;
+  }
+  __syncthreads();
+  const int off = warp > 0 ? sc[warp - 1] : 0;
+  total = sc[31];
+  __syncthreads();
+  return off + x - v;
+}
+
+// Stable counting sort of positions by group (one 1024-thread CTA per head):
+// perm lists the members of G_0, G_1, ... each in ascending position order;
+// goff[r] .. goff[r+1] delimits G_r.
+__global__ void __launch_bounds__(1024) group_sort_kernel(const int* kappa, int T, int t, int* perm, int* goff,
+                                                          int* cursor) {
+  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int* kb = kappa + (long long)b * T;
+  int* pb = perm + (long long)b * T;
+  int* gb = goff + (long long)b * (t + 1);
+  int* cb = cursor + (long long)b * t;
+  __shared__ int sc[32];
+  for (int r = tid; r < t; r += 1024) cb[r] = 0;
+  __syncthreads();
+  for (int j = tid; j < T; j += 1024) atomicAdd(&cb[kb[j]], 1);
+  __syncthreads();
+  int base = 0;
+  for (int r0 = 0; r0 < t; r0 += 1024) {
+    const int r = r0 + tid;
+    const int c = (r < t) ? cb[r] : 0;
+    int tot;
+    const int ex = block_excl_scan_1024_m(c, sc, tot) + base;
+    if (r < t) { gb[r] = ex; cb[r] = ex; }
+    base += tot;
+  }
+  if (tid == 0) gb[t] = base;
+  __syncthreads();
+  const unsigned int lt = (1u << lane) - 1u;
+  for (int j0 = 0; j0 < T; j0 += 1024) {
+    const int j = j0 + tid;
+    const int key = (j < T) ? kb[j] : -1;
+    const unsigned int peers = __match_any_sync(0xffffffffu, key);
+    const int rank = __popc(peers & lt);
+    const bool leader = (__ffs(peers) - 1) == lane;
+    int pos = 0;
+    for (int w = 0; w < 32; ++w) {
+      if (warp == w) {
+        if (key >= 0) pos = cb[key] + rank;
+        __syncwarp();
+        if (key >= 0 && leader) cb[key] += __popc(peers);
+      }
+      __syncthreads();
+    }
+    if (key >= 0) pb[pos] = j;
+  }
+}
+
+// One warp per group r: mu_r = sum_{G_r} w_j k_j / sum_{G_r} w_j with
+// w_j = e^{log phi_j - max_{G_r} log phi} (Eq. mass_centroid), members summed in
+// ascending position order; c_r = k_{s_r} + lambda_m (mu_r - k_{s_r}), which is
+// (1 - lambda_m) k_{s_r} + lambda_m mu_r of Eq. key_merge.
+__global__ void __launch_bounds__(256) group_merge_kernel(const bf16* K, const int* anchors, const int* perm,
+                                                          const int* goff, const float* logphi, float lambda_m,
+                                                          float* C_k, int T, int t) {
+  const int b = blockIdx.y, r = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (r >= t) return;
+  const int* pb = perm + (long long)b * T;
+  const int* gb = goff + (long long)b * (t + 1);
+  const float* lp = logphi + (long long)b * T;
+  const bf16* Kb = K + (long long)b * T * 128;
+  const int beg = gb[r], end = gb[r + 1];
+  float gm = -INFINITY;
+  for (int q = beg + lane; q < end; q += 32) gm = fmaxf(gm, lp[pb[q]]);
+  gm = warp_max(gm);
+  float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f, ws = 0.f;
+#pragma unroll 4
+  for (int q = beg; q < end; ++q) {
+    const int j = pb[q];
+    const float om = expf(lp[j] - gm);
+    const uint2 raw = *(const uint2*)(Kb + (long long)j * 128 + lane * 4);
+    const bf16* h = (const bf16*)&raw;
+    a0 = fmaf(om, to_f32(h[0]), a0);
+    a1 = fmaf(om, to_f32(h[1]), a1);
+    a2 = fmaf(om, to_f32(h[2]), a2);
+    a3 = fmaf(om, to_f32(h[3]), a3);
+    ws += om;
+  }
+  const int s = anchors[(long long)b * t + r];
+  const uint2 raw = *(const uint2*)(Kb + (long long)s * 128 + lane * 4);
+  const bf16* h = (const bf16*)&raw;
+  const float k0 = to_f32(h[0]), k1 = to_f32(h[1]), k2 = to_f32(h[2]), k3 = to_f32(h[3]);
+  const float iw = 1.0f / ws;
+  float4 c;
+  c.x = fmaf(lambda_m, a0 * iw - k0, k0);
+  c.y = fmaf(lambda_m, a1 * iw - k1, k1);
+  c.z = fmaf(lambda_m, a2 * iw - k2, k2);
+  c.w = fmaf(lambda_m, a3 * iw - k3, k3);
+  *(float4*)(C_k + ((long long)b * t + r) * 128 + lane * 4) = c;
+}
+
+int launch_merge(const Dims& D, float lambda_m, const bf16* K, const int* anchors, const int* kappa,
+                 const float* logphi, int* perm, int* goff, int* cursor, float* C_k, cudaStream_t st) {
+  group_sort_kernel<<<D.H, 1024, 0, st>>>(kappa, D.T, D.t, perm, goff, cursor);
+  group_merge_kernel<<<dim3(cdiv(D.t, 8), D.H), 256, 0, st>>>(K, anchors, perm, goff, logphi, lambda_m, C_k,
+                                                              D.T, D.t);
+  return 2;
+}
+
+}  // namespace arckv

@@ -1,0 +1,163 @@
+// Top-t anchor selection (App. A.6 Eq. persistent_support) and small shared
+// row / reduction kernels.
+#include "kernels.h"
+
+namespace arckv {
+
+// Exclusive prefix sum over a 1024-thread block; `sc` holds 32 ints.
+__device__ __forceinline__ int block_excl_scan_1024(int v, int* sc, int& total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) sc[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = sc[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    sc[lane] = w;
+  }
+  __syncthreads();
+  const int off = warp > 0 ? sc[warp - 1] : 0;
+  total = sc[31];
+  __syncthreads();
+  return off + x - v;
+}
+
+// One 1024-thread CTA per head.  MSB-first radix select (8-bit digits) of the
+// t-th largest score on the ordered bit patterns, then an order-preserving
+// compaction: every position with a larger score, plus the lowest-position
+// ones among those equal to the threshold (ties -> lower position), written
+// in ascending position order.
+__global__ void __launch_bounds__(1024) top_t_kernel(const float* s, int T, int t, int* anchors,
+                                                     DevStatus* stt) {
+  const int b = blockIdx.x, tid = threadIdx.x;
+  const float* sb = s + (long long)b * T;
+  int* out = anchors + (long long)b * t;
+  __shared__ int hist[256];
+  __shared__ int sc[32];
+  __shared__ unsigned int sh_prefix;
+  __shared__ int sh_rem;
+  unsigned int prefix = 0u, mask = 0u;
+  int rem = t;
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 24 - 8 * pass;
+    if (tid < 256) hist[tid] = 0;
+    __syncthreads();
+    for (int j = tid; j < T; j += 1024) {
+      const float v = sb[j];
+      if (pass == 0 && !isfinite(v)) set_status(stt, ARCKV_ERR_NONFINITE);
+      const unsigned int key = f32_ordered(v);
+      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1);
+    }
+    __syncthreads();
+    if (tid == 0) {
+      int cum = 0, D = 0;
+      for (int dg = 255; dg >= 0; --dg) {
+        if (cum + hist[dg] >= rem) { D = dg; break; }
+        cum += hist[dg];
+      }
+      sh_prefix = prefix | ((unsigned int)D << shift);
+      sh_rem = rem - cum;
+    }
+    __syncthreads();
+    prefix = sh_prefix;
+    rem = sh_rem;
+    mask |= 0xffu << shift;
+  }
+  int base = 0, eqseen = 0;
+  for (int j0 = 0; j0 < T; j0 += 1024) {
+    const int j = j0 + tid;
+    const unsigned int key = (j < T) ? f32_ordered(sb[j]) : 0u;
+    const int eq = (j < T && key == prefix) ? 1 : 0;
+    int eqtot, tot;
+    const int eqrank = block_excl_scan_1024(eq, sc, eqtot) + eqseen;
+    const int take = (j < T && (key > prefix || (eq && eqrank < rem))) ? 1 : 0;
+    const int pos = block_excl_scan_1024(take, sc, tot) + base;
+    if (take && pos < t) out[pos] = j;
+    base += tot;
+    eqseen += eqtot;
+  }
+  if (tid == 0 && base != t) set_status(stt, ARCKV_ERR_INVALID_ARG);
+}
+
+int launch_top_t(const Dims& D, const float* s, int* anchors, DevStatus* stt, cudaStream_t st) {
+  top_t_kernel<<<D.H, 1024, 0, st>>>(s, D.T, D.t, anchors, stt);
+  return 1;
+}
+
+// Caller-supplied anchors (copied into the workspace) must be strictly
+// ascending positions in [0, T).  A violation is recorded as
+// ARCKV_ERR_INVALID_ARG and every entry is clamped to [0, T) so that later
+// kernels never index outside the cache.  One CTA per head.
+__global__ void check_anchors_kernel(int* anchors, int T, int t, DevStatus* stt) {
+  int* a = anchors + (long long)blockIdx.x * t;
+  bool bad = false;
+  for (int r = threadIdx.x; r < t; r += blockDim.x) {
+    const int v = a[r];
+    bad |= (v < 0 || v >= T || (r > 0 && a[r - 1] >= v));
+  }
+  __syncthreads();
+  for (int r = threadIdx.x; r < t; r += blockDim.x) a[r] = min(max(a[r], 0), T - 1);
+  if (bad) set_status(stt, ARCKV_ERR_INVALID_ARG);
+}
+
+int launch_check_anchors(const Dims& D, int* anchors, DevStatus* stt, cudaStream_t st) {
+  check_anchors_kernel<<<D.H, 256, 0, st>>>(anchors, D.T, D.t, stt);
+  return 1;
+}
+
+// Per row: shift = max_c X, sum = sum_c exp(X - shift), mul = 1 / sum (one warp per row).
+__global__ void row_stats_kernel(const float* X, float* shift, float* mul, float* sum, int rows, int cols) {
+  const int b = blockIdx.y, row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const float* x = X + ((long long)b * rows + row) * cols;
+  float mx = -INFINITY, sm = 0.f;
+  for (int c = lane; c < cols; c += 32) {
+    const float v = x[c];
+    if (v > mx) { sm = (mx == -INFINITY ? 0.f : sm * expf(mx - v)) + 1.f; mx = v; }
+    else sm += expf(v - mx);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float om = __shfl_xor_sync(0xffffffffu, mx, o), os = __shfl_xor_sync(0xffffffffu, sm, o);
+    lse_combine(mx, sm, om, os);
+  }
+  if (lane == 0) {
+    const long long k = (long long)b * rows + row;
+    shift[k] = mx;
+    if (mul) mul[k] = 1.0f / sm;
+    if (sum) sum[k] = sm;
+  }
+}
+
+int launch_row_stats(int H, int rows, int cols, const float* X, float* shift, float* mul, float* sum,
+                     cudaStream_t st) {
+  row_stats_kernel<<<dim3(cdiv(rows, 8), H), 256, 0, st>>>(X, shift, mul, sum, rows, cols);
+  return 1;
+}
+
+// out[i] = sum over slices (in slice order) of part[slice][i].
+__global__ void split_reduce_kernel(const float* part, float* out, long long count, int splits) {
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < count;
+       i += (long long)gridDim.x * blockDim.x) {
+    float a = 0.f;
+    for (int s = 0; s < splits; ++s) a += part[(long long)s * count + i];
+    out[i] = a;
+  }
+}
+
+int launch_split_reduce(int H, int M, int N, int splits, const float* part, float* out, cudaStream_t st) {
+  const long long count = (long long)H * M * N;
+  split_reduce_kernel<<<min(cdiv(count, 256), 152 * 16), 256, 0, st>>>(part, out, count, splits);
+  return 1;
+}
+
+}  // namespace arckv

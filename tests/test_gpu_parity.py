@@ -1,0 +1,233 @@
+"""GPU-vs-oracle parity of arckv_compact / arckv_attend through the C ABI.
+
+Tolerances are those stated in ``oracle/parity.py``.  Integer decisions
+(anchors, assignment) are compared tie-aware; the floating-point outputs of
+the merge and the fits are compared on the oracle's own decisions, passed to
+the GPU through ``anchors_in`` / ``assign_in``.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from oracle import parity
+import paper_2609_36835_gb300 as pk
+from paper_2609_36835_gb300 import workload
+
+pytestmark = pytest.mark.gpu
+
+BAND = 1e-5   # relative score gap at the t-th score inside which anchors may trade places
+TAU = 1e-4    # similarity gap inside which the assignment may differ (fp32 profile GEMM)
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu(lib):
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    torch.cuda.set_device(0)
+
+
+def _ocfg(cfg: pk.Config):
+    return oracle.OracleConfig(t=cfg.t, lambda_m=cfg.lambda_m, scale=(cfg.logit_scale or None),
+                               ridge_w=cfg.ridge_w, ridge_v=cfg.ridge_v, eps_w=cfg.eps_w, b_min=cfg.b_min,
+                               b_max=cfg.b_max, G=cfg.G)
+
+
+def _pair64(arr, h, G):
+    f64 = synth.bf16_to_f64
+    K, V, Q = f64(arr["K"][h]), f64(arr["V"][h]), f64(arr["Q"][h])
+    Xr = np.repeat(f64(arr["X"]), G, axis=0)
+    W = {f: f64(arr[f][h]) for f in pk.INDEXER_FIELDS}
+    return K, V, Q, Xr, W
+
+
+def _run(cfg, ten, **kw):
+    out = pk.compact_layer(cfg, ten["K"], ten["V"], ten["Q"], ten["X"], workload.indexer_dict(ten), **kw)
+    torch.cuda.synchronize()
+    return out
+
+
+def _np(x):
+    return x.detach().cpu().numpy()
+
+
+def check_layer(w, heads, sample, T=None, n_pos=None, t=None, layer=0, n_hold=64, **cfgkw):
+    """Full path on all ``heads``; oracle comparison on the ``sample`` heads."""
+    arr = workload.layer_inputs_np(w, layer, heads, T=T, n_pos=n_pos)
+    ten = workload.to_device(arr, "cuda")
+    cfg = workload.layer_config(w, len(heads), T=T, n_pos=n_pos, t=t, **cfgkw)
+    out = _run(cfg, ten, want_scores=True, want_assign=True)
+    scale = cfg.logit_scale or 1.0 / np.sqrt(cfg.d)
+    refs = {}
+    for h in sample:
+        K, V, Q, Xr, W = _pair64(arr, h, cfg.G)
+        ref = oracle.compact_pair(K, V, Q, Xr, W, _ocfg(cfg), H_I=cfg.H_I)
+        refs[h] = ref
+        e_inf, e_top = parity.score_errors(_np(out["scores"][h]).astype(np.float64), ref["scores"], cfg.t)
+        assert e_inf <= 1e-3 and e_top <= 1e-3, ("scores", h, e_inf, e_top)
+        ok, nd, gap = parity.anchors_match(_np(out["anchors"][h]), ref["anchors"], ref["scores"], cfg.t, BAND)
+        assert ok, ("anchors", h, nd, gap)
+    # downstream stages on the oracle's decisions (other heads keep the GPU's own)
+    S_in = out["anchors"].clone()
+    A_in = out["assign"].clone()
+    for h in sample:
+        S_in[h] = torch.as_tensor(refs[h]["anchors"], dtype=torch.int32)
+        A_in[h] = torch.as_tensor(refs[h]["assign"], dtype=torch.int32)
+    out2 = _run(cfg, ten, anchors_in=S_in, assign_in=A_in)
+    out3 = _run(cfg, ten, anchors_in=S_in, want_assign=True)
+    Qh = np.stack([synth.make_heldout(w, layer, h, arr["K"][i], n_hold) for i, h in enumerate(heads)])
+    O = pk.attend(workload.bf16_tensor(Qh, "cuda"), out2["C_k"], out2["beta"], out2["C_v"], cfg.logit_scale)
+    for h in sample:
+        ref = refs[h]
+        assert parity.rel_fro(_np(out2["C_k"][h]), ref["C_k"]) <= 2e-3
+        eb, rest_ok = parity.beta_errors(_np(out2["beta"][h]), ref["beta"], ref["w_star"])
+        assert eb <= 2e-3 and rest_ok, ("beta", h, eb, rest_ok)
+        assert parity.rel_fro(_np(out2["C_v"][h]), ref["C_v"]) <= 2e-3
+        O_ref = oracle.compact_attention(synth.bf16_to_f64(Qh[h]), ref["C_k"], ref["beta"], ref["C_v"], scale)
+        assert parity.rel_fro(_np(O[h]), O_ref) <= 2e-3
+        K, V, Q, Xr, W = _pair64(arr, h, cfg.G)
+        u, _ = oracle.response_profiles(oracle.attention_logits(Q, K, scale))
+        sim = u.T @ u[:, ref["anchors"]]
+        ok, n_mis, n_tie, worst = parity.assignment_valid(_np(out3["assign"][h]), sim, ref["anchors"], TAU)
+        assert ok, ("assign", h, n_mis, n_tie, worst)
+    return cfg, arr, ten, out, out2
+
+
+def test_small_single_head_workload():
+    """T = 1024, one KV head, n = 256, t = 102 (the small workload in full)."""
+    check_layer(synth.WORKLOADS["single_head_T1024"], [0], [0])
+
+
+def test_ragged_tiles_two_heads():
+    """T, n and t not multiples of the 128-wide tiles; two heads batched."""
+    check_layer(synth.WORKLOADS["llama8b_layer_T8192"], [0, 3], [0, 1], T=1000, n_pos=50, t=77)
+
+
+def test_full_llama_layer_sampled_heads():
+    """One Llama-3.1-8B layer at full size (8 KV heads, T = 8192, n = 1024,
+    t = 819) in the launch configuration the benchmark times; oracle on two heads."""
+    check_layer(synth.WORKLOADS["llama8b_layer_T8192"], list(range(8)), [0, 7])
+
+
+def test_full_context_layer_retention_2pct():
+    w = synth.WORKLOADS["llama8b_T8192_r02"]
+    check_layer(w, list(range(8)), [5], layer=17)
+
+
+def test_odd_shapes_single_index_head():
+    """One index head, a narrow activation width and sizes off every tile."""
+    w = synth.Workload("odd_shapes", 11, 1, 2, 333, 7, 5, shape=synth.IndexerShape(H_I=1, d_x=72))
+    check_layer(w, [0, 1], [1])
+
+
+@pytest.mark.parametrize("t", [1, 2])
+def test_tiny_budgets(t):
+    check_layer(synth.WORKLOADS["single_head_T1024"], [0], [0], T=200, n_pos=16, t=t)
+
+
+@pytest.mark.parametrize("lam", [0.0, 1.0])
+def test_merge_endpoints(lam):
+    w = synth.WORKLOADS["single_head_T1024"]
+    cfg, arr, ten, out, out2 = check_layer(w, [0], [0], T=500, n_pos=32, t=40, lambda_m=lam)
+    if lam == 0.0:   # C_k = K_S exactly
+        K = synth.bf16_to_f32(arr["K"][0])
+        S = _np(out["anchors"][0])
+        assert np.array_equal(_np(_run(cfg, ten)["C_k"][0]), K[S])
+
+
+def test_identity_budget_reproduces_cache():
+    """t = T: every group is a singleton, so C_k = K bit for bit; with a
+    well-conditioned logit scale and no ridge, beta ~ 0 and C_v ~ V."""
+    w = synth.WORKLOADS["single_head_T1024"]
+    arr = workload.layer_inputs_np(w, 0, [0], T=64, n_pos=64)
+    ten = workload.to_device(arr, "cuda")
+    cfg = workload.layer_config(w, 1, T=64, n_pos=64, t=64, logit_scale=0.005, ridge_w=0.0, ridge_v=0.0,
+                                lambda_m=0.6)
+    out = _run(cfg, ten)
+    K = synth.bf16_to_f32(arr["K"][0])
+    assert np.array_equal(_np(out["anchors"][0]), np.arange(64))
+    assert np.array_equal(_np(out["C_k"][0]), K)
+    assert np.max(np.abs(_np(out["beta"][0]))) <= 1e-3
+    assert parity.rel_fro(_np(out["C_v"][0]), synth.bf16_to_f32(arr["V"][0])) <= 2e-3
+
+
+def test_bitwise_reproducible():
+    w = synth.WORKLOADS["llama8b_layer_T8192"]
+    arr = workload.layer_inputs_np(w, 1, [0, 1], T=2048, n_pos=64)
+    ten = workload.to_device(arr, "cuda")
+    cfg = workload.layer_config(w, 2, T=2048, n_pos=64, t=205)
+    a = _run(cfg, ten, want_scores=True, want_assign=True)
+    b = _run(cfg, ten, want_scores=True, want_assign=True)
+    for k in ("scores", "anchors", "assign", "C_k", "beta", "C_v"):
+        assert torch.equal(a[k], b[k]), k
+
+
+def test_nonblocking_then_query_status():
+    w = synth.WORKLOADS["single_head_T1024"]
+    arr = workload.layer_inputs_np(w, 0, [0], T=256, n_pos=16)
+    ten = workload.to_device(arr, "cuda")
+    cfg = workload.layer_config(w, 1, T=256, n_pos=16, t=20, flags=pk.FLAG_NONBLOCKING)
+    ws = torch.empty(pk.workspace_bytes(cfg), dtype=torch.uint8, device="cuda")
+    out = _run(cfg, ten, ws=ws)
+    assert out["status"] == 0
+    assert pk.arckv_query_status(ws) == 0
+    blocking = workload.layer_config(w, 1, T=256, n_pos=16, t=20)
+    ref = _run(blocking, ten)
+    assert torch.equal(out["C_v"], ref["C_v"])
+
+
+def test_nonfinite_input_is_reported():
+    w = synth.WORKLOADS["single_head_T1024"]
+    arr = workload.layer_inputs_np(w, 0, [0], T=256, n_pos=16)
+    ten = workload.to_device(arr, "cuda")
+    ten["K"][0, 17, 3] = float("nan")
+    cfg = workload.layer_config(w, 1, T=256, n_pos=16, t=20)
+    out = _run(cfg, ten, check=False)
+    assert out["status"] == 5
+    # the context stays usable
+    ten2 = workload.to_device(arr, "cuda")
+    assert _run(cfg, ten2)["status"] == 0
+
+
+def test_singular_fit_returns_not_spd():
+    """Q = 0 makes every logit 0 and Phi_C the all-ones matrix, whose Gram
+    n 11^T is singular for t >= 2; with ridge_w = 0 the factorisation meets an
+    exactly zero pivot and the call returns ARCKV_ERR_NOT_SPD."""
+    w = synth.WORKLOADS["single_head_T1024"]
+    arr = workload.layer_inputs_np(w, 0, [0], T=128, n_pos=64)
+    ten = workload.to_device(arr, "cuda")
+    ten["Q"].zero_()
+    cfg = workload.layer_config(w, 1, T=128, n_pos=64, t=4, ridge_w=0.0)
+    S = torch.tensor([[0, 1, 2, 3]], dtype=torch.int32, device="cuda")
+    out = _run(cfg, ten, anchors_in=S, check=False)
+    assert out["status"] == 4
+    assert _run(workload.layer_config(w, 1, T=128, n_pos=64, t=4), workload.to_device(arr, "cuda"))["status"] == 0
+
+
+def test_invalid_overrides_are_rejected_on_device():
+    w = synth.WORKLOADS["single_head_T1024"]
+    arr = workload.layer_inputs_np(w, 0, [0], T=128, n_pos=8)
+    ten = workload.to_device(arr, "cuda")
+    cfg = workload.layer_config(w, 1, T=128, n_pos=8, t=4)
+    bad = torch.tensor([[5, 3, 9, 400]], dtype=torch.int32, device="cuda")
+    assert _run(cfg, ten, anchors_in=bad, check=False)["status"] == 1
+    S = torch.tensor([[1, 5, 9, 100]], dtype=torch.int32, device="cuda")
+    A = torch.full((1, 128), 7, dtype=torch.int32, device="cuda")
+    assert _run(cfg, ten, anchors_in=S, assign_in=A, check=False)["status"] == 1
+    assert _run(cfg, ten)["status"] == 0
+
+
+@pytest.mark.parametrize("H,n,t", [(3, 200, 77), (1, 1, 1), (2, 130, 300)])
+def test_attend_matches_oracle(H, n, t):
+    rng = np.random.default_rng(H * 1000 + t)
+    Qb = synth.bf16_round((rng.normal(size=(H, n, 128)) * 3).astype(np.float32))
+    Ck = rng.normal(size=(H, t, 128)).astype(np.float32)
+    beta = rng.normal(size=(H, t)).astype(np.float32)
+    Cv = rng.normal(size=(H, t, 128)).astype(np.float32)
+    O = pk.attend(workload.bf16_tensor(Qb, "cuda"), torch.from_numpy(Ck).cuda(), torch.from_numpy(beta).cuda(),
+                  torch.from_numpy(Cv).cuda())
+    for h in range(H):
+        ref = oracle.compact_attention(synth.bf16_to_f64(Qb[h]), Ck[h].astype(np.float64),
+                                       beta[h].astype(np.float64), Cv[h].astype(np.float64), 1.0 / np.sqrt(128))
+        assert parity.rel_fro(_np(O[h]), ref) <= 2e-3
