@@ -174,6 +174,36 @@ arckv_status arckv_attend(int32_t H_kv, int32_t n, int32_t t, int32_t d, float l
                           const void* Q, const float* C_k, const float* beta, const float* C_v,
                           float* O, void* ws, size_t ws_bytes, uint32_t flags, void* stream);
 
+/*
+ * Allocation-free compact attention.  The paper has no counterpart: this is a
+ * deployment variant of arckv_attend for callers that cannot allocate device
+ * memory when they call it -- for example an inference-engine plugin whose
+ * execute step must not allocate, or a serving loop that has fixed its memory
+ * budget up front and cannot risk an allocation failing or fragmenting memory
+ * mid-request.  It computes exactly what arckv_attend computes, with the same
+ * kernels, arguments (minus the workspace) and errors.
+ *
+ * Scratch: one fixed array of ARCKV_ATTEND_STATIC_MAX_FLOATS floats (32 MiB)
+ * compiled into libarckv.so as a device global.  Every GPU on which the library
+ * is loaded holds it until the process exits; the call itself allocates
+ * nothing (no cudaMalloc, no allocating library routine).  A problem needs
+ * arckv_attend_static_floats(H_kv, n, t, d) floats of it; larger problems are
+ * rejected with ARCKV_ERR_WORKSPACE before anything is enqueued.
+ *
+ * The first call on a device looks up the array's device address with that
+ * device current (cudaGetSymbolAddress) and caches it; make that first call
+ * before any stream capture.  All calls share the one array and it keeps the
+ * previous call's contents (the call clears what must start at zero): calls
+ * whose GPU work overlaps -- on different streams, or from several host
+ * threads -- race on it, so serialise them.  The call always synchronises
+ * `stream` and returns the device status.
+ */
+#define ARCKV_ATTEND_STATIC_MAX_FLOATS (8u << 20)
+size_t arckv_attend_static_floats(int32_t H_kv, int32_t n, int32_t t, int32_t d);
+arckv_status arckv_attend_static(int32_t H_kv, int32_t n, int32_t t, int32_t d, float logit_scale,
+                                 const void* Q, const float* C_k, const float* beta, const float* C_v,
+                                 float* O, void* stream);
+
 /* Read (and clear) the device status word of a workspace after a
  * non-blocking call; synchronises `stream`. */
 arckv_status arckv_query_status(void* ws, void* stream);

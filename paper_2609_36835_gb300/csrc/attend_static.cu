@@ -1,0 +1,75 @@
+// arckv_attend_static: compact attention with no caller workspace and no
+// allocation at call time.  Its scratch is one file-scope __device__ array
+// that the CUDA module loader places in every context that loads this
+// library; the array stays resident until the process exits.
+#include <algorithm>
+#include <mutex>
+
+#include "kernels.h"
+
+namespace {
+
+// status word (256 bytes) + compact logits + split-K partials, in floats
+constexpr size_t kStaticScratchFloats = ARCKV_ATTEND_STATIC_MAX_FLOATS;
+
+__device__ __align__(256) float g_attend_scratch[kStaticScratchFloats];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+float* g_scratch_addr[kMaxDevices];  // per device, filled by the first call on that device
+
+// The symbol's device address, looked up once per device with that device
+// current.  In host code `g_attend_scratch` names a host-side shadow, never
+// the device memory, so kernels only ever receive this looked-up address.
+arckv_status scratch_for_current_device(float** out) {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return ARCKV_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_mu);
+  if (!g_scratch_addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_attend_scratch) != cudaSuccess || !p) return ARCKV_ERR_CUDA;
+    g_scratch_addr[dev] = (float*)p;
+  }
+  *out = g_scratch_addr[dev];
+  return ARCKV_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t arckv_attend_static_floats(int32_t H_kv, int32_t n, int32_t t, int32_t d) {
+  if (H_kv < 1 || n < 1 || t < 1 || d != 128) return 0;
+  const size_t splits = (size_t)std::max(1, std::min(arckv::kSplitK, (t + 127) / 128));
+  return 64 + ((size_t)H_kv * n * t + 63) / 64 * 64 + splits * H_kv * n * 128;
+}
+
+arckv_status arckv_attend_static(int32_t H_kv, int32_t n, int32_t t, int32_t d, float logit_scale, const void* Q,
+                                 const float* C_k, const float* beta, const float* C_v, float* O, void* stream) {
+  if (d != 128) return ARCKV_ERR_UNSUPPORTED;
+  const size_t need = arckv_attend_static_floats(H_kv, n, t, d);
+  if (need == 0) return ARCKV_ERR_SHAPE;
+  if (need > kStaticScratchFloats) return ARCKV_ERR_WORKSPACE;
+  if (!Q || !C_k || !beta || !C_v || !O) return ARCKV_ERR_INVALID_ARG;
+  if (!(logit_scale >= 0.f) || !isfinite(logit_scale)) return ARCKV_ERR_INVALID_ARG;
+  float* base = nullptr;
+  arckv_status s = scratch_for_current_device(&base);
+  if (s != ARCKV_OK) return s;
+  cudaStream_t st = (cudaStream_t)stream;
+  arckv::DevStatus* stt = (arckv::DevStatus*)base;
+  float* LC = base + 64;
+  float* split = LC + ((size_t)H_kv * n * t + 63) / 64 * 64;
+  const float scale = logit_scale > 0.f ? logit_scale : 1.0f / sqrtf((float)d);
+  cudaGetLastError();
+  // the array keeps the previous call's contents: the status word must start at zero
+  if (cudaMemsetAsync(stt, 0, sizeof(arckv::DevStatus), st) != cudaSuccess) return ARCKV_ERR_CUDA;
+  arckv::launch_attend(H_kv, n, t, scale, (const arckv::bf16*)Q, C_k, beta, C_v, O, LC, split, st);
+  arckv::launch_check_finite(O, (long long)H_kv * n * d, stt, st);
+  if (cudaGetLastError() != cudaSuccess) return ARCKV_ERR_CUDA;
+  unsigned int code = 0;
+  if (cudaMemcpyAsync(&code, stt, sizeof(code), cudaMemcpyDeviceToHost, st) != cudaSuccess) return ARCKV_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return ARCKV_ERR_CUDA;
+  return (arckv_status)code;
+}
+
+}  // extern "C"
