@@ -15,7 +15,7 @@ inline size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct Layout {
   size_t status, kbar, Uk, Uv, vq, cctx, qbar, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
-      US, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, split, total;
+      US, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z, split, total;
 };
 
 Dims dims_of(const arckv_config& c) {
@@ -85,6 +85,9 @@ Layout plan(const arckv_config& c) {
   L.Gram = take(H * t * t * f);
   L.Linv = take(H * nblk * kCholNB * kCholNB * f);
   L.rhs = take(H * t * f);
+  L.wsol = take(H * t * f);
+  L.R = take(H * t * 128 * f);
+  L.Z = take(H * t * 128 * f);
   L.split = take((size_t)kSplitK * H * (n > t ? n : t) * 128 * f);
   L.total = o;
   return L;
@@ -202,7 +205,7 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
   nl += launch_merge(D, cfg->lambda_m, Kb, anchors, kappa, F(L.logphi), I32(L.perm), I32(L.goff), I32(L.cursor),
                      C_k, st);
   mark(5);
-  FitBufs B{F(L.LC), F(L.Phi), F(L.Gram), F(L.Linv), F(L.rhs), F(L.split)};
+  FitBufs B{F(L.LC), F(L.Phi), F(L.Gram), F(L.Linv), F(L.rhs), F(L.wsol), F(L.R), F(L.Z), F(L.split)};
   nl += launch_fits(D, scale, cfg->ridge_w, cfg->ridge_v, cfg->eps_w, cfg->b_min, cfg->b_max, Qb, C_k, F(L.z),
                     F(L.m), F(L.Y), B, beta, C_v, stt, st);
   nl += launch_check_finite(C_k, (long long)D.H * D.t * D.d, stt, st);

@@ -60,6 +60,10 @@ __global__ void ridge_kernel(float* Gram, int t, float ridge, DevStatus* stt) {
 
 // Factor the (already updated) diagonal block k in shared memory, write L_kk
 // into A and its inverse into Linv[b][k] (64 x 64, identity beyond the matrix).
+// Left-looking by columns: at column c every row r >= c forms
+// A_rc - sum_{q<c} L_rq L_cq with four threads per row, the pivot row takes the
+// square root and the rows below divide.  The inverse is formed row by row:
+// Li_ij = (delta_ij - sum_{l=j}^{i-1} L_il Li_lj) / L_ii, all j of a row at once.
 __global__ void __launch_bounds__(256) potrf_diag_kernel(float* A, int t, int k, float* Linv, int nblk,
                                                          DevStatus* stt) {
   const int b = blockIdx.x, tid = threadIdx.x;
@@ -71,42 +75,43 @@ __global__ void __launch_bounds__(256) potrf_diag_kernel(float* A, int t, int k,
   for (int e = tid; e < NB * NB; e += 256) {
     const int r = e / NB, c = e % NB;
     L[r][c] = (r < kb && c <= r) ? Ab[(long long)(k0 + r) * t + k0 + c] : (r == c ? 1.f : 0.f);
+    Li[r][c] = 0.f;
   }
   if (tid == 0) bad = 0;
   __syncthreads();
+  const int r = tid >> 2, p = tid & 3;
   for (int c = 0; c < NB; ++c) {
-    if (tid == 0) {
-      float p = L[c][c];
-      if (!(p > 0.f) || !isfinite(p)) { bad = 1; p = 1.f; }
-      L[c][c] = sqrtf(p);
+    // columns < c are final (the previous iteration ended with a barrier)
+    float v = 0.f;
+    if (r >= c)
+      for (int q = p; q < c; q += 4) v = fmaf(L[r][q], L[c][q], v);
+    v += __shfl_xor_sync(0xffffffffu, v, 1);
+    v += __shfl_xor_sync(0xffffffffu, v, 2);
+    v = (r >= c) ? L[r][c] - v : 0.f;
+    if (r == c && p == 0) {
+      if (!(v > 0.f) || !isfinite(v)) { bad = 1; v = 1.f; }
+      L[c][c] = sqrtf(v);
     }
     __syncthreads();
-    const float dinv = 1.0f / L[c][c];
-    for (int r = c + 1 + tid; r < NB; r += 256) L[r][c] *= dinv;
-    __syncthreads();
-    const int w = NB - c - 1;
-    for (int e = tid; e < w * w; e += 256) {
-      const int rr = c + 1 + e / w, cc = c + 1 + e % w;
-      if (cc <= rr) L[rr][cc] = fmaf(-L[rr][c], L[cc][c], L[rr][cc]);
-    }
+    if (r > c && p == 0) L[r][c] = v / L[c][c];
     __syncthreads();
   }
   if (tid == 0 && bad) set_status(stt, ARCKV_ERR_NOT_SPD);
-  if (tid < NB) {
-    const int j = tid;
-    for (int i = 0; i < NB; ++i) {
-      if (i < j) { Li[i][j] = 0.f; continue; }
-      float s = (i == j) ? 1.f : 0.f;
-      for (int l = j; l < i; ++l) s = fmaf(-L[i][l], Li[l][j], s);
-      Li[i][j] = s / L[i][i];
-    }
+  const int j = tid >> 2;
+  for (int i = 0; i < NB; ++i) {
+    float v = 0.f;
+    if (j < i)
+      for (int l = j + p; l < i; l += 4) v = fmaf(L[i][l], Li[l][j], v);
+    v += __shfl_xor_sync(0xffffffffu, v, 1);
+    v += __shfl_xor_sync(0xffffffffu, v, 2);
+    if (j <= i && p == 0) Li[i][j] = ((i == j ? 1.f : 0.f) - v) / L[i][i];
+    __syncthreads();
   }
-  __syncthreads();
   float* Lo = Linv + ((long long)b * nblk + k) * NB * NB;
   for (int e = tid; e < NB * NB; e += 256) {
-    const int r = e / NB, c = e % NB;
-    Lo[e] = Li[r][c];
-    if (r < kb && c <= r) Ab[(long long)(k0 + r) * t + k0 + c] = L[r][c];
+    const int rr = e / NB, cc = e % NB;
+    Lo[e] = Li[rr][cc];
+    if (rr < kb && cc <= rr) Ab[(long long)(k0 + rr) * t + k0 + cc] = L[rr][cc];
   }
 }
 
@@ -139,164 +144,198 @@ __global__ void __launch_bounds__(256) trsm_kernel(float* A, int t, int k, const
   }
 }
 
-// A_ij -= L_ik L_jk^T for the lower blocks k < j <= i of the trailing matrix.
-__global__ void __launch_bounds__(256) syrk_kernel(float* A, int t, int k) {
-  const int b = blockIdx.y, tid = threadIdx.x;
-  const int x = blockIdx.x;
-  int ii = (int)((sqrtf(8.f * x + 1.f) - 1.f) * 0.5f);
-  while (ii * (ii + 1) / 2 > x) --ii;
-  while ((ii + 1) * (ii + 2) / 2 <= x) ++ii;
-  const int jj = x - ii * (ii + 1) / 2;
-  const int i0 = (k + 1 + ii) * NB, j0 = (k + 1 + jj) * NB, k0 = k * NB;
-  const int rb = min(NB, t - i0), cb = min(NB, t - j0);
-  float* Ab = A + (long long)b * t * t;
-  __shared__ float Li[NB][NB + 1];
-  __shared__ float Lj[NB][NB + 1];
-  for (int e = tid; e < NB * NB; e += 256) {
-    const int r = e / NB, c = e % NB;
-    Li[r][c] = (r < rb) ? Ab[(long long)(i0 + r) * t + k0 + c] : 0.f;
-    Lj[r][c] = (r < cb) ? Ab[(long long)(j0 + r) * t + k0 + c] : 0.f;
+// 64 x 64 tile product helper: acc[p][q] += sum_l X[ry+p][l] * Y[l][cx+q] with
+// X, Y in shared memory ([64][65] layout), ry = (tid>>4)*4, cx = (tid&15)*4.
+__device__ __forceinline__ void tile_mm(const float (*X)[NB + 1], const float (*Y)[NB + 1], float (&acc)[4][4],
+                                        bool transX) {
+  const int ry = (threadIdx.x >> 4) * 4, cx = (threadIdx.x & 15) * 4;
+  for (int l = 0; l < NB; ++l) {
+    float a[4], c[4];
+#pragma unroll
+    for (int p = 0; p < 4; ++p) { a[p] = transX ? X[l][ry + p] : X[ry + p][l]; c[p] = Y[l][cx + p]; }
+#pragma unroll
+    for (int p = 0; p < 4; ++p)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) acc[p][q] = fmaf(a[p], c[q], acc[p][q]);
   }
-  __syncthreads();
+}
+
+// Trailing update of step k.  Blocks [0, ntri): A_ij -= L_ik L_jk^T for the
+// lower blocks k < j <= i.  Blocks [ntri, ntri + m * nct): the forward
+// substitution of the right-hand side B (t x nrhs, row stride ldb):
+// B_i -= L_ik (Linv_kk B_k) for block rows i > k and 64-column tiles of B.
+// B_k itself is only read in this launch (every tile recomputes Linv_kk B_k).
+__global__ void __launch_bounds__(256) update_kernel(float* A, int t, int k, const float* Linv, int nblk,
+                                                     float* B, int ldb, int nrhs, long long bbs) {
+  const int b = blockIdx.y, tid = threadIdx.x;
+  const int m = nblk - k - 1, ntri = m * (m + 1) / 2, k0 = k * NB;
+  float* Ab = A + (long long)b * t * t;
+  __shared__ float S1[NB][NB + 1];
+  __shared__ float S2[NB][NB + 1];
   const int ry = (tid >> 4) * 4, cx = (tid & 15) * 4;
   float acc[4][4];
 #pragma unroll
   for (int p = 0; p < 4; ++p)
 #pragma unroll
     for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
-  for (int l = 0; l < NB; ++l) {
-    float a[4], c[4];
-#pragma unroll
-    for (int p = 0; p < 4; ++p) { a[p] = Li[ry + p][l]; c[p] = Lj[cx + p][l]; }
+  const int x = blockIdx.x;
+  if (x < ntri) {
+    int ii = (int)((sqrtf(8.f * x + 1.f) - 1.f) * 0.5f);
+    while (ii * (ii + 1) / 2 > x) --ii;
+    while ((ii + 1) * (ii + 2) / 2 <= x) ++ii;
+    const int jj = x - ii * (ii + 1) / 2;
+    const int i0 = (k + 1 + ii) * NB, j0 = (k + 1 + jj) * NB;
+    const int rb = min(NB, t - i0), cb = min(NB, t - j0);
+    for (int e = tid; e < NB * NB; e += 256) {
+      const int r = e / NB, c = e % NB;
+      S1[r][c] = (r < rb) ? Ab[(long long)(i0 + r) * t + k0 + c] : 0.f;   // L_ik
+      S2[c][r] = (r < cb) ? Ab[(long long)(j0 + r) * t + k0 + c] : 0.f;   // L_jk^T
+    }
+    __syncthreads();
+    tile_mm(S1, S2, acc, false);
 #pragma unroll
     for (int p = 0; p < 4; ++p)
 #pragma unroll
-      for (int q = 0; q < 4; ++q) acc[p][q] = fmaf(a[p], c[q], acc[p][q]);
+      for (int q = 0; q < 4; ++q)
+        if (ry + p < rb && cx + q < cb) Ab[(long long)(i0 + ry + p) * t + j0 + cx + q] -= acc[p][q];
+    return;
   }
+  const int nct = (nrhs + NB - 1) / NB;
+  const int y = x - ntri, i = k + 1 + y / nct, c0 = (y % nct) * NB;
+  const int i0 = i * NB, rb = min(NB, t - i0), nc = min(NB, nrhs - c0);
+  float* Bb = B + (long long)b * bbs;
+  const float* Lk = Linv + ((long long)b * nblk + k) * NB * NB;
+  for (int e = tid; e < NB * NB; e += 256) {
+    const int r = e / NB, c = e % NB;
+    S1[r][c] = Lk[e];
+    S2[r][c] = (c < nc) ? Bb[(long long)(k0 + r) * ldb + c0 + c] : 0.f;   // block k is full (k < nblk-1)
+  }
+  __syncthreads();
+  tile_mm(S1, S2, acc, false);   // y = Linv_kk B_k
+  __syncthreads();
+#pragma unroll
+  for (int p = 0; p < 4; ++p)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) S2[ry + p][cx + q] = acc[p][q];
+  for (int e = tid; e < NB * NB; e += 256) {
+    const int r = e / NB, c = e % NB;
+    S1[r][c] = (r < rb) ? Ab[(long long)(i0 + r) * t + k0 + c] : 0.f;    // L_ik
+  }
+  __syncthreads();
+#pragma unroll
+  for (int p = 0; p < 4; ++p)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
+  tile_mm(S1, S2, acc, false);
 #pragma unroll
   for (int p = 0; p < 4; ++p)
 #pragma unroll
     for (int q = 0; q < 4; ++q)
-      if (ry + p < rb && cx + q < cb) Ab[(long long)(i0 + ry + p) * t + j0 + cx + q] -= acc[p][q];
+      if (ry + p < rb && cx + q < nc) Bb[(long long)(i0 + ry + p) * ldb + c0 + cx + q] -= acc[p][q];
 }
 
-// Solve L L^T X = B in place (X holds B), columns [32 blockIdx.x, +32) of an
-// nrhs-column right-hand side with row stride ldx; one CTA per (column tile, head).
-__global__ void __launch_bounds__(256) chol_solve_kernel(const float* A, const float* Linv, float* X, int t,
-                                                         int ldx, int nrhs, long long xbs, int nblk) {
+// Backward substitution, step k (block rows from the last down): with
+// Y_k = Linv_kk B_k (B after the forward updates) and Z_k the accumulated
+// -sum_{j>k} L_jk^T X_j,  X_k = Linv_kk^T (Y_k + Z_k).  Block (i = k) writes X_k;
+// blocks i < k apply Z_i -= L_ki^T X_k.  B_k and Z_k are only read here.
+__global__ void __launch_bounds__(256) backward_kernel(const float* A, int t, int k, const float* Linv, int nblk,
+                                                       const float* B, float* Z, float* X, int ldb, int nrhs,
+                                                       long long bbs) {
   const int b = blockIdx.y, tid = threadIdx.x;
-  const int c0 = blockIdx.x * 32, nc = min(32, nrhs - c0);
+  const int nct = (nrhs + NB - 1) / NB;
+  const int i = blockIdx.x / nct, c0 = (blockIdx.x % nct) * NB;
+  const int k0 = k * NB, kb = min(NB, t - k0), nc = min(NB, nrhs - c0);
   const float* Ab = A + (long long)b * t * t;
-  const float* Lb = Linv + (long long)b * nblk * NB * NB;
-  float* Xb = X + (long long)b * xbs;
-  __shared__ float Lt[NB][NB + 1];
-  __shared__ float Yt[NB][33];
-  const int r = tid >> 2, cc = (tid & 3) * 8;
-  float acc[8];
-  // forward: Y_k = Linv_kk (B_k - sum_{j<k} L_kj Y_j)
-  for (int k = 0; k < nblk; ++k) {
-    const int k0 = k * NB, kb = min(NB, t - k0);
+  const float* Bb = B + (long long)b * bbs;
+  float* Zb = Z + (long long)b * bbs;
+  float* Xb = X + (long long)b * bbs;
+  const float* Lk = Linv + ((long long)b * nblk + k) * NB * NB;
+  __shared__ float S1[NB][NB + 1];
+  __shared__ float S2[NB][NB + 1];
+  const int ry = (tid >> 4) * 4, cx = (tid & 15) * 4;
+  float acc[4][4];
 #pragma unroll
-    for (int q = 0; q < 8; ++q)
-      acc[q] = (r < kb && cc + q < nc) ? Xb[(long long)(k0 + r) * ldx + c0 + cc + q] : 0.f;
-    for (int j = 0; j < k; ++j) {
-      const int j0 = j * NB;
-      __syncthreads();
-      for (int e = tid; e < NB * NB; e += 256) {
-        const int rr = e / NB, l = e % NB;
-        Lt[rr][l] = (rr < kb) ? Ab[(long long)(k0 + rr) * t + j0 + l] : 0.f;
-      }
-      for (int e = tid; e < NB * 32; e += 256) {
-        const int l = e >> 5, c = e & 31;
-        Yt[l][c] = (c < nc) ? Xb[(long long)(j0 + l) * ldx + c0 + c] : 0.f;
-      }
-      __syncthreads();
-      for (int l = 0; l < NB; ++l) {
-        const float a = Lt[r][l];
+  for (int p = 0; p < 4; ++p)
 #pragma unroll
-        for (int q = 0; q < 8; ++q) acc[q] = fmaf(-a, Yt[l][cc + q], acc[q]);
-      }
-    }
-    __syncthreads();
-    const float* Lk = Lb + (long long)k * NB * NB;
-    for (int e = tid; e < NB * NB; e += 256) Lt[e / NB][e % NB] = Lk[e];
-#pragma unroll
-    for (int q = 0; q < 8; ++q) Yt[r][cc + q] = acc[q];
-    __syncthreads();
-#pragma unroll
-    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
-    for (int l = 0; l <= r; ++l) {
-      const float a = Lt[r][l];
-#pragma unroll
-      for (int q = 0; q < 8; ++q) acc[q] = fmaf(a, Yt[l][cc + q], acc[q]);
-    }
-#pragma unroll
-    for (int q = 0; q < 8; ++q)
-      if (r < kb && cc + q < nc) Xb[(long long)(k0 + r) * ldx + c0 + cc + q] = acc[q];
-    __syncthreads();
+    for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
+  for (int e = tid; e < NB * NB; e += 256) {
+    const int r = e / NB, c = e % NB;
+    S1[r][c] = Lk[e];
+    S2[r][c] = (r < kb && c < nc) ? Bb[(long long)(k0 + r) * ldb + c0 + c] : 0.f;
   }
-  // backward: X_k = Linv_kk^T (Y_k - sum_{j>k} L_jk^T X_j)
-  for (int k = nblk - 1; k >= 0; --k) {
-    const int k0 = k * NB, kb = min(NB, t - k0);
+  __syncthreads();
+  tile_mm(S1, S2, acc, false);          // Y_k = Linv_kk B_k
+  __syncthreads();
 #pragma unroll
-    for (int q = 0; q < 8; ++q)
-      acc[q] = (r < kb && cc + q < nc) ? Xb[(long long)(k0 + r) * ldx + c0 + cc + q] : 0.f;
-    for (int j = k + 1; j < nblk; ++j) {
-      const int j0 = j * NB, jb = min(NB, t - j0);
-      __syncthreads();
-      for (int e = tid; e < NB * NB; e += 256) {
-        const int l = e / NB, rr = e % NB;
-        Lt[l][rr] = (l < jb) ? Ab[(long long)(j0 + l) * t + k0 + rr] : 0.f;
-      }
-      for (int e = tid; e < NB * 32; e += 256) {
-        const int l = e >> 5, c = e & 31;
-        Yt[l][c] = (l < jb && c < nc) ? Xb[(long long)(j0 + l) * ldx + c0 + c] : 0.f;
-      }
-      __syncthreads();
-      for (int l = 0; l < NB; ++l) {
-        const float a = Lt[l][r];
+  for (int p = 0; p < 4; ++p)
 #pragma unroll
-        for (int q = 0; q < 8; ++q) acc[q] = fmaf(-a, Yt[l][cc + q], acc[q]);
-      }
-    }
-    __syncthreads();
-    const float* Lk = Lb + (long long)k * NB * NB;
-    for (int e = tid; e < NB * NB; e += 256) Lt[e / NB][e % NB] = Lk[e];
+    for (int q = 0; q < 4; ++q)
+      S2[ry + p][cx + q] = acc[p][q] + ((ry + p < kb && cx + q < nc)
+                                            ? Zb[(long long)(k0 + ry + p) * ldb + c0 + cx + q] : 0.f);
+  __syncthreads();
 #pragma unroll
-    for (int q = 0; q < 8; ++q) Yt[r][cc + q] = acc[q];
-    __syncthreads();
+  for (int p = 0; p < 4; ++p)
 #pragma unroll
-    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
-    for (int l = r; l < NB; ++l) {
-      const float a = Lt[l][r];
+    for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
+  tile_mm(S1, S2, acc, true);           // X_k = Linv_kk^T (Y_k + Z_k)
+  if (i == k) {
 #pragma unroll
-      for (int q = 0; q < 8; ++q) acc[q] = fmaf(a, Yt[l][cc + q], acc[q]);
-    }
+    for (int p = 0; p < 4; ++p)
 #pragma unroll
-    for (int q = 0; q < 8; ++q)
-      if (r < kb && cc + q < nc) Xb[(long long)(k0 + r) * ldx + c0 + cc + q] = acc[q];
-    __syncthreads();
+      for (int q = 0; q < 4; ++q)
+        if (ry + p < kb && cx + q < nc) Xb[(long long)(k0 + ry + p) * ldb + c0 + cx + q] = acc[p][q];
+    return;
   }
+  __syncthreads();
+#pragma unroll
+  for (int p = 0; p < 4; ++p)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) S2[ry + p][cx + q] = acc[p][q];
+  const int i0 = i * NB;   // i < k: a full block
+  for (int e = tid; e < NB * NB; e += 256) {
+    const int r = e / NB, c = e % NB;
+    S1[r][c] = (r < kb) ? Ab[(long long)(k0 + r) * t + i0 + c] : 0.f;     // L_ki[r][c]
+  }
+  __syncthreads();
+#pragma unroll
+  for (int p = 0; p < 4; ++p)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
+  tile_mm(S1, S2, acc, true);           // L_ki^T X_k
+#pragma unroll
+  for (int p = 0; p < 4; ++p)
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      if (cx + q < nc) Zb[(long long)(i0 + ry + p) * ldb + c0 + cx + q] -= acc[p][q];
 }
 
-static int cholesky_solve(int H, int t, float* Gram, float* Linv, float* X, int ldx, int nrhs, long long xbs,
-                          float ridge, DevStatus* stt, cudaStream_t st) {
+// Solve (Gram + lam I) X = B for each head: ridge, blocked Cholesky with the
+// forward substitution of B fused into the trailing updates, then backward
+// substitution.  B (t x nrhs, stride ldb) is overwritten; Z is scratch of the
+// same shape; X receives the solution.
+static int cholesky_solve(int H, int t, float* Gram, float* Linv, float* B, float* Z, float* X, int ldb,
+                          int nrhs, long long bbs, float ridge, DevStatus* stt, cudaStream_t st) {
   int nl = 0;
   ridge_kernel<<<H, 256, 0, st>>>(Gram, t, ridge, stt);
   ++nl;
-  const int nblk = cdiv(t, NB);
+  const int nblk = cdiv(t, NB), nct = cdiv(nrhs, NB);
   for (int k = 0; k < nblk; ++k) {
     potrf_diag_kernel<<<H, 256, 0, st>>>(Gram, t, k, Linv, nblk, stt);
     ++nl;
     const int m = nblk - k - 1;
     if (m > 0) {
       trsm_kernel<<<dim3(m, H), 256, 0, st>>>(Gram, t, k, Linv, nblk);
-      syrk_kernel<<<dim3(m * (m + 1) / 2, H), 256, 0, st>>>(Gram, t, k);
+      update_kernel<<<dim3(m * (m + 1) / 2 + m * nct, H), 256, 0, st>>>(Gram, t, k, Linv, nblk, B, ldb, nrhs,
+                                                                          bbs);
       nl += 2;
     }
   }
-  chol_solve_kernel<<<dim3(cdiv(nrhs, 32), H), 256, 0, st>>>(Gram, Linv, X, t, ldx, nrhs, xbs, nblk);
-  return nl + 1;
+  cudaMemsetAsync(Z, 0, sizeof(float) * (size_t)H * bbs, st);
+  for (int k = nblk - 1; k >= 0; --k) {
+    backward_kernel<<<dim3((k + 1) * nct, H), 256, 0, st>>>(Gram, t, k, Linv, nblk, B, Z, X, ldb, nrhs, bbs);
+    ++nl;
+  }
+  return nl;
 }
 
 __global__ void beta_kernel(const float* w, float* beta, long long count, float eps_w, float b_min, float b_max) {
@@ -342,9 +381,9 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
   ++nl;
   mass_rhs_kernel<<<dim3(cdiv(D.t, 128), D.H), 128, 0, st>>>(B.Phi, m, B.rhs, D.n, D.t);
   ++nl;
-  nl += cholesky_solve(D.H, D.t, B.Gram, B.Linv, B.rhs, 1, 1, D.t, ridge_w, stt, st);
+  nl += cholesky_solve(D.H, D.t, B.Gram, B.Linv, B.rhs, B.Z, B.wsol, 1, 1, D.t, ridge_w, stt, st);
   const long long ht = (long long)D.H * D.t;
-  beta_kernel<<<cdiv(ht, 256), 256, 0, st>>>(B.rhs, beta, ht, eps_w, b_min, b_max);
+  beta_kernel<<<cdiv(ht, 256), 256, 0, st>>>(B.wsol, beta, ht, eps_w, b_min, b_max);
   ++nl;
   // value system: P^ over the compact keys with the fitted bias
   softmax_bias_kernel<<<dim3(cdiv(D.n, 8), D.H), 256, 0, st>>>(B.LC, beta, B.Phi, D.n, D.t);
@@ -356,8 +395,8 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
   launch_gemm(ColK<float>{B.Phi, nt, D.t}, ColK<float>{Y, nd, D.d},
               EpiStore{B.split, td, (long long)D.H * td, D.d, 1.f, false}, D.H, D.t, D.d, D.n, kSplitK, st);
   ++nl;
-  nl += launch_split_reduce(D.H, D.t, D.d, kSplitK, B.split, C_v, st);
-  nl += cholesky_solve(D.H, D.t, B.Gram, B.Linv, C_v, D.d, D.d, td, ridge_v, stt, st);
+  nl += launch_split_reduce(D.H, D.t, D.d, kSplitK, B.split, B.R, st);
+  nl += cholesky_solve(D.H, D.t, B.Gram, B.Linv, B.R, B.Z, C_v, D.d, D.d, td, ridge_v, stt, st);
   return nl;
 }
 

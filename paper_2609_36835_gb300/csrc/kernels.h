@@ -45,7 +45,7 @@ int launch_merge(const Dims& D, float lambda_m, const bf16* K, const int* anchor
 
 // ---- fits (App. A.9) -----------------------------------------------------
 struct FitBufs {
-  float *LC, *Phi, *Gram, *Linv, *rhs, *split;
+  float *LC, *Phi, *Gram, *Linv, *rhs, *wsol, *R, *Z, *split;
 };
 int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float eps_w, float b_min,
                 float b_max, const bf16* Q, const float* C_k, const float* z, const float* m,

@@ -12,34 +12,53 @@
 
 namespace arckv {
 
-// One thread per column j: M_j = max_i l_ij, s1 = sum_i e^{l_ij - M_j},
-// s2 = sum_i e^{2(l_ij - M_j)}; log phi_j = M_j + log s1 - log n; then
-// U_ij = e^{l_ij - M_j} / sqrt(s2) is written over l.
-__global__ void __launch_bounds__(128) col_stats_kernel(float* L, float* logphi, int n, int T) {
-  const int b = blockIdx.y, j = blockIdx.x * 128 + threadIdx.x;
-  if (j >= T) return;
+// Column statistics, 32 columns per CTA and 8 row slices per column: each
+// (slice, column) thread keeps an online (M, s1, s2) over its rows, the eight
+// slices are combined in slice order, then
+//   M_j = max_i l_ij,  s1 = sum_i e^{l_ij - M_j},  s2 = sum_i e^{2(l_ij - M_j)},
+//   log phi_j = M_j + log s1 - log n,
+// and U_ij = e^{l_ij - M_j} / sqrt(s2) is written over l.
+__global__ void __launch_bounds__(256) col_stats_kernel(float* L, float* logphi, int n, int T) {
+  const int b = blockIdx.y, lane = threadIdx.x & 31, slice = threadIdx.x >> 5;
+  const int j = blockIdx.x * 32 + lane;
+  __shared__ float sm[8][32], s1s[8][32], s2s[8][32];
   float* Lb = L + (long long)b * n * T + j;
+  const int rows = (n + 7) / 8, i0 = slice * rows, i1 = min(n, i0 + rows);
   float mx = -INFINITY, s1 = 0.f, s2 = 0.f;
-#pragma unroll 4
-  for (int i = 0; i < n; ++i) {
-    const float v = Lb[(long long)i * T];
-    if (v > mx) {
-      const float r = (mx == -INFINITY) ? 0.f : expf(mx - v);
-      s1 = fmaf(s1, r, 1.f);
-      s2 = fmaf(s2, r * r, 1.f);
-      mx = v;
-    } else {
-      const float e = expf(v - mx);
-      s1 += e;
-      s2 = fmaf(e, e, s2);
+  if (j < T) {
+    for (int i = i0; i < i1; ++i) {
+      const float v = Lb[(long long)i * T];
+      if (v > mx) {
+        const float r = (mx == -INFINITY) ? 0.f : expf(mx - v);
+        s1 = fmaf(s1, r, 1.f);
+        s2 = fmaf(s2, r * r, 1.f);
+        mx = v;
+      } else {
+        const float e = expf(v - mx);
+        s1 += e;
+        s2 = fmaf(e, e, s2);
+      }
     }
   }
-  logphi[(long long)b * T + j] = mx + logf(s1) - logf((float)n);
-  const float inv = 1.0f / sqrtf(s2);
-#pragma unroll 4
-  for (int i = 0; i < n; ++i) {
-    float* p = Lb + (long long)i * T;
-    *p = expf(*p - mx) * inv;
+  sm[slice][lane] = mx;
+  s1s[slice][lane] = s1;
+  s2s[slice][lane] = s2;
+  __syncthreads();
+  float M = -INFINITY;
+  for (int q = 0; q < 8; ++q) M = fmaxf(M, sm[q][lane]);
+  float S1 = 0.f, S2 = 0.f;
+  for (int q = 0; q < 8; ++q) {
+    if (sm[q][lane] == -INFINITY) continue;
+    const float r = expf(sm[q][lane] - M);
+    S1 = fmaf(s1s[q][lane], r, S1);
+    S2 = fmaf(s2s[q][lane], r * r, S2);
+  }
+  if (j >= T) return;
+  if (slice == 0) logphi[(long long)b * T + j] = M + logf(S1) - logf((float)n);
+  const float inv = 1.0f / sqrtf(S2);
+  for (int i = i0; i < i1; ++i) {
+    float* q = Lb + (long long)i * T;
+    *q = expf(*q - M) * inv;
   }
 }
 
@@ -57,7 +76,7 @@ int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const 
   launch_gemm(P, ColK<bf16>{V, Td, D.d}, EpiStore{split, nd, (long long)D.H * nd, D.d, 1.f, false}, D.H, D.n,
               D.d, D.T, kSplitK, st);
   launch_split_reduce(D.H, D.n, D.d, kSplitK, split, Y, st);
-  col_stats_kernel<<<dim3(cdiv(D.T, 128), D.H), 128, 0, st>>>(L, logphi, D.n, D.T);
+  col_stats_kernel<<<dim3(cdiv(D.T, 32), D.H), 256, 0, st>>>(L, logphi, D.n, D.T);
   return 5;
 }
 
@@ -203,26 +222,32 @@ __global__ void __launch_bounds__(1024) group_sort_kernel(const int* kappa, int 
   }
 }
 
-// One warp per group r: mu_r = sum_{G_r} w_j k_j / sum_{G_r} w_j with
-// w_j = e^{log phi_j - max_{G_r} log phi} (Eq. mass_centroid), members summed in
-// ascending position order; c_r = k_{s_r} + lambda_m (mu_r - k_{s_r}), which is
+// One CTA per group r: mu_r = sum_{G_r} w_j k_j / sum_{G_r} w_j with
+// w_j = e^{log phi_j - max_{G_r} log phi} (Eq. mass_centroid).  Warp w sums the
+// members w, w+8, ... (ascending position order inside G_r) over 4 dims per
+// lane; the eight partial sums are added in warp order, so the result does not
+// depend on scheduling.  c_r = k_{s_r} + lambda_m (mu_r - k_{s_r}), which is
 // (1 - lambda_m) k_{s_r} + lambda_m mu_r of Eq. key_merge.
 __global__ void __launch_bounds__(256) group_merge_kernel(const bf16* K, const int* anchors, const int* perm,
                                                           const int* goff, const float* logphi, float lambda_m,
                                                           float* C_k, int T, int t) {
-  const int b = blockIdx.y, r = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
-  if (r >= t) return;
+  const int b = blockIdx.y, r = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int* pb = perm + (long long)b * T;
   const int* gb = goff + (long long)b * (t + 1);
   const float* lp = logphi + (long long)b * T;
   const bf16* Kb = K + (long long)b * T * 128;
   const int beg = gb[r], end = gb[r + 1];
+  __shared__ float red[8][129];
+  __shared__ float gmax_s[8];
   float gm = -INFINITY;
-  for (int q = beg + lane; q < end; q += 32) gm = fmaxf(gm, lp[pb[q]]);
+  for (int q = beg + threadIdx.x; q < end; q += 256) gm = fmaxf(gm, lp[pb[q]]);
   gm = warp_max(gm);
+  if (lane == 0) gmax_s[warp] = gm;
+  __syncthreads();
+  gm = gmax_s[0];
+  for (int w = 1; w < 8; ++w) gm = fmaxf(gm, gmax_s[w]);
   float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f, ws = 0.f;
-#pragma unroll 4
-  for (int q = beg; q < end; ++q) {
+  for (int q = beg + warp; q < end; q += 8) {
     const int j = pb[q];
     const float om = expf(lp[j] - gm);
     const uint2 raw = *(const uint2*)(Kb + (long long)j * 128 + lane * 4);
@@ -233,24 +258,28 @@ __global__ void __launch_bounds__(256) group_merge_kernel(const bf16* K, const i
     a3 = fmaf(om, to_f32(h[3]), a3);
     ws += om;
   }
+  red[warp][lane * 4 + 0] = a0;
+  red[warp][lane * 4 + 1] = a1;
+  red[warp][lane * 4 + 2] = a2;
+  red[warp][lane * 4 + 3] = a3;
+  if (lane == 0) red[warp][128] = ws;
+  __syncthreads();
+  if (threadIdx.x >= 128) return;
+  const int dcol = threadIdx.x;
+  float acc = 0.f, wsum = 0.f;
+  for (int w = 0; w < 8; ++w) {
+    acc += red[w][dcol];
+    wsum += red[w][128];
+  }
   const int s = anchors[(long long)b * t + r];
-  const uint2 raw = *(const uint2*)(Kb + (long long)s * 128 + lane * 4);
-  const bf16* h = (const bf16*)&raw;
-  const float k0 = to_f32(h[0]), k1 = to_f32(h[1]), k2 = to_f32(h[2]), k3 = to_f32(h[3]);
-  const float iw = 1.0f / ws;
-  float4 c;
-  c.x = fmaf(lambda_m, a0 * iw - k0, k0);
-  c.y = fmaf(lambda_m, a1 * iw - k1, k1);
-  c.z = fmaf(lambda_m, a2 * iw - k2, k2);
-  c.w = fmaf(lambda_m, a3 * iw - k3, k3);
-  *(float4*)(C_k + ((long long)b * t + r) * 128 + lane * 4) = c;
+  const float k = to_f32(Kb[(long long)s * 128 + dcol]);
+  C_k[((long long)b * t + r) * 128 + dcol] = fmaf(lambda_m, acc * (1.0f / wsum) - k, k);
 }
 
 int launch_merge(const Dims& D, float lambda_m, const bf16* K, const int* anchors, const int* kappa,
                  const float* logphi, int* perm, int* goff, int* cursor, float* C_k, cudaStream_t st) {
   group_sort_kernel<<<D.H, 1024, 0, st>>>(kappa, D.T, D.t, perm, goff, cursor);
-  group_merge_kernel<<<dim3(cdiv(D.t, 8), D.H), 256, 0, st>>>(K, anchors, perm, goff, logphi, lambda_m, C_k,
-                                                              D.T, D.t);
+  group_merge_kernel<<<dim3(D.t, D.H), 256, 0, st>>>(K, anchors, perm, goff, logphi, lambda_m, C_k, D.T, D.t);
   return 2;
 }
 

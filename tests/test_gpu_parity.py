@@ -137,19 +137,24 @@ def test_merge_endpoints(lam):
 
 
 def test_identity_budget_reproduces_cache():
-    """t = T: every group is a singleton, so C_k = K bit for bit; with a
-    well-conditioned logit scale and no ridge, beta ~ 0 and C_v ~ V."""
+    """t = T: every group is a singleton, so C_k = K bit for bit.  With the
+    keys themselves as reference queries (Gaussian keys, no attention sink)
+    Phi_C is near the identity and the unregularised fits are well
+    conditioned, so beta = 0 and C_v = V up to fp32 rounding."""
     w = synth.WORKLOADS["single_head_T1024"]
-    arr = workload.layer_inputs_np(w, 0, [0], T=64, n_pos=64)
+    arr = workload.layer_inputs_np(w, 0, [0], T=64, n_pos=16)
+    rng = np.random.default_rng(5)
+    arr["K"] = synth.bf16_round(rng.normal(size=(1, 64, 128)).astype(np.float32))
+    arr["V"] = synth.bf16_round(rng.normal(size=(1, 64, 128)).astype(np.float32))
+    arr["Q"] = arr["K"].copy()
     ten = workload.to_device(arr, "cuda")
-    cfg = workload.layer_config(w, 1, T=64, n_pos=64, t=64, logit_scale=0.005, ridge_w=0.0, ridge_v=0.0,
-                                lambda_m=0.6)
+    cfg = workload.layer_config(w, 1, T=64, n_pos=16, t=64, ridge_w=0.0, ridge_v=0.0, lambda_m=0.6)
     out = _run(cfg, ten)
     K = synth.bf16_to_f32(arr["K"][0])
     assert np.array_equal(_np(out["anchors"][0]), np.arange(64))
     assert np.array_equal(_np(out["C_k"][0]), K)
-    assert np.max(np.abs(_np(out["beta"][0]))) <= 1e-3
-    assert parity.rel_fro(_np(out["C_v"][0]), synth.bf16_to_f32(arr["V"][0])) <= 2e-3
+    assert np.max(np.abs(_np(out["beta"][0]))) <= 1e-5
+    assert parity.rel_fro(_np(out["C_v"][0]), synth.bf16_to_f32(arr["V"][0])) <= 1e-5
 
 
 def test_bitwise_reproducible():
