@@ -34,9 +34,26 @@ if str(ROOT) not in sys.path:
 METRIC = "compaction s/context and context tokens/s at Llama-3.1-8B shape; % roofline"
 UNIT = "context tokens/s"
 DEFAULT_WORKLOAD = "llama8b_T8192_r10"
-SM_COUNT, FP32_LANES_PER_SM = 152, 128
-PROFILE_SUMMARY = ROOT / "profiles" / "index_logits_llama8b_layer_T8192.md"
-DOMINANT_SOURCE = ROOT / "paper_2609_36835_gb300" / "csrc" / "indexer.cu"
+PROFILE_SUMMARY = ROOT / "profiles" / "index_logits_tc_llama8b_layer_T8192.md"
+DOMINANT_SOURCES = [ROOT / "paper_2609_36835_gb300" / "csrc" / f for f in ("tc_index.cu", "tc_gemm.cuh", "tc.cuh")]
+FALLBACK_BF16_SUSTAINED_TFLOPS = 1700.0
+
+
+def measured_peaks():
+    """Measured GB300 peaks (MEASURED_PEAKS.json), else the fallback."""
+    p = ROOT / "MEASURED_PEAKS.json"
+    try:
+        d = json.loads(p.read_text())
+        return float(d["bf16_tflops_sustained"]), float(d["hbm_gbs"]), "measured"
+    except (OSError, ValueError, KeyError):
+        return FALLBACK_BF16_SUSTAINED_TFLOPS, 6800.0, "fallback"
+
+
+def dominant_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in DOMINANT_SOURCES:
+        h.update(f.read_bytes())
+    return h.hexdigest()
 
 
 def parse_args(argv=None):
@@ -201,8 +218,7 @@ def profiled_traffic():
     h = re.search(r"source_sha256:\s*([0-9a-f]{64})", text)
     if not m or not h:
         return None
-    cur = hashlib.sha256(DOMINANT_SOURCE.read_bytes()).hexdigest()
-    return float(m.group(1)) if h.group(1) == cur else None
+    return float(m.group(1)) if h.group(1) == dominant_source_hash() else None
 
 
 # ------------------------------------------------------------ reference arm
@@ -336,17 +352,18 @@ def run_gpu(args, dist: Dist):
             logits_ms.append(evs[1].elapsed_time(evs[2]))
     stage_ms = [x / args.steps for x in stage_ms]
 
-    # roofline of the dominant kernel (index logits, one launch per layer)
+    # roofline of the dominant kernel (index logits, one launch per layer): a
+    # split-bf16 tcgen05 GEMM issuing three bf16 MMAs per useful product
     flops = 2.0 * w.H_kv * w.n * w.T * w.shape.H_I * w.shape.d_I
     avg_s = statistics.mean(logits_ms) / 1e3
-    sm_max = 2070.0
-    peak_fp32 = SM_COUNT * FP32_LANES_PER_SM * 2 * sm_max * 1e6 / 1e12
+    peak, _, peak_src = measured_peaks()
     achieved = flops / avg_s / 1e12
-    traffic = profiled_traffic()
-    roofline = {"kernel": "index_logits_kernel", "bound": "alu", "achieved": achieved, "peak": peak_fp32,
-                "unit": "TFLOP/s", "frac": achieved / peak_fp32, "traffic": traffic,
-                "flops_per_launch": flops, "launch_ms": avg_s * 1e3,
-                "peak_note": "fp32 FMA: 152 SMs x 128 lanes x 2 flop x 2070 MHz (derived, not measured)"}
+    roofline = {"kernel": "tc_gemm_kernel<128, split, TcEpiIndex> (index logits, Eq. pairwise_index_score)",
+                "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                "traffic": profiled_traffic(), "flops_per_launch": flops, "launch_ms": avg_s * 1e3,
+                "issued_tflops": 3.0 * achieved, "issued_frac": 3.0 * achieved / peak,
+                "peak_note": "bf16 dense, sustained, of %s (MEASURED_PEAKS.json); achieved counts useful flops, "
+                             "issued counts the 3 bf16 MMAs of each split-bf16 product" % peak_src}
 
     # end to end: pinned host inputs -> device -> compaction -> host outputs, every step
     pinned = [workload.to_device(a, pin=True) for a in host]

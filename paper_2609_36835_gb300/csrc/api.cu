@@ -14,8 +14,8 @@ constexpr size_t kAlign = 256;
 inline size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct Layout {
-  size_t status, kbar, Uk, Uv, vq, cctx, qbar, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
-      US, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z, split, total;
+  size_t status, kbar_hi, kbar_lo, Uk, Uv, vq, cctx, qbar_hi, qbar_lo, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
+      colM, colInvN, Ut_hi, Ut_lo, S_hi, S_lo, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z, split, total;
 };
 
 Dims dims_of(const arckv_config& c) {
@@ -55,12 +55,14 @@ Layout plan(const arckv_config& c) {
   size_t o = 0;
   auto take = [&](size_t bytes) { size_t r = o; o += up(bytes); return r; };
   L.status = take(sizeof(DevStatus));
-  L.kbar = take(H * T * HD * f);
+  L.kbar_hi = take(H * T * HD * 2);
+  L.kbar_lo = take(H * T * HD * 2);
   L.Uk = take(H * T * 128 * f);
   L.Uv = take(H * T * 128 * f);
   L.vq = take(H * n * 128 * f);
   L.cctx = take(H * n * 128 * f);
-  L.qbar = take(H * n * HD * f);
+  L.qbar_hi = take(H * n * HD * 2);
+  L.qbar_lo = take(H * n * HD * 2);
   L.wts = take(H * (size_t)D.n_pos * D.H_I * f);
   L.NT = take(H * n * T * f);
   L.rA = take(H * n * f);
@@ -74,7 +76,13 @@ Layout plan(const arckv_config& c) {
   L.invm = take(H * n * f);
   L.Y = take(H * n * 128 * f);
   L.logphi = take(H * T * f);
-  L.US = take(H * n * t * f);
+  const size_t ldn = (n + 7) / 8 * 8;
+  L.colM = take(H * T * f);
+  L.colInvN = take(H * T * f);
+  L.Ut_hi = take(H * T * ldn * 2);
+  L.Ut_lo = take(H * T * ldn * 2);
+  L.S_hi = take(H * t * ldn * 2);
+  L.S_lo = take(H * t * ldn * 2);
   L.best = take(H * T * 8);
   L.kappa = take(H * T * 4);
   L.perm = take(H * T * 4);
@@ -174,14 +182,18 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
   int* anchors = I32(L.anchors);
   mark(0);
   if (!given_anchors) {
+    auto B16 = [&](size_t off) { return (bf16*)(w + off); };
     nl += launch_key_features(D, Kb, Vb, (const bf16*)idx->L_k, (const bf16*)idx->L_v, (const bf16*)idx->U_k,
-                              (const bf16*)idx->U_v, F(L.kbar), F(L.Uk), F(L.Uv), st);
+                              (const bf16*)idx->U_v, B16(L.kbar_hi), B16(L.kbar_lo), F(L.Uk), F(L.Uv), st);
     nl += launch_query_features(D, Qb, (const bf16*)X_ref, (const bf16*)idx->U_q, (const bf16*)idx->L_q,
                                 (const bf16*)idx->L_c, (const bf16*)idx->L_x, (const bf16*)idx->b_x, F(L.Uk),
-                                F(L.Uv), F(L.vq), F(L.NT), F(L.rA), F(L.rB), F(L.split), F(L.cctx), F(L.qbar),
-                                F(L.wts), st);
+                                F(L.Uv), F(L.vq), F(L.NT), F(L.rA), F(L.rB), F(L.split), F(L.cctx),
+                                B16(L.qbar_hi), B16(L.qbar_lo), F(L.wts), st);
     mark(1);
-    nl += launch_index_logits(D, F(L.qbar), F(L.kbar), F(L.wts), F(L.NT), (float2*)(w + L.part), st);
+    const int nli = launch_index_logits(D, B16(L.qbar_hi), B16(L.qbar_lo), B16(L.kbar_hi), B16(L.kbar_lo),
+                                        F(L.wts), F(L.NT), (float2*)(w + L.part), stt, st);
+    if (nli < 0) return ARCKV_ERR_CUDA;
+    nl += nli;
     mark(2);
     nl += launch_index_pool(D, F(L.NT), (const float2*)(w + L.part), F(L.lse), F(L.s), st);
     nl += launch_top_t(D, F(L.s), anchors, stt, st);
@@ -192,11 +204,17 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
     nl += launch_check_anchors(D, anchors, stt, st);
   }
   mark(3);
-  nl += launch_reference_attention(D, scale, Qb, Kb, Vb, F(L.NT), F(L.z), F(L.m), F(L.invm), F(L.split), F(L.Y),
-                                   F(L.logphi), st);
+  const int nlr = launch_reference_attention(D, scale, Qb, Kb, Vb, F(L.NT), F(L.z), F(L.m), F(L.invm), F(L.split),
+                                             F(L.Y), F(L.logphi), F(L.colM), F(L.colInvN), stt, st);
+  if (nlr < 0) return ARCKV_ERR_CUDA;
+  nl += nlr;
   int* kappa = I32(L.kappa);
   if (!given_assign) {
-    nl += launch_assign(D, F(L.NT), anchors, F(L.US), (unsigned long long*)(w + L.best), kappa, st);
+    auto B16 = [&](size_t off) { return (bf16*)(w + off); };
+    const int nla = launch_assign_tc(D, F(L.NT), F(L.colM), F(L.colInvN), anchors, B16(L.Ut_hi), B16(L.Ut_lo),
+                                     B16(L.S_hi), B16(L.S_lo), (unsigned long long*)(w + L.best), kappa, stt, st);
+    if (nla < 0) return ARCKV_ERR_CUDA;
+    nl += nla;
   } else {
     cudaMemcpyAsync(kappa, aux->assign_in, sizeof(int) * (size_t)D.H * D.T, cudaMemcpyDeviceToDevice, st);
     nl += launch_check_assign(D, kappa, anchors, stt, st);

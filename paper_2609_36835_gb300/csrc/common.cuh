@@ -33,6 +33,13 @@ __device__ __forceinline__ float f32_from_ordered(unsigned int u) {
   return __uint_as_float((u & 0x80000000u) ? (u & 0x7fffffffu) : ~u);
 }
 
+// bf16 pair (hi, lo) with hi = bf16(x) and lo = bf16(x - hi): x = hi + lo to
+// within 2^-16 relative, the operand format of the split tensor-core GEMMs.
+__device__ __forceinline__ void split_bf16(float x, bf16& hi, bf16& lo) {
+  hi = __float2bfloat16_rn(x);
+  lo = __float2bfloat16_rn(x - __bfloat162float(hi));
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);

@@ -264,34 +264,33 @@ struct EpiBlockNorm {
   }
 };
 
-// Row-wise argmax over the tile's columns, merged across column tiles with a
-// 64-bit atomicMax of (ordered value << 32) | (0xffffffff - column): the
-// largest value wins and equal values go to the smallest column.
-struct EpiArgmax {
-  unsigned long long* best;
-  long long bbs;
-  __device__ __forceinline__ void apply(int b, int, int m0, int n0, int M, int N, float (&acc)[8][8],
+// EpiBlockNorm with a split-bf16 output pair instead of fp32.
+struct EpiBlockNormSplit {
+  bf16* Hi;
+  bf16* Lo;
+  long long cbs;
+  int ldc;
+  __device__ __forceinline__ void apply(int b, int, int m0, int n0, int M, int, float (&acc)[8][8],
                                         float*) const {
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      float bv = -INFINITY;
-      int bn = 0x7fffffff;
+      float ss = 0.f;
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int n = n0 + tile_col(j);
-        if (n < N && (acc[i][j] > bv || (acc[i][j] == bv && n < bn))) { bv = acc[i][j]; bn = n; }
-      }
+      for (int j = 0; j < 8; ++j) ss = fmaf(acc[i][j], acc[i][j], ss);
 #pragma unroll
-      for (int o = 1; o < 16; o <<= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-        const int on = __shfl_xor_sync(0xffffffffu, bn, o);
-        if (ov > bv || (ov == bv && on < bn)) { bv = ov; bn = on; }
-      }
+      for (int o = 1; o < 16; o <<= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+      const float sc = 1.0f / sqrtf(ss * (1.0f / 128.0f) + 1e-6f);
       const int m = m0 + tile_row(i);
-      if ((threadIdx.x & 15) == 0 && m < M && bn != 0x7fffffff) {
-        const unsigned long long key =
-            ((unsigned long long)f32_ordered(bv) << 32) | (unsigned long long)(0xffffffffu - (unsigned int)bn);
-        atomicMax(best + (long long)b * bbs + m, key);
+      if (m >= M) continue;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int n = n0 + (threadIdx.x & 15) * 4 + h * 64;
+        const long long off = (long long)b * cbs + (long long)m * ldc + n;
+        __align__(8) bf16 hi[4], lo[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) split_bf16(acc[i][h * 4 + q] * sc, hi[q], lo[q]);
+        *(uint2*)(Hi + off) = *(const uint2*)hi;
+        *(uint2*)(Lo + off) = *(const uint2*)lo;
       }
     }
   }

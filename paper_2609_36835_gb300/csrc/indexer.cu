@@ -5,7 +5,7 @@
 // c_i = softmax_j((U_q q_i).(Uk_j)) Uv (Eq. value_context);
 // q_bar_i,a = N((L_q q_i + L_c c_i)_a); w_i,a = (L_x x_r + b_x)_a
 // (Eq. indexer_projection); I_ij = sum_a w_ia LeakyReLU_0.1(q_bar_ia.k_bar_ja / sqrt(d_I))
-// (Eq. pairwise_index_score); pi = row softmax of I and
+// (Eq. pairwise_index_score, in tc_index.cu); pi = row softmax of I and
 // s_j = (mean_i pi_ij^2)^(1/2) (Eq. indexer_pooling).
 #include "gemm.cuh"
 #include "kernels.h"
@@ -13,12 +13,14 @@
 namespace arckv {
 
 int launch_key_features(const Dims& D, const bf16* K, const bf16* V, const bf16* L_k, const bf16* L_v,
-                        const bf16* U_k, const bf16* U_v, float* kbar, float* Uk, float* Uv, cudaStream_t st) {
+                        const bf16* U_k, const bf16* U_v, bf16* kbar_hi, bf16* kbar_lo, float* Uk, float* Uv,
+                        cudaStream_t st) {
   const long long Td = (long long)D.T * D.d, Wd = (long long)D.HD * D.d;
-  // z = [k | v] [L_k | L_v]^T, RMS-normalised per 128-wide block
+  // z = [k | v] [L_k | L_v]^T, RMS-normalised per 128-wide block, stored as a split-bf16 pair
   CatRowK<bf16, bf16> A{{K, Td, D.d}, {V, Td, D.d}, D.d};
   CatRowK<bf16, bf16> B{{L_k, Wd, D.d}, {L_v, Wd, D.d}, D.d};
-  launch_gemm(A, B, EpiBlockNorm{kbar, (long long)D.T * D.HD, D.HD}, D.H, D.T, D.HD, 2 * D.d, 1, st);
+  launch_gemm(A, B, EpiBlockNormSplit{kbar_hi, kbar_lo, (long long)D.T * D.HD, D.HD}, D.H, D.T, D.HD, 2 * D.d, 1,
+              st);
   const long long Ud = (long long)D.d_A * D.d;
   launch_gemm(RowK<bf16>{K, Td, D.d}, RowK<bf16>{U_k, Ud, D.d},
               EpiStore{Uk, (long long)D.T * D.d_A, 0, D.d_A, 1.f, false}, D.H, D.T, D.d_A, D.d, 1, st);
@@ -52,7 +54,7 @@ __global__ void __launch_bounds__(256) index_weights_kernel(const bf16* X, const
 int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf16* U_q, const bf16* L_q,
                           const bf16* L_c, const bf16* L_x, const bf16* b_x, const float* Uk,
                           const float* Uv, float* vq, float* logits, float* rshift, float* rmul,
-                          float* split, float* cctx, float* qbar, float* wts, cudaStream_t st) {
+                          float* split, float* cctx, bf16* qbar_hi, bf16* qbar_lo, float* wts, cudaStream_t st) {
   int nl = 0;
   const long long nd = (long long)D.n * D.d, nA = (long long)D.n * D.d_A, TA = (long long)D.T * D.d_A;
   // vq = U_q q
@@ -73,83 +75,12 @@ int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf1
   // q_bar = N(L_q q + L_c c) per block
   CatRowK<bf16, float> A{{Q, nd, D.d}, {cctx, nA, D.d_A}, D.d};
   CatRowK<bf16, bf16> B{{L_q, (long long)D.HD * D.d, D.d}, {L_c, (long long)D.HD * D.d_A, D.d_A}, D.d};
-  launch_gemm(A, B, EpiBlockNorm{qbar, (long long)D.n * D.HD, D.HD}, D.H, D.n, D.HD, D.d + D.d_A, 1, st);
+  launch_gemm(A, B, EpiBlockNormSplit{qbar_hi, qbar_lo, (long long)D.n * D.HD, D.HD}, D.H, D.n, D.HD,
+              D.d + D.d_A, 1, st);
   ++nl;
   index_weights_kernel<<<dim3(D.n_pos, D.H), 256, 0, st>>>(X, L_x, b_x, wts, D.d_x, D.H_I, D.n_pos);
   ++nl;
   return nl;
-}
-
-// I tile = sum_a w_a LeakyReLU(q_bar_a k_bar_a^T / sqrt(d_I)); also writes the
-// per-(row, column tile) (max, sum exp) partials of the row softmax.
-__global__ void __launch_bounds__(GNT) index_logits_kernel(const float* qbar, const float* kbar,
-                                                           const float* wts, float* I, float2* part, int n,
-                                                           int T, int H_I, int G, int n_pos) {
-  __shared__ __align__(16) float sA[2 * GBK * GSST];
-  __shared__ __align__(16) float sB[2 * GBK * GSST];
-  const int b = blockIdx.z, m0 = blockIdx.y * GBM, n0 = blockIdx.x * GBN;
-  const int HD = H_I * 128;
-  RowK<float> la{qbar, (long long)n * HD, HD};
-  RowK<float> lb{kbar, (long long)T * HD, HD};
-  la.bind(b, m0, n);
-  lb.bind(b, n0, T);
-  float Iacc[8][8], acc[8][8];
-#pragma unroll
-  for (int i = 0; i < 8; ++i)
-#pragma unroll
-    for (int j = 0; j < 8; ++j) Iacc[i][j] = 0.f;
-  const float inv_sqrt_dI = 1.0f / sqrtf(128.0f);
-  const float* wb = wts + (long long)b * n_pos * H_I;
-  for (int a = 0; a < H_I; ++a) {
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-#pragma unroll
-      for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
-    gemm_mainloop(la, lb, a * 128, (a + 1) * 128, acc, sA, sB);
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int m = m0 + tile_row(i);
-      const float wv = (m < n) ? wb[(m / G) * H_I + a] : 0.f;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const float x = acc[i][j] * inv_sqrt_dI;
-        Iacc[i][j] = fmaf(wv, x >= 0.f ? x : 0.1f * x, Iacc[i][j]);
-      }
-    }
-  }
-  float* Ib = I + (long long)b * n * T;
-  const bool vec = (T & 3) == 0;
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int m = m0 + tile_row(i);
-    float mx = -INFINITY;
-#pragma unroll
-    for (int j = 0; j < 8; ++j)
-      if (n0 + tile_col(j) < T) mx = fmaxf(mx, Iacc[i][j]);
-    float sm = 0.f;
-#pragma unroll
-    for (int j = 0; j < 8; ++j)
-      if (n0 + tile_col(j) < T) sm += expf(Iacc[i][j] - mx);
-#pragma unroll
-    for (int o = 1; o < 16; o <<= 1) {
-      const float om = __shfl_xor_sync(0xffffffffu, mx, o), os = __shfl_xor_sync(0xffffffffu, sm, o);
-      lse_combine(mx, sm, om, os);
-    }
-    if (m >= n) continue;
-    if ((threadIdx.x & 15) == 0) part[((long long)b * n + m) * gridDim.x + blockIdx.x] = make_float2(mx, sm);
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int c = n0 + (threadIdx.x & 15) * 4 + h * 64;
-      float* dst = Ib + (long long)m * T + c;
-      if (vec && c + 4 <= T) {
-        *(float4*)dst = make_float4(Iacc[i][h * 4], Iacc[i][h * 4 + 1], Iacc[i][h * 4 + 2], Iacc[i][h * 4 + 3]);
-      } else {
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-          if (c + q < T) dst[q] = Iacc[i][h * 4 + q];
-      }
-    }
-  }
 }
 
 // lse[b][i] = log sum_j exp(I_ij) from the column-tile partials; one warp per row.
@@ -194,13 +125,6 @@ __global__ void __launch_bounds__(256) pool_kernel(const float* I, const float* 
     }
   }
   if (j < T) s[(long long)b * T + j] = sqrtf((a0 + a1) / (float)n);
-}
-
-int launch_index_logits(const Dims& D, const float* qbar, const float* kbar, const float* wts, float* I,
-                        float2* part, cudaStream_t st) {
-  dim3 grid(cdiv(D.T, GBN), cdiv(D.n, GBM), D.H);
-  index_logits_kernel<<<grid, GNT, 0, st>>>(qbar, kbar, wts, I, part, D.n, D.T, D.H_I, D.G, D.n_pos);
-  return 1;
 }
 
 int launch_index_pool(const Dims& D, const float* I, const float2* part, float* lse, float* s, cudaStream_t st) {

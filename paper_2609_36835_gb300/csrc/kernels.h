@@ -15,15 +15,19 @@ constexpr int kCholNB = 64;  // Cholesky block size
 // ---- indexer (Sec. 3.3, App. A.1) --------------------------------------
 // k_bar = N(L_k k + L_v v) per d_I block; Uk = U_k k; Uv = U_v v.
 int launch_key_features(const Dims& D, const bf16* K, const bf16* V, const bf16* L_k, const bf16* L_v,
-                        const bf16* U_k, const bf16* U_v, float* kbar, float* Uk, float* Uv, cudaStream_t st);
+                        const bf16* U_k, const bf16* U_v, bf16* kbar_hi, bf16* kbar_lo, float* Uk, float* Uv,
+                        cudaStream_t st);
 // value context c (Eq. value_context), q_bar (Eq. indexer_projection), w.
 int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf16* U_q, const bf16* L_q,
                           const bf16* L_c, const bf16* L_x, const bf16* b_x, const float* Uk,
                           const float* Uv, float* vq, float* logits, float* rshift, float* rmul,
-                          float* split, float* cctx, float* qbar, float* wts, cudaStream_t st);
-// I (Eq. pairwise_index_score) and per-(row, column tile) softmax partials.
-int launch_index_logits(const Dims& D, const float* qbar, const float* kbar, const float* wts, float* I,
-                        float2* part, cudaStream_t st);
+                          float* split, float* cctx, bf16* qbar_hi, bf16* qbar_lo, float* wts, cudaStream_t st);
+// I (Eq. pairwise_index_score) on tcgen05 with split-bf16 operands, and the
+// per-(row, 128-column tile) softmax partials.  Returns launches, or -1 when a
+// TMA descriptor cannot be encoded.
+int launch_index_logits(const Dims& D, const bf16* qbar_hi, const bf16* qbar_lo, const bf16* kbar_hi,
+                        const bf16* kbar_lo, const float* wts, float* I, float2* part, DevStatus* stt,
+                        cudaStream_t st);
 // row log-sum-exp and pooled s (Eq. indexer_pooling).
 int launch_index_pool(const Dims& D, const float* I, const float2* part, float* lse, float* s, cudaStream_t st);
 
@@ -32,13 +36,18 @@ int launch_top_t(const Dims& D, const float* s, int* anchors, DevStatus* stt, cu
 int launch_check_anchors(const Dims& D, int* anchors, DevStatus* stt, cudaStream_t st);
 
 // ---- reference attention, assignment, merge (Sec. 3.4) ------------------
-// l = scale Q K^T into `L`; z, m (row max / mass); Y = softmax(l) V;
-// column statistics log phi and the normalised profiles U written over `L`.
+// l = scale Q K^T into `L` (tcgen05); z, m (row max / mass); Y = softmax(l) V;
+// column statistics log phi, M_j and 1/||e^{l_:j - M_j}||.  -1 when a TMA
+// descriptor cannot be encoded.
 int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const bf16* K, const bf16* V,
                                float* L, float* z, float* m, float* invm, float* split, float* Y,
-                               float* logphi, cudaStream_t st);
-int launch_assign(const Dims& D, const float* U, const int* anchors, float* US, unsigned long long* best,
-                  int* kappa, cudaStream_t st);
+                               float* logphi, float* colM, float* colInvN, DevStatus* stt, cudaStream_t st);
+int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* K, float* L, DevStatus* stt,
+                         cudaStream_t st);
+// Assignment on tcgen05: transposed split-bf16 profiles, anchor rows, argmax GEMM.
+int launch_assign_tc(const Dims& D, const float* L, const float* colM, const float* colInvN, const int* anchors,
+                     bf16* Ut_hi, bf16* Ut_lo, bf16* S_hi, bf16* S_lo, unsigned long long* best, int* kappa,
+                     DevStatus* stt, cudaStream_t st);
 int launch_check_assign(const Dims& D, int* kappa, const int* anchors, DevStatus* stt, cudaStream_t st);
 int launch_merge(const Dims& D, float lambda_m, const bf16* K, const int* anchors, const int* kappa,
                  const float* logphi, int* perm, int* goff, int* cursor, float* C_k, cudaStream_t st);

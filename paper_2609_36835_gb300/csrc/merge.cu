@@ -16,13 +16,14 @@ namespace arckv {
 // (slice, column) thread keeps an online (M, s1, s2) over its rows, the eight
 // slices are combined in slice order, then
 //   M_j = max_i l_ij,  s1 = sum_i e^{l_ij - M_j},  s2 = sum_i e^{2(l_ij - M_j)},
-//   log phi_j = M_j + log s1 - log n,
-// and U_ij = e^{l_ij - M_j} / sqrt(s2) is written over l.
-__global__ void __launch_bounds__(256) col_stats_kernel(float* L, float* logphi, int n, int T) {
+//   log phi_j = M_j + log s1 - log n,  invN_j = 1 / sqrt(s2),
+// so that the normalised profile is U_ij = e^{l_ij - M_j} invN_j.
+__global__ void __launch_bounds__(256) col_stats_kernel(const float* L, float* logphi, float* colM,
+                                                        float* colInvN, int n, int T) {
   const int b = blockIdx.y, lane = threadIdx.x & 31, slice = threadIdx.x >> 5;
   const int j = blockIdx.x * 32 + lane;
   __shared__ float sm[8][32], s1s[8][32], s2s[8][32];
-  float* Lb = L + (long long)b * n * T + j;
+  const float* Lb = L + (long long)b * n * T + j;
   const int rows = (n + 7) / 8, i0 = slice * rows, i1 = min(n, i0 + rows);
   float mx = -INFINITY, s1 = 0.f, s2 = 0.f;
   if (j < T) {
@@ -44,6 +45,7 @@ __global__ void __launch_bounds__(256) col_stats_kernel(float* L, float* logphi,
   s1s[slice][lane] = s1;
   s2s[slice][lane] = s2;
   __syncthreads();
+  if (slice != 0 || j >= T) return;
   float M = -INFINITY;
   for (int q = 0; q < 8; ++q) M = fmaxf(M, sm[q][lane]);
   float S1 = 0.f, S2 = 0.f;
@@ -53,22 +55,18 @@ __global__ void __launch_bounds__(256) col_stats_kernel(float* L, float* logphi,
     S1 = fmaf(s1s[q][lane], r, S1);
     S2 = fmaf(s2s[q][lane], r * r, S2);
   }
-  if (j >= T) return;
-  if (slice == 0) logphi[(long long)b * T + j] = M + logf(S1) - logf((float)n);
-  const float inv = 1.0f / sqrtf(S2);
-  for (int i = i0; i < i1; ++i) {
-    float* q = Lb + (long long)i * T;
-    *q = expf(*q - M) * inv;
-  }
+  const long long o = (long long)b * T + j;
+  logphi[o] = M + logf(S1) - logf((float)n);
+  colM[o] = M;
+  colInvN[o] = 1.0f / sqrtf(S2);
 }
 
 int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const bf16* K, const bf16* V,
                                float* L, float* z, float* m, float* invm, float* split, float* Y,
-                               float* logphi, cudaStream_t st) {
+                               float* logphi, float* colM, float* colInvN, DevStatus* stt, cudaStream_t st) {
   const long long nd = (long long)D.n * D.d, Td = (long long)D.T * D.d, nT = (long long)D.n * D.T;
-  // l = scale * Q K^T
-  launch_gemm(RowK<bf16>{Q, nd, D.d}, RowK<bf16>{K, Td, D.d}, EpiStore{L, nT, 0, D.T, scale, false}, D.H, D.n,
-              D.T, D.d, 1, st);
+  // l = scale * Q K^T on the tensor cores
+  if (launch_ref_logits_tc(D, scale, Q, K, L, stt, st) < 0) return -1;
   // z_i = max_j l_ij (z^fit of Eq. mass_fit), m_i = sum_j e^{l_ij - z_i} = (Phi_K 1)_i
   launch_row_stats(D.H, D.n, D.T, L, z, invm, m, st);
   // Y = softmax(l) V
@@ -76,48 +74,8 @@ int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const 
   launch_gemm(P, ColK<bf16>{V, Td, D.d}, EpiStore{split, nd, (long long)D.H * nd, D.d, 1.f, false}, D.H, D.n,
               D.d, D.T, kSplitK, st);
   launch_split_reduce(D.H, D.n, D.d, kSplitK, split, Y, st);
-  col_stats_kernel<<<dim3(cdiv(D.T, 32), D.H), 256, 0, st>>>(L, logphi, D.n, D.T);
+  col_stats_kernel<<<dim3(cdiv(D.T, 32), D.H), 256, 0, st>>>(L, logphi, colM, colInvN, D.n, D.T);
   return 5;
-}
-
-// US[b][i][r] = U[b][i][S_r]
-__global__ void gather_anchor_cols_kernel(const float* U, const int* anchors, float* US, int n, int T, int t) {
-  const int b = blockIdx.y, i = blockIdx.x;
-  const float* u = U + ((long long)b * n + i) * T;
-  const int* S = anchors + (long long)b * t;
-  float* o = US + ((long long)b * n + i) * t;
-  for (int r = threadIdx.x; r < t; r += blockDim.x) o[r] = u[S[r]];
-}
-
-__global__ void decode_assign_kernel(const unsigned long long* best, int* kappa, long long count) {
-  for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < count;
-       k += (long long)gridDim.x * blockDim.x) {
-    const unsigned long long v = best[k];
-    kappa[k] = v ? (int)(0xffffffffu - (unsigned int)(v & 0xffffffffull)) : 0;
-  }
-}
-
-// kappa(s_r) = r (Eq. anchor_assignment)
-__global__ void anchor_self_assign_kernel(const int* anchors, int* kappa, int T, int t, int H) {
-  const long long total = (long long)H * t;
-  for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < total;
-       k += (long long)gridDim.x * blockDim.x) {
-    const long long b = k / t;
-    kappa[b * T + anchors[k]] = (int)(k - b * t);
-  }
-}
-
-int launch_assign(const Dims& D, const float* U, const int* anchors, float* US, unsigned long long* best,
-                  int* kappa, cudaStream_t st) {
-  gather_anchor_cols_kernel<<<dim3(D.n, D.H), 256, 0, st>>>(U, anchors, US, D.n, D.T, D.t);
-  cudaMemsetAsync(best, 0, sizeof(unsigned long long) * (size_t)D.H * D.T, st);
-  // sim(j, r) = u_j . u_{s_r}: A(j, i) = U[i][j], B(r, i) = US[i][r]
-  launch_gemm(ColK<float>{U, (long long)D.n * D.T, D.T}, ColK<float>{US, (long long)D.n * D.t, D.t},
-              EpiArgmax{best, D.T}, D.H, D.T, D.t, D.n, 1, st);
-  const long long cnt = (long long)D.H * D.T;
-  decode_assign_kernel<<<min(cdiv(cnt, 256), 152 * 8), 256, 0, st>>>(best, kappa, cnt);
-  anchor_self_assign_kernel<<<cdiv((long long)D.H * D.t, 256), 256, 0, st>>>(anchors, kappa, D.T, D.t, D.H);
-  return 4;
 }
 
 // Caller-supplied assignment (copied into the workspace): values in [0, t)

@@ -1,0 +1,133 @@
+// Tensor-core stages of Sec. 3.4:
+//   * reference logits l = scale Q K^T (bf16 operands are exact, one MMA per
+//     product, fp32 accumulation);
+//   * the anchor assignment kappa(j) = argmax_r u_j . u_{s_r}
+//     (Eq. anchor_assignment) as a split-bf16 GEMM of the transposed profiles
+//     U^T [T x n] against the anchor rows U_S^T [t x n] whose epilogue keeps
+//     the row maximum (lowest r on ties) and merges it across column tiles
+//     with a 64-bit atomicMax; the T x t similarity is never stored.
+#include "kernels.h"
+#include "tc_gemm.cuh"
+
+namespace arckv {
+
+struct TcEpiArgmax {
+  unsigned long long* best;
+  long long bbs;
+  struct State {
+    float bv;
+    int bi, ncols, n0;
+    bool row_ok;
+  };
+  __device__ __forceinline__ void init(State& s, int, int row, int n0, int M, int N) const {
+    s.bv = -INFINITY;
+    s.bi = -1;
+    s.ncols = N - n0;
+    s.n0 = n0;
+    s.row_ok = row < M;
+  }
+  __device__ __forceinline__ void consume(State& s, int, int j, float (&v)[32]) const {
+#pragma unroll
+    for (int q = 0; q < 32; ++q)
+      if (j * 32 + q < s.ncols && v[q] > s.bv) {
+        s.bv = v[q];
+        s.bi = s.n0 + j * 32 + q;
+      }
+  }
+  __device__ __forceinline__ void finish(State& s, int b, int row, int, int, int) const {
+    if (!s.row_ok || s.bi < 0) return;
+    const unsigned long long key =
+        ((unsigned long long)f32_ordered(s.bv) << 32) | (unsigned long long)(0xffffffffu - (unsigned int)s.bi);
+    atomicMax(best + (long long)b * bbs + row, key);
+  }
+};
+
+int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* K, float* L, DevStatus* stt,
+                         cudaStream_t st) {
+  CUtensorMap mA, mB;
+  if (!encode_bf16_map_3d(&mA, Q, D.d, D.n, D.H, 128) || !encode_bf16_map_3d(&mB, K, D.d, D.T, D.H, 128)) return -1;
+  TcEpiStore epi{L, (long long)D.n * D.T, D.T, scale};
+  if (launch_tc_gemm<128, false>(mA, mB, mA, mB, epi, D.H, D.n, D.T, D.d, 128, stt, st) != cudaSuccess) return -1;
+  return 1;
+}
+
+// One CTA per (32 x 32 tile of l, head): U_ij = exp(l_ij - M_j) * invN_j, split
+// into bf16 (hi, lo) and written transposed, Ut[b][j][i] (row stride ldn >= n;
+// the pad columns n..ldn-1 are written as zeros).
+__global__ void __launch_bounds__(256) profiles_t_kernel(const float* L, const float* colM, const float* colInvN,
+                                                         bf16* Ut_hi, bf16* Ut_lo, int n, int T, int ldn) {
+  const int b = blockIdx.z, j0 = blockIdx.x * 32, i0 = blockIdx.y * 32;
+  __shared__ float tile[32][33];
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  const float* Lb = L + (long long)b * n * T;
+  for (int r = ty; r < 32; r += 8) {
+    const int i = i0 + r, j = j0 + tx;
+    float u = 0.f;
+    if (i < n && j < T) u = expf(Lb[(long long)i * T + j] - colM[(long long)b * T + j]) * colInvN[(long long)b * T + j];
+    tile[r][tx] = u;
+  }
+  __syncthreads();
+  for (int r = ty; r < 32; r += 8) {
+    const int j = j0 + r, i = i0 + tx;
+    if (j < T && i < ldn) {
+      bf16 hi, lo;
+      split_bf16(tile[tx][r], hi, lo);
+      const long long o = ((long long)b * T + j) * ldn + i;
+      Ut_hi[o] = hi;
+      Ut_lo[o] = lo;
+    }
+  }
+}
+
+// UtS[b][r] = Ut[b][S_r] (hi and lo rows).
+__global__ void gather_anchor_rows_kernel(const bf16* Ut_hi, const bf16* Ut_lo, const int* anchors, bf16* S_hi,
+                                          bf16* S_lo, int T, int t, int ldn) {
+  const int b = blockIdx.y, r = blockIdx.x;
+  const int j = anchors[(long long)b * t + r];
+  const long long src = ((long long)b * T + j) * ldn, dst = ((long long)b * t + r) * ldn;
+  for (int i = threadIdx.x; i < ldn; i += blockDim.x) {
+    S_hi[dst + i] = Ut_hi[src + i];
+    S_lo[dst + i] = Ut_lo[src + i];
+  }
+}
+
+__global__ void decode_assign_kernel2(const unsigned long long* best, int* kappa, long long count) {
+  for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < count;
+       k += (long long)gridDim.x * blockDim.x) {
+    const unsigned long long v = best[k];
+    kappa[k] = v ? (int)(0xffffffffu - (unsigned int)(v & 0xffffffffull)) : 0;
+  }
+}
+
+__global__ void anchor_self_assign_kernel2(const int* anchors, int* kappa, int T, int t, int H) {
+  const long long total = (long long)H * t;
+  for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < total;
+       k += (long long)gridDim.x * blockDim.x) {
+    const long long b = k / t;
+    kappa[b * T + anchors[k]] = (int)(k - b * t);
+  }
+}
+
+int launch_assign_tc(const Dims& D, const float* L, const float* colM, const float* colInvN, const int* anchors,
+                     bf16* Ut_hi, bf16* Ut_lo, bf16* S_hi, bf16* S_lo, unsigned long long* best, int* kappa,
+                     DevStatus* stt, cudaStream_t st) {
+  const int ldn = (D.n + 7) / 8 * 8;
+  profiles_t_kernel<<<dim3(cdiv(D.T, 32), cdiv(ldn, 32), D.H), 256, 0, st>>>(L, colM, colInvN, Ut_hi, Ut_lo, D.n,
+                                                                             D.T, ldn);
+  gather_anchor_rows_kernel<<<dim3(D.t, D.H), 128, 0, st>>>(Ut_hi, Ut_lo, anchors, S_hi, S_lo, D.T, D.t, ldn);
+  cudaMemsetAsync(best, 0, sizeof(unsigned long long) * (size_t)D.H * D.T, st);
+  CUtensorMap mA, mA2, mB, mB2;
+  if (!encode_bf16_map_3d(&mA, Ut_hi, ldn, D.T, D.H, 128) || !encode_bf16_map_3d(&mA2, Ut_lo, ldn, D.T, D.H, 128) ||
+      !encode_bf16_map_3d(&mB, S_hi, ldn, D.t, D.H, 128) || !encode_bf16_map_3d(&mB2, S_lo, ldn, D.t, D.H, 128))
+    return -1;
+  TcEpiArgmax epi{best, D.T};
+  const int kfull = (ldn + 63) / 64 * 64;
+  if (launch_tc_gemm<128, true>(mA, mB, mA2, mB2, epi, D.H, D.T, D.t, ldn, kfull, stt, st) != cudaSuccess)
+    return -1;
+  const long long cnt = (long long)D.H * D.T;
+  decode_assign_kernel2<<<min(cdiv(cnt, 256), 152 * 8), 256, 0, st>>>(best, kappa, cnt);
+  anchor_self_assign_kernel2<<<cdiv((long long)D.H * D.t, 256), 256, 0, st>>>(anchors, kappa, D.T, D.t, D.H);
+  return 5;
+}
+
+}  // namespace arckv

@@ -1,0 +1,226 @@
+// Warp-specialised tcgen05 GEMM for sm_103a:
+//
+//   D[b](m, n) = sum_k A[b](m, k) B[b](n, k)      (A, B bf16, K-major, D fp32 in TMEM)
+//
+// One CTA computes a 128 x BN tile.  Warp 0 streams 64-wide K slabs of A and B
+// into a STAGES-deep ring of 128-byte-swizzled shared tiles with TMA; warp 1
+// issues tcgen05.mma (M = 128, N = BN, K = 16) into one of two TMEM
+// accumulators; warps 2..5 drain the accumulator with tcgen05.ld, one TMEM
+// lane (= one output row) per thread, and hand it to the epilogue.
+//
+// With SPLIT, each operand is given as a pair (hi, lo) of bf16 tensors with
+// x ~= hi + lo (hi = bf16(x), lo = bf16(x - hi)), and every K step issues
+// hi*hi + hi*lo + lo*hi: an fp32-accurate product on the bf16 tensor pipe
+// (the dropped lo*lo term is below 2^-16 relative).
+//
+// K is consumed in chunks of `chunk_k` (a multiple of 64): each chunk gets a
+// fresh accumulator and the epilogue sees every chunk separately, which lets
+// a non-linearity act between chunks (the per-index-head LeakyReLU of
+// Eq. pairwise_index_score).  The two TMEM buffers alternate between chunks,
+// so the MMA of chunk c+1 overlaps the epilogue of chunk c.
+//
+// Epilogue interface (all per thread = per output row):
+//   struct State;                                     registers of one row
+//   void init(State&, int b, int row, int n0, int M, int N);
+//   void consume(State&, int chunk, int j, float (&v)[32]);  columns n0+32j..
+//   void finish(State&, int b, int row, int n0, int M, int N);
+#pragma once
+#include "tc.cuh"
+
+namespace arckv {
+
+template <int BN, bool SPLIT>
+struct TcCfg {
+  static constexpr int TILE_A = 128 * 128;  // bytes: 128 rows x 64 bf16
+  static constexpr int TILE_B = BN * 128;
+  static constexpr int STAGE = (TILE_A + TILE_B) * (SPLIT ? 2 : 1);
+  static constexpr int STAGES = SPLIT ? 3 : 4;
+  static constexpr int SMEM = STAGES * STAGE + 1024;
+  static constexpr uint32_t TMEM_COLS = 2 * BN;
+};
+
+template <int BN, bool SPLIT, class Epi>
+__global__ void __launch_bounds__(192, 1)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
+                   const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mB2, Epi epi, int M,
+                   int N, int K, int chunk_k, DevStatus* stt) {
+  using C = TcCfg<BN, SPLIT>;
+  constexpr int STAGES = C::STAGES;
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ uint64_t full[STAGES], empty[STAGES], accf[2], acce[2], drain;
+  __shared__ uint32_t tmem_slot;
+  __shared__ int abort_flag;
+  const uint32_t raw = tc::smem_u32(smem_raw);
+  uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.z, m0 = blockIdx.y * 128, n0 = blockIdx.x * BN;
+  const int nk = (K + 63) / 64;
+  const int kpc = chunk_k / 64;
+  const int nchunks = (nk + kpc - 1) / kpc;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      tc::mbar_init(&full[s], 1);
+      tc::mbar_init(&empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&accf[i], 1);
+      tc::mbar_init(&acce[i], 4);
+    }
+    tc::mbar_init(&drain, 1);
+    abort_flag = 0;
+    tc::mbar_fence_init();
+  }
+  if (warp == 1) tc::tmem_alloc(&tmem_slot, C::TMEM_COLS);
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = tmem_slot;
+  volatile int* abortp = &abort_flag;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tc::tma_prefetch(&mA);
+      tc::tma_prefetch(&mB);
+      if (SPLIT) {
+        tc::tma_prefetch(&mA2);
+        tc::tma_prefetch(&mB2);
+      }
+      int issued = 0;
+      for (int kb = 0; kb < nk; ++kb) {
+        const int s = kb % STAGES;
+        if (kb >= STAGES && !tc::mbar_wait(&empty[s], ((kb / STAGES) - 1) & 1, abortp, stt)) break;
+        uint8_t* st = base + s * C::STAGE;
+        tc::mbar_arrive_expect_tx(&full[s], C::STAGE);
+        tc::tma_load_3d(st, &mA, kb * 64, m0, b, &full[s]);
+        tc::tma_load_3d(st + C::TILE_A, &mB, kb * 64, n0, b, &full[s]);
+        if (SPLIT) {
+          tc::tma_load_3d(st + C::TILE_A + C::TILE_B, &mA2, kb * 64, m0, b, &full[s]);
+          tc::tma_load_3d(st + 2 * C::TILE_A + C::TILE_B, &mB2, kb * 64, n0, b, &full[s]);
+        }
+        issued = kb + 1;
+      }
+      // every issued copy lands before the CTA may exit
+      volatile int never = 0;
+      for (int kb = issued > STAGES ? issued - STAGES : 0; kb < issued; ++kb)
+        tc::mbar_wait(&full[kb % STAGES], (kb / STAGES) & 1, &never, stt);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = tc::idesc_bf16_f32(BN);
+      bool ok = true;
+      for (int c = 0; c < nchunks && ok; ++c) {
+        const int buf = c & 1;
+        if (c >= 2 && !tc::mbar_wait(&acce[buf], ((c >> 1) - 1) & 1, abortp, stt)) break;
+        tc::fence_after_sync();
+        const uint32_t d = tmem + (uint32_t)(buf * BN);
+        const int kb0 = c * kpc, kb1 = min(nk, kb0 + kpc);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          const int s = kb % STAGES;
+          if (!tc::mbar_wait(&full[s], (kb / STAGES) & 1, abortp, stt)) {
+            ok = false;
+            break;
+          }
+          tc::fence_after_sync();
+          const uint32_t a = tc::smem_u32(base + s * C::STAGE), bb = a + C::TILE_A;
+#pragma unroll
+          for (int ks = 0; ks < 4; ++ks) {
+            const uint64_t ad = tc::sdesc_k128(a + ks * 32), bd = tc::sdesc_k128(bb + ks * 32);
+            tc::mma_f16(d, ad, bd, idesc, (kb > kb0 || ks > 0) ? 1u : 0u);
+            if (SPLIT) {
+              const uint64_t ad2 = tc::sdesc_k128(a + C::TILE_A + C::TILE_B + ks * 32);
+              const uint64_t bd2 = tc::sdesc_k128(bb + C::TILE_A + C::TILE_B + ks * 32);
+              tc::mma_f16(d, ad, bd2, idesc, 1u);
+              tc::mma_f16(d, ad2, bd, idesc, 1u);
+            }
+          }
+          tc::mma_commit(&empty[s]);
+        }
+        if (ok) tc::mma_commit(&accf[buf]);
+      }
+      // all MMAs this thread issued have completed before teardown
+      tc::mma_commit(&drain);
+      volatile int never = 0;
+      tc::mbar_wait(&drain, 0, &never, stt);
+    }
+  } else {
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int row = q * 32 + lane;
+    typename Epi::State es;
+    epi.init(es, b, m0 + row, n0, M, N);
+    bool ok = true;
+    for (int c = 0; c < nchunks; ++c) {
+      const int buf = c & 1;
+      ok = tc::mbar_wait(&accf[buf], (c >> 1) & 1, abortp, stt);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) break;
+      tc::fence_after_sync();
+#pragma unroll
+      for (int j = 0; j < BN / 32; ++j) {
+        float v[32];
+        tc::tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN + j * 32), v);
+        epi.consume(es, c, j, v);
+      }
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&acce[buf]);
+    }
+    if (ok) epi.finish(es, b, m0 + row, n0, M, N);
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 1) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+// Host: launch over H batches; maps are built by the caller (encode_bf16_map_3d,
+// box rows 128 for A and BN for B).
+template <int BN, bool SPLIT, class Epi>
+inline cudaError_t launch_tc_gemm(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mA2,
+                                  const CUtensorMap& mB2, const Epi& epi, int H, int M, int N, int K, int chunk_k,
+                                  DevStatus* stt, cudaStream_t st) {
+  using C = TcCfg<BN, SPLIT>;
+  auto kern = tc_gemm_kernel<BN, SPLIT, Epi>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  dim3 grid(cdiv(N, BN), cdiv(M, 128), H);
+  kern<<<grid, 192, C::SMEM, st>>>(mA, mB, mA2, mB2, epi, M, N, K, chunk_k, stt);
+  return cudaGetLastError();
+}
+
+// Plain fp32 store epilogue: C[b][row][col] = alpha * acc.
+struct TcEpiStore {
+  float* C;
+  long long cbs;
+  int ldc;
+  float alpha;
+  struct State {
+    float* dst;
+    bool row_ok, vec;
+    int ncols;
+  };
+  __device__ __forceinline__ void init(State& s, int b, int row, int n0, int M, int N) const {
+    s.dst = C + (long long)b * cbs + (long long)row * ldc + n0;
+    s.row_ok = row < M;
+    s.ncols = N - n0;
+    s.vec = ((ldc & 3) == 0) && ((((uintptr_t)C) & 15) == 0) && ((cbs & 3) == 0) && ((n0 & 3) == 0);
+  }
+  __device__ __forceinline__ void consume(State& s, int, int j, float (&v)[32]) const {
+    if (!s.row_ok) return;
+    float* d = s.dst + j * 32;
+    if (s.vec && j * 32 + 32 <= s.ncols) {
+#pragma unroll
+      for (int q = 0; q < 32; q += 4)
+        *(float4*)(d + q) = make_float4(alpha * v[q], alpha * v[q + 1], alpha * v[q + 2], alpha * v[q + 3]);
+    } else {
+#pragma unroll
+      for (int q = 0; q < 32; ++q)
+        if (j * 32 + q < s.ncols) d[q] = alpha * v[q];
+    }
+  }
+  __device__ __forceinline__ void finish(State&, int, int, int, int, int) const {}
+};
+
+}  // namespace arckv

@@ -1,0 +1,79 @@
+// Index logits on tcgen05 (Sec. 3.3; App. A.1 Eq. pairwise_index_score):
+//
+//   I_ij = sum_a w_ia LeakyReLU_0.1(q_bar_ia . k_bar_ja / sqrt(d_I))
+//
+// as one split-bf16 tensor-core GEMM of q_bar [n x H_I d_I] against
+// k_bar [T x H_I d_I] whose K dimension is consumed one index head (d_I = 128
+// columns) at a time: every head's partial dot products land in their own
+// TMEM accumulator and the epilogue folds them through the LeakyReLU and the
+// row's head weight w_ia before the next head is added.  The epilogue then
+// writes the I tile and the tile's row-softmax partials (max, sum of exp).
+#include "kernels.h"
+#include "tc_gemm.cuh"
+
+namespace arckv {
+
+struct TcEpiIndex {
+  const float* wts;  // [H][n_pos][H_I]
+  float* I;          // [H][n][T]
+  float2* part;      // [H][n][ntiles]
+  int n, T, H_I, G, n_pos, ntiles;
+  struct State {
+    float acc[128];
+    const float* wrow;
+    float w;
+    bool row_ok;
+  };
+  __device__ __forceinline__ void init(State& s, int b, int row, int, int M, int) const {
+    s.row_ok = row < M;
+    s.wrow = wts + ((long long)b * n_pos + (s.row_ok ? row / G : 0)) * H_I;
+    s.w = 0.f;
+#pragma unroll
+    for (int q = 0; q < 128; ++q) s.acc[q] = 0.f;
+  }
+  __device__ __forceinline__ void consume(State& s, int chunk, int j, float (&v)[32]) const {
+    if (j == 0) s.w = s.row_ok ? s.wrow[chunk] : 0.f;
+    const float inv = 0.08838834764831845f;  // 1 / sqrt(d_I), d_I = 128
+#pragma unroll
+    for (int q = 0; q < 32; ++q) {
+      const float x = v[q] * inv;
+      s.acc[j * 32 + q] = fmaf(s.w, x >= 0.f ? x : 0.1f * x, s.acc[j * 32 + q]);
+    }
+  }
+  __device__ __forceinline__ void finish(State& s, int b, int row, int n0, int, int N) const {
+    if (!s.row_ok) return;
+    const int nc = min(128, N - n0);
+    float mx = -INFINITY;
+#pragma unroll
+    for (int q = 0; q < 128; ++q)
+      if (q < nc) mx = fmaxf(mx, s.acc[q]);
+    float sm = 0.f;
+#pragma unroll
+    for (int q = 0; q < 128; ++q)
+      if (q < nc) sm += expf(s.acc[q] - mx);
+    part[((long long)b * n + row) * ntiles + n0 / 128] = make_float2(mx, sm);
+    float* dst = I + ((long long)b * n + row) * T + n0;
+    if ((T & 3) == 0 && nc == 128) {
+#pragma unroll
+      for (int q = 0; q < 128; q += 4) *(float4*)(dst + q) = make_float4(s.acc[q], s.acc[q + 1], s.acc[q + 2], s.acc[q + 3]);
+    } else {
+#pragma unroll
+      for (int q = 0; q < 128; ++q)
+        if (q < nc) dst[q] = s.acc[q];
+    }
+  }
+};
+
+int launch_index_logits(const Dims& D, const bf16* qbar_hi, const bf16* qbar_lo, const bf16* kbar_hi,
+                        const bf16* kbar_lo, const float* wts, float* I, float2* part, DevStatus* stt,
+                        cudaStream_t st) {
+  CUtensorMap mA, mA2, mB, mB2;
+  if (!encode_bf16_map_3d(&mA, qbar_hi, D.HD, D.n, D.H, 128) || !encode_bf16_map_3d(&mA2, qbar_lo, D.HD, D.n, D.H, 128) ||
+      !encode_bf16_map_3d(&mB, kbar_hi, D.HD, D.T, D.H, 128) || !encode_bf16_map_3d(&mB2, kbar_lo, D.HD, D.T, D.H, 128))
+    return -1;
+  TcEpiIndex epi{wts, I, part, D.n, D.T, D.H_I, D.G, D.n_pos, cdiv(D.T, 128)};
+  if (launch_tc_gemm<128, true>(mA, mB, mA2, mB2, epi, D.H, D.n, D.T, D.HD, 128, stt, st) != cudaSuccess) return -1;
+  return 1;
+}
+
+}  // namespace arckv
