@@ -14,8 +14,9 @@ constexpr size_t kAlign = 256;
 inline size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct Layout {
-  size_t status, kbar_hi, kbar_lo, Uk, Uv, vq, cctx, qbar_hi, qbar_lo, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
-      colM, colInvN, Ut_hi, Ut_lo, S_hi, S_lo, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z, split, total;
+  size_t status, W1, W2, kbar_hi, kbar_lo, Uk, Uv, vq, cctx, qbar_hi, qbar_lo, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
+      colM, colInvN, Ut_hi, Ut_lo, S_hi, S_lo, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z,
+      YT_hi, YT_lo, split, total;
 };
 
 Dims dims_of(const arckv_config& c) {
@@ -55,6 +56,8 @@ Layout plan(const arckv_config& c) {
   size_t o = 0;
   auto take = [&](size_t bytes) { size_t r = o; o += up(bytes); return r; };
   L.status = take(sizeof(DevStatus));
+  L.W1 = take(H * (HD + 256) * 128 * 2);
+  L.W2 = take(H * (HD + 256) * 128 * 2);
   L.kbar_hi = take(H * T * HD * 2);
   L.kbar_lo = take(H * T * HD * 2);
   L.Uk = take(H * T * 128 * f);
@@ -96,6 +99,8 @@ Layout plan(const arckv_config& c) {
   L.wsol = take(H * t * f);
   L.R = take(H * t * 128 * f);
   L.Z = take(H * t * 128 * f);
+  L.YT_hi = take(H * 128 * ldn * 2);
+  L.YT_lo = take(H * 128 * ldn * 2);
   L.split = take((size_t)kSplitK * H * (n > t ? n : t) * 128 * f);
   L.total = o;
   return L;
@@ -183,8 +188,11 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
   mark(0);
   if (!given_anchors) {
     auto B16 = [&](size_t off) { return (bf16*)(w + off); };
-    nl += launch_key_features(D, Kb, Vb, (const bf16*)idx->L_k, (const bf16*)idx->L_v, (const bf16*)idx->U_k,
-                              (const bf16*)idx->U_v, B16(L.kbar_hi), B16(L.kbar_lo), F(L.Uk), F(L.Uv), st);
+    const int nlk = launch_key_features_tc(D, Kb, Vb, (const bf16*)idx->L_k, (const bf16*)idx->L_v,
+                                           (const bf16*)idx->U_k, (const bf16*)idx->U_v, B16(L.W1), B16(L.W2),
+                                           B16(L.kbar_hi), B16(L.kbar_lo), F(L.Uk), F(L.Uv), stt, st);
+    if (nlk < 0) return ARCKV_ERR_CUDA;
+    nl += nlk;
     nl += launch_query_features(D, Qb, (const bf16*)X_ref, (const bf16*)idx->U_q, (const bf16*)idx->L_q,
                                 (const bf16*)idx->L_c, (const bf16*)idx->L_x, (const bf16*)idx->b_x, F(L.Uk),
                                 F(L.Uv), F(L.vq), F(L.NT), F(L.rA), F(L.rB), F(L.split), F(L.cctx),
@@ -223,9 +231,12 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
   nl += launch_merge(D, cfg->lambda_m, Kb, anchors, kappa, F(L.logphi), I32(L.perm), I32(L.goff), I32(L.cursor),
                      C_k, st);
   mark(5);
-  FitBufs B{F(L.LC), F(L.Phi), F(L.Gram), F(L.Linv), F(L.rhs), F(L.wsol), F(L.R), F(L.Z), F(L.split)};
-  nl += launch_fits(D, scale, cfg->ridge_w, cfg->ridge_v, cfg->eps_w, cfg->b_min, cfg->b_max, Qb, C_k, F(L.z),
-                    F(L.m), F(L.Y), B, beta, C_v, stt, st);
+  FitBufs B{F(L.LC),  F(L.Phi), F(L.Gram), F(L.Linv), F(L.rhs), F(L.wsol), F(L.R), F(L.Z), F(L.split),
+            (bf16*)(w + L.S_hi), (bf16*)(w + L.S_lo), (bf16*)(w + L.YT_hi), (bf16*)(w + L.YT_lo)};
+  const int nlf = launch_fits(D, scale, cfg->ridge_w, cfg->ridge_v, cfg->eps_w, cfg->b_min, cfg->b_max, Qb, C_k,
+                              F(L.z), F(L.m), F(L.Y), B, beta, C_v, stt, st);
+  if (nlf < 0) return ARCKV_ERR_CUDA;
+  nl += nlf;
   nl += launch_check_finite(C_k, (long long)D.H * D.t * D.d, stt, st);
   nl += launch_check_finite(beta, (long long)D.H * D.t, stt, st);
   nl += launch_check_finite(C_v, (long long)D.H * D.t * D.d, stt, st);

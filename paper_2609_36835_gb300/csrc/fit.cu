@@ -12,6 +12,7 @@
 // backward substitution.
 #include "gemm.cuh"
 #include "kernels.h"
+#include "tc_gemm.cuh"
 
 namespace arckv {
 
@@ -60,33 +61,33 @@ __global__ void ridge_kernel(float* Gram, int t, float ridge, DevStatus* stt) {
 
 // Factor the (already updated) diagonal block k in shared memory, write L_kk
 // into A and its inverse into Linv[b][k] (64 x 64, identity beyond the matrix).
-// Left-looking by columns: at column c every row r >= c forms
-// A_rc - sum_{q<c} L_rq L_cq with four threads per row, the pivot row takes the
-// square root and the rows below divide.  The inverse is formed row by row:
+// Left-looking by columns with 16 threads per row: at column c every row
+// r >= c forms A_rc - sum_{q<c} L_rq L_cq, the pivot row takes the square
+// root and the rows below divide.  The inverse is formed row by row:
 // Li_ij = (delta_ij - sum_{l=j}^{i-1} L_il Li_lj) / L_ii, all j of a row at once.
-__global__ void __launch_bounds__(256) potrf_diag_kernel(float* A, int t, int k, float* Linv, int nblk,
-                                                         DevStatus* stt) {
+__global__ void __launch_bounds__(1024) potrf_diag_kernel(float* A, int t, int k, float* Linv, int nblk,
+                                                          DevStatus* stt) {
   const int b = blockIdx.x, tid = threadIdx.x;
   float* Ab = A + (long long)b * t * t;
   const int k0 = k * NB, kb = min(NB, t - k0);
   __shared__ float L[NB][NB + 1];
   __shared__ float Li[NB][NB + 1];
   __shared__ int bad;
-  for (int e = tid; e < NB * NB; e += 256) {
+  for (int e = tid; e < NB * NB; e += 1024) {
     const int r = e / NB, c = e % NB;
     L[r][c] = (r < kb && c <= r) ? Ab[(long long)(k0 + r) * t + k0 + c] : (r == c ? 1.f : 0.f);
     Li[r][c] = 0.f;
   }
   if (tid == 0) bad = 0;
   __syncthreads();
-  const int r = tid >> 2, p = tid & 3;
+  const int r = tid >> 4, p = tid & 15;
   for (int c = 0; c < NB; ++c) {
     // columns < c are final (the previous iteration ended with a barrier)
     float v = 0.f;
     if (r >= c)
-      for (int q = p; q < c; q += 4) v = fmaf(L[r][q], L[c][q], v);
-    v += __shfl_xor_sync(0xffffffffu, v, 1);
-    v += __shfl_xor_sync(0xffffffffu, v, 2);
+      for (int q = p; q < c; q += 16) v = fmaf(L[r][q], L[c][q], v);
+#pragma unroll
+    for (int o = 1; o < 16; o <<= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     v = (r >= c) ? L[r][c] - v : 0.f;
     if (r == c && p == 0) {
       if (!(v > 0.f) || !isfinite(v)) { bad = 1; v = 1.f; }
@@ -97,18 +98,18 @@ __global__ void __launch_bounds__(256) potrf_diag_kernel(float* A, int t, int k,
     __syncthreads();
   }
   if (tid == 0 && bad) set_status(stt, ARCKV_ERR_NOT_SPD);
-  const int j = tid >> 2;
+  const int j = tid >> 4;
   for (int i = 0; i < NB; ++i) {
     float v = 0.f;
     if (j < i)
-      for (int l = j + p; l < i; l += 4) v = fmaf(L[i][l], Li[l][j], v);
-    v += __shfl_xor_sync(0xffffffffu, v, 1);
-    v += __shfl_xor_sync(0xffffffffu, v, 2);
+      for (int l = j + p; l < i; l += 16) v = fmaf(L[i][l], Li[l][j], v);
+#pragma unroll
+    for (int o = 1; o < 16; o <<= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     if (j <= i && p == 0) Li[i][j] = ((i == j ? 1.f : 0.f) - v) / L[i][i];
     __syncthreads();
   }
   float* Lo = Linv + ((long long)b * nblk + k) * NB * NB;
-  for (int e = tid; e < NB * NB; e += 256) {
+  for (int e = tid; e < NB * NB; e += 1024) {
     const int rr = e / NB, cc = e % NB;
     Lo[e] = Li[rr][cc];
     if (rr < kb && cc <= rr) Ab[(long long)(k0 + rr) * t + k0 + cc] = L[rr][cc];
@@ -320,7 +321,7 @@ static int cholesky_solve(int H, int t, float* Gram, float* Linv, float* B, floa
   ++nl;
   const int nblk = cdiv(t, NB), nct = cdiv(nrhs, NB);
   for (int k = 0; k < nblk; ++k) {
-    potrf_diag_kernel<<<H, 256, 0, st>>>(Gram, t, k, Linv, nblk, stt);
+    potrf_diag_kernel<<<H, 1024, 0, st>>>(Gram, t, k, Linv, nblk, stt);
     ++nl;
     const int m = nblk - k - 1;
     if (m > 0) {
@@ -363,6 +364,45 @@ __global__ void softmax_bias_kernel(const float* LC, const float* beta, float* P
   for (int c = lane; c < t; c += 32) o[c] = expf(x[c] + be[c] - mx) * inv;
 }
 
+// dst_hi/lo[b][c][r] = split(src[b][r][c]) for r < rows, zero for rows <= r < ldr:
+// the transposed, K-major split-bf16 operand of the Gram GEMMs.
+__global__ void __launch_bounds__(256) transpose_split_kernel(const float* src, int rows, int cols, bf16* dst_hi,
+                                                              bf16* dst_lo, int ldr) {
+  const int b = blockIdx.z, c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+  __shared__ float tile[32][33];
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  const float* sb = src + (long long)b * rows * cols;
+  for (int q = ty; q < 32; q += 8) {
+    const int r = r0 + q, c = c0 + tx;
+    tile[q][tx] = (r < rows && c < cols) ? sb[(long long)r * cols + c] : 0.f;
+  }
+  __syncthreads();
+  for (int q = ty; q < 32; q += 8) {
+    const int c = c0 + q, r = r0 + tx;
+    if (c < cols && r < ldr) {
+      bf16 hi, lo;
+      split_bf16(tile[tx][q], hi, lo);
+      const long long o = ((long long)b * cols + c) * ldr + r;
+      dst_hi[o] = hi;
+      dst_lo[o] = lo;
+    }
+  }
+}
+
+// C[b] (M x N, row stride ldc) = X^T Z over the n reference rows, with X^T and
+// Z^T given as transposed split-bf16 operands [M][ldn] and [N][ldn].
+static int gram_tc(int H, int M, int N, int ldn, const bf16* Xh, const bf16* Xl, const bf16* Zh, const bf16* Zl,
+                   float* C, int ldc, DevStatus* stt, cudaStream_t st) {
+  CUtensorMap mA, mA2, mB, mB2;
+  if (!encode_bf16_map_3d(&mA, Xh, ldn, M, H, 128) || !encode_bf16_map_3d(&mA2, Xl, ldn, M, H, 128) ||
+      !encode_bf16_map_3d(&mB, Zh, ldn, N, H, 128) || !encode_bf16_map_3d(&mB2, Zl, ldn, N, H, 128))
+    return -1;
+  TcEpiStore epi{C, (long long)M * ldc, ldc, 1.f};
+  const int kfull = (ldn + 63) / 64 * 64;
+  if (launch_tc_gemm<128, kSplit>(mA, mB, mA2, mB2, epi, H, M, N, ldn, kfull, stt, st) != cudaSuccess) return -1;
+  return 1;
+}
+
 int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float eps_w, float b_min,
                 float b_max, const bf16* Q, const float* C_k, const float* z, const float* m,
                 const float* Y, const FitBufs& B, float* beta, float* C_v, DevStatus* stt, cudaStream_t st) {
@@ -375,7 +415,11 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
   const long long cnt = (long long)D.H * nt;
   phi_kernel<<<min(cdiv(cnt, 256), 152 * 16), 256, 0, st>>>(B.LC, z, B.Phi, D.n, D.t, cnt);
   ++nl;
-  // beta system
+  // beta system: Gram = Phi_C^T Phi_C in fp32 (SIMT, lower tiles mirrored).  Its
+  // condition number reaches ~1e6 on long caches, beyond what the split-bf16
+  // tensor-core product (~1e-5 relative per entry) resolves within tolerance.
+  const int ldn = (D.n + 7) / 8 * 8;
+  const dim3 tgrid(cdiv(D.t, 32), cdiv(ldn, 32), D.H);
   launch_gemm<true>(ColK<float>{B.Phi, nt, D.t}, ColK<float>{B.Phi, nt, D.t}, EpiStore{B.Gram, tt, 0, D.t, 1.f, true},
                     D.H, D.t, D.t, D.n, 1, st);
   ++nl;
@@ -385,17 +429,19 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
   const long long ht = (long long)D.H * D.t;
   beta_kernel<<<cdiv(ht, 256), 256, 0, st>>>(B.wsol, beta, ht, eps_w, b_min, b_max);
   ++nl;
-  // value system: P^ over the compact keys with the fitted bias
+  // value system: P^ over the compact keys with the fitted bias; its Gram and
+  // P^T Y on the tensor cores from transposed split-bf16 operands
   softmax_bias_kernel<<<dim3(cdiv(D.n, 8), D.H), 256, 0, st>>>(B.LC, beta, B.Phi, D.n, D.t);
   ++nl;
-  launch_gemm<true>(ColK<float>{B.Phi, nt, D.t}, ColK<float>{B.Phi, nt, D.t}, EpiStore{B.Gram, tt, 0, D.t, 1.f, true},
-                    D.H, D.t, D.t, D.n, 1, st);
-  ++nl;
+  transpose_split_kernel<<<tgrid, 256, 0, st>>>(B.Phi, D.n, D.t, B.PT_hi, B.PT_lo, ldn);
+  transpose_split_kernel<<<dim3(cdiv(D.d, 32), cdiv(ldn, 32), D.H), 256, 0, st>>>(Y, D.n, D.d, B.YT_hi, B.YT_lo,
+                                                                                    ldn);
+  nl += 2;
+  if (gram_tc(D.H, D.t, D.t, ldn, B.PT_hi, B.PT_lo, B.PT_hi, B.PT_lo, B.Gram, D.t, stt, st) < 0) return -1;
+  // R = P^T Y
   const long long td = (long long)D.t * D.d;
-  launch_gemm(ColK<float>{B.Phi, nt, D.t}, ColK<float>{Y, nd, D.d},
-              EpiStore{B.split, td, (long long)D.H * td, D.d, 1.f, false}, D.H, D.t, D.d, D.n, kSplitK, st);
-  ++nl;
-  nl += launch_split_reduce(D.H, D.t, D.d, kSplitK, B.split, B.R, st);
+  if (gram_tc(D.H, D.t, D.d, ldn, B.PT_hi, B.PT_lo, B.YT_hi, B.YT_lo, B.R, D.d, stt, st) < 0) return -1;
+  nl += 2;
   nl += cholesky_solve(D.H, D.t, B.Gram, B.Linv, B.R, B.Z, C_v, D.d, D.d, td, ridge_v, stt, st);
   return nl;
 }

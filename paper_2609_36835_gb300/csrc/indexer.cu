@@ -12,23 +12,6 @@
 
 namespace arckv {
 
-int launch_key_features(const Dims& D, const bf16* K, const bf16* V, const bf16* L_k, const bf16* L_v,
-                        const bf16* U_k, const bf16* U_v, bf16* kbar_hi, bf16* kbar_lo, float* Uk, float* Uv,
-                        cudaStream_t st) {
-  const long long Td = (long long)D.T * D.d, Wd = (long long)D.HD * D.d;
-  // z = [k | v] [L_k | L_v]^T, RMS-normalised per 128-wide block, stored as a split-bf16 pair
-  CatRowK<bf16, bf16> A{{K, Td, D.d}, {V, Td, D.d}, D.d};
-  CatRowK<bf16, bf16> B{{L_k, Wd, D.d}, {L_v, Wd, D.d}, D.d};
-  launch_gemm(A, B, EpiBlockNormSplit{kbar_hi, kbar_lo, (long long)D.T * D.HD, D.HD}, D.H, D.T, D.HD, 2 * D.d, 1,
-              st);
-  const long long Ud = (long long)D.d_A * D.d;
-  launch_gemm(RowK<bf16>{K, Td, D.d}, RowK<bf16>{U_k, Ud, D.d},
-              EpiStore{Uk, (long long)D.T * D.d_A, 0, D.d_A, 1.f, false}, D.H, D.T, D.d_A, D.d, 1, st);
-  launch_gemm(RowK<bf16>{V, Td, D.d}, RowK<bf16>{U_v, Ud, D.d},
-              EpiStore{Uv, (long long)D.T * D.d_A, 0, D.d_A, 1.f, false}, D.H, D.T, D.d_A, D.d, 1, st);
-  return 3;
-}
-
 // w[b][r][a] = L_x[b][a] . x_r + b_x[b][a]: one CTA per (position, head).
 __global__ void __launch_bounds__(256) index_weights_kernel(const bf16* X, const bf16* L_x, const bf16* b_x,
                                                             float* wts, int d_x, int H_I, int n_pos) {

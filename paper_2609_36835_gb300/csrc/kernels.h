@@ -13,10 +13,11 @@ constexpr int kSplitK = 8;   // K slices of the skinny (N = 128) long-K products
 constexpr int kCholNB = 64;  // Cholesky block size
 
 // ---- indexer (Sec. 3.3, App. A.1) --------------------------------------
-// k_bar = N(L_k k + L_v v) per d_I block; Uk = U_k k; Uv = U_v v.
-int launch_key_features(const Dims& D, const bf16* K, const bf16* V, const bf16* L_k, const bf16* L_v,
-                        const bf16* U_k, const bf16* U_v, bf16* kbar_hi, bf16* kbar_lo, float* Uk, float* Uv,
-                        cudaStream_t st);
+// k_bar = N(L_k k + L_v v) per d_I block (split bf16); Uk = U_k k; Uv = U_v v
+// (one tcgen05 GEMM over [K | V]; W1, W2 are stacked-weight scratch).
+int launch_key_features_tc(const Dims& D, const bf16* K, const bf16* V, const bf16* L_k, const bf16* L_v,
+                           const bf16* U_k, const bf16* U_v, bf16* W1, bf16* W2, bf16* kbar_hi, bf16* kbar_lo,
+                           float* Uk, float* Uv, DevStatus* stt, cudaStream_t st);
 // value context c (Eq. value_context), q_bar (Eq. indexer_projection), w.
 int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf16* U_q, const bf16* L_q,
                           const bf16* L_c, const bf16* L_x, const bf16* b_x, const float* Uk,
@@ -55,7 +56,9 @@ int launch_merge(const Dims& D, float lambda_m, const bf16* K, const int* anchor
 // ---- fits (App. A.9) -----------------------------------------------------
 struct FitBufs {
   float *LC, *Phi, *Gram, *Linv, *rhs, *wsol, *R, *Z, *split;
+  bf16 *PT_hi, *PT_lo, *YT_hi, *YT_lo;  // transposed split-bf16 operands ([t][ldn], [d][ldn])
 };
+// Returns launches, or -1 when a TMA descriptor cannot be encoded.
 int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float eps_w, float b_min,
                 float b_max, const bf16* Q, const float* C_k, const float* z, const float* m,
                 const float* Y, const FitBufs& B, float* beta, float* C_v, DevStatus* stt, cudaStream_t st);

@@ -47,7 +47,7 @@ int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* 
   CUtensorMap mA, mB;
   if (!encode_bf16_map_3d(&mA, Q, D.d, D.n, D.H, 128) || !encode_bf16_map_3d(&mB, K, D.d, D.T, D.H, 128)) return -1;
   TcEpiStore epi{L, (long long)D.n * D.T, D.T, scale};
-  if (launch_tc_gemm<128, false>(mA, mB, mA, mB, epi, D.H, D.n, D.T, D.d, 128, stt, st) != cudaSuccess) return -1;
+  if (launch_tc_gemm<128, kPlain>(mA, mB, mA, mB, epi, D.H, D.n, D.T, D.d, 128, stt, st) != cudaSuccess) return -1;
   return 1;
 }
 
@@ -122,7 +122,7 @@ int launch_assign_tc(const Dims& D, const float* L, const float* colM, const flo
     return -1;
   TcEpiArgmax epi{best, D.T};
   const int kfull = (ldn + 63) / 64 * 64;
-  if (launch_tc_gemm<128, true>(mA, mB, mA2, mB2, epi, D.H, D.T, D.t, ldn, kfull, stt, st) != cudaSuccess)
+  if (launch_tc_gemm<128, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.T, D.t, ldn, kfull, stt, st) != cudaSuccess)
     return -1;
   const long long cnt = (long long)D.H * D.T;
   decode_assign_kernel2<<<min(cdiv(cnt, 256), 152 * 8), 256, 0, st>>>(best, kappa, cnt);

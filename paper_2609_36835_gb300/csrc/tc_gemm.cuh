@@ -8,10 +8,14 @@
 // accumulators; warps 2..5 drain the accumulator with tcgen05.ld, one TMEM
 // lane (= one output row) per thread, and hand it to the epilogue.
 //
-// With SPLIT, each operand is given as a pair (hi, lo) of bf16 tensors with
-// x ~= hi + lo (hi = bf16(x), lo = bf16(x - hi)), and every K step issues
-// hi*hi + hi*lo + lo*hi: an fp32-accurate product on the bf16 tensor pipe
-// (the dropped lo*lo term is below 2^-16 relative).
+// MODE selects how the second pair of maps (mA2, mB2) is used:
+//   kPlain  -- not used;
+//   kSplit  -- each operand is a pair (hi, lo) of bf16 tensors with
+//              x ~= hi + lo (hi = bf16(x), lo = bf16(x - hi)) and every K step
+//              issues hi*hi + hi*lo + lo*hi: an fp32-accurate product on the
+//              bf16 tensor pipe (the dropped lo*lo term is below 2^-16 relative);
+//   kConcat -- the operands are concatenated along K: K < K1 comes from
+//              (mA, mB), K >= K1 from (mA2, mB2) (K1 a multiple of 64).
 //
 // K is consumed in chunks of `chunk_k` (a multiple of 64): each chunk gets a
 // fresh accumulator and the epilogue sees every chunk separately, which lets
@@ -29,8 +33,11 @@
 
 namespace arckv {
 
-template <int BN, bool SPLIT>
+enum TcMode { kPlain = 0, kSplit = 1, kConcat = 2 };
+
+template <int BN, int MODE>
 struct TcCfg {
+  static constexpr bool SPLIT = MODE == kSplit;
   static constexpr int TILE_A = 128 * 128;  // bytes: 128 rows x 64 bf16
   static constexpr int TILE_B = BN * 128;
   static constexpr int STAGE = (TILE_A + TILE_B) * (SPLIT ? 2 : 1);
@@ -39,12 +46,13 @@ struct TcCfg {
   static constexpr uint32_t TMEM_COLS = 2 * BN;
 };
 
-template <int BN, bool SPLIT, class Epi>
+template <int BN, int MODE, class Epi>
 __global__ void __launch_bounds__(192, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
                    const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mB2, Epi epi, int M,
-                   int N, int K, int chunk_k, DevStatus* stt) {
-  using C = TcCfg<BN, SPLIT>;
+                   int N, int K, int chunk_k, int K1, DevStatus* stt) {
+  using C = TcCfg<BN, MODE>;
+  constexpr bool SPLIT = C::SPLIT;
   constexpr int STAGES = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
   __shared__ uint64_t full[STAGES], empty[STAGES], accf[2], acce[2], drain;
@@ -82,7 +90,7 @@ __global__ void __launch_bounds__(192, 1)
     if (lane == 0) {
       tc::tma_prefetch(&mA);
       tc::tma_prefetch(&mB);
-      if (SPLIT) {
+      if (MODE != kPlain) {
         tc::tma_prefetch(&mA2);
         tc::tma_prefetch(&mB2);
       }
@@ -92,8 +100,13 @@ __global__ void __launch_bounds__(192, 1)
         if (kb >= STAGES && !tc::mbar_wait(&empty[s], ((kb / STAGES) - 1) & 1, abortp, stt)) break;
         uint8_t* st = base + s * C::STAGE;
         tc::mbar_arrive_expect_tx(&full[s], C::STAGE);
-        tc::tma_load_3d(st, &mA, kb * 64, m0, b, &full[s]);
-        tc::tma_load_3d(st + C::TILE_A, &mB, kb * 64, n0, b, &full[s]);
+        if (MODE == kConcat && kb * 64 >= K1) {
+          tc::tma_load_3d(st, &mA2, kb * 64 - K1, m0, b, &full[s]);
+          tc::tma_load_3d(st + C::TILE_A, &mB2, kb * 64 - K1, n0, b, &full[s]);
+        } else {
+          tc::tma_load_3d(st, &mA, kb * 64, m0, b, &full[s]);
+          tc::tma_load_3d(st + C::TILE_A, &mB, kb * 64, n0, b, &full[s]);
+        }
         if (SPLIT) {
           tc::tma_load_3d(st + C::TILE_A + C::TILE_B, &mA2, kb * 64, m0, b, &full[s]);
           tc::tma_load_3d(st + 2 * C::TILE_A + C::TILE_B, &mB2, kb * 64, n0, b, &full[s]);
@@ -177,16 +190,16 @@ __global__ void __launch_bounds__(192, 1)
 
 // Host: launch over H batches; maps are built by the caller (encode_bf16_map_3d,
 // box rows 128 for A and BN for B).
-template <int BN, bool SPLIT, class Epi>
+template <int BN, int MODE, class Epi>
 inline cudaError_t launch_tc_gemm(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mA2,
                                   const CUtensorMap& mB2, const Epi& epi, int H, int M, int N, int K, int chunk_k,
-                                  DevStatus* stt, cudaStream_t st) {
-  using C = TcCfg<BN, SPLIT>;
-  auto kern = tc_gemm_kernel<BN, SPLIT, Epi>;
+                                  DevStatus* stt, cudaStream_t st, int K1 = 0) {
+  using C = TcCfg<BN, MODE>;
+  auto kern = tc_gemm_kernel<BN, MODE, Epi>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
   dim3 grid(cdiv(N, BN), cdiv(M, 128), H);
-  kern<<<grid, 192, C::SMEM, st>>>(mA, mB, mA2, mB2, epi, M, N, K, chunk_k, stt);
+  kern<<<grid, 192, C::SMEM, st>>>(mA, mB, mA2, mB2, epi, M, N, K, chunk_k, K1, stt);
   return cudaGetLastError();
 }
 

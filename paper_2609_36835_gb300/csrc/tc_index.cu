@@ -72,7 +72,7 @@ int launch_index_logits(const Dims& D, const bf16* qbar_hi, const bf16* qbar_lo,
       !encode_bf16_map_3d(&mB, kbar_hi, D.HD, D.T, D.H, 128) || !encode_bf16_map_3d(&mB2, kbar_lo, D.HD, D.T, D.H, 128))
     return -1;
   TcEpiIndex epi{wts, I, part, D.n, D.T, D.H_I, D.G, D.n_pos, cdiv(D.T, 128)};
-  if (launch_tc_gemm<128, true>(mA, mB, mA2, mB2, epi, D.H, D.n, D.T, D.HD, 128, stt, st) != cudaSuccess) return -1;
+  if (launch_tc_gemm<128, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.n, D.T, D.HD, 128, stt, st) != cudaSuccess) return -1;
   return 1;
 }
 
