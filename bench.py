@@ -64,6 +64,8 @@ def parse_args(argv=None):
     ap.add_argument("--impl", choices=("gpu", "reference"), default="gpu")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--streams", type=int, default=4,
+                    help="CUDA streams (each with its own workspace) the layers of a context are spread over")
     ap.add_argument("--cpu-pairs", type=int, default=4, help="(layer, head) pairs the oracle baseline times")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-layer", action="store_true",
@@ -280,20 +282,43 @@ def run_gpu(args, dist: Dist):
 
     host = [workload.layer_inputs_np(w, l, list(range(w.H_kv))) for l in layers]
     dev_in = [workload.to_device(a, dev) for a in host]
-    ws = torch.empty(pk.workspace_bytes(cfg), dtype=torch.uint8, device=dev)
+    # layers are independent: they are spread round-robin over `n_str` streams,
+    # each with its own workspace (arckv_compact is reentrant per workspace/stream)
+    n_str = max(1, min(args.streams, len(layers)))
+    wss = [torch.empty(pk.workspace_bytes(cfg), dtype=torch.uint8, device=dev) for _ in range(n_str)]
     f32 = dict(dtype=torch.float32, device=dev)
     outs = [{"C_k": torch.empty(w.H_kv, w.t, 128, **f32), "beta": torch.empty(w.H_kv, w.t, **f32),
              "C_v": torch.empty(w.H_kv, w.t, 128, **f32)} for _ in layers]
     stream = torch.cuda.current_stream(dev)
+    streams = [stream] + [torch.cuda.Stream(dev) for _ in range(n_str - 1)]
 
     def compact(i, events=None, c=cfg, ins=None, out=None):
         t = ins if ins is not None else dev_in[i]
         o = out if out is not None else outs[i]
+        ws, s_i = wss[i % n_str], streams[i % n_str]
         st, nl = pk.arckv_compact(c, t["K"], t["V"], t["Q"], t["X"], workload.indexer_dict(t), o["C_k"],
-                                  o["beta"], o["C_v"], ws, ws.numel(), stream=stream, stage_events=events)
+                                  o["beta"], o["C_v"], ws, ws.numel(), stream=s_i, stage_events=events)
         if st != 0:
             raise pk.ArckvError(st, "arckv_compact")
         return nl
+
+    def fork():
+        e = torch.cuda.Event()
+        e.record(stream)
+        for s_i in streams[1:]:
+            s_i.wait_event(e)
+
+    def join():
+        for s_i in streams[1:]:
+            e = torch.cuda.Event()
+            e.record(s_i)
+            stream.wait_event(e)
+
+    def statuses():
+        for ws, s_i in zip(wss, streams):
+            code = pk.arckv_query_status(ws, s_i)
+            if code != 0:
+                raise pk.ArckvError(code, "timed region")
 
     if args.profile_layer:
         compact(0, c=cfg_block)
@@ -306,20 +331,27 @@ def run_gpu(args, dist: Dist):
     for i in range(len(layers)):
         compact(i, c=cfg_block)
 
-    def new_events(k):
+    def new_events(k, s_i=None):
         evs = [torch.cuda.Event(enable_timing=True) for _ in range(k)]
         for e in evs:
-            e.record(stream)
+            e.record(s_i if s_i is not None else stream)
         return evs
 
-    for _ in range(args.warmup):
+    def step(handles=None):
+        n = 0
+        fork()
         for i in range(len(layers)):
-            compact(i)
+            n += compact(i, handles[i] if handles is not None else None)
+        join()
+        return n
+
+    for _ in range(args.warmup):
+        step()
     torch.cuda.synchronize()
 
     n_ev = pk.NUM_STAGES + 1
-    ev_sets = [[new_events(n_ev) for _ in layers] for _ in range(args.steps)]
-    handles = [[[e.cuda_event for e in evs] for evs in step] for step in ev_sets]
+    ev_sets = [[new_events(n_ev, streams[i % n_str]) for i in range(len(layers))] for _ in range(args.steps)]
+    handles = [[[e.cuda_event for e in evs] for evs in st_] for st_ in ev_sets]
     t_start, t_end = new_events(2)
     launches = 0
     clocks = ClockSampler(dist.local_rank)
@@ -329,8 +361,7 @@ def run_gpu(args, dist: Dist):
     torch.cuda.synchronize()
     t_start.record(stream)
     for s in range(args.steps):
-        for i in range(len(layers)):
-            launches += compact(i, handles[s][i])
+        launches += step(handles[s])
     t_end.record(stream)
     torch.cuda.synchronize()
     dist.barrier()
@@ -338,10 +369,8 @@ def run_gpu(args, dist: Dist):
     ms_total = t_start.elapsed_time(t_end)
     ms_total = dist.max(ms_total, dev)
     ms_step = ms_total / args.steps
-    # status of the timed calls: one blocking read
-    st = pk.arckv_query_status(ws, stream)
-    if st != 0:
-        raise pk.ArckvError(st, "timed region")
+    # status of the timed calls: one blocking read per workspace
+    statuses()
 
     stage_ms = [[0.0] * pk.NUM_STAGES for _ in range(1)][0]
     logits_ms = []
@@ -372,12 +401,15 @@ def run_gpu(args, dist: Dist):
     d2h = sum(t.numel() * t.element_size() for o in host_out for t in o.values())
 
     def e2e_step():
+        fork()
         for i in range(len(layers)):
-            for k, t in pinned[i].items():
-                dev_in[i][k].copy_(t, non_blocking=True)
-            compact(i)
-            for k, t in outs[i].items():
-                host_out[i][k].copy_(t, non_blocking=True)
+            with torch.cuda.stream(streams[i % n_str]):
+                for k, t in pinned[i].items():
+                    dev_in[i][k].copy_(t, non_blocking=True)
+                compact(i)
+                for k, t in outs[i].items():
+                    host_out[i][k].copy_(t, non_blocking=True)
+        join()
 
     e2e_step()
     torch.cuda.synchronize()
@@ -390,8 +422,7 @@ def run_gpu(args, dist: Dist):
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = dist.max(e0.elapsed_time(e1), dev) / args.e2e_steps
-    if pk.arckv_query_status(ws, stream) != 0:
-        raise RuntimeError("e2e status")
+    statuses()
 
     value = dist.world * w.T / (ms_step / 1e3)
     line = {
@@ -401,7 +432,9 @@ def run_gpu(args, dist: Dist):
         "config": workload_config(w, "inputs larger than L2 (%.2f GB per context)" %
                                   (h2d / 1e9)),
         "s_per_context": ms_step / 1e3,
+        "streams": n_str,
         "stage_ms_per_step": dict(zip(pk.STAGE_NAMES, stage_ms)),
+        "stage_note": "per-layer event spans summed over layers; with several streams the spans overlap",
         "gpu_launches": launches,
         "roofline": roofline,
         "e2e": {"value": dist.world * w.T / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,

@@ -8,8 +8,9 @@
 //        (P^T P^ + lam_v I) C_v = P^T Y, Y = softmax(scale Q K^T) V   (Eq. value_lstsq)
 // with lam = ridge * trace(Gram) / t.  Both systems are solved by a blocked
 // right-looking Cholesky factorisation (64 x 64 blocks; each diagonal block
-// is factored and inverted in shared memory) followed by blocked forward and
-// backward substitution.
+// is factored and inverted in shared memory) with the forward substitution
+// fused into the trailing updates, then blocked back substitution, all in one
+// cluster launch per system (chol_cluster_kernel).
 #include "gemm.cuh"
 #include "kernels.h"
 #include "tc_gemm.cuh"
@@ -37,306 +38,290 @@ __global__ void mass_rhs_kernel(const float* Phi, const float* m, float* rhs, in
   rhs[(long long)b * t + r] = a;
 }
 
-// Gram += ridge * trace(Gram) / t * I, one CTA per head.
-__global__ void ridge_kernel(float* Gram, int t, float ridge, DevStatus* stt) {
-  const int b = blockIdx.x;
-  float* G = Gram + (long long)b * t * t;
-  __shared__ float red[32];
-  float a = 0.f;
-  for (int r = threadIdx.x; r < t; r += blockDim.x) a += G[(long long)r * t + r];
-  a = warp_sum(a);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = a;
-  __syncthreads();
-  if (threadIdx.x < 32) {
-    float v = (threadIdx.x < (blockDim.x >> 5)) ? red[threadIdx.x] : 0.f;
-    v = warp_sum(v);
-    if (threadIdx.x == 0) red[0] = v;
-  }
-  __syncthreads();
-  const float tr = red[0];
-  if (!isfinite(tr)) set_status(stt, ARCKV_ERR_NONFINITE);
-  const float lam = ridge * tr / (float)t;
-  for (int r = threadIdx.x; r < t; r += blockDim.x) G[(long long)r * t + r] += lam;
+// ---------------------------------------------------------------------------
+// Cluster Cholesky solver: (Gram + lam I) X = B for every head in ONE launch.
+// One cluster of kCL CTAs per head; the matrix, its factor and the right-hand
+// sides live in global memory (L2-resident at these sizes) and are read with
+// ld.global.cg so that no CTA sees a stale L1 line of another CTA's writes.
+// Phases of each 64-wide block step k are separated by hardware cluster
+// barriers (release / acquire at cluster scope):
+//   trsm    L_ik = A_ik Linv_kk^T for block rows i > k (round robin);
+//   update  A_ij -= L_ik L_jk^T (k < j <= i) and B_i -= L_ik (Linv_kk B_k);
+//           the CTA that owns block k+1 updates the diagonal block first and
+//           factors it at once, overlapping the serial factorisation with the
+//           other CTAs' updates;
+// then block back substitution X_k = Linv_kk^T (Linv_kk B_k + Z_k),
+// Z_i -= L_ki^T X_k (i < k).  lam = ridge * trace(Gram) / t is added to the
+// diagonal as each diagonal block is factored.
+constexpr int kCL = 8;
+constexpr int kCT = 512;
+constexpr int kTileF = NB * (NB + 1);
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ unsigned cluster_rank() {
+  unsigned r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
 }
 
-// Factor the (already updated) diagonal block k in shared memory, write L_kk
-// into A and its inverse into Linv[b][k] (64 x 64, identity beyond the matrix).
-// Left-looking by columns with 16 threads per row: at column c every row
-// r >= c forms A_rc - sum_{q<c} L_rq L_cq, the pivot row takes the square
-// root and the rows below divide.  The inverse is formed row by row:
-// Li_ij = (delta_ij - sum_{l=j}^{i-1} L_il Li_lj) / L_ii, all j of a row at once.
-__global__ void __launch_bounds__(1024) potrf_diag_kernel(float* A, int t, int k, float* Linv, int nblk,
-                                                          DevStatus* stt) {
-  const int b = blockIdx.x, tid = threadIdx.x;
-  float* Ab = A + (long long)b * t * t;
-  const int k0 = k * NB, kb = min(NB, t - k0);
-  __shared__ float L[NB][NB + 1];
-  __shared__ float Li[NB][NB + 1];
-  __shared__ int bad;
-  for (int e = tid; e < NB * NB; e += 1024) {
+// S[r][c] = G[(r0 + r) * ld + c0 + c] (or its transpose with `trans`), zero outside
+// rows < rmax, cols < cmax of the source block.
+__device__ __forceinline__ void ld_tile(float (*S)[NB + 1], const float* G, long long ld, int r0, int c0, int rmax,
+                                        int cmax, bool trans) {
+  for (int e = threadIdx.x; e < NB * NB; e += kCT) {
     const int r = e / NB, c = e % NB;
-    L[r][c] = (r < kb && c <= r) ? Ab[(long long)(k0 + r) * t + k0 + c] : (r == c ? 1.f : 0.f);
+    const float v = (r < rmax && c < cmax) ? __ldcg(G + (long long)(r0 + r) * ld + c0 + c) : 0.f;
+    if (trans) S[c][r] = v;
+    else S[r][c] = v;
+  }
+}
+
+// acc[p][q] = sum_l X[ry+p][l] Y[l][cx+q], ry = (tid >> 4) * 2, cx = (tid & 15) * 4.
+__device__ __forceinline__ void mm64(const float (*X)[NB + 1], const float (*Y)[NB + 1], float (&acc)[2][4]) {
+  const int ry = (threadIdx.x >> 4) * 2, cx = (threadIdx.x & 15) * 4;
+#pragma unroll
+  for (int p = 0; p < 2; ++p)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
+#pragma unroll 8
+  for (int l = 0; l < NB; ++l) {
+    // rows of the [64][65] tiles are 260 bytes apart: scalar loads only
+    const float a0 = X[ry][l], a1 = X[ry + 1][l];
+    const float c0 = Y[l][cx], c1 = Y[l][cx + 1], c2 = Y[l][cx + 2], c3 = Y[l][cx + 3];
+    acc[0][0] = fmaf(a0, c0, acc[0][0]); acc[0][1] = fmaf(a0, c1, acc[0][1]);
+    acc[0][2] = fmaf(a0, c2, acc[0][2]); acc[0][3] = fmaf(a0, c3, acc[0][3]);
+    acc[1][0] = fmaf(a1, c0, acc[1][0]); acc[1][1] = fmaf(a1, c1, acc[1][1]);
+    acc[1][2] = fmaf(a1, c2, acc[1][2]); acc[1][3] = fmaf(a1, c3, acc[1][3]);
+  }
+}
+
+// Factor diagonal block k (lower part of A_kk + lam I) in shared memory; write
+// L_kk into A and its inverse into Linv[k].  8 threads per row.
+__device__ void factor_diag(float* Ab, float* Lb, int t, int k, float lam, float (*L)[NB + 1],
+                            float (*Li)[NB + 1], int* bad) {
+  const int tid = threadIdx.x, k0 = k * NB, kb = min(NB, t - k0);
+  for (int e = tid; e < NB * NB; e += kCT) {
+    const int r = e / NB, c = e % NB;
+    L[r][c] = (r < kb && c <= r) ? __ldcg(Ab + (long long)(k0 + r) * t + k0 + c) + (r == c ? lam : 0.f)
+                                 : (r == c ? 1.f : 0.f);
     Li[r][c] = 0.f;
   }
-  if (tid == 0) bad = 0;
   __syncthreads();
-  const int r = tid >> 4, p = tid & 15;
+  const int r = tid >> 3, p = tid & 7;
   for (int c = 0; c < NB; ++c) {
-    // columns < c are final (the previous iteration ended with a barrier)
     float v = 0.f;
     if (r >= c)
-      for (int q = p; q < c; q += 16) v = fmaf(L[r][q], L[c][q], v);
-#pragma unroll
-    for (int o = 1; o < 16; o <<= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+      for (int q = p; q < c; q += 8) v = fmaf(L[r][q], L[c][q], v);
+    v += __shfl_xor_sync(0xffffffffu, v, 1);
+    v += __shfl_xor_sync(0xffffffffu, v, 2);
+    v += __shfl_xor_sync(0xffffffffu, v, 4);
     v = (r >= c) ? L[r][c] - v : 0.f;
     if (r == c && p == 0) {
-      if (!(v > 0.f) || !isfinite(v)) { bad = 1; v = 1.f; }
+      if (!(v > 0.f) || !isfinite(v)) { *bad = 1; v = 1.f; }
       L[c][c] = sqrtf(v);
     }
     __syncthreads();
     if (r > c && p == 0) L[r][c] = v / L[c][c];
     __syncthreads();
   }
-  if (tid == 0 && bad) set_status(stt, ARCKV_ERR_NOT_SPD);
-  const int j = tid >> 4;
   for (int i = 0; i < NB; ++i) {
     float v = 0.f;
-    if (j < i)
-      for (int l = j + p; l < i; l += 16) v = fmaf(L[i][l], Li[l][j], v);
-#pragma unroll
-    for (int o = 1; o < 16; o <<= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    if (j <= i && p == 0) Li[i][j] = ((i == j ? 1.f : 0.f) - v) / L[i][i];
+    if (r < i)
+      for (int l = r + p; l < i; l += 8) v = fmaf(L[i][l], Li[l][r], v);
+    v += __shfl_xor_sync(0xffffffffu, v, 1);
+    v += __shfl_xor_sync(0xffffffffu, v, 2);
+    v += __shfl_xor_sync(0xffffffffu, v, 4);
+    if (r <= i && p == 0) Li[i][r] = ((i == r ? 1.f : 0.f) - v) / L[i][i];
     __syncthreads();
   }
-  float* Lo = Linv + ((long long)b * nblk + k) * NB * NB;
-  for (int e = tid; e < NB * NB; e += 1024) {
+  float* Lo = Lb + (long long)k * NB * NB;
+  for (int e = tid; e < NB * NB; e += kCT) {
     const int rr = e / NB, cc = e % NB;
     Lo[e] = Li[rr][cc];
     if (rr < kb && cc <= rr) Ab[(long long)(k0 + rr) * t + k0 + cc] = L[rr][cc];
   }
+  __syncthreads();
 }
 
-// L_ik = A_ik Linv_kk^T for the block rows below k.
-__global__ void __launch_bounds__(256) trsm_kernel(float* A, int t, int k, const float* Linv, int nblk) {
-  const int b = blockIdx.y, tid = threadIdx.x;
-  const int i = k + 1 + blockIdx.x, i0 = i * NB, rb = min(NB, t - i0), k0 = k * NB;
-  float* Ab = A + (long long)b * t * t;
-  __shared__ float Aik[NB][NB + 1];
-  __shared__ float Li[NB][NB + 1];
-  const float* Lk = Linv + ((long long)b * nblk + k) * NB * NB;
-  for (int e = tid; e < NB * NB; e += 256) {
-    const int r = e / NB, c = e % NB;
-    Aik[r][c] = (r < rb) ? Ab[(long long)(i0 + r) * t + k0 + c] : 0.f;
-    Li[r][c] = Lk[e];
+__global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
+    chol_cluster_kernel(float* A, float* Linv, float* B, float* Z, float* X, int t, int nrhs, int ldb,
+                        long long bbs, float ridge, DevStatus* stt) {
+  extern __shared__ float sm[];
+  float (*S1)[NB + 1] = (float (*)[NB + 1])sm;
+  float (*S2)[NB + 1] = (float (*)[NB + 1])(sm + kTileF);
+  float (*S3)[NB + 1] = (float (*)[NB + 1])(sm + 2 * kTileF);
+  __shared__ float red[kCT / 32];
+  __shared__ int bad;
+  const int head = blockIdx.x / kCL;
+  const int rank = (int)cluster_rank();
+  const int tid = threadIdx.x;
+  const int nblk = (t + NB - 1) / NB, nct = (nrhs + NB - 1) / NB;
+  float* Ab = A + (long long)head * t * t;
+  float* Lb = Linv + (long long)head * nblk * NB * NB;
+  float* Bb = B + (long long)head * bbs;
+  float* Zb = Z + (long long)head * bbs;
+  float* Xb = X + (long long)head * bbs;
+  const int ry = (tid >> 4) * 2, cx = (tid & 15) * 4;
+  float acc[2][4];
+
+  // lam = ridge * trace / t (every CTA forms it; the trace precedes all writes)
+  float tr = 0.f;
+  for (int r = tid; r < t; r += kCT) tr += __ldcg(Ab + (long long)r * t + r);
+  tr = warp_sum(tr);
+  if ((tid & 31) == 0) red[tid >> 5] = tr;
+  if (tid == 0) bad = 0;
+  __syncthreads();
+  if (tid < 32) {
+    float v = tid < kCT / 32 ? red[tid] : 0.f;
+    v = warp_sum(v);
+    if (tid == 0) red[0] = v;
   }
   __syncthreads();
-  const int r = tid >> 2;
-  float out[16];
-#pragma unroll
-  for (int q = 0; q < 16; ++q) out[q] = 0.f;
-  for (int l = 0; l < NB; ++l) {
-    const float a = Aik[r][l];
-#pragma unroll
-    for (int q = 0; q < 16; ++q) out[q] = fmaf(a, Li[(tid & 3) + 4 * q][l], out[q]);
-  }
-  if (r < rb) {
-#pragma unroll
-    for (int q = 0; q < 16; ++q) Ab[(long long)(i0 + r) * t + k0 + (tid & 3) + 4 * q] = out[q];
-  }
-}
+  const float trace = red[0];
+  const float lam = ridge * trace / (float)t;
+  if (rank == 0 && tid == 0 && !isfinite(trace)) set_status(stt, ARCKV_ERR_NONFINITE);
+  // zero Z (rows split over the cluster) and factor the first diagonal block
+  for (long long e = (long long)rank * kCT + tid; e < (long long)t * ldb; e += (long long)kCL * kCT) Zb[e] = 0.f;
+  cluster_sync_all();   // everyone has read the unmodified diagonal for the trace
+  if (rank == 0) factor_diag(Ab, Lb, t, 0, lam, S1, S2, &bad);
+  cluster_sync_all();
 
-// 64 x 64 tile product helper: acc[p][q] += sum_l X[ry+p][l] * Y[l][cx+q] with
-// X, Y in shared memory ([64][65] layout), ry = (tid>>4)*4, cx = (tid&15)*4.
-__device__ __forceinline__ void tile_mm(const float (*X)[NB + 1], const float (*Y)[NB + 1], float (&acc)[4][4],
-                                        bool transX) {
-  const int ry = (threadIdx.x >> 4) * 4, cx = (threadIdx.x & 15) * 4;
-  for (int l = 0; l < NB; ++l) {
-    float a[4], c[4];
+  for (int k = 0; k < nblk; ++k) {
+    const int m = nblk - k - 1, k0 = k * NB;
+    // trsm: L_ik = A_ik Linv_kk^T
+    for (int x = rank; x < m; x += kCL) {
+      const int i0 = (k + 1 + x) * NB, rb = min(NB, t - i0);
+      ld_tile(S1, Ab, t, i0, k0, rb, NB, false);
+      ld_tile(S2, Lb + (long long)k * NB * NB, NB, 0, 0, NB, NB, true);   // S2[l][c] = Linv[c][l]
+      __syncthreads();
+      mm64(S1, S2, acc);
 #pragma unroll
-    for (int p = 0; p < 4; ++p) { a[p] = transX ? X[l][ry + p] : X[ry + p][l]; c[p] = Y[l][cx + p]; }
+      for (int p = 0; p < 2; ++p)
 #pragma unroll
-    for (int p = 0; p < 4; ++p)
-#pragma unroll
-      for (int q = 0; q < 4; ++q) acc[p][q] = fmaf(a[p], c[q], acc[p][q]);
-  }
-}
-
-// Trailing update of step k.  Blocks [0, ntri): A_ij -= L_ik L_jk^T for the
-// lower blocks k < j <= i.  Blocks [ntri, ntri + m * nct): the forward
-// substitution of the right-hand side B (t x nrhs, row stride ldb):
-// B_i -= L_ik (Linv_kk B_k) for block rows i > k and 64-column tiles of B.
-// B_k itself is only read in this launch (every tile recomputes Linv_kk B_k).
-__global__ void __launch_bounds__(256) update_kernel(float* A, int t, int k, const float* Linv, int nblk,
-                                                     float* B, int ldb, int nrhs, long long bbs) {
-  const int b = blockIdx.y, tid = threadIdx.x;
-  const int m = nblk - k - 1, ntri = m * (m + 1) / 2, k0 = k * NB;
-  float* Ab = A + (long long)b * t * t;
-  __shared__ float S1[NB][NB + 1];
-  __shared__ float S2[NB][NB + 1];
-  const int ry = (tid >> 4) * 4, cx = (tid & 15) * 4;
-  float acc[4][4];
-#pragma unroll
-  for (int p = 0; p < 4; ++p)
-#pragma unroll
-    for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
-  const int x = blockIdx.x;
-  if (x < ntri) {
-    int ii = (int)((sqrtf(8.f * x + 1.f) - 1.f) * 0.5f);
-    while (ii * (ii + 1) / 2 > x) --ii;
-    while ((ii + 1) * (ii + 2) / 2 <= x) ++ii;
-    const int jj = x - ii * (ii + 1) / 2;
-    const int i0 = (k + 1 + ii) * NB, j0 = (k + 1 + jj) * NB;
-    const int rb = min(NB, t - i0), cb = min(NB, t - j0);
-    for (int e = tid; e < NB * NB; e += 256) {
-      const int r = e / NB, c = e % NB;
-      S1[r][c] = (r < rb) ? Ab[(long long)(i0 + r) * t + k0 + c] : 0.f;   // L_ik
-      S2[c][r] = (r < cb) ? Ab[(long long)(j0 + r) * t + k0 + c] : 0.f;   // L_jk^T
+        for (int q = 0; q < 4; ++q)
+          if (ry + p < rb) Ab[(long long)(i0 + ry + p) * t + k0 + cx + q] = acc[p][q];
+      __syncthreads();
     }
-    __syncthreads();
-    tile_mm(S1, S2, acc, false);
+    cluster_sync_all();
+    if (m == 0) break;
+    // update: syrk tiles (ii >= jj over the m trailing blocks) then rhs tiles
+    const int ntri = m * (m + 1) / 2, ntot = ntri + m * nct, owner = (k + 1) % kCL;
+    for (int pass = 0; pass < 2; ++pass) {
+      // pass 0: the owner of block k+1 updates and factors the diagonal block (x = 0)
+      int xb, xs;
+      if (pass == 0) { if (rank != owner) continue; xb = 0; xs = 1; }
+      else { xb = rank; xs = kCL; }
+      for (int x = xb; x < (pass == 0 ? 1 : ntot); x += xs) {
+        if (pass == 1 && x == 0) continue;
+        if (x < ntri) {
+          int ii = (int)((sqrtf(8.f * x + 1.f) - 1.f) * 0.5f);
+          while (ii * (ii + 1) / 2 > x) --ii;
+          while ((ii + 1) * (ii + 2) / 2 <= x) ++ii;
+          const int jj = x - ii * (ii + 1) / 2;
+          const int i0 = (k + 1 + ii) * NB, j0 = (k + 1 + jj) * NB;
+          const int rb = min(NB, t - i0), cb = min(NB, t - j0);
+          ld_tile(S1, Ab, t, i0, k0, rb, NB, false);    // L_ik
+          ld_tile(S2, Ab, t, j0, k0, cb, NB, true);     // S2[l][c] = L_jk[c][l]
+          __syncthreads();
+          mm64(S1, S2, acc);
 #pragma unroll
-    for (int p = 0; p < 4; ++p)
+          for (int p = 0; p < 2; ++p)
 #pragma unroll
-      for (int q = 0; q < 4; ++q)
-        if (ry + p < rb && cx + q < cb) Ab[(long long)(i0 + ry + p) * t + j0 + cx + q] -= acc[p][q];
-    return;
+            for (int q = 0; q < 4; ++q)
+              if (ry + p < rb && cx + q < cb) {
+                float* a = Ab + (long long)(i0 + ry + p) * t + j0 + cx + q;
+                *a = __ldcg(a) - acc[p][q];
+              }
+          __syncthreads();
+          if (pass == 0) factor_diag(Ab, Lb, t, k + 1, lam, S1, S2, &bad);
+        } else {
+          const int y = x - ntri, i = k + 1 + y / nct, c0 = (y % nct) * NB;
+          const int i0 = i * NB, rb = min(NB, t - i0), nc = min(NB, nrhs - c0);
+          ld_tile(S1, Lb + (long long)k * NB * NB, NB, 0, 0, NB, NB, false);   // Linv_kk
+          ld_tile(S2, Bb, ldb, k0, c0, NB, nc, false);                        // B_k (full block)
+          __syncthreads();
+          mm64(S1, S2, acc);                                                  // y = Linv_kk B_k
+          __syncthreads();                                                    // S1 is reloaded below
+#pragma unroll
+          for (int p = 0; p < 2; ++p)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) S3[ry + p][cx + q] = acc[p][q];
+          ld_tile(S1, Ab, t, i0, k0, rb, NB, false);                         // L_ik
+          __syncthreads();
+          mm64(S1, S3, acc);
+#pragma unroll
+          for (int p = 0; p < 2; ++p)
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              if (ry + p < rb && cx + q < nc) {
+                float* bp = Bb + (long long)(i0 + ry + p) * ldb + c0 + cx + q;
+                *bp = __ldcg(bp) - acc[p][q];
+              }
+          __syncthreads();
+        }
+      }
+    }
+    cluster_sync_all();
   }
-  const int nct = (nrhs + NB - 1) / NB;
-  const int y = x - ntri, i = k + 1 + y / nct, c0 = (y % nct) * NB;
-  const int i0 = i * NB, rb = min(NB, t - i0), nc = min(NB, nrhs - c0);
-  float* Bb = B + (long long)b * bbs;
-  const float* Lk = Linv + ((long long)b * nblk + k) * NB * NB;
-  for (int e = tid; e < NB * NB; e += 256) {
-    const int r = e / NB, c = e % NB;
-    S1[r][c] = Lk[e];
-    S2[r][c] = (c < nc) ? Bb[(long long)(k0 + r) * ldb + c0 + c] : 0.f;   // block k is full (k < nblk-1)
+  // back substitution
+  for (int k = nblk - 1; k >= 0; --k) {
+    const int k0 = k * NB, kb = min(NB, t - k0);
+    for (int x = rank; x < (k + 1) * nct; x += kCL) {
+      const int i = x / nct, c0 = (x % nct) * NB, nc = min(NB, nrhs - c0);
+      ld_tile(S1, Lb + (long long)k * NB * NB, NB, 0, 0, NB, NB, false);     // Linv_kk
+      ld_tile(S2, Bb, ldb, k0, c0, kb, nc, false);
+      __syncthreads();
+      mm64(S1, S2, acc);                                                    // Y_k = Linv_kk B_k
+      __syncthreads();                                                      // S2 is reloaded below
+#pragma unroll
+      for (int p = 0; p < 2; ++p)
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          S3[ry + p][cx + q] = acc[p][q] + ((ry + p < kb && cx + q < nc)
+                                                ? __ldcg(Zb + (long long)(k0 + ry + p) * ldb + c0 + cx + q) : 0.f);
+      ld_tile(S2, Lb + (long long)k * NB * NB, NB, 0, 0, NB, NB, true);      // S2[r][l] = Linv[l][r]
+      __syncthreads();
+      mm64(S2, S3, acc);                                                    // X_k = Linv^T (Y_k + Z_k)
+      __syncthreads();
+      if (i == k) {
+#pragma unroll
+        for (int p = 0; p < 2; ++p)
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            if (ry + p < kb && cx + q < nc) Xb[(long long)(k0 + ry + p) * ldb + c0 + cx + q] = acc[p][q];
+      } else {
+#pragma unroll
+        for (int p = 0; p < 2; ++p)
+#pragma unroll
+          for (int q = 0; q < 4; ++q) S3[ry + p][cx + q] = acc[p][q];
+        const int i0 = i * NB;
+        ld_tile(S1, Ab, t, k0, i0, kb, NB, true);                            // S1[r][l] = L_ki[l][r]
+        __syncthreads();
+        mm64(S1, S3, acc);                                                  // L_ki^T X_k
+#pragma unroll
+        for (int p = 0; p < 2; ++p)
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            if (cx + q < nc) {
+              float* zp = Zb + (long long)(i0 + ry + p) * ldb + c0 + cx + q;
+              *zp = __ldcg(zp) - acc[p][q];
+            }
+      }
+      __syncthreads();
+    }
+    cluster_sync_all();
   }
-  __syncthreads();
-  tile_mm(S1, S2, acc, false);   // y = Linv_kk B_k
-  __syncthreads();
-#pragma unroll
-  for (int p = 0; p < 4; ++p)
-#pragma unroll
-    for (int q = 0; q < 4; ++q) S2[ry + p][cx + q] = acc[p][q];
-  for (int e = tid; e < NB * NB; e += 256) {
-    const int r = e / NB, c = e % NB;
-    S1[r][c] = (r < rb) ? Ab[(long long)(i0 + r) * t + k0 + c] : 0.f;    // L_ik
-  }
-  __syncthreads();
-#pragma unroll
-  for (int p = 0; p < 4; ++p)
-#pragma unroll
-    for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
-  tile_mm(S1, S2, acc, false);
-#pragma unroll
-  for (int p = 0; p < 4; ++p)
-#pragma unroll
-    for (int q = 0; q < 4; ++q)
-      if (ry + p < rb && cx + q < nc) Bb[(long long)(i0 + ry + p) * ldb + c0 + cx + q] -= acc[p][q];
+  if (tid == 0 && bad) set_status(stt, ARCKV_ERR_NOT_SPD);
 }
 
-// Backward substitution, step k (block rows from the last down): with
-// Y_k = Linv_kk B_k (B after the forward updates) and Z_k the accumulated
-// -sum_{j>k} L_jk^T X_j,  X_k = Linv_kk^T (Y_k + Z_k).  Block (i = k) writes X_k;
-// blocks i < k apply Z_i -= L_ki^T X_k.  B_k and Z_k are only read here.
-__global__ void __launch_bounds__(256) backward_kernel(const float* A, int t, int k, const float* Linv, int nblk,
-                                                       const float* B, float* Z, float* X, int ldb, int nrhs,
-                                                       long long bbs) {
-  const int b = blockIdx.y, tid = threadIdx.x;
-  const int nct = (nrhs + NB - 1) / NB;
-  const int i = blockIdx.x / nct, c0 = (blockIdx.x % nct) * NB;
-  const int k0 = k * NB, kb = min(NB, t - k0), nc = min(NB, nrhs - c0);
-  const float* Ab = A + (long long)b * t * t;
-  const float* Bb = B + (long long)b * bbs;
-  float* Zb = Z + (long long)b * bbs;
-  float* Xb = X + (long long)b * bbs;
-  const float* Lk = Linv + ((long long)b * nblk + k) * NB * NB;
-  __shared__ float S1[NB][NB + 1];
-  __shared__ float S2[NB][NB + 1];
-  const int ry = (tid >> 4) * 4, cx = (tid & 15) * 4;
-  float acc[4][4];
-#pragma unroll
-  for (int p = 0; p < 4; ++p)
-#pragma unroll
-    for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
-  for (int e = tid; e < NB * NB; e += 256) {
-    const int r = e / NB, c = e % NB;
-    S1[r][c] = Lk[e];
-    S2[r][c] = (r < kb && c < nc) ? Bb[(long long)(k0 + r) * ldb + c0 + c] : 0.f;
-  }
-  __syncthreads();
-  tile_mm(S1, S2, acc, false);          // Y_k = Linv_kk B_k
-  __syncthreads();
-#pragma unroll
-  for (int p = 0; p < 4; ++p)
-#pragma unroll
-    for (int q = 0; q < 4; ++q)
-      S2[ry + p][cx + q] = acc[p][q] + ((ry + p < kb && cx + q < nc)
-                                            ? Zb[(long long)(k0 + ry + p) * ldb + c0 + cx + q] : 0.f);
-  __syncthreads();
-#pragma unroll
-  for (int p = 0; p < 4; ++p)
-#pragma unroll
-    for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
-  tile_mm(S1, S2, acc, true);           // X_k = Linv_kk^T (Y_k + Z_k)
-  if (i == k) {
-#pragma unroll
-    for (int p = 0; p < 4; ++p)
-#pragma unroll
-      for (int q = 0; q < 4; ++q)
-        if (ry + p < kb && cx + q < nc) Xb[(long long)(k0 + ry + p) * ldb + c0 + cx + q] = acc[p][q];
-    return;
-  }
-  __syncthreads();
-#pragma unroll
-  for (int p = 0; p < 4; ++p)
-#pragma unroll
-    for (int q = 0; q < 4; ++q) S2[ry + p][cx + q] = acc[p][q];
-  const int i0 = i * NB;   // i < k: a full block
-  for (int e = tid; e < NB * NB; e += 256) {
-    const int r = e / NB, c = e % NB;
-    S1[r][c] = (r < kb) ? Ab[(long long)(k0 + r) * t + i0 + c] : 0.f;     // L_ki[r][c]
-  }
-  __syncthreads();
-#pragma unroll
-  for (int p = 0; p < 4; ++p)
-#pragma unroll
-    for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
-  tile_mm(S1, S2, acc, true);           // L_ki^T X_k
-#pragma unroll
-  for (int p = 0; p < 4; ++p)
-#pragma unroll
-    for (int q = 0; q < 4; ++q)
-      if (cx + q < nc) Zb[(long long)(i0 + ry + p) * ldb + c0 + cx + q] -= acc[p][q];
-}
-
-// Solve (Gram + lam I) X = B for each head: ridge, blocked Cholesky with the
-// forward substitution of B fused into the trailing updates, then backward
-// substitution.  B (t x nrhs, stride ldb) is overwritten; Z is scratch of the
-// same shape; X receives the solution.
 static int cholesky_solve(int H, int t, float* Gram, float* Linv, float* B, float* Z, float* X, int ldb,
                           int nrhs, long long bbs, float ridge, DevStatus* stt, cudaStream_t st) {
-  int nl = 0;
-  ridge_kernel<<<H, 256, 0, st>>>(Gram, t, ridge, stt);
-  ++nl;
-  const int nblk = cdiv(t, NB), nct = cdiv(nrhs, NB);
-  for (int k = 0; k < nblk; ++k) {
-    potrf_diag_kernel<<<H, 1024, 0, st>>>(Gram, t, k, Linv, nblk, stt);
-    ++nl;
-    const int m = nblk - k - 1;
-    if (m > 0) {
-      trsm_kernel<<<dim3(m, H), 256, 0, st>>>(Gram, t, k, Linv, nblk);
-      update_kernel<<<dim3(m * (m + 1) / 2 + m * nct, H), 256, 0, st>>>(Gram, t, k, Linv, nblk, B, ldb, nrhs,
-                                                                          bbs);
-      nl += 2;
-    }
-  }
-  cudaMemsetAsync(Z, 0, sizeof(float) * (size_t)H * bbs, st);
-  for (int k = nblk - 1; k >= 0; --k) {
-    backward_kernel<<<dim3((k + 1) * nct, H), 256, 0, st>>>(Gram, t, k, Linv, nblk, B, Z, X, ldb, nrhs, bbs);
-    ++nl;
-  }
-  return nl;
+  const int smem = 3 * kTileF * (int)sizeof(float);
+  cudaFuncSetAttribute(chol_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  chol_cluster_kernel<<<kCL * H, kCT, smem, st>>>(Gram, Linv, B, Z, X, t, nrhs, ldb, bbs, ridge, stt);
+  return 1;
 }
 
 __global__ void beta_kernel(const float* w, float* beta, long long count, float eps_w, float b_min, float b_max) {
