@@ -14,9 +14,9 @@ constexpr size_t kAlign = 256;
 inline size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct Layout {
-  size_t status, W1, W2, kbar_hi, kbar_lo, Uk, Uv, vq, cctx, qbar_hi, qbar_lo, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
+  size_t status, kbar_hi, kbar_lo, vq, qpp, q_h, q_m, q_l, av, VT, p_h, p_m, p_l, cctx, qbar_hi, qbar_lo, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
       colM, colInvN, Ut_hi, Ut_lo, S_hi, S_lo, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z,
-      YT_hi, YT_lo, split, total;
+      YT_hi, YT_lo, total;
 };
 
 Dims dims_of(const arckv_config& c) {
@@ -56,13 +56,19 @@ Layout plan(const arckv_config& c) {
   size_t o = 0;
   auto take = [&](size_t bytes) { size_t r = o; o += up(bytes); return r; };
   L.status = take(sizeof(DevStatus));
-  L.W1 = take(H * (HD + 256) * 128 * 2);
-  L.W2 = take(H * (HD + 256) * 128 * 2);
+  const size_t ldT = (T + 7) / 8 * 8;
   L.kbar_hi = take(H * T * HD * 2);
   L.kbar_lo = take(H * T * HD * 2);
-  L.Uk = take(H * T * 128 * f);
-  L.Uv = take(H * T * 128 * f);
   L.vq = take(H * n * 128 * f);
+  L.qpp = take(H * n * 128 * f);
+  L.q_h = take(H * n * 128 * 2);
+  L.q_m = take(H * n * 128 * 2);
+  L.q_l = take(H * n * 128 * 2);
+  L.av = take(H * n * 128 * f);
+  L.VT = take(H * 128 * ldT * 2);
+  L.p_h = take(H * n * ldT * 2);
+  L.p_m = take(H * n * ldT * 2);
+  L.p_l = take(H * n * ldT * 2);
   L.cctx = take(H * n * 128 * f);
   L.qbar_hi = take(H * n * HD * 2);
   L.qbar_lo = take(H * n * HD * 2);
@@ -101,7 +107,6 @@ Layout plan(const arckv_config& c) {
   L.Z = take(H * t * 128 * f);
   L.YT_hi = take(H * 128 * ldn * 2);
   L.YT_lo = take(H * 128 * ldn * 2);
-  L.split = take((size_t)kSplitK * H * (n > t ? n : t) * 128 * f);
   L.total = o;
   return L;
 }
@@ -185,18 +190,22 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
   cudaGetLastError();  // clear a stale error from earlier, unrelated work
   if (cudaMemsetAsync(stt, 0, sizeof(DevStatus), st) != cudaSuccess) return ARCKV_ERR_CUDA;
   int* anchors = I32(L.anchors);
+  auto B16 = [&](size_t off) { return (bf16*)(w + off); };
   mark(0);
+  nl += launch_transpose_v(D, Vb, B16(L.VT), st);
   if (!given_anchors) {
-    auto B16 = [&](size_t off) { return (bf16*)(w + off); };
-    const int nlk = launch_key_features_tc(D, Kb, Vb, (const bf16*)idx->L_k, (const bf16*)idx->L_v,
-                                           (const bf16*)idx->U_k, (const bf16*)idx->U_v, B16(L.W1), B16(L.W2),
-                                           B16(L.kbar_hi), B16(L.kbar_lo), F(L.Uk), F(L.Uv), stt, st);
+    const int nlk = launch_key_features_tc(D, Kb, Vb, (const bf16*)idx->L_k, (const bf16*)idx->L_v, B16(L.kbar_hi),
+                                           B16(L.kbar_lo), stt, st);
     if (nlk < 0) return ARCKV_ERR_CUDA;
     nl += nlk;
-    nl += launch_query_features(D, Qb, (const bf16*)X_ref, (const bf16*)idx->U_q, (const bf16*)idx->L_q,
-                                (const bf16*)idx->L_c, (const bf16*)idx->L_x, (const bf16*)idx->b_x, F(L.Uk),
-                                F(L.Uv), F(L.vq), F(L.NT), F(L.rA), F(L.rB), F(L.split), F(L.cctx),
-                                B16(L.qbar_hi), B16(L.qbar_lo), F(L.wts), st);
+    QueryBufs QB{F(L.vq), F(L.qpp), F(L.NT), F(L.rA), F(L.rB), F(L.av), F(L.cctx),
+                 B16(L.q_h), B16(L.q_m), B16(L.q_l), B16(L.p_h), B16(L.p_m), B16(L.p_l)};
+    const int nlq = launch_query_features(D, Qb, (const bf16*)X_ref, Kb, B16(L.VT), (const bf16*)idx->U_q,
+                                          (const bf16*)idx->U_k, (const bf16*)idx->U_v, (const bf16*)idx->L_q,
+                                          (const bf16*)idx->L_c, (const bf16*)idx->L_x, (const bf16*)idx->b_x, QB,
+                                          B16(L.qbar_hi), B16(L.qbar_lo), F(L.wts), stt, st);
+    if (nlq < 0) return ARCKV_ERR_CUDA;
+    nl += nlq;
     mark(1);
     const int nli = launch_index_logits(D, B16(L.qbar_hi), B16(L.qbar_lo), B16(L.kbar_hi), B16(L.kbar_lo),
                                         F(L.wts), F(L.NT), (float2*)(w + L.part), stt, st);
@@ -212,13 +221,13 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
     nl += launch_check_anchors(D, anchors, stt, st);
   }
   mark(3);
-  const int nlr = launch_reference_attention(D, scale, Qb, Kb, Vb, F(L.NT), F(L.z), F(L.m), F(L.invm), F(L.split),
-                                             F(L.Y), F(L.logphi), F(L.colM), F(L.colInvN), stt, st);
+  const int nlr = launch_reference_attention(D, scale, Qb, Kb, B16(L.VT), F(L.NT), F(L.z), F(L.m), F(L.invm),
+                                             B16(L.p_h), B16(L.p_m), B16(L.p_l), F(L.Y), F(L.logphi), F(L.colM),
+                                             F(L.colInvN), stt, st);
   if (nlr < 0) return ARCKV_ERR_CUDA;
   nl += nlr;
   int* kappa = I32(L.kappa);
   if (!given_assign) {
-    auto B16 = [&](size_t off) { return (bf16*)(w + off); };
     const int nla = launch_assign_tc(D, F(L.NT), F(L.colM), F(L.colInvN), anchors, B16(L.Ut_hi), B16(L.Ut_lo),
                                      B16(L.S_hi), B16(L.S_lo), (unsigned long long*)(w + L.best), kappa, stt, st);
     if (nla < 0) return ARCKV_ERR_CUDA;
@@ -231,7 +240,7 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
   nl += launch_merge(D, cfg->lambda_m, Kb, anchors, kappa, F(L.logphi), I32(L.perm), I32(L.goff), I32(L.cursor),
                      C_k, st);
   mark(5);
-  FitBufs B{F(L.LC),  F(L.Phi), F(L.Gram), F(L.Linv), F(L.rhs), F(L.wsol), F(L.R), F(L.Z), F(L.split),
+  FitBufs B{F(L.LC),  F(L.Phi), F(L.Gram), F(L.Linv), F(L.rhs), F(L.wsol), F(L.R), F(L.Z),
             (bf16*)(w + L.S_hi), (bf16*)(w + L.S_lo), (bf16*)(w + L.YT_hi), (bf16*)(w + L.YT_lo)};
   const int nlf = launch_fits(D, scale, cfg->ridge_w, cfg->ridge_v, cfg->eps_w, cfg->b_min, cfg->b_max, Qb, C_k,
                               F(L.z), F(L.m), F(L.Y), B, beta, C_v, stt, st);

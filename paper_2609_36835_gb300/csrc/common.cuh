@@ -40,6 +40,16 @@ __device__ __forceinline__ void split_bf16(float x, bf16& hi, bf16& lo) {
   lo = __float2bfloat16_rn(x - __bfloat162float(hi));
 }
 
+// bf16 triple (h, m, l) with x = h + m + l to within 2^-24 relative: an fp32
+// value carried exactly enough for fp32-grade tensor-core products against an
+// exact bf16 operand.
+__device__ __forceinline__ void split3_bf16(float x, bf16& h, bf16& m, bf16& l) {
+  h = __float2bfloat16_rn(x);
+  const float r1 = x - __bfloat162float(h);
+  m = __float2bfloat16_rn(r1);
+  l = __float2bfloat16_rn(r1 - __bfloat162float(m));
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);

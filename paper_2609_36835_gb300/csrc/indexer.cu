@@ -34,31 +34,34 @@ __global__ void __launch_bounds__(256) index_weights_kernel(const bf16* X, const
   }
 }
 
-int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf16* U_q, const bf16* L_q,
-                          const bf16* L_c, const bf16* L_x, const bf16* b_x, const float* Uk,
-                          const float* Uv, float* vq, float* logits, float* rshift, float* rmul,
-                          float* split, float* cctx, bf16* qbar_hi, bf16* qbar_lo, float* wts, cudaStream_t st) {
+int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf16* K, const bf16* VT,
+                          const bf16* U_q, const bf16* U_k, const bf16* U_v, const bf16* L_q, const bf16* L_c,
+                          const bf16* L_x, const bf16* b_x, const QueryBufs& B, bf16* qbar_hi, bf16* qbar_lo,
+                          float* wts, DevStatus* stt, cudaStream_t st) {
   int nl = 0;
-  const long long nd = (long long)D.n * D.d, nA = (long long)D.n * D.d_A, TA = (long long)D.T * D.d_A;
-  // vq = U_q q
-  launch_gemm(RowK<bf16>{Q, nd, D.d}, RowK<bf16>{U_q, (long long)D.d_A * D.d, D.d},
-              EpiStore{vq, nA, 0, D.d_A, 1.f, false}, D.H, D.n, D.d_A, D.d, 1, st);
+  const long long nd = (long long)D.n * D.d, nA = (long long)D.n * D.d_A, dd = (long long)D.d_A * D.d;
+  // vq = U_q q;  q'' = U_k^T vq, so that (U_q q_i).(U_k k_j) = q''_i . k_j
+  launch_gemm(RowK<bf16>{Q, nd, D.d}, RowK<bf16>{U_q, dd, D.d}, EpiStore{B.vq, nA, 0, D.d_A, 1.f, false}, D.H, D.n,
+              D.d_A, D.d, 1, st);
+  launch_gemm(RowK<float>{B.vq, nA, D.d_A}, ColK<bf16>{U_k, dd, D.d}, EpiStore{B.qpp, nd, 0, D.d, 1.f, false}, D.H,
+              D.n, D.d, D.d_A, 1, st);
+  nl += 2;
+  // value-attention logits on the tensor cores, unscaled as printed in Eq. value_context
+  int r = launch_value_logits_tc(D, B.qpp, B.q_h, B.q_m, B.q_l, K, B.logits, stt, st);
+  if (r < 0) return -1;
+  nl += r;
+  nl += launch_row_stats(D.H, D.n, D.T, B.logits, B.rshift, B.rmul, nullptr, st);
+  // A^V V on the tensor cores, then c = (A^V V) U_v^T = A^V (U_v V)
+  r = launch_probs_v_tc(D, B.logits, B.rshift, B.rmul, B.p_h, B.p_m, B.p_l, VT, B.av, stt, st);
+  if (r < 0) return -1;
+  nl += r;
+  launch_gemm(RowK<float>{B.av, nd, D.d}, RowK<bf16>{U_v, dd, D.d}, EpiStore{B.cctx, nA, 0, D.d_A, 1.f, false},
+              D.H, D.n, D.d_A, D.d, 1, st);
   ++nl;
-  // value-attention logits (U_q q_i).(U_k k_j), unscaled as printed in Eq. value_context
-  launch_gemm(RowK<float>{vq, nA, D.d_A}, RowK<float>{Uk, TA, D.d_A},
-              EpiStore{logits, (long long)D.n * D.T, 0, D.T, 1.f, false}, D.H, D.n, D.T, D.d_A, 1, st);
-  ++nl;
-  nl += launch_row_stats(D.H, D.n, D.T, logits, rshift, rmul, nullptr, st);
-  // c = A^V Uv, split over T
-  RowKExp P{{logits, (long long)D.n * D.T, D.T}, rshift, rmul, D.n, 1.f};
-  launch_gemm(P, ColK<float>{Uv, TA, D.d_A},
-              EpiStore{split, nA, (long long)D.H * nA, D.d_A, 1.f, false}, D.H, D.n, D.d_A, D.T, kSplitK, st);
-  ++nl;
-  nl += launch_split_reduce(D.H, D.n, D.d_A, kSplitK, split, cctx, st);
-  // q_bar = N(L_q q + L_c c) per block
-  CatRowK<bf16, float> A{{Q, nd, D.d}, {cctx, nA, D.d_A}, D.d};
-  CatRowK<bf16, bf16> B{{L_q, (long long)D.HD * D.d, D.d}, {L_c, (long long)D.HD * D.d_A, D.d_A}, D.d};
-  launch_gemm(A, B, EpiBlockNormSplit{qbar_hi, qbar_lo, (long long)D.n * D.HD, D.HD}, D.H, D.n, D.HD,
+  // q_bar = N(L_q q + L_c c) per block, as a split-bf16 pair
+  CatRowK<bf16, float> A{{Q, nd, D.d}, {B.cctx, nA, D.d_A}, D.d};
+  CatRowK<bf16, bf16> W{{L_q, (long long)D.HD * D.d, D.d}, {L_c, (long long)D.HD * D.d_A, D.d_A}, D.d};
+  launch_gemm(A, W, EpiBlockNormSplit{qbar_hi, qbar_lo, (long long)D.n * D.HD, D.HD}, D.H, D.n, D.HD,
               D.d + D.d_A, 1, st);
   ++nl;
   index_weights_kernel<<<dim3(D.n_pos, D.H), 256, 0, st>>>(X, L_x, b_x, wts, D.d_x, D.H_I, D.n_pos);

@@ -13,16 +13,28 @@ constexpr int kSplitK = 8;   // K slices of the skinny (N = 128) long-K products
 constexpr int kCholNB = 64;  // Cholesky block size
 
 // ---- indexer (Sec. 3.3, App. A.1) --------------------------------------
-// k_bar = N(L_k k + L_v v) per d_I block (split bf16); Uk = U_k k; Uv = U_v v
-// (one tcgen05 GEMM over [K | V]; W1, W2 are stacked-weight scratch).
+// k_bar = N(L_k k + L_v v) per d_I block, as a split-bf16 pair (one tcgen05
+// GEMM over [K | V] against [L_k | L_v]).
 int launch_key_features_tc(const Dims& D, const bf16* K, const bf16* V, const bf16* L_k, const bf16* L_v,
-                           const bf16* U_k, const bf16* U_v, bf16* W1, bf16* W2, bf16* kbar_hi, bf16* kbar_lo,
-                           float* Uk, float* Uv, DevStatus* stt, cudaStream_t st);
+                           bf16* kbar_hi, bf16* kbar_lo, DevStatus* stt, cudaStream_t st);
+// Scratch of the query-side features.
+struct QueryBufs {
+  float *vq, *qpp, *logits, *rshift, *rmul, *av, *cctx;
+  bf16 *q_h, *q_m, *q_l, *p_h, *p_m, *p_l;
+};
 // value context c (Eq. value_context), q_bar (Eq. indexer_projection), w.
-int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf16* U_q, const bf16* L_q,
-                          const bf16* L_c, const bf16* L_x, const bf16* b_x, const float* Uk,
-                          const float* Uv, float* vq, float* logits, float* rshift, float* rmul,
-                          float* split, float* cctx, bf16* qbar_hi, bf16* qbar_lo, float* wts, cudaStream_t st);
+// VT is V transposed ([H][d][ldT] bf16, launch_transpose_v).  -1 on a TMA failure.
+int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf16* K, const bf16* VT,
+                          const bf16* U_q, const bf16* U_k, const bf16* U_v, const bf16* L_q, const bf16* L_c,
+                          const bf16* L_x, const bf16* b_x, const QueryBufs& B, bf16* qbar_hi, bf16* qbar_lo,
+                          float* wts, DevStatus* stt, cudaStream_t st);
+// softmax products with fp32-grade split-3 operands (tc_attn.cu)
+int launch_transpose_v(const Dims& D, const bf16* V, bf16* VT, cudaStream_t st);
+int launch_value_logits_tc(const Dims& D, const float* qpp, bf16* q_h, bf16* q_m, bf16* q_l, const bf16* K,
+                           float* logits, DevStatus* stt, cudaStream_t st);
+// out [H][n][128] = (exp(X - shift) * mul) V over rows of X [H][n][T].
+int launch_probs_v_tc(const Dims& D, const float* X, const float* shift, const float* mul, bf16* p_h, bf16* p_m,
+                      bf16* p_l, const bf16* VT, float* out, DevStatus* stt, cudaStream_t st);
 // I (Eq. pairwise_index_score) on tcgen05 with split-bf16 operands, and the
 // per-(row, 128-column tile) softmax partials.  Returns launches, or -1 when a
 // TMA descriptor cannot be encoded.
@@ -37,12 +49,13 @@ int launch_top_t(const Dims& D, const float* s, int* anchors, DevStatus* stt, cu
 int launch_check_anchors(const Dims& D, int* anchors, DevStatus* stt, cudaStream_t st);
 
 // ---- reference attention, assignment, merge (Sec. 3.4) ------------------
-// l = scale Q K^T into `L` (tcgen05); z, m (row max / mass); Y = softmax(l) V;
-// column statistics log phi, M_j and 1/||e^{l_:j - M_j}||.  -1 when a TMA
-// descriptor cannot be encoded.
-int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const bf16* K, const bf16* V,
-                               float* L, float* z, float* m, float* invm, float* split, float* Y,
-                               float* logphi, float* colM, float* colInvN, DevStatus* stt, cudaStream_t st);
+// l = scale Q K^T into `L` (tcgen05); z, m (row max / mass); Y = softmax(l) V
+// (tcgen05, split-3 probabilities against VT); column statistics log phi,
+// M_j and 1/||e^{l_:j - M_j}||.  -1 when a TMA descriptor cannot be encoded.
+int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const bf16* K, const bf16* VT,
+                               float* L, float* z, float* m, float* invm, bf16* p_h, bf16* p_m, bf16* p_l,
+                               float* Y, float* logphi, float* colM, float* colInvN, DevStatus* stt,
+                               cudaStream_t st);
 int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* K, float* L, DevStatus* stt,
                          cudaStream_t st);
 // Assignment on tcgen05: transposed split-bf16 profiles, anchor rows, argmax GEMM.
@@ -55,7 +68,7 @@ int launch_merge(const Dims& D, float lambda_m, const bf16* K, const int* anchor
 
 // ---- fits (App. A.9) -----------------------------------------------------
 struct FitBufs {
-  float *LC, *Phi, *Gram, *Linv, *rhs, *wsol, *R, *Z, *split;
+  float *LC, *Phi, *Gram, *Linv, *rhs, *wsol, *R, *Z;
   bf16 *PT_hi, *PT_lo, *YT_hi, *YT_lo;  // transposed split-bf16 operands ([t][ldn], [d][ldn])
 };
 // Returns launches, or -1 when a TMA descriptor cannot be encoded.

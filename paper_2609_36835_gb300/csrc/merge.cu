@@ -61,21 +61,19 @@ __global__ void __launch_bounds__(256) col_stats_kernel(const float* L, float* l
   colInvN[o] = 1.0f / sqrtf(S2);
 }
 
-int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const bf16* K, const bf16* V,
-                               float* L, float* z, float* m, float* invm, float* split, float* Y,
-                               float* logphi, float* colM, float* colInvN, DevStatus* stt, cudaStream_t st) {
-  const long long nd = (long long)D.n * D.d, Td = (long long)D.T * D.d, nT = (long long)D.n * D.T;
+int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const bf16* K, const bf16* VT,
+                               float* L, float* z, float* m, float* invm, bf16* p_h, bf16* p_m, bf16* p_l,
+                               float* Y, float* logphi, float* colM, float* colInvN, DevStatus* stt,
+                               cudaStream_t st) {
   // l = scale * Q K^T on the tensor cores
   if (launch_ref_logits_tc(D, scale, Q, K, L, stt, st) < 0) return -1;
   // z_i = max_j l_ij (z^fit of Eq. mass_fit), m_i = sum_j e^{l_ij - z_i} = (Phi_K 1)_i
   launch_row_stats(D.H, D.n, D.T, L, z, invm, m, st);
   // Y = softmax(l) V
-  RowKExp P{{L, nT, D.T}, z, invm, D.n, 1.f};
-  launch_gemm(P, ColK<bf16>{V, Td, D.d}, EpiStore{split, nd, (long long)D.H * nd, D.d, 1.f, false}, D.H, D.n,
-              D.d, D.T, kSplitK, st);
-  launch_split_reduce(D.H, D.n, D.d, kSplitK, split, Y, st);
+  const int r = launch_probs_v_tc(D, L, z, invm, p_h, p_m, p_l, VT, Y, stt, st);
+  if (r < 0) return -1;
   col_stats_kernel<<<dim3(cdiv(D.T, 32), D.H), 256, 0, st>>>(L, logphi, colM, colInvN, D.n, D.T);
-  return 5;
+  return 3 + r;
 }
 
 // Caller-supplied assignment (copied into the workspace): values in [0, t)

@@ -15,7 +15,11 @@
 //              issues hi*hi + hi*lo + lo*hi: an fp32-accurate product on the
 //              bf16 tensor pipe (the dropped lo*lo term is below 2^-16 relative);
 //   kConcat -- the operands are concatenated along K: K < K1 comes from
-//              (mA, mB), K >= K1 from (mA2, mB2) (K1 a multiple of 64).
+//              (mA, mB), K >= K1 from (mA2, mB2) (K1 a multiple of 64);
+//   kSplit3A -- A is a triple (h, m, l) of bf16 tensors with x = h + m + l to
+//              within 2^-24 relative (mA, mA2, mA3) and B is exact bf16 (mB):
+//              every K step issues h*B + m*B + l*B, fp32-grade products for an
+//              fp32 operand against a bf16 input.
 //
 // K is consumed in chunks of `chunk_k` (a multiple of 64): each chunk gets a
 // fresh accumulator and the epilogue sees every chunk separately, which lets
@@ -33,15 +37,16 @@
 
 namespace arckv {
 
-enum TcMode { kPlain = 0, kSplit = 1, kConcat = 2 };
+enum TcMode { kPlain = 0, kSplit = 1, kConcat = 2, kSplit3A = 3 };
 
 template <int BN, int MODE>
 struct TcCfg {
   static constexpr bool SPLIT = MODE == kSplit;
   static constexpr int TILE_A = 128 * 128;  // bytes: 128 rows x 64 bf16
   static constexpr int TILE_B = BN * 128;
-  static constexpr int STAGE = (TILE_A + TILE_B) * (SPLIT ? 2 : 1);
-  static constexpr int STAGES = SPLIT ? 3 : 4;
+  static constexpr int STAGE = MODE == kSplit ? 2 * (TILE_A + TILE_B)
+                               : MODE == kSplit3A ? 3 * TILE_A + TILE_B : TILE_A + TILE_B;
+  static constexpr int STAGES = (MODE == kSplit || MODE == kSplit3A) ? 3 : 4;
   static constexpr int SMEM = STAGES * STAGE + 1024;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
 };
@@ -49,8 +54,9 @@ struct TcCfg {
 template <int BN, int MODE, class Epi>
 __global__ void __launch_bounds__(192, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
-                   const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mB2, Epi epi, int M,
-                   int N, int K, int chunk_k, int K1, DevStatus* stt) {
+                   const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mB2,
+                   const __grid_constant__ CUtensorMap mA3, Epi epi, int M, int N, int K, int chunk_k, int K1,
+                   DevStatus* stt) {
   using C = TcCfg<BN, MODE>;
   constexpr bool SPLIT = C::SPLIT;
   constexpr int STAGES = C::STAGES;
@@ -90,9 +96,13 @@ __global__ void __launch_bounds__(192, 1)
     if (lane == 0) {
       tc::tma_prefetch(&mA);
       tc::tma_prefetch(&mB);
-      if (MODE != kPlain) {
+      if (MODE == kSplit || MODE == kConcat) {
         tc::tma_prefetch(&mA2);
         tc::tma_prefetch(&mB2);
+      }
+      if (MODE == kSplit3A) {
+        tc::tma_prefetch(&mA2);
+        tc::tma_prefetch(&mA3);
       }
       int issued = 0;
       for (int kb = 0; kb < nk; ++kb) {
@@ -110,6 +120,10 @@ __global__ void __launch_bounds__(192, 1)
         if (SPLIT) {
           tc::tma_load_3d(st + C::TILE_A + C::TILE_B, &mA2, kb * 64, m0, b, &full[s]);
           tc::tma_load_3d(st + 2 * C::TILE_A + C::TILE_B, &mB2, kb * 64, n0, b, &full[s]);
+        }
+        if (MODE == kSplit3A) {
+          tc::tma_load_3d(st + C::TILE_A + C::TILE_B, &mA2, kb * 64, m0, b, &full[s]);
+          tc::tma_load_3d(st + 2 * C::TILE_A + C::TILE_B, &mA3, kb * 64, m0, b, &full[s]);
         }
         issued = kb + 1;
       }
@@ -145,6 +159,12 @@ __global__ void __launch_bounds__(192, 1)
               const uint64_t bd2 = tc::sdesc_k128(bb + C::TILE_A + C::TILE_B + ks * 32);
               tc::mma_f16(d, ad, bd2, idesc, 1u);
               tc::mma_f16(d, ad2, bd, idesc, 1u);
+            }
+            if (MODE == kSplit3A) {
+              const uint64_t am = tc::sdesc_k128(a + C::TILE_A + C::TILE_B + ks * 32);
+              const uint64_t al = tc::sdesc_k128(a + 2 * C::TILE_A + C::TILE_B + ks * 32);
+              tc::mma_f16(d, am, bd, idesc, 1u);
+              tc::mma_f16(d, al, bd, idesc, 1u);
             }
           }
           tc::mma_commit(&empty[s]);
@@ -193,13 +213,13 @@ __global__ void __launch_bounds__(192, 1)
 template <int BN, int MODE, class Epi>
 inline cudaError_t launch_tc_gemm(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mA2,
                                   const CUtensorMap& mB2, const Epi& epi, int H, int M, int N, int K, int chunk_k,
-                                  DevStatus* stt, cudaStream_t st, int K1 = 0) {
+                                  DevStatus* stt, cudaStream_t st, int K1 = 0, const CUtensorMap* mA3 = nullptr) {
   using C = TcCfg<BN, MODE>;
   auto kern = tc_gemm_kernel<BN, MODE, Epi>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
   dim3 grid(cdiv(N, BN), cdiv(M, 128), H);
-  kern<<<grid, 192, C::SMEM, st>>>(mA, mB, mA2, mB2, epi, M, N, K, chunk_k, K1, stt);
+  kern<<<grid, 192, C::SMEM, st>>>(mA, mB, mA2, mB2, mA3 ? *mA3 : mA, epi, M, N, K, chunk_k, K1, stt);
   return cudaGetLastError();
 }
 

@@ -43,8 +43,8 @@ def _cfg(**kw):
 
 def test_workspace_bytes_sizes_and_rejections(lib):
     ws = pk.workspace_bytes(_cfg())
-    # the n x T spill, k_bar and the t x t Gram dominate
-    assert 0.6e9 < ws < 1.2e9
+    # the n x T fp32 spill, its split-3 bf16 probabilities, k_bar and the t x t Gram dominate
+    assert 0.8e9 < ws < 2.0e9
     assert pk.workspace_bytes(_cfg(t=9000)) == 0           # t > T
     assert pk.workspace_bytes(_cfg(t=0)) == 0
     assert pk.workspace_bytes(_cfg(d=64)) == 0             # unsupported head dim
