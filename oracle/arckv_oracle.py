@@ -164,13 +164,18 @@ def response_profiles_literal(l: np.ndarray):
     return E / np.linalg.norm(E, axis=0, keepdims=True)
 
 
-def assign_to_anchors(u: np.ndarray, S: np.ndarray) -> np.ndarray:
+def assign_to_anchors(u: np.ndarray, S: np.ndarray, rows: int = 8192) -> np.ndarray:
     """Eq. (anchor_assignment): kappa(s_r) = r; kappa(j) = argmax_r u_j . u_{s_r}
-    for j not in S (ties -> smallest r)."""
-    sim = u.T @ u[:, S]                       # [T, t]
-    kappa = np.argmax(sim, axis=1)            # first maximum = smallest r
+    for j not in S (ties -> smallest r).  Each key's argmax is independent, so
+    the T x t similarity table is formed ``rows`` keys at a time."""
+    T = u.shape[1]
+    uS = u[:, S]
+    kappa = np.empty(T, dtype=np.int64)
+    for j0 in range(0, T, rows):
+        sim = u[:, j0:j0 + rows].T @ uS           # [rows, t]
+        kappa[j0:j0 + rows] = np.argmax(sim, axis=1)  # first maximum = smallest r
     kappa[S] = np.arange(S.shape[0])
-    return kappa.astype(np.int64)
+    return kappa
 
 
 def log_mass_weights(l: np.ndarray) -> np.ndarray:

@@ -68,6 +68,32 @@ def assignment_valid(kappa_gpu: np.ndarray, sim: np.ndarray, S: np.ndarray, tau:
     return (n_dec_mis == 0 and anchors_ok and worst <= tau), n_dec_mis, n_tie, worst
 
 
+def assignment_valid_profiles(kappa_gpu: np.ndarray, u: np.ndarray, S: np.ndarray, tau: float, rows: int = 8192):
+    """assignment_valid over the profile matrix u [n, T], forming the
+    similarity table a block of keys at a time (for long caches)."""
+    T = u.shape[1]
+    uS = u[:, S]
+    is_anchor = np.zeros(T, bool)
+    is_anchor[S] = True
+    n_mis = n_tie = 0
+    worst = 0.0
+    for j0 in range(0, T, rows):
+        sim = u[:, j0:j0 + rows].T @ uS
+        kg = kappa_gpu[j0:j0 + rows]
+        best = sim.max(axis=1)
+        srt = np.sort(sim, axis=1)
+        gap = srt[:, -1] - (srt[:, -2] if sim.shape[1] > 1 else -np.inf)
+        anc = is_anchor[j0:j0 + rows]
+        got = sim[np.arange(sim.shape[0]), kg]
+        dec = (~anc) & (gap > tau)
+        kref = np.argmax(sim, axis=1)
+        n_mis += int(np.sum(dec & (kg != kref)))
+        n_tie += int(np.sum((~anc) & (~dec) & (kg != kref)))
+        worst = max(worst, float(np.max(np.where(anc, 0.0, best - got))))
+    anchors_ok = bool(np.all(kappa_gpu[S] == np.arange(len(S))))
+    return (n_mis == 0 and anchors_ok and worst <= tau), n_mis, n_tie, worst
+
+
 def beta_errors(beta_gpu: np.ndarray, beta: np.ndarray, w_star: np.ndarray):
     """(relative l2 error on the supported entries, ok flag for the rest)."""
     wmax = float(np.max(w_star))

@@ -16,7 +16,7 @@ inline size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 struct Layout {
   size_t status, kbar_hi, kbar_lo, vq, qpp, q_h, q_m, q_l, av, VT, p_h, p_m, p_l, cctx, qbar_hi, qbar_lo, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
       colM, colInvN, Ut_hi, Ut_lo, S_hi, S_lo, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z,
-      YT_hi, YT_lo, total;
+      YT_hi, YT_lo, G64, L64, B64, Z64, X64, total;
 };
 
 Dims dims_of(const arckv_config& c) {
@@ -97,7 +97,7 @@ Layout plan(const arckv_config& c) {
   L.perm = take(H * T * 4);
   L.goff = take(H * (t + 1) * 4);
   L.cursor = take(H * t * 4);
-  L.LC = take(H * n * t * f);
+  L.LC = take(H * n * (t > 128 ? t : 128) * f);   // also holds the n x d dual solution when t > n
   L.Phi = take(H * n * t * f);
   L.Gram = take(H * t * t * f);
   L.Linv = take(H * nblk * kCholNB * kCholNB * f);
@@ -107,6 +107,13 @@ Layout plan(const arckv_config& c) {
   L.Z = take(H * t * 128 * f);
   L.YT_hi = take(H * 128 * ldn * 2);
   L.YT_lo = take(H * 128 * ldn * 2);
+  // fp64 dual-form scratch, only when t > n
+  const size_t nd64 = t > n ? n : 0, nbn = (nd64 + kCholNB - 1) / kCholNB;
+  L.G64 = take(H * nd64 * nd64 * 8);
+  L.L64 = take(H * nbn * kCholNB * kCholNB * 8);
+  L.B64 = take(H * nd64 * 128 * 8);
+  L.Z64 = take(H * nd64 * 128 * 8);
+  L.X64 = take(H * nd64 * 128 * 8);
   L.total = o;
   return L;
 }
@@ -241,7 +248,9 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
                      C_k, st);
   mark(5);
   FitBufs B{F(L.LC),  F(L.Phi), F(L.Gram), F(L.Linv), F(L.rhs), F(L.wsol), F(L.R), F(L.Z),
-            (bf16*)(w + L.S_hi), (bf16*)(w + L.S_lo), (bf16*)(w + L.YT_hi), (bf16*)(w + L.YT_lo)};
+            (bf16*)(w + L.S_hi), (bf16*)(w + L.S_lo), (bf16*)(w + L.YT_hi), (bf16*)(w + L.YT_lo),
+            (double*)(w + L.G64), (double*)(w + L.L64), (double*)(w + L.B64), (double*)(w + L.Z64),
+            (double*)(w + L.X64)};
   const int nlf = launch_fits(D, scale, cfg->ridge_w, cfg->ridge_v, cfg->eps_w, cfg->b_min, cfg->b_max, Qb, C_k,
                               F(L.z), F(L.m), F(L.Y), B, beta, C_v, stt, st);
   if (nlf < 0) return ARCKV_ERR_CUDA;

@@ -51,11 +51,21 @@ __global__ void mass_rhs_kernel(const float* Phi, const float* m, float* rhs, in
 //           factors it at once, overlapping the serial factorisation with the
 //           other CTAs' updates;
 // then block back substitution X_k = Linv_kk^T (Linv_kk B_k + Z_k),
-// Z_i -= L_ki^T X_k (i < k).  lam = ridge * trace(Gram) / t is added to the
-// diagonal as each diagonal block is factored.
+// Z_i -= L_ki^T X_k (i < k).  lam = ridge * trace(Gram) / tdiv is added to the
+// diagonal as each diagonal block is factored (tdiv = t, or the primal size
+// when the dual system is solved).
 constexpr int kCL = 8;
 constexpr int kCT = 512;
 constexpr int kTileF = NB * (NB + 1);
+
+__device__ __forceinline__ float fma_r(float a, float b, float c) { return fmaf(a, b, c); }
+__device__ __forceinline__ double fma_r(double a, double b, double c) { return fma(a, b, c); }
+template <typename R>
+__device__ __forceinline__ R warp_sum_r(R v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
 
 __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
@@ -68,18 +78,20 @@ __device__ __forceinline__ unsigned cluster_rank() {
 
 // S[r][c] = G[(r0 + r) * ld + c0 + c] (or its transpose with `trans`), zero outside
 // rows < rmax, cols < cmax of the source block.
-__device__ __forceinline__ void ld_tile(float (*S)[NB + 1], const float* G, long long ld, int r0, int c0, int rmax,
-                                        int cmax, bool trans) {
+template <typename R>
+__device__ __forceinline__ void ld_tile(R (*S)[NB + 1], const R* G, long long ld, int r0, int c0, int rmax, int cmax,
+                                        bool trans) {
   for (int e = threadIdx.x; e < NB * NB; e += kCT) {
     const int r = e / NB, c = e % NB;
-    const float v = (r < rmax && c < cmax) ? __ldcg(G + (long long)(r0 + r) * ld + c0 + c) : 0.f;
+    const R v = (r < rmax && c < cmax) ? __ldcg(G + (long long)(r0 + r) * ld + c0 + c) : R(0);
     if (trans) S[c][r] = v;
     else S[r][c] = v;
   }
 }
 
 // acc[p][q] = sum_l X[ry+p][l] Y[l][cx+q], ry = (tid >> 4) * 2, cx = (tid & 15) * 4.
-__device__ __forceinline__ void mm64(const float (*X)[NB + 1], const float (*Y)[NB + 1], float (&acc)[2][4]) {
+template <typename R>
+__device__ __forceinline__ void mm64(const R (*X)[NB + 1], const R (*Y)[NB + 1], R (&acc)[2][4]) {
   const int ry = (threadIdx.x >> 4) * 2, cx = (threadIdx.x & 15) * 4;
 #pragma unroll
   for (int p = 0; p < 2; ++p)
@@ -88,55 +100,55 @@ __device__ __forceinline__ void mm64(const float (*X)[NB + 1], const float (*Y)[
 #pragma unroll 8
   for (int l = 0; l < NB; ++l) {
     // rows of the [64][65] tiles are 260 bytes apart: scalar loads only
-    const float a0 = X[ry][l], a1 = X[ry + 1][l];
-    const float c0 = Y[l][cx], c1 = Y[l][cx + 1], c2 = Y[l][cx + 2], c3 = Y[l][cx + 3];
-    acc[0][0] = fmaf(a0, c0, acc[0][0]); acc[0][1] = fmaf(a0, c1, acc[0][1]);
-    acc[0][2] = fmaf(a0, c2, acc[0][2]); acc[0][3] = fmaf(a0, c3, acc[0][3]);
-    acc[1][0] = fmaf(a1, c0, acc[1][0]); acc[1][1] = fmaf(a1, c1, acc[1][1]);
-    acc[1][2] = fmaf(a1, c2, acc[1][2]); acc[1][3] = fmaf(a1, c3, acc[1][3]);
+    const R a0 = X[ry][l], a1 = X[ry + 1][l];
+    const R c0 = Y[l][cx], c1 = Y[l][cx + 1], c2 = Y[l][cx + 2], c3 = Y[l][cx + 3];
+    acc[0][0] = fma_r(a0, c0, acc[0][0]); acc[0][1] = fma_r(a0, c1, acc[0][1]);
+    acc[0][2] = fma_r(a0, c2, acc[0][2]); acc[0][3] = fma_r(a0, c3, acc[0][3]);
+    acc[1][0] = fma_r(a1, c0, acc[1][0]); acc[1][1] = fma_r(a1, c1, acc[1][1]);
+    acc[1][2] = fma_r(a1, c2, acc[1][2]); acc[1][3] = fma_r(a1, c3, acc[1][3]);
   }
 }
 
 // Factor diagonal block k (lower part of A_kk + lam I) in shared memory; write
 // L_kk into A and its inverse into Linv[k].  8 threads per row.
-__device__ void factor_diag(float* Ab, float* Lb, int t, int k, float lam, float (*L)[NB + 1],
-                            float (*Li)[NB + 1], int* bad) {
+template <typename R>
+__device__ void factor_diag(R* Ab, R* Lb, int t, int k, R lam, R (*L)[NB + 1], R (*Li)[NB + 1], int* bad) {
   const int tid = threadIdx.x, k0 = k * NB, kb = min(NB, t - k0);
   for (int e = tid; e < NB * NB; e += kCT) {
     const int r = e / NB, c = e % NB;
-    L[r][c] = (r < kb && c <= r) ? __ldcg(Ab + (long long)(k0 + r) * t + k0 + c) + (r == c ? lam : 0.f)
-                                 : (r == c ? 1.f : 0.f);
-    Li[r][c] = 0.f;
+    L[r][c] = (r < kb && c <= r) ? __ldcg(Ab + (long long)(k0 + r) * t + k0 + c) + (r == c ? lam : R(0))
+                                 : (r == c ? R(1) : R(0));
+    Li[r][c] = R(0);
   }
   __syncthreads();
   const int r = tid >> 3, p = tid & 7;
   for (int c = 0; c < NB; ++c) {
-    float v = 0.f;
+    R v = R(0);
     if (r >= c)
-      for (int q = p; q < c; q += 8) v = fmaf(L[r][q], L[c][q], v);
+      for (int q = p; q < c; q += 8) v = fma_r(L[r][q], L[c][q], v);
     v += __shfl_xor_sync(0xffffffffu, v, 1);
     v += __shfl_xor_sync(0xffffffffu, v, 2);
     v += __shfl_xor_sync(0xffffffffu, v, 4);
-    v = (r >= c) ? L[r][c] - v : 0.f;
+    v = (r >= c) ? L[r][c] - v : R(0);
     if (r == c && p == 0) {
-      if (!(v > 0.f) || !isfinite(v)) { *bad = 1; v = 1.f; }
-      L[c][c] = sqrtf(v);
+      if (!(v > R(0)) || !isfinite(v)) { *bad = 1; v = R(1); }
+      L[c][c] = sqrt(v);
     }
     __syncthreads();
     if (r > c && p == 0) L[r][c] = v / L[c][c];
     __syncthreads();
   }
   for (int i = 0; i < NB; ++i) {
-    float v = 0.f;
+    R v = R(0);
     if (r < i)
-      for (int l = r + p; l < i; l += 8) v = fmaf(L[i][l], Li[l][r], v);
+      for (int l = r + p; l < i; l += 8) v = fma_r(L[i][l], Li[l][r], v);
     v += __shfl_xor_sync(0xffffffffu, v, 1);
     v += __shfl_xor_sync(0xffffffffu, v, 2);
     v += __shfl_xor_sync(0xffffffffu, v, 4);
-    if (r <= i && p == 0) Li[i][r] = ((i == r ? 1.f : 0.f) - v) / L[i][i];
+    if (r <= i && p == 0) Li[i][r] = ((i == r ? R(1) : R(0)) - v) / L[i][i];
     __syncthreads();
   }
-  float* Lo = Lb + (long long)k * NB * NB;
+  R* Lo = Lb + (long long)k * NB * NB;
   for (int e = tid; e < NB * NB; e += kCT) {
     const int rr = e / NB, cc = e % NB;
     Lo[e] = Li[rr][cc];
@@ -145,45 +157,47 @@ __device__ void factor_diag(float* Ab, float* Lb, int t, int k, float lam, float
   __syncthreads();
 }
 
+template <typename R>
 __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
-    chol_cluster_kernel(float* A, float* Linv, float* B, float* Z, float* X, int t, int nrhs, int ldb,
-                        long long bbs, float ridge, DevStatus* stt) {
-  extern __shared__ float sm[];
-  float (*S1)[NB + 1] = (float (*)[NB + 1])sm;
-  float (*S2)[NB + 1] = (float (*)[NB + 1])(sm + kTileF);
-  float (*S3)[NB + 1] = (float (*)[NB + 1])(sm + 2 * kTileF);
-  __shared__ float red[kCT / 32];
+    chol_cluster_kernel(R* A, R* Linv, R* B, R* Z, R* X, int t, int nrhs, int ldb, long long bbs, R ridge, R tdiv,
+                        DevStatus* stt) {
+  extern __shared__ __align__(16) unsigned char smraw[];
+  R* sm = (R*)smraw;
+  R (*S1)[NB + 1] = (R (*)[NB + 1])sm;
+  R (*S2)[NB + 1] = (R (*)[NB + 1])(sm + kTileF);
+  R (*S3)[NB + 1] = (R (*)[NB + 1])(sm + 2 * kTileF);
+  __shared__ R red[kCT / 32];
   __shared__ int bad;
   const int head = blockIdx.x / kCL;
   const int rank = (int)cluster_rank();
   const int tid = threadIdx.x;
   const int nblk = (t + NB - 1) / NB, nct = (nrhs + NB - 1) / NB;
-  float* Ab = A + (long long)head * t * t;
-  float* Lb = Linv + (long long)head * nblk * NB * NB;
-  float* Bb = B + (long long)head * bbs;
-  float* Zb = Z + (long long)head * bbs;
-  float* Xb = X + (long long)head * bbs;
+  R* Ab = A + (long long)head * t * t;
+  R* Lb = Linv + (long long)head * nblk * NB * NB;
+  R* Bb = B + (long long)head * bbs;
+  R* Zb = Z + (long long)head * bbs;
+  R* Xb = X + (long long)head * bbs;
   const int ry = (tid >> 4) * 2, cx = (tid & 15) * 4;
-  float acc[2][4];
+  R acc[2][4];
 
   // lam = ridge * trace / t (every CTA forms it; the trace precedes all writes)
-  float tr = 0.f;
+  R tr = R(0);
   for (int r = tid; r < t; r += kCT) tr += __ldcg(Ab + (long long)r * t + r);
-  tr = warp_sum(tr);
+  tr = warp_sum_r(tr);
   if ((tid & 31) == 0) red[tid >> 5] = tr;
   if (tid == 0) bad = 0;
   __syncthreads();
   if (tid < 32) {
-    float v = tid < kCT / 32 ? red[tid] : 0.f;
-    v = warp_sum(v);
+    R v = tid < kCT / 32 ? red[tid] : R(0);
+    v = warp_sum_r(v);
     if (tid == 0) red[0] = v;
   }
   __syncthreads();
-  const float trace = red[0];
-  const float lam = ridge * trace / (float)t;
+  const R trace = red[0];
+  const R lam = ridge * trace / tdiv;
   if (rank == 0 && tid == 0 && !isfinite(trace)) set_status(stt, ARCKV_ERR_NONFINITE);
   // zero Z (rows split over the cluster) and factor the first diagonal block
-  for (long long e = (long long)rank * kCT + tid; e < (long long)t * ldb; e += (long long)kCL * kCT) Zb[e] = 0.f;
+  for (long long e = (long long)rank * kCT + tid; e < (long long)t * ldb; e += (long long)kCL * kCT) Zb[e] = R(0);
   cluster_sync_all();   // everyone has read the unmodified diagonal for the trace
   if (rank == 0) factor_diag(Ab, Lb, t, 0, lam, S1, S2, &bad);
   cluster_sync_all();
@@ -231,7 +245,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
 #pragma unroll
             for (int q = 0; q < 4; ++q)
               if (ry + p < rb && cx + q < cb) {
-                float* a = Ab + (long long)(i0 + ry + p) * t + j0 + cx + q;
+                R* a = Ab + (long long)(i0 + ry + p) * t + j0 + cx + q;
                 *a = __ldcg(a) - acc[p][q];
               }
           __syncthreads();
@@ -256,7 +270,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
 #pragma unroll
             for (int q = 0; q < 4; ++q)
               if (ry + p < rb && cx + q < nc) {
-                float* bp = Bb + (long long)(i0 + ry + p) * ldb + c0 + cx + q;
+                R* bp = Bb + (long long)(i0 + ry + p) * ldb + c0 + cx + q;
                 *bp = __ldcg(bp) - acc[p][q];
               }
           __syncthreads();
@@ -280,7 +294,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
 #pragma unroll
         for (int q = 0; q < 4; ++q)
           S3[ry + p][cx + q] = acc[p][q] + ((ry + p < kb && cx + q < nc)
-                                                ? __ldcg(Zb + (long long)(k0 + ry + p) * ldb + c0 + cx + q) : 0.f);
+                                                ? __ldcg(Zb + (long long)(k0 + ry + p) * ldb + c0 + cx + q) : R(0));
       ld_tile(S2, Lb + (long long)k * NB * NB, NB, 0, 0, NB, NB, true);      // S2[r][l] = Linv[l][r]
       __syncthreads();
       mm64(S2, S3, acc);                                                    // X_k = Linv^T (Y_k + Z_k)
@@ -305,7 +319,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
 #pragma unroll
           for (int q = 0; q < 4; ++q)
             if (cx + q < nc) {
-              float* zp = Zb + (long long)(i0 + ry + p) * ldb + c0 + cx + q;
+              R* zp = Zb + (long long)(i0 + ry + p) * ldb + c0 + cx + q;
               *zp = __ldcg(zp) - acc[p][q];
             }
       }
@@ -316,11 +330,13 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
   if (tid == 0 && bad) set_status(stt, ARCKV_ERR_NOT_SPD);
 }
 
-static int cholesky_solve(int H, int t, float* Gram, float* Linv, float* B, float* Z, float* X, int ldb,
-                          int nrhs, long long bbs, float ridge, DevStatus* stt, cudaStream_t st) {
-  const int smem = 3 * kTileF * (int)sizeof(float);
-  cudaFuncSetAttribute(chol_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  chol_cluster_kernel<<<kCL * H, kCT, smem, st>>>(Gram, Linv, B, Z, X, t, nrhs, ldb, bbs, ridge, stt);
+template <typename R>
+static int cholesky_solve(int H, int t, R* Gram, R* Linv, R* B, R* Z, R* X, int ldb, int nrhs, long long bbs,
+                          float ridge, DevStatus* stt, cudaStream_t st, int tdiv = 0) {
+  const int smem = 3 * kTileF * (int)sizeof(R);
+  cudaFuncSetAttribute(chol_cluster_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  chol_cluster_kernel<R><<<kCL * H, kCT, smem, st>>>(Gram, Linv, B, Z, X, t, nrhs, ldb, bbs, (R)ridge,
+                                                     (R)(tdiv > 0 ? tdiv : t), stt);
   return 1;
 }
 
@@ -388,6 +404,126 @@ static int gram_tc(int H, int M, int N, int ldn, const bf16* Xh, const bf16* Xl,
   return 1;
 }
 
+// C[b] = X X^T in fp64 (X fp32 [rows][K]); 64 x 64 lower tiles, mirrored.
+__global__ void __launch_bounds__(256) syrk64_kernel(const float* X, double* C, int rows, int K) {
+  const int b = blockIdx.z, i0 = blockIdx.y * 64, j0 = blockIdx.x * 64;
+  if (j0 > i0) return;
+  const float* Xb = X + (long long)b * rows * K;
+  double* Cb = C + (long long)b * rows * rows;
+  __shared__ double As[16][65], Bs[16][65];
+  const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
+  double acc[4][4];
+#pragma unroll
+  for (int p = 0; p < 4; ++p)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) acc[p][q] = 0.0;
+  for (int k0 = 0; k0 < K; k0 += 16) {
+    for (int e = threadIdx.x; e < 64 * 16; e += 256) {
+      const int r = e >> 4, kk = e & 15, k = k0 + kk;
+      As[kk][r] = (i0 + r < rows && k < K) ? (double)Xb[(long long)(i0 + r) * K + k] : 0.0;
+      Bs[kk][r] = (j0 + r < rows && k < K) ? (double)Xb[(long long)(j0 + r) * K + k] : 0.0;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < 16; ++kk) {
+      double a[4], c[4];
+#pragma unroll
+      for (int p = 0; p < 4; ++p) { a[p] = As[kk][ty * 4 + p]; c[p] = Bs[kk][tx * 4 + p]; }
+#pragma unroll
+      for (int p = 0; p < 4; ++p)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) acc[p][q] = fma(a[p], c[q], acc[p][q]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int p = 0; p < 4; ++p)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = i0 + ty * 4 + p, j = j0 + tx * 4 + q;
+      if (i < rows && j < rows) {
+        Cb[(long long)i * rows + j] = acc[p][q];
+        Cb[(long long)j * rows + i] = acc[p][q];
+      }
+    }
+}
+
+__global__ void widen_kernel(const float* x, double* y, long long count) {
+  for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < count;
+       k += (long long)gridDim.x * blockDim.x)
+    y[k] = (double)x[k];
+}
+
+// out[b][r][c] = sum_i X[b][i][r] Y[b][i][c] accumulated in fp64 (X fp32 [n][t],
+// Y fp64 [n][ncol], out fp32 [t][ncol]); 64 x 32 output tiles.
+__global__ void __launch_bounds__(256) xty64_kernel(const float* X, const double* Y, float* out, int n, int t,
+                                                    int ncol) {
+  const int b = blockIdx.z, r0 = blockIdx.x * 64, c0 = blockIdx.y * 32;
+  const float* Xb = X + (long long)b * n * t;
+  const double* Yb = Y + (long long)b * n * ncol;
+  __shared__ double Xs[16][64], Ys[16][33];
+  const int tr = threadIdx.x & 63, tc = threadIdx.x >> 6;   // 64 rows x 4 column groups of 8
+  double acc[8];
+#pragma unroll
+  for (int q = 0; q < 8; ++q) acc[q] = 0.0;
+  for (int i0 = 0; i0 < n; i0 += 16) {
+    for (int e = threadIdx.x; e < 16 * 64; e += 256) {
+      const int ii = e >> 6, r = e & 63;
+      Xs[ii][r] = (i0 + ii < n && r0 + r < t) ? (double)Xb[(long long)(i0 + ii) * t + r0 + r] : 0.0;
+    }
+    for (int e = threadIdx.x; e < 16 * 32; e += 256) {
+      const int ii = e >> 5, c = e & 31;
+      Ys[ii][c] = (i0 + ii < n && c0 + c < ncol) ? Yb[(long long)(i0 + ii) * ncol + c0 + c] : 0.0;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int ii = 0; ii < 16; ++ii) {
+      const double xv = Xs[ii][tr];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) acc[q] = fma(xv, Ys[ii][tc * 8 + q], acc[q]);
+    }
+    __syncthreads();
+  }
+  const int r = r0 + tr;
+  if (r >= t) return;
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    const int c = c0 + tc * 8 + q;
+    if (c < ncol) out[((long long)b * t + r) * ncol + c] = (float)acc[q];
+  }
+}
+
+// Dual (push-through) form of both ridge fits for t > n, where the primal
+// t x t normal matrices have rank <= n:
+//   (Phi^T Phi + lam I) w = Phi^T m   <=>   w = Phi^T a,  (Phi Phi^T + lam I) a = m
+//   (P^T P + lam I) C_v = P^T Y       <=>   C_v = P^T A,  (P P^T + lam I) A = Y
+// with the same lam = ridge * trace / t (trace(Phi^T Phi) = trace(Phi Phi^T)),
+// so the solutions equal the primal ones; the systems are n x n.  These
+// systems reach condition numbers ~1e8 on 128K caches (lam relative to t
+// diagonal entries, n of them carrying the mass), so the n x n Grams, the
+// solves and the back-projections run in fp64 (Phi and P^ stay fp32).
+static int fits_dual(const Dims& D, float ridge_w, float ridge_v, float eps_w, float b_min, float b_max,
+                     const float* m, const float* Y, const FitBufs& B, float* beta, float* C_v, DevStatus* stt,
+                     cudaStream_t st) {
+  const long long nt = (long long)D.n * D.t, nd = (long long)D.n * D.d;
+  const dim3 sgrid(cdiv(D.n, 64), cdiv(D.n, 64), D.H);
+  // beta system
+  syrk64_kernel<<<sgrid, 256, 0, st>>>(B.Phi, B.G64, D.n, D.t);
+  widen_kernel<<<cdiv((long long)D.H * D.n, 256), 256, 0, st>>>(m, B.B64, (long long)D.H * D.n);
+  cholesky_solve<double>(D.H, D.n, B.G64, B.L64, B.B64, B.Z64, B.X64, 1, 1, D.n, ridge_w, stt, st, D.t);
+  xty64_kernel<<<dim3(cdiv(D.t, 64), 1, D.H), 256, 0, st>>>(B.Phi, B.X64, B.rhs, D.n, D.t, 1);   // w = Phi^T a
+  const long long ht = (long long)D.H * D.t;
+  beta_kernel<<<cdiv(ht, 256), 256, 0, st>>>(B.rhs, beta, ht, eps_w, b_min, b_max);
+  // value system
+  softmax_bias_kernel<<<dim3(cdiv(D.n, 8), D.H), 256, 0, st>>>(B.LC, beta, B.Phi, D.n, D.t);
+  syrk64_kernel<<<sgrid, 256, 0, st>>>(B.Phi, B.G64, D.n, D.t);
+  widen_kernel<<<cdiv((long long)D.H * nd, 256), 256, 0, st>>>(Y, B.B64, (long long)D.H * nd);
+  cholesky_solve<double>(D.H, D.n, B.G64, B.L64, B.B64, B.Z64, B.X64, D.d, D.d, nd, ridge_v, stt, st, D.t);
+  xty64_kernel<<<dim3(cdiv(D.t, 64), cdiv(D.d, 32), D.H), 256, 0, st>>>(B.Phi, B.X64, C_v, D.n, D.t, D.d);
+  (void)nt;
+  return 12;
+}
+
 int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float eps_w, float b_min,
                 float b_max, const bf16* Q, const float* C_k, const float* z, const float* m,
                 const float* Y, const FitBufs& B, float* beta, float* C_v, DevStatus* stt, cudaStream_t st) {
@@ -400,6 +536,7 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
   const long long cnt = (long long)D.H * nt;
   phi_kernel<<<min(cdiv(cnt, 256), 152 * 16), 256, 0, st>>>(B.LC, z, B.Phi, D.n, D.t, cnt);
   ++nl;
+  if (D.t > D.n) return nl + fits_dual(D, ridge_w, ridge_v, eps_w, b_min, b_max, m, Y, B, beta, C_v, stt, st);
   // beta system: Gram = Phi_C^T Phi_C in fp32 (SIMT, lower tiles mirrored).  Its
   // condition number reaches ~1e6 on long caches, beyond what the split-bf16
   // tensor-core product (~1e-5 relative per entry) resolves within tolerance.

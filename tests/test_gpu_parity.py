@@ -88,8 +88,7 @@ def check_layer(w, heads, sample, T=None, n_pos=None, t=None, layer=0, n_hold=64
         assert parity.rel_fro(_np(O[h]), O_ref) <= 2e-3
         K, V, Q, Xr, W = _pair64(arr, h, cfg.G)
         u, _ = oracle.response_profiles(oracle.attention_logits(Q, K, scale))
-        sim = u.T @ u[:, ref["anchors"]]
-        ok, n_mis, n_tie, worst = parity.assignment_valid(_np(out3["assign"][h]), sim, ref["anchors"], TAU)
+        ok, n_mis, n_tie, worst = parity.assignment_valid_profiles(_np(out3["assign"][h]), u, ref["anchors"], TAU)
         assert ok, ("assign", h, n_mis, n_tie, worst)
     return cfg, arr, ten, out, out2
 
@@ -113,6 +112,24 @@ def test_full_llama_layer_sampled_heads():
 def test_full_context_layer_retention_2pct():
     w = synth.WORKLOADS["llama8b_T8192_r02"]
     check_layer(w, list(range(8)), [5], layer=17)
+
+
+def test_budget_above_reference_rows_uses_dual_fits():
+    """t > n: the t x t normal matrices have rank <= n, the fits run in their
+    n x n dual form (same ridge solution); compared with the primal oracle."""
+    check_layer(synth.WORKLOADS["llama8b_layer_T8192"], [1, 6], [0, 1], T=1500, n_pos=40, t=300)
+
+
+def test_long_context_32k_sampled_head():
+    """The 32K workload (T = 32768, n = 2048, t = 1638, outlier channels
+    reseeded per layer) on one KV head of layer 9."""
+    check_layer(synth.WORKLOADS["llama8b_T32768_r05"], [2], [0], layer=9, n_hold=32)
+
+
+def test_long_context_128k_sampled_head():
+    """The 128K workload (T = 131072, n = 2048, t = 13107 > n, dual-form fits)
+    on one KV head of layer 31."""
+    check_layer(synth.WORKLOADS["llama8b_T131072_r10"], [7], [0], layer=31, n_hold=32)
 
 
 def test_odd_shapes_single_index_head():
