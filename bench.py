@@ -381,16 +381,32 @@ def run_gpu(args, dist: Dist):
             logits_ms.append(evs[1].elapsed_time(evs[2]))
     stage_ms = [x / args.steps for x in stage_ms]
 
+    # the same kernel timed alone: layer 0 on one stream, blocking calls
+    iso_ms = []
+    iso_ev = new_events(n_ev)
+    iso_h = [e.cuda_event for e in iso_ev]
+    for _ in range(5):
+        st_, _ = pk.arckv_compact(cfg_block, dev_in[0]["K"], dev_in[0]["V"], dev_in[0]["Q"], dev_in[0]["X"],
+                                  workload.indexer_dict(dev_in[0]), outs[0]["C_k"], outs[0]["beta"], outs[0]["C_v"],
+                                  wss[0], wss[0].numel(), stream=stream, stage_events=iso_h)
+        if st_ != 0:
+            raise pk.ArckvError(st_, "isolated layer")
+        iso_ms.append(iso_ev[1].elapsed_time(iso_ev[2]))
+
     # roofline of the dominant kernel (index logits, one launch per layer): a
     # split-bf16 tcgen05 GEMM issuing three bf16 MMAs per useful product
     flops = 2.0 * w.H_kv * w.n * w.T * w.shape.H_I * w.shape.d_I
     avg_s = statistics.mean(logits_ms) / 1e3
+    iso_s = statistics.median(iso_ms) / 1e3
     peak, _, peak_src = measured_peaks()
     achieved = flops / avg_s / 1e12
     roofline = {"kernel": "tc_gemm_kernel<128, split, TcEpiIndex> (index logits, Eq. pairwise_index_score)",
                 "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                 "traffic": profiled_traffic(), "flops_per_launch": flops, "launch_ms": avg_s * 1e3,
                 "issued_tflops": 3.0 * achieved, "issued_frac": 3.0 * achieved / peak,
+                "launch_ms_isolated": iso_s * 1e3, "frac_isolated": flops / iso_s / 1e12 / peak,
+                "timing_note": "launch_ms: live CUDA events over the timed region, where 4 streams share the GPU; "
+                               "launch_ms_isolated: the same launch with the GPU to itself (median of 5)",
                 "peak_note": "bf16 dense, sustained, of %s (MEASURED_PEAKS.json); achieved counts useful flops, "
                              "issued counts the 3 bf16 MMAs of each split-bf16 product" % peak_src}
 
