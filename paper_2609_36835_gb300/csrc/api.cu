@@ -206,7 +206,7 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
     if (nlk < 0) return ARCKV_ERR_CUDA;
     nl += nlk;
     QueryBufs QB{F(L.vq), F(L.qpp), F(L.NT), F(L.rA), F(L.rB), F(L.av), F(L.cctx),
-                 B16(L.q_h), B16(L.q_m), B16(L.q_l), B16(L.p_h), B16(L.p_m), B16(L.p_l)};
+                 B16(L.q_h), B16(L.q_m), B16(L.q_l), B16(L.p_h), B16(L.p_m), B16(L.p_l), (float2*)(w + L.part)};
     const int nlq = launch_query_features(D, Qb, (const bf16*)X_ref, Kb, B16(L.VT), (const bf16*)idx->U_q,
                                           (const bf16*)idx->U_k, (const bf16*)idx->U_v, (const bf16*)idx->L_q,
                                           (const bf16*)idx->L_c, (const bf16*)idx->L_x, (const bf16*)idx->b_x, QB,
@@ -228,7 +228,8 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
     nl += launch_check_anchors(D, anchors, stt, st);
   }
   mark(3);
-  const int nlr = launch_reference_attention(D, scale, Qb, Kb, B16(L.VT), F(L.NT), F(L.z), F(L.m), F(L.invm),
+  const int nlr = launch_reference_attention(D, scale, Qb, Kb, B16(L.VT), F(L.NT), (float2*)(w + L.part), F(L.z),
+                                             F(L.m), F(L.invm),
                                              B16(L.p_h), B16(L.p_m), B16(L.p_l), F(L.Y), F(L.logphi), F(L.colM),
                                              F(L.colInvN), stt, st);
   if (nlr < 0) return ARCKV_ERR_CUDA;

@@ -47,10 +47,10 @@ int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf1
               D.n, D.d, D.d_A, 1, st);
   nl += 2;
   // value-attention logits on the tensor cores, unscaled as printed in Eq. value_context
-  int r = launch_value_logits_tc(D, B.qpp, B.q_h, B.q_m, B.q_l, K, B.logits, stt, st);
+  int r = launch_value_logits_tc(D, B.qpp, B.q_h, B.q_m, B.q_l, K, B.logits, B.part, stt, st);
   if (r < 0) return -1;
   nl += r;
-  nl += launch_row_stats(D.H, D.n, D.T, B.logits, B.rshift, B.rmul, nullptr, st);
+  nl += launch_part_stats(D.H, D.n, cdiv(D.T, 128), B.part, B.rshift, B.rmul, nullptr, st);
   // A^V V on the tensor cores, then c = (A^V V) U_v^T = A^V (U_v V)
   r = launch_probs_v_tc(D, B.logits, B.rshift, B.rmul, B.p_h, B.p_m, B.p_l, VT, B.av, stt, st);
   if (r < 0) return -1;
@@ -84,39 +84,46 @@ __global__ void lse_reduce_kernel(const float2* part, float* lse, int n, int nti
   if (lane == 0) lse[(long long)b * n + row] = mx + logf(sm);
 }
 
-// s_j = sqrt(mean_i exp(2 (I_ij - lse_i))); one thread per column, rows in order.
+// s_j = sqrt(mean_i exp(2 (I_ij - lse_i))).  A CTA owns 32 columns; warp w
+// sums the rows i = w, w+8, ... of its column (four independent partial sums
+// per thread) and the eight warp sums are added in warp order.
 __global__ void __launch_bounds__(256) pool_kernel(const float* I, const float* lse, float* s, int n, int T) {
-  const int b = blockIdx.y, j = blockIdx.x * 256 + threadIdx.x;
-  __shared__ float ls[256];
-  const float* Ib = I + (long long)b * n * T;
+  const int b = blockIdx.y, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int j = blockIdx.x * 32 + lane;
+  __shared__ float red[8][33];
+  const float* Ib = I + (long long)b * n * T + j;
   const float* lb = lse + (long long)b * n;
-  float a0 = 0.f, a1 = 0.f;
-  for (int i0 = 0; i0 < n; i0 += 256) {
-    __syncthreads();
-    if (i0 + (int)threadIdx.x < n) ls[threadIdx.x] = lb[i0 + threadIdx.x];
-    __syncthreads();
-    const int cnt = min(256, n - i0);
-    if (j < T) {
-      int q = 0;
-      for (; q + 1 < cnt; q += 2) {
-        const float p0 = expf(Ib[(long long)(i0 + q) * T + j] - ls[q]);
-        const float p1 = expf(Ib[(long long)(i0 + q + 1) * T + j] - ls[q + 1]);
-        a0 = fmaf(p0, p0, a0);
-        a1 = fmaf(p1, p1, a1);
-      }
-      if (q < cnt) {
-        const float p0 = expf(Ib[(long long)(i0 + q) * T + j] - ls[q]);
-        a0 = fmaf(p0, p0, a0);
-      }
+  float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+  if (j < T) {
+    int i = warp;
+    for (; i + 24 < n; i += 32) {
+      const float p0 = expf(Ib[(long long)i * T] - lb[i]);
+      const float p1 = expf(Ib[(long long)(i + 8) * T] - lb[i + 8]);
+      const float p2 = expf(Ib[(long long)(i + 16) * T] - lb[i + 16]);
+      const float p3 = expf(Ib[(long long)(i + 24) * T] - lb[i + 24]);
+      a0 = fmaf(p0, p0, a0);
+      a1 = fmaf(p1, p1, a1);
+      a2 = fmaf(p2, p2, a2);
+      a3 = fmaf(p3, p3, a3);
+    }
+    for (; i < n; i += 8) {
+      const float p0 = expf(Ib[(long long)i * T] - lb[i]);
+      a0 = fmaf(p0, p0, a0);
     }
   }
-  if (j < T) s[(long long)b * T + j] = sqrtf((a0 + a1) / (float)n);
+  red[warp][lane] = (a0 + a1) + (a2 + a3);
+  __syncthreads();
+  if (warp == 0 && j < T) {
+    float a = 0.f;
+    for (int w = 0; w < 8; ++w) a += red[w][lane];
+    s[(long long)b * T + j] = sqrtf(a / (float)n);
+  }
 }
 
 int launch_index_pool(const Dims& D, const float* I, const float2* part, float* lse, float* s, cudaStream_t st) {
   const int ntiles = cdiv(D.T, GBN);
   lse_reduce_kernel<<<dim3(cdiv(D.n, 8), D.H), 256, 0, st>>>(part, lse, D.n, ntiles);
-  pool_kernel<<<dim3(cdiv(D.T, 256), D.H), 256, 0, st>>>(I, lse, s, D.n, D.T);
+  pool_kernel<<<dim3(cdiv(D.T, 32), D.H), 256, 0, st>>>(I, lse, s, D.n, D.T);
   return 2;
 }
 

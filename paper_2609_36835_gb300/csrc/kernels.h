@@ -21,6 +21,7 @@ int launch_key_features_tc(const Dims& D, const bf16* K, const bf16* V, const bf
 struct QueryBufs {
   float *vq, *qpp, *logits, *rshift, *rmul, *av, *cctx;
   bf16 *q_h, *q_m, *q_l, *p_h, *p_m, *p_l;
+  float2* part;  // per-(row, 128-column tile) softmax partials of the logits
 };
 // value context c (Eq. value_context), q_bar (Eq. indexer_projection), w.
 // VT is V transposed ([H][d][ldT] bf16, launch_transpose_v).  -1 on a TMA failure.
@@ -31,7 +32,7 @@ int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf1
 // softmax products with fp32-grade split-3 operands (tc_attn.cu)
 int launch_transpose_v(const Dims& D, const bf16* V, bf16* VT, cudaStream_t st);
 int launch_value_logits_tc(const Dims& D, const float* qpp, bf16* q_h, bf16* q_m, bf16* q_l, const bf16* K,
-                           float* logits, DevStatus* stt, cudaStream_t st);
+                           float* logits, float2* part, DevStatus* stt, cudaStream_t st);
 // out [H][n][128] = (exp(X - shift) * mul) V over rows of X [H][n][T].
 int launch_probs_v_tc(const Dims& D, const float* X, const float* shift, const float* mul, bf16* p_h, bf16* p_m,
                       bf16* p_l, const bf16* VT, float* out, DevStatus* stt, cudaStream_t st);
@@ -53,11 +54,11 @@ int launch_check_anchors(const Dims& D, int* anchors, DevStatus* stt, cudaStream
 // (tcgen05, split-3 probabilities against VT); column statistics log phi,
 // M_j and 1/||e^{l_:j - M_j}||.  -1 when a TMA descriptor cannot be encoded.
 int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const bf16* K, const bf16* VT,
-                               float* L, float* z, float* m, float* invm, bf16* p_h, bf16* p_m, bf16* p_l,
-                               float* Y, float* logphi, float* colM, float* colInvN, DevStatus* stt,
+                               float* L, float2* part, float* z, float* m, float* invm, bf16* p_h, bf16* p_m,
+                               bf16* p_l, float* Y, float* logphi, float* colM, float* colInvN, DevStatus* stt,
                                cudaStream_t st);
-int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* K, float* L, DevStatus* stt,
-                         cudaStream_t st);
+int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* K, float* L, float2* part,
+                         DevStatus* stt, cudaStream_t st);
 // Assignment on tcgen05: transposed split-bf16 profiles, anchor rows, argmax GEMM.
 int launch_assign_tc(const Dims& D, const float* L, const float* colM, const float* colInvN, const int* anchors,
                      bf16* Ut_hi, bf16* Ut_lo, bf16* S_hi, bf16* S_lo, unsigned long long* best, int* kappa,
@@ -83,8 +84,8 @@ int launch_attend(int H, int n, int t, float scale, const bf16* Q, const float* 
                   const float* C_v, float* O, float* LC, float* split, cudaStream_t st);
 
 // Shared small kernels.
-int launch_row_stats(int H, int rows, int cols, const float* X, float* shift, float* mul, float* sum,
-                     cudaStream_t st);
+int launch_part_stats(int H, int rows, int ntiles, const float2* part, float* shift, float* mul, float* sum,
+                      cudaStream_t st);
 int launch_split_reduce(int H, int M, int N, int splits, const float* part, float* out, cudaStream_t st);
 
 }  // namespace arckv

@@ -62,13 +62,13 @@ __global__ void __launch_bounds__(256) col_stats_kernel(const float* L, float* l
 }
 
 int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const bf16* K, const bf16* VT,
-                               float* L, float* z, float* m, float* invm, bf16* p_h, bf16* p_m, bf16* p_l,
-                               float* Y, float* logphi, float* colM, float* colInvN, DevStatus* stt,
+                               float* L, float2* part, float* z, float* m, float* invm, bf16* p_h, bf16* p_m,
+                               bf16* p_l, float* Y, float* logphi, float* colM, float* colInvN, DevStatus* stt,
                                cudaStream_t st) {
-  // l = scale * Q K^T on the tensor cores
-  if (launch_ref_logits_tc(D, scale, Q, K, L, stt, st) < 0) return -1;
+  // l = scale * Q K^T on the tensor cores, with per-tile row softmax partials
+  if (launch_ref_logits_tc(D, scale, Q, K, L, part, stt, st) < 0) return -1;
   // z_i = max_j l_ij (z^fit of Eq. mass_fit), m_i = sum_j e^{l_ij - z_i} = (Phi_K 1)_i
-  launch_row_stats(D.H, D.n, D.T, L, z, invm, m, st);
+  launch_part_stats(D.H, D.n, cdiv(D.T, 128), part, z, invm, m, st);
   // Y = softmax(l) V
   const int r = launch_probs_v_tc(D, L, z, invm, p_h, p_m, p_l, VT, Y, stt, st);
   if (r < 0) return -1;

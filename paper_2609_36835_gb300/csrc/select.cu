@@ -114,17 +114,14 @@ int launch_check_anchors(const Dims& D, int* anchors, DevStatus* stt, cudaStream
   return 1;
 }
 
-// Per row: shift = max_c X, sum = sum_c exp(X - shift), mul = 1 / sum (one warp per row).
-__global__ void row_stats_kernel(const float* X, float* shift, float* mul, float* sum, int rows, int cols) {
+// Row statistics from per-tile softmax partials part[b][row][tile] = (max, sum):
+// shift = max, sum = total sum of exp(x - shift), mul = 1 / sum.  One warp per row.
+__global__ void part_stats_kernel(const float2* part, float* shift, float* mul, float* sum, int rows, int ntiles) {
   const int b = blockIdx.y, row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (row >= rows) return;
-  const float* x = X + ((long long)b * rows + row) * cols;
+  const float2* p = part + ((long long)b * rows + row) * ntiles;
   float mx = -INFINITY, sm = 0.f;
-  for (int c = lane; c < cols; c += 32) {
-    const float v = x[c];
-    if (v > mx) { sm = (mx == -INFINITY ? 0.f : sm * expf(mx - v)) + 1.f; mx = v; }
-    else sm += expf(v - mx);
-  }
+  for (int k = lane; k < ntiles; k += 32) lse_combine(mx, sm, p[k].x, p[k].y);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     const float om = __shfl_xor_sync(0xffffffffu, mx, o), os = __shfl_xor_sync(0xffffffffu, sm, o);
@@ -138,9 +135,9 @@ __global__ void row_stats_kernel(const float* X, float* shift, float* mul, float
   }
 }
 
-int launch_row_stats(int H, int rows, int cols, const float* X, float* shift, float* mul, float* sum,
-                     cudaStream_t st) {
-  row_stats_kernel<<<dim3(cdiv(rows, 8), H), 256, 0, st>>>(X, shift, mul, sum, rows, cols);
+int launch_part_stats(int H, int rows, int ntiles, const float2* part, float* shift, float* mul, float* sum,
+                      cudaStream_t st) {
+  part_stats_kernel<<<dim3(cdiv(rows, 8), H), 256, 0, st>>>(part, shift, mul, sum, rows, ntiles);
   return 1;
 }
 

@@ -66,10 +66,16 @@ static int gemm_split3a(int H, int rows, int N, int K, int ldk, const bf16* h, c
 }
 
 int launch_value_logits_tc(const Dims& D, const float* qpp, bf16* q_h, bf16* q_m, bf16* q_l, const bf16* K,
-                           float* logits, DevStatus* stt, cudaStream_t st) {
+                           float* logits, float2* part, DevStatus* stt, cudaStream_t st) {
   const long long cnt = (long long)D.H * D.n * 128;
   split3_kernel<<<min(cdiv(cnt, 256), 152 * 8), 256, 0, st>>>(qpp, q_h, q_m, q_l, cnt);
-  if (gemm_split3a(D.H, D.n, D.T, 128, 128, q_h, q_m, q_l, K, logits, D.T, 1.f, stt, st) < 0) return -1;
+  CUtensorMap mA, mA2, mA3, mB;
+  if (!encode_bf16_map_3d(&mA, q_h, 128, D.n, D.H, 128) || !encode_bf16_map_3d(&mA2, q_m, 128, D.n, D.H, 128) ||
+      !encode_bf16_map_3d(&mA3, q_l, 128, D.n, D.H, 128) || !encode_bf16_map_3d(&mB, K, 128, D.T, D.H, 128))
+    return -1;
+  TcEpiStoreRowPart epi{{logits, (long long)D.n * D.T, D.T, 1.f}, part, cdiv(D.T, 128), 128};
+  if (launch_tc_gemm<128, kSplit3A>(mA, mB, mA2, mA, epi, D.H, D.n, D.T, 128, 128, stt, st, 0, &mA3) != cudaSuccess)
+    return -1;
   return 2;
 }
 

@@ -256,4 +256,40 @@ struct TcEpiStore {
   __device__ __forceinline__ void finish(State&, int, int, int, int, int) const {}
 };
 
+// TcEpiStore that also writes each row's softmax partials over the tile's
+// columns: part[b][row][n0 / BN] = (max, sum exp(x - max)) of alpha * acc.
+struct TcEpiStoreRowPart {
+  TcEpiStore st;
+  float2* part;
+  int ntiles, BNt;
+  struct State {
+    TcEpiStore::State s;
+    float mx, sm;
+    long long prow;
+  };
+  __device__ __forceinline__ void init(State& s, int b, int row, int n0, int M, int N) const {
+    st.init(s.s, b, row, n0, M, N);
+    s.mx = -INFINITY;
+    s.sm = 0.f;
+    s.prow = ((long long)b * M + row) * ntiles + n0 / BNt;
+  }
+  __device__ __forceinline__ void consume(State& s, int c, int j, float (&v)[32]) const {
+    st.consume(s.s, c, j, v);
+    float m = s.mx;
+#pragma unroll
+    for (int q = 0; q < 32; ++q)
+      if (j * 32 + q < s.s.ncols) m = fmaxf(m, st.alpha * v[q]);
+    if (m == -INFINITY) return;
+    float a = s.sm * expf(s.mx - m);
+#pragma unroll
+    for (int q = 0; q < 32; ++q)
+      if (j * 32 + q < s.s.ncols) a += expf(st.alpha * v[q] - m);
+    s.mx = m;
+    s.sm = a;
+  }
+  __device__ __forceinline__ void finish(State& s, int, int, int, int, int) const {
+    if (s.s.row_ok) part[s.prow] = make_float2(s.mx, s.sm);
+  }
+};
+
 }  // namespace arckv
