@@ -11,6 +11,8 @@
 // is factored and inverted in shared memory) with the forward substitution
 // fused into the trailing updates, then blocked back substitution, all in one
 // cluster launch per system (chol_cluster_kernel).
+#include <cooperative_groups.h>
+
 #include "gemm.cuh"
 #include "kernels.h"
 #include "tc_gemm.cuh"
@@ -56,10 +58,19 @@ __global__ void mass_rhs_kernel(const float* Phi, const float* m, float* rhs, in
 // when the dual system is solved).
 constexpr int kCL = 8;
 constexpr int kCT = 512;
-constexpr int kTileF = NB * (NB + 1);
+// Shared tiles are [NB][NBP] with rows padded to a 16-byte multiple, so that
+// mm64 can read them with vector loads.
+template <typename R>
+constexpr int NBP = NB + 16 / (int)sizeof(R);
+template <typename R>
+using Tile = R (*)[NBP<R>];
+template <typename R>
+constexpr int kTileF = NB * NBP<R>;
 
 __device__ __forceinline__ float fma_r(float a, float b, float c) { return fmaf(a, b, c); }
 __device__ __forceinline__ double fma_r(double a, double b, double c) { return fma(a, b, c); }
+__device__ __forceinline__ float rcp_r(float x) { return __frcp_rn(x); }
+__device__ __forceinline__ double rcp_r(double x) { return __drcp_rn(x); }
 template <typename R>
 __device__ __forceinline__ R warp_sum_r(R v) {
 #pragma unroll
@@ -76,98 +87,272 @@ __device__ __forceinline__ unsigned cluster_rank() {
   return r;
 }
 
-// S[r][c] = G[(r0 + r) * ld + c0 + c] (or its transpose with `trans`), zero outside
-// rows < rmax, cols < cmax of the source block.
+// S[r][c] = G[(r0 + r) * ld + c0 + c] (or S[c][r] with `trans`), zero outside
+// rows < rmax, cols < cmax of the source block.  Every thread issues its eight
+// loads before its first shared store, so the L2 latency is paid once per tile.
+// The transposed form maps a warp to 4 rows x 8 columns, so its shared stores
+// hit 32 distinct banks.
 template <typename R>
-__device__ __forceinline__ void ld_tile(R (*S)[NB + 1], const R* G, long long ld, int r0, int c0, int rmax, int cmax,
+__device__ __forceinline__ void ld_tile(Tile<R> S, const R* G, long long ld, int r0, int c0, int rmax, int cmax,
                                         bool trans) {
-  for (int e = threadIdx.x; e < NB * NB; e += kCT) {
-    const int r = e / NB, c = e % NB;
-    const R v = (r < rmax && c < cmax) ? __ldcg(G + (long long)(r0 + r) * ld + c0 + c) : R(0);
-    if (trans) S[c][r] = v;
-    else S[r][c] = v;
+  constexpr int NE = NB * NB / kCT;
+  R v[NE];
+  int rr[NE], cc[NE];
+#pragma unroll
+  for (int q = 0; q < NE; ++q) {
+    const int e = threadIdx.x + q * kCT;
+    if (!trans) {
+      rr[q] = e / NB;
+      cc[q] = e % NB;
+    } else {
+      const int lane = e & 31, w = e >> 5;
+      cc[q] = (w & 7) * 8 + (lane & 7);
+      rr[q] = (w >> 3) * 4 + (lane >> 3);
+    }
+    v[q] = (rr[q] < rmax && cc[q] < cmax) ? __ldcg(G + (long long)(r0 + rr[q]) * ld + c0 + cc[q]) : R(0);
+  }
+#pragma unroll
+  for (int q = 0; q < NE; ++q) {
+    if (trans) S[cc[q]][rr[q]] = v[q];
+    else S[rr[q]][cc[q]] = v[q];
   }
 }
 
-// acc[p][q] = sum_l X[ry+p][l] Y[l][cx+q], ry = (tid >> 4) * 2, cx = (tid & 15) * 4.
+// P[p*ld + q] -= acc[p][q] for p < pn, q < qn (all loads issued before the stores)
 template <typename R>
-__device__ __forceinline__ void mm64(const R (*X)[NB + 1], const R (*Y)[NB + 1], R (&acc)[2][4]) {
+__device__ __forceinline__ void rmw_sub(R* P, long long ld, int pn, int qn, const R (&acc)[2][4]) {
+  R old[2][4];
+#pragma unroll
+  for (int p = 0; p < 2; ++p)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) old[p][q] = (p < pn && q < qn) ? __ldcg(P + p * ld + q) : R(0);
+#pragma unroll
+  for (int p = 0; p < 2; ++p)
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      if (p < pn && q < qn) P[p * ld + q] = old[p][q] - acc[p][q];
+}
+
+__device__ __forceinline__ void lds2(float (&a)[2], const float* p) {
+  const float2 v = *(const float2*)p;
+  a[0] = v.x; a[1] = v.y;
+}
+__device__ __forceinline__ void lds4(float (&a)[4], const float* p) {
+  const float4 v = *(const float4*)p;
+  a[0] = v.x; a[1] = v.y; a[2] = v.z; a[3] = v.w;
+}
+__device__ __forceinline__ void lds2(double (&a)[2], const double* p) {
+  const double2 v = *(const double2*)p;
+  a[0] = v.x; a[1] = v.y;
+}
+__device__ __forceinline__ void lds4(double (&a)[4], const double* p) {
+  const double2 v = *(const double2*)p, u = *(const double2*)(p + 2);
+  a[0] = v.x; a[1] = v.y; a[2] = u.x; a[3] = u.y;
+}
+
+// acc[p][q] = sum_l XT[l][ry+p] Y[l][cx+q], ry = (tid >> 4) * 2, cx = (tid & 15) * 4:
+// the left operand is held transposed so that each l takes one 2-wide and one
+// 4-wide shared load.
+template <typename R>
+__device__ __forceinline__ void mm64(Tile<R> XT, Tile<R> Y, R (&acc)[2][4]) {
   const int ry = (threadIdx.x >> 4) * 2, cx = (threadIdx.x & 15) * 4;
 #pragma unroll
   for (int p = 0; p < 2; ++p)
 #pragma unroll
-    for (int q = 0; q < 4; ++q) acc[p][q] = 0.f;
+    for (int q = 0; q < 4; ++q) acc[p][q] = R(0);
 #pragma unroll 8
   for (int l = 0; l < NB; ++l) {
-    // rows of the [64][65] tiles are 260 bytes apart: scalar loads only
-    const R a0 = X[ry][l], a1 = X[ry + 1][l];
-    const R c0 = Y[l][cx], c1 = Y[l][cx + 1], c2 = Y[l][cx + 2], c3 = Y[l][cx + 3];
-    acc[0][0] = fma_r(a0, c0, acc[0][0]); acc[0][1] = fma_r(a0, c1, acc[0][1]);
-    acc[0][2] = fma_r(a0, c2, acc[0][2]); acc[0][3] = fma_r(a0, c3, acc[0][3]);
-    acc[1][0] = fma_r(a1, c0, acc[1][0]); acc[1][1] = fma_r(a1, c1, acc[1][1]);
-    acc[1][2] = fma_r(a1, c2, acc[1][2]); acc[1][3] = fma_r(a1, c3, acc[1][3]);
+    R a[2], c[4];
+    lds2(a, &XT[l][ry]);
+    lds4(c, &Y[l][cx]);
+#pragma unroll
+    for (int p = 0; p < 2; ++p)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) acc[p][q] = fma_r(a[p], c[q], acc[p][q]);
   }
 }
 
-// Factor diagonal block k (lower part of A_kk + lam I) in shared memory; write
-// L_kk into A and its inverse into Linv[k].  8 threads per row.
+// Load the lower part of A_kk + lam I into the tile L (identity beyond the
+// matrix when kb < NB; zero above the diagonal).
 template <typename R>
-__device__ void factor_diag(R* Ab, R* Lb, int t, int k, R lam, R (*L)[NB + 1], R (*Li)[NB + 1], int* bad) {
-  const int tid = threadIdx.x, k0 = k * NB, kb = min(NB, t - k0);
-  for (int e = tid; e < NB * NB; e += kCT) {
-    const int r = e / NB, c = e % NB;
-    L[r][c] = (r < kb && c <= r) ? __ldcg(Ab + (long long)(k0 + r) * t + k0 + c) + (r == c ? lam : R(0))
-                                 : (r == c ? R(1) : R(0));
-    Li[r][c] = R(0);
+__device__ __forceinline__ void load_diag(Tile<R> L, const R* Ab, int t, int k0, int kb, R lam) {
+  constexpr int NE = NB * NB / kCT;
+  R v[NE];
+#pragma unroll
+  for (int q = 0; q < NE; ++q) {
+    const int e = threadIdx.x + q * kCT, r = e / NB, c = e % NB;
+    v[q] = (r < kb && c <= r) ? __ldcg(Ab + (long long)(k0 + r) * t + k0 + c) + (r == c ? lam : R(0))
+                              : (r == c ? R(1) : R(0));
   }
-  __syncthreads();
-  const int r = tid >> 3, p = tid & 7;
-  for (int c = 0; c < NB; ++c) {
-    R v = R(0);
-    if (r >= c)
-      for (int q = p; q < c; q += 8) v = fma_r(L[r][q], L[c][q], v);
-    v += __shfl_xor_sync(0xffffffffu, v, 1);
-    v += __shfl_xor_sync(0xffffffffu, v, 2);
-    v += __shfl_xor_sync(0xffffffffu, v, 4);
-    v = (r >= c) ? L[r][c] - v : R(0);
-    if (r == c && p == 0) {
-      if (!(v > R(0)) || !isfinite(v)) { *bad = 1; v = R(1); }
-      L[c][c] = sqrt(v);
-    }
-    __syncthreads();
-    if (r > c && p == 0) L[r][c] = v / L[c][c];
-    __syncthreads();
+#pragma unroll
+  for (int q = 0; q < NE; ++q) {
+    const int e = threadIdx.x + q * kCT;
+    L[e / NB][e % NB] = v[q];
   }
-  for (int i = 0; i < NB; ++i) {
-    R v = R(0);
-    if (r < i)
-      for (int l = r + p; l < i; l += 8) v = fma_r(L[i][l], Li[l][r], v);
-    v += __shfl_xor_sync(0xffffffffu, v, 1);
-    v += __shfl_xor_sync(0xffffffffu, v, 2);
-    v += __shfl_xor_sync(0xffffffffu, v, 4);
-    if (r <= i && p == 0) Li[i][r] = ((i == r ? R(1) : R(0)) - v) / L[i][i];
-    __syncthreads();
-  }
+}
+
+// Write L_kk (lower part, rows < kb) into A and the full tile Li into Linv[k].
+template <typename R>
+__device__ __forceinline__ void store_diag(Tile<R> L, Tile<R> Li, R* Ab, R* Lb, int t, int k, int kb) {
   R* Lo = Lb + (long long)k * NB * NB;
-  for (int e = tid; e < NB * NB; e += kCT) {
+  const int k0 = k * NB;
+  for (int e = threadIdx.x; e < NB * NB; e += kCT) {
     const int rr = e / NB, cc = e % NB;
     Lo[e] = Li[rr][cc];
     if (rr < kb && cc <= rr) Ab[(long long)(k0 + rr) * t + k0 + cc] = L[rr][cc];
   }
+}
+
+// Factor diagonal block k (lower part of A_kk + lam I) in shared memory and
+// invert the factor: L_kk goes into A and L_kk^-1 into Linv[k].
+//   factor:  right-looking and unscaled, one barrier per column: step c
+//            subtracts a_rc a_jc / a_cc from every (r, j) with c < j <= r (the
+//            lower triangle is dealt to the threads); the thread that finishes
+//            a_c+1,c+1 publishes its reciprocal (pad column NB + 1); the column
+//            scaling by sqrt(a_cc) follows in one pass;
+//   inverse: each warp forms four columns of L^-1 by forward substitution
+//            (column j of L^-1 solves L x = e_j), reading L^T from Li.
+// Pad rows beyond the matrix (kb < NB) are the identity.
+template <typename R>
+__device__ void factor_diag(R* Ab, R* Lb, int t, int k, R lam, Tile<R> L, Tile<R> Li, int* bad) {
+  static_assert(kCT == 16 * 32, "the inverse deals 64 columns to 16 warps");
+  const int tid = threadIdx.x, k0 = k * NB, kb = min(NB, t - k0);
+  load_diag(L, Ab, t, k0, kb, lam);
   __syncthreads();
+  constexpr int NT = NB * (NB + 1) / 2, NQ = (NT + kCT - 1) / kCT;
+  int er[NQ], ej[NQ];
+#pragma unroll
+  for (int q = 0; q < NQ; ++q) {
+    const int e = tid + q * kCT;
+    int rr = (int)((sqrtf(8.f * e + 1.f) - 1.f) * 0.5f);
+    while (rr * (rr + 1) / 2 > e) --rr;
+    while ((rr + 1) * (rr + 2) / 2 <= e) ++rr;
+    er[q] = e < NT ? rr : -1;
+    ej[q] = e < NT ? e - rr * (rr + 1) / 2 : -1;   // -1: no entry (never > c)
+  }
+  auto pivot_inv = [](R v) { return (v > R(0) && isfinite(v)) ? rcp_r(v) : R(1); };
+  if (tid == 0) L[0][NB + 1] = pivot_inv(L[0][0]);
+  __syncthreads();
+  for (int c = 0; c < NB - 1; ++c) {
+    R a[NQ], b[NQ], d[NQ];
+    const R pinv = L[c][NB + 1];
+#pragma unroll
+    for (int q = 0; q < NQ; ++q)
+      if (ej[q] > c) {
+        a[q] = L[er[q]][c];
+        b[q] = L[ej[q]][c];
+        d[q] = L[er[q]][ej[q]];
+      }
+#pragma unroll
+    for (int q = 0; q < NQ; ++q)
+      if (ej[q] > c) {
+        const R v = fma_r(-a[q] * pinv, b[q], d[q]);
+        L[er[q]][ej[q]] = v;
+        if (er[q] == c + 1 && ej[q] == c + 1) L[c + 1][NB + 1] = pivot_inv(v);
+      }
+    __syncthreads();
+  }
+  R nv[NQ];
+#pragma unroll
+  for (int q = 0; q < NQ; ++q)
+    if (er[q] >= 0) {
+      const int rr = er[q], j = ej[q];
+      R pj = L[j][j];
+      if (!(pj > R(0)) || !isfinite(pj)) {
+        if (rr == j && j < kb) *bad = 1;
+        pj = R(1);
+      }
+      const R dj = sqrt(pj), djinv = rcp_r(dj);
+      nv[q] = (rr == j) ? dj : L[rr][j] * djinv;
+      if (rr == j) L[j][NB] = djinv;   // the pad column holds 1 / L_jj for the inverse
+    }
+  __syncthreads();
+#pragma unroll
+  for (int q = 0; q < NQ; ++q)
+    if (er[q] >= 0) {
+      L[er[q]][ej[q]] = nv[q];
+      Li[ej[q]][er[q]] = nv[q];   // Li holds L^T until the inverse replaces it
+    }
+  __syncthreads();
+  {  // columns of L^-1: warp w takes j = w, 63 - w, 16 + w, 47 - w (130 substitution steps each)
+    const int w = tid >> 5, lane = tid & 31;
+    const int js[4] = {w, NB - 1 - w, 16 + w, 47 - w};
+    R x0[4], x1[4];   // rows lane and lane + 32 of the four columns
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      x0[u] = (lane == js[u]) ? R(1) : R(0);
+      x1[u] = (lane + 32 == js[u]) ? R(1) : R(0);
+    }
+    for (int i = w; i < NB; ++i) {
+      const R dinv = L[i][NB];
+      const R l0 = Li[i][lane], l1 = Li[i][lane + 32];   // L[lane][i], L[lane + 32][i]
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if (i < js[u]) continue;
+        const R src = i < 32 ? x0[u] : x1[u];
+        const R xi = __shfl_sync(0xffffffffu, src, i & 31) * dinv;
+        if (lane == i) x0[u] = xi;
+        else if (lane > i) x0[u] = fma_r(-l0, xi, x0[u]);
+        if (lane + 32 == i) x1[u] = xi;
+        else if (lane + 32 > i) x1[u] = fma_r(-l1, xi, x1[u]);
+      }
+    }
+    __syncthreads();   // every warp has finished reading L^T from Li
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      Li[lane][js[u]] = x0[u];
+      Li[lane + 32][js[u]] = x1[u];
+    }
+  }
+  __syncthreads();
+  store_diag(L, Li, Ab, Lb, t, k, kb);
+  __syncthreads();
+}
+
+// S[r][c] = G1[(r0 + r) * ld + c0 + c] + G2[...] (zero outside rows < rmax, cols < cmax)
+template <typename R>
+__device__ __forceinline__ void ld_tile_sum(Tile<R> S, const R* G1, const R* G2, long long ld, int r0, int c0,
+                                            int rmax, int cmax) {
+  constexpr int NE = NB * NB / kCT;
+  R v[NE], u[NE];
+#pragma unroll
+  for (int q = 0; q < NE; ++q) {
+    const int e = threadIdx.x + q * kCT, r = e / NB, c = e % NB;
+    const bool ok = r < rmax && c < cmax;
+    const long long o = (long long)(r0 + r) * ld + c0 + c;
+    v[q] = ok ? __ldcg(G1 + o) : R(0);
+    u[q] = ok ? __ldcg(G2 + o) : R(0);
+  }
+#pragma unroll
+  for (int q = 0; q < NE; ++q) {
+    const int e = threadIdx.x + q * kCT;
+    S[e / NB][e % NB] = v[q] + u[q];
+  }
+}
+
+// P[p*ld + q] = acc[p][q] for p < pn, q < qn
+template <typename R>
+__device__ __forceinline__ void st_acc(R* P, long long ld, int pn, int qn, const R (&acc)[2][4]) {
+#pragma unroll
+  for (int p = 0; p < 2; ++p)
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      if (p < pn && q < qn) P[p * ld + q] = acc[p][q];
 }
 
 template <typename R>
 __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     chol_cluster_kernel(R* A, R* Linv, R* B, R* Z, R* X, int t, int nrhs, int ldb, long long bbs, R ridge, R tdiv,
                         DevStatus* stt) {
+  namespace cg = cooperative_groups;
   extern __shared__ __align__(16) unsigned char smraw[];
   R* sm = (R*)smraw;
-  R (*S1)[NB + 1] = (R (*)[NB + 1])sm;
-  R (*S2)[NB + 1] = (R (*)[NB + 1])(sm + kTileF);
-  R (*S3)[NB + 1] = (R (*)[NB + 1])(sm + 2 * kTileF);
+  Tile<R> S1 = (Tile<R>)sm;
+  Tile<R> S2 = (Tile<R>)(sm + kTileF<R>);
+  Tile<R> S3 = (Tile<R>)(sm + 2 * kTileF<R>);
   __shared__ R red[kCT / 32];
-  __shared__ int bad;
+  __shared__ int bad, grab;
+  __shared__ int ctr[2];   // rank 0's pair deals the tiles of alternate dynamic phases
   const int head = blockIdx.x / kCL;
   const int rank = (int)cluster_rank();
   const int tid = threadIdx.x;
@@ -179,13 +364,26 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
   R* Xb = X + (long long)head * bbs;
   const int ry = (tid >> 4) * 2, cx = (tid & 15) * 4;
   R acc[2][4];
+  int* ctr0 = cg::this_cluster().map_shared_rank(ctr, 0);
+  int ep = 0;   // dynamic phase number; phase ep draws from ctr0[ep & 1]
+  // next tile of the current dynamic phase (block-uniform)
+  auto next_tile = [&]() -> int {
+    __syncthreads();
+    if (tid == 0) grab = atomicAdd(ctr0 + (ep & 1), 1);
+    __syncthreads();
+    return grab;
+  };
 
   // lam = ridge * trace / t (every CTA forms it; the trace precedes all writes)
   R tr = R(0);
   for (int r = tid; r < t; r += kCT) tr += __ldcg(Ab + (long long)r * t + r);
   tr = warp_sum_r(tr);
   if ((tid & 31) == 0) red[tid >> 5] = tr;
-  if (tid == 0) bad = 0;
+  if (tid == 0) {
+    bad = 0;
+    ctr[0] = 0;
+    ctr[1] = 0;
+  }
   __syncthreads();
   if (tid < 32) {
     R v = tid < kCT / 32 ? red[tid] : R(0);
@@ -198,133 +396,122 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
   if (rank == 0 && tid == 0 && !isfinite(trace)) set_status(stt, ARCKV_ERR_NONFINITE);
   // zero Z (rows split over the cluster) and factor the first diagonal block
   for (long long e = (long long)rank * kCT + tid; e < (long long)t * ldb; e += (long long)kCL * kCT) Zb[e] = R(0);
-  cluster_sync_all();   // everyone has read the unmodified diagonal for the trace
-  if (rank == 0) factor_diag(Ab, Lb, t, 0, lam, S1, S2, &bad);
-  cluster_sync_all();
+  cluster_sync_all();   // everyone has read the unmodified diagonal for the trace; counters are set
 
-  for (int k = 0; k < nblk; ++k) {
-    const int m = nblk - k - 1, k0 = k * NB;
-    // trsm: L_ik = A_ik Linv_kk^T
-    for (int x = rank; x < m; x += kCL) {
-      const int i0 = (k + 1 + x) * NB, rb = min(NB, t - i0);
-      ld_tile(S1, Ab, t, i0, k0, rb, NB, false);
-      ld_tile(S2, Lb + (long long)k * NB * NB, NB, 0, 0, NB, NB, true);   // S2[l][c] = Linv[c][l]
+  // trailing-update tiles of step k: x < ntri is the syrk tile (ii >= jj) of
+  // the m trailing blocks, A_ij -= L_ik L_jk^T; the rest are rhs tiles
+  // B_i -= L_ik Y_k with Y_k = Linv_kk B_k formed in the trsm phase
+  auto update_tile = [&](int k, int x, int ntri) {
+    const int k0 = k * NB;
+    if (x < ntri) {
+      int ii = (int)((sqrtf(8.f * x + 1.f) - 1.f) * 0.5f);
+      while (ii * (ii + 1) / 2 > x) --ii;
+      while ((ii + 1) * (ii + 2) / 2 <= x) ++ii;
+      const int jj = x - ii * (ii + 1) / 2;
+      const int i0 = (k + 1 + ii) * NB, j0 = (k + 1 + jj) * NB;
+      const int rb = min(NB, t - i0), cb = min(NB, t - j0);
+      ld_tile(S1, Ab, t, i0, k0, rb, NB, true);     // S1[l][r] = L_ik[r][l]
+      ld_tile(S2, Ab, t, j0, k0, cb, NB, true);     // S2[l][c] = L_jk[c][l]
       __syncthreads();
       mm64(S1, S2, acc);
-#pragma unroll
-      for (int p = 0; p < 2; ++p)
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-          if (ry + p < rb) Ab[(long long)(i0 + ry + p) * t + k0 + cx + q] = acc[p][q];
+      rmw_sub(Ab + (long long)(i0 + ry) * t + j0 + cx, t, rb - ry, cb - cx, acc);
+    } else {
+      const int y = x - ntri, i = k + 1 + y / nct, c0 = (y % nct) * NB;
+      const int i0 = i * NB, rb = min(NB, t - i0), nc = min(NB, nrhs - c0);
+      ld_tile(S1, Ab, t, i0, k0, rb, NB, true);     // S1[l][r] = L_ik[r][l]
+      ld_tile(S2, Bb, ldb, k0, c0, NB, nc, false);  // Y_k (block k < nblk - 1 is full)
+      __syncthreads();
+      mm64(S1, S2, acc);
+      rmw_sub(Bb + (long long)(i0 + ry) * ldb + c0 + cx, ldb, rb - ry, nc - cx, acc);
+    }
+    __syncthreads();
+  };
+
+  // step k = -1 only factors the first diagonal block (one call site keeps the
+  // register-resident factorisation inlined once)
+  for (int k = -1; k < nblk; ++k) {
+    const int m = nblk - k - 1, k0 = k * NB, kb = min(NB, t - k0);
+    const R* Lk = Lb + (long long)k * NB * NB;
+    // trsm phase: L_ik = A_ik Linv_kk^T (x < m) and Y_k = Linv_kk B_k, written over B_k
+    for (int x = rank; k >= 0 && x < m + nct; x += kCL) {
+      if (x < m) {
+        const int i0 = (k + 1 + x) * NB, rb = min(NB, t - i0);
+        ld_tile(S1, Ab, t, i0, k0, rb, NB, true);                    // S1[l][r] = A_ik[r][l]
+        ld_tile(S2, Lk, NB, 0, 0, NB, NB, true);                     // S2[l][c] = Linv[c][l]
+        __syncthreads();
+        mm64(S1, S2, acc);
+        st_acc(Ab + (long long)(i0 + ry) * t + k0 + cx, t, rb - ry, NB, acc);
+      } else {
+        const int c0 = (x - m) * NB, nc = min(NB, nrhs - c0);
+        ld_tile(S1, Lk, NB, 0, 0, NB, NB, true);                     // S1[l][r] = Linv[r][l]
+        ld_tile(S2, Bb, ldb, k0, c0, kb, nc, false);
+        __syncthreads();
+        mm64(S1, S2, acc);
+        st_acc(Bb + (long long)(k0 + ry) * ldb + c0 + cx, ldb, kb - ry, nc - cx, acc);
+      }
       __syncthreads();
     }
-    cluster_sync_all();
-    if (m == 0) break;
-    // update: syrk tiles (ii >= jj over the m trailing blocks) then rhs tiles
-    const int ntri = m * (m + 1) / 2, ntot = ntri + m * nct, owner = (k + 1) % kCL;
-    for (int pass = 0; pass < 2; ++pass) {
-      // pass 0: the owner of block k+1 updates and factors the diagonal block (x = 0)
-      int xb, xs;
-      if (pass == 0) { if (rank != owner) continue; xb = 0; xs = 1; }
-      else { xb = rank; xs = kCL; }
-      for (int x = xb; x < (pass == 0 ? 1 : ntot); x += xs) {
-        if (pass == 1 && x == 0) continue;
-        if (x < ntri) {
-          int ii = (int)((sqrtf(8.f * x + 1.f) - 1.f) * 0.5f);
-          while (ii * (ii + 1) / 2 > x) --ii;
-          while ((ii + 1) * (ii + 2) / 2 <= x) ++ii;
-          const int jj = x - ii * (ii + 1) / 2;
-          const int i0 = (k + 1 + ii) * NB, j0 = (k + 1 + jj) * NB;
-          const int rb = min(NB, t - i0), cb = min(NB, t - j0);
-          ld_tile(S1, Ab, t, i0, k0, rb, NB, false);    // L_ik
-          ld_tile(S2, Ab, t, j0, k0, cb, NB, true);     // S2[l][c] = L_jk[c][l]
-          __syncthreads();
-          mm64(S1, S2, acc);
-#pragma unroll
-          for (int p = 0; p < 2; ++p)
-#pragma unroll
-            for (int q = 0; q < 4; ++q)
-              if (ry + p < rb && cx + q < cb) {
-                R* a = Ab + (long long)(i0 + ry + p) * t + j0 + cx + q;
-                *a = __ldcg(a) - acc[p][q];
-              }
-          __syncthreads();
-          if (pass == 0) factor_diag(Ab, Lb, t, k + 1, lam, S1, S2, &bad);
-        } else {
-          const int y = x - ntri, i = k + 1 + y / nct, c0 = (y % nct) * NB;
-          const int i0 = i * NB, rb = min(NB, t - i0), nc = min(NB, nrhs - c0);
-          ld_tile(S1, Lb + (long long)k * NB * NB, NB, 0, 0, NB, NB, false);   // Linv_kk
-          ld_tile(S2, Bb, ldb, k0, c0, NB, nc, false);                        // B_k (full block)
-          __syncthreads();
-          mm64(S1, S2, acc);                                                  // y = Linv_kk B_k
-          __syncthreads();                                                    // S1 is reloaded below
-#pragma unroll
-          for (int p = 0; p < 2; ++p)
-#pragma unroll
-            for (int q = 0; q < 4; ++q) S3[ry + p][cx + q] = acc[p][q];
-          ld_tile(S1, Ab, t, i0, k0, rb, NB, false);                         // L_ik
-          __syncthreads();
-          mm64(S1, S3, acc);
-#pragma unroll
-          for (int p = 0; p < 2; ++p)
-#pragma unroll
-            for (int q = 0; q < 4; ++q)
-              if (ry + p < rb && cx + q < nc) {
-                R* bp = Bb + (long long)(i0 + ry + p) * ldb + c0 + cx + q;
-                *bp = __ldcg(bp) - acc[p][q];
-              }
-          __syncthreads();
-        }
-      }
+    if (k >= 0) {
+      cluster_sync_all();
+      if (m == 0) break;
     }
+    // update phase: the owner of block k+1 updates and factors the diagonal
+    // block first (overlapping the serial factorisation with the other CTAs'
+    // updates); every CTA then draws the remaining tiles from the counter
+    const int ntri = k >= 0 ? m * (m + 1) / 2 : 0, ntot = k >= 0 ? ntri + m * nct : 0;
+    if (rank == 0 && tid == 0) ctr[(ep + 1) & 1] = 0;
+    if (rank == (k + 1) % kCL) {
+      if (k >= 0) update_tile(k, 0, ntri);
+      factor_diag(Ab, Lb, t, k + 1, lam, S1, S2, &bad);
+    }
+    for (;;) {
+      const int x = 1 + next_tile();
+      if (x >= ntot) break;
+      update_tile(k, x, ntri);
+    }
+    ++ep;
     cluster_sync_all();
   }
-  // back substitution
-  for (int k = nblk - 1; k >= 0; --k) {
+
+  // back substitution: X_k = Linv_kk^T (Y_k + Z_k) and Z_i -= L_ki^T X_k (i < k).
+  // The owner of block k-1 applies X_k to Z_{k-1} first and forms X_{k-1} at
+  // once; the other Z tiles are drawn from the counter.
+  auto form_x = [&](int k) {
     const int k0 = k * NB, kb = min(NB, t - k0);
-    for (int x = rank; x < (k + 1) * nct; x += kCL) {
-      const int i = x / nct, c0 = (x % nct) * NB, nc = min(NB, nrhs - c0);
-      ld_tile(S1, Lb + (long long)k * NB * NB, NB, 0, 0, NB, NB, false);     // Linv_kk
-      ld_tile(S2, Bb, ldb, k0, c0, kb, nc, false);
+    for (int c0 = 0; c0 < nrhs; c0 += NB) {
+      const int nc = min(NB, nrhs - c0);
+      ld_tile(S1, Lb + (long long)k * NB * NB, NB, 0, 0, NB, NB, false);   // S1[l][r] = Linv[l][r]
+      ld_tile_sum(S2, Bb, Zb, ldb, k0, c0, kb, nc);                        // Y_k + Z_k
       __syncthreads();
-      mm64(S1, S2, acc);                                                    // Y_k = Linv_kk B_k
-      __syncthreads();                                                      // S2 is reloaded below
-#pragma unroll
-      for (int p = 0; p < 2; ++p)
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-          S3[ry + p][cx + q] = acc[p][q] + ((ry + p < kb && cx + q < nc)
-                                                ? __ldcg(Zb + (long long)(k0 + ry + p) * ldb + c0 + cx + q) : R(0));
-      ld_tile(S2, Lb + (long long)k * NB * NB, NB, 0, 0, NB, NB, true);      // S2[r][l] = Linv[l][r]
-      __syncthreads();
-      mm64(S2, S3, acc);                                                    // X_k = Linv^T (Y_k + Z_k)
-      __syncthreads();
-      if (i == k) {
-#pragma unroll
-        for (int p = 0; p < 2; ++p)
-#pragma unroll
-          for (int q = 0; q < 4; ++q)
-            if (ry + p < kb && cx + q < nc) Xb[(long long)(k0 + ry + p) * ldb + c0 + cx + q] = acc[p][q];
-      } else {
-#pragma unroll
-        for (int p = 0; p < 2; ++p)
-#pragma unroll
-          for (int q = 0; q < 4; ++q) S3[ry + p][cx + q] = acc[p][q];
-        const int i0 = i * NB;
-        ld_tile(S1, Ab, t, k0, i0, kb, NB, true);                            // S1[r][l] = L_ki[l][r]
-        __syncthreads();
-        mm64(S1, S3, acc);                                                  // L_ki^T X_k
-#pragma unroll
-        for (int p = 0; p < 2; ++p)
-#pragma unroll
-          for (int q = 0; q < 4; ++q)
-            if (cx + q < nc) {
-              R* zp = Zb + (long long)(i0 + ry + p) * ldb + c0 + cx + q;
-              *zp = __ldcg(zp) - acc[p][q];
-            }
-      }
+      mm64(S1, S2, acc);
+      st_acc(Xb + (long long)(k0 + ry) * ldb + c0 + cx, ldb, kb - ry, nc - cx, acc);
       __syncthreads();
     }
+  };
+  auto z_tile = [&](int k, int i, int c0) {
+    const int k0 = k * NB, kb = min(NB, t - k0), i0 = i * NB, nc = min(NB, nrhs - c0);
+    ld_tile(S1, Ab, t, k0, i0, kb, NB, false);     // S1[l][r] = L_ki[l][r]
+    ld_tile(S2, Xb, ldb, k0, c0, kb, nc, false);   // X_k
+    __syncthreads();
+    mm64(S1, S2, acc);
+    rmw_sub(Zb + (long long)(i0 + ry) * ldb + c0 + cx, ldb, NB - ry, nc - cx, acc);   // block i < k is full
+    __syncthreads();
+  };
+  if (rank == (nblk - 1) % kCL) form_x(nblk - 1);
+  cluster_sync_all();
+  for (int k = nblk - 1; k >= 1; --k) {
+    if (rank == 0 && tid == 0) ctr[(ep + 1) & 1] = 0;
+    if (rank == (k - 1) % kCL) {
+      for (int c0 = 0; c0 < nrhs; c0 += NB) z_tile(k, k - 1, c0);
+      form_x(k - 1);
+    }
+    const int ntz = (k - 1) * nct;
+    for (;;) {
+      const int g = next_tile();
+      if (g >= ntz) break;
+      z_tile(k, g / nct, (g % nct) * NB);
+    }
+    ++ep;
     cluster_sync_all();
   }
   if (tid == 0 && bad) set_status(stt, ARCKV_ERR_NOT_SPD);
@@ -333,7 +520,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
 template <typename R>
 static int cholesky_solve(int H, int t, R* Gram, R* Linv, R* B, R* Z, R* X, int ldb, int nrhs, long long bbs,
                           float ridge, DevStatus* stt, cudaStream_t st, int tdiv = 0) {
-  const int smem = 3 * kTileF * (int)sizeof(R);
+  const int smem = 3 * kTileF<R> * (int)sizeof(R);
   cudaFuncSetAttribute(chol_cluster_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   chol_cluster_kernel<R><<<kCL * H, kCT, smem, st>>>(Gram, Linv, B, Z, X, t, nrhs, ldb, bbs, (R)ridge,
                                                      (R)(tdiv > 0 ? tdiv : t), stt);
