@@ -56,7 +56,7 @@ __global__ void mass_rhs_kernel(const float* Phi, const float* m, float* rhs, in
 // Z_i -= L_ki^T X_k (i < k).  lam = ridge * trace(Gram) / tdiv is added to the
 // diagonal as each diagonal block is factored (tdiv = t, or the primal size
 // when the dual system is solved).
-constexpr int kCL = 8;
+constexpr int kCL = 4;
 constexpr int kCT = 512;
 // Shared tiles are [NB][NBP] with rows padded to a 16-byte multiple, so that
 // mm64 can read them with vector loads.
@@ -207,9 +207,8 @@ __device__ __forceinline__ void store_diag(Tile<R> L, Tile<R> Li, R* Ab, R* Lb, 
 // invert the factor: L_kk goes into A and L_kk^-1 into Linv[k].
 //   factor:  right-looking and unscaled, one barrier per column: step c
 //            subtracts a_rc a_jc / a_cc from every (r, j) with c < j <= r (the
-//            lower triangle is dealt to the threads); the thread that finishes
-//            a_c+1,c+1 publishes its reciprocal (pad column NB + 1); the column
-//            scaling by sqrt(a_cc) follows in one pass;
+//            lower triangle is dealt to the threads; each forms 1 / a_cc
+//            itself); the column scaling by sqrt(a_cc) follows in one pass;
 //   inverse: each warp forms four columns of L^-1 by forward substitution
 //            (column j of L^-1 solves L x = e_j), reading L^T from Li.
 // Pad rows beyond the matrix (kb < NB) are the identity.
@@ -231,11 +230,9 @@ __device__ void factor_diag(R* Ab, R* Lb, int t, int k, R lam, Tile<R> L, Tile<R
     ej[q] = e < NT ? e - rr * (rr + 1) / 2 : -1;   // -1: no entry (never > c)
   }
   auto pivot_inv = [](R v) { return (v > R(0) && isfinite(v)) ? rcp_r(v) : R(1); };
-  if (tid == 0) L[0][NB + 1] = pivot_inv(L[0][0]);
-  __syncthreads();
   for (int c = 0; c < NB - 1; ++c) {
     R a[NQ], b[NQ], d[NQ];
-    const R pinv = L[c][NB + 1];
+    const R pinv = pivot_inv(L[c][c]);
 #pragma unroll
     for (int q = 0; q < NQ; ++q)
       if (ej[q] > c) {
@@ -248,7 +245,6 @@ __device__ void factor_diag(R* Ab, R* Lb, int t, int k, R lam, Tile<R> L, Tile<R
       if (ej[q] > c) {
         const R v = fma_r(-a[q] * pinv, b[q], d[q]);
         L[er[q]][ej[q]] = v;
-        if (er[q] == c + 1 && ej[q] == c + 1) L[c + 1][NB + 1] = pivot_inv(v);
       }
     __syncthreads();
   }
