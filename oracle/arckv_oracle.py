@@ -28,6 +28,8 @@ Readings of points the paper leaves open (each is listed in the design doc):
 * both least-squares fits are solved with a ridge lam = ridge * tr(Gram)/t;
   ridge = 0 is the paper's unregularised solve for beta (Eq. mass_fit).
 * eps_w, b_min, b_max (unstated in Eq. mass_fit) default to e^-20, -20, 20.
+* chunked selection (App. A.3, ``chunk_len`` > 0, T above 10,000) rounds
+  t T_c / T half to even, in exact integer arithmetic.
 
 Parity pins for every function live in ``tests/test_oracle_pins.py``.
 """
@@ -41,7 +43,8 @@ import scipy.linalg
 
 __all__ = [
     "OracleConfig", "indexer_param_count", "rms_normalize", "value_context",
-    "indexer_projections", "indexer_logits", "indexer_pool", "top_t",
+    "indexer_projections", "indexer_logits", "indexer_pool", "top_t", "CHUNK_THRESHOLD",
+    "round_half_even_ratio", "chunk_budgets", "anchor_count", "top_t_chunked",
     "attention_logits", "full_attention", "response_profiles", "response_profiles_literal",
     "assign_to_anchors", "log_mass_weights", "mass_weights_literal", "merge_keys", "fit_beta", "fit_values", "compact_attention",
     "hard_subset_attention", "output_loss", "mass_error", "compact_pair",
@@ -59,6 +62,7 @@ class OracleConfig:
     b_min: float = -20.0
     b_max: float = 20.0
     G: int = 4
+    chunk_len: int = 0             # App. A.3 fixed chunking (0: global top-t)
 
 
 # ---------------------------------------------------------------- indexer
@@ -130,6 +134,45 @@ def top_t(s: np.ndarray, t: int) -> np.ndarray:
     position), returned in ascending position order."""
     order = np.lexsort((np.arange(s.shape[0]), -s))
     return np.sort(order[:t]).astype(np.int64)
+
+
+CHUNK_THRESHOLD = 10_000   # App. A.3: fixed chunking applies only when T_a > 10,000
+
+
+def round_half_even_ratio(num: int, den: int) -> int:
+    """round(num / den) for integers num >= 0, den > 0, a tie going to the even
+    neighbour; exact integer arithmetic (App. A.3 rounds t T_c / T_a)."""
+    q, r = divmod(int(num), int(den))
+    if 2 * r > den or (2 * r == den and q % 2 == 1):
+        q += 1
+    return q
+
+
+def chunk_budgets(T: int, t: int, chunk_len: int, threshold: int = CHUNK_THRESHOLD):
+    """App. A.3: with fixed chunking enabled (chunk_len > 0) and T_a = T above
+    the threshold, the score vector is cut into contiguous chunks of length
+    chunk_len (the last one shorter) and chunk c keeps
+    t_c = clip_[1, T_c](round(t T_c / T)) anchors.  Returns [(start, T_c, t_c)];
+    a single global chunk when chunking is off or bypassed."""
+    if chunk_len <= 0 or T <= threshold:
+        return [(0, T, t)]
+    out = []
+    for start in range(0, T, chunk_len):
+        Tc = min(chunk_len, T - start)
+        out.append((start, Tc, min(max(round_half_even_ratio(t * Tc, T), 1), Tc)))
+    return out
+
+
+def anchor_count(T: int, t: int, chunk_len: int, threshold: int = CHUNK_THRESHOLD) -> int:
+    """Realized |S| = sum_c t_c (App. A.3: may differ slightly from t)."""
+    return sum(tc for _, _, tc in chunk_budgets(T, t, chunk_len, threshold))
+
+
+def top_t_chunked(s: np.ndarray, t: int, chunk_len: int, threshold: int = CHUNK_THRESHOLD) -> np.ndarray:
+    """App. A.3: the union over chunks of each chunk's local top-t_c (ties ->
+    lower position), in ascending position order."""
+    parts = [start + top_t(s[start:start + Tc], tc) for start, Tc, tc in chunk_budgets(s.shape[0], t, chunk_len, threshold)]
+    return np.concatenate(parts).astype(np.int64)
 
 
 # ------------------------------------------------------- attention / merge
@@ -282,7 +325,7 @@ def compact_pair(K, V, Q, X_rows, W, cfg: OracleConfig, anchors_in: Optional[np.
     if anchors_in is None:
         I = indexer_logits(Q, X_rows, K, V, W, H_I, d_I)
         _, s = indexer_pool(I)
-        S = top_t(s, cfg.t)
+        S = top_t_chunked(s, cfg.t, cfg.chunk_len)
         out["scores"] = s
     else:
         S = np.asarray(anchors_in, dtype=np.int64)

@@ -180,6 +180,55 @@ def test_top_t_brute_force_and_ties():
     assert list(oracle.top_t(np.array([1.0, 3.0, 3.0, 3.0]), 2)) == [1, 2]
 
 
+def test_chunk_budgets_closed_forms():
+    """App. A.3 budgets t_c = clip_[1,T_c](round(t T_c / T_a)), ties to even,
+    chunking only above T_a = 10,000."""
+    # the 32K and 128K workloads: 1638 / 4 = 409.5 -> 410 (even); 13107 / 16 = 819.19 -> 819
+    assert [tc for _, _, tc in oracle.chunk_budgets(32768, 1638, 8192)] == [410] * 4
+    assert oracle.anchor_count(32768, 1638, 8192) == 1640
+    assert oracle.anchor_count(131072, 13107, 8192) == 16 * 819
+    # exact halves go to the even neighbour: 2.5 -> 2, 3.5 -> 4
+    assert oracle.chunk_budgets(20000, 5, 10000) == [(0, 10000, 2), (10000, 10000, 2)]
+    assert oracle.chunk_budgets(20000, 7, 10000) == [(0, 10000, 4), (10000, 10000, 4)]
+    # ragged last chunk: 819.2 -> 819 twice, 361.6 -> 362
+    assert oracle.chunk_budgets(20000, 2000, 8192) == [(0, 8192, 819), (8192, 8192, 819), (16384, 3616, 362)]
+    # clip to at least one anchor per chunk
+    assert oracle.chunk_budgets(30000, 1, 8192) == [(0, 8192, 1), (8192, 8192, 1), (16384, 8192, 1), (24576, 5424, 1)]
+    # bypass at or below the threshold, and when chunking is off
+    assert oracle.chunk_budgets(10000, 100, 4096) == [(0, 10000, 100)]
+    assert oracle.chunk_budgets(50000, 100, 0) == [(0, 50000, 100)]
+    assert oracle.round_half_even_ratio(5, 2) == 2 and oracle.round_half_even_ratio(7, 2) == 4
+    assert oracle.round_half_even_ratio(0, 3) == 0 and oracle.round_half_even_ratio(5, 3) == 2
+
+
+def test_top_t_chunked_brute_force_and_ties():
+    """Each chunk keeps exactly t_c positions: its t_c largest scores, equal
+    scores to the lower position; the union is ascending."""
+    rng = np.random.default_rng(5)
+    for T, L, t in ((10500, 1000, 350), (12001, 4096, 1200), (10001, 3000, 7)):
+        s = rng.integers(0, 40, size=T).astype(float)   # many exact ties
+        S = oracle.top_t_chunked(s, t, L)
+        assert np.all(np.diff(S) > 0)
+        total = 0
+        for start in range(0, T, L):
+            Tc = min(L, T - start)
+            inside = S[(S >= start) & (S < start + Tc)] - start
+            ranked = sorted(range(Tc), key=lambda j: (-s[start + j], j))
+            assert list(inside) == sorted(ranked[:len(inside)])
+            num, den = t * Tc, T
+            if 2 * (num % den) != den:   # not an exact half: the nearest integer, clipped
+                assert len(inside) == min(max((2 * num + den) // (2 * den), 1), Tc)
+            total += len(inside)
+        assert total == len(S) == oracle.anchor_count(T, t, L)
+
+
+def test_top_t_chunked_reduces_to_global():
+    rng = np.random.default_rng(6)
+    s = rng.standard_normal(12000)
+    assert np.array_equal(oracle.top_t_chunked(s, 900, 12000), oracle.top_t(s, 900))   # one chunk
+    assert np.array_equal(oracle.top_t_chunked(s[:9000], 900, 2048), oracle.top_t(s[:9000], 900))   # bypass
+
+
 # ------------------------------------------------------- attention / merge
 
 def test_full_attention_two_keys_closed_form():
