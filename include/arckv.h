@@ -74,8 +74,15 @@ typedef enum {
  *   d_x   reference-activation width (multiple of 8)
  *   H_I   index heads (1..16), d_I index-head width (must be 128),
  *   d_A   value-attention width (must be 128)                       (App. A.1)
- *   t     anchors per head, 1 <= t <= T                             (Sec. 3.1)
- *   chunk_len  0 = global top-t (the only mode implemented)          (App. A.3)
+ *   t     anchor budget per head, 1 <= t <= T                       (Sec. 3.1)
+ *   chunk_len  >= 0; 0 = one global top-t.  With chunk_len > 0 and T above
+ *         10,000 the scores are cut into contiguous chunks of chunk_len (the
+ *         last one shorter, at most 65535 chunks) and chunk c keeps its top
+ *         t_c = clip_[1, T_c](round(t T_c / T)) positions, rounding exactly
+ *         with halves to even; S is their union.  The realized anchor count
+ *         t' = sum_c t_c (arckv_anchor_count) may differ slightly from t, and
+ *         every [t] extent below is then t'.  Assignment, merge and fits stay
+ *         global over the whole cache.                              (App. A.3)
  * Scalars:
  *   lambda_m  key-merging coefficient in [0, 1]                      (Eq. key_merge)
  *   logit_scale  factor on every model-attention logit q.k; the paper writes
@@ -113,7 +120,7 @@ typedef struct {
  * Optional inputs / outputs of arckv_compact (the pointer itself may be NULL;
  * every field may be NULL).
  *   scores     out fp32 [H_kv][T]  pooled indexer scores s (Eq. indexer_pooling)
- *   anchors    out int32 [H_kv][t] anchor positions S, ascending
+ *   anchors    out int32 [H_kv][t] anchor positions S, ascending (t = t', above)
  *   assign     out int32 [H_kv][T] group index kappa(j) in [0, t)
  *   anchors_in in  int32 [H_kv][t] strictly ascending positions in [0, T):
  *              replaces indexer scoring and selection (the hard branch of
@@ -138,6 +145,11 @@ typedef struct {
 /* Workspace bytes arckv_compact needs for `cfg` (0 if cfg is invalid).
  * Host-only; no CUDA call. */
 size_t arckv_workspace_bytes(const arckv_config* cfg);
+
+/* Realized anchors per head t' (App. A.3): t without chunking, else the sum
+ * of the per-chunk budgets; 0 if cfg is invalid.  Host-only; no CUDA call.
+ * C_k, beta, C_v, anchors and anchors_in have t' rows per head. */
+int32_t arckv_anchor_count(const arckv_config* cfg);
 
 /*
  * Compact one layer (all H_kv heads).

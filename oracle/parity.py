@@ -5,7 +5,8 @@ Tolerances (applied by the tests, stated here once):
     relative error <= 1e-3 on the oracle's top-2t scores;
   * anchor sets: identical, except that positions whose oracle score lies
     within ``band`` (relative to the oracle's t-th largest score) of that
-    threshold may be exchanged for one another (a tie band);
+    threshold may be exchanged for one another (a tie band); with chunked
+    selection the same holds within each chunk at its own t_c-th score;
   * assignment (an argmax whose exact ties are frequent): where the oracle's
     best and second-best similarities differ by more than ``tau`` the GPU
     must agree; elsewhere the GPU's choice must be within ``tau`` of the best;
@@ -46,6 +47,23 @@ def anchors_match(S_gpu: np.ndarray, S: np.ndarray, s: np.ndarray, t: int, band:
         return True, 0, 0.0
     gaps = [abs(s[j] - thr) / thr for j in diff]
     return bool(max(gaps) <= band), len(diff), float(max(gaps))
+
+
+def anchors_match_chunked(S_gpu: np.ndarray, S: np.ndarray, s: np.ndarray, chunks, band: float):
+    """anchors_match within every chunk (start, T_c, t_c) of the chunked
+    selection of App. A.3, the tie band taken at the chunk's own t_c-th score.
+    Returns (ok, exchanged positions, widest relative gap)."""
+    n_ex, widest = 0, 0.0
+    for start, Tc, tc in chunks:
+        def part(X):
+            X = np.asarray(X)
+            return X[(X >= start) & (X < start + Tc)] - start
+        ok, nd, gap = anchors_match(part(S_gpu), part(S), s[start:start + Tc], tc, band)
+        if not ok:
+            return False, nd, gap
+        n_ex += nd
+        widest = max(widest, gap)
+    return len(S_gpu) == len(S), n_ex, widest
 
 
 def assignment_valid(kappa_gpu: np.ndarray, sim: np.ndarray, S: np.ndarray, tau: float):

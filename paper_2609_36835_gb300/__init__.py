@@ -14,7 +14,7 @@ from pathlib import Path
 from typing import Dict, Optional, Sequence
 
 __all__ = [
-    "Config", "ArckvError", "STATUS", "NUM_STAGES", "STAGE_NAMES", "load_library", "workspace_bytes",
+    "Config", "ArckvError", "STATUS", "NUM_STAGES", "STAGE_NAMES", "load_library", "workspace_bytes", "anchor_count",
     "attend_workspace_bytes", "arckv_compact", "arckv_attend", "arckv_query_status", "status_string",
     "compact_layer", "attend", "INDEXER_FIELDS",
 ]
@@ -101,6 +101,8 @@ def load_library():
     P = ctypes.c_void_p
     lib.arckv_workspace_bytes.argtypes = [ctypes.POINTER(_Config)]
     lib.arckv_workspace_bytes.restype = ctypes.c_size_t
+    lib.arckv_anchor_count.argtypes = [ctypes.POINTER(_Config)]
+    lib.arckv_anchor_count.restype = ctypes.c_int32
     lib.arckv_compact.argtypes = [ctypes.POINTER(_Config), P, P, P, P, ctypes.POINTER(_Indexer), P, P, P,
                                   ctypes.POINTER(_Aux), P, ctypes.c_size_t, P]
     lib.arckv_compact.restype = ctypes.c_int
@@ -124,6 +126,12 @@ def status_string(code: int) -> str:
 def workspace_bytes(cfg: Config) -> int:
     c = cfg.c_struct()
     return int(load_library().arckv_workspace_bytes(ctypes.byref(c)))
+
+
+def anchor_count(cfg: Config) -> int:
+    """Realized anchors per head t' (App. A.3 chunking; = cfg.t without it), 0 if invalid."""
+    c = cfg.c_struct()
+    return int(load_library().arckv_anchor_count(ctypes.byref(c)))
 
 
 def attend_workspace_bytes(H_kv: int, n: int, t: int, d: int = 128) -> int:
@@ -201,15 +209,16 @@ def compact_layer(cfg: Config, K, V, Q_ref, X_ref, idx: Dict[str, object], *, ws
         raise ArckvError(2, "arckv_workspace_bytes")
     if ws is None:
         ws = _alloc_ws(need, dev)
+    tp = anchor_count(cfg)
     out = {
-        "C_k": torch.empty(cfg.H_kv, cfg.t, cfg.d, **f32),
-        "beta": torch.empty(cfg.H_kv, cfg.t, **f32),
-        "C_v": torch.empty(cfg.H_kv, cfg.t, cfg.d, **f32),
+        "C_k": torch.empty(cfg.H_kv, tp, cfg.d, **f32),
+        "beta": torch.empty(cfg.H_kv, tp, **f32),
+        "C_v": torch.empty(cfg.H_kv, tp, cfg.d, **f32),
     }
     if want_scores:
         out["scores"] = torch.empty(cfg.H_kv, cfg.T, **f32)
     if want_anchors:
-        out["anchors"] = torch.empty(cfg.H_kv, cfg.t, dtype=torch.int32, device=dev)
+        out["anchors"] = torch.empty(cfg.H_kv, tp, dtype=torch.int32, device=dev)
     if want_assign:
         out["assign"] = torch.empty(cfg.H_kv, cfg.T, dtype=torch.int32, device=dev)
     st, nl = arckv_compact(cfg, K, V, Q_ref, X_ref, idx, out["C_k"], out["beta"], out["C_v"], ws, ws.numel(),

@@ -22,7 +22,9 @@ struct Layout {
 Dims dims_of(const arckv_config& c) {
   Dims D;
   D.H = c.H_kv; D.G = c.G; D.T = c.T; D.d = c.d; D.n_pos = c.n_pos; D.n = c.n_pos * c.G; D.d_x = c.d_x;
-  D.H_I = c.H_I; D.d_I = c.d_I; D.d_A = c.d_A; D.t = c.t; D.HD = c.H_I * c.d_I;
+  D.H_I = c.H_I; D.d_I = c.d_I; D.d_A = c.d_A; D.HD = c.H_I * c.d_I;
+  D.chunk = effective_chunk(c.T, c.chunk_len);
+  D.t = realized_anchors(c.T, c.t, c.chunk_len);   // = t without chunking
   return D;
 }
 
@@ -32,11 +34,14 @@ arckv_status validate(const arckv_config* c) {
   if (c->H_kv < 1 || c->G < 1 || c->T < 1 || c->n_pos < 1 || c->t < 1 || c->t > c->T) return ARCKV_ERR_SHAPE;
   if (c->H_I < 1 || c->H_I > 16 || c->d_x < 8 || (c->d_x % 8) != 0) return ARCKV_ERR_SHAPE;
   if (c->d != 128 || c->d_I != 128 || c->d_A != 128) return ARCKV_ERR_UNSUPPORTED;
-  if (c->chunk_len != 0) return ARCKV_ERR_UNSUPPORTED;
+  if (c->chunk_len < 0) return ARCKV_ERR_INVALID_ARG;
+  const int L = effective_chunk(c->T, c->chunk_len);
+  if (L > 0 && (c->T + (long long)L - 1) / L > 65535) return ARCKV_ERR_SHAPE;   // chunks per head
+  const long long tr = realized_anchors(c->T, c->t, c->chunk_len);
   // per-head element counts index with 32-bit ints inside the kernels
   const long long n = (long long)c->n_pos * c->G;
   if (n > (1 << 24) || (long long)c->T > (1 << 26) || n * c->T >= (1LL << 31) ||
-      (long long)c->t * c->t >= (1LL << 31) || (long long)c->T * c->H_I * 128 >= (1LL << 31) ||
+      (long long)c->t * c->t >= (1LL << 31) || tr * tr >= (1LL << 31) || (long long)c->T * c->H_I * 128 >= (1LL << 31) ||
       (long long)c->H_kv * kSplitK > 65535)
     return ARCKV_ERR_SHAPE;
   if (!(c->lambda_m >= 0.f && c->lambda_m <= 1.f)) return ARCKV_ERR_INVALID_ARG;
@@ -139,6 +144,11 @@ size_t arckv_workspace_bytes(const arckv_config* cfg) {
   return plan(*cfg).total;
 }
 
+int32_t arckv_anchor_count(const arckv_config* cfg) {
+  if (validate(cfg) != ARCKV_OK) return 0;
+  return realized_anchors(cfg->T, cfg->t, cfg->chunk_len);
+}
+
 const char* arckv_status_string(arckv_status s) {
   switch (s) {
     case ARCKV_OK: return "ok";
@@ -220,7 +230,8 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
     nl += nli;
     mark(2);
     nl += launch_index_pool(D, F(L.NT), (const float2*)(w + L.part), F(L.lse), F(L.s), st);
-    nl += launch_top_t(D, F(L.s), anchors, stt, st);
+    nl += launch_top_t(D, cfg->t, F(L.s), anchors, stt, st);
+    nl += launch_check_anchors(D, anchors, stt, st);   // a selection fault becomes a status, not a stray index
   } else {
     mark(1);
     mark(2);

@@ -7,7 +7,29 @@ namespace arckv {
 
 struct Dims {
   int H, G, T, d, n_pos, n, d_x, H_I, d_I, d_A, t, HD;
+  int chunk;   // effective chunk length of the anchor selection (0: one global top-t)
 };
+
+// App. A.3 fixed chunking: with chunk length L > 0 and T_a = T above 10,000
+// the scores are cut into contiguous chunks (the last one shorter) and chunk c
+// keeps t_c = clip_[1, T_c](round(t T_c / T)) anchors, the rounding exact and
+// half to even.  t is then the realized sum of the t_c.
+constexpr int kChunkThreshold = 10000;
+__host__ __device__ inline int chunk_budget(int T, int t, int Tc) {
+  const long long num = (long long)t * Tc;
+  long long q = num / T;
+  const long long r = num % T;
+  if (2 * r > T || (2 * r == T && (q & 1))) ++q;
+  return (int)(q < 1 ? 1 : (q > Tc ? Tc : q));
+}
+inline int effective_chunk(int T, int chunk_len) { return (chunk_len > 0 && T > kChunkThreshold) ? chunk_len : 0; }
+inline int realized_anchors(int T, int t, int chunk_len) {
+  const int L = effective_chunk(T, chunk_len);
+  if (L == 0) return t;
+  int total = 0;
+  for (int start = 0; start < T; start += L) total += chunk_budget(T, t, T - start < L ? T - start : L);
+  return total;
+}
 
 constexpr int kSplitK = 8;   // K slices of the skinny (N = 128) long-K products
 constexpr int kCholNB = 64;  // Cholesky block size
@@ -46,7 +68,8 @@ int launch_index_logits(const Dims& D, const bf16* qbar_hi, const bf16* qbar_lo,
 int launch_index_pool(const Dims& D, const float* I, const float2* part, float* lse, float* s, cudaStream_t st);
 
 // ---- selection (Eq. persistent_support) ----------------------------------
-int launch_top_t(const Dims& D, const float* s, int* anchors, DevStatus* stt, cudaStream_t st);
+// t_budget: the configured t (the per-chunk budgets derive from it); D.t is the realized count
+int launch_top_t(const Dims& D, int t_budget, const float* s, int* anchors, DevStatus* stt, cudaStream_t st);
 int launch_check_anchors(const Dims& D, int* anchors, DevStatus* stt, cudaStream_t st);
 
 // ---- reference attention, assignment, merge (Sec. 3.4) ------------------

@@ -31,16 +31,24 @@ __device__ __forceinline__ int block_excl_scan_1024(int v, int* sc, int& total) 
   return off + x - v;
 }
 
-// One 1024-thread CTA per head.  MSB-first radix select (8-bit digits) of the
-// t-th largest score on the ordered bit patterns, then an order-preserving
-// compaction: every position with a larger score, plus the lowest-position
-// ones among those equal to the threshold (ties -> lower position), written
-// in ascending position order.
-__global__ void __launch_bounds__(1024) top_t_kernel(const float* s, int T, int t, int* anchors,
+// One 1024-thread CTA per (chunk, head).  MSB-first radix select (8-bit
+// digits) of the t_c-th largest score of the chunk on the ordered bit
+// patterns, then an order-preserving compaction: every position with a larger
+// score, plus the lowest-position ones among those equal to the threshold
+// (ties -> lower position), written in ascending position order after the
+// anchors of the chunks before it.  L = 0: one chunk, the whole cache, t_c = t.
+__global__ void __launch_bounds__(1024) top_t_kernel(const float* s, int Tall, int tb, int L, int tp, int* anchors,
                                                      DevStatus* stt) {
-  const int b = blockIdx.x, tid = threadIdx.x;
-  const float* sb = s + (long long)b * T;
-  int* out = anchors + (long long)b * t;
+  const int b = blockIdx.y, c = blockIdx.x, tid = threadIdx.x;
+  int cstart = 0, T = Tall, t = tb, off = 0;   // chunk start, length, budget, output offset
+  if (L > 0) {
+    cstart = c * L;
+    T = min(L, Tall - cstart);
+    t = chunk_budget(Tall, tb, T);
+    for (int q = 0; q < c; ++q) off += chunk_budget(Tall, tb, min(L, Tall - q * L));
+  }
+  const float* sb = s + (long long)b * Tall + cstart;
+  int* out = anchors + (long long)b * tp + off;
   __shared__ int hist[256];
   __shared__ int sc[32];
   __shared__ unsigned int sh_prefix;
@@ -81,15 +89,16 @@ __global__ void __launch_bounds__(1024) top_t_kernel(const float* s, int T, int 
     const int eqrank = block_excl_scan_1024(eq, sc, eqtot) + eqseen;
     const int take = (j < T && (key > prefix || (eq && eqrank < rem))) ? 1 : 0;
     const int pos = block_excl_scan_1024(take, sc, tot) + base;
-    if (take && pos < t) out[pos] = j;
+    if (take && pos < t) out[pos] = cstart + j;
     base += tot;
     eqseen += eqtot;
   }
   if (tid == 0 && base != t) set_status(stt, ARCKV_ERR_INVALID_ARG);
 }
 
-int launch_top_t(const Dims& D, const float* s, int* anchors, DevStatus* stt, cudaStream_t st) {
-  top_t_kernel<<<D.H, 1024, 0, st>>>(s, D.T, D.t, anchors, stt);
+int launch_top_t(const Dims& D, int t_budget, const float* s, int* anchors, DevStatus* stt, cudaStream_t st) {
+  const int nch = D.chunk > 0 ? cdiv(D.T, D.chunk) : 1;
+  top_t_kernel<<<dim3(nch, D.H), 1024, 0, st>>>(s, D.T, D.chunk > 0 ? t_budget : D.t, D.chunk, D.t, anchors, stt);
   return 1;
 }
 

@@ -4,8 +4,10 @@ the host before anything is enqueued."""
 import re
 from pathlib import Path
 
+import numpy as np
 import pytest
 
+import oracle
 import synth
 import paper_2609_36835_gb300 as pk
 from paper_2609_36835_gb300 import workload
@@ -48,20 +50,43 @@ def test_workspace_bytes_sizes_and_rejections(lib):
     assert pk.workspace_bytes(_cfg(t=9000)) == 0           # t > T
     assert pk.workspace_bytes(_cfg(t=0)) == 0
     assert pk.workspace_bytes(_cfg(d=64)) == 0             # unsupported head dim
-    assert pk.workspace_bytes(_cfg(chunk_len=8192)) == 0   # chunked selection not built
+    assert pk.workspace_bytes(_cfg(chunk_len=4096)) == ws  # T = 8192 <= 10,000: chunking is bypassed
     assert pk.attend_workspace_bytes(8, 1024, 819) > 0
     assert pk.attend_workspace_bytes(8, 1024, 0) == 0
 
 
 @pytest.mark.parametrize("kw,code", [
     (dict(t=9000), 2), (dict(T=0), 2), (dict(H_I=17), 2), (dict(d_x=4095), 2), (dict(d=64), 8),
-    (dict(chunk_len=4096), 8), (dict(lambda_m=1.5), 1), (dict(ridge_w=-1.0), 1), (dict(eps_w=0.0), 1),
+    (dict(chunk_len=-1), 1), (dict(T=1 << 20, chunk_len=8), 2), (dict(lambda_m=1.5), 1), (dict(ridge_w=-1.0), 1), (dict(eps_w=0.0), 1),
     (dict(b_min=3.0, b_max=2.0), 1), (dict(flags=0x80), 1),
 ])
 def test_compact_rejects_bad_config_without_gpu(lib, kw, code):
     idx = {f: 1 for f in pk.INDEXER_FIELDS}
     st, nl = pk.arckv_compact(_cfg(**kw), 1, 1, 1, 1, idx, 1, 1, 1, 256, 1 << 40, stream=0)
     assert st == code and nl == 0
+
+
+def test_anchor_count_matches_the_oracle_budgets(lib):
+    """Realized anchors per head (App. A.3), integer-exact against the oracle."""
+    w32 = synth.WORKLOADS["llama8b_T32768_r05"]
+    assert pk.anchor_count(workload.layer_config(w32, 8, chunk_len=8192)) == 1640
+    assert pk.anchor_count(workload.layer_config(w32, 8)) == 1638
+    w128 = synth.WORKLOADS["llama8b_T131072_r10"]
+    assert pk.anchor_count(workload.layer_config(w128, 8, chunk_len=8192)) == 13104
+    assert pk.anchor_count(_cfg(chunk_len=4096)) == 819          # bypassed at T = 8192
+    assert pk.anchor_count(_cfg(t=0)) == 0
+    rng = np.random.default_rng(0)
+    for _ in range(200):
+        T = int(rng.integers(10001, 200000))
+        L = int(rng.integers(512, 40000))
+        t = int(rng.integers(1, min(T // 4, 30000)))   # t^2 < 2^31 keeps the config valid
+        assert pk.anchor_count(_cfg(T=T, t=t, chunk_len=L)) == oracle.anchor_count(T, t, L), (T, t, L)
+    # exact halves go to the even neighbour
+    assert pk.anchor_count(_cfg(T=20000, t=5, chunk_len=10000)) == 4
+    assert pk.anchor_count(_cfg(T=20000, t=7, chunk_len=10000)) == 8
+    ws_c = pk.workspace_bytes(workload.layer_config(w32, 8, chunk_len=8192))
+    ws_g = pk.workspace_bytes(workload.layer_config(w32, 8))
+    assert ws_c > ws_g > 0   # two more anchors per head
 
 
 def test_compact_rejects_null_pointers_and_small_workspace(lib):

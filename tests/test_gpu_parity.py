@@ -31,7 +31,7 @@ def _gpu(lib):
 def _ocfg(cfg: pk.Config):
     return oracle.OracleConfig(t=cfg.t, lambda_m=cfg.lambda_m, scale=(cfg.logit_scale or None),
                                ridge_w=cfg.ridge_w, ridge_v=cfg.ridge_v, eps_w=cfg.eps_w, b_min=cfg.b_min,
-                               b_max=cfg.b_max, G=cfg.G)
+                               b_max=cfg.b_max, G=cfg.G, chunk_len=cfg.chunk_len)
 
 
 def _pair64(arr, h, G):
@@ -66,7 +66,9 @@ def check_layer(w, heads, sample, T=None, n_pos=None, t=None, layer=0, n_hold=64
         refs[h] = ref
         e_inf, e_top = parity.score_errors(_np(out["scores"][h]).astype(np.float64), ref["scores"], cfg.t)
         assert e_inf <= 1e-3 and e_top <= 1e-3, ("scores", h, e_inf, e_top)
-        ok, nd, gap = parity.anchors_match(_np(out["anchors"][h]), ref["anchors"], ref["scores"], cfg.t, BAND)
+        chunks = oracle.chunk_budgets(cfg.T, cfg.t, cfg.chunk_len)
+        assert out["anchors"].shape[1] == len(ref["anchors"]) == sum(tc for _, _, tc in chunks)
+        ok, nd, gap = parity.anchors_match_chunked(_np(out["anchors"][h]), ref["anchors"], ref["scores"], chunks, BAND)
         assert ok, ("anchors", h, nd, gap)
     # downstream stages on the oracle's decisions (other heads keep the GPU's own)
     S_in = out["anchors"].clone()
@@ -130,6 +132,24 @@ def test_long_context_128k_sampled_head():
     """The 128K workload (T = 131072, n = 2048, t = 13107 > n, dual-form fits)
     on one KV head of layer 31."""
     check_layer(synth.WORKLOADS["llama8b_T131072_r10"], [7], [0], layer=31, n_hold=32)
+
+
+def test_chunked_selection_32k_sampled_head():
+    """App. A.3 chunked selection on the 32K workload: four 8192-chunks keep
+    round(1638 / 4) = 410 anchors each (t' = 1640); merge and fits global."""
+    cfg, *_ = check_layer(synth.WORKLOADS["llama8b_T32768_r05"], [4], [0], layer=3, n_hold=32, chunk_len=8192)
+    assert pk.anchor_count(cfg) == 1640
+
+
+def test_chunked_selection_ragged_last_chunk():
+    """T = 20000 in chunks of 8192, 8192 and 3616 (budgets 819, 819, 362) on
+    two heads, reference rows off the tile grid."""
+    check_layer(synth.WORKLOADS["llama8b_layer_T8192"], [2, 5], [0, 1], T=20000, n_pos=60, t=2000, chunk_len=8192)
+
+
+def test_chunked_selection_one_anchor_per_chunk():
+    """Budgets clipped up to one anchor per chunk: T = 12000, chunks of 4096, t = 3."""
+    check_layer(synth.WORKLOADS["llama8b_layer_T8192"], [1], [0], T=12000, n_pos=20, t=3, chunk_len=4096)
 
 
 def test_odd_shapes_single_index_head():
