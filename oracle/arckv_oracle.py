@@ -43,7 +43,7 @@ import scipy.linalg
 
 __all__ = [
     "OracleConfig", "indexer_param_count", "rms_normalize", "value_context",
-    "indexer_projections", "indexer_logits", "indexer_pool", "top_t", "CHUNK_THRESHOLD",
+    "indexer_projections", "indexer_logits", "indexer_pool", "top_t", "CHUNK_THRESHOLD", "joint_compact_attention",
     "round_half_even_ratio", "chunk_budgets", "anchor_count", "top_t_chunked",
     "attention_logits", "full_attention", "response_profiles", "response_profiles_literal",
     "assign_to_anchors", "log_mass_weights", "mass_weights_literal", "merge_keys", "fit_beta", "fit_values", "compact_attention",
@@ -290,6 +290,16 @@ def fit_values(Q, K, V, C_k, beta, cfg: OracleConfig, scale: float):
 def compact_attention(Q, C_k, beta, C_v, scale: float) -> np.ndarray:
     """Eq. (compact_attention): O^ = softmax(Q C_k^T + 1 beta^T) C_v."""
     return _softmax_rows(attention_logits(Q, C_k, scale) + beta[None, :]) @ C_v
+
+
+def joint_compact_attention(Q, C_k, beta, C_v, K_fixed, V_fixed, scale: float) -> np.ndarray:
+    """Eq. (concatenated_attention_preservation), right-hand side: attention
+    over the stacked keys [C_k; K_fixed] and values [C_v; V_fixed] with the
+    bias b = [beta; 0_F] on the logits (App. A.7).  Either block may be empty."""
+    keys = np.concatenate([C_k, K_fixed], axis=0)
+    vals = np.concatenate([C_v, V_fixed], axis=0)
+    b = np.concatenate([beta, np.zeros(K_fixed.shape[0])])
+    return _softmax_rows(attention_logits(Q, keys, scale) + b[None, :]) @ vals
 
 
 def hard_subset_attention(Q, K, V, S, scale: float) -> np.ndarray:

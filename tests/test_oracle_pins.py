@@ -446,6 +446,38 @@ def test_compact_attention_reduces_to_full_and_hard_subset():
     assert np.allclose(oracle.compact_attention(Q, K, b, V, SC), O2, rtol=1e-12)
 
 
+def test_joint_attention_concatenation_and_bias():
+    """App. A.7: with C_k = K_A, beta = 0, C_v = V_A the joint right-hand side
+    is full attention over the stacked cache [K_A; K_f]; a compact key with
+    beta = log 2 stands for two copies of itself; empty blocks reduce to the
+    compact operator and to plain attention."""
+    rng = np.random.default_rng(7)
+    KA, VA = rng.standard_normal((9, 16)), rng.standard_normal((9, 16))
+    Kf, Vf = rng.standard_normal((5, 16)), rng.standard_normal((5, 16))
+    Q = rng.standard_normal((4, 16))
+    sc = 0.3
+    _, O_full = oracle.full_attention(Q, np.vstack([KA, Kf]), np.vstack([VA, Vf]), sc)
+    assert np.allclose(oracle.joint_compact_attention(Q, KA, np.zeros(9), VA, Kf, Vf, sc), O_full, rtol=1e-12, atol=1e-12)
+    # duplicate key 2 of the compact block: beta_2 = log 2 on a single copy
+    Kdup, Vdup = np.vstack([KA, KA[2:3], Kf]), np.vstack([VA, VA[2:3], Vf])
+    _, O_dup = oracle.full_attention(Q, Kdup, Vdup, sc)
+    beta = np.zeros(9)
+    beta[2] = np.log(2.0)
+    assert np.allclose(oracle.joint_compact_attention(Q, KA, beta, VA, Kf, Vf, sc), O_dup, rtol=1e-12, atol=1e-12)
+    # explicit loops: o_i = sum_j e^{a_ij} v_j / sum_j e^{a_ij}
+    O_loop = np.zeros((4, 16))
+    for i in range(4):
+        a = [sc * Q[i] @ KA[j] + beta[j] for j in range(9)] + [sc * Q[i] @ Kf[j] for j in range(5)]
+        e = np.exp(np.array(a) - max(a))
+        O_loop[i] = (e[:9] @ VA + e[9:] @ Vf) / e.sum()
+    assert np.allclose(oracle.joint_compact_attention(Q, KA, beta, VA, Kf, Vf, sc), O_loop, rtol=1e-12, atol=1e-12)
+    e0 = np.zeros((0, 16))
+    assert np.allclose(oracle.joint_compact_attention(Q, KA, beta, VA, e0, e0, sc),
+                       oracle.compact_attention(Q, KA, beta, VA, sc), rtol=1e-13, atol=1e-13)
+    assert np.allclose(oracle.joint_compact_attention(Q, e0, np.zeros(0), e0, Kf, Vf, sc),
+                       oracle.full_attention(Q, Kf, Vf, sc)[1], rtol=1e-13, atol=1e-13)
+
+
 def test_diagnostics():
     y = np.array([[3.0, 4.0]])
     assert oracle.output_loss(y * 1.1, y) == pytest.approx(0.01, rel=1e-12)
