@@ -63,6 +63,7 @@ typedef enum {
 
 /* Flags (arckv_config.flags). */
 #define ARCKV_FLAG_NONBLOCKING 0x1u /* do not synchronise; see arckv_query_status */
+#define ARCKV_FLAG_COMPACT_BF16 0x2u /* arckv_attend_joint: C_k, C_v are bf16, not fp32 */
 
 /*
  * Problem description for one layer.  Sizes:
@@ -185,6 +186,30 @@ size_t arckv_attend_workspace_bytes(int32_t H_kv, int32_t n, int32_t t, int32_t 
 arckv_status arckv_attend(int32_t H_kv, int32_t n, int32_t t, int32_t d, float logit_scale,
                           const void* Q, const float* C_k, const float* beta, const float* C_v,
                           float* O, void* ws, size_t ws_bytes, uint32_t flags, void* stream);
+
+/* Workspace bytes of arckv_attend_joint (0 if the sizes are invalid). Host-only. */
+size_t arckv_attend_joint_workspace_bytes(int32_t H, int32_t n, int32_t t, int32_t F, int32_t d);
+
+/*
+ * Attention over a compact block followed by an uncompressed block (App. A.7
+ * Eq. concatenated_attention_preservation):
+ *   O[h] = softmax(logit_scale * Q[h] [C_k[h]; K_fixed[h]]^T + [beta[h]; 0_F]) [C_v[h]; V_fixed[h]]
+ * for H independent heads (a decode batch folds into H: head = sequence x KV head).
+ *   Q        bf16 [H][n][d]        n >= 1 query rows per head
+ *   C_k, C_v [H][t][d] fp32, or bf16 with ARCKV_FLAG_COMPACT_BF16; beta fp32 [H][t]
+ *   K_fixed, V_fixed  bf16 [H][F][d]  the uncompressed block (zero bias)
+ *   O        out fp32 [H][n][d]
+ * t >= 0, F >= 0, t + F >= 1, d == 128.  With t == 0 the compact arguments
+ * may be NULL and the call is plain attention over K_fixed / V_fixed (the
+ * full-cache baseline); with F == 0 it is the compact operator of
+ * arckv_attend.  Every array pointer must be 16-byte aligned
+ * (ARCKV_ERR_INVALID_ARG otherwise).  `flags` takes ARCKV_FLAG_NONBLOCKING
+ * and ARCKV_FLAG_COMPACT_BF16; ws as for arckv_attend.
+ */
+arckv_status arckv_attend_joint(int32_t H, int32_t n, int32_t t, int32_t F, int32_t d, float logit_scale,
+                                const void* Q, const void* C_k, const float* beta, const void* C_v,
+                                const void* K_fixed, const void* V_fixed, float* O, void* ws, size_t ws_bytes,
+                                uint32_t flags, void* stream);
 
 /*
  * Allocation-free compact attention.  The paper has no counterpart: this is a

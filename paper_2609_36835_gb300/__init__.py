@@ -16,7 +16,8 @@ from typing import Dict, Optional, Sequence
 __all__ = [
     "Config", "ArckvError", "STATUS", "NUM_STAGES", "STAGE_NAMES", "load_library", "workspace_bytes", "anchor_count",
     "attend_workspace_bytes", "arckv_compact", "arckv_attend", "arckv_query_status", "status_string",
-    "compact_layer", "attend", "INDEXER_FIELDS",
+    "compact_layer", "attend", "INDEXER_FIELDS", "attend_joint", "arckv_attend_joint",
+    "attend_joint_workspace_bytes", "FLAG_COMPACT_BF16",
 ]
 
 _LIB_PATH = Path(__file__).resolve().parent / "libarckv.so"
@@ -28,6 +29,7 @@ STATUS = {
     8: "ARCKV_ERR_UNSUPPORTED",
 }
 FLAG_NONBLOCKING = 0x1
+FLAG_COMPACT_BF16 = 0x2
 NUM_STAGES = 6
 STAGE_NAMES = ("indexer_features", "index_logits", "pool_top_t", "refattn_assign", "merge", "fits")
 INDEXER_FIELDS = ("L_q", "L_k", "L_x", "b_x", "U_q", "U_k", "U_v", "L_c", "L_v")
@@ -111,6 +113,11 @@ def load_library():
     lib.arckv_attend.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_float,
                                  P, P, P, P, P, P, ctypes.c_size_t, ctypes.c_uint32, P]
     lib.arckv_attend.restype = ctypes.c_int
+    lib.arckv_attend_joint_workspace_bytes.argtypes = [ctypes.c_int32] * 5
+    lib.arckv_attend_joint_workspace_bytes.restype = ctypes.c_size_t
+    lib.arckv_attend_joint.argtypes = [ctypes.c_int32] * 5 + [ctypes.c_float] + [P] * 8 + [ctypes.c_size_t,
+                                                                                         ctypes.c_uint32, P]
+    lib.arckv_attend_joint.restype = ctypes.c_int
     lib.arckv_query_status.argtypes = [P, P]
     lib.arckv_query_status.restype = ctypes.c_int
     lib.arckv_status_string.argtypes = [ctypes.c_int]
@@ -184,6 +191,19 @@ def arckv_attend(H_kv: int, n: int, t: int, d: int, logit_scale: float, Q, C_k, 
                                 _ptr(O), _ptr(ws), int(ws_bytes), int(flags), _stream_handle(stream)))
 
 
+def attend_joint_workspace_bytes(H: int, n: int, t: int, F: int, d: int = 128) -> int:
+    return int(load_library().arckv_attend_joint_workspace_bytes(H, n, t, F, d))
+
+
+def arckv_attend_joint(H: int, n: int, t: int, F: int, d: int, logit_scale: float, Q, C_k, beta, C_v, K_fixed,
+                       V_fixed, O, ws, ws_bytes: int, flags: int = 0, stream=None) -> int:
+    """Direct binding of ``arckv_attend_joint``; returns the status code."""
+    lib = load_library()
+    return int(lib.arckv_attend_joint(H, n, t, F, d, float(logit_scale), _ptr(Q), _ptr(C_k), _ptr(beta), _ptr(C_v),
+                                      _ptr(K_fixed), _ptr(V_fixed), _ptr(O), _ptr(ws), int(ws_bytes), int(flags),
+                                      _stream_handle(stream)))
+
+
 def arckv_query_status(ws, stream=None) -> int:
     return int(load_library().arckv_query_status(_ptr(ws), _stream_handle(stream)))
 
@@ -245,4 +265,26 @@ def attend(Q, C_k, beta, C_v, logit_scale: float = 0.0, *, ws=None, stream=None,
     st = arckv_attend(H, n, t, d, logit_scale, Q, C_k, beta, C_v, O, ws, ws.numel(), stream=stream)
     if check and st != 0:
         raise ArckvError(st, "arckv_attend")
+    return O
+
+
+def attend_joint(Q, C_k=None, beta=None, C_v=None, K_fixed=None, V_fixed=None, logit_scale: float = 0.0, *, ws=None,
+                 stream=None, check: bool = True):
+    """O = softmax(scale Q [C_k; K_fixed]^T + [beta; 0]) [C_v; V_fixed] (App. A.7) for Q [H, n, 128] bf16.
+    C_k / C_v fp32 or bf16 (both the same); either block may be omitted."""
+    import torch
+    H, n, d = Q.shape
+    t = 0 if C_k is None else C_k.shape[1]
+    F = 0 if K_fixed is None else K_fixed.shape[1]
+    need = attend_joint_workspace_bytes(H, n, t, F, d)
+    if need == 0:
+        raise ArckvError(2, "arckv_attend_joint_workspace_bytes")
+    if ws is None:
+        ws = _alloc_ws(need, Q.device)
+    flags = FLAG_COMPACT_BF16 if (C_k is not None and C_k.dtype == torch.bfloat16) else 0
+    O = torch.empty(H, n, d, dtype=torch.float32, device=Q.device)
+    st = arckv_attend_joint(H, n, t, F, d, logit_scale, Q, C_k, beta, C_v, K_fixed, V_fixed, O, ws, ws.numel(),
+                            flags=flags, stream=stream)
+    if check and st != 0:
+        raise ArckvError(st, "arckv_attend_joint")
     return O

@@ -317,4 +317,46 @@ arckv_status arckv_attend(int32_t H_kv, int32_t n, int32_t t, int32_t d, float l
   return read_status(ws, st);
 }
 
+size_t arckv_attend_joint_workspace_bytes(int32_t H, int32_t n, int32_t t, int32_t F, int32_t d) {
+  if (H < 1 || n < 1 || t < 0 || F < 0 || (long long)t + F < 1 || d != 128) return 0;
+  if ((long long)t + F >= (1LL << 30) || (long long)H * n >= (1LL << 31) || cdiv(n, 4) > 65535 || H > 65535) return 0;
+  const JointSplit js = joint_split(H, n, t, F);
+  const size_t rows = (size_t)H * js.nsplit * n;
+  return up(sizeof(DevStatus)) + up(rows * 128 * 4) + up(rows * 8);
+}
+
+arckv_status arckv_attend_joint(int32_t H, int32_t n, int32_t t, int32_t F, int32_t d, float logit_scale,
+                                const void* Q, const void* C_k, const float* beta, const void* C_v,
+                                const void* K_fixed, const void* V_fixed, float* O, void* ws, size_t ws_bytes,
+                                uint32_t flags, void* stream) {
+  if (flags & ~(ARCKV_FLAG_NONBLOCKING | ARCKV_FLAG_COMPACT_BF16)) return ARCKV_ERR_INVALID_ARG;
+  if (d != 128) return ARCKV_ERR_UNSUPPORTED;
+  const size_t need = arckv_attend_joint_workspace_bytes(H, n, t, F, d);
+  if (need == 0) return ARCKV_ERR_SHAPE;
+  if (!Q || !O || (t > 0 && (!C_k || !beta || !C_v)) || (F > 0 && (!K_fixed || !V_fixed)))
+    return ARCKV_ERR_INVALID_ARG;
+  // rows are read as 16-byte vectors
+  auto misaligned = [](const void* p) { return p && ((uintptr_t)p % 16) != 0; };
+  if (misaligned(C_k) || misaligned(C_v) || misaligned(K_fixed) || misaligned(V_fixed) || misaligned(O))
+    return ARCKV_ERR_INVALID_ARG;
+  if (!(logit_scale >= 0.f) || !isfinite(logit_scale)) return ARCKV_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < need || ((uintptr_t)ws % kAlign) != 0) return ARCKV_ERR_WORKSPACE;
+  cudaStream_t st = (cudaStream_t)stream;
+  char* w = (char*)ws;
+  DevStatus* stt = (DevStatus*)w;
+  const JointSplit js = joint_split(H, n, t, F);
+  const size_t rows = (size_t)H * js.nsplit * n;
+  float* Opart = (float*)(w + up(sizeof(DevStatus)));
+  float2* ml = (float2*)(w + up(sizeof(DevStatus)) + up(rows * 128 * 4));
+  const float scale = logit_scale > 0.f ? logit_scale : 1.0f / sqrtf((float)d);
+  cudaGetLastError();
+  if (cudaMemsetAsync(stt, 0, sizeof(DevStatus), st) != cudaSuccess) return ARCKV_ERR_CUDA;
+  launch_attend_joint(H, n, t, F, scale, (const bf16*)Q, C_k, beta, C_v, (flags & ARCKV_FLAG_COMPACT_BF16) != 0,
+                      (const bf16*)K_fixed, (const bf16*)V_fixed, O, Opart, ml, st);
+  launch_check_finite(O, (long long)H * n * d, stt, st);
+  if (cudaGetLastError() != cudaSuccess) return ARCKV_ERR_CUDA;
+  if (flags & ARCKV_FLAG_NONBLOCKING) return ARCKV_OK;
+  return read_status(ws, st);
+}
+
 }  // extern "C"

@@ -1,0 +1,286 @@
+// Attention over a compact block followed by an uncompressed block (App. A.7
+// Eq. concatenated_attention_preservation):
+//
+//   O_i = sum_j e^{a_ij} v_j / sum_j e^{a_ij},   a_ij = scale q_i.k_j + b_j,
+//   k, v, b = [C_k; K_fixed], [C_v; V_fixed], [beta; 0_F]
+//
+// for H independent heads of n query rows (a decode batch folds into H).
+// The operation streams every key and value once and does ~2 FMA per byte of
+// bf16 cache: it is HBM-bound, so it runs on the SIMT pipes as a split-key
+// ("flash-decoding") pass, not as a GEMM:
+//   attend_split_kernel: CTA (key split, 4-row block, head); per 64-key tile
+//     - logits: thread (key tid/4, 32-dim quarter tid%4) loads its slice of the
+//       key straight from HBM (16-byte vectors, a warp reads 8 whole rows),
+//       dots it with the 4 query rows held in shared memory, and the 4
+//       quarters are combined with two shuffles;
+//     - online softmax per row (running max m, running sum l);
+//     - values: warp w takes keys w, w+8, ... of the tile, lane l dims
+//       4l..4l+3, so a warp reads whole value rows; the accumulators are
+//       rescaled by e^{m_old - m_new};
+//   attend_combine_kernel: per (head, row) merges the splits' (m, l, o).
+// t = 0 gives plain attention over the uncompressed block (the full-cache
+// baseline of the decode measurement); F = 0 the compact operator of Sec. 3.1.
+#include <algorithm>
+
+#include "kernels.h"
+
+namespace arckv {
+
+constexpr int kJR = 4;        // query rows per CTA
+constexpr int kJTile = 64;    // keys per tile
+constexpr int kJThreads = 256;
+
+__device__ __forceinline__ void load32(const float* p, float (&x)[32]) {
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    const float4 v = __ldg((const float4*)p + q);
+    x[4 * q] = v.x; x[4 * q + 1] = v.y; x[4 * q + 2] = v.z; x[4 * q + 3] = v.w;
+  }
+}
+__device__ __forceinline__ void load32(const bf16* p, float (&x)[32]) {
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const uint4 v = __ldg((const uint4*)p + q);
+    const __nv_bfloat162* h = (const __nv_bfloat162*)&v;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float2 f = __bfloat1622float2(h[e]);
+      x[8 * q + 2 * e] = f.x;
+      x[8 * q + 2 * e + 1] = f.y;
+    }
+  }
+}
+__device__ __forceinline__ void load4(const float* p, float (&x)[4]) {
+  const float4 v = __ldg((const float4*)p);
+  x[0] = v.x; x[1] = v.y; x[2] = v.z; x[3] = v.w;
+}
+__device__ __forceinline__ void load4(const bf16* p, float (&x)[4]) {
+  const uint2 v = __ldg((const uint2*)p);
+  const float2 a = __bfloat1622float2(*(const __nv_bfloat162*)&v.x), b = __bfloat1622float2(*(const __nv_bfloat162*)&v.y);
+  x[0] = a.x; x[1] = a.y; x[2] = b.x; x[3] = b.y;
+}
+
+// sum_q qv[q] k[q] over a 32-dim slice held as loaded (fp32, or packed bf16 pairs)
+struct KSlice32F {
+  float x[32];
+  __device__ __forceinline__ void load(const float* p) { load32(p, x); }
+  __device__ __forceinline__ void zero() {
+#pragma unroll
+    for (int q = 0; q < 32; ++q) x[q] = 0.f;
+  }
+  __device__ __forceinline__ float dot(const float4* qv) const {
+    float a = 0.f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const float4 y = qv[q];
+      a = fmaf(y.x, x[4 * q], a);
+      a = fmaf(y.y, x[4 * q + 1], a);
+      a = fmaf(y.z, x[4 * q + 2], a);
+      a = fmaf(y.w, x[4 * q + 3], a);
+    }
+    return a;
+  }
+};
+struct KSlice32H {
+  uint4 x[4];
+  __device__ __forceinline__ void load(const bf16* p) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) x[q] = __ldg((const uint4*)p + q);
+  }
+  __device__ __forceinline__ void zero() {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) x[q] = make_uint4(0u, 0u, 0u, 0u);
+  }
+  __device__ __forceinline__ float dot(const float4* qv) const {
+    float a = 0.f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const __nv_bfloat162* h = (const __nv_bfloat162*)&x[q];
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const float2 f0 = __bfloat1622float2(h[2 * e]), f1 = __bfloat1622float2(h[2 * e + 1]);
+        const float4 y = qv[2 * q + e];
+        a = fmaf(y.x, f0.x, a);
+        a = fmaf(y.y, f0.y, a);
+        a = fmaf(y.z, f1.x, a);
+        a = fmaf(y.w, f1.y, a);
+      }
+    }
+    return a;
+  }
+};
+template <typename TC> struct KSliceOf { using type = KSlice32F; };
+template <> struct KSliceOf<bf16> { using type = KSlice32H; };
+
+// The tiles of keys [jlo, jhi) of one block: key j is row j - koff of Kb / Vb,
+// with bias[j] (bias == nullptr: zero).  Updates the running (m, l) in sM / sL
+// and the per-thread accumulators acc.
+template <typename KT>
+__device__ __forceinline__ void attend_tiles(const KT* Kb, const KT* Vb, const float* bias, int jlo, int jhi,
+                                             int koff, float (*sQ)[128], float (*sP)[kJTile], float* sM, float* sL,
+                                             float* sF, float (&acc)[kJR][4]) {
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  for (int j0 = jlo; j0 < jhi; j0 += kJTile) {
+    {  // logits of the tile
+      const int jj = tid >> 2, p = tid & 3, j = j0 + jj;
+      typename KSliceOf<KT>::type k;
+      if (j < jhi) k.load(Kb + (long long)(j - koff) * 128 + p * 32);
+      else k.zero();
+      float part[kJR];
+#pragma unroll
+      for (int r = 0; r < kJR; ++r) {
+        float a = k.dot((const float4*)&sQ[r][p * 32]);
+        a += __shfl_xor_sync(0xffffffffu, a, 1);
+        a += __shfl_xor_sync(0xffffffffu, a, 2);
+        part[r] = a;
+      }
+      if (p == 0) {
+        const float b = (j < jhi && bias) ? __ldg(bias + j) : 0.f;
+#pragma unroll
+        for (int r = 0; r < kJR; ++r) sP[r][jj] = (j < jhi) ? part[r] + b : -INFINITY;
+      }
+    }
+    __syncthreads();
+    if (w < kJR) {  // online softmax of row w over the tile (at least one key is valid)
+      const float a0 = sP[w][lane], a1 = sP[w][lane + 32];
+      const float mold = sM[w], mnew = fmaxf(mold, warp_max(fmaxf(a0, a1)));
+      const float e0 = expf(a0 - mnew), e1 = expf(a1 - mnew);
+      sP[w][lane] = e0;
+      sP[w][lane + 32] = e1;
+      const float ssum = warp_sum(e0 + e1);
+      if (lane == 0) {
+        const float f = expf(mold - mnew);   // 0 on the first tile (mold = -inf)
+        sF[w] = f;
+        sL[w] = sL[w] * f + ssum;
+        sM[w] = mnew;
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int r = 0; r < kJR; ++r) {
+      const float f = sF[r];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) acc[r][q] *= f;
+    }
+#pragma unroll 4
+    for (int i = 0; i < kJTile / 8; ++i) {
+      const int jj = w + 8 * i, j = j0 + jj;
+      if (j < jhi) {
+        float v[4];
+        load4(Vb + (long long)(j - koff) * 128 + lane * 4, v);
+#pragma unroll
+        for (int r = 0; r < kJR; ++r) {
+          const float pr = sP[r][jj];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) acc[r][q] = fmaf(pr, v[q], acc[r][q]);
+        }
+      }
+    }
+    __syncthreads();
+  }
+}
+
+// Partial results of key split sp: Opart[h][sp][i][:] = sum_j e^{a_ij - m} v_j
+// (unnormalised) and ml[h][sp][i] = (m, l = sum_j e^{a_ij - m}).  The split's
+// key range is cut at t so that every tile holds one block's keys.
+template <typename TC>
+__global__ void __launch_bounds__(kJThreads, 3) attend_split_kernel(const bf16* Q, int n, const TC* Ck, const float* beta,
+                                                                    const TC* Cv, int t, const bf16* Kf, const bf16* Vf,
+                                                                    int F, float scale, int per_split, int nsplit,
+                                                                    float* Opart, float2* ml) {
+  const int h = blockIdx.z, r0 = blockIdx.y * kJR, sp = blockIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  const int L = t + F, jb = sp * per_split, je = min(L, jb + per_split);
+  __shared__ __align__(16) float sQ[kJR][128];
+  __shared__ float sP[kJR][kJTile];
+  __shared__ float sM[kJR], sL[kJR], sF[kJR];
+  __shared__ __align__(16) float sAcc[kJThreads / 32][kJR][128];
+  for (int e = tid; e < kJR * 128; e += kJThreads) {
+    const int r = e >> 7, dd = e & 127;
+    sQ[r][dd] = (r0 + r < n) ? scale * __bfloat162float(Q[((long long)h * n + r0 + r) * 128 + dd]) : 0.f;
+  }
+  if (tid < kJR) {
+    sM[tid] = -INFINITY;
+    sL[tid] = 0.f;
+  }
+  float acc[kJR][4];
+#pragma unroll
+  for (int r = 0; r < kJR; ++r)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) acc[r][q] = 0.f;
+  __syncthreads();
+  if (jb < t)
+    attend_tiles<TC>(Ck + (long long)h * t * 128, Cv + (long long)h * t * 128, beta + (long long)h * t, jb,
+                     min(je, t), 0, sQ, sP, sM, sL, sF, acc);
+  if (je > t)
+    attend_tiles<bf16>(Kf + (long long)h * F * 128, Vf + (long long)h * F * 128, nullptr, max(jb, t), je, t, sQ, sP,
+                       sM, sL, sF, acc);
+#pragma unroll
+  for (int r = 0; r < kJR; ++r) *(float4*)&sAcc[w][r][lane * 4] = make_float4(acc[r][0], acc[r][1], acc[r][2], acc[r][3]);
+  __syncthreads();
+  for (int e = tid; e < kJR * 128; e += kJThreads) {
+    const int r = e >> 7, dd = e & 127;
+    if (r0 + r >= n) continue;
+    float o = 0.f;
+#pragma unroll
+    for (int q = 0; q < kJThreads / 32; ++q) o += sAcc[q][r][dd];
+    const long long row = ((long long)h * nsplit + sp) * n + r0 + r;
+    Opart[row * 128 + dd] = o;
+    if (dd == 0) ml[row] = make_float2(sM[r], sL[r]);
+  }
+}
+
+// O[h][i] = sum_s e^{m_s - m} Opart_s / sum_s e^{m_s - m} l_s (one warp per row, lane dims 4l..4l+3)
+__global__ void __launch_bounds__(256) attend_combine_kernel(const float* Opart, const float2* ml, int n, int nsplit,
+                                                             long long rows, float* O) {
+  const long long g = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (g >= rows) return;
+  const long long h = g / n, i = g % n;
+  float m = -INFINITY;
+  for (int s = 0; s < nsplit; ++s) m = fmaxf(m, ml[(h * nsplit + s) * n + i].x);
+  float l = 0.f, o0 = 0.f, o1 = 0.f, o2 = 0.f, o3 = 0.f;
+  for (int s = 0; s < nsplit; ++s) {
+    const long long row = (h * nsplit + s) * n + i;
+    const float2 v = ml[row];
+    const float f = expf(v.x - m);
+    l = fmaf(v.y, f, l);
+    const float4 op = *(const float4*)(Opart + row * 128 + lane * 4);
+    o0 = fmaf(f, op.x, o0);
+    o1 = fmaf(f, op.y, o1);
+    o2 = fmaf(f, op.z, o2);
+    o3 = fmaf(f, op.w, o3);
+  }
+  const float inv = 1.0f / l;
+  *(float4*)(O + g * 128 + lane * 4) = make_float4(o0 * inv, o1 * inv, o2 * inv, o3 * inv);
+}
+
+JointSplit joint_split(int H, int n, int t, int F) {
+  JointSplit s;
+  const int L = t + F, rb = cdiv(n, kJR);
+  const long long ctas = (long long)H * rb;
+  const int want = (int)std::max<long long>(1, (152LL * 8 + ctas - 1) / ctas);   // about 8 CTAs per SM
+  const int ntiles = cdiv(L, kJTile);
+  const int nsp = std::min(want, ntiles);
+  s.per_split = cdiv(ntiles, nsp) * kJTile;
+  s.nsplit = cdiv(L, s.per_split);
+  return s;
+}
+
+int launch_attend_joint(int H, int n, int t, int F, float scale, const bf16* Q, const void* Ck, const float* beta,
+                        const void* Cv, bool compact_bf16, const bf16* Kf, const bf16* Vf, float* O, float* Opart,
+                        float2* ml, cudaStream_t st) {
+  const JointSplit s = joint_split(H, n, t, F);
+  const dim3 grid(s.nsplit, cdiv(n, kJR), H);
+  if (compact_bf16)
+    attend_split_kernel<bf16><<<grid, kJThreads, 0, st>>>(Q, n, (const bf16*)Ck, beta, (const bf16*)Cv, t, Kf, Vf, F,
+                                                          scale, s.per_split, s.nsplit, Opart, ml);
+  else
+    attend_split_kernel<float><<<grid, kJThreads, 0, st>>>(Q, n, (const float*)Ck, beta, (const float*)Cv, t, Kf, Vf,
+                                                           F, scale, s.per_split, s.nsplit, Opart, ml);
+  const long long rows = (long long)H * n;
+  attend_combine_kernel<<<(unsigned)cdiv(rows, 8), 256, 0, st>>>(Opart, ml, n, s.nsplit, rows, O);
+  return 2;
+}
+
+}  // namespace arckv

@@ -106,6 +106,19 @@ int launch_check_finite(const float* x, long long count, DevStatus* stt, cudaStr
 int launch_attend(int H, int n, int t, float scale, const bf16* Q, const float* C_k, const float* beta,
                   const float* C_v, float* O, float* LC, float* split, cudaStream_t st);
 
+// ---- joint attention with an uncompressed block (App. A.7) -------------
+// Key splits of the split-key pass (deterministic in H, n, t, F).
+struct JointSplit {
+  int per_split, nsplit;
+};
+JointSplit joint_split(int H, int n, int t, int F);
+// O [H][n][128] fp32 = softmax(scale Q [C_k; K_f]^T + [beta; 0]) [C_v; V_f];
+// C_k, C_v fp32 or (compact_bf16) bf16 [H][t][128]; K_f, V_f bf16 [H][F][128];
+// scratch Opart [H][nsplit][n][128] fp32 and ml [H][nsplit][n].
+int launch_attend_joint(int H, int n, int t, int F, float scale, const bf16* Q, const void* Ck, const float* beta,
+                        const void* Cv, bool compact_bf16, const bf16* Kf, const bf16* Vf, float* O, float* Opart,
+                        float2* ml, cudaStream_t st);
+
 // Shared small kernels.
 int launch_part_stats(int H, int rows, int ntiles, const float2* part, float* shift, float* mul, float* sum,
                       cudaStream_t st);

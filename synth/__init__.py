@@ -20,6 +20,12 @@ evaluation, which are not available; Sec. 3.1, App. A.1, App. A.5):
 * reference activations x_r: N(0,1)^{d_x}, one per reference position,
   shared by the G query heads of that position and by all KV heads of a layer;
 * held-out queries: same law as the reference queries, separate stream;
+* stand-in compact caches for attention tests (no fit involved): C_k = the
+  keys at a uniformly drawn anchor subset plus N(0, 0.1^2) noise, C_v = the
+  values there, beta ~ U(-2, 1);
+* decode batches (timing and full-size attention parity): keys, values and
+  queries N(0,1) in bf16 drawn on the device by a seeded torch generator
+  (Philox on CUDA), stand-in compact caches drawn the same way;
 * indexer weights in the shapes of Eqs. (indexer_parameters) and
   (value_indexer_parameters): U_q, U_k, U_v, L_q, L_k, L_v ~ N(0, 1/d),
   L_c ~ N(0, 1/d_A), L_x ~ N(0, 1/d_x), b_x ~ N(0, 0.1^2).
@@ -37,7 +43,7 @@ import numpy as np
 __all__ = [
     "Workload", "WORKLOADS", "IndexerShape", "bf16_round", "bf16_to_f64",
     "bf16_to_f32", "make_pair", "make_layer_activations", "make_heldout",
-    "make_indexer",
+    "make_indexer", "make_compact_cache", "decode_batch_device",
 ]
 
 D_HEAD = 128
@@ -90,7 +96,7 @@ WORKLOADS: Dict[str, Workload] = {
 }
 
 # stream ids (one Philox key per tensor family)
-_S_KEYS, _S_VALS, _S_QREF, _S_XREF, _S_HOLD, _S_IDX, _S_OUTL = range(1, 8)
+_S_KEYS, _S_VALS, _S_QREF, _S_XREF, _S_HOLD, _S_IDX, _S_OUTL, _S_CCACHE = range(1, 9)
 
 
 def _rng(*key: int) -> np.random.Generator:
@@ -205,3 +211,34 @@ def make_pair(w: Workload, layer: int, head: int, T: Optional[int] = None,
 def make_heldout(w: Workload, layer: int, head: int, K_bf16: np.ndarray, n: int) -> np.ndarray:
     """Held-out queries (same law as Q_ref, separate stream): [n, d] bf16 bits."""
     return _queries_like_keys(K_bf16, n, _rng(w.wid, layer, head, _S_HOLD))
+
+
+def make_compact_cache(w: Workload, layer: int, head: int, K_bf16: np.ndarray, V_bf16: np.ndarray,
+                       t: int) -> Dict[str, np.ndarray]:
+    """A stand-in compact cache of t rows (fp32) for attention tests: the
+    keys at t distinct random positions plus N(0, 0.1^2) noise, the values
+    there, beta ~ U(-2, 1).  No part of the compaction method is involved."""
+    g = _rng(w.wid, layer, head, _S_CCACHE)
+    S = np.sort(g.choice(K_bf16.shape[0], size=t, replace=False))
+    C_k = (bf16_to_f64(K_bf16[S]) + 0.1 * g.standard_normal((t, D_HEAD))).astype(np.float32)
+    C_v = bf16_to_f64(V_bf16[S]).astype(np.float32)
+    beta = g.uniform(-2.0, 1.0, size=t).astype(np.float32)
+    return {"C_k": C_k, "C_v": C_v, "beta": beta}
+
+
+def decode_batch_device(seed: int, H: int, G: int, T: int, t: int, F: int, device, compact_bf16: bool = True):
+    """One decode step's inputs on the device, drawn by a seeded torch
+    generator: Q [H, G, d], full cache K, V [H, T, d] and an uncompressed block
+    K_f, V_f [H, F, d] (bf16, N(0,1)); a stand-in compact cache C_k, C_v
+    [H, t, d] (bf16 or fp32, N(0,1)) and beta [H, t] ~ U(-2, 1)."""
+    import torch
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed)
+    def nrm(*shape, dt=torch.bfloat16):
+        return torch.randn(*shape, generator=gen, device=device, dtype=torch.float32).to(dt)
+    cdt = torch.bfloat16 if compact_bf16 else torch.float32
+    out = {"Q": nrm(H, G, D_HEAD), "K": nrm(H, T, D_HEAD), "V": nrm(H, T, D_HEAD),
+           "C_k": nrm(H, t, D_HEAD, dt=cdt), "C_v": nrm(H, t, D_HEAD, dt=cdt),
+           "beta": torch.rand(H, t, generator=gen, device=device) * 3.0 - 2.0,
+           "K_f": nrm(H, F, D_HEAD), "V_f": nrm(H, F, D_HEAD)}
+    return out

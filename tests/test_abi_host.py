@@ -23,7 +23,8 @@ def declared_functions():
 def test_header_declares_the_boundary():
     names = declared_functions()
     for n in ("arckv_compact", "arckv_attend", "arckv_workspace_bytes", "arckv_attend_workspace_bytes",
-              "arckv_query_status", "arckv_status_string"):
+              "arckv_query_status", "arckv_status_string", "arckv_anchor_count", "arckv_attend_joint",
+              "arckv_attend_joint_workspace_bytes"):
         assert n in names
 
 
@@ -110,3 +111,19 @@ def test_attend_rejects_bad_arguments_without_gpu(lib):
     assert pk.arckv_attend(2, 16, 8, 128, 0.0, 1, 1, 1, 1, 1, 256, need - 1, stream=0) == 3
     assert pk.arckv_attend(2, 16, 8, 128, -1.0, 1, 1, 1, 1, 1, 256, need, stream=0) == 1
     assert pk.arckv_attend(2, 16, 8, 128, 0.0, 1, 1, 1, 1, 1, 256, need, flags=4, stream=0) == 1
+
+
+def test_attend_joint_rejects_bad_arguments_without_gpu(lib):
+    need = pk.attend_joint_workspace_bytes(2, 4, 8, 8)
+    assert need > 0
+    args = dict(H=2, n=4, t=8, F=8, d=128, logit_scale=0.0, Q=256, C_k=256, beta=256, C_v=256, K_fixed=256,
+                V_fixed=256, O=256, ws=256, ws_bytes=need, stream=0)
+    call = lambda **kw: pk.arckv_attend_joint(**dict(args, **kw))
+    assert call(d=64) == 8
+    assert call(t=0, F=0) == 2
+    assert call(C_k=None) == 1
+    assert call(K_fixed=None) == 1
+    assert call(C_v=264) == 1            # not 16-byte aligned
+    assert call(ws_bytes=need - 1) == 3
+    assert call(flags=0x4) == 1
+    assert call(logit_scale=-1.0) == 1
