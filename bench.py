@@ -68,6 +68,10 @@ def parse_args(argv=None):
                     help="CUDA streams (each with its own workspace) the layers of a context are spread over")
     ap.add_argument("--cpu-pairs", type=int, default=4, help="(layer, head) pairs the oracle baseline times")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--decode", action="store_true",
+                    help="time one decode step of attention (App. D shape) instead of the compaction")
+    ap.add_argument("--decode-contexts", default="4096,8192,16384,32768")
+    ap.add_argument("--decode-iters", type=int, default=50)
     ap.add_argument("--profile-layer", action="store_true",
                     help="compact layer 0 twice and exit (a small case for ncu captures)")
     return ap.parse_args(argv)
@@ -473,6 +477,92 @@ def run_gpu(args, dist: Dist):
     return 0
 
 
+def run_decode(args, dist: Dist):
+    """One decode step of attention for a batch of 64 Llama-3.1-8B sequences
+    (8 KV heads x 4 query heads, head dim 128) per layer: full bf16 cache
+    (plain attention, t = 0) against a 20 % compact cache (bf16 C_k, C_v and
+    the bias beta), both through arckv_attend_joint, plus the full-length
+    bias-aware path (the whole cache passed as the compact block).  Inputs are
+    larger than L2 at every context, so calls run back to back."""
+    import torch
+    import synth
+    import paper_2609_36835_gb300 as pk
+
+    if dist.rank != 0:
+        return 0
+    torch.cuda.set_device(0)
+    pk.load_library()
+    B, H_kv, G, d = 64, 8, 4, 128
+    H = B * H_kv
+    _, hbm_peak, peak_src = measured_peaks()
+    flags = pk.FLAG_NONBLOCKING | pk.FLAG_COMPACT_BF16
+    stream = torch.cuda.current_stream()
+
+    def timed(fn):
+        for _ in range(max(3, args.warmup)):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.decode_iters):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / args.decode_iters   # us per call
+
+    rows = []
+    clocks = ClockSampler(0)
+    clocks.start()
+    for T in [int(x) for x in args.decode_contexts.split(",")]:
+        t = int(round(0.2 * T))
+        x = synth.decode_batch_device(1000 + T, H, G, T, t, 0, "cuda", compact_bf16=True)
+        O = torch.empty(H, G, d, dtype=torch.float32, device="cuda")
+        def call(t_, F_, Ck, beta, Cv, Kf, Vf, fl):
+            ws = torch.empty(pk.attend_joint_workspace_bytes(H, G, t_, F_), dtype=torch.uint8, device="cuda")
+            def fn():
+                st = pk.arckv_attend_joint(H, G, t_, F_, d, 0.0, x["Q"], Ck, beta, Cv, Kf, Vf, O, ws, ws.numel(),
+                                           flags=fl, stream=stream)
+                if st != 0:
+                    raise pk.ArckvError(st, "arckv_attend_joint")
+            return fn
+        us_full = timed(call(0, T, None, None, None, x["K"], x["V"], pk.FLAG_NONBLOCKING))
+        us_comp = timed(call(t, 0, x["C_k"], x["beta"], x["C_v"], None, None, flags))
+        beta_full = torch.zeros(H, T, dtype=torch.float32, device="cuda")
+        us_bias = timed(call(T, 0, x["K"], beta_full, x["V"], None, None, flags))
+        io = H * G * d * (2 + 4)                     # Q in, O out
+        b_full = H * T * d * 2 * 2 + io              # K and V, bf16
+        b_comp = H * t * d * 2 * 2 + H * t * 4 + io  # C_k, C_v bf16 and beta fp32
+        b_bias = H * T * d * 2 * 2 + H * T * 4 + io
+        rows.append({"T": T, "t": t, "full_us": round(us_full, 2), "compact_us": round(us_comp, 2),
+                     "full_bias_us": round(us_bias, 2), "speedup": round(us_full / us_comp, 3),
+                     "bias_path_vs_full": round(us_bias / us_full, 3),
+                     "kv_gb_full": round(b_full / 1e9, 3), "kv_gb_compact": round(b_comp / 1e9, 3),
+                     "full_gbs": round(b_full / us_full / 1e3, 1), "compact_gbs": round(b_comp / us_comp / 1e3, 1),
+                     "full_frac": round(b_full / us_full / 1e3 / hbm_peak, 3),
+                     "compact_frac": round(b_comp / us_comp / 1e3 / hbm_peak, 3)})
+        del x, beta_full
+        torch.cuda.empty_cache()
+    clk = clocks.stop()
+    last = rows[-1]
+    line = {
+        "metric": "decode-step attention latency per layer, batch 64, Llama-3.1-8B GQA (8 KV x 4 q heads), "
+                  "20% compact cache with beta vs full cache",
+        "value": last["compact_us"], "unit": "us/layer", "higher_is_better": False, "n_gpus": 1,
+        "steps": args.decode_iters, "warmup": max(3, args.warmup), "dtype": "bf16 cache, f32 accumulate",
+        "data": "synthetic (seeded N(0,1) bf16 caches on the device)",
+        "config": {"workload": "decode step: 64 sequences x 8 KV heads x 4 query rows, head_dim 128, t = 0.2 T",
+                   "l2": "inputs larger than L2 at every context; calls back to back"},
+        "contexts": rows,
+        "roofline": {"kernel": "attend_split_kernel (split-key decode attention)", "bound": "hbm",
+                     "achieved": last["compact_gbs"], "peak": hbm_peak, "unit": "GB/s",
+                     "frac": last["compact_frac"], "traffic": None,
+                     "peak_note": "HBM copy bandwidth, of %s (MEASURED_PEAKS.json)" % peak_src},
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main(argv=None):
     args = parse_args(argv)
     if args.warmup < 3 and not args.profile_layer:
@@ -480,6 +570,8 @@ def main(argv=None):
     dist = Dist()
     if args.impl == "reference":
         return run_reference(args, dist)
+    if args.decode:
+        return run_decode(args, dist)
     return run_gpu(args, dist)
 
 

@@ -352,7 +352,7 @@ arckv_status arckv_attend_joint(int32_t H, int32_t n, int32_t t, int32_t F, int3
   cudaGetLastError();
   if (cudaMemsetAsync(stt, 0, sizeof(DevStatus), st) != cudaSuccess) return ARCKV_ERR_CUDA;
   launch_attend_joint(H, n, t, F, scale, (const bf16*)Q, C_k, beta, C_v, (flags & ARCKV_FLAG_COMPACT_BF16) != 0,
-                      (const bf16*)K_fixed, (const bf16*)V_fixed, O, Opart, ml, st);
+                      (const bf16*)K_fixed, (const bf16*)V_fixed, O, Opart, ml, stt, st);
   launch_check_finite(O, (long long)H * n * d, stt, st);
   if (cudaGetLastError() != cudaSuccess) return ARCKV_ERR_CUDA;
   if (flags & ARCKV_FLAG_NONBLOCKING) return ARCKV_OK;

@@ -20,9 +20,19 @@
 //   attend_combine_kernel: per (head, row) merges the splits' (m, l, o).
 // t = 0 gives plain attention over the uncompressed block (the full-cache
 // baseline of the decode measurement); F = 0 the compact operator of Sec. 3.1.
+//
+// bf16 caches (both blocks bf16) take attend_bulk_kernel instead: one thread
+// streams each 64-key tile of K and V (16 KB each, contiguous rows) into a
+// 3-stage shared-memory ring with cp.async.bulk, so that every CTA keeps up
+// to 64 KB in flight, and the warps read the tiles two keys per instruction
+// (512 contiguous bytes: no bank conflicts).  Lane l holds query dims
+// 8 (l%16) .. +7 of the 4 rows in registers; the 16 partial dot products of a
+// lane (4 keys x 4 rows) are summed over the 16 lanes of each half-warp by a
+// transposing butterfly (15 shuffles).
 #include <algorithm>
 
 #include "kernels.h"
+#include "tc.cuh"
 
 namespace arckv {
 
@@ -230,6 +240,223 @@ __global__ void __launch_bounds__(kJThreads, 3) attend_split_kernel(const bf16* 
   }
 }
 
+constexpr int kBStages = 3;
+constexpr int kBTileBytes = kJTile * 128 * 2;   // one bf16 tile of K (or V)
+
+// Partial results of key split sp as in attend_split_kernel, for bf16 blocks.
+__global__ void __launch_bounds__(kJThreads, 2) attend_bulk_kernel(const bf16* Q, int n, const bf16* Ck,
+                                                                   const float* beta, const bf16* Cv, int t,
+                                                                   const bf16* Kf, const bf16* Vf, int F, float scale,
+                                                                   int per_split, int nsplit, float* Opart,
+                                                                   float2* ml, DevStatus* stt) {
+  extern __shared__ __align__(128) unsigned char smraw[];
+  bf16* sK = (bf16*)smraw;                                       // [stage][64][128]
+  bf16* sV = (bf16*)(smraw + kBStages * kBTileBytes);            // [stage][64][128]
+  __shared__ __align__(8) uint64_t bar[kBStages];
+  __shared__ float sP[kJR][kJTile];
+  __shared__ float sM[kJR], sL[kJR], sF[kJR];
+  __shared__ int abort_flag;
+  const int h = blockIdx.z, r0 = blockIdx.y * kJR, sp = blockIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5, hl = lane & 15, hh = lane >> 4;
+  const int L = t + F, jb = sp * per_split, je = min(L, jb + per_split);
+  // tiles: the compact keys [jb, min(je, t)) then the uncompressed ones [max(jb, t), je)
+  const int c_lo = jb, c_hi = min(je, t), f_lo = max(jb, t), f_hi = je;
+  const int n1 = c_hi > c_lo ? (c_hi - c_lo + kJTile - 1) / kJTile : 0;
+  const int ntile = n1 + (f_hi > f_lo ? (f_hi - f_lo + kJTile - 1) / kJTile : 0);
+  const bf16* Ckh = Ck + (long long)h * t * 128;
+  const bf16* Cvh = Cv + (long long)h * t * 128;
+  const bf16* Kfh = Kf + (long long)h * F * 128;
+  const bf16* Vfh = Vf + (long long)h * F * 128;
+  const float* bh = beta + (long long)h * t;
+  // tile i -> (first key j0, keys nk, compact?)
+  auto tile_of = [&](int i, int& j0, int& nk, bool& comp) {
+    comp = i < n1;
+    j0 = comp ? c_lo + i * kJTile : f_lo + (i - n1) * kJTile;
+    nk = min(kJTile, (comp ? c_hi : f_hi) - j0);
+  };
+  auto issue = [&](int i) {   // one thread: both tiles of tile i into stage i % S
+    int j0, nk;
+    bool comp;
+    tile_of(i, j0, nk, comp);
+    const int s = i % kBStages;
+    const uint32_t bytes = (uint32_t)nk * 256u;
+    tc::mbar_arrive_expect_tx(&bar[s], 2 * bytes);
+    const long long row = comp ? j0 : (long long)(j0 - t);
+    tc::bulk_load(sK + (size_t)s * kJTile * 128, (comp ? Ckh : Kfh) + row * 128, bytes, &bar[s]);
+    tc::bulk_load(sV + (size_t)s * kJTile * 128, (comp ? Cvh : Vfh) + row * 128, bytes, &bar[s]);
+  };
+  if (tid == 0) {
+    for (int s = 0; s < kBStages; ++s) tc::mbar_init(&bar[s], 1);
+    tc::mbar_fence_init();
+    abort_flag = 0;
+  }
+  if (tid < kJR) {
+    sM[tid] = -INFINITY;
+    sL[tid] = 0.f;
+  }
+  __syncthreads();
+  if (tid == 0)
+    for (int i = 0; i < min(kBStages, ntile); ++i) issue(i);
+  // the 4 query rows at dims 8 hl .. 8 hl + 7, pre-scaled
+  float q[kJR][8];
+#pragma unroll
+  for (int r = 0; r < kJR; ++r)
+#pragma unroll
+    for (int e = 0; e < 8; ++e)
+      q[r][e] = (r0 + r < n) ? scale * __bfloat162float(Q[((long long)h * n + r0 + r) * 128 + hl * 8 + e]) : 0.f;
+  float acc[kJR][8];
+#pragma unroll
+  for (int r = 0; r < kJR; ++r)
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[r][e] = 0.f;
+  int done = 0;   // tiles consumed
+  for (int i = 0; i < ntile; ++i) {
+    int j0, nk;
+    bool comp;
+    tile_of(i, j0, nk, comp);
+    const int s = i % kBStages;
+    const bool ok = tc::mbar_wait(&bar[s], (uint32_t)((i / kBStages) & 1), &abort_flag, stt);
+    if (__syncthreads_or(!ok)) break;
+    const bf16* Kt = sK + (size_t)s * kJTile * 128;
+    const bf16* Vt = sV + (size_t)s * kJTile * 128;
+    {  // logits: warp w takes keys 8w .. 8w+7, two per load (lane half hh)
+      float v[16];
+#pragma unroll
+      for (int qq = 0; qq < 4; ++qq) {
+        const int kk = 8 * w + 2 * qq + hh;
+        const uint4 raw = *(const uint4*)(Kt + kk * 128 + hl * 8);
+        const __nv_bfloat162* h2 = (const __nv_bfloat162*)&raw;
+        float k8[8];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = __bfloat1622float2(h2[e]);
+          k8[2 * e] = f.x;
+          k8[2 * e + 1] = f.y;
+        }
+#pragma unroll
+        for (int r = 0; r < kJR; ++r) {
+          float a = 0.f;
+#pragma unroll
+          for (int e = 0; e < 8; ++e) a = fmaf(q[r][e], k8[e], a);
+          v[qq * 4 + r] = a;
+        }
+      }
+      // transposing butterfly over the 16 lanes of the half-warp: lane hl ends
+      // with the sum of entry hl (key 2 (hl >> 2) + hh of the warp, row hl & 3)
+#pragma unroll
+      for (int i8 = 0; i8 < 8; ++i8) {
+        const bool up = hl & 8;
+        const float mine = up ? v[8 + i8] : v[i8], other = up ? v[i8] : v[8 + i8];
+        v[i8] = mine + __shfl_xor_sync(0xffffffffu, other, 8);
+      }
+#pragma unroll
+      for (int i4 = 0; i4 < 4; ++i4) {
+        const bool up = hl & 4;
+        const float mine = up ? v[4 + i4] : v[i4], other = up ? v[i4] : v[4 + i4];
+        v[i4] = mine + __shfl_xor_sync(0xffffffffu, other, 4);
+      }
+#pragma unroll
+      for (int i2 = 0; i2 < 2; ++i2) {
+        const bool up = hl & 2;
+        const float mine = up ? v[2 + i2] : v[i2], other = up ? v[i2] : v[2 + i2];
+        v[i2] = mine + __shfl_xor_sync(0xffffffffu, other, 2);
+      }
+      {
+        const bool up = hl & 1;
+        const float mine = up ? v[1] : v[0], other = up ? v[0] : v[1];
+        v[0] = mine + __shfl_xor_sync(0xffffffffu, other, 1);
+      }
+      const int kk = 8 * w + 2 * (hl >> 2) + hh, r = hl & 3;
+      const bool valid = kk < nk;
+      const float b = (valid && comp) ? __ldg(bh + j0 + kk) : 0.f;
+      sP[r][kk] = valid ? v[0] + b : -INFINITY;
+    }
+    __syncthreads();
+    if (w < kJR) {  // online softmax of row w over the tile (at least one key is valid)
+      const float a0 = sP[w][lane], a1 = sP[w][lane + 32];
+      const float mold = sM[w], mnew = fmaxf(mold, warp_max(fmaxf(a0, a1)));
+      const float e0 = expf(a0 - mnew), e1 = expf(a1 - mnew);
+      sP[w][lane] = e0;
+      sP[w][lane + 32] = e1;
+      const float ssum = warp_sum(e0 + e1);
+      if (lane == 0) {
+        const float f = expf(mold - mnew);   // 0 on the first tile (mold = -inf)
+        sF[w] = f;
+        sL[w] = sL[w] * f + ssum;
+        sM[w] = mnew;
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int r = 0; r < kJR; ++r) {
+      const float f = sF[r];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[r][e] *= f;
+    }
+#pragma unroll
+    for (int qq = 0; qq < 4; ++qq) {   // values: the same keys, dims 8 hl .. 8 hl + 7
+      const int kk = 8 * w + 2 * qq + hh;
+      if (kk < nk) {
+        const uint4 raw = *(const uint4*)(Vt + kk * 128 + hl * 8);
+        const __nv_bfloat162* h2 = (const __nv_bfloat162*)&raw;
+        float v8[8];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = __bfloat1622float2(h2[e]);
+          v8[2 * e] = f.x;
+          v8[2 * e + 1] = f.y;
+        }
+#pragma unroll
+        for (int r = 0; r < kJR; ++r) {
+          const float pr = sP[r][kk];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) acc[r][e] = fmaf(pr, v8[e], acc[r][e]);
+        }
+      }
+    }
+    __syncthreads();   // stage s and sP are free
+    done = i + 1;
+    if (tid == 0 && i + kBStages < ntile) issue(i + kBStages);
+  }
+  if (done < ntile) {
+    // a wait gave up (status recorded): let the copies already issued land
+    // (bounded) before the CTA's shared memory goes away, and write nothing
+    if (tid == 0) {
+      const unsigned long long t0 = tc::globaltimer();
+      for (int i = done; i < min(ntile, done + kBStages); ++i)
+        while (!tc::mbar_try_wait(&bar[i % kBStages], (uint32_t)((i / kBStages) & 1)) &&
+               tc::globaltimer() - t0 < tc::kWaitLimitNs) {
+        }
+    }
+    __syncthreads();
+    return;
+  }
+  // lanes l and l ^ 16 hold the same dims over different keys
+#pragma unroll
+  for (int r = 0; r < kJR; ++r)
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[r][e] += __shfl_xor_sync(0xffffffffu, acc[r][e], 16);
+  float* sAcc = (float*)smraw;   // [8 warps][kJR][128], over the drained stages
+  if (hh == 0) {
+#pragma unroll
+    for (int r = 0; r < kJR; ++r) {
+      *(float4*)&sAcc[(w * kJR + r) * 128 + hl * 8] = make_float4(acc[r][0], acc[r][1], acc[r][2], acc[r][3]);
+      *(float4*)&sAcc[(w * kJR + r) * 128 + hl * 8 + 4] = make_float4(acc[r][4], acc[r][5], acc[r][6], acc[r][7]);
+    }
+  }
+  __syncthreads();
+  for (int e = tid; e < kJR * 128; e += kJThreads) {
+    const int r = e >> 7, dd = e & 127;
+    if (r0 + r >= n) continue;
+    float o = 0.f;
+#pragma unroll
+    for (int q8 = 0; q8 < kJThreads / 32; ++q8) o += sAcc[(q8 * kJR + r) * 128 + dd];
+    const long long row = ((long long)h * nsplit + sp) * n + r0 + r;
+    Opart[row * 128 + dd] = o;
+    if (dd == 0) ml[row] = make_float2(sM[r], sL[r]);
+  }
+}
+
 // O[h][i] = sum_s e^{m_s - m} Opart_s / sum_s e^{m_s - m} l_s (one warp per row, lane dims 4l..4l+3)
 __global__ void __launch_bounds__(256) attend_combine_kernel(const float* Opart, const float2* ml, int n, int nsplit,
                                                              long long rows, float* O) {
@@ -269,13 +496,15 @@ JointSplit joint_split(int H, int n, int t, int F) {
 
 int launch_attend_joint(int H, int n, int t, int F, float scale, const bf16* Q, const void* Ck, const float* beta,
                         const void* Cv, bool compact_bf16, const bf16* Kf, const bf16* Vf, float* O, float* Opart,
-                        float2* ml, cudaStream_t st) {
+                        float2* ml, DevStatus* stt, cudaStream_t st) {
   const JointSplit s = joint_split(H, n, t, F);
   const dim3 grid(s.nsplit, cdiv(n, kJR), H);
-  if (compact_bf16)
-    attend_split_kernel<bf16><<<grid, kJThreads, 0, st>>>(Q, n, (const bf16*)Ck, beta, (const bf16*)Cv, t, Kf, Vf, F,
-                                                          scale, s.per_split, s.nsplit, Opart, ml);
-  else
+  if (compact_bf16 || t == 0) {
+    const int smem = 2 * kBStages * kBTileBytes;
+    cudaFuncSetAttribute(attend_bulk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    attend_bulk_kernel<<<grid, kJThreads, smem, st>>>(Q, n, (const bf16*)Ck, beta, (const bf16*)Cv, t, Kf, Vf, F,
+                                                      scale, s.per_split, s.nsplit, Opart, ml, stt);
+  } else
     attend_split_kernel<float><<<grid, kJThreads, 0, st>>>(Q, n, (const float*)Ck, beta, (const float*)Cv, t, Kf, Vf,
                                                            F, scale, s.per_split, s.nsplit, Opart, ml);
   const long long rows = (long long)H * n;

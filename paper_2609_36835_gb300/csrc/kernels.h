@@ -117,7 +117,7 @@ JointSplit joint_split(int H, int n, int t, int F);
 // scratch Opart [H][nsplit][n][128] fp32 and ml [H][nsplit][n].
 int launch_attend_joint(int H, int n, int t, int F, float scale, const bf16* Q, const void* Ck, const float* beta,
                         const void* Cv, bool compact_bf16, const bf16* Kf, const bf16* Vf, float* O, float* Opart,
-                        float2* ml, cudaStream_t st);
+                        float2* ml, DevStatus* stt, cudaStream_t st);
 
 // Shared small kernels.
 int launch_part_stats(int H, int rows, int ntiles, const float2* part, float* shift, float* mul, float* sum,
