@@ -2,7 +2,8 @@
 //
 //   D[b](m, n) = sum_k A[b](m, k) B[b](n, k)      (A, B bf16, K-major, D fp32 in TMEM)
 //
-// One CTA computes a 128 x BN tile.  Warp 0 streams 64-wide K slabs of A and B
+// Persistent: one CTA per SM walks the 128 x BN output tiles (b, row tile,
+// column tile; columns fastest) in a grid-stride loop.  Warp 0 streams 64-wide K slabs of A and B
 // into a STAGES-deep ring of 128-byte-swizzled shared tiles with TMA; warp 1
 // issues tcgen05.mma (M = 128, N = BN, K = 16) into one of two TMEM
 // accumulators; warps 2..5 drain the accumulator with tcgen05.ld, one TMEM
@@ -25,7 +26,10 @@
 // fresh accumulator and the epilogue sees every chunk separately, which lets
 // a non-linearity act between chunks (the per-index-head LeakyReLU of
 // Eq. pairwise_index_score).  The two TMEM buffers alternate between chunks,
-// so the MMA of chunk c+1 overlaps the epilogue of chunk c.
+// so the MMA of chunk c+1 overlaps the epilogue of chunk c -- also across
+// tiles: the stage ring, the chunk counter and the accumulator alternation run
+// on over a CTA's tiles, so a tile's last epilogue overlaps the next tile's
+// first MMAs and no tile pays a prologue.
 //
 // Epilogue interface (all per thread = per output row):
 //   struct State;                                     registers of one row
@@ -33,6 +37,8 @@
 //   void consume(State&, int chunk, int j, float (&v)[32]);  columns n0+32j..
 //   void finish(State&, int b, int row, int n0, int M, int N);
 #pragma once
+#include <algorithm>
+
 #include "tc.cuh"
 
 namespace arckv {
@@ -55,7 +61,7 @@ template <int BN, int MODE, class Epi>
 __global__ void __launch_bounds__(192, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
                    const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mB2,
-                   const __grid_constant__ CUtensorMap mA3, Epi epi, int M, int N, int K, int chunk_k, int K1,
+                   const __grid_constant__ CUtensorMap mA3, Epi epi, int H, int M, int N, int K, int chunk_k, int K1,
                    DevStatus* stt) {
   using C = TcCfg<BN, MODE>;
   constexpr bool SPLIT = C::SPLIT;
@@ -67,10 +73,18 @@ __global__ void __launch_bounds__(192, 1)
   const uint32_t raw = tc::smem_u32(smem_raw);
   uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int b = blockIdx.z, m0 = blockIdx.y * 128, n0 = blockIdx.x * BN;
   const int nk = (K + 63) / 64;
   const int kpc = chunk_k / 64;
   const int nchunks = (nk + kpc - 1) / kpc;
+  // persistent: CTA c takes tiles c, c + grid, ...; tile = (b, row tile, column tile), columns fastest
+  const int Mt = (M + 127) / 128, Nt = (N + BN - 1) / BN;
+  const int ntiles = H * Mt * Nt;
+  auto tile_coords = [&](int tl, int& b, int& m0, int& n0) {
+    b = tl / (Mt * Nt);
+    const int r = tl - b * (Mt * Nt);
+    m0 = (r / Nt) * 128;
+    n0 = (r % Nt) * BN;
+  };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -104,72 +118,86 @@ __global__ void __launch_bounds__(192, 1)
         tc::tma_prefetch(&mA2);
         tc::tma_prefetch(&mA3);
       }
-      int issued = 0;
-      for (int kb = 0; kb < nk; ++kb) {
-        const int s = kb % STAGES;
-        if (kb >= STAGES && !tc::mbar_wait(&empty[s], ((kb / STAGES) - 1) & 1, abortp, stt)) break;
-        uint8_t* st = base + s * C::STAGE;
-        tc::mbar_arrive_expect_tx(&full[s], C::STAGE);
-        if (MODE == kConcat && kb * 64 >= K1) {
-          tc::tma_load_3d(st, &mA2, kb * 64 - K1, m0, b, &full[s]);
-          tc::tma_load_3d(st + C::TILE_A, &mB2, kb * 64 - K1, n0, b, &full[s]);
-        } else {
-          tc::tma_load_3d(st, &mA, kb * 64, m0, b, &full[s]);
-          tc::tma_load_3d(st + C::TILE_A, &mB, kb * 64, n0, b, &full[s]);
+      int g = 0;   // K slabs issued by this CTA (ring position across tiles)
+      bool ok = true;
+      for (int tl = blockIdx.x; tl < ntiles && ok; tl += gridDim.x) {
+        int b, m0, n0;
+        tile_coords(tl, b, m0, n0);
+        for (int kb = 0; kb < nk; ++kb) {
+          const int s = g % STAGES;
+          if (g >= STAGES && !tc::mbar_wait(&empty[s], ((g / STAGES) - 1) & 1, abortp, stt)) {
+            ok = false;
+            break;
+          }
+          uint8_t* st = base + s * C::STAGE;
+          tc::mbar_arrive_expect_tx(&full[s], C::STAGE);
+          if (MODE == kConcat && kb * 64 >= K1) {
+            tc::tma_load_3d(st, &mA2, kb * 64 - K1, m0, b, &full[s]);
+            tc::tma_load_3d(st + C::TILE_A, &mB2, kb * 64 - K1, n0, b, &full[s]);
+          } else {
+            tc::tma_load_3d(st, &mA, kb * 64, m0, b, &full[s]);
+            tc::tma_load_3d(st + C::TILE_A, &mB, kb * 64, n0, b, &full[s]);
+          }
+          if (SPLIT) {
+            tc::tma_load_3d(st + C::TILE_A + C::TILE_B, &mA2, kb * 64, m0, b, &full[s]);
+            tc::tma_load_3d(st + 2 * C::TILE_A + C::TILE_B, &mB2, kb * 64, n0, b, &full[s]);
+          }
+          if (MODE == kSplit3A) {
+            tc::tma_load_3d(st + C::TILE_A + C::TILE_B, &mA2, kb * 64, m0, b, &full[s]);
+            tc::tma_load_3d(st + 2 * C::TILE_A + C::TILE_B, &mA3, kb * 64, m0, b, &full[s]);
+          }
+          ++g;
         }
-        if (SPLIT) {
-          tc::tma_load_3d(st + C::TILE_A + C::TILE_B, &mA2, kb * 64, m0, b, &full[s]);
-          tc::tma_load_3d(st + 2 * C::TILE_A + C::TILE_B, &mB2, kb * 64, n0, b, &full[s]);
-        }
-        if (MODE == kSplit3A) {
-          tc::tma_load_3d(st + C::TILE_A + C::TILE_B, &mA2, kb * 64, m0, b, &full[s]);
-          tc::tma_load_3d(st + 2 * C::TILE_A + C::TILE_B, &mA3, kb * 64, m0, b, &full[s]);
-        }
-        issued = kb + 1;
       }
       // every issued copy lands before the CTA may exit
       volatile int never = 0;
-      for (int kb = issued > STAGES ? issued - STAGES : 0; kb < issued; ++kb)
-        tc::mbar_wait(&full[kb % STAGES], (kb / STAGES) & 1, &never, stt);
+      for (int k = g > STAGES ? g - STAGES : 0; k < g; ++k)
+        tc::mbar_wait(&full[k % STAGES], (k / STAGES) & 1, &never, stt);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = tc::idesc_bf16_f32(BN);
       bool ok = true;
-      for (int c = 0; c < nchunks && ok; ++c) {
-        const int buf = c & 1;
-        if (c >= 2 && !tc::mbar_wait(&acce[buf], ((c >> 1) - 1) & 1, abortp, stt)) break;
-        tc::fence_after_sync();
-        const uint32_t d = tmem + (uint32_t)(buf * BN);
-        const int kb0 = c * kpc, kb1 = min(nk, kb0 + kpc);
-        for (int kb = kb0; kb < kb1; ++kb) {
-          const int s = kb % STAGES;
-          if (!tc::mbar_wait(&full[s], (kb / STAGES) & 1, abortp, stt)) {
+      int g = 0, cg = 0;   // K slabs and chunks consumed by this CTA, across tiles
+      for (int tl = blockIdx.x; tl < ntiles && ok; tl += gridDim.x) {
+        for (int c = 0; c < nchunks && ok; ++c, ++cg) {
+          const int buf = cg & 1;
+          if (cg >= 2 && !tc::mbar_wait(&acce[buf], ((cg >> 1) - 1) & 1, abortp, stt)) {
             ok = false;
             break;
           }
           tc::fence_after_sync();
-          const uint32_t a = tc::smem_u32(base + s * C::STAGE), bb = a + C::TILE_A;
+          const uint32_t d = tmem + (uint32_t)(buf * BN);
+          const int kb0 = c * kpc, kb1 = min(nk, kb0 + kpc);
+          for (int kb = kb0; kb < kb1; ++kb, ++g) {
+            const int s = g % STAGES;
+            if (!tc::mbar_wait(&full[s], (g / STAGES) & 1, abortp, stt)) {
+              ok = false;
+              break;
+            }
+            tc::fence_after_sync();
+            const uint32_t a = tc::smem_u32(base + s * C::STAGE), bb = a + C::TILE_A;
 #pragma unroll
-          for (int ks = 0; ks < 4; ++ks) {
-            const uint64_t ad = tc::sdesc_k128(a + ks * 32), bd = tc::sdesc_k128(bb + ks * 32);
-            tc::mma_f16(d, ad, bd, idesc, (kb > kb0 || ks > 0) ? 1u : 0u);
-            if (SPLIT) {
-              const uint64_t ad2 = tc::sdesc_k128(a + C::TILE_A + C::TILE_B + ks * 32);
-              const uint64_t bd2 = tc::sdesc_k128(bb + C::TILE_A + C::TILE_B + ks * 32);
-              tc::mma_f16(d, ad, bd2, idesc, 1u);
-              tc::mma_f16(d, ad2, bd, idesc, 1u);
+            for (int ks = 0; ks < 4; ++ks) {
+              const uint64_t ad = tc::sdesc_k128(a + ks * 32), bd = tc::sdesc_k128(bb + ks * 32);
+              tc::mma_f16(d, ad, bd, idesc, (kb > kb0 || ks > 0) ? 1u : 0u);
+              if (SPLIT) {
+                const uint64_t ad2 = tc::sdesc_k128(a + C::TILE_A + C::TILE_B + ks * 32);
+                const uint64_t bd2 = tc::sdesc_k128(bb + C::TILE_A + C::TILE_B + ks * 32);
+                tc::mma_f16(d, ad, bd2, idesc, 1u);
+                tc::mma_f16(d, ad2, bd, idesc, 1u);
+              }
+              if (MODE == kSplit3A) {
+                const uint64_t am = tc::sdesc_k128(a + C::TILE_A + C::TILE_B + ks * 32);
+                const uint64_t al = tc::sdesc_k128(a + 2 * C::TILE_A + C::TILE_B + ks * 32);
+                tc::mma_f16(d, am, bd, idesc, 1u);
+                tc::mma_f16(d, al, bd, idesc, 1u);
+              }
             }
-            if (MODE == kSplit3A) {
-              const uint64_t am = tc::sdesc_k128(a + C::TILE_A + C::TILE_B + ks * 32);
-              const uint64_t al = tc::sdesc_k128(a + 2 * C::TILE_A + C::TILE_B + ks * 32);
-              tc::mma_f16(d, am, bd, idesc, 1u);
-              tc::mma_f16(d, al, bd, idesc, 1u);
-            }
+            tc::mma_commit(&empty[s]);
           }
-          tc::mma_commit(&empty[s]);
+          if (ok) tc::mma_commit(&accf[buf]);
         }
-        if (ok) tc::mma_commit(&accf[buf]);
       }
       // all MMAs this thread issued have completed before teardown
       tc::mma_commit(&drain);
@@ -179,26 +207,31 @@ __global__ void __launch_bounds__(192, 1)
   } else {
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     const int row = q * 32 + lane;
-    typename Epi::State es;
-    epi.init(es, b, m0 + row, n0, M, N);
     bool ok = true;
-    for (int c = 0; c < nchunks; ++c) {
-      const int buf = c & 1;
-      ok = tc::mbar_wait(&accf[buf], (c >> 1) & 1, abortp, stt);
-      ok = __all_sync(0xffffffffu, ok);
-      if (!ok) break;
-      tc::fence_after_sync();
+    int cg = 0;
+    for (int tl = blockIdx.x; tl < ntiles && ok; tl += gridDim.x) {
+      int b, m0, n0;
+      tile_coords(tl, b, m0, n0);
+      typename Epi::State es;
+      epi.init(es, b, m0 + row, n0, M, N);
+      for (int c = 0; c < nchunks; ++c, ++cg) {
+        const int buf = cg & 1;
+        ok = tc::mbar_wait(&accf[buf], (cg >> 1) & 1, abortp, stt);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) break;
+        tc::fence_after_sync();
 #pragma unroll
-      for (int j = 0; j < BN / 32; ++j) {
-        float v[32];
-        tc::tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN + j * 32), v);
-        epi.consume(es, c, j, v);
+        for (int j = 0; j < BN / 32; ++j) {
+          float v[32];
+          tc::tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN + j * 32), v);
+          epi.consume(es, c, j, v);
+        }
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&acce[buf]);
       }
-      tc::fence_before_sync();
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&acce[buf]);
+      if (ok) epi.finish(es, b, m0 + row, n0, M, N);
     }
-    if (ok) epi.finish(es, b, m0 + row, n0, M, N);
   }
   tc::fence_before_sync();
   __syncthreads();
@@ -207,6 +240,10 @@ __global__ void __launch_bounds__(192, 1)
     tc::tmem_dealloc(tmem, C::TMEM_COLS);
   }
 }
+
+// Resident CTAs of the persistent GEMM: one per SM (the stage ring takes most
+// of the shared memory), looked up once per device.
+int tc_gemm_sm_count();
 
 // Host: launch over H batches; maps are built by the caller (encode_bf16_map_3d,
 // box rows 128 for A and BN for B).
@@ -218,8 +255,9 @@ inline cudaError_t launch_tc_gemm(const CUtensorMap& mA, const CUtensorMap& mB, 
   auto kern = tc_gemm_kernel<BN, MODE, Epi>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
-  dim3 grid(cdiv(N, BN), cdiv(M, 128), H);
-  kern<<<grid, 192, C::SMEM, st>>>(mA, mB, mA2, mB2, mA3 ? *mA3 : mA, epi, M, N, K, chunk_k, K1, stt);
+  const long long ntiles = (long long)cdiv(N, BN) * cdiv(M, 128) * H;
+  const int grid = (int)std::min<long long>(ntiles, tc_gemm_sm_count());
+  kern<<<grid, 192, C::SMEM, st>>>(mA, mB, mA2, mB2, mA3 ? *mA3 : mA, epi, H, M, N, K, chunk_k, K1, stt);
   return cudaGetLastError();
 }
 

@@ -35,4 +35,18 @@ bool encode_bf16_map_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint6
   return r == CUDA_SUCCESS;
 }
 
+int tc_gemm_sm_count() {
+  static std::mutex mu;
+  static int cache[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
+  std::lock_guard<std::mutex> lock(mu);
+  if (cache[dev] == 0) {
+    int v = 0;
+    cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+    cache[dev] = v > 0 ? v : 1;
+  }
+  return cache[dev];
+}
+
 }  // namespace arckv
