@@ -42,7 +42,7 @@ __global__ void mass_rhs_kernel(const float* Phi, const float* m, float* rhs, in
 
 // ---------------------------------------------------------------------------
 // Cluster Cholesky solver: (Gram + lam I) X = B for every head in ONE launch.
-// One cluster of kCL CTAs per head; the matrix, its factor and the right-hand
+// One cluster of kCL CTAs (cluster_size) per head; the matrix, its factor and the right-hand
 // sides live in global memory (L2-resident at these sizes) and are read with
 // ld.global.cg so that no CTA sees a stale L1 line of another CTA's writes.
 // Phases of each 64-wide block step k are separated by hardware cluster
@@ -56,7 +56,10 @@ __global__ void mass_rhs_kernel(const float* Phi, const float* m, float* rhs, in
 // Z_i -= L_ki^T X_k (i < k).  lam = ridge * trace(Gram) / tdiv is added to the
 // diagonal as each diagonal block is factored (tdiv = t, or the primal size
 // when the dual system is solved).
-constexpr int kCL = 4;
+// CTAs per cluster (one cluster per head): 4 up to 16 blocks (t <= 1024) --
+// half the SMs of 8 at nearly the same latency, which leaves room for the
+// concurrent layers -- and 8 for longer systems, whose tile work dominates.
+constexpr int cluster_size(int t) { return (t + NB - 1) / NB > 16 ? 8 : 4; }
 constexpr int kCT = 512;
 // Shared tiles are [NB][NBP] with rows padded to a 16-byte multiple, so that
 // mm64 can read them with vector loads.
@@ -204,103 +207,120 @@ __device__ __forceinline__ void store_diag(Tile<R> L, Tile<R> Li, R* Ab, R* Lb, 
 }
 
 // Factor diagonal block k (lower part of A_kk + lam I) in shared memory and
-// invert the factor: L_kk goes into A and L_kk^-1 into Linv[k].
-//   factor:  right-looking and unscaled, one barrier per column: step c
-//            subtracts a_rc a_jc / a_cc from every (r, j) with c < j <= r (the
-//            lower triangle is dealt to the threads; each forms 1 / a_cc
-//            itself); the column scaling by sqrt(a_cc) follows in one pass;
-//   inverse: each warp forms four columns of L^-1 by forward substitution
-//            (column j of L^-1 solves L x = e_j), reading L^T from Li.
-// Pad rows beyond the matrix (kb < NB) are the identity.
+// invert the factor: L_kk goes into A and L_kk^-1 into Linv[k].  Blocked in
+// four 16-wide panels, every phase on all warps:
+//   panel p: factor its 16 x 16 diagonal block (unscaled right-looking, one
+//            element per thread, one barrier per column; then the column
+//            scaling by sqrt(a_cc)) and invert it (forward substitution by
+//            columns, one barrier per row); L_panel = A_panel X_pp^T below it;
+//            trailing update A -= L_panel L_panel^T;
+//   inverse: off-diagonal 16 x 16 blocks X_ij = -X_ii sum_{m=j}^{i-1} L_im X_mj,
+//            level by level (i - j = 1, 2, 3).
+// Tiles: L (the block; pad column NB holds 1 / l_cc), Li (the inverse), T
+// (scratch).  Pad rows beyond the matrix (kb < NB) are the identity.
 template <typename R>
-__device__ void factor_diag(R* Ab, R* Lb, int t, int k, R lam, Tile<R> L, Tile<R> Li, int* bad) {
-  static_assert(kCT == 16 * 32, "the inverse deals 64 columns to 16 warps");
+__device__ void factor_diag(R* Ab, R* Lb, int t, int k, R lam, Tile<R> L, Tile<R> Li, Tile<R> T, int* bad) {
+  static_assert(kCT == 512 && NB == 64, "thread map of the 16-wide panels");
   const int tid = threadIdx.x, k0 = k * NB, kb = min(NB, t - k0);
   load_diag(L, Ab, t, k0, kb, lam);
+  for (int e = tid; e < NB * NB; e += kCT) Li[e / NB][e % NB] = R(0);
   __syncthreads();
-  constexpr int NT = NB * (NB + 1) / 2, NQ = (NT + kCT - 1) / kCT;
-  int er[NQ], ej[NQ];
+  const bool blk = tid < 256;
+  const int er = (tid >> 4) & 15, ec = tid & 15;   // element of a 16 x 16 block (threads < 256)
+  for (int p = 0; p < 4; ++p) {
+    const int c0 = 16 * p;
+    for (int j = 0; j < 15; ++j) {   // factor the diagonal block
+      if (blk && ec > j && er >= ec) {
+        R piv = L[c0 + j][c0 + j];
+        if (!(piv > R(0)) || !isfinite(piv)) piv = R(1);
+        L[c0 + er][c0 + ec] = fma_r(-L[c0 + er][c0 + j] * rcp_r(piv), L[c0 + ec][c0 + j], L[c0 + er][c0 + ec]);
+      }
+      __syncthreads();
+    }
+    R v = R(0);
+    if (blk && er >= ec) {   // column scaling
+      R pc = L[c0 + ec][c0 + ec];
+      if (!(pc > R(0)) || !isfinite(pc)) {
+        if (er == ec && c0 + ec < kb) *bad = 1;
+        pc = R(1);
+      }
+      const R d = sqrt(pc);
+      v = (er == ec) ? d : L[c0 + er][c0 + ec] * rcp_r(d);
+    }
+    __syncthreads();
+    if (blk && er >= ec) {
+      L[c0 + er][c0 + ec] = v;
+      if (er == ec) {
+        L[c0 + er][NB] = rcp_r(v);
+        Li[c0 + er][c0 + er] = R(1);
+      }
+    }
+    __syncthreads();
+    for (int i = 0; i < 15; ++i) {   // Y = I; y_lj -= l_li y_ij / l_ii for l > i, j <= i
+      if (blk && er > i && ec <= i)
+        Li[c0 + er][c0 + ec] = fma_r(-L[c0 + er][c0 + i] * L[c0 + i][NB], Li[c0 + i][c0 + ec], Li[c0 + er][c0 + ec]);
+      __syncthreads();
+    }
+    if (blk && ec <= er) Li[c0 + er][c0 + ec] *= L[c0 + er][NB];   // X_pp = diag(1 / l_rr) Y
+    __syncthreads();
+    if (p == 3) break;
+    {  // panel below: L[r][c0 + c] = sum_m A[r][c0 + m] X_pp[c][m] (all reads before the writes)
+      const int rows = NB - c0 - 16;
+      R o[2];
+      int pr[2], pcol[2];
 #pragma unroll
-  for (int q = 0; q < NQ; ++q) {
-    const int e = tid + q * kCT;
-    int rr = (int)((sqrtf(8.f * e + 1.f) - 1.f) * 0.5f);
-    while (rr * (rr + 1) / 2 > e) --rr;
-    while ((rr + 1) * (rr + 2) / 2 <= e) ++rr;
-    er[q] = e < NT ? rr : -1;
-    ej[q] = e < NT ? e - rr * (rr + 1) / 2 : -1;   // -1: no entry (never > c)
+      for (int q = 0; q < 2; ++q) {
+        const int e = tid + q * kCT;
+        pr[q] = -1;
+        if (e < rows * 16) {
+          const int r = c0 + 16 + e / 16, c = e % 16;
+          R a = R(0);
+          for (int m = 0; m <= c; ++m) a = fma_r(L[r][c0 + m], Li[c0 + c][c0 + m], a);
+          o[q] = a;
+          pr[q] = r;
+          pcol[q] = c;
+        }
+      }
+      __syncthreads();
+#pragma unroll
+      for (int q = 0; q < 2; ++q)
+        if (pr[q] >= 0) L[pr[q]][c0 + pcol[q]] = o[q];
+      __syncthreads();
+    }
+    {  // trailing update: L[r][c] -= sum_m L[r][c0 + m] L[c][c0 + m], c0 + 16 <= c <= r
+      const int c1 = c0 + 16, wdt = NB - c1, ntri = wdt * (wdt + 1) / 2;
+      for (int e = tid; e < ntri; e += kCT) {
+        int r = (int)((sqrtf(8.f * e + 1.f) - 1.f) * 0.5f);
+        while (r * (r + 1) / 2 > e) --r;
+        while ((r + 1) * (r + 2) / 2 <= e) ++r;
+        const int c = e - r * (r + 1) / 2;
+        R a = L[c1 + r][c1 + c];
+#pragma unroll
+        for (int m = 0; m < 16; ++m) a = fma_r(-L[c1 + r][c0 + m], L[c1 + c][c0 + m], a);
+        L[c1 + r][c1 + c] = a;
+      }
+      __syncthreads();
+    }
   }
-  auto pivot_inv = [](R v) { return (v > R(0) && isfinite(v)) ? rcp_r(v) : R(1); };
-  for (int c = 0; c < NB - 1; ++c) {
-    R a[NQ], b[NQ], d[NQ];
-    const R pinv = pivot_inv(L[c][c]);
+  for (int lv = 1; lv < 4; ++lv) {   // off-diagonal blocks of the inverse, level i - j = lv
+    const int nbk = 4 - lv;
+    for (int e = tid; e < nbk * 256; e += kCT) {
+      const int j = e >> 8, i = j + lv, r = (e >> 4) & 15, c = e & 15;
+      R a = R(0);
+      for (int m = j; m < i; ++m)
 #pragma unroll
-    for (int q = 0; q < NQ; ++q)
-      if (ej[q] > c) {
-        a[q] = L[er[q]][c];
-        b[q] = L[ej[q]][c];
-        d[q] = L[er[q]][ej[q]];
-      }
-#pragma unroll
-    for (int q = 0; q < NQ; ++q)
-      if (ej[q] > c) {
-        const R v = fma_r(-a[q] * pinv, b[q], d[q]);
-        L[er[q]][ej[q]] = v;
-      }
+        for (int q = 0; q < 16; ++q) a = fma_r(L[16 * i + r][16 * m + q], Li[16 * m + q][16 * j + c], a);
+      T[16 * i + r][16 * j + c] = a;
+    }
+    __syncthreads();
+    for (int e = tid; e < nbk * 256; e += kCT) {
+      const int j = e >> 8, i = j + lv, r = (e >> 4) & 15, c = e & 15;
+      R a = R(0);
+      for (int q = 0; q <= r; ++q) a = fma_r(Li[16 * i + r][16 * i + q], T[16 * i + q][16 * j + c], a);
+      Li[16 * i + r][16 * j + c] = -a;
+    }
     __syncthreads();
   }
-  R nv[NQ];
-#pragma unroll
-  for (int q = 0; q < NQ; ++q)
-    if (er[q] >= 0) {
-      const int rr = er[q], j = ej[q];
-      R pj = L[j][j];
-      if (!(pj > R(0)) || !isfinite(pj)) {
-        if (rr == j && j < kb) *bad = 1;
-        pj = R(1);
-      }
-      const R dj = sqrt(pj), djinv = rcp_r(dj);
-      nv[q] = (rr == j) ? dj : L[rr][j] * djinv;
-      if (rr == j) L[j][NB] = djinv;   // the pad column holds 1 / L_jj for the inverse
-    }
-  __syncthreads();
-#pragma unroll
-  for (int q = 0; q < NQ; ++q)
-    if (er[q] >= 0) {
-      L[er[q]][ej[q]] = nv[q];
-      Li[ej[q]][er[q]] = nv[q];   // Li holds L^T until the inverse replaces it
-    }
-  __syncthreads();
-  {  // columns of L^-1: warp w takes j = w, 63 - w, 16 + w, 47 - w (130 substitution steps each)
-    const int w = tid >> 5, lane = tid & 31;
-    const int js[4] = {w, NB - 1 - w, 16 + w, 47 - w};
-    R x0[4], x1[4];   // rows lane and lane + 32 of the four columns
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      x0[u] = (lane == js[u]) ? R(1) : R(0);
-      x1[u] = (lane + 32 == js[u]) ? R(1) : R(0);
-    }
-    for (int i = w; i < NB; ++i) {
-      const R dinv = L[i][NB];
-      const R l0 = Li[i][lane], l1 = Li[i][lane + 32];   // L[lane][i], L[lane + 32][i]
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        if (i < js[u]) continue;
-        const R src = i < 32 ? x0[u] : x1[u];
-        const R xi = __shfl_sync(0xffffffffu, src, i & 31) * dinv;
-        if (lane == i) x0[u] = xi;
-        else if (lane > i) x0[u] = fma_r(-l0, xi, x0[u]);
-        if (lane + 32 == i) x1[u] = xi;
-        else if (lane + 32 > i) x1[u] = fma_r(-l1, xi, x1[u]);
-      }
-    }
-    __syncthreads();   // every warp has finished reading L^T from Li
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      Li[lane][js[u]] = x0[u];
-      Li[lane + 32][js[u]] = x1[u];
-    }
-  }
-  __syncthreads();
   store_diag(L, Li, Ab, Lb, t, k, kb);
   __syncthreads();
 }
@@ -336,7 +356,7 @@ __device__ __forceinline__ void st_acc(R* P, long long ld, int pn, int qn, const
       if (p < pn && q < qn) P[p * ld + q] = acc[p][q];
 }
 
-template <typename R>
+template <typename R, int kCL>
 __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     chol_cluster_kernel(R* A, R* Linv, R* B, R* Z, R* X, int t, int nrhs, int ldb, long long bbs, R ridge, R tdiv,
                         DevStatus* stt) {
@@ -458,7 +478,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     if (rank == 0 && tid == 0) ctr[(ep + 1) & 1] = 0;
     if (rank == (k + 1) % kCL) {
       if (k >= 0) update_tile(k, 0, ntri);
-      factor_diag(Ab, Lb, t, k + 1, lam, S1, S2, &bad);
+      factor_diag(Ab, Lb, t, k + 1, lam, S1, S2, S3, &bad);
     }
     for (;;) {
       const int x = 1 + next_tile();
@@ -517,9 +537,14 @@ template <typename R>
 static int cholesky_solve(int H, int t, R* Gram, R* Linv, R* B, R* Z, R* X, int ldb, int nrhs, long long bbs,
                           float ridge, DevStatus* stt, cudaStream_t st, int tdiv = 0) {
   const int smem = 3 * kTileF<R> * (int)sizeof(R);
-  cudaFuncSetAttribute(chol_cluster_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  chol_cluster_kernel<R><<<kCL * H, kCT, smem, st>>>(Gram, Linv, B, Z, X, t, nrhs, ldb, bbs, (R)ridge,
-                                                     (R)(tdiv > 0 ? tdiv : t), stt);
+  const R td = (R)(tdiv > 0 ? tdiv : t);
+  if (cluster_size(t) == 8) {
+    cudaFuncSetAttribute(chol_cluster_kernel<R, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    chol_cluster_kernel<R, 8><<<8 * H, kCT, smem, st>>>(Gram, Linv, B, Z, X, t, nrhs, ldb, bbs, (R)ridge, td, stt);
+  } else {
+    cudaFuncSetAttribute(chol_cluster_kernel<R, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    chol_cluster_kernel<R, 4><<<4 * H, kCT, smem, st>>>(Gram, Linv, B, Z, X, t, nrhs, ldb, bbs, (R)ridge, td, stt);
+  }
   return 1;
 }
 
