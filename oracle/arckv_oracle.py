@@ -28,6 +28,9 @@ Readings of points the paper leaves open (each is listed in the design doc):
 * both least-squares fits are solved with a ridge lam = ridge * tr(Gram)/t;
   ridge = 0 is the paper's unregularised solve for beta (Eq. mass_fit).
 * eps_w, b_min, b_max (unstated in Eq. mass_fit) default to e^-20, -20, 20.
+* the epsilon of the HA/VI selectors and of E(S) (App. B.1, unstated) is 1e-6;
+  the leave-one-out change of a row's dominant column is evaluated in its
+  exact algebraic form p_a ||v_a - O^(-a)|| (see leave_one_out_changes).
 * chunked selection (App. A.3, ``chunk_len`` > 0, T above 10,000) rounds
   t T_c / T half to even, in exact integer arithmetic.
 
@@ -44,7 +47,8 @@ import scipy.linalg
 __all__ = [
     "OracleConfig", "indexer_param_count", "rms_normalize", "value_context",
     "indexer_projections", "indexer_logits", "indexer_pool", "top_t", "CHUNK_THRESHOLD", "joint_compact_attention",
-    "round_half_even_ratio", "chunk_budgets", "anchor_count", "top_t_chunked",
+    "round_half_even_ratio", "chunk_budgets", "anchor_count", "top_t_chunked", "SELECTOR_EPS", "ha_scores",
+    "leave_one_out_changes", "vi_scores", "truncated_output_error",
     "attention_logits", "full_attention", "response_profiles", "response_profiles_literal",
     "assign_to_anchors", "log_mass_weights", "mass_weights_literal", "merge_keys", "fit_beta", "fit_values", "compact_attention",
     "hard_subset_attention", "output_loss", "mass_error", "compact_pair",
@@ -63,6 +67,7 @@ class OracleConfig:
     b_max: float = 20.0
     G: int = 4
     chunk_len: int = 0             # App. A.3 fixed chunking (0: global top-t)
+    selector: str = "indexer"      # "indexer" (Sec. 3.3), or "ha" / "vi" (App. B.1)
 
 
 # ---------------------------------------------------------------- indexer
@@ -307,6 +312,71 @@ def hard_subset_attention(Q, K, V, S, scale: float) -> np.ndarray:
     return _softmax_rows(attention_logits(Q, K[S], scale)) @ V[S]
 
 
+# ------------------------------------------------- HA / VI selectors, E(S)
+
+SELECTOR_EPS = 1e-6   # the epsilon of Eqs. background_value_selectors / background_truncated_error (unstated)
+
+
+def ha_scores(Q, K, scale: float) -> np.ndarray:
+    """App. B.1 Eq. (background_value_selectors): s^HA_j = (mean_i p_ij^2)^(1/2),
+    p = softmax(scale Q K^T)."""
+    P = _softmax_rows(attention_logits(Q, K, scale))
+    return np.sqrt(np.mean(P * P, axis=0))
+
+
+def leave_one_out_changes(Q, K, V, scale: float) -> np.ndarray:
+    """D_ij = ||O_i - O_i^(-j)|| = p_ij / (1 - p_ij) ||v_j - O_i|| (App. B.1), with
+    1 - p_ij = sum_{u != j} p_iu.  For the column a_i holding a row's largest
+    logit the same quantity is evaluated as p_ia ||v_a - O_i^(-a)|| (exact
+    algebra: O_i = p_ia v_a + (1 - p_ia) O_i^(-a)), O_i^(-a) being attention over
+    the other keys with its own max shift -- where p_ia rounds to 1 and v_a to
+    O_i, the printed form is 0 / 0 in any floating point."""
+    l = attention_logits(Q, K, scale)
+    n, T = l.shape
+    z = l.max(axis=1, keepdims=True)
+    e = np.exp(l - z)
+    msum = e.sum(axis=1, keepdims=True)
+    O = (e @ V) / msum
+    # non-dominant columns: p / (1 - p) = e / (sum_{u != j} e_u)
+    vv = np.sum(V * V, axis=1)[None, :]
+    oo = np.sum(O * O, axis=1)[:, None]
+    dist2 = np.maximum(vv - 2.0 * (O @ V.T) + oo, 0.0)
+    a = np.argmax(l, axis=1)
+    den = msum - e
+    den[np.arange(n), a] = 1.0          # the dominant columns are evaluated below
+    D = e / den * np.sqrt(dist2)
+    for i in range(n):
+        rest = np.delete(np.arange(T), a[i])
+        if rest.size == 0:
+            D[i, a[i]] = np.inf
+            continue
+        lr = l[i, rest]
+        z2 = lr.max()
+        er = np.exp(lr - z2)
+        O_minus = (er @ V[rest]) / er.sum()
+        p_a = 1.0 / (1.0 + er.sum() * np.exp(z2 - z[i, 0]))
+        D[i, a[i]] = p_a * np.linalg.norm(V[a[i]] - O_minus)
+    return D
+
+
+def vi_scores(Q, K, V, scale: float, eps: float = SELECTOR_EPS) -> np.ndarray:
+    """App. B.1 Eq. (background_value_selectors):
+    s^VI_j = (mean_i D_ij^2 / (||O_i||^2 + eps))^(1/2)."""
+    D = leave_one_out_changes(Q, K, V, scale)
+    O = full_attention(Q, K, V, scale)[1]
+    oo = np.sum(O * O, axis=1)[:, None]
+    return np.sqrt(np.mean(D * D / (oo + eps), axis=0))
+
+
+def truncated_output_error(Q_eval, K, V, S, scale: float, eps: float = SELECTOR_EPS) -> float:
+    """App. B.1 Eq. (background_truncated_error): O~_i(S) = sum_{j in S} p_ij v_j
+    with p, O from the full cache; E(S) = mean_i ||O_i - O~_i|| / (||O_i|| + eps)."""
+    P, O = full_attention(Q_eval, K, V, scale)
+    S = np.asarray(S, dtype=np.int64)
+    O_t = P[:, S] @ V[S]
+    return float(np.mean(np.linalg.norm(O - O_t, axis=1) / (np.linalg.norm(O, axis=1) + eps)))
+
+
 # ------------------------------------------------------------ diagnostics
 
 def output_loss(y_hat: np.ndarray, y: np.ndarray) -> float:
@@ -333,8 +403,13 @@ def compact_pair(K, V, Q, X_rows, W, cfg: OracleConfig, anchors_in: Optional[np.
     scale = cfg.scale if cfg.scale is not None else 1.0 / np.sqrt(d)
     out: Dict[str, np.ndarray] = {}
     if anchors_in is None:
-        I = indexer_logits(Q, X_rows, K, V, W, H_I, d_I)
-        _, s = indexer_pool(I)
+        if cfg.selector == "indexer":
+            I = indexer_logits(Q, X_rows, K, V, W, H_I, d_I)
+            _, s = indexer_pool(I)
+        elif cfg.selector == "ha":
+            s = ha_scores(Q, K, scale)
+        else:
+            s = vi_scores(Q, K, V, scale)
         S = top_t_chunked(s, cfg.t, cfg.chunk_len)
         out["scores"] = s
     else:

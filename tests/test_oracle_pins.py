@@ -478,6 +478,68 @@ def test_joint_attention_concatenation_and_bias():
                        oracle.full_attention(Q, Kf, Vf, sc)[1], rtol=1e-13, atol=1e-13)
 
 
+def _loo_brute(Q, K, V, sc):
+    """D_ij by removing key j and renormalising over the rest (App. B.1 definition)."""
+    n, T = Q.shape[0], K.shape[0]
+    _, O = oracle.full_attention(Q, K, V, sc)
+    D = np.zeros((n, T))
+    for j in range(T):
+        keep = [u for u in range(T) if u != j]
+        _, Oj = oracle.full_attention(Q, K[keep], V[keep], sc)
+        D[:, j] = np.linalg.norm(O - Oj, axis=1)
+    return D
+
+
+def test_leave_one_out_changes_brute_force_incl_dominant_keys():
+    rng = np.random.default_rng(8)
+    K, V, Q = rng.standard_normal((7, 4)), rng.standard_normal((7, 4)), rng.standard_normal((5, 4))
+    assert np.allclose(oracle.leave_one_out_changes(Q, K, V, 0.7), _loo_brute(Q, K, V, 0.7), rtol=1e-9, atol=1e-12)
+    # a dominant key: logit gaps near 60, where p rounds to 1 and the printed ratio is 0 / 0
+    K2 = K.copy()
+    K2[3] = 25.0 * Q[0] / np.linalg.norm(Q[0])
+    D = oracle.leave_one_out_changes(Q, K2, V, 1.0)
+    assert np.all(np.isfinite(D))
+    assert np.allclose(D, _loo_brute(Q, K2, V, 1.0), rtol=1e-9, atol=1e-12)
+
+
+def test_ha_vi_scores_closed_forms_and_brute_force():
+    rng = np.random.default_rng(9)
+    T = 6
+    K, V = rng.standard_normal((T, 4)), rng.standard_normal((T, 4))
+    # zero queries: uniform attention, s^HA = 1/T
+    assert np.allclose(oracle.ha_scores(np.zeros((3, 4)), K, 1.0), 1.0 / T, rtol=1e-14)
+    Q = rng.standard_normal((5, 4))
+    D = _loo_brute(Q, K, V, 0.5)
+    _, O = oracle.full_attention(Q, K, V, 0.5)
+    vi = np.sqrt(np.mean(D ** 2 / (np.sum(O ** 2, axis=1)[:, None] + oracle.SELECTOR_EPS), axis=0))
+    assert np.allclose(oracle.vi_scores(Q, K, V, 0.5), vi, rtol=1e-9)
+    P = np.exp(0.5 * Q @ K.T)
+    P /= P.sum(axis=1, keepdims=True)
+    assert np.allclose(oracle.ha_scores(Q, K, 0.5), [np.sqrt(np.mean([P[i, j] ** 2 for i in range(5)])) for j in range(T)])
+    # one key duplicated: two identical columns get identical scores
+    K3, V3 = np.vstack([K, K[1:2]]), np.vstack([V, V[1:2]])
+    assert oracle.ha_scores(Q, K3, 0.5)[1] == pytest.approx(oracle.ha_scores(Q, K3, 0.5)[T], rel=1e-12)
+    assert oracle.vi_scores(Q, K3, V3, 0.5)[1] == pytest.approx(oracle.vi_scores(Q, K3, V3, 0.5)[T], rel=1e-9)
+
+
+def test_truncated_output_error_closed_forms():
+    rng = np.random.default_rng(10)
+    K, V, Q = rng.standard_normal((9, 4)), rng.standard_normal((9, 4)), rng.standard_normal((6, 4))
+    assert oracle.truncated_output_error(Q, K, V, np.arange(9), 0.5) == pytest.approx(0.0, abs=1e-14)
+    _, O = oracle.full_attention(Q, K, V, 0.5)
+    no = np.linalg.norm(O, axis=1)
+    assert oracle.truncated_output_error(Q, K, V, np.array([], dtype=int), 0.5) == pytest.approx(
+        np.mean(no / (no + oracle.SELECTOR_EPS)), rel=1e-14)
+    S = [1, 4, 7]
+    err = []
+    for i in range(6):
+        a = 0.5 * K @ Q[i]
+        p = np.exp(a - a.max()); p /= p.sum()
+        o_t = sum(p[j] * V[j] for j in S)
+        err.append(np.linalg.norm(O[i] - o_t) / (np.linalg.norm(O[i]) + oracle.SELECTOR_EPS))
+    assert oracle.truncated_output_error(Q, K, V, S, 0.5) == pytest.approx(np.mean(err), rel=1e-12)
+
+
 def test_diagnostics():
     y = np.array([[3.0, 4.0]])
     assert oracle.output_loss(y * 1.1, y) == pytest.approx(0.01, rel=1e-12)
