@@ -92,12 +92,27 @@ typedef enum {
  *   ridge_w, ridge_v  >= 0: the beta and C_v normal matrices are solved as
  *             (Gram + lam I) with lam = ridge * trace(Gram) / t
  *   eps_w > 0, b_min <= b_max: the guards of Eq. mass_fit
+ * Anchor scores: selector (below).
  */
 typedef struct {
   int32_t H_kv, G, T, d, n_pos, d_x, H_I, d_I, d_A, t, chunk_len;
   float lambda_m, logit_scale, ridge_w, ridge_v, eps_w, b_min, b_max;
   uint32_t flags;
+  int32_t selector;
 } arckv_config;
+
+/* arckv_config.selector: how anchors are scored before top-t.
+ *   ARCKV_SELECTOR_INDEXER  the value-aware indexer (Sec. 3.3) -- ARC-KV
+ *   ARCKV_SELECTOR_HA       highest attention: s_j = (mean_i p_ij^2)^(1/2),
+ *                           p = softmax(logit_scale Q_ref K^T)          (App. B.1)
+ *   ARCKV_SELECTOR_VI       value influence: s_j = (mean_i D_ij^2 / (||O_i||^2 + 1e-6))^(1/2),
+ *                           D_ij = ||O_i - O_i^(-j)|| = p_ij / (1 - p_ij) ||v_j - O_i||,
+ *                           O = p V; needs T >= 2                      (App. B.1)
+ * HA and VI use no indexer weights and no X_ref (those pointers may be NULL);
+ * the rest of the path (assignment, merge, fits) is unchanged. */
+#define ARCKV_SELECTOR_INDEXER 0
+#define ARCKV_SELECTOR_HA 1
+#define ARCKV_SELECTOR_VI 2
 
 /*
  * Frozen indexer parameters of the H_kv heads of one layer, bf16, stacked

@@ -17,7 +17,7 @@ __all__ = [
     "Config", "ArckvError", "STATUS", "NUM_STAGES", "STAGE_NAMES", "load_library", "workspace_bytes", "anchor_count",
     "attend_workspace_bytes", "arckv_compact", "arckv_attend", "arckv_query_status", "status_string",
     "compact_layer", "attend", "INDEXER_FIELDS", "attend_joint", "arckv_attend_joint",
-    "attend_joint_workspace_bytes", "FLAG_COMPACT_BF16",
+    "attend_joint_workspace_bytes", "FLAG_COMPACT_BF16", "SELECTOR_INDEXER", "SELECTOR_HA", "SELECTOR_VI",
 ]
 
 _LIB_PATH = Path(__file__).resolve().parent / "libarckv.so"
@@ -30,6 +30,7 @@ STATUS = {
 }
 FLAG_NONBLOCKING = 0x1
 FLAG_COMPACT_BF16 = 0x2
+SELECTOR_INDEXER, SELECTOR_HA, SELECTOR_VI = 0, 1, 2
 NUM_STAGES = 6
 STAGE_NAMES = ("indexer_features", "index_logits", "pool_top_t", "refattn_assign", "merge", "fits")
 INDEXER_FIELDS = ("L_q", "L_k", "L_x", "b_x", "U_q", "U_k", "U_v", "L_c", "L_v")
@@ -46,7 +47,7 @@ class _Config(ctypes.Structure):
                  ("H_kv", "G", "T", "d", "n_pos", "d_x", "H_I", "d_I", "d_A", "t", "chunk_len")] +
                 [(n, ctypes.c_float) for n in
                  ("lambda_m", "logit_scale", "ridge_w", "ridge_v", "eps_w", "b_min", "b_max")] +
-                [("flags", ctypes.c_uint32)])
+                [("flags", ctypes.c_uint32), ("selector", ctypes.c_int32)])
 
 
 class _Indexer(ctypes.Structure):
@@ -80,6 +81,7 @@ class Config:
     b_min: float = -20.0
     b_max: float = 20.0
     flags: int = 0
+    selector: int = 0             # SELECTOR_INDEXER / SELECTOR_HA / SELECTOR_VI (App. B.1)
 
     @property
     def n(self) -> int:
@@ -88,7 +90,7 @@ class Config:
     def c_struct(self) -> _Config:
         return _Config(self.H_kv, self.G, self.T, self.d, self.n_pos, self.d_x, self.H_I, self.d_I, self.d_A,
                        self.t, self.chunk_len, self.lambda_m, self.logit_scale, self.ridge_w, self.ridge_v,
-                       self.eps_w, self.b_min, self.b_max, self.flags)
+                       self.eps_w, self.b_min, self.b_max, self.flags, self.selector)
 
 
 def load_library():

@@ -35,6 +35,8 @@ arckv_status validate(const arckv_config* c) {
   if (c->H_I < 1 || c->H_I > 16 || c->d_x < 8 || (c->d_x % 8) != 0) return ARCKV_ERR_SHAPE;
   if (c->d != 128 || c->d_I != 128 || c->d_A != 128) return ARCKV_ERR_UNSUPPORTED;
   if (c->chunk_len < 0) return ARCKV_ERR_INVALID_ARG;
+  if (c->selector < ARCKV_SELECTOR_INDEXER || c->selector > ARCKV_SELECTOR_VI) return ARCKV_ERR_INVALID_ARG;
+  if (c->selector == ARCKV_SELECTOR_VI && c->T < 2) return ARCKV_ERR_SHAPE;
   const int L = effective_chunk(c->T, c->chunk_len);
   if (L > 0 && (c->T + (long long)L - 1) / L > 65535) return ARCKV_ERR_SHAPE;   // chunks per head
   const long long tr = realized_anchors(c->T, c->t, c->chunk_len);
@@ -178,11 +180,12 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
                            const arckv_aux* aux, void* ws, size_t ws_bytes, void* stream) {
   arckv_status vs = validate(cfg);
   if (vs != ARCKV_OK) return vs;
-  if (!K || !V || !Q_ref || !X_ref || !idx || !C_k || !beta || !C_v) return ARCKV_ERR_INVALID_ARG;
+  if (!K || !V || !Q_ref || !C_k || !beta || !C_v) return ARCKV_ERR_INVALID_ARG;
   const bool given_anchors = aux && aux->anchors_in;
   const bool given_assign = aux && aux->assign_in;
   if (given_assign && !given_anchors) return ARCKV_ERR_INVALID_ARG;
-  if (!given_anchors && (!idx->L_q || !idx->L_k || !idx->L_x || !idx->b_x || !idx->U_q || !idx->U_k ||
+  const bool use_indexer = !given_anchors && cfg->selector == ARCKV_SELECTOR_INDEXER;
+  if (use_indexer && (!idx || !X_ref || !idx->L_q || !idx->L_k || !idx->L_x || !idx->b_x || !idx->U_q || !idx->U_k ||
                          !idx->U_v || !idx->L_c || !idx->L_v))
     return ARCKV_ERR_INVALID_ARG;
   const Layout L = plan(*cfg);
@@ -210,7 +213,37 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
   auto B16 = [&](size_t off) { return (bf16*)(w + off); };
   mark(0);
   nl += launch_transpose_v(D, Vb, B16(L.VT), st);
-  if (!given_anchors) {
+  // the reference attention (a5) does not depend on S: with the HA / VI
+  // selectors it runs first and its logits give the scores
+  bool ref_done = false;
+  auto reference_attention = [&]() -> int {
+    ref_done = true;
+    return launch_reference_attention(D, scale, Qb, Kb, B16(L.VT), F(L.NT), (float2*)(w + L.part), F(L.z), F(L.m),
+                                      F(L.invm), B16(L.p_h), B16(L.p_m), B16(L.p_l), F(L.Y), F(L.logphi),
+                                      F(L.colM), F(L.colInvN), stt, st);
+  };
+  if (!given_anchors && !use_indexer) {
+    mark(1);
+    mark(2);
+    const int nlr0 = reference_attention();
+    if (nlr0 < 0) return ARCKV_ERR_CUDA;
+    nl += nlr0;
+    if (cfg->selector == ARCKV_SELECTOR_HA) {
+      // p = softmax(l): the same pooling as the index scores, on l's row partials
+      nl += launch_index_pool(D, F(L.NT), (const float2*)(w + L.part), F(L.lse), F(L.s), st);
+    } else {
+      float* vq = F(L.vq);   // n-sized rows in the (unused) indexer buffers
+      const size_t hn = (size_t)D.H * D.n;
+      ViBufs VB{(int*)vq, vq + hn, vq + 2 * hn, vq + 3 * hn, vq + 4 * hn, F(L.qpp), F(L.best), F(L.Ut_hi),
+                B16(L.p_h), B16(L.p_m), B16(L.p_l), B16(L.q_h), B16(L.q_m), B16(L.q_l)};
+      const int nlv = launch_vi_scores(D, F(L.NT), F(L.z), F(L.m), F(L.Y), Vb, B16(L.VT), VB, F(L.s), 1e-6f, stt,
+                                       st);
+      if (nlv < 0) return ARCKV_ERR_CUDA;
+      nl += nlv;
+    }
+    nl += launch_top_t(D, cfg->t, F(L.s), anchors, stt, st);
+    nl += launch_check_anchors(D, anchors, stt, st);
+  } else if (!given_anchors) {
     const int nlk = launch_key_features_tc(D, Kb, Vb, (const bf16*)idx->L_k, (const bf16*)idx->L_v, B16(L.kbar_hi),
                                            B16(L.kbar_lo), stt, st);
     if (nlk < 0) return ARCKV_ERR_CUDA;
@@ -239,12 +272,11 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
     nl += launch_check_anchors(D, anchors, stt, st);
   }
   mark(3);
-  const int nlr = launch_reference_attention(D, scale, Qb, Kb, B16(L.VT), F(L.NT), (float2*)(w + L.part), F(L.z),
-                                             F(L.m), F(L.invm),
-                                             B16(L.p_h), B16(L.p_m), B16(L.p_l), F(L.Y), F(L.logphi), F(L.colM),
-                                             F(L.colInvN), stt, st);
-  if (nlr < 0) return ARCKV_ERR_CUDA;
-  nl += nlr;
+  if (!ref_done) {
+    const int nlr = reference_attention();
+    if (nlr < 0) return ARCKV_ERR_CUDA;
+    nl += nlr;
+  }
   int* kappa = I32(L.kappa);
   if (!given_assign) {
     const int nla = launch_assign_tc(D, F(L.NT), F(L.colM), F(L.colInvN), anchors, B16(L.Ut_hi), B16(L.Ut_lo),

@@ -57,7 +57,10 @@ int launch_value_logits_tc(const Dims& D, const float* qpp, bf16* q_h, bf16* q_m
                            float* logits, float2* part, DevStatus* stt, cudaStream_t st);
 // out [H][n][128] = (exp(X - shift) * mul) V over rows of X [H][n][T].
 int launch_probs_v_tc(const Dims& D, const float* X, const float* shift, const float* mul, bf16* p_h, bf16* p_m,
-                      bf16* p_l, const bf16* VT, float* out, DevStatus* stt, cudaStream_t st);
+                      bf16* p_l, const bf16* VT, float* out, DevStatus* stt, cudaStream_t st,
+                      const int* skip = nullptr);
+// x (count floats) -> bf16 triple h + m + l
+int launch_split3(const float* x, bf16* h, bf16* m, bf16* l, long long count, cudaStream_t st);
 // I (Eq. pairwise_index_score) on tcgen05 with split-bf16 operands, and the
 // per-(row, 128-column tile) softmax partials.  Returns launches, or -1 when a
 // TMA descriptor cannot be encoded.
@@ -105,6 +108,19 @@ int launch_check_finite(const float* x, long long count, DevStatus* stt, cudaStr
 // ---- compact attention (Eq. compact_attention) ----------------------------
 int launch_attend(int H, int n, int t, float scale, const bf16* Q, const float* C_k, const float* beta,
                   const float* C_v, float* O, float* LC, float* split, cudaStream_t st);
+
+// ---- HA / VI anchor scores (App. B.1) ----------------------------------
+// Scratch of launch_vi_scores: per row amax, z2, mul2, Da, oo [H][n]; O^(-a) Om
+// [H][n][128]; the split probabilities p_* [H][n][ldT] and Y's split y_*
+// [H][n][128]; vv [H][T]; colpart [H][ceil(n/32)][T].
+struct ViBufs {
+  int* amax;
+  float *z2, *mul2, *Da, *oo, *Om, *vv, *colpart;
+  bf16 *p_h, *p_m, *p_l, *y_h, *y_m, *y_l;
+};
+// s [H][T] = VI scores from the reference logits L, row stats z, m, Y = softmax(L) V.
+int launch_vi_scores(const Dims& D, const float* L, const float* z, const float* m, const float* Y, const bf16* V,
+                     const bf16* VT, const ViBufs& B, float* s, float eps, DevStatus* stt, cudaStream_t st);
 
 // ---- joint attention with an uncompressed block (App. A.7) -------------
 // Key splits of the split-key pass (deterministic in H, n, t, F).

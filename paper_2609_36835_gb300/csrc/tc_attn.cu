@@ -20,16 +20,17 @@ __global__ void split3_kernel(const float* x, bf16* h, bf16* m, bf16* l, long lo
 }
 
 // P = exp(X - shift_row) * mul_row as a bf16 triple [H][rows][ldc] (zero in the
-// pad columns cols..ldc-1).
-__global__ void probs_split3_kernel(const float* X, const float* shift, const float* mul, bf16* h, bf16* m, bf16* l,
-                                    int rows, int cols, int ldc) {
+// pad columns cols..ldc-1, and in column skip[row] when skip is given).
+__global__ void probs_split3_kernel(const float* X, const float* shift, const float* mul, const int* skip, bf16* h,
+                                    bf16* m, bf16* l, int rows, int cols, int ldc) {
   const int b = blockIdx.z, row = blockIdx.y;
   const long long rr = (long long)b * rows + row;
   const float sh = shift[rr], mu = mul[rr];
+  const int sk = skip ? skip[rr] : -1;
   const float* x = X + rr * cols;
   const long long o = rr * ldc;
   for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < ldc; c += gridDim.x * blockDim.x) {
-    const float p = (c < cols) ? expf(x[c] - sh) * mu : 0.f;
+    const float p = (c < cols && c != sk) ? expf(x[c] - sh) * mu : 0.f;
     split3_bf16(p, h[o + c], m[o + c], l[o + c]);
   }
 }
@@ -79,6 +80,11 @@ int launch_value_logits_tc(const Dims& D, const float* qpp, bf16* q_h, bf16* q_m
   return 2;
 }
 
+int launch_split3(const float* x, bf16* h, bf16* m, bf16* l, long long count, cudaStream_t st) {
+  split3_kernel<<<min(cdiv(count, 256), 152 * 8), 256, 0, st>>>(x, h, m, l, count);
+  return 1;
+}
+
 int launch_transpose_v(const Dims& D, const bf16* V, bf16* VT, cudaStream_t st) {
   const int ldT = (D.T + 7) / 8 * 8;
   transpose_v_kernel<<<dim3(cdiv(ldT, 32), 4, D.H), 256, 0, st>>>(V, VT, D.T, ldT);
@@ -86,10 +92,10 @@ int launch_transpose_v(const Dims& D, const bf16* V, bf16* VT, cudaStream_t st) 
 }
 
 int launch_probs_v_tc(const Dims& D, const float* X, const float* shift, const float* mul, bf16* p_h, bf16* p_m,
-                      bf16* p_l, const bf16* VT, float* out, DevStatus* stt, cudaStream_t st) {
+                      bf16* p_l, const bf16* VT, float* out, DevStatus* stt, cudaStream_t st, const int* skip) {
   const int ldT = (D.T + 7) / 8 * 8;
-  probs_split3_kernel<<<dim3(cdiv(ldT, 256 * 4), D.n, D.H), 256, 0, st>>>(X, shift, mul, p_h, p_m, p_l, D.n, D.T,
-                                                                          ldT);
+  probs_split3_kernel<<<dim3(cdiv(ldT, 256 * 4), D.n, D.H), 256, 0, st>>>(X, shift, mul, skip, p_h, p_m, p_l, D.n,
+                                                                          D.T, ldT);
   if (gemm_split3a(D.H, D.n, 128, ldT, ldT, p_h, p_m, p_l, VT, out, 128, 1.f, stt, st) < 0) return -1;
   return 2;
 }

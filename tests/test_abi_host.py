@@ -58,7 +58,8 @@ def test_workspace_bytes_sizes_and_rejections(lib):
 
 @pytest.mark.parametrize("kw,code", [
     (dict(t=9000), 2), (dict(T=0), 2), (dict(H_I=17), 2), (dict(d_x=4095), 2), (dict(d=64), 8),
-    (dict(chunk_len=-1), 1), (dict(T=1 << 20, chunk_len=8), 2), (dict(lambda_m=1.5), 1), (dict(ridge_w=-1.0), 1), (dict(eps_w=0.0), 1),
+    (dict(chunk_len=-1), 1), (dict(T=1 << 20, chunk_len=8), 2), (dict(selector=3), 1), (dict(selector=-1), 1),
+    (dict(selector=2, T=1, t=1), 2), (dict(lambda_m=1.5), 1), (dict(ridge_w=-1.0), 1), (dict(eps_w=0.0), 1),
     (dict(b_min=3.0, b_max=2.0), 1), (dict(flags=0x80), 1),
 ])
 def test_compact_rejects_bad_config_without_gpu(lib, kw, code):

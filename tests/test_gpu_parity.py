@@ -31,7 +31,8 @@ def _gpu(lib):
 def _ocfg(cfg: pk.Config):
     return oracle.OracleConfig(t=cfg.t, lambda_m=cfg.lambda_m, scale=(cfg.logit_scale or None),
                                ridge_w=cfg.ridge_w, ridge_v=cfg.ridge_v, eps_w=cfg.eps_w, b_min=cfg.b_min,
-                               b_max=cfg.b_max, G=cfg.G, chunk_len=cfg.chunk_len)
+                               b_max=cfg.b_max, G=cfg.G, chunk_len=cfg.chunk_len,
+                               selector={0: "indexer", 1: "ha", 2: "vi"}[cfg.selector])
 
 
 def _pair64(arr, h, G):
@@ -83,9 +84,19 @@ def check_layer(w, heads, sample, T=None, n_pos=None, t=None, layer=0, n_hold=64
     for h in sample:
         ref = refs[h]
         assert parity.rel_fro(_np(out2["C_k"][h]), ref["C_k"]) <= 2e-3
-        eb, rest_ok = parity.beta_errors(_np(out2["beta"][h]), ref["beta"], ref["w_star"])
-        assert eb <= 2e-3 and rest_ok, ("beta", h, eb, rest_ok)
-        assert parity.rel_fro(_np(out2["C_v"][h]), ref["C_v"]) <= 2e-3
+        if cfg.selector == pk.SELECTOR_INDEXER:
+            eb, rest_ok = parity.beta_errors(_np(out2["beta"][h]), ref["beta"], ref["w_star"])
+            assert eb <= 2e-3 and rest_ok, ("beta", h, eb, rest_ok)
+        else:   # ill-conditioned anchor sets: the mass weights e^beta (see oracle/parity.py)
+            em = parity.mass_weight_error(_np(out2["beta"][h]), ref["beta"])
+            assert em <= 2e-3, ("mass weights", h, em)
+        if cfg.selector == pk.SELECTOR_INDEXER:
+            assert parity.rel_fro(_np(out2["C_v"][h]), ref["C_v"]) <= 2e-3
+        else:   # stage-isolated: the oracle's C_v fit on the GPU's own beta
+            K_, V_, Q_, _, _ = _pair64(arr, h, cfg.G)
+            Cv_ref = oracle.fit_values(Q_, K_, V_, ref["C_k"], _np(out2["beta"][h]).astype(np.float64), _ocfg(cfg),
+                                       scale)["C_v"]
+            assert parity.rel_fro(_np(out2["C_v"][h]), Cv_ref) <= 2e-3
         O_ref = oracle.compact_attention(synth.bf16_to_f64(Qh[h]), ref["C_k"], ref["beta"], ref["C_v"], scale)
         assert parity.rel_fro(_np(O[h]), O_ref) <= 2e-3
         K, V, Q, Xr, W = _pair64(arr, h, cfg.G)
@@ -150,6 +161,20 @@ def test_chunked_selection_ragged_last_chunk():
 def test_chunked_selection_one_anchor_per_chunk():
     """Budgets clipped up to one anchor per chunk: T = 12000, chunks of 4096, t = 3."""
     check_layer(synth.WORKLOADS["llama8b_layer_T8192"], [1], [0], T=12000, n_pos=20, t=3, chunk_len=4096)
+
+
+@pytest.mark.parametrize("selector", [pk.SELECTOR_HA, pk.SELECTOR_VI])
+def test_ha_vi_selectors_small(selector):
+    """App. B.1 selectors on the small workload, ragged shapes: scores, anchors
+    (tie-aware) and the downstream stages on the oracle's anchors."""
+    check_layer(synth.WORKLOADS["single_head_T1024"], [0], [0], selector=selector)
+    check_layer(synth.WORKLOADS["llama8b_layer_T8192"], [1, 4], [0, 1], T=1000, n_pos=50, t=77, selector=selector)
+
+
+@pytest.mark.parametrize("selector", [pk.SELECTOR_HA, pk.SELECTOR_VI])
+def test_ha_vi_selectors_full_layer_sampled_heads(selector):
+    """HA / VI on a full Llama layer (8 heads, T = 8192, n = 1024, t = 819); oracle on two heads."""
+    check_layer(synth.WORKLOADS["llama8b_layer_T8192"], list(range(8)), [2, 6], selector=selector)
 
 
 def test_odd_shapes_single_index_head():
