@@ -226,6 +226,24 @@ arckv_status arckv_attend_joint(int32_t H, int32_t n, int32_t t, int32_t F, int3
                                 const void* K_fixed, const void* V_fixed, float* O, void* ws, size_t ws_bytes,
                                 uint32_t flags, void* stream);
 
+/* Workspace bytes of arckv_truncated_error (0 if the sizes are invalid). Host-only. */
+size_t arckv_truncated_error_workspace_bytes(int32_t H, int32_t n, int32_t T, int32_t t, int32_t d);
+
+/*
+ * Truncated-output error of anchor sets (App. B.1 Eq. background_truncated_error),
+ * the held-out measure by which selectors are compared:
+ *   p = softmax(logit_scale Q_eval[h] K[h]^T) over the full cache, O = p V,
+ *   O~_i(S) = sum_{j in S[h]} p_ij v_j,
+ *   E[h] = mean_i ||O_i - O~_i(S)|| / (||O_i|| + 1e-6)
+ *   Q_eval bf16 [H][n][d]; K, V bf16 [H][T][d] (16-byte aligned);
+ *   S int32 [H][t] distinct positions in [0, T) (t = 0: empty sets);
+ *   E out fp32 [H].  d == 128.  `flags` takes ARCKV_FLAG_NONBLOCKING;
+ *   out-of-range positions record ARCKV_ERR_INVALID_ARG (and are clamped).
+ */
+arckv_status arckv_truncated_error(int32_t H, int32_t n, int32_t T, int32_t t, int32_t d, float logit_scale,
+                                   const void* Q_eval, const void* K, const void* V, const int32_t* S, float* E,
+                                   void* ws, size_t ws_bytes, uint32_t flags, void* stream);
+
 /*
  * Allocation-free compact attention.  The paper has no counterpart: this is a
  * deployment variant of arckv_attend for callers that cannot allocate device

@@ -17,7 +17,7 @@ __all__ = [
     "Config", "ArckvError", "STATUS", "NUM_STAGES", "STAGE_NAMES", "load_library", "workspace_bytes", "anchor_count",
     "attend_workspace_bytes", "arckv_compact", "arckv_attend", "arckv_query_status", "status_string",
     "compact_layer", "attend", "INDEXER_FIELDS", "attend_joint", "arckv_attend_joint",
-    "attend_joint_workspace_bytes", "FLAG_COMPACT_BF16", "SELECTOR_INDEXER", "SELECTOR_HA", "SELECTOR_VI",
+    "attend_joint_workspace_bytes", "FLAG_COMPACT_BF16", "truncated_error", "arckv_truncated_error", "SELECTOR_INDEXER", "SELECTOR_HA", "SELECTOR_VI",
 ]
 
 _LIB_PATH = Path(__file__).resolve().parent / "libarckv.so"
@@ -120,6 +120,11 @@ def load_library():
     lib.arckv_attend_joint.argtypes = [ctypes.c_int32] * 5 + [ctypes.c_float] + [P] * 8 + [ctypes.c_size_t,
                                                                                          ctypes.c_uint32, P]
     lib.arckv_attend_joint.restype = ctypes.c_int
+    lib.arckv_truncated_error_workspace_bytes.argtypes = [ctypes.c_int32] * 5
+    lib.arckv_truncated_error_workspace_bytes.restype = ctypes.c_size_t
+    lib.arckv_truncated_error.argtypes = [ctypes.c_int32] * 5 + [ctypes.c_float] + [P] * 5 + [P, ctypes.c_size_t,
+                                                                                              ctypes.c_uint32, P]
+    lib.arckv_truncated_error.restype = ctypes.c_int
     lib.arckv_query_status.argtypes = [P, P]
     lib.arckv_query_status.restype = ctypes.c_int
     lib.arckv_status_string.argtypes = [ctypes.c_int]
@@ -206,6 +211,14 @@ def arckv_attend_joint(H: int, n: int, t: int, F: int, d: int, logit_scale: floa
                                       _stream_handle(stream)))
 
 
+def arckv_truncated_error(H: int, n: int, T: int, t: int, d: int, logit_scale: float, Q_eval, K, V, S, E, ws,
+                          ws_bytes: int, flags: int = 0, stream=None) -> int:
+    """Direct binding of ``arckv_truncated_error``; returns the status code."""
+    lib = load_library()
+    return int(lib.arckv_truncated_error(H, n, T, t, d, float(logit_scale), _ptr(Q_eval), _ptr(K), _ptr(V), _ptr(S),
+                                         _ptr(E), _ptr(ws), int(ws_bytes), int(flags), _stream_handle(stream)))
+
+
 def arckv_query_status(ws, stream=None) -> int:
     return int(load_library().arckv_query_status(_ptr(ws), _stream_handle(stream)))
 
@@ -290,3 +303,20 @@ def attend_joint(Q, C_k=None, beta=None, C_v=None, K_fixed=None, V_fixed=None, l
     if check and st != 0:
         raise ArckvError(st, "arckv_attend_joint")
     return O
+
+
+def truncated_error(Q_eval, K, V, S, logit_scale: float = 0.0, *, stream=None, check: bool = True):
+    """E(S) per head (App. B.1) for Q_eval [H, n, 128], K, V [H, T, 128] bf16 and anchors S [H, t] int32."""
+    import torch
+    H, n, d = Q_eval.shape
+    T = K.shape[1]
+    t = 0 if S is None else S.shape[1]
+    need = int(load_library().arckv_truncated_error_workspace_bytes(H, n, T, t, d))
+    if need == 0:
+        raise ArckvError(2, "arckv_truncated_error_workspace_bytes")
+    ws = _alloc_ws(need, Q_eval.device)
+    E = torch.empty(H, dtype=torch.float32, device=Q_eval.device)
+    st = arckv_truncated_error(H, n, T, t, d, logit_scale, Q_eval, K, V, S, E, ws, ws.numel(), stream=stream)
+    if check and st != 0:
+        raise ArckvError(st, "arckv_truncated_error")
+    return E

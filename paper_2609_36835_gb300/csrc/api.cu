@@ -391,4 +391,37 @@ arckv_status arckv_attend_joint(int32_t H, int32_t n, int32_t t, int32_t F, int3
   return read_status(ws, st);
 }
 
+size_t arckv_truncated_error_workspace_bytes(int32_t H, int32_t n, int32_t T, int32_t t, int32_t d) {
+  if (H < 1 || n < 1 || T < 1 || t < 0 || t > T || d != 128) return 0;
+  if ((long long)H * T >= (1LL << 40) || (long long)H * n >= (1LL << 31) || cdiv(n, 4) > 65535 || H > 65535) return 0;
+  return up(sizeof(DevStatus)) + up((size_t)H * T) + up((size_t)H * n * 4);
+}
+
+arckv_status arckv_truncated_error(int32_t H, int32_t n, int32_t T, int32_t t, int32_t d, float logit_scale,
+                                   const void* Q_eval, const void* K, const void* V, const int32_t* S, float* E,
+                                   void* ws, size_t ws_bytes, uint32_t flags, void* stream) {
+  if (flags & ~ARCKV_FLAG_NONBLOCKING) return ARCKV_ERR_INVALID_ARG;
+  if (d != 128) return ARCKV_ERR_UNSUPPORTED;
+  const size_t need = arckv_truncated_error_workspace_bytes(H, n, T, t, d);
+  if (need == 0) return ARCKV_ERR_SHAPE;
+  if (!Q_eval || !K || !V || !E || (t > 0 && !S)) return ARCKV_ERR_INVALID_ARG;
+  if ((((uintptr_t)K) % 16) || (((uintptr_t)V) % 16)) return ARCKV_ERR_INVALID_ARG;
+  if (!(logit_scale >= 0.f) || !isfinite(logit_scale)) return ARCKV_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < need || ((uintptr_t)ws % kAlign) != 0) return ARCKV_ERR_WORKSPACE;
+  cudaStream_t st = (cudaStream_t)stream;
+  char* w = (char*)ws;
+  DevStatus* stt = (DevStatus*)w;
+  unsigned char* inS = (unsigned char*)(w + up(sizeof(DevStatus)));
+  float* err = (float*)(w + up(sizeof(DevStatus)) + up((size_t)H * T));
+  const float scale = logit_scale > 0.f ? logit_scale : 1.0f / sqrtf((float)d);
+  cudaGetLastError();
+  if (cudaMemsetAsync(stt, 0, sizeof(DevStatus), st) != cudaSuccess) return ARCKV_ERR_CUDA;
+  launch_truncated_error(H, n, T, t, scale, 1e-6f, (const bf16*)Q_eval, (const bf16*)K, (const bf16*)V, S, E, inS,
+                         err, stt, st);
+  launch_check_finite(E, H, stt, st);
+  if (cudaGetLastError() != cudaSuccess) return ARCKV_ERR_CUDA;
+  if (flags & ARCKV_FLAG_NONBLOCKING) return ARCKV_OK;
+  return read_status(ws, st);
+}
+
 }  // extern "C"

@@ -482,6 +482,163 @@ __global__ void __launch_bounds__(256) attend_combine_kernel(const float* Opart,
   *(float4*)(O + g * 128 + lane * 4) = make_float4(o0 * inv, o1 * inv, o2 * inv, o3 * inv);
 }
 
+// ---------------------------------------------------------------------------
+// Truncated-output error of an anchor set (App. B.1 Eq. background_truncated_error):
+//   O_i = sum_j p_ij v_j, O~_i(S) = sum_{j in S} p_ij v_j (p over the full cache),
+//   err_i = ||O_i - O~_i|| / (||O_i|| + eps).
+// One CTA per (4-row block, head) makes one pass over the keys: the logits and
+// online softmax of attend_tiles, and two value accumulators (all keys; keys in S).
+__global__ void __launch_bounds__(kJThreads) trunc_err_kernel(const bf16* Q, int n, const bf16* K, const bf16* V,
+                                                              int T, const unsigned char* inS, float scale, float eps,
+                                                              float* err) {
+  const int h = blockIdx.y, r0 = blockIdx.x * kJR;
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  __shared__ __align__(16) float sQ[kJR][128];
+  __shared__ float sP[kJR][kJTile];
+  __shared__ float sM[kJR], sL[kJR], sF[kJR];
+  __shared__ __align__(16) float sAcc[2][kJThreads / 32][kJR][128];
+  const bf16* Kh = K + (long long)h * T * 128;
+  const bf16* Vh = V + (long long)h * T * 128;
+  const unsigned char* mh = inS + (long long)h * T;
+  for (int e = tid; e < kJR * 128; e += kJThreads) {
+    const int r = e >> 7, dd = e & 127;
+    sQ[r][dd] = (r0 + r < n) ? scale * __bfloat162float(Q[((long long)h * n + r0 + r) * 128 + dd]) : 0.f;
+  }
+  if (tid < kJR) {
+    sM[tid] = -INFINITY;
+    sL[tid] = 0.f;
+  }
+  float acc[kJR][4], accs[kJR][4];
+#pragma unroll
+  for (int r = 0; r < kJR; ++r)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) acc[r][q] = accs[r][q] = 0.f;
+  __syncthreads();
+  for (int j0 = 0; j0 < T; j0 += kJTile) {
+    {
+      const int jj = tid >> 2, p = tid & 3, j = j0 + jj;
+      KSlice32H k;
+      if (j < T) k.load(Kh + (long long)j * 128 + p * 32);
+      else k.zero();
+      float part[kJR];
+#pragma unroll
+      for (int r = 0; r < kJR; ++r) {
+        float a = k.dot((const float4*)&sQ[r][p * 32]);
+        a += __shfl_xor_sync(0xffffffffu, a, 1);
+        a += __shfl_xor_sync(0xffffffffu, a, 2);
+        part[r] = a;
+      }
+      if (p == 0) {
+#pragma unroll
+        for (int r = 0; r < kJR; ++r) sP[r][jj] = (j < T) ? part[r] : -INFINITY;
+      }
+    }
+    __syncthreads();
+    if (w < kJR) {
+      const float a0 = sP[w][lane], a1 = sP[w][lane + 32];
+      const float mold = sM[w], mnew = fmaxf(mold, warp_max(fmaxf(a0, a1)));
+      const float e0 = expf(a0 - mnew), e1 = expf(a1 - mnew);
+      sP[w][lane] = e0;
+      sP[w][lane + 32] = e1;
+      const float ssum = warp_sum(e0 + e1);
+      if (lane == 0) {
+        const float f = expf(mold - mnew);
+        sF[w] = f;
+        sL[w] = sL[w] * f + ssum;
+        sM[w] = mnew;
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int r = 0; r < kJR; ++r) {
+      const float f = sF[r];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        acc[r][q] *= f;
+        accs[r][q] *= f;
+      }
+    }
+    for (int i = 0; i < kJTile / 8; ++i) {
+      const int jj = w + 8 * i, j = j0 + jj;
+      if (j < T) {
+        float v[4];
+        load4(Vh + (long long)j * 128 + lane * 4, v);
+        const bool in = mh[j] != 0;
+#pragma unroll
+        for (int r = 0; r < kJR; ++r) {
+          const float pr = sP[r][jj];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            acc[r][q] = fmaf(pr, v[q], acc[r][q]);
+            if (in) accs[r][q] = fmaf(pr, v[q], accs[r][q]);
+          }
+        }
+      }
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int r = 0; r < kJR; ++r) {
+    *(float4*)&sAcc[0][w][r][lane * 4] = make_float4(acc[r][0], acc[r][1], acc[r][2], acc[r][3]);
+    *(float4*)&sAcc[1][w][r][lane * 4] = make_float4(accs[r][0], accs[r][1], accs[r][2], accs[r][3]);
+  }
+  __syncthreads();
+  if (w < kJR && r0 + w < n) {   // warp r: row r's norms over its 128 dims
+    const int r = w;
+    const float inv = 1.0f / sL[r];
+    float dd = 0.f, oo = 0.f;
+    for (int c = lane; c < 128; c += 32) {
+      float o = 0.f, os = 0.f;
+#pragma unroll
+      for (int q = 0; q < kJThreads / 32; ++q) {
+        o += sAcc[0][q][r][c];
+        os += sAcc[1][q][r][c];
+      }
+      o *= inv;
+      os *= inv;
+      dd = fmaf(o - os, o - os, dd);
+      oo = fmaf(o, o, oo);
+    }
+    dd = warp_sum(dd);
+    oo = warp_sum(oo);
+    if (lane == 0) err[(long long)h * n + r0 + r] = sqrtf(dd) / (sqrtf(oo) + eps);
+  }
+}
+
+// inS[h][j] = 1 for the anchors S[h][:] (clamped into [0, T); out-of-range entries record INVALID_ARG)
+__global__ void anchor_mask_kernel(const int* S, int t, int T, int H, unsigned char* inS, DevStatus* stt) {
+  for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < (long long)H * t;
+       k += (long long)gridDim.x * blockDim.x) {
+    const long long h = k / t;
+    int j = S[k];
+    if (j < 0 || j >= T) {
+      set_status(stt, ARCKV_ERR_INVALID_ARG);
+      j = min(max(j, 0), T - 1);
+    }
+    inS[h * T + j] = 1;
+  }
+}
+
+// E[h] = mean_i err[h][i] (fixed order)
+__global__ void row_mean_kernel(const float* err, int n, int H, float* E) {
+  const int h = blockIdx.x * blockDim.x + threadIdx.x;
+  if (h >= H) return;
+  float a = 0.f;
+  for (int i = 0; i < n; ++i) a += err[(long long)h * n + i];
+  E[h] = a / (float)n;
+}
+
+int launch_truncated_error(int H, int n, int T, int t, float scale, float eps, const bf16* Q, const bf16* K,
+                           const bf16* V, const int* S, float* E, unsigned char* inS, float* err, DevStatus* stt,
+                           cudaStream_t st) {
+  cudaMemsetAsync(inS, 0, (size_t)H * T, st);
+  if (t > 0)
+    anchor_mask_kernel<<<std::min(cdiv((long long)H * t, 256), 152 * 4), 256, 0, st>>>(S, t, T, H, inS, stt);
+  trunc_err_kernel<<<dim3(cdiv(n, kJR), H), kJThreads, 0, st>>>(Q, n, K, V, T, inS, scale, eps, err);
+  row_mean_kernel<<<cdiv(H, 128), 128, 0, st>>>(err, n, H, E);
+  return 3;
+}
+
 JointSplit joint_split(int H, int n, int t, int F) {
   JointSplit s;
   const int L = t + F, rb = cdiv(n, kJR);

@@ -110,6 +110,11 @@ int launch_attend(int H, int n, int t, float scale, const bf16* Q, const float* 
                   const float* C_v, float* O, float* LC, float* split, cudaStream_t st);
 
 // ---- HA / VI anchor scores (App. B.1) ----------------------------------
+// E[h] = mean_i ||O_i - O~_i(S)|| / (||O_i|| + eps) (Eq. background_truncated_error);
+// scratch inS [H][T] bytes, err [H][n].
+int launch_truncated_error(int H, int n, int T, int t, float scale, float eps, const bf16* Q, const bf16* K,
+                           const bf16* V, const int* S, float* E, unsigned char* inS, float* err, DevStatus* stt,
+                           cudaStream_t st);
 // Scratch of launch_vi_scores: per row amax, z2, mul2, Da, oo [H][n]; O^(-a) Om
 // [H][n][128]; the split probabilities p_* [H][n][ldT] and Y's split y_*
 // [H][n][128]; vv [H][T]; colpart [H][ceil(n/32)][T].

@@ -132,3 +132,31 @@ def test_decode_batch_full_size_sampled_heads():
         assert parity.rel_fro(O_full[h].cpu().numpy(), ref_full) <= TOL
         ref_c = oracle.compact_attention(Q, f(d["C_k"]), f(d["beta"]), f(d["C_v"]), SC)
         assert parity.rel_fro(O_comp[h].cpu().numpy(), ref_c) <= TOL
+
+
+@pytest.mark.parametrize("layer_heads,T,n_pos,t", [((0, [0, 3]), 1000, 50, 77), ((2, list(range(8))), 8192, 256, 819)])
+def test_truncated_output_error_of_the_three_selectors(layer_heads, T, n_pos, t):
+    """E(S) (App. B.1) on held-out queries for the anchor sets of the indexer,
+    HA and VI selectors, against the oracle (relative 1e-4)."""
+    layer, heads = layer_heads
+    w = synth.WORKLOADS["llama8b_layer_T8192"]
+    arr = workload.layer_inputs_np(w, layer, heads, T=T, n_pos=n_pos)
+    ten = workload.to_device(arr, "cuda")
+    Qh = np.stack([synth.make_heldout(w, layer, h, arr["K"][i], 64) for i, h in enumerate(heads)])
+    Qt = workload.bf16_tensor(Qh, "cuda")
+    results = {}
+    for sel in (pk.SELECTOR_INDEXER, pk.SELECTOR_HA, pk.SELECTOR_VI):
+        cfg = workload.layer_config(w, len(heads), T=T, n_pos=n_pos, t=t, selector=sel)
+        out = pk.compact_layer(cfg, ten["K"], ten["V"], ten["Q"], ten["X"], workload.indexer_dict(ten))
+        E = pk.truncated_error(Qt, ten["K"], ten["V"], out["anchors"]).cpu().numpy()
+        S = out["anchors"].cpu().numpy()
+        for i in (0, len(heads) - 1):
+            ref = oracle.truncated_output_error(synth.bf16_to_f64(Qh[i]), synth.bf16_to_f64(arr["K"][i]),
+                                                synth.bf16_to_f64(arr["V"][i]), S[i], SC)
+            assert abs(E[i] - ref) <= 1e-4 * ref, (sel, i, E[i], ref)
+        results[sel] = E
+    # empty and full sets: E = mean ||O|| / (||O|| + eps) ~ 1 and E = 0
+    Sall = torch.arange(T, dtype=torch.int32, device="cuda").repeat(len(heads), 1)
+    assert np.all(pk.truncated_error(Qt, ten["K"], ten["V"], Sall).cpu().numpy() < 1e-5)
+    E0 = pk.truncated_error(Qt, ten["K"], ten["V"], None).cpu().numpy()
+    assert np.allclose(E0, 1.0, atol=1e-5)
