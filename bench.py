@@ -68,6 +68,11 @@ def parse_args(argv=None):
                     help="CUDA streams (each with its own workspace) the layers of a context are spread over")
     ap.add_argument("--cpu-pairs", type=int, default=4, help="(layer, head) pairs the oracle baseline times")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--selector", choices=("indexer", "ha", "vi"), default="indexer",
+                    help="anchor scores: the ARC-KV indexer (default) or the HA / VI selectors of App. B.1")
+    ap.add_argument("--chunk-len", type=int, default=0, help="App. A.3 chunked selection (0: global top-t)")
+    ap.add_argument("--eval-selectors", action="store_true",
+                    help="held-out truncated-output error E(S) of the three selectors on one layer (App. B.1)")
     ap.add_argument("--decode", action="store_true",
                     help="time one decode step of attention (App. D shape) instead of the compaction")
     ap.add_argument("--decode-contexts", default="4096,8192,16384,32768")
@@ -195,7 +200,7 @@ def blas_threads() -> int:
     return len(os.sched_getaffinity(0))
 
 
-def oracle_pair_seconds(w, pairs):
+def oracle_pair_seconds(w, pairs, selector="indexer", chunk_len=0):
     """Time the fp64 oracle (as it stands) on (layer, head) pairs at full size."""
     import numpy as np
     import oracle
@@ -209,7 +214,7 @@ def oracle_pair_seconds(w, pairs):
         K, V, Q = f64(p["K"]), f64(p["V"]), f64(p["Q"])
         Xr = np.repeat(f64(X), w.G, axis=0)
         t0 = time.perf_counter()
-        oracle.compact_pair(K, V, Q, Xr, W, oracle.OracleConfig(t=w.t))
+        oracle.compact_pair(K, V, Q, Xr, W, oracle.OracleConfig(t=w.t, selector=selector, chunk_len=chunk_len))
         times.append(time.perf_counter() - t0)
     return times
 
@@ -236,8 +241,8 @@ def run_reference(args, dist: Dist):
     w = synth.WORKLOADS[args.workload]
     pairs = [(l, h) for l in range(w.layers) for h in range(w.H_kv)]
     pick = [pairs[(i * 37) % len(pairs)] for i in range(args.warmup + args.steps)]
-    oracle_pair_seconds(w, pick[:args.warmup])
-    times = oracle_pair_seconds(w, pick[args.warmup:])
+    oracle_pair_seconds(w, pick[:args.warmup], args.selector, args.chunk_len)
+    times = oracle_pair_seconds(w, pick[args.warmup:], args.selector, args.chunk_len)
     per_pair = statistics.mean(times)
     s_ctx = per_pair * len(pairs)
     value = w.T / s_ctx
@@ -281,8 +286,9 @@ def run_gpu(args, dist: Dist):
     layers = context_layers(w.layers, dist.rank)
     if args.profile_layer:
         layers = layers[:1]
-    cfg = workload.layer_config(w, w.H_kv, flags=pk.FLAG_NONBLOCKING)
-    cfg_block = workload.layer_config(w, w.H_kv)
+    sel = {"indexer": pk.SELECTOR_INDEXER, "ha": pk.SELECTOR_HA, "vi": pk.SELECTOR_VI}[args.selector]
+    cfg = workload.layer_config(w, w.H_kv, flags=pk.FLAG_NONBLOCKING, selector=sel, chunk_len=args.chunk_len)
+    cfg_block = workload.layer_config(w, w.H_kv, selector=sel, chunk_len=args.chunk_len)
 
     host = [workload.layer_inputs_np(w, l, list(range(w.H_kv))) for l in layers]
     dev_in = [workload.to_device(a, dev) for a in host]
@@ -291,8 +297,9 @@ def run_gpu(args, dist: Dist):
     n_str = max(1, min(args.streams, len(layers)))
     wss = [torch.empty(pk.workspace_bytes(cfg), dtype=torch.uint8, device=dev) for _ in range(n_str)]
     f32 = dict(dtype=torch.float32, device=dev)
-    outs = [{"C_k": torch.empty(w.H_kv, w.t, 128, **f32), "beta": torch.empty(w.H_kv, w.t, **f32),
-             "C_v": torch.empty(w.H_kv, w.t, 128, **f32)} for _ in layers]
+    tp = pk.anchor_count(cfg)   # = w.t without chunking
+    outs = [{"C_k": torch.empty(w.H_kv, tp, 128, **f32), "beta": torch.empty(w.H_kv, tp, **f32),
+             "C_v": torch.empty(w.H_kv, tp, 128, **f32)} for _ in layers]
     stream = torch.cuda.current_stream(dev)
     streams = [stream] + [torch.cuda.Stream(dev) for _ in range(n_str - 1)]
 
@@ -449,8 +456,8 @@ def run_gpu(args, dist: Dist):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded Llama-3.1-8B-shaped caches)",
-        "config": workload_config(w, "inputs larger than L2 (%.2f GB per context)" %
-                                  (h2d / 1e9)),
+        "config": dict(workload_config(w, "inputs larger than L2 (%.2f GB per context)" % (h2d / 1e9)),
+                       selector=args.selector, chunk_len=args.chunk_len, anchors_per_head=tp),
         "s_per_context": ms_step / 1e3,
         "streams": n_str,
         "stage_ms_per_step": dict(zip(pk.STAGE_NAMES, stage_ms)),
@@ -464,7 +471,7 @@ def run_gpu(args, dist: Dist):
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
         spread = [(0, 0), (w.layers - 1, w.H_kv - 1), (w.layers // 2, 3 % w.H_kv), (w.layers // 4, 5 % w.H_kv)]
         pairs = spread[:max(1, min(len(spread), args.cpu_pairs))]
-        times = oracle_pair_seconds(w, pairs)
+        times = oracle_pair_seconds(w, pairs, args.selector, args.chunk_len)
         per_pair = statistics.mean(times)
         n_pairs = w.layers * w.H_kv
         line["cpu_baseline"] = {
@@ -563,6 +570,44 @@ def run_decode(args, dist: Dist):
     return 0
 
 
+def run_eval_selectors(args, dist: Dist):
+    """App. B.1 on synthetic caches: compact one layer with each selector, then
+    the held-out truncated-output error E(S) of each anchor set (64 held-out
+    queries per head, drawn like the reference queries)."""
+    import numpy as np
+    import torch
+    import synth
+    import paper_2609_36835_gb300 as pk
+    from paper_2609_36835_gb300 import workload
+
+    if dist.rank != 0:
+        return 0
+    torch.cuda.set_device(0)
+    pk.load_library()
+    w = synth.WORKLOADS[args.workload]
+    rows = {}
+    for layer in (0, w.layers // 2, w.layers - 1):
+        heads = list(range(w.H_kv))
+        arr = workload.layer_inputs_np(w, layer, heads)
+        ten = workload.to_device(arr, "cuda")
+        Qh = np.stack([synth.make_heldout(w, layer, h, arr["K"][i], 64) for i, h in enumerate(heads)])
+        Qt = workload.bf16_tensor(Qh, "cuda")
+        for name, sel in (("indexer", pk.SELECTOR_INDEXER), ("ha", pk.SELECTOR_HA), ("vi", pk.SELECTOR_VI)):
+            cfg = workload.layer_config(w, w.H_kv, selector=sel)
+            out = pk.compact_layer(cfg, ten["K"], ten["V"], ten["Q"], ten["X"], workload.indexer_dict(ten))
+            E = pk.truncated_error(Qt, ten["K"], ten["V"], out["anchors"]).cpu().numpy()
+            rows.setdefault(name, []).extend(float(x) for x in E)
+    mean = {k: float(np.mean(v)) for k, v in rows.items()}
+    line = {"metric": "held-out truncated-output error E(S), App. B.1 (lower is better)", "unit": "relative error",
+            "higher_is_better": False, "config": {"workload": args.workload, "layers": [0, w.layers // 2, w.layers - 1],
+                                                  "heads": w.H_kv, "t": w.t, "held_out_queries": 64},
+            "data": "synthetic (seeded Llama-3.1-8B-shaped caches)",
+            "E_mean": mean, "E_per_pair": rows,
+            "vi_vs_ha_relative_reduction": (mean["ha"] - mean["vi"]) / mean["ha"]}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main(argv=None):
     args = parse_args(argv)
     if args.warmup < 3 and not args.profile_layer:
@@ -572,6 +617,8 @@ def main(argv=None):
         return run_reference(args, dist)
     if args.decode:
         return run_decode(args, dist)
+    if args.eval_selectors:
+        return run_eval_selectors(args, dist)
     return run_gpu(args, dist)
 
 
