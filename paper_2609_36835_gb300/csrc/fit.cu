@@ -29,15 +29,33 @@ __global__ void phi_kernel(const float* LC, const float* z, float* Phi, int n, i
   }
 }
 
-// rhs[b][r] = sum_i Phi[b][i][r] m[b][i]   (Phi_C^T Phi_K 1)
-__global__ void mass_rhs_kernel(const float* Phi, const float* m, float* rhs, int n, int t) {
-  const int b = blockIdx.y, r = blockIdx.x * blockDim.x + threadIdx.x;
-  if (r >= t) return;
+// rhs[b][r] = sum_i Phi[b][i][r] m[b][i]   (Phi_C^T Phi_K 1).  A CTA owns 32
+// columns; warp w sums the rows i = w, w+8, ... (four partial sums) and the
+// eight warp sums are added in warp order.
+__global__ void __launch_bounds__(256) mass_rhs_kernel(const float* Phi, const float* m, float* rhs, int n, int t) {
+  const int b = blockIdx.y, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int r = blockIdx.x * 32 + lane;
+  __shared__ float red[8][33];
   const float* P = Phi + (long long)b * n * t + r;
   const float* mb = m + (long long)b * n;
-  float a = 0.f;
-  for (int i = 0; i < n; ++i) a = fmaf(P[(long long)i * t], mb[i], a);
-  rhs[(long long)b * t + r] = a;
+  float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+  if (r < t) {
+    int i = warp;
+    for (; i + 24 < n; i += 32) {
+      a0 = fmaf(P[(long long)i * t], mb[i], a0);
+      a1 = fmaf(P[(long long)(i + 8) * t], mb[i + 8], a1);
+      a2 = fmaf(P[(long long)(i + 16) * t], mb[i + 16], a2);
+      a3 = fmaf(P[(long long)(i + 24) * t], mb[i + 24], a3);
+    }
+    for (; i < n; i += 8) a0 = fmaf(P[(long long)i * t], mb[i], a0);
+  }
+  red[warp][lane] = (a0 + a1) + (a2 + a3);
+  __syncthreads();
+  if (warp == 0 && r < t) {
+    float a = 0.f;
+    for (int w = 0; w < 8; ++w) a += red[w][lane];
+    rhs[(long long)b * t + r] = a;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -121,18 +139,26 @@ __device__ __forceinline__ void ld_tile(Tile<R> S, const R* G, long long ld, int
   }
 }
 
+// Thread tile of the 64 x 64 products: kTP rows x kTQ columns at (tile_ry, tile_cx).
+// A warp covers 16 rows x 16 columns, so each k step of mm64 costs it one
+// 16-byte load of the transposed left operand (4 rows) and one 8-byte load of
+// the right one (2 columns): two shared wavefronts for 8 FMAs per thread.
+constexpr int kTP = 4, kTQ = 2;
+__device__ __forceinline__ int tile_ry() { return (threadIdx.x >> 7) * 16 + ((threadIdx.x >> 3) & 3) * 4; }
+__device__ __forceinline__ int tile_cx() { return ((threadIdx.x >> 5) & 3) * 16 + (threadIdx.x & 7) * 2; }
+
 // P[p*ld + q] -= acc[p][q] for p < pn, q < qn (all loads issued before the stores)
 template <typename R>
-__device__ __forceinline__ void rmw_sub(R* P, long long ld, int pn, int qn, const R (&acc)[2][4]) {
-  R old[2][4];
+__device__ __forceinline__ void rmw_sub(R* P, long long ld, int pn, int qn, const R (&acc)[kTP][kTQ]) {
+  R old[kTP][kTQ];
 #pragma unroll
-  for (int p = 0; p < 2; ++p)
+  for (int p = 0; p < kTP; ++p)
 #pragma unroll
-    for (int q = 0; q < 4; ++q) old[p][q] = (p < pn && q < qn) ? __ldcg(P + p * ld + q) : R(0);
+    for (int q = 0; q < kTQ; ++q) old[p][q] = (p < pn && q < qn) ? __ldcg(P + p * ld + q) : R(0);
 #pragma unroll
-  for (int p = 0; p < 2; ++p)
+  for (int p = 0; p < kTP; ++p)
 #pragma unroll
-    for (int q = 0; q < 4; ++q)
+    for (int q = 0; q < kTQ; ++q)
       if (p < pn && q < qn) P[p * ld + q] = old[p][q] - acc[p][q];
 }
 
@@ -153,25 +179,25 @@ __device__ __forceinline__ void lds4(double (&a)[4], const double* p) {
   a[0] = v.x; a[1] = v.y; a[2] = u.x; a[3] = u.y;
 }
 
-// acc[p][q] = sum_l XT[l][ry+p] Y[l][cx+q], ry = (tid >> 4) * 2, cx = (tid & 15) * 4:
-// the left operand is held transposed so that each l takes one 2-wide and one
-// 4-wide shared load.
+// acc[p][q] = sum_l XT[l][ry+p] Y[l][cx+q] (ry = tile_ry(), cx = tile_cx()): the left
+// operand is held transposed so that each l takes one 4-wide and one 2-wide
+// shared load.
 template <typename R>
-__device__ __forceinline__ void mm64(Tile<R> XT, Tile<R> Y, R (&acc)[2][4]) {
-  const int ry = (threadIdx.x >> 4) * 2, cx = (threadIdx.x & 15) * 4;
+__device__ __forceinline__ void mm64(Tile<R> XT, Tile<R> Y, R (&acc)[kTP][kTQ]) {
+  const int ry = tile_ry(), cx = tile_cx();
 #pragma unroll
-  for (int p = 0; p < 2; ++p)
+  for (int p = 0; p < kTP; ++p)
 #pragma unroll
-    for (int q = 0; q < 4; ++q) acc[p][q] = R(0);
+    for (int q = 0; q < kTQ; ++q) acc[p][q] = R(0);
 #pragma unroll 8
   for (int l = 0; l < NB; ++l) {
-    R a[2], c[4];
-    lds2(a, &XT[l][ry]);
-    lds4(c, &Y[l][cx]);
+    R a[4], c[2];
+    lds4(a, &XT[l][ry]);
+    lds2(c, &Y[l][cx]);
 #pragma unroll
-    for (int p = 0; p < 2; ++p)
+    for (int p = 0; p < kTP; ++p)
 #pragma unroll
-      for (int q = 0; q < 4; ++q) acc[p][q] = fma_r(a[p], c[q], acc[p][q]);
+      for (int q = 0; q < kTQ; ++q) acc[p][q] = fma_r(a[p], c[q], acc[p][q]);
   }
 }
 
@@ -348,11 +374,11 @@ __device__ __forceinline__ void ld_tile_sum(Tile<R> S, const R* G1, const R* G2,
 
 // P[p*ld + q] = acc[p][q] for p < pn, q < qn
 template <typename R>
-__device__ __forceinline__ void st_acc(R* P, long long ld, int pn, int qn, const R (&acc)[2][4]) {
+__device__ __forceinline__ void st_acc(R* P, long long ld, int pn, int qn, const R (&acc)[kTP][kTQ]) {
 #pragma unroll
-  for (int p = 0; p < 2; ++p)
+  for (int p = 0; p < kTP; ++p)
 #pragma unroll
-    for (int q = 0; q < 4; ++q)
+    for (int q = 0; q < kTQ; ++q)
       if (p < pn && q < qn) P[p * ld + q] = acc[p][q];
 }
 
@@ -378,8 +404,8 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
   R* Bb = B + (long long)head * bbs;
   R* Zb = Z + (long long)head * bbs;
   R* Xb = X + (long long)head * bbs;
-  const int ry = (tid >> 4) * 2, cx = (tid & 15) * 4;
-  R acc[2][4];
+  const int ry = tile_ry(), cx = tile_cx();
+  R acc[kTP][kTQ];
   int* ctr0 = cg::this_cluster().map_shared_rank(ctr, 0);
   int ep = 0;   // dynamic phase number; phase ep draws from ctr0[ep & 1]
   // next tile of the current dynamic phase (block-uniform)
@@ -753,7 +779,7 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
   launch_gemm<true>(ColK<float>{B.Phi, nt, D.t}, ColK<float>{B.Phi, nt, D.t}, EpiStore{B.Gram, tt, 0, D.t, 1.f, true},
                     D.H, D.t, D.t, D.n, 1, st);
   ++nl;
-  mass_rhs_kernel<<<dim3(cdiv(D.t, 128), D.H), 128, 0, st>>>(B.Phi, m, B.rhs, D.n, D.t);
+  mass_rhs_kernel<<<dim3(cdiv(D.t, 32), D.H), 256, 0, st>>>(B.Phi, m, B.rhs, D.n, D.t);
   ++nl;
   nl += cholesky_solve(D.H, D.t, B.Gram, B.Linv, B.rhs, B.Z, B.wsol, 1, 1, D.t, ridge_w, stt, st);
   const long long ht = (long long)D.H * D.t;

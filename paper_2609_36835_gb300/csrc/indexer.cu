@@ -13,25 +13,31 @@
 namespace arckv {
 
 // w[b][r][a] = L_x[b][a] . x_r + b_x[b][a]: one CTA per (position, head).
-__global__ void __launch_bounds__(256) index_weights_kernel(const bf16* X, const bf16* L_x, const bf16* b_x,
+__global__ void __launch_bounds__(512) index_weights_kernel(const bf16* X, const bf16* L_x, const bf16* b_x,
                                                             float* wts, int d_x, int H_I, int n_pos) {
-  const int r = blockIdx.x, b = blockIdx.y;
+  // one warp per index head a: w_ra = L_x[a] . x_r + b_x[a]
+  const int r = blockIdx.x, b = blockIdx.y, a = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (a >= H_I) return;
   const bf16* x = X + (long long)r * d_x;
-  __shared__ float red[8];
-  for (int a = 0; a < H_I; ++a) {
-    const bf16* l = L_x + ((long long)b * H_I + a) * d_x;
-    float acc = 0.f;
-    for (int k = threadIdx.x; k < d_x; k += blockDim.x) acc = fmaf(to_f32(x[k]), to_f32(l[k]), acc);
-    acc = warp_sum(acc);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      float s = 0.f;
-      for (int w = 0; w < (int)(blockDim.x >> 5); ++w) s += red[w];
-      wts[((long long)b * n_pos + r) * H_I + a] = s + to_f32(b_x[b * H_I + a]);
+  const bf16* l = L_x + ((long long)b * H_I + a) * d_x;
+  float acc = 0.f;
+  if ((((uintptr_t)x | (uintptr_t)l) & 15) == 0) {   // rows are d_x % 8 == 0 elements long
+    for (int k = lane * 8; k < d_x; k += 256) {
+      const uint4 xv = *(const uint4*)(x + k), lv = *(const uint4*)(l + k);
+      const __nv_bfloat162* xh = (const __nv_bfloat162*)&xv;
+      const __nv_bfloat162* lh = (const __nv_bfloat162*)&lv;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 xf = __bfloat1622float2(xh[e]), lf = __bfloat1622float2(lh[e]);
+        acc = fmaf(xf.x, lf.x, acc);
+        acc = fmaf(xf.y, lf.y, acc);
+      }
     }
-    __syncthreads();
+  } else {
+    for (int k = lane; k < d_x; k += 32) acc = fmaf(to_f32(x[k]), to_f32(l[k]), acc);
   }
+  acc = warp_sum(acc);
+  if (lane == 0) wts[((long long)b * n_pos + r) * H_I + a] = acc + to_f32(b_x[b * H_I + a]);
 }
 
 int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf16* K, const bf16* VT,
@@ -64,7 +70,7 @@ int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf1
   launch_gemm(A, W, EpiBlockNormSplit{qbar_hi, qbar_lo, (long long)D.n * D.HD, D.HD}, D.H, D.n, D.HD,
               D.d + D.d_A, 1, st);
   ++nl;
-  index_weights_kernel<<<dim3(D.n_pos, D.H), 256, 0, st>>>(X, L_x, b_x, wts, D.d_x, D.H_I, D.n_pos);
+  index_weights_kernel<<<dim3(D.n_pos, D.H), 32 * D.H_I, 0, st>>>(X, L_x, b_x, wts, D.d_x, D.H_I, D.n_pos);
   ++nl;
   return nl;
 }

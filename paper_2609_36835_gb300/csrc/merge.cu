@@ -27,7 +27,23 @@ __global__ void __launch_bounds__(256) col_stats_kernel(const float* L, float* l
   const int rows = (n + 7) / 8, i0 = slice * rows, i1 = min(n, i0 + rows);
   float mx = -INFINITY, s1 = 0.f, s2 = 0.f;
   if (j < T) {
-    for (int i = i0; i < i1; ++i) {
+    // four rows per step: one rescale of the running sums per step
+    int i = i0;
+    for (; i + 3 < i1; i += 4) {
+      const float v0 = Lb[(long long)i * T], v1 = Lb[(long long)(i + 1) * T];
+      const float v2 = Lb[(long long)(i + 2) * T], v3 = Lb[(long long)(i + 3) * T];
+      const float m4 = fmaxf(fmaxf(v0, v1), fmaxf(v2, v3));
+      if (m4 > mx) {
+        const float r = (mx == -INFINITY) ? 0.f : expf(mx - m4);
+        s1 *= r;
+        s2 *= r * r;
+        mx = m4;
+      }
+      const float e0 = expf(v0 - mx), e1 = expf(v1 - mx), e2 = expf(v2 - mx), e3 = expf(v3 - mx);
+      s1 += (e0 + e1) + (e2 + e3);
+      s2 += (e0 * e0 + e1 * e1) + (e2 * e2 + e3 * e3);
+    }
+    for (; i < i1; ++i) {
       const float v = Lb[(long long)i * T];
       if (v > mx) {
         const float r = (mx == -INFINITY) ? 0.f : expf(mx - v);

@@ -51,30 +51,35 @@ int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* 
   return 1;
 }
 
-// One CTA per (32 x 32 tile of l, head): U_ij = exp(l_ij - M_j) * invN_j, split
-// into bf16 (hi, lo) and written transposed, Ut[b][j][i] (row stride ldn >= n;
-// the pad columns n..ldn-1 are written as zeros).
+// One CTA per (64 rows i x 32 columns j of l, head): U_ij = exp(l_ij - M_j) * invN_j,
+// split into bf16 (hi, lo) and written transposed, Ut[b][j][i] (row stride
+// ldn >= n, a multiple of 8; the pad columns n..ldn-1 are written as zeros).
+// Reads are 128-byte row segments; each warp writes 64 i-values of one j as
+// bf16 pairs (128 bytes per tensor).
 __global__ void __launch_bounds__(256) profiles_t_kernel(const float* L, const float* colM, const float* colInvN,
                                                          bf16* Ut_hi, bf16* Ut_lo, int n, int T, int ldn) {
-  const int b = blockIdx.z, j0 = blockIdx.x * 32, i0 = blockIdx.y * 32;
-  __shared__ float tile[32][33];
+  const int b = blockIdx.z, j0 = blockIdx.x * 32, i0 = blockIdx.y * 64;
+  __shared__ float tile[64][33];
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
   const float* Lb = L + (long long)b * n * T;
-  for (int r = ty; r < 32; r += 8) {
-    const int i = i0 + r, j = j0 + tx;
+  const int j = j0 + tx;
+  const float cm = j < T ? colM[(long long)b * T + j] : 0.f, ci = j < T ? colInvN[(long long)b * T + j] : 0.f;
+  for (int r = ty; r < 64; r += 8) {
+    const int i = i0 + r;
     float u = 0.f;
-    if (i < n && j < T) u = expf(Lb[(long long)i * T + j] - colM[(long long)b * T + j]) * colInvN[(long long)b * T + j];
+    if (i < n && j < T) u = expf(Lb[(long long)i * T + j] - cm) * ci;
     tile[r][tx] = u;
   }
   __syncthreads();
-  for (int r = ty; r < 32; r += 8) {
-    const int j = j0 + r, i = i0 + tx;
-    if (j < T && i < ldn) {
-      bf16 hi, lo;
-      split_bf16(tile[tx][r], hi, lo);
-      const long long o = ((long long)b * T + j) * ldn + i;
-      Ut_hi[o] = hi;
-      Ut_lo[o] = lo;
+  for (int c = ty; c < 32; c += 8) {
+    const int jj = j0 + c, i = i0 + 2 * tx;
+    if (jj < T && i < ldn) {   // ldn even: i + 1 < ldn as well
+      bf16 h0, l0, h1, l1;
+      split_bf16(tile[2 * tx][c], h0, l0);
+      split_bf16(tile[2 * tx + 1][c], h1, l1);
+      const long long o = ((long long)b * T + jj) * ldn + i;
+      *(__nv_bfloat162*)(Ut_hi + o) = __halves2bfloat162(h0, h1);
+      *(__nv_bfloat162*)(Ut_lo + o) = __halves2bfloat162(l0, l1);
     }
   }
 }
@@ -112,7 +117,7 @@ int launch_assign_tc(const Dims& D, const float* L, const float* colM, const flo
                      bf16* Ut_hi, bf16* Ut_lo, bf16* S_hi, bf16* S_lo, unsigned long long* best, int* kappa,
                      DevStatus* stt, cudaStream_t st) {
   const int ldn = (D.n + 7) / 8 * 8;
-  profiles_t_kernel<<<dim3(cdiv(D.T, 32), cdiv(ldn, 32), D.H), 256, 0, st>>>(L, colM, colInvN, Ut_hi, Ut_lo, D.n,
+  profiles_t_kernel<<<dim3(cdiv(D.T, 32), cdiv(ldn, 64), D.H), 256, 0, st>>>(L, colM, colInvN, Ut_hi, Ut_lo, D.n,
                                                                              D.T, ldn);
   gather_anchor_rows_kernel<<<dim3(D.t, D.H), 128, 0, st>>>(Ut_hi, Ut_lo, anchors, S_hi, S_lo, D.T, D.t, ldn);
   cudaMemsetAsync(best, 0, sizeof(unsigned long long) * (size_t)D.H * D.T, st);
