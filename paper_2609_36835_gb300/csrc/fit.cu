@@ -109,34 +109,67 @@ __device__ __forceinline__ unsigned cluster_rank() {
 }
 
 // S[r][c] = G[(r0 + r) * ld + c0 + c] (or S[c][r] with `trans`), zero outside
-// rows < rmax, cols < cmax of the source block.  Every thread issues its eight
-// loads before its first shared store, so the L2 latency is paid once per tile.
-// The transposed form maps a warp to 4 rows x 8 columns, so its shared stores
-// hit 32 distinct banks.
+// rows < rmax, cols < cmax of the source block.  Split into a fetch (eight
+// loads per thread into registers) and a put (the shared stores), so that a
+// caller loading two tiles issues all sixteen loads before its first store and
+// pays the L2 latency once.  The transposed form maps a warp to 4 rows x 8
+// columns, so its shared stores hit 32 distinct banks.
+template <typename R>
+struct TileRegs {
+  static constexpr int NE = NB * NB / kCT;
+  R v[NE];
+  bool trans;
+};
+// element q of this thread: (row, col) of the source block
+__device__ __forceinline__ void tile_pos(int q, bool trans, int& r, int& c) {
+  const int e = threadIdx.x + q * kCT;
+  if (!trans) {
+    r = e / NB;
+    c = e % NB;
+  } else {
+    const int lane = e & 31, w = e >> 5;
+    c = (w & 7) * 8 + (lane & 7);
+    r = (w >> 3) * 4 + (lane >> 3);
+  }
+}
+template <typename R>
+__device__ __forceinline__ void tile_fetch(TileRegs<R>& f, const R* G, long long ld, int r0, int c0, int rmax,
+                                           int cmax, bool trans) {
+  f.trans = trans;
+#pragma unroll
+  for (int q = 0; q < TileRegs<R>::NE; ++q) {
+    int r, c;
+    tile_pos(q, trans, r, c);
+    f.v[q] = (r < rmax && c < cmax) ? __ldcg(G + (long long)(r0 + r) * ld + c0 + c) : R(0);
+  }
+}
+template <typename R>
+__device__ __forceinline__ void tile_put(Tile<R> S, const TileRegs<R>& f) {
+#pragma unroll
+  for (int q = 0; q < TileRegs<R>::NE; ++q) {
+    int r, c;
+    tile_pos(q, f.trans, r, c);
+    if (f.trans) S[c][r] = f.v[q];
+    else S[r][c] = f.v[q];
+  }
+}
 template <typename R>
 __device__ __forceinline__ void ld_tile(Tile<R> S, const R* G, long long ld, int r0, int c0, int rmax, int cmax,
                                         bool trans) {
-  constexpr int NE = NB * NB / kCT;
-  R v[NE];
-  int rr[NE], cc[NE];
-#pragma unroll
-  for (int q = 0; q < NE; ++q) {
-    const int e = threadIdx.x + q * kCT;
-    if (!trans) {
-      rr[q] = e / NB;
-      cc[q] = e % NB;
-    } else {
-      const int lane = e & 31, w = e >> 5;
-      cc[q] = (w & 7) * 8 + (lane & 7);
-      rr[q] = (w >> 3) * 4 + (lane >> 3);
-    }
-    v[q] = (rr[q] < rmax && cc[q] < cmax) ? __ldcg(G + (long long)(r0 + rr[q]) * ld + c0 + cc[q]) : R(0);
-  }
-#pragma unroll
-  for (int q = 0; q < NE; ++q) {
-    if (trans) S[cc[q]][rr[q]] = v[q];
-    else S[rr[q]][cc[q]] = v[q];
-  }
+  TileRegs<R> f;
+  tile_fetch(f, G, ld, r0, c0, rmax, cmax, trans);
+  tile_put(S, f);
+}
+// two tiles, one L2 round trip
+template <typename R>
+__device__ __forceinline__ void ld_tiles(Tile<R> S1, const R* G1, long long ld1, int r1, int c1, int rm1, int cm1,
+                                         bool tr1, Tile<R> S2, const R* G2, long long ld2, int r2, int c2, int rm2,
+                                         int cm2, bool tr2) {
+  TileRegs<R> f1, f2;
+  tile_fetch(f1, G1, ld1, r1, c1, rm1, cm1, tr1);
+  tile_fetch(f2, G2, ld2, r2, c2, rm2, cm2, tr2);
+  tile_put(S1, f1);
+  tile_put(S2, f2);
 }
 
 // Thread tile of the 64 x 64 products: kTP rows x kTQ columns at (tile_ry, tile_cx).
@@ -392,6 +425,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
   Tile<R> S1 = (Tile<R>)sm;
   Tile<R> S2 = (Tile<R>)(sm + kTileF<R>);
   Tile<R> S3 = (Tile<R>)(sm + 2 * kTileF<R>);
+  Tile<R> S4 = (Tile<R>)(sm + 3 * kTileF<R>);
   __shared__ R red[kCT / 32];
   __shared__ int bad, grab;
   __shared__ int ctr[2];   // rank 0's pair deals the tiles of alternate dynamic phases
@@ -443,31 +477,74 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
   // trailing-update tiles of step k: x < ntri is the syrk tile (ii >= jj) of
   // the m trailing blocks, A_ij -= L_ik L_jk^T; the rest are rhs tiles
   // B_i -= L_ik Y_k with Y_k = Linv_kk B_k formed in the trsm phase
-  auto update_tile = [&](int k, int x, int ntri) {
+  // where tile x of step k reads its operands and writes its result
+  struct UpdDesc {
+    const R* Ga;   // L_ik (rows i0.., cols k0..), loaded transposed
+    const R* Gb;   // L_jk (transposed) or Y_k (as is)
+    R* dst;        // A_ij or B_i at the thread's first row / column
+    long long ldb_, ldd;
+    int i0, rb, br0, bc0, brm, bcm, pn, qn;
+    bool btrans;
+  };
+  auto describe = [&](int k, int x, int ntri, UpdDesc& u) {
     const int k0 = k * NB;
+    u.Ga = Ab;
     if (x < ntri) {
       int ii = (int)((sqrtf(8.f * x + 1.f) - 1.f) * 0.5f);
       while (ii * (ii + 1) / 2 > x) --ii;
       while ((ii + 1) * (ii + 2) / 2 <= x) ++ii;
       const int jj = x - ii * (ii + 1) / 2;
       const int i0 = (k + 1 + ii) * NB, j0 = (k + 1 + jj) * NB;
-      const int rb = min(NB, t - i0), cb = min(NB, t - j0);
-      ld_tile(S1, Ab, t, i0, k0, rb, NB, true);     // S1[l][r] = L_ik[r][l]
-      ld_tile(S2, Ab, t, j0, k0, cb, NB, true);     // S2[l][c] = L_jk[c][l]
-      __syncthreads();
-      mm64(S1, S2, acc);
-      rmw_sub(Ab + (long long)(i0 + ry) * t + j0 + cx, t, rb - ry, cb - cx, acc);
+      u.i0 = i0;
+      u.rb = min(NB, t - i0);
+      const int cb = min(NB, t - j0);
+      u.Gb = Ab; u.ldb_ = t; u.br0 = j0; u.bc0 = k0; u.brm = cb; u.bcm = NB; u.btrans = true;
+      u.dst = Ab + (long long)(i0 + ry) * t + j0 + cx; u.ldd = t; u.pn = u.rb - ry; u.qn = cb - cx;
     } else {
       const int y = x - ntri, i = k + 1 + y / nct, c0 = (y % nct) * NB;
-      const int i0 = i * NB, rb = min(NB, t - i0), nc = min(NB, nrhs - c0);
-      ld_tile(S1, Ab, t, i0, k0, rb, NB, true);     // S1[l][r] = L_ik[r][l]
-      ld_tile(S2, Bb, ldb, k0, c0, NB, nc, false);  // Y_k (block k < nblk - 1 is full)
-      __syncthreads();
-      mm64(S1, S2, acc);
-      rmw_sub(Bb + (long long)(i0 + ry) * ldb + c0 + cx, ldb, rb - ry, nc - cx, acc);
+      const int i0 = i * NB, nc = min(NB, nrhs - c0);
+      u.i0 = i0;
+      u.rb = min(NB, t - i0);
+      u.Gb = Bb; u.ldb_ = ldb; u.br0 = k0; u.bc0 = c0; u.brm = NB; u.bcm = nc; u.btrans = false;   // block k is full
+      u.dst = Bb + (long long)(i0 + ry) * ldb + c0 + cx; u.ldd = ldb; u.pn = u.rb - ry; u.qn = nc - cx;
+    }
+  };
+  // trailing-update tiles x0 and (when x1 < ntot) x1 of step k: all operand
+  // loads in one L2 round trip, both products, both read-modify-writes
+  auto update_tiles = [&](int k, int x0, int x1, int ntot, int ntri) {
+    const int k0 = k * NB;
+    const bool two = x1 < ntot;
+    UpdDesc u0, u1;
+    describe(k, x0, ntri, u0);
+    if (two) describe(k, x1, ntri, u1);
+    {
+      TileRegs<R> fa0, fb0, fa1, fb1;
+      tile_fetch(fa0, u0.Ga, t, u0.i0, k0, u0.rb, NB, true);
+      tile_fetch(fb0, u0.Gb, u0.ldb_, u0.br0, u0.bc0, u0.brm, u0.bcm, u0.btrans);
+      if (two) {
+        tile_fetch(fa1, u1.Ga, t, u1.i0, k0, u1.rb, NB, true);
+        tile_fetch(fb1, u1.Gb, u1.ldb_, u1.br0, u1.bc0, u1.brm, u1.bcm, u1.btrans);
+      }
+      tile_put(S1, fa0);
+      tile_put(S2, fb0);
+      if (two) {
+        tile_put(S3, fa1);
+        tile_put(S4, fb1);
+      }
+    }
+    __syncthreads();
+    mm64(S1, S2, acc);
+    if (two) {
+      R acc1[kTP][kTQ];
+      mm64(S3, S4, acc1);
+      rmw_sub(u0.dst, u0.ldd, u0.pn, u0.qn, acc);
+      rmw_sub(u1.dst, u1.ldd, u1.pn, u1.qn, acc1);
+    } else {
+      rmw_sub(u0.dst, u0.ldd, u0.pn, u0.qn, acc);
     }
     __syncthreads();
   };
+
 
   // step k = -1 only factors the first diagonal block (one call site keeps the
   // register-resident factorisation inlined once)
@@ -478,15 +555,15 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     for (int x = rank; k >= 0 && x < m + nct; x += kCL) {
       if (x < m) {
         const int i0 = (k + 1 + x) * NB, rb = min(NB, t - i0);
-        ld_tile(S1, Ab, t, i0, k0, rb, NB, true);                    // S1[l][r] = A_ik[r][l]
-        ld_tile(S2, Lk, NB, 0, 0, NB, NB, true);                     // S2[l][c] = Linv[c][l]
+        ld_tiles(S1, Ab, t, i0, k0, rb, NB, true,                    // S1[l][r] = A_ik[r][l]
+                 S2, Lk, (long long)NB, 0, 0, NB, NB, true);         // S2[l][c] = Linv[c][l]
         __syncthreads();
         mm64(S1, S2, acc);
         st_acc(Ab + (long long)(i0 + ry) * t + k0 + cx, t, rb - ry, NB, acc);
       } else {
         const int c0 = (x - m) * NB, nc = min(NB, nrhs - c0);
-        ld_tile(S1, Lk, NB, 0, 0, NB, NB, true);                     // S1[l][r] = Linv[r][l]
-        ld_tile(S2, Bb, ldb, k0, c0, kb, nc, false);
+        ld_tiles(S1, Lk, (long long)NB, 0, 0, NB, NB, true,          // S1[l][r] = Linv[r][l]
+                 S2, Bb, ldb, k0, c0, kb, nc, false);
         __syncthreads();
         mm64(S1, S2, acc);
         st_acc(Bb + (long long)(k0 + ry) * ldb + c0 + cx, ldb, kb - ry, nc - cx, acc);
@@ -503,13 +580,13 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     const int ntri = k >= 0 ? m * (m + 1) / 2 : 0, ntot = k >= 0 ? ntri + m * nct : 0;
     if (rank == 0 && tid == 0) ctr[(ep + 1) & 1] = 0;
     if (rank == (k + 1) % kCL) {
-      if (k >= 0) update_tile(k, 0, ntri);
+      if (k >= 0) update_tiles(k, 0, ntot, ntot, ntri);
       factor_diag(Ab, Lb, t, k + 1, lam, S1, S2, S3, &bad);
     }
-    for (;;) {
-      const int x = 1 + next_tile();
+    for (;;) {   // tiles are drawn two at a time
+      const int x = 1 + 2 * next_tile();
       if (x >= ntot) break;
-      update_tile(k, x, ntri);
+      update_tiles(k, x, x + 1, ntot, ntri);
     }
     ++ep;
     cluster_sync_all();
@@ -532,8 +609,8 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
   };
   auto z_tile = [&](int k, int i, int c0) {
     const int k0 = k * NB, kb = min(NB, t - k0), i0 = i * NB, nc = min(NB, nrhs - c0);
-    ld_tile(S1, Ab, t, k0, i0, kb, NB, false);     // S1[l][r] = L_ki[l][r]
-    ld_tile(S2, Xb, ldb, k0, c0, kb, nc, false);   // X_k
+    ld_tiles(S1, Ab, t, k0, i0, kb, NB, false,     // S1[l][r] = L_ki[l][r]
+             S2, Xb, ldb, k0, c0, kb, nc, false);  // X_k
     __syncthreads();
     mm64(S1, S2, acc);
     rmw_sub(Zb + (long long)(i0 + ry) * ldb + c0 + cx, ldb, NB - ry, nc - cx, acc);   // block i < k is full
@@ -562,7 +639,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
 template <typename R>
 static int cholesky_solve(int H, int t, R* Gram, R* Linv, R* B, R* Z, R* X, int ldb, int nrhs, long long bbs,
                           float ridge, DevStatus* stt, cudaStream_t st, int tdiv = 0) {
-  const int smem = 3 * kTileF<R> * (int)sizeof(R);
+  const int smem = 4 * kTileF<R> * (int)sizeof(R);
   const R td = (R)(tdiv > 0 ? tdiv : t);
   if (cluster_size(t) == 8) {
     cudaFuncSetAttribute(chol_cluster_kernel<R, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
