@@ -117,6 +117,12 @@ __device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_
       : "memory");
 }
 
+// Make this thread's generic-proxy shared-memory writes visible to the async
+// proxy (tcgen05.mma operand reads) before it signals the MMA issuer.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 // Arrive on `bar` once every MMA this thread issued so far has completed.
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
@@ -166,5 +172,10 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int n) {
 // (dim0 contiguous) with a box of {64, box1, 1} and 128-byte swizzle.
 bool encode_bf16_map_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1, uint64_t dim2,
                         uint32_t box1);
+
+// Host: encode a 3-D tiled TMA map over an fp32 tensor [dim2][dim1][dim0]
+// with a box of {box0, box1, 1}, no swizzle (rows land box0 * 4 bytes apart).
+bool encode_f32_map_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1, uint64_t dim2,
+                       uint32_t box0, uint32_t box1);
 
 }  // namespace arckv

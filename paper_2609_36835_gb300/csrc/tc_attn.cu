@@ -91,8 +91,234 @@ int launch_transpose_v(const Dims& D, const bf16* V, bf16* VT, cudaStream_t st) 
   return 1;
 }
 
+// ---------------------------------------------------------------------------
+// Fused O = P V with P = exp(X - shift_row) * mul_row, X the fp32 logits
+// [H][rows][T] and V the bf16 cache (as V^T [H][128][ldT]).  P never reaches
+// memory: TMA streams 128 x 64 slabs of X into a raw ring; eight converter
+// warps form P there, split it into the bf16 triple (h, m, l) and write the
+// three operand tiles straight into the 128-byte-swizzled K-major layout the
+// MMA reads; one thread issues h V + m V + l V per 16-wide K step into a
+// 128 x 128 fp32 TMEM accumulator; a fifth warp streams the V^T slabs.  The
+// products are those of the unfused split-3 GEMM, in the same order.
+//
+// CTA = (row tile of 128, K split); with two K splits the halves are added
+// into a zeroed output with fp32 atomics (two addends onto 0: the sum does not
+// depend on their order).
+namespace {
+constexpr int kPvRawBytes = 128 * 64 * 4;   // one fp32 slab of X
+constexpr int kPvTile = 128 * 128;          // one bf16 128 x 64 operand tile
+constexpr int kPvRS = 3;                    // raw ring depth
+constexpr int kPvOS = 2;                    // operand ring depth (h, m, l, V^T)
+constexpr int kPvOpBytes = 4 * kPvTile;
+constexpr int kPvConv = 8;                  // converter warps 2..9
+constexpr int kPvThreads = 32 * (kPvConv + 3);
+constexpr int kPvSmem = kPvRS * kPvRawBytes + kPvOS * kPvOpBytes + 1024;
+}  // namespace
+
+__global__ void __launch_bounds__(kPvThreads, 1)
+    probs_v_kernel(const __grid_constant__ CUtensorMap mX, const __grid_constant__ CUtensorMap mVT,
+                   const float* shift, const float* mul, const int* skip, float* O, int rows, int T, int splits,
+                   DevStatus* stt) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ uint64_t rfull[kPvRS], rempty[kPvRS], vfull[kPvOS], ofull[kPvOS], oempty[kPvOS], accf, drain;
+  __shared__ uint32_t tmem_slot;
+  __shared__ int abort_flag;
+  const uint32_t r0 = tc::smem_u32(smem_raw);
+  uint8_t* rbase = smem_raw + (((r0 + 1023u) & ~1023u) - r0);
+  uint8_t* obase = rbase + kPvRS * kPvRawBytes;   // 1024-byte aligned: the ring is a multiple of 1 KB
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int mt = (rows + 127) / 128;
+  const int tile = blockIdx.x / splits, sp = blockIdx.x - tile * splits;
+  const int b = tile / mt, m0 = (tile - b * mt) * 128;
+  const int nk = (T + 63) / 64;
+  const int kb0 = (int)((long long)nk * sp / splits), kb1 = (int)((long long)nk * (sp + 1) / splits);
+  const int nkb = kb1 - kb0;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kPvRS; ++s) {
+      tc::mbar_init(&rfull[s], 1);
+      tc::mbar_init(&rempty[s], kPvConv);
+    }
+    for (int s = 0; s < kPvOS; ++s) {
+      tc::mbar_init(&vfull[s], 1);
+      tc::mbar_init(&ofull[s], kPvConv);
+      tc::mbar_init(&oempty[s], 1);
+    }
+    tc::mbar_init(&accf, 1);
+    tc::mbar_init(&drain, 1);
+    abort_flag = 0;
+    tc::mbar_fence_init();
+  }
+  if (warp == 1) tc::tmem_alloc(&tmem_slot, 128);
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = tmem_slot;
+  volatile int* abortp = &abort_flag;
+
+  if (warp == 0) {
+    // X slabs
+    if (lane == 0) {
+      tc::tma_prefetch(&mX);
+      int g = 0;
+      for (; g < nkb; ++g) {
+        const int s = g % kPvRS;
+        if (g >= kPvRS && !tc::mbar_wait(&rempty[s], ((g / kPvRS) - 1) & 1, abortp, stt)) break;
+        tc::mbar_arrive_expect_tx(&rfull[s], kPvRawBytes);
+        tc::tma_load_3d(rbase + s * kPvRawBytes, &mX, (kb0 + g) * 64, m0, b, &rfull[s]);
+      }
+      volatile int never = 0;
+      for (int k = g > kPvRS ? g - kPvRS : 0; k < g; ++k) tc::mbar_wait(&rfull[k % kPvRS], (k / kPvRS) & 1, &never, stt);
+    }
+  } else if (warp == kPvConv + 2) {
+    // V^T slabs
+    if (lane == 0) {
+      tc::tma_prefetch(&mVT);
+      int g = 0;
+      for (; g < nkb; ++g) {
+        const int s = g % kPvOS;
+        if (g >= kPvOS && !tc::mbar_wait(&oempty[s], ((g / kPvOS) - 1) & 1, abortp, stt)) break;
+        tc::mbar_arrive_expect_tx(&vfull[s], kPvTile);
+        tc::tma_load_3d(obase + s * kPvOpBytes + 3 * kPvTile, &mVT, (kb0 + g) * 64, 0, b, &vfull[s]);
+      }
+      volatile int never = 0;
+      for (int k = g > kPvOS ? g - kPvOS : 0; k < g; ++k) tc::mbar_wait(&vfull[k % kPvOS], (k / kPvOS) & 1, &never, stt);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = tc::idesc_bf16_f32(128);
+      bool ok = true;
+      for (int g = 0; g < nkb && ok; ++g) {
+        const int s = g % kPvOS;
+        const uint32_t ph = (g / kPvOS) & 1;
+        if (!tc::mbar_wait(&vfull[s], ph, abortp, stt) || !tc::mbar_wait(&ofull[s], ph, abortp, stt)) {
+          ok = false;
+          break;
+        }
+        tc::fence_after_sync();
+        const uint32_t a = tc::smem_u32(obase + s * kPvOpBytes), bv = a + 3 * kPvTile;
+#pragma unroll
+        for (int ks = 0; ks < 4; ++ks) {
+          const uint64_t bd = tc::sdesc_k128(bv + ks * 32);
+#pragma unroll
+          for (int part = 0; part < 3; ++part)
+            tc::mma_f16(tmem, tc::sdesc_k128(a + part * kPvTile + ks * 32), bd, idesc,
+                        (g > 0 || ks > 0 || part > 0) ? 1u : 0u);
+        }
+        tc::mma_commit(&oempty[s]);
+      }
+      if (ok) tc::mma_commit(&accf);
+      tc::mma_commit(&drain);
+      volatile int never = 0;
+      tc::mbar_wait(&drain, 0, &never, stt);
+    }
+  } else {
+    // converters: warp cw owns rows 16 cw .. 16 cw + 15 of the tile; lane l
+    // holds row 16 cw + l's shift, scale and skipped column (l < 16)
+    const int cw = warp - 2;
+    float zr = 0.f, mr = 0.f;   // rows past the end: P = 0
+    int kr = -1;
+    if (lane < 16) {
+      const int row = m0 + cw * 16 + lane;
+      if (row < rows) {
+        const long long rr = (long long)b * rows + row;
+        zr = shift[rr];
+        mr = mul[rr];
+        kr = skip ? skip[rr] : -1;
+      }
+    }
+    bool ok = true;
+    for (int g = 0; g < nkb; ++g) {
+      const int rs = g % kPvRS, os = g % kPvOS;
+      ok = tc::mbar_wait(&rfull[rs], (g / kPvRS) & 1, abortp, stt);
+      if (ok && g >= kPvOS) ok = tc::mbar_wait(&oempty[os], ((g / kPvOS) - 1) & 1, abortp, stt);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) break;
+      const float* R = (const float*)(rbase + rs * kPvRawBytes);
+      uint8_t* A = obase + os * kPvOpBytes;
+      const int c = (kb0 + g) * 64 + 2 * lane;   // this lane's two columns
+#pragma unroll 4
+      for (int q = 0; q < 16; ++q) {
+        const int r = cw * 16 + q;
+        const float z = __shfl_sync(0xffffffffu, zr, q), mu = __shfl_sync(0xffffffffu, mr, q);
+        const int sk = __shfl_sync(0xffffffffu, kr, q);
+        const float2 x = *(const float2*)(R + r * 64 + 2 * lane);
+        const float p0 = (c < T && c != sk) ? expf(x.x - z) * mu : 0.f;
+        const float p1 = (c + 1 < T && c + 1 != sk) ? expf(x.y - z) * mu : 0.f;
+        const __nv_bfloat162 h = __floats2bfloat162_rn(p0, p1);
+        const float2 hf = __bfloat1622float2(h);
+        const float e0 = p0 - hf.x, e1 = p1 - hf.y;
+        const __nv_bfloat162 m = __floats2bfloat162_rn(e0, e1);
+        const float2 mf = __bfloat1622float2(m);
+        const __nv_bfloat162 l = __floats2bfloat162_rn(e0 - mf.x, e1 - mf.y);
+        // 128-byte swizzle: 16-byte chunk (lane / 4) of row r sits at chunk (lane / 4) ^ (r % 8)
+        const uint32_t off = (uint32_t)r * 128u + ((((uint32_t)lane >> 2) ^ ((uint32_t)r & 7u)) << 4) +
+                             (((uint32_t)lane & 3u) << 2);
+        *(__nv_bfloat162*)(A + off) = h;
+        *(__nv_bfloat162*)(A + kPvTile + off) = m;
+        *(__nv_bfloat162*)(A + 2 * kPvTile + off) = l;
+      }
+      tc::fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        tc::mbar_arrive(&rempty[rs]);
+        tc::mbar_arrive(&ofull[os]);
+      }
+    }
+    if (ok) ok = tc::mbar_wait(&accf, 0, abortp, stt);
+    ok = __all_sync(0xffffffffu, ok);
+    if (ok) {
+      tc::fence_after_sync();
+      const int qd = warp & 3, half = cw >> 2;   // TMEM lane quarter; column half
+      const int row = m0 + qd * 32 + lane;
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        float v[32];
+        tc::tmem_ld32(tmem + ((uint32_t)(qd * 32) << 16) + (uint32_t)(half * 64 + j * 32), v);
+        if (row < rows) {
+          float* d = O + ((long long)b * rows + row) * 128 + half * 64 + j * 32;
+          if (splits > 1) {
+#pragma unroll
+            for (int e = 0; e < 32; ++e) atomicAdd(d + e, v[e]);
+          } else {
+#pragma unroll
+            for (int e = 0; e < 32; e += 4) *(float4*)(d + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
+          }
+        }
+      }
+    }
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 1) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(tmem, 128);
+  }
+}
+
+// The fused product when X can be tiled by TMA (T a multiple of 4, 16-byte
+// aligned base); returns launches issued, 0 when not applicable, -1 on error.
+static int launch_probs_v_fused(const Dims& D, const float* X, const float* shift, const float* mul, const int* skip,
+                                const bf16* VT, float* out, DevStatus* stt, cudaStream_t st) {
+  if ((D.T & 3) != 0 || ((uintptr_t)X & 15u) != 0 || ((uintptr_t)out & 15u) != 0) return 0;
+  const int ldT = (D.T + 7) / 8 * 8;
+  CUtensorMap mX, mVT;
+  if (!encode_f32_map_3d(&mX, X, D.T, D.n, D.H, 64, 128) || !encode_bf16_map_3d(&mVT, VT, ldT, 128, D.H, 128))
+    return -1;
+  const int tiles = D.H * cdiv(D.n, 128), nk = cdiv(D.T, 64);
+  const int splits = (2 * tiles <= tc_gemm_sm_count() && nk >= 2) ? 2 : 1;
+  if (cudaFuncSetAttribute(probs_v_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kPvSmem) != cudaSuccess)
+    return -1;
+  if (splits > 1 && cudaMemsetAsync(out, 0, sizeof(float) * (size_t)D.H * D.n * 128, st) != cudaSuccess) return -1;
+  probs_v_kernel<<<tiles * splits, kPvThreads, kPvSmem, st>>>(mX, mVT, shift, mul, skip, out, D.n, D.T, splits, stt);
+  return cudaGetLastError() == cudaSuccess ? 1 : -1;
+}
+
 int launch_probs_v_tc(const Dims& D, const float* X, const float* shift, const float* mul, bf16* p_h, bf16* p_m,
                       bf16* p_l, const bf16* VT, float* out, DevStatus* stt, cudaStream_t st, const int* skip) {
+  const int fused = launch_probs_v_fused(D, X, shift, mul, skip, VT, out, stt, st);
+  if (fused != 0) return fused;
+  // X rows not TMA-tileable: P as a bf16 triple in memory, then the split-3 GEMM
   const int ldT = (D.T + 7) / 8 * 8;
   probs_split3_kernel<<<dim3(cdiv(ldT, 256 * 4), D.n, D.H), 256, 0, st>>>(X, shift, mul, skip, p_h, p_m, p_l, D.n,
                                                                           D.T, ldT);

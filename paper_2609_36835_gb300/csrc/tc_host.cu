@@ -12,8 +12,7 @@ PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_once;
 }  // namespace
 
-bool encode_bf16_map_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1, uint64_t dim2,
-                        uint32_t box1) {
+static bool encoder_ready() {
   std::call_once(g_once, [] {
     void* fn = nullptr;
     cudaDriverEntryPointQueryResult q;
@@ -22,7 +21,12 @@ bool encode_bf16_map_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint6
         q == cudaDriverEntryPointSuccess)
       g_encode = (PFN_cuTensorMapEncodeTiled_v12000)fn;
   });
-  if (!g_encode) return false;
+  return g_encode != nullptr;
+}
+
+bool encode_bf16_map_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1, uint64_t dim2,
+                        uint32_t box1) {
+  if (!encoder_ready()) return false;
   // TMA requires a 16-byte aligned base and row strides that are multiples of 16 bytes
   if (((uintptr_t)base & 15u) != 0 || (dim0 * 2) % 16 != 0) return false;
   const cuuint64_t gdim[3] = {dim0, dim1, dim2};
@@ -31,6 +35,21 @@ bool encode_bf16_map_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint6
   const cuuint32_t estride[3] = {1, 1, 1};
   const CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), gdim, gstride, box,
                               estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+bool encode_f32_map_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1, uint64_t dim2,
+                       uint32_t box0, uint32_t box1) {
+  if (!encoder_ready()) return false;
+  if (((uintptr_t)base & 15u) != 0 || (dim0 * 4) % 16 != 0 || (box0 * 4) % 16 != 0 || box0 > 256 || box1 > 256)
+    return false;
+  const cuuint64_t gdim[3] = {dim0, dim1, dim2};
+  const cuuint64_t gstride[2] = {dim0 * 4, dim0 * dim1 * 4};
+  const cuuint32_t box[3] = {box0, box1, 1};
+  const cuuint32_t estride[3] = {1, 1, 1};
+  const CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<void*>(base), gdim, gstride, box,
+                              estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
                               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }

@@ -122,6 +122,12 @@ def test_full_llama_layer_sampled_heads():
     check_layer(synth.WORKLOADS["llama8b_layer_T8192"], list(range(8)), [0, 7])
 
 
+def test_many_row_tiles_single_k_split():
+    """8 heads x 10 row tiles of reference rows (n = 1200): more row tiles than
+    half the SMs, so the fused probability products run without a K split."""
+    check_layer(synth.WORKLOADS["llama8b_layer_T8192"], list(range(8)), [3], T=2048, n_pos=300, t=205)
+
+
 def test_full_context_layer_retention_2pct():
     w = synth.WORKLOADS["llama8b_T8192_r02"]
     check_layer(w, list(range(8)), [5], layer=17)
@@ -169,6 +175,8 @@ def test_ha_vi_selectors_small(selector):
     (tie-aware) and the downstream stages on the oracle's anchors."""
     check_layer(synth.WORKLOADS["single_head_T1024"], [0], [0], selector=selector)
     check_layer(synth.WORKLOADS["llama8b_layer_T8192"], [1, 4], [0, 1], T=1000, n_pos=50, t=77, selector=selector)
+    # T not a multiple of 4: the probability products take the unfused path
+    check_layer(synth.WORKLOADS["llama8b_layer_T8192"], [3], [0], T=999, n_pos=30, t=50, selector=selector)
 
 
 @pytest.mark.parametrize("selector", [pk.SELECTOR_HA, pk.SELECTOR_VI])
