@@ -73,9 +73,10 @@ Layout plan(const arckv_config& c) {
   L.q_l = take(H * n * 128 * 2);
   L.av = take(H * n * 128 * f);
   L.VT = take(H * 128 * ldT * 2);
-  L.p_h = take(H * n * ldT * 2);
-  L.p_m = take(H * n * ldT * 2);
-  L.p_l = take(H * n * ldT * 2);
+  const size_t ptrip = probs_fused((int)T) ? 0 : H * n * ldT * 2;   // probability triple (unfused path only)
+  L.p_h = take(ptrip);
+  L.p_m = take(ptrip);
+  L.p_l = take(ptrip);
   L.cctx = take(H * n * 128 * f);
   L.qbar_hi = take(H * n * HD * 2);
   L.qbar_lo = take(H * n * HD * 2);

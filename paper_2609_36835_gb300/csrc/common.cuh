@@ -24,6 +24,27 @@ __device__ __forceinline__ void set_status(DevStatus* st, unsigned int code) {
 __device__ __forceinline__ float to_f32(float x) { return x; }
 __device__ __forceinline__ float to_f32(bf16 x) { return __bfloat162float(x); }
 
+// e^x evaluated as 2^(x log2 e): callers fold log2 e into an FMA with their
+// shift (e^(x - m) = ex2(x * kLog2e - m * kLog2e)) and take one MUFU ex2
+// (relative error ~2^-22; flushes subnormal results to zero).
+constexpr float kLog2e = 1.4426950408889634f;
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// bf16x2 triple of two fp32 values (split3_bf16 elementwise, packed pairs).
+__device__ __forceinline__ void split3_bf16x2(float a, float b, __nv_bfloat162& h, __nv_bfloat162& m,
+                                              __nv_bfloat162& l) {
+  h = __floats2bfloat162_rn(a, b);
+  const float2 hf = __bfloat1622float2(h);
+  const float ea = a - hf.x, eb = b - hf.y;
+  m = __floats2bfloat162_rn(ea, eb);
+  const float2 mf = __bfloat1622float2(m);
+  l = __floats2bfloat162_rn(ea - mf.x, eb - mf.y);
+}
+
 // Monotone map of fp32 onto uint32 (total order of finite values).
 __device__ __forceinline__ unsigned int f32_ordered(float f) {
   unsigned int u = __float_as_uint(f);

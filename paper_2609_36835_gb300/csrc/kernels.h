@@ -22,6 +22,9 @@ __host__ __device__ inline int chunk_budget(int T, int t, int Tc) {
   if (2 * r > T || (2 * r == T && (q & 1))) ++q;
   return (int)(q < 1 ? 1 : (q > Tc ? Tc : q));
 }
+// softmax(X) V products run fused (no probability triple in memory) when the
+// fp32 logit rows can be tiled by TMA: T a multiple of 4
+inline bool probs_fused(int T) { return (T & 3) == 0; }
 inline int effective_chunk(int T, int chunk_len) { return (chunk_len > 0 && T > kChunkThreshold) ? chunk_len : 0; }
 inline int realized_anchors(int T, int t, int chunk_len) {
   const int L = effective_chunk(T, chunk_len);

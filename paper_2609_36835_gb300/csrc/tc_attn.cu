@@ -94,8 +94,8 @@ int launch_transpose_v(const Dims& D, const bf16* V, bf16* VT, cudaStream_t st) 
 // ---------------------------------------------------------------------------
 // Fused O = P V with P = exp(X - shift_row) * mul_row, X the fp32 logits
 // [H][rows][T] and V the bf16 cache (as V^T [H][128][ldT]).  P never reaches
-// memory: TMA streams 128 x 64 slabs of X into a raw ring; eight converter
-// warps form P there, split it into the bf16 triple (h, m, l) and write the
+// memory: TMA streams 128 x 64 slabs of X into a raw ring; sixteen converter
+// warps form P there (e^x as 2^(x log2 e), one MUFU op per element), split it into the bf16 triple (h, m, l) and write the
 // three operand tiles straight into the 128-byte-swizzled K-major layout the
 // MMA reads; one thread issues h V + m V + l V per 16-wide K step into a
 // 128 x 128 fp32 TMEM accumulator; a fifth warp streams the V^T slabs.  The
@@ -110,11 +110,12 @@ constexpr int kPvTile = 128 * 128;          // one bf16 128 x 64 operand tile
 constexpr int kPvRS = 3;                    // raw ring depth
 constexpr int kPvOS = 2;                    // operand ring depth (h, m, l, V^T)
 constexpr int kPvOpBytes = 4 * kPvTile;
-constexpr int kPvConv = 8;                  // converter warps 2..9
+constexpr int kPvConv = 16;                 // converter warps 2..17, 8 rows each
 constexpr int kPvThreads = 32 * (kPvConv + 3);
 constexpr int kPvSmem = kPvRS * kPvRawBytes + kPvOS * kPvOpBytes + 1024;
 }  // namespace
 
+template <bool kSkip>
 __global__ void __launch_bounds__(kPvThreads, 1)
     probs_v_kernel(const __grid_constant__ CUtensorMap mX, const __grid_constant__ CUtensorMap mVT,
                    const float* shift, const float* mul, const int* skip, float* O, int rows, int T, int splits,
@@ -213,18 +214,22 @@ __global__ void __launch_bounds__(kPvThreads, 1)
       tc::mbar_wait(&drain, 0, &never, stt);
     }
   } else {
-    // converters: warp cw owns rows 16 cw .. 16 cw + 15 of the tile; lane l
-    // holds row 16 cw + l's shift, scale and skipped column (l < 16)
-    const int cw = warp - 2;
-    float zr = 0.f, mr = 0.f;   // rows past the end: P = 0
-    int kr = -1;
-    if (lane < 16) {
-      const int row = m0 + cw * 16 + lane;
+    // converters: warp cw owns rows 8 cw .. 8 cw + 7 of the tile, two rows per
+    // step (lanes 0-15 the first, 16-31 the second), four columns per lane
+    const int cw = warp - 2, hl = lane >> 4, cl = lane & 15;
+    float zl[4], mu[4];   // per step: shift * log2 e and scale of this lane's row (0, 0 past the end: P = 0)
+    int sk[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int row = m0 + cw * 8 + 2 * u + hl;
+      zl[u] = 0.f;
+      mu[u] = 0.f;
+      sk[u] = -1;
       if (row < rows) {
         const long long rr = (long long)b * rows + row;
-        zr = shift[rr];
-        mr = mul[rr];
-        kr = skip ? skip[rr] : -1;
+        zl[u] = shift[rr] * kLog2e;
+        mu[u] = mul[rr];
+        if (kSkip) sk[u] = skip[rr];
       }
     }
     bool ok = true;
@@ -236,27 +241,28 @@ __global__ void __launch_bounds__(kPvThreads, 1)
       if (!ok) break;
       const float* R = (const float*)(rbase + rs * kPvRawBytes);
       uint8_t* A = obase + os * kPvOpBytes;
-      const int c = (kb0 + g) * 64 + 2 * lane;   // this lane's two columns
-#pragma unroll 4
-      for (int q = 0; q < 16; ++q) {
-        const int r = cw * 16 + q;
-        const float z = __shfl_sync(0xffffffffu, zr, q), mu = __shfl_sync(0xffffffffu, mr, q);
-        const int sk = __shfl_sync(0xffffffffu, kr, q);
-        const float2 x = *(const float2*)(R + r * 64 + 2 * lane);
-        const float p0 = (c < T && c != sk) ? expf(x.x - z) * mu : 0.f;
-        const float p1 = (c + 1 < T && c + 1 != sk) ? expf(x.y - z) * mu : 0.f;
-        const __nv_bfloat162 h = __floats2bfloat162_rn(p0, p1);
-        const float2 hf = __bfloat1622float2(h);
-        const float e0 = p0 - hf.x, e1 = p1 - hf.y;
-        const __nv_bfloat162 m = __floats2bfloat162_rn(e0, e1);
-        const float2 mf = __bfloat1622float2(m);
-        const __nv_bfloat162 l = __floats2bfloat162_rn(e0 - mf.x, e1 - mf.y);
-        // 128-byte swizzle: 16-byte chunk (lane / 4) of row r sits at chunk (lane / 4) ^ (r % 8)
-        const uint32_t off = (uint32_t)r * 128u + ((((uint32_t)lane >> 2) ^ ((uint32_t)r & 7u)) << 4) +
-                             (((uint32_t)lane & 3u) << 2);
-        *(__nv_bfloat162*)(A + off) = h;
-        *(__nv_bfloat162*)(A + kPvTile + off) = m;
-        *(__nv_bfloat162*)(A + 2 * kPvTile + off) = l;
+      const int c = (kb0 + g) * 64 + 4 * cl;   // this lane's first column
+      const bool edge = kSkip || c + 4 > T;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int r = cw * 8 + 2 * u + hl;
+        const float4 x = *(const float4*)(R + r * 64 + 4 * cl);
+        float p[4] = {ex2_approx(fmaf(x.x, kLog2e, -zl[u])) * mu[u], ex2_approx(fmaf(x.y, kLog2e, -zl[u])) * mu[u],
+                      ex2_approx(fmaf(x.z, kLog2e, -zl[u])) * mu[u], ex2_approx(fmaf(x.w, kLog2e, -zl[u])) * mu[u]};
+        if (edge) {
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            if (c + e >= T || c + e == sk[u]) p[e] = 0.f;
+        }
+        __nv_bfloat162 h0, m0_, l0, h1, m1, l1;
+        split3_bf16x2(p[0], p[1], h0, m0_, l0);
+        split3_bf16x2(p[2], p[3], h1, m1, l1);
+        // 128-byte swizzle: 16-byte chunk cl / 2 of row r sits at chunk (cl / 2) ^ (r % 8)
+        const uint32_t off = (uint32_t)r * 128u + ((((uint32_t)cl >> 1) ^ ((uint32_t)r & 7u)) << 4) +
+                             (((uint32_t)cl & 1u) << 3);
+        *(uint2*)(A + off) = make_uint2(*(uint32_t*)&h0, *(uint32_t*)&h1);
+        *(uint2*)(A + kPvTile + off) = make_uint2(*(uint32_t*)&m0_, *(uint32_t*)&m1);
+        *(uint2*)(A + 2 * kPvTile + off) = make_uint2(*(uint32_t*)&l0, *(uint32_t*)&l1);
       }
       tc::fence_proxy_async_smem();
       __syncwarp();
@@ -269,21 +275,18 @@ __global__ void __launch_bounds__(kPvThreads, 1)
     ok = __all_sync(0xffffffffu, ok);
     if (ok) {
       tc::fence_after_sync();
-      const int qd = warp & 3, half = cw >> 2;   // TMEM lane quarter; column half
+      const int qd = warp & 3, cg = cw >> 2;   // TMEM lane quarter; 32-column group
       const int row = m0 + qd * 32 + lane;
+      float v[32];
+      tc::tmem_ld32(tmem + ((uint32_t)(qd * 32) << 16) + (uint32_t)(cg * 32), v);
+      if (row < rows) {
+        float* d = O + ((long long)b * rows + row) * 128 + cg * 32;
+        if (splits > 1) {
 #pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        float v[32];
-        tc::tmem_ld32(tmem + ((uint32_t)(qd * 32) << 16) + (uint32_t)(half * 64 + j * 32), v);
-        if (row < rows) {
-          float* d = O + ((long long)b * rows + row) * 128 + half * 64 + j * 32;
-          if (splits > 1) {
+          for (int e = 0; e < 32; ++e) atomicAdd(d + e, v[e]);
+        } else {
 #pragma unroll
-            for (int e = 0; e < 32; ++e) atomicAdd(d + e, v[e]);
-          } else {
-#pragma unroll
-            for (int e = 0; e < 32; e += 4) *(float4*)(d + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
-          }
+          for (int e = 0; e < 32; e += 4) *(float4*)(d + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
         }
       }
     }
@@ -296,28 +299,27 @@ __global__ void __launch_bounds__(kPvThreads, 1)
   }
 }
 
-// The fused product when X can be tiled by TMA (T a multiple of 4, 16-byte
-// aligned base); returns launches issued, 0 when not applicable, -1 on error.
+// The fused product (probs_fused(T): X rows tileable by TMA); returns the
+// launches issued or -1 (also for base pointers off the 16-byte grid).
 static int launch_probs_v_fused(const Dims& D, const float* X, const float* shift, const float* mul, const int* skip,
                                 const bf16* VT, float* out, DevStatus* stt, cudaStream_t st) {
-  if ((D.T & 3) != 0 || ((uintptr_t)X & 15u) != 0 || ((uintptr_t)out & 15u) != 0) return 0;
+  if (((uintptr_t)X & 15u) != 0 || ((uintptr_t)out & 15u) != 0) return -1;
   const int ldT = (D.T + 7) / 8 * 8;
   CUtensorMap mX, mVT;
   if (!encode_f32_map_3d(&mX, X, D.T, D.n, D.H, 64, 128) || !encode_bf16_map_3d(&mVT, VT, ldT, 128, D.H, 128))
     return -1;
   const int tiles = D.H * cdiv(D.n, 128), nk = cdiv(D.T, 64);
   const int splits = (2 * tiles <= tc_gemm_sm_count() && nk >= 2) ? 2 : 1;
-  if (cudaFuncSetAttribute(probs_v_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kPvSmem) != cudaSuccess)
-    return -1;
+  auto kern = skip ? probs_v_kernel<true> : probs_v_kernel<false>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kPvSmem) != cudaSuccess) return -1;
   if (splits > 1 && cudaMemsetAsync(out, 0, sizeof(float) * (size_t)D.H * D.n * 128, st) != cudaSuccess) return -1;
-  probs_v_kernel<<<tiles * splits, kPvThreads, kPvSmem, st>>>(mX, mVT, shift, mul, skip, out, D.n, D.T, splits, stt);
+  kern<<<tiles * splits, kPvThreads, kPvSmem, st>>>(mX, mVT, shift, mul, skip, out, D.n, D.T, splits, stt);
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
 }
 
 int launch_probs_v_tc(const Dims& D, const float* X, const float* shift, const float* mul, bf16* p_h, bf16* p_m,
                       bf16* p_l, const bf16* VT, float* out, DevStatus* stt, cudaStream_t st, const int* skip) {
-  const int fused = launch_probs_v_fused(D, X, shift, mul, skip, VT, out, stt, st);
-  if (fused != 0) return fused;
+  if (probs_fused(D.T)) return launch_probs_v_fused(D, X, shift, mul, skip, VT, out, stt, st);
   // X rows not TMA-tileable: P as a bf16 triple in memory, then the split-3 GEMM
   const int ldT = (D.T + 7) / 8 * 8;
   probs_split3_kernel<<<dim3(cdiv(ldT, 256 * 4), D.n, D.H), 256, 0, st>>>(X, shift, mul, skip, p_h, p_m, p_l, D.n,

@@ -295,7 +295,8 @@ struct TcEpiStore {
 };
 
 // TcEpiStore that also writes each row's softmax partials over the tile's
-// columns: part[b][row][n0 / BN] = (max, sum exp(x - max)) of alpha * acc.
+// columns: part[b][row][n0 / BN] = (max, sum exp(x - max)) of alpha * acc
+// (exp as 2^(x log2 e) on the MUFU unit).
 struct TcEpiStoreRowPart {
   TcEpiStore st;
   float2* part;
@@ -313,17 +314,24 @@ struct TcEpiStoreRowPart {
   }
   __device__ __forceinline__ void consume(State& s, int c, int j, float (&v)[32]) const {
     st.consume(s.s, c, j, v);
-    float m = s.mx;
+    const int nc = s.s.ncols - j * 32;   // columns of this chunk inside the matrix
+    if (nc <= 0) return;
 #pragma unroll
-    for (int q = 0; q < 32; ++q)
-      if (j * 32 + q < s.s.ncols) m = fmaxf(m, st.alpha * v[q]);
-    if (m == -INFINITY) return;
-    float a = s.sm * expf(s.mx - m);
+    for (int q = 0; q < 32; ++q) v[q] = (q < nc) ? st.alpha * v[q] : -INFINITY;
+    // independent max / sum chains (a serial chain would stall the single
+    // epilogue warp of each sub-partition on every dependent instruction)
+    float m8[8];
 #pragma unroll
-    for (int q = 0; q < 32; ++q)
-      if (j * 32 + q < s.s.ncols) a += expf(st.alpha * v[q] - m);
-    s.mx = m;
-    s.sm = a;
+    for (int k = 0; k < 8; ++k) m8[k] = fmaxf(fmaxf(v[k], v[k + 8]), fmaxf(v[k + 16], v[k + 24]));
+    const float m = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])), fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
+    const float mn = fmaxf(s.mx, m);
+    if (mn == -INFINITY) return;
+    const float ml = mn * kLog2e;
+    float a4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int q = 0; q < 32; ++q) a4[q & 3] += ex2_approx(fmaf(v[q], kLog2e, -ml));
+    s.sm = fmaf(s.sm, ex2_approx(fmaf(s.mx, kLog2e, -ml)), (a4[0] + a4[1]) + (a4[2] + a4[3]));
+    s.mx = mn;
   }
   __device__ __forceinline__ void finish(State& s, int, int, int, int, int) const {
     if (s.s.row_ok) part[s.prow] = make_float2(s.mx, s.sm);

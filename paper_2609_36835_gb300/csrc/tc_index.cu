@@ -43,14 +43,21 @@ struct TcEpiIndex {
   __device__ __forceinline__ void finish(State& s, int b, int row, int n0, int, int N) const {
     if (!s.row_ok) return;
     const int nc = min(128, N - n0);
-    float mx = -INFINITY;
+    // eight independent max / sum chains over the tile's columns
+    float m8[8], a8[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) m8[k] = -INFINITY;
 #pragma unroll
     for (int q = 0; q < 128; ++q)
-      if (q < nc) mx = fmaxf(mx, s.acc[q]);
-    float sm = 0.f;
+      if (q < nc) m8[q & 7] = fmaxf(m8[q & 7], s.acc[q]);
+    const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])), fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
+    const float ml = mx * kLog2e;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) a8[k] = 0.f;
 #pragma unroll
     for (int q = 0; q < 128; ++q)
-      if (q < nc) sm += expf(s.acc[q] - mx);
+      if (q < nc) a8[q & 7] += ex2_approx(fmaf(s.acc[q], kLog2e, -ml));
+    const float sm = ((a8[0] + a8[1]) + (a8[2] + a8[3])) + ((a8[4] + a8[5]) + (a8[6] + a8[7]));
     part[((long long)b * n + row) * ntiles + n0 / 128] = make_float2(mx, sm);
     float* dst = I + ((long long)b * n + row) * T + n0;
     if ((T & 3) == 0 && nc == 128) {
