@@ -83,6 +83,24 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, i
       : "memory");
 }
 
+// 3-D tiled store shared -> global of one box (x innermost; x, y, z >= 0;
+// the parts of the box outside the tensor are not written), tracked by this
+// thread's bulk async-group.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* src, int x, int y, int z) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+                   (uint64_t)map),
+               "r"(smem_u32(src)), "r"(x), "r"(y), "r"(z)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// Wait until at most N of this thread's bulk groups still read shared memory.
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+// Wait until all of this thread's bulk groups have completed.
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
 // Contiguous bulk copy global -> shared of `bytes` (both addresses 16-byte
 // aligned, bytes a multiple of 16), completing on `bar`.
 __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
@@ -174,8 +192,10 @@ bool encode_bf16_map_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint6
                         uint32_t box1);
 
 // Host: encode a 3-D tiled TMA map over an fp32 tensor [dim2][dim1][dim0]
-// with a box of {box0, box1, 1}, no swizzle (rows land box0 * 4 bytes apart).
+// (rows ld elements apart, batches bs elements apart) with a box of
+// {box0, box1, 1}; without swizzle the box rows land box0 * 4 bytes apart,
+// with swz128 (box0 = 32) the 16-byte chunks of row r are permuted by r % 8.
 bool encode_f32_map_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1, uint64_t dim2,
-                       uint32_t box0, uint32_t box1);
+                       uint32_t box0, uint32_t box1, uint64_t ld = 0, uint64_t bs = 0, bool swz128 = false);
 
 }  // namespace arckv

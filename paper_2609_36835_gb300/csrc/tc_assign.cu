@@ -46,8 +46,9 @@ int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* 
                          DevStatus* stt, cudaStream_t st) {
   CUtensorMap mA, mB;
   if (!encode_bf16_map_3d(&mA, Q, D.d, D.n, D.H, 128) || !encode_bf16_map_3d(&mB, K, D.d, D.T, D.H, 128)) return -1;
-  TcEpiStoreRowPart epi{{L, (long long)D.n * D.T, D.T, scale}, part, cdiv(D.T, 128), 128};
-  if (launch_tc_gemm<128, kPlain>(mA, mB, mA, mB, epi, D.H, D.n, D.T, D.d, 128, stt, st) != cudaSuccess) return -1;
+  if (launch_tc_logits_rowpart<kPlain>(mA, mB, mA, mB, nullptr, L, scale, part, D.H, D.n, D.T, D.d, stt, st) !=
+      cudaSuccess)
+    return -1;
   return 1;
 }
 

@@ -74,8 +74,8 @@ int launch_value_logits_tc(const Dims& D, const float* qpp, bf16* q_h, bf16* q_m
   if (!encode_bf16_map_3d(&mA, q_h, 128, D.n, D.H, 128) || !encode_bf16_map_3d(&mA2, q_m, 128, D.n, D.H, 128) ||
       !encode_bf16_map_3d(&mA3, q_l, 128, D.n, D.H, 128) || !encode_bf16_map_3d(&mB, K, 128, D.T, D.H, 128))
     return -1;
-  TcEpiStoreRowPart epi{{logits, (long long)D.n * D.T, D.T, 1.f}, part, cdiv(D.T, 128), 128};
-  if (launch_tc_gemm<128, kSplit3A>(mA, mB, mA2, mA, epi, D.H, D.n, D.T, 128, 128, stt, st, 0, &mA3) != cudaSuccess)
+  if (launch_tc_logits_rowpart<kSplit3A>(mA, mB, mA2, mA, &mA3, logits, 1.f, part, D.H, D.n, D.T, 128, stt, st) !=
+      cudaSuccess)
     return -1;
   return 2;
 }

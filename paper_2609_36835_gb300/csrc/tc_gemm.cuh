@@ -36,14 +36,29 @@
 //   void init(State&, int b, int row, int n0, int M, int N);
 //   void consume(State&, int chunk, int j, float (&v)[32]);  columns n0+32j..
 //   void finish(State&, int b, int row, int n0, int M, int N);
+// An epilogue that declares kStageBytes gets that much shared memory per
+// epilogue warp (1024-byte aligned) through attach(State&, uint8_t*, int*)
+// after init, for staging TMA stores, with a per-thread count of the stores
+// issued so far (kept across tiles, so staging buffers alternate by issued
+// store); the kernel waits for its bulk stores before it exits.
 #pragma once
 #include <algorithm>
+#include <type_traits>
 
 #include "tc.cuh"
 
 namespace arckv {
 
 enum TcMode { kPlain = 0, kSplit = 1, kConcat = 2, kSplit3A = 3 };
+
+template <class E, class = void>
+struct EpiStage {
+  static constexpr int bytes = 0;
+};
+template <class E>
+struct EpiStage<E, std::void_t<decltype(E::kStageBytes)>> {
+  static constexpr int bytes = E::kStageBytes;
+};
 
 template <int BN, int MODE>
 struct TcCfg {
@@ -61,9 +76,10 @@ template <int BN, int MODE, class Epi>
 __global__ void __launch_bounds__(192, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
                    const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mB2,
-                   const __grid_constant__ CUtensorMap mA3, Epi epi, int H, int M, int N, int K, int chunk_k, int K1,
-                   DevStatus* stt) {
+                   const __grid_constant__ CUtensorMap mA3, const __grid_constant__ Epi epi, int H, int M, int N, int K,
+                   int chunk_k, int K1, DevStatus* stt) {
   using C = TcCfg<BN, MODE>;
+  constexpr int SB = EpiStage<Epi>::bytes;
   constexpr bool SPLIT = C::SPLIT;
   constexpr int STAGES = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -209,11 +225,13 @@ __global__ void __launch_bounds__(192, 1)
     const int row = q * 32 + lane;
     bool ok = true;
     int cg = 0;
+    int stores = 0;   // staged stores issued by this warp (identical in all its lanes)
     for (int tl = blockIdx.x; tl < ntiles && ok; tl += gridDim.x) {
       int b, m0, n0;
       tile_coords(tl, b, m0, n0);
       typename Epi::State es;
       epi.init(es, b, m0 + row, n0, M, N);
+      if constexpr (SB > 0) epi.attach(es, base + STAGES * C::STAGE + (warp - 2) * SB, &stores);
       for (int c = 0; c < nchunks; ++c, ++cg) {
         const int buf = cg & 1;
         ok = tc::mbar_wait(&accf[buf], (cg >> 1) & 1, abortp, stt);
@@ -231,6 +249,10 @@ __global__ void __launch_bounds__(192, 1)
         if (lane == 0) tc::mbar_arrive(&acce[buf]);
       }
       if (ok) epi.finish(es, b, m0 + row, n0, M, N);
+    }
+    if constexpr (SB > 0) {
+      if (lane == 0) tc::bulk_wait_all();
+      __syncwarp();
     }
   }
   tc::fence_before_sync();
@@ -252,12 +274,14 @@ inline cudaError_t launch_tc_gemm(const CUtensorMap& mA, const CUtensorMap& mB, 
                                   const CUtensorMap& mB2, const Epi& epi, int H, int M, int N, int K, int chunk_k,
                                   DevStatus* stt, cudaStream_t st, int K1 = 0, const CUtensorMap* mA3 = nullptr) {
   using C = TcCfg<BN, MODE>;
+  constexpr int smem = C::SMEM + 4 * EpiStage<Epi>::bytes;
+  static_assert(smem <= 227 * 1024, "stage ring and epilogue staging exceed shared memory");
   auto kern = tc_gemm_kernel<BN, MODE, Epi>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const long long ntiles = (long long)cdiv(N, BN) * cdiv(M, 128) * H;
   const int grid = (int)std::min<long long>(ntiles, tc_gemm_sm_count());
-  kern<<<grid, 192, C::SMEM, st>>>(mA, mB, mA2, mB2, mA3 ? *mA3 : mA, epi, H, M, N, K, chunk_k, K1, stt);
+  kern<<<grid, 192, smem, st>>>(mA, mB, mA2, mB2, mA3 ? *mA3 : mA, epi, H, M, N, K, chunk_k, K1, stt);
   return cudaGetLastError();
 }
 
@@ -294,27 +318,90 @@ struct TcEpiStore {
   __device__ __forceinline__ void finish(State&, int, int, int, int, int) const {}
 };
 
-// TcEpiStore that also writes each row's softmax partials over the tile's
-// columns: part[b][row][n0 / BN] = (max, sum exp(x - max)) of alpha * acc
-// (exp as 2^(x log2 e) on the MUFU unit).
-struct TcEpiStoreRowPart {
-  TcEpiStore st;
+// Staged TMA store of one warp's 32 rows x 32 columns at (x, y, b): the rows
+// go into a 128-byte-swizzled staging buffer (conflict-free 16-byte stores)
+// and one lane issues the tiled bulk store.  Two buffers alternate by issued
+// store; before a buffer is rewritten, at most one store (the other
+// buffer's) may still be reading.  Boxes wholly outside [0, N) x [0, M) are
+// skipped (warp-uniform).  v is scaled by alpha.
+__device__ __forceinline__ void staged_store_32x32(const CUtensorMap* map, uint8_t* stage, int* stores, int x, int y,
+                                                   int b, int M, int N, const float* v, float alpha) {
+  if (y >= M || x >= N) return;
+  const int lane = threadIdx.x & 31;
+  uint8_t* buf = stage + (*stores & 1) * 4096;
+  if (lane == 0) tc::bulk_wait_read<1>();
+  __syncwarp();
+#pragma unroll
+  for (int k = 0; k < 8; ++k)
+    *(float4*)(buf + lane * 128 + ((k ^ (lane & 7)) << 4)) =
+        make_float4(alpha * v[4 * k], alpha * v[4 * k + 1], alpha * v[4 * k + 2], alpha * v[4 * k + 3]);
+  tc::fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0) {
+    tc::tma_store_3d(map, buf, x, y, b);
+    tc::bulk_commit();
+  }
+  ++*stores;
+}
+
+// fp32 store through shared memory and TMA (staged_store_32x32 per chunk):
+// a chunk's store overlaps the next chunk.  C is [H][M][N] with row stride
+// ldc (a multiple of 4) in `map`.
+struct TcEpiStoreTma {
+  CUtensorMap map;   // box {32, 32, 1}, 128-byte swizzle
+  float alpha;
+  int M, N;
+  static constexpr int kStageBytes = 2 * 32 * 128;
+  struct State {
+    uint8_t* stage;
+    int* stores;
+    int b, y, n0;
+  };
+  __device__ __forceinline__ void init(State& s, int b, int row, int n0, int, int) const {
+    s.b = b;
+    s.y = row & ~31;
+    s.n0 = n0;
+  }
+  __device__ __forceinline__ void attach(State& s, uint8_t* stage, int* stores) const {
+    s.stage = stage;
+    s.stores = stores;
+  }
+  __device__ __forceinline__ void consume(State& s, int, int j, float (&v)[32]) const {
+    staged_store_32x32(&map, s.stage, s.stores, s.n0 + 32 * j, s.y, s.b, M, N, v, alpha);
+  }
+  __device__ __forceinline__ void finish(State&, int, int, int, int, int) const {}
+};
+
+// A store epilogue (TcEpiStore or TcEpiStoreTma) that also writes each row's
+// softmax partials over the tile's columns: part[b][row][n0 / BN] =
+// (max, sum exp(x - max)) of alpha * acc (exp as 2^(x log2 e) on the MUFU unit).
+template <class Store>
+struct TcEpiRowPartT {
+  Store st;
   float2* part;
   int ntiles, BNt;
+  static constexpr int kStageBytes = EpiStage<Store>::bytes;
   struct State {
-    TcEpiStore::State s;
+    typename Store::State s;
     float mx, sm;
     long long prow;
+    int ncols;
+    bool row_ok;
   };
   __device__ __forceinline__ void init(State& s, int b, int row, int n0, int M, int N) const {
     st.init(s.s, b, row, n0, M, N);
     s.mx = -INFINITY;
     s.sm = 0.f;
     s.prow = ((long long)b * M + row) * ntiles + n0 / BNt;
+    s.ncols = N - n0;
+    s.row_ok = row < M;
+  }
+  __device__ __forceinline__ void attach(State& s, uint8_t* stage, int* stores) const {
+    st.attach(s.s, stage, stores);
   }
   __device__ __forceinline__ void consume(State& s, int c, int j, float (&v)[32]) const {
     st.consume(s.s, c, j, v);
-    const int nc = s.s.ncols - j * 32;   // columns of this chunk inside the matrix
+    const int nc = s.ncols - j * 32;   // columns of this chunk inside the matrix
     if (nc <= 0) return;
 #pragma unroll
     for (int q = 0; q < 32; ++q) v[q] = (q < nc) ? st.alpha * v[q] : -INFINITY;
@@ -334,8 +421,35 @@ struct TcEpiStoreRowPart {
     s.mx = mn;
   }
   __device__ __forceinline__ void finish(State& s, int, int, int, int, int) const {
-    if (s.s.row_ok) part[s.prow] = make_float2(s.mx, s.sm);
+    if (s.row_ok) part[s.prow] = make_float2(s.mx, s.sm);
   }
 };
+using TcEpiStoreRowPart = TcEpiRowPartT<TcEpiStore>;
+using TcEpiStoreRowPartTma = TcEpiRowPartT<TcEpiStoreTma>;
+
+// Row-partial logits L = alpha * (A B^T) [H][M][N] (row stride N) through the
+// TMA-store epilogue when N is a multiple of 4 (row pitch on the 16-byte grid),
+// else through plain stores.
+template <int MODE>
+inline cudaError_t launch_tc_logits_rowpart(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mA2,
+                                            const CUtensorMap& mB2, const CUtensorMap* mA3, float* L, float alpha,
+                                            float2* part, int H, int M, int N, int K, DevStatus* stt,
+                                            cudaStream_t st) {
+  const int ntiles = cdiv(N, 128);
+  if ((N & 3) == 0 && (((uintptr_t)L) & 15u) == 0) {
+    TcEpiStoreRowPartTma epi{};
+    epi.st.alpha = alpha;
+    epi.st.M = M;
+    epi.st.N = N;
+    epi.part = part;
+    epi.ntiles = ntiles;
+    epi.BNt = 128;
+    if (!encode_f32_map_3d(&epi.st.map, L, N, M, H, 32, 32, N, (uint64_t)M * N, true))
+      return cudaErrorInvalidValue;
+    return launch_tc_gemm<128, MODE>(mA, mB, mA2, mB2, epi, H, M, N, K, K, stt, st, 0, mA3);
+  }
+  TcEpiStoreRowPart epi{{L, (long long)M * N, N, alpha}, part, ntiles, 128};
+  return launch_tc_gemm<128, MODE>(mA, mB, mA2, mB2, epi, H, M, N, K, K, stt, st, 0, mA3);
+}
 
 }  // namespace arckv

@@ -7,20 +7,27 @@
 // columns) at a time: every head's partial dot products land in their own
 // TMEM accumulator and the epilogue folds them through the LeakyReLU and the
 // row's head weight w_ia before the next head is added.  The epilogue then
-// writes the I tile and the tile's row-softmax partials (max, sum of exp).
+// writes the tile's row-softmax partials (max, sum of exp) and the I tile.
 #include "kernels.h"
 #include "tc_gemm.cuh"
 
 namespace arckv {
 
-struct TcEpiIndex {
+// kTma: the I tile leaves through TMA stores staged in shared memory (32 x 32
+// boxes, two buffers per epilogue warp); else each row writes its 128 values.
+template <bool kTma>
+struct TcEpiIndexT {
   const float* wts;  // [H][n_pos][H_I]
   float* I;          // [H][n][T]
   float2* part;      // [H][n][ntiles]
   int n, T, H_I, G, n_pos, ntiles;
+  CUtensorMap map;   // kTma: I as [H][n][T], box {32, 32, 1}, 128-byte swizzle
+  static constexpr int kStageBytes = kTma ? 2 * 32 * 128 : 0;
   struct State {
     float acc[128];
     const float* wrow;
+    uint8_t* stage;
+    int* stores;
     float w;
     bool row_ok;
   };
@@ -30,6 +37,10 @@ struct TcEpiIndex {
     s.w = 0.f;
 #pragma unroll
     for (int q = 0; q < 128; ++q) s.acc[q] = 0.f;
+  }
+  __device__ __forceinline__ void attach(State& s, uint8_t* stage, int* stores) const {
+    s.stage = stage;
+    s.stores = stores;
   }
   __device__ __forceinline__ void consume(State& s, int chunk, int j, float (&v)[32]) const {
     if (j == 0) s.w = s.row_ok ? s.wrow[chunk] : 0.f;
@@ -41,32 +52,43 @@ struct TcEpiIndex {
     }
   }
   __device__ __forceinline__ void finish(State& s, int b, int row, int n0, int, int N) const {
-    if (!s.row_ok) return;
     const int nc = min(128, N - n0);
-    // eight independent max / sum chains over the tile's columns
-    float m8[8], a8[8];
+    if (s.row_ok) {
+      // eight independent max / sum chains over the tile's columns
+      float m8[8], a8[8];
 #pragma unroll
-    for (int k = 0; k < 8; ++k) m8[k] = -INFINITY;
-#pragma unroll
-    for (int q = 0; q < 128; ++q)
-      if (q < nc) m8[q & 7] = fmaxf(m8[q & 7], s.acc[q]);
-    const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])), fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
-    const float ml = mx * kLog2e;
-#pragma unroll
-    for (int k = 0; k < 8; ++k) a8[k] = 0.f;
-#pragma unroll
-    for (int q = 0; q < 128; ++q)
-      if (q < nc) a8[q & 7] += ex2_approx(fmaf(s.acc[q], kLog2e, -ml));
-    const float sm = ((a8[0] + a8[1]) + (a8[2] + a8[3])) + ((a8[4] + a8[5]) + (a8[6] + a8[7]));
-    part[((long long)b * n + row) * ntiles + n0 / 128] = make_float2(mx, sm);
-    float* dst = I + ((long long)b * n + row) * T + n0;
-    if ((T & 3) == 0 && nc == 128) {
-#pragma unroll
-      for (int q = 0; q < 128; q += 4) *(float4*)(dst + q) = make_float4(s.acc[q], s.acc[q + 1], s.acc[q + 2], s.acc[q + 3]);
-    } else {
+      for (int k = 0; k < 8; ++k) m8[k] = -INFINITY;
 #pragma unroll
       for (int q = 0; q < 128; ++q)
-        if (q < nc) dst[q] = s.acc[q];
+        if (q < nc) m8[q & 7] = fmaxf(m8[q & 7], s.acc[q]);
+      const float mx =
+          fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])), fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
+      const float ml = mx * kLog2e;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) a8[k] = 0.f;
+#pragma unroll
+      for (int q = 0; q < 128; ++q)
+        if (q < nc) a8[q & 7] += ex2_approx(fmaf(s.acc[q], kLog2e, -ml));
+      const float sm = ((a8[0] + a8[1]) + (a8[2] + a8[3])) + ((a8[4] + a8[5]) + (a8[6] + a8[7]));
+      part[((long long)b * n + row) * ntiles + n0 / 128] = make_float2(mx, sm);
+    }
+    if constexpr (kTma) {
+      // rows past n and columns past T fall outside the tensor map: not written
+      const int y = row & ~31;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) staged_store_32x32(&map, s.stage, s.stores, n0 + 32 * j, y, b, n, T, s.acc + 32 * j, 1.f);
+    } else {
+      if (!s.row_ok) return;
+      float* dst = I + ((long long)b * n + row) * T + n0;
+      if ((T & 3) == 0 && nc == 128) {
+#pragma unroll
+        for (int q = 0; q < 128; q += 4)
+          *(float4*)(dst + q) = make_float4(s.acc[q], s.acc[q + 1], s.acc[q + 2], s.acc[q + 3]);
+      } else {
+#pragma unroll
+        for (int q = 0; q < 128; ++q)
+          if (q < nc) dst[q] = s.acc[q];
+      }
     }
   }
 };
@@ -78,7 +100,14 @@ int launch_index_logits(const Dims& D, const bf16* qbar_hi, const bf16* qbar_lo,
   if (!encode_bf16_map_3d(&mA, qbar_hi, D.HD, D.n, D.H, 128) || !encode_bf16_map_3d(&mA2, qbar_lo, D.HD, D.n, D.H, 128) ||
       !encode_bf16_map_3d(&mB, kbar_hi, D.HD, D.T, D.H, 128) || !encode_bf16_map_3d(&mB2, kbar_lo, D.HD, D.T, D.H, 128))
     return -1;
-  TcEpiIndex epi{wts, I, part, D.n, D.T, D.H_I, D.G, D.n_pos, cdiv(D.T, 128)};
+  if ((D.T & 3) == 0 && ((uintptr_t)I & 15u) == 0) {
+    TcEpiIndexT<true> epi{wts, I, part, D.n, D.T, D.H_I, D.G, D.n_pos, cdiv(D.T, 128), {}};
+    if (!encode_f32_map_3d(&epi.map, I, D.T, D.n, D.H, 32, 32, D.T, (uint64_t)D.n * D.T, true)) return -1;
+    if (launch_tc_gemm<128, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.n, D.T, D.HD, 128, stt, st) != cudaSuccess)
+      return -1;
+    return 1;
+  }
+  TcEpiIndexT<false> epi{wts, I, part, D.n, D.T, D.H_I, D.G, D.n_pos, cdiv(D.T, 128), {}};
   if (launch_tc_gemm<128, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.n, D.T, D.HD, 128, stt, st) != cudaSuccess) return -1;
   return 1;
 }
