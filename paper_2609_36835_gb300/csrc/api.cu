@@ -295,7 +295,7 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
   FitBufs B{F(L.LC),  F(L.Phi), F(L.Gram), F(L.Linv), F(L.rhs), F(L.wsol), F(L.R), F(L.Z),
             (bf16*)(w + L.S_hi), (bf16*)(w + L.S_lo), (bf16*)(w + L.YT_hi), (bf16*)(w + L.YT_lo),
             (double*)(w + L.G64), (double*)(w + L.L64), (double*)(w + L.B64), (double*)(w + L.Z64),
-            (double*)(w + L.X64)};
+            (double*)(w + L.X64), (bf16*)(w + L.Ut_hi)};   // Ut_hi [H][T][ldn] is free after the assignment
   const int nlf = launch_fits(D, scale, cfg->ridge_w, cfg->ridge_v, cfg->eps_w, cfg->b_min, cfg->b_max, Qb, C_k,
                               F(L.z), F(L.m), F(L.Y), B, beta, C_v, stt, st);
   if (nlf < 0) return ARCKV_ERR_CUDA;

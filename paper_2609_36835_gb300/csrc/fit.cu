@@ -701,6 +701,43 @@ __global__ void __launch_bounds__(256) transpose_split_kernel(const float* src, 
   }
 }
 
+// Transposed bf16 triple of src [rows][cols] (fp32): dst_{h,m,l}[b][c][r]
+// (row stride ldr >= rows; the pad r in [rows, ldr) is written as zeros).
+__global__ void __launch_bounds__(256) transpose_split3_kernel(const float* src, int rows, int cols, bf16* dh, bf16* dm,
+                                                               bf16* dl, int ldr) {
+  const int b = blockIdx.z, c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+  __shared__ float tile[32][33];
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  const float* sb = src + (long long)b * rows * cols;
+  for (int q = ty; q < 32; q += 8) {
+    const int r = r0 + q, c = c0 + tx;
+    tile[q][tx] = (r < rows && c < cols) ? sb[(long long)r * cols + c] : 0.f;
+  }
+  __syncthreads();
+  for (int q = ty; q < 32; q += 8) {
+    const int c = c0 + q, r = r0 + tx;
+    if (c < cols && r < ldr) {
+      const long long o = ((long long)b * cols + c) * ldr + r;
+      split3_bf16(tile[tx][q], dh[o], dm[o], dl[o]);
+    }
+  }
+}
+
+// C[b] (t x t, row stride t) = X^T X over the n reference rows, X^T given as a
+// transposed bf16 triple [t][ldn]: the kSplit3S tensor-core Gram.
+static int gram3_tc(int H, int t, int ldn, const bf16* Xh, const bf16* Xm, const bf16* Xl, float* C, DevStatus* stt,
+                    cudaStream_t st) {
+  CUtensorMap mA, mA2, mA3;
+  if (!encode_bf16_map_3d(&mA, Xh, ldn, t, H, 128) || !encode_bf16_map_3d(&mA2, Xm, ldn, t, H, 128) ||
+      !encode_bf16_map_3d(&mA3, Xl, ldn, t, H, 128))
+    return -1;
+  TcEpiStore epi{C, (long long)t * t, t, 1.f};
+  const int kfull = (ldn + 63) / 64 * 64;
+  if (launch_tc_gemm<128, kSplit3S>(mA, mA, mA2, mA2, epi, H, t, t, ldn, kfull, stt, st, 0, &mA3) != cudaSuccess)
+    return -1;
+  return 1;
+}
+
 // C[b] (M x N, row stride ldc) = X^T Z over the n reference rows, with X^T and
 // Z^T given as transposed split-bf16 operands [M][ldn] and [N][ldn].
 static int gram_tc(int H, int M, int N, int ldn, const bf16* Xh, const bf16* Xl, const bf16* Zh, const bf16* Zl,
@@ -839,7 +876,7 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
                 float b_max, const bf16* Q, const float* C_k, const float* z, const float* m,
                 const float* Y, const FitBufs& B, float* beta, float* C_v, DevStatus* stt, cudaStream_t st) {
   int nl = 0;
-  const long long nd = (long long)D.n * D.d, nt = (long long)D.n * D.t, tt = (long long)D.t * D.t;
+  const long long nd = (long long)D.n * D.d, nt = (long long)D.n * D.t;
   // logits of the compact keys: scale Q C_k^T
   launch_gemm(RowK<bf16>{Q, nd, D.d}, RowK<float>{C_k, (long long)D.t * D.d, D.d},
               EpiStore{B.LC, nt, 0, D.t, scale, false}, D.H, D.n, D.t, D.d, 1, st);
@@ -848,14 +885,15 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
   phi_kernel<<<min(cdiv(cnt, 256), 152 * 16), 256, 0, st>>>(B.LC, z, B.Phi, D.n, D.t, cnt);
   ++nl;
   if (D.t > D.n) return nl + fits_dual(D, ridge_w, ridge_v, eps_w, b_min, b_max, m, Y, B, beta, C_v, stt, st);
-  // beta system: Gram = Phi_C^T Phi_C in fp32 (SIMT, lower tiles mirrored).  Its
-  // condition number reaches ~1e6 on long caches, beyond what the split-bf16
-  // tensor-core product (~1e-5 relative per entry) resolves within tolerance.
+  // beta system: Gram = Phi_C^T Phi_C.  Its condition number reaches ~1e6 on
+  // long caches, beyond what a split-bf16 pair (~1e-5 relative per entry)
+  // resolves within tolerance: the operand enters as a bf16 triple and the
+  // tensor-core Gram keeps every product term down to 2^-24 (kSplit3S).
   const int ldn = (D.n + 7) / 8 * 8;
   const dim3 tgrid(cdiv(D.t, 32), cdiv(ldn, 32), D.H);
-  launch_gemm<true>(ColK<float>{B.Phi, nt, D.t}, ColK<float>{B.Phi, nt, D.t}, EpiStore{B.Gram, tt, 0, D.t, 1.f, true},
-                    D.H, D.t, D.t, D.n, 1, st);
-  ++nl;
+  transpose_split3_kernel<<<tgrid, 256, 0, st>>>(B.Phi, D.n, D.t, B.PT_hi, B.PT_mid, B.PT_lo, ldn);
+  if (gram3_tc(D.H, D.t, ldn, B.PT_hi, B.PT_mid, B.PT_lo, B.Gram, stt, st) < 0) return -1;
+  nl += 2;
   mass_rhs_kernel<<<dim3(cdiv(D.t, 32), D.H), 256, 0, st>>>(B.Phi, m, B.rhs, D.n, D.t);
   ++nl;
   nl += cholesky_solve(D.H, D.t, B.Gram, B.Linv, B.rhs, B.Z, B.wsol, 1, 1, D.t, ridge_w, stt, st);

@@ -101,6 +101,7 @@ struct FitBufs {
   float *LC, *Phi, *Gram, *Linv, *rhs, *wsol, *R, *Z;
   bf16 *PT_hi, *PT_lo, *YT_hi, *YT_lo;  // transposed split-bf16 operands ([t][ldn], [d][ldn])
   double *G64, *L64, *B64, *Z64, *X64;   // fp64 dual-form scratch (t > n only): [n][n], blocks, [n][d] x 3
+  bf16* PT_mid;                         // middle part of the transposed triple of Phi_C ([t][ldn])
 };
 // Returns launches, or -1 when a TMA descriptor cannot be encoded.
 int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float eps_w, float b_min,

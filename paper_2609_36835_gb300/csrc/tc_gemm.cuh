@@ -20,7 +20,11 @@
 //   kSplit3A -- A is a triple (h, m, l) of bf16 tensors with x = h + m + l to
 //              within 2^-24 relative (mA, mA2, mA3) and B is exact bf16 (mB):
 //              every K step issues h*B + m*B + l*B, fp32-grade products for an
-//              fp32 operand against a bf16 input.
+//              fp32 operand against a bf16 input;
+//   kSplit3S -- a Gram of one fp32 operand with itself: A and B are both the
+//              triple (mA, mA2, mA3), read at rows m0 and n0, and every K step
+//              issues hh + hm + mh + hl + lh + mm (the dropped ml, lm, ll terms
+//              are below 2^-24 relative): fp32-grade X X^T on the bf16 pipe.
 //
 // K is consumed in chunks of `chunk_k` (a multiple of 64): each chunk gets a
 // fresh accumulator and the epilogue sees every chunk separately, which lets
@@ -49,7 +53,7 @@
 
 namespace arckv {
 
-enum TcMode { kPlain = 0, kSplit = 1, kConcat = 2, kSplit3A = 3 };
+enum TcMode { kPlain = 0, kSplit = 1, kConcat = 2, kSplit3A = 3, kSplit3S = 4 };
 
 template <class E, class = void>
 struct EpiStage {
@@ -65,9 +69,11 @@ struct TcCfg {
   static constexpr bool SPLIT = MODE == kSplit;
   static constexpr int TILE_A = 128 * 128;  // bytes: 128 rows x 64 bf16
   static constexpr int TILE_B = BN * 128;
-  static constexpr int STAGE = MODE == kSplit ? 2 * (TILE_A + TILE_B)
-                               : MODE == kSplit3A ? 3 * TILE_A + TILE_B : TILE_A + TILE_B;
-  static constexpr int STAGES = (MODE == kSplit || MODE == kSplit3A) ? 3 : 4;
+  static constexpr int STAGE = MODE == kSplit     ? 2 * (TILE_A + TILE_B)
+                               : MODE == kSplit3A ? 3 * TILE_A + TILE_B
+                               : MODE == kSplit3S ? 3 * (TILE_A + TILE_B)
+                                                  : TILE_A + TILE_B;
+  static constexpr int STAGES = MODE == kSplit3S ? 2 : (MODE == kSplit || MODE == kSplit3A) ? 3 : 4;
   static constexpr int SMEM = STAGES * STAGE + 1024;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
 };
@@ -130,7 +136,7 @@ __global__ void __launch_bounds__(192, 1)
         tc::tma_prefetch(&mA2);
         tc::tma_prefetch(&mB2);
       }
-      if (MODE == kSplit3A) {
+      if (MODE == kSplit3A || MODE == kSplit3S) {
         tc::tma_prefetch(&mA2);
         tc::tma_prefetch(&mA3);
       }
@@ -150,6 +156,14 @@ __global__ void __launch_bounds__(192, 1)
           if (MODE == kConcat && kb * 64 >= K1) {
             tc::tma_load_3d(st, &mA2, kb * 64 - K1, m0, b, &full[s]);
             tc::tma_load_3d(st + C::TILE_A, &mB2, kb * 64 - K1, n0, b, &full[s]);
+          } else if (MODE == kSplit3S) {
+            // [A_h][B_h][A_m][B_m][A_l][B_l]
+            const CUtensorMap* mp[3] = {&mA, &mA2, &mA3};
+#pragma unroll
+            for (int p = 0; p < 3; ++p) {
+              tc::tma_load_3d(st + p * (C::TILE_A + C::TILE_B), mp[p], kb * 64, m0, b, &full[s]);
+              tc::tma_load_3d(st + p * (C::TILE_A + C::TILE_B) + C::TILE_A, mp[p], kb * 64, n0, b, &full[s]);
+            }
           } else {
             tc::tma_load_3d(st, &mA, kb * 64, m0, b, &full[s]);
             tc::tma_load_3d(st + C::TILE_A, &mB, kb * 64, n0, b, &full[s]);
@@ -208,6 +222,16 @@ __global__ void __launch_bounds__(192, 1)
                 const uint64_t al = tc::sdesc_k128(a + 2 * C::TILE_A + C::TILE_B + ks * 32);
                 tc::mma_f16(d, am, bd, idesc, 1u);
                 tc::mma_f16(d, al, bd, idesc, 1u);
+              }
+              if (MODE == kSplit3S) {
+                constexpr uint32_t P = C::TILE_A + C::TILE_B;
+                const uint64_t am = tc::sdesc_k128(a + P + ks * 32), bm = tc::sdesc_k128(bb + P + ks * 32);
+                const uint64_t al = tc::sdesc_k128(a + 2 * P + ks * 32), bl = tc::sdesc_k128(bb + 2 * P + ks * 32);
+                tc::mma_f16(d, ad, bm, idesc, 1u);
+                tc::mma_f16(d, am, bd, idesc, 1u);
+                tc::mma_f16(d, ad, bl, idesc, 1u);
+                tc::mma_f16(d, al, bd, idesc, 1u);
+                tc::mma_f16(d, am, bm, idesc, 1u);
               }
             }
             tc::mma_commit(&empty[s]);

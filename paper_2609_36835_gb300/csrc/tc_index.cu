@@ -28,13 +28,14 @@ struct TcEpiIndexT {
     const float* wrow;
     uint8_t* stage;
     int* stores;
-    float w;
+    float w, wn;   // this head's weight / sqrt(d_I); the next head's weight (prefetched)
     bool row_ok;
   };
   __device__ __forceinline__ void init(State& s, int b, int row, int, int M, int) const {
     s.row_ok = row < M;
     s.wrow = wts + ((long long)b * n_pos + (s.row_ok ? row / G : 0)) * H_I;
     s.w = 0.f;
+    s.wn = s.row_ok ? s.wrow[0] : 0.f;
 #pragma unroll
     for (int q = 0; q < 128; ++q) s.acc[q] = 0.f;
   }
@@ -43,13 +44,13 @@ struct TcEpiIndexT {
     s.stores = stores;
   }
   __device__ __forceinline__ void consume(State& s, int chunk, int j, float (&v)[32]) const {
-    if (j == 0) s.w = s.row_ok ? s.wrow[chunk] : 0.f;
-    const float inv = 0.08838834764831845f;  // 1 / sqrt(d_I), d_I = 128
-#pragma unroll
-    for (int q = 0; q < 32; ++q) {
-      const float x = v[q] * inv;
-      s.acc[j * 32 + q] = fmaf(s.w, x >= 0.f ? x : 0.1f * x, s.acc[j * 32 + q]);
+    // w LeakyReLU(v / sqrt(d_I)) = (w / sqrt(d_I)) max(v, 0.1 v)
+    if (j == 0) {
+      s.w = s.wn * 0.08838834764831845f;   // 1 / sqrt(d_I), d_I = 128
+      s.wn = (s.row_ok && chunk + 1 < H_I) ? s.wrow[chunk + 1] : 0.f;
     }
+#pragma unroll
+    for (int q = 0; q < 32; ++q) s.acc[j * 32 + q] = fmaf(s.w, fmaxf(v[q], 0.1f * v[q]), s.acc[j * 32 + q]);
   }
   __device__ __forceinline__ void finish(State& s, int b, int row, int n0, int, int N) const {
     const int nc = min(128, N - n0);
