@@ -15,7 +15,7 @@ inline size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct Layout {
   size_t status, kbar_hi, kbar_lo, vq, qpp, q_h, q_m, q_l, av, VT, p_h, p_m, p_l, cctx, qbar_hi, qbar_lo, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
-      colM, colInvN, Ut_hi, Ut_lo, S_hi, S_lo, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z,
+      Ut_hi, Ut_lo, S_hi, S_lo, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z,
       YT_hi, YT_lo, G64, L64, B64, Z64, X64, total;
 };
 
@@ -94,8 +94,6 @@ Layout plan(const arckv_config& c) {
   L.Y = take(H * n * 128 * f);
   L.logphi = take(H * T * f);
   const size_t ldn = (n + 7) / 8 * 8;
-  L.colM = take(H * T * f);
-  L.colInvN = take(H * T * f);
   L.Ut_hi = take(H * T * ldn * 2);
   L.Ut_lo = take(H * T * ldn * 2);
   L.S_hi = take(H * t * ldn * 2);
@@ -220,8 +218,7 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
   auto reference_attention = [&]() -> int {
     ref_done = true;
     return launch_reference_attention(D, scale, Qb, Kb, B16(L.VT), F(L.NT), (float2*)(w + L.part), F(L.z), F(L.m),
-                                      F(L.invm), B16(L.p_h), B16(L.p_m), B16(L.p_l), F(L.Y), F(L.logphi),
-                                      F(L.colM), F(L.colInvN), stt, st);
+                                      F(L.invm), B16(L.p_h), B16(L.p_m), B16(L.p_l), F(L.Y), stt, st);
   };
   if (!given_anchors && !use_indexer) {
     mark(1);
@@ -280,11 +277,14 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
   }
   int* kappa = I32(L.kappa);
   if (!given_assign) {
-    const int nla = launch_assign_tc(D, F(L.NT), F(L.colM), F(L.colInvN), anchors, B16(L.Ut_hi), B16(L.Ut_lo),
-                                     B16(L.S_hi), B16(L.S_lo), (unsigned long long*)(w + L.best), kappa, stt, st);
+    const int nla = launch_assign_tc(D, F(L.NT), F(L.logphi), anchors, B16(L.Ut_hi), B16(L.Ut_lo), B16(L.S_hi),
+                                     B16(L.S_lo), (unsigned long long*)(w + L.best), kappa, stt, st);
     if (nla < 0) return ARCKV_ERR_CUDA;
     nl += nla;
   } else {
+    const int nlc = launch_col_profiles(D, F(L.NT), F(L.logphi), nullptr, nullptr, st);   // log phi only
+    if (nlc < 0) return ARCKV_ERR_CUDA;
+    nl += nlc;
     cudaMemcpyAsync(kappa, aux->assign_in, sizeof(int) * (size_t)D.H * D.T, cudaMemcpyDeviceToDevice, st);
     nl += launch_check_assign(D, kappa, anchors, stt, st);
   }

@@ -84,14 +84,16 @@ int launch_check_anchors(const Dims& D, int* anchors, DevStatus* stt, cudaStream
 // M_j and 1/||e^{l_:j - M_j}||.  -1 when a TMA descriptor cannot be encoded.
 int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const bf16* K, const bf16* VT,
                                float* L, float2* part, float* z, float* m, float* invm, bf16* p_h, bf16* p_m,
-                               bf16* p_l, float* Y, float* logphi, float* colM, float* colInvN, DevStatus* stt,
-                               cudaStream_t st);
+                               bf16* p_l, float* Y, DevStatus* stt, cudaStream_t st);
 int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* K, float* L, float2* part,
                          DevStatus* stt, cudaStream_t st);
-// Assignment on tcgen05: transposed split-bf16 profiles, anchor rows, argmax GEMM.
-int launch_assign_tc(const Dims& D, const float* L, const float* colM, const float* colInvN, const int* anchors,
-                     bf16* Ut_hi, bf16* Ut_lo, bf16* S_hi, bf16* S_lo, unsigned long long* best, int* kappa,
-                     DevStatus* stt, cudaStream_t st);
+// Column statistics of the reference logits L: log phi [H][T] (mass weights of
+// the merge) and, when Ut_hi is given, the transposed split-bf16 profiles.
+int launch_col_profiles(const Dims& D, const float* L, float* logphi, bf16* Ut_hi, bf16* Ut_lo, cudaStream_t st);
+// Assignment on tcgen05: column statistics and transposed split-bf16 profiles
+// (log phi written on the way), anchor rows, argmax GEMM.
+int launch_assign_tc(const Dims& D, const float* L, float* logphi, const int* anchors, bf16* Ut_hi, bf16* Ut_lo,
+                     bf16* S_hi, bf16* S_lo, unsigned long long* best, int* kappa, DevStatus* stt, cudaStream_t st);
 int launch_check_assign(const Dims& D, int* kappa, const int* anchors, DevStatus* stt, cudaStream_t st);
 int launch_merge(const Dims& D, float lambda_m, const bf16* K, const int* anchors, const int* kappa,
                  const float* logphi, int* perm, int* goff, int* cursor, float* C_k, cudaStream_t st);

@@ -6,81 +6,16 @@
 // (a normalised column) and the ratios phi_j / sum_{G_r} phi_j are invariant to
 // any per-column shift, so the kernels shift column j by its own maximum M_j,
 // which keeps every column representable in fp32 when the logit range
-// exceeds the fp32 exponent range.
+// exceeds the fp32 exponent range (column statistics and profiles: the
+// col_profiles kernel of the assignment stage).
 #include "gemm.cuh"
 #include "kernels.h"
 
 namespace arckv {
 
-// Column statistics, 32 columns per CTA and 8 row slices per column: each
-// (slice, column) thread keeps an online (M, s1, s2) over its rows, the eight
-// slices are combined in slice order, then
-//   M_j = max_i l_ij,  s1 = sum_i e^{l_ij - M_j},  s2 = sum_i e^{2(l_ij - M_j)},
-//   log phi_j = M_j + log s1 - log n,  invN_j = 1 / sqrt(s2),
-// so that the normalised profile is U_ij = e^{l_ij - M_j} invN_j.
-__global__ void __launch_bounds__(256) col_stats_kernel(const float* L, float* logphi, float* colM,
-                                                        float* colInvN, int n, int T) {
-  const int b = blockIdx.y, lane = threadIdx.x & 31, slice = threadIdx.x >> 5;
-  const int j = blockIdx.x * 32 + lane;
-  __shared__ float sm[8][32], s1s[8][32], s2s[8][32];
-  const float* Lb = L + (long long)b * n * T + j;
-  const int rows = (n + 7) / 8, i0 = slice * rows, i1 = min(n, i0 + rows);
-  float mx = -INFINITY, s1 = 0.f, s2 = 0.f;
-  if (j < T) {
-    // four rows per step: one rescale of the running sums per step
-    int i = i0;
-    for (; i + 3 < i1; i += 4) {
-      const float v0 = Lb[(long long)i * T], v1 = Lb[(long long)(i + 1) * T];
-      const float v2 = Lb[(long long)(i + 2) * T], v3 = Lb[(long long)(i + 3) * T];
-      const float m4 = fmaxf(fmaxf(v0, v1), fmaxf(v2, v3));
-      if (m4 > mx) {
-        const float r = (mx == -INFINITY) ? 0.f : expf(mx - m4);
-        s1 *= r;
-        s2 *= r * r;
-        mx = m4;
-      }
-      const float e0 = expf(v0 - mx), e1 = expf(v1 - mx), e2 = expf(v2 - mx), e3 = expf(v3 - mx);
-      s1 += (e0 + e1) + (e2 + e3);
-      s2 += (e0 * e0 + e1 * e1) + (e2 * e2 + e3 * e3);
-    }
-    for (; i < i1; ++i) {
-      const float v = Lb[(long long)i * T];
-      if (v > mx) {
-        const float r = (mx == -INFINITY) ? 0.f : expf(mx - v);
-        s1 = fmaf(s1, r, 1.f);
-        s2 = fmaf(s2, r * r, 1.f);
-        mx = v;
-      } else {
-        const float e = expf(v - mx);
-        s1 += e;
-        s2 = fmaf(e, e, s2);
-      }
-    }
-  }
-  sm[slice][lane] = mx;
-  s1s[slice][lane] = s1;
-  s2s[slice][lane] = s2;
-  __syncthreads();
-  if (slice != 0 || j >= T) return;
-  float M = -INFINITY;
-  for (int q = 0; q < 8; ++q) M = fmaxf(M, sm[q][lane]);
-  float S1 = 0.f, S2 = 0.f;
-  for (int q = 0; q < 8; ++q) {
-    if (sm[q][lane] == -INFINITY) continue;
-    const float r = expf(sm[q][lane] - M);
-    S1 = fmaf(s1s[q][lane], r, S1);
-    S2 = fmaf(s2s[q][lane], r * r, S2);
-  }
-  const long long o = (long long)b * T + j;
-  logphi[o] = M + logf(S1) - logf((float)n);
-  colM[o] = M;
-  colInvN[o] = 1.0f / sqrtf(S2);
-}
-
 int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const bf16* K, const bf16* VT,
                                float* L, float2* part, float* z, float* m, float* invm, bf16* p_h, bf16* p_m,
-                               bf16* p_l, float* Y, float* logphi, float* colM, float* colInvN, DevStatus* stt,
-                               cudaStream_t st) {
+                               bf16* p_l, float* Y, DevStatus* stt, cudaStream_t st) {
   // l = scale * Q K^T on the tensor cores, with per-tile row softmax partials
   if (launch_ref_logits_tc(D, scale, Q, K, L, part, stt, st) < 0) return -1;
   // z_i = max_j l_ij (z^fit of Eq. mass_fit), m_i = sum_j e^{l_ij - z_i} = (Phi_K 1)_i
@@ -88,8 +23,7 @@ int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const 
   // Y = softmax(l) V
   const int r = launch_probs_v_tc(D, L, z, invm, p_h, p_m, p_l, VT, Y, stt, st);
   if (r < 0) return -1;
-  col_stats_kernel<<<dim3(cdiv(D.T, 32), D.H), 256, 0, st>>>(L, logphi, colM, colInvN, D.n, D.T);
-  return 3 + r;
+  return 2 + r;
 }
 
 // Caller-supplied assignment (copied into the workspace): values in [0, t)

@@ -52,37 +52,113 @@ int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* 
   return 1;
 }
 
-// One CTA per (64 rows i x 32 columns j of l, head): U_ij = exp(l_ij - M_j) * invN_j,
-// split into bf16 (hi, lo) and written transposed, Ut[b][j][i] (row stride
-// ldn >= n, a multiple of 8; the pad columns n..ldn-1 are written as zeros).
-// Reads are 128-byte row segments; each warp writes 64 i-values of one j as
-// bf16 pairs (128 bytes per tensor).
-__global__ void __launch_bounds__(256) profiles_t_kernel(const float* L, const float* colM, const float* colInvN,
-                                                         bf16* Ut_hi, bf16* Ut_lo, int n, int T, int ldn) {
-  const int b = blockIdx.z, j0 = blockIdx.x * 32, i0 = blockIdx.y * 64;
+// Column statistics of the reference logits and the transposed response
+// profiles (Sec. 3.4, Eq. response_profile), one CTA per (32 columns, head):
+//   pass 1: per column the online (M_j, s1, s2) over the n rows, the 16 row
+//     slices (warps) combined in slice order,
+//       M_j = max_i l_ij,  s1 = sum_i e^{l_ij - M_j},  s2 = sum_i e^{2(l_ij - M_j)},
+//       log phi_j = M_j + log s1 - log n  (the mass of Eq. mass_centroid),
+//       invN_j = 1 / sqrt(s2);
+//   pass 2 (Ut_hi given): U_ij = e^{l_ij - M_j} invN_j, re-read from L2 (the
+//     strip was just streamed in), split into bf16 (hi, lo) and written
+//     transposed, Ut[b][j][i] (row stride ldn >= n, a multiple of 8; the pad
+//     columns n..ldn-1 are written as zeros).
+// e^x is taken as 2^(x log2 e) after the subtraction.
+__global__ void __launch_bounds__(512) col_profiles_kernel(const float* L, float* logphi, bf16* Ut_hi, bf16* Ut_lo,
+                                                           int n, int T, int ldn) {
+  const int b = blockIdx.y, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int j0 = blockIdx.x * 32, j = j0 + lane;
+  __shared__ float red[3][16][32];
+  __shared__ float cstat[2][32];
   __shared__ float tile[64][33];
-  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
-  const float* Lb = L + (long long)b * n * T;
-  const int j = j0 + tx;
-  const float cm = j < T ? colM[(long long)b * T + j] : 0.f, ci = j < T ? colInvN[(long long)b * T + j] : 0.f;
-  for (int r = ty; r < 64; r += 8) {
-    const int i = i0 + r;
-    float u = 0.f;
-    if (i < n && j < T) u = expf(Lb[(long long)i * T + j] - cm) * ci;
-    tile[r][tx] = u;
-  }
-  __syncthreads();
-  for (int c = ty; c < 32; c += 8) {
-    const int jj = j0 + c, i = i0 + 2 * tx;
-    if (jj < T && i < ldn) {   // ldn even: i + 1 < ldn as well
-      bf16 h0, l0, h1, l1;
-      split_bf16(tile[2 * tx][c], h0, l0);
-      split_bf16(tile[2 * tx + 1][c], h1, l1);
-      const long long o = ((long long)b * T + jj) * ldn + i;
-      *(__nv_bfloat162*)(Ut_hi + o) = __halves2bfloat162(h0, h1);
-      *(__nv_bfloat162*)(Ut_lo + o) = __halves2bfloat162(l0, l1);
+  const float* Lb = L + (long long)b * n * T + j;
+  float mx = -INFINITY, s1 = 0.f, s2 = 0.f;
+  if (j < T) {
+    int i = w;
+    for (; i + 48 < n; i += 64) {   // rows i, i + 16, i + 32, i + 48: one rescale per step
+      const float v0 = Lb[(long long)i * T], v1 = Lb[(long long)(i + 16) * T];
+      const float v2 = Lb[(long long)(i + 32) * T], v3 = Lb[(long long)(i + 48) * T];
+      const float m4 = fmaxf(fmaxf(v0, v1), fmaxf(v2, v3));
+      if (m4 > mx) {
+        const float r = (mx == -INFINITY) ? 0.f : ex2_approx((mx - m4) * kLog2e);
+        s1 *= r;
+        s2 *= r * r;
+        mx = m4;
+      }
+      const float e0 = ex2_approx((v0 - mx) * kLog2e), e1 = ex2_approx((v1 - mx) * kLog2e);
+      const float e2 = ex2_approx((v2 - mx) * kLog2e), e3 = ex2_approx((v3 - mx) * kLog2e);
+      s1 += (e0 + e1) + (e2 + e3);
+      s2 += (e0 * e0 + e1 * e1) + (e2 * e2 + e3 * e3);
+    }
+    for (; i < n; i += 16) {
+      const float v = Lb[(long long)i * T];
+      if (v > mx) {
+        const float r = (mx == -INFINITY) ? 0.f : ex2_approx((mx - v) * kLog2e);
+        s1 = fmaf(s1, r, 1.f);
+        s2 = fmaf(s2, r * r, 1.f);
+        mx = v;
+      } else {
+        const float e = ex2_approx((v - mx) * kLog2e);
+        s1 += e;
+        s2 = fmaf(e, e, s2);
+      }
     }
   }
+  red[0][w][lane] = mx;
+  red[1][w][lane] = s1;
+  red[2][w][lane] = s2;
+  __syncthreads();
+  if (w == 0) {
+    float M = -INFINITY;
+    for (int q = 0; q < 16; ++q) M = fmaxf(M, red[0][q][lane]);
+    float S1 = 0.f, S2 = 0.f;
+    for (int q = 0; q < 16; ++q) {
+      if (red[0][q][lane] == -INFINITY) continue;
+      const float r = ex2_approx((red[0][q][lane] - M) * kLog2e);
+      S1 = fmaf(red[1][q][lane], r, S1);
+      S2 = fmaf(red[2][q][lane], r * r, S2);
+    }
+    if (j < T) logphi[(long long)b * T + j] = M + logf(S1) - logf((float)n);
+    cstat[0][lane] = M;
+    cstat[1][lane] = j < T ? 1.0f / sqrtf(S2) : 0.f;
+  }
+  __syncthreads();
+  if (Ut_hi == nullptr) return;
+  const float cm = cstat[0][lane], ci = cstat[1][lane];
+  for (int i0 = 0; i0 < ldn; i0 += 64) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int r = w + 16 * k, i = i0 + r;
+      tile[r][lane] = (i < n && j < T) ? ex2_approx((Lb[(long long)i * T] - cm) * kLog2e) * ci : 0.f;
+    }
+    __syncthreads();
+    // warp w writes columns 2w and 2w + 1, lane l rows i0 + 2l and i0 + 2l + 1 (ldn even)
+#pragma unroll
+    for (int c = 2 * w; c < 2 * w + 2; ++c) {
+      const int jj = j0 + c, i = i0 + 2 * lane;
+      if (jj < T && i < ldn) {
+        bf16 h0, l0, h1, l1;
+        split_bf16(tile[2 * lane][c], h0, l0);
+        split_bf16(tile[2 * lane + 1][c], h1, l1);
+        const long long o = ((long long)b * T + jj) * ldn + i;
+        *(__nv_bfloat162*)(Ut_hi + o) = __halves2bfloat162(h0, h1);
+        *(__nv_bfloat162*)(Ut_lo + o) = __halves2bfloat162(l0, l1);
+      }
+    }
+    __syncthreads();
+  }
+}
+
+int launch_col_profiles(const Dims& D, const float* L, float* logphi, bf16* Ut_hi, bf16* Ut_lo, cudaStream_t st) {
+  const int ldn = (D.n + 7) / 8 * 8;
+  // each CTA re-reads its n x 32 strip from L2: with n > 1024 a shared-memory
+  // reservation keeps at most two CTAs per SM so the live strips fit in L2
+  const int smem = D.n > 1024 ? 80 * 1024 : 0;
+  if (smem > 0 && cudaFuncSetAttribute(col_profiles_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+                      cudaSuccess)
+    return -1;
+  col_profiles_kernel<<<dim3(cdiv(D.T, 32), D.H), 512, smem, st>>>(L, logphi, Ut_hi, Ut_lo, D.n, D.T, ldn);
+  return 1;
 }
 
 // UtS[b][r] = Ut[b][S_r] (hi and lo rows).
@@ -114,12 +190,10 @@ __global__ void anchor_self_assign_kernel2(const int* anchors, int* kappa, int T
   }
 }
 
-int launch_assign_tc(const Dims& D, const float* L, const float* colM, const float* colInvN, const int* anchors,
-                     bf16* Ut_hi, bf16* Ut_lo, bf16* S_hi, bf16* S_lo, unsigned long long* best, int* kappa,
-                     DevStatus* stt, cudaStream_t st) {
+int launch_assign_tc(const Dims& D, const float* L, float* logphi, const int* anchors, bf16* Ut_hi, bf16* Ut_lo,
+                     bf16* S_hi, bf16* S_lo, unsigned long long* best, int* kappa, DevStatus* stt, cudaStream_t st) {
   const int ldn = (D.n + 7) / 8 * 8;
-  profiles_t_kernel<<<dim3(cdiv(D.T, 32), cdiv(ldn, 64), D.H), 256, 0, st>>>(L, colM, colInvN, Ut_hi, Ut_lo, D.n,
-                                                                             D.T, ldn);
+  if (launch_col_profiles(D, L, logphi, Ut_hi, Ut_lo, st) < 0) return -1;
   gather_anchor_rows_kernel<<<dim3(D.t, D.H), 128, 0, st>>>(Ut_hi, Ut_lo, anchors, S_hi, S_lo, D.T, D.t, ldn);
   cudaMemsetAsync(best, 0, sizeof(unsigned long long) * (size_t)D.H * D.T, st);
   CUtensorMap mA, mA2, mB, mB2;
