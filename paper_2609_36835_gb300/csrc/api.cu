@@ -15,7 +15,7 @@ inline size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct Layout {
   size_t status, kbar_hi, kbar_lo, vq, qpp, q_h, q_m, q_l, av, VT, p_h, p_m, p_l, cctx, qbar_hi, qbar_lo, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
-      Ut_hi, Ut_lo, S_hi, S_lo, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z,
+      qcat, wcat, Ut_hi, Ut_lo, S_hi, S_lo, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z,
       YT_hi, YT_lo, G64, L64, B64, Z64, X64, total;
 };
 
@@ -78,6 +78,8 @@ Layout plan(const arckv_config& c) {
   L.p_m = take(ptrip);
   L.p_l = take(ptrip);
   L.cctx = take(H * n * 128 * f);
+  L.qcat = take(H * n * 512 * 2);
+  L.wcat = take(H * HD * 512 * 2);
   L.qbar_hi = take(H * n * HD * 2);
   L.qbar_lo = take(H * n * HD * 2);
   L.wts = take(H * (size_t)D.n_pos * D.H_I * f);
@@ -246,8 +248,9 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
                                            B16(L.kbar_lo), stt, st);
     if (nlk < 0) return ARCKV_ERR_CUDA;
     nl += nlk;
-    QueryBufs QB{F(L.vq), F(L.qpp), F(L.NT), F(L.rA), F(L.rB), F(L.av), F(L.cctx),
-                 B16(L.q_h), B16(L.q_m), B16(L.q_l), B16(L.p_h), B16(L.p_m), B16(L.p_l), (float2*)(w + L.part)};
+    QueryBufs QB{F(L.vq),     F(L.qpp),   F(L.NT),    F(L.rA),    F(L.rB),    F(L.av),
+                 F(L.cctx),   B16(L.q_h), B16(L.q_m), B16(L.q_l), B16(L.p_h), B16(L.p_m),
+                 B16(L.p_l),  (float2*)(w + L.part), B16(L.qcat), B16(L.wcat)};
     const int nlq = launch_query_features(D, Qb, (const bf16*)X_ref, Kb, B16(L.VT), (const bf16*)idx->U_q,
                                           (const bf16*)idx->U_k, (const bf16*)idx->U_v, (const bf16*)idx->L_q,
                                           (const bf16*)idx->L_c, (const bf16*)idx->L_x, (const bf16*)idx->b_x, QB,

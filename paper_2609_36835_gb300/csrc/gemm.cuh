@@ -6,9 +6,9 @@
 // 8 x 8 register micro-tile (rows ty*4 + {0..3} and 64 + ty*4 + {0..3},
 // columns tx*4 + {0..3} and 64 + tx*4 + {0..3}).  K is walked in slabs of 16,
 // double-buffered through registers into K-major shared tiles.  Operands are
-// described by small loader structs (row-K, column-K, concatenated, and an
-// exp-transformed row-K operand) that convert bf16 or fp32 inputs to fp32 on
-// the fly and zero-fill every element outside [0, M|N) x [kb, ke).
+// described by small loader structs (row-K, column-K) that convert bf16 or
+// fp32 inputs to fp32 on the fly and zero-fill every element outside
+// [0, M|N) x [kb, ke).
 #pragma once
 #include "common.cuh"
 
@@ -108,44 +108,6 @@ struct ColK {
   }
 };
 
-// Two row-K operands concatenated along K at K1 (K1 a multiple of GBK).
-template <typename T1, typename T2>
-struct CatRowK {
-  RowK<T1> a;
-  RowK<T2> b;
-  int K1;
-  __device__ __forceinline__ void bind(int bb, int r0, int R) { a.bind(bb, r0, R); b.bind(bb, r0, R); }
-  __device__ __forceinline__ void fetch(int k0, int kend, float (&v)[8]) const {
-    if (k0 < K1) a.fetch(k0, min(kend, K1), v);
-    else b.fetch(k0 - K1, kend - K1, v);
-  }
-  __device__ __forceinline__ void store(float* S, const float (&v)[8]) const { a.store(S, v); }
-};
-
-// Row-K fp32 operand seen through v -> exp(alpha * v - shift[r]) * mul[r].
-struct RowKExp {
-  RowK<float> x;
-  const float* shift;
-  const float* mul;
-  long long sbs;
-  float alpha;
-  const float* sh;
-  const float* mu;
-  __device__ __forceinline__ void bind(int b, int r0, int R) {
-    x.bind(b, r0, R);
-    sh = shift + (long long)b * sbs;
-    mu = mul + (long long)b * sbs;
-  }
-  __device__ __forceinline__ void fetch(int k0, int kend, float (&v)[8]) const {
-    x.fetch(k0, kend, v);
-    const int r = x.row();
-    const float s = (r < x.R) ? sh[r] : 0.f, m = (r < x.R) ? mu[r] : 0.f;
-#pragma unroll
-    for (int q = 0; q < 8; ++q) v[q] = x.inb(k0, kend, q) ? expf(alpha * v[q] - s) * m : 0.f;
-  }
-  __device__ __forceinline__ void store(float* S, const float (&v)[8]) const { x.store(S, v); }
-};
-
 __device__ __forceinline__ int tile_row(int i) { return (threadIdx.x >> 4) * 4 + (i & 3) + (i >> 2) * 64; }
 __device__ __forceinline__ int tile_col(int j) { return (threadIdx.x & 15) * 4 + (j & 3) + (j >> 2) * 64; }
 
@@ -230,67 +192,6 @@ struct EpiStore {
           for (int q = 0; q < 4; ++q)
             if (n + q < N) base[(long long)(n + q) * ldc + m] = vv[q];
         }
-      }
-    }
-  }
-};
-
-// Per-row RMS normalisation over the tile's 128 columns (one d_I block):
-// C = acc / sqrt(sum(acc^2) / 128 + 1e-6)   (App. A.1, the N(.) of Eq. indexer_projection)
-struct EpiBlockNorm {
-  float* C;
-  long long cbs;
-  int ldc;
-  __device__ __forceinline__ void apply(int b, int, int m0, int n0, int M, int, float (&acc)[8][8],
-                                        float*) const {
-    float* base = C + (long long)b * cbs;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      float ss = 0.f;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) ss = fmaf(acc[i][j], acc[i][j], ss);
-#pragma unroll
-      for (int o = 1; o < 16; o <<= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-      const float sc = 1.0f / sqrtf(ss * (1.0f / 128.0f) + 1e-6f);
-      const int m = m0 + tile_row(i);
-      if (m >= M) continue;
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int n = n0 + (threadIdx.x & 15) * 4 + h * 64;
-        *(float4*)(base + (long long)m * ldc + n) =
-            make_float4(acc[i][h * 4] * sc, acc[i][h * 4 + 1] * sc, acc[i][h * 4 + 2] * sc, acc[i][h * 4 + 3] * sc);
-      }
-    }
-  }
-};
-
-// EpiBlockNorm with a split-bf16 output pair instead of fp32.
-struct EpiBlockNormSplit {
-  bf16* Hi;
-  bf16* Lo;
-  long long cbs;
-  int ldc;
-  __device__ __forceinline__ void apply(int b, int, int m0, int n0, int M, int, float (&acc)[8][8],
-                                        float*) const {
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      float ss = 0.f;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) ss = fmaf(acc[i][j], acc[i][j], ss);
-#pragma unroll
-      for (int o = 1; o < 16; o <<= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-      const float sc = 1.0f / sqrtf(ss * (1.0f / 128.0f) + 1e-6f);
-      const int m = m0 + tile_row(i);
-      if (m >= M) continue;
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int n = n0 + (threadIdx.x & 15) * 4 + h * 64;
-        const long long off = (long long)b * cbs + (long long)m * ldc + n;
-        __align__(8) bf16 hi[4], lo[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) split_bf16(acc[i][h * 4 + q] * sc, hi[q], lo[q]);
-        *(uint2*)(Hi + off) = *(const uint2*)hi;
-        *(uint2*)(Lo + off) = *(const uint2*)lo;
       }
     }
   }

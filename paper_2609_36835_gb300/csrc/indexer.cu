@@ -65,11 +65,9 @@ int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf1
               D.H, D.n, D.d_A, D.d, 1, st);
   ++nl;
   // q_bar = N(L_q q + L_c c) per block, as a split-bf16 pair
-  CatRowK<bf16, float> A{{Q, nd, D.d}, {B.cctx, nA, D.d_A}, D.d};
-  CatRowK<bf16, bf16> W{{L_q, (long long)D.HD * D.d, D.d}, {L_c, (long long)D.HD * D.d_A, D.d_A}, D.d};
-  launch_gemm(A, W, EpiBlockNormSplit{qbar_hi, qbar_lo, (long long)D.n * D.HD, D.HD}, D.H, D.n, D.HD,
-              D.d + D.d_A, 1, st);
-  ++nl;
+  r = launch_query_proj_tc(D, Q, B.cctx, L_q, L_c, B.qcat, B.wcat, qbar_hi, qbar_lo, stt, st);
+  if (r < 0) return -1;
+  nl += r;
   index_weights_kernel<<<dim3(D.n_pos, D.H), 32 * D.H_I, 0, st>>>(X, L_x, b_x, wts, D.d_x, D.H_I, D.n_pos);
   ++nl;
   return nl;

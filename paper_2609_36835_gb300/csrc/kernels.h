@@ -40,6 +40,8 @@ constexpr int kCholNB = 64;  // Cholesky block size
 // ---- indexer (Sec. 3.3, App. A.1) --------------------------------------
 // k_bar = N(L_k k + L_v v) per d_I block, as a split-bf16 pair (one tcgen05
 // GEMM over [K | V] against [L_k | L_v]).
+int launch_query_proj_tc(const Dims& D, const bf16* Q, const float* cctx, const bf16* L_q, const bf16* L_c,
+                         bf16* qcat, bf16* wcat, bf16* qbar_hi, bf16* qbar_lo, DevStatus* stt, cudaStream_t st);
 int launch_key_features_tc(const Dims& D, const bf16* K, const bf16* V, const bf16* L_k, const bf16* L_v,
                            bf16* kbar_hi, bf16* kbar_lo, DevStatus* stt, cudaStream_t st);
 // Scratch of the query-side features.
@@ -47,6 +49,7 @@ struct QueryBufs {
   float *vq, *qpp, *logits, *rshift, *rmul, *av, *cctx;
   bf16 *q_h, *q_m, *q_l, *p_h, *p_m, *p_l;
   float2* part;  // per-(row, 128-column tile) softmax partials of the logits
+  bf16 *qcat, *wcat;   // K-concatenated operands of the q_bar GEMM ([n][512], [HD][512])
 };
 // value context c (Eq. value_context), q_bar (Eq. indexer_projection), w.
 // VT is V transposed ([H][d][ldT] bf16, launch_transpose_v).  -1 on a TMA failure.
