@@ -35,7 +35,8 @@ METRIC = "compaction s/context and context tokens/s at Llama-3.1-8B shape; % roo
 UNIT = "context tokens/s"
 DEFAULT_WORKLOAD = "llama8b_T8192_r10"
 PROFILE_SUMMARY = ROOT / "profiles" / "index_logits_tc_llama8b_layer_T8192.md"
-DOMINANT_SOURCES = [ROOT / "paper_2609_36835_gb300" / "csrc" / f for f in ("tc_index.cu", "tc_gemm.cuh", "tc.cuh")]
+DOMINANT_SOURCES = [ROOT / "paper_2609_36835_gb300" / "csrc" / f
+                    for f in ("tc_index.cu", "tc_gemm.cuh", "tc.cuh", "common.cuh")]
 FALLBACK_BF16_SUSTAINED_TFLOPS = 1700.0
 
 

@@ -58,7 +58,7 @@ arckv_status validate(const arckv_config* c) {
 Layout plan(const arckv_config& c) {
   const Dims D = dims_of(c);
   const size_t H = D.H, T = D.T, n = D.n, t = D.t, HD = D.HD, f = 4;
-  const size_t nblk = (t + kCholNB - 1) / kCholNB, ntile = (T + 127) / 128;
+  const size_t nblk = (t + kCholNB - 1) / kCholNB, ntile = (T + 63) / 64;   // softmax partials: 128 columns each, or kIndexPartW >= 64
   Layout L;
   size_t o = 0;
   auto take = [&](size_t bytes) { size_t r = o; o += up(bytes); return r; };
@@ -230,7 +230,7 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
     nl += nlr0;
     if (cfg->selector == ARCKV_SELECTOR_HA) {
       // p = softmax(l): the same pooling as the index scores, on l's row partials
-      nl += launch_index_pool(D, F(L.NT), (const float2*)(w + L.part), F(L.lse), F(L.s), st);
+      nl += launch_index_pool(D, F(L.NT), (const float2*)(w + L.part), cdiv(D.T, 128), F(L.lse), F(L.s), st);
     } else {
       float* vq = F(L.vq);   // n-sized rows in the (unused) indexer buffers
       const size_t hn = (size_t)D.H * D.n;
@@ -263,7 +263,8 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
     if (nli < 0) return ARCKV_ERR_CUDA;
     nl += nli;
     mark(2);
-    nl += launch_index_pool(D, F(L.NT), (const float2*)(w + L.part), F(L.lse), F(L.s), st);
+    nl += launch_index_pool(D, F(L.NT), (const float2*)(w + L.part), cdiv(D.T, kIndexPartW), F(L.lse), F(L.s),
+                            st);
     nl += launch_top_t(D, cfg->t, F(L.s), anchors, stt, st);
     nl += launch_check_anchors(D, anchors, stt, st);   // a selection fault becomes a status, not a stray index
   } else {

@@ -124,8 +124,8 @@ __global__ void __launch_bounds__(256) pool_kernel(const float* I, const float* 
   }
 }
 
-int launch_index_pool(const Dims& D, const float* I, const float2* part, float* lse, float* s, cudaStream_t st) {
-  const int ntiles = cdiv(D.T, GBN);
+int launch_index_pool(const Dims& D, const float* I, const float2* part, int ntiles, float* lse, float* s,
+                      cudaStream_t st) {
   lse_reduce_kernel<<<dim3(cdiv(D.n, 8), D.H), 256, 0, st>>>(part, lse, D.n, ntiles);
   pool_kernel<<<dim3(cdiv(D.T, 32), D.H), 256, 0, st>>>(I, lse, s, D.n, D.T);
   return 2;

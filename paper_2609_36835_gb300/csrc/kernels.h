@@ -74,7 +74,10 @@ int launch_index_logits(const Dims& D, const bf16* qbar_hi, const bf16* qbar_lo,
                         const bf16* kbar_lo, const float* wts, float* I, float2* part, DevStatus* stt,
                         cudaStream_t st);
 // row log-sum-exp and pooled s (Eq. indexer_pooling).
-int launch_index_pool(const Dims& D, const float* I, const float2* part, float* lse, float* s, cudaStream_t st);
+// Index-logit softmax partials cover kIndexPartW columns each ([H][n][ceil(T / kIndexPartW)]).
+constexpr int kIndexPartW = 128;
+int launch_index_pool(const Dims& D, const float* I, const float2* part, int ntiles, float* lse, float* s,
+                      cudaStream_t st);
 
 // ---- selection (Eq. persistent_support) ----------------------------------
 // t_budget: the configured t (the per-chunk budgets derive from it); D.t is the realized count

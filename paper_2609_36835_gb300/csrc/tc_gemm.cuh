@@ -40,6 +40,10 @@
 //   void init(State&, int b, int row, int n0, int M, int N);
 //   void consume(State&, int chunk, int j, float (&v)[32]);  columns n0+32j..
 //   void finish(State&, int b, int row, int n0, int M, int N);
+// An epilogue that declares kEpiWarps = 8 gets two warps per TMEM lane
+// quarter: warps 2..5 drain the first BN/2 columns and warps 6..9 the rest,
+// and each sees a tile of BN/2 columns (init/finish get its first column;
+// consume's j counts 32-column chunks within it).
 // An epilogue that declares kStageBytes gets that much shared memory per
 // epilogue warp (1024-byte aligned) through attach(State&, uint8_t*, int*)
 // after init, for staging TMA stores, with a per-thread count of the stores
@@ -54,6 +58,15 @@
 namespace arckv {
 
 enum TcMode { kPlain = 0, kSplit = 1, kConcat = 2, kSplit3A = 3, kSplit3S = 4 };
+
+template <class E, class = void>
+struct EpiWarps {
+  static constexpr int value = 4;
+};
+template <class E>
+struct EpiWarps<E, std::void_t<decltype(E::kEpiWarps)>> {
+  static constexpr int value = E::kEpiWarps;
+};
 
 template <class E, class = void>
 struct EpiStage {
@@ -79,13 +92,16 @@ struct TcCfg {
 };
 
 template <int BN, int MODE, class Epi>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(64 + 32 * EpiWarps<Epi>::value, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
                    const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mB2,
                    const __grid_constant__ CUtensorMap mA3, const __grid_constant__ Epi epi, int H, int M, int N, int K,
                    int chunk_k, int K1, DevStatus* stt) {
   using C = TcCfg<BN, MODE>;
   constexpr int SB = EpiStage<Epi>::bytes;
+  constexpr int NE = EpiWarps<Epi>::value;   // epilogue warps: 4 or 8
+  constexpr int JG = BN / 32 / (NE / 4);     // 32-column chunks per epilogue warp
+  static_assert(NE == 4 || NE == 8, "4 or 8 epilogue warps");
   constexpr bool SPLIT = C::SPLIT;
   constexpr int STAGES = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -115,7 +131,7 @@ __global__ void __launch_bounds__(192, 1)
     }
     for (int i = 0; i < 2; ++i) {
       tc::mbar_init(&accf[i], 1);
-      tc::mbar_init(&acce[i], 4);
+      tc::mbar_init(&acce[i], NE);
     }
     tc::mbar_init(&drain, 1);
     abort_flag = 0;
@@ -245,34 +261,35 @@ __global__ void __launch_bounds__(192, 1)
       tc::mbar_wait(&drain, 0, &never, stt);
     }
   } else {
-    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int q = warp & 3;              // TMEM lane quarter this warp may access
+    const int cg = ((warp - 2) >> 2) * JG;   // first 32-column chunk of this warp
     const int row = q * 32 + lane;
     bool ok = true;
-    int cg = 0;
+    int kc = 0;
     int stores = 0;   // staged stores issued by this warp (identical in all its lanes)
     for (int tl = blockIdx.x; tl < ntiles && ok; tl += gridDim.x) {
       int b, m0, n0;
       tile_coords(tl, b, m0, n0);
       typename Epi::State es;
-      epi.init(es, b, m0 + row, n0, M, N);
+      epi.init(es, b, m0 + row, n0 + cg * 32, M, N);
       if constexpr (SB > 0) epi.attach(es, base + STAGES * C::STAGE + (warp - 2) * SB, &stores);
-      for (int c = 0; c < nchunks; ++c, ++cg) {
-        const int buf = cg & 1;
-        ok = tc::mbar_wait(&accf[buf], (cg >> 1) & 1, abortp, stt);
+      for (int c = 0; c < nchunks; ++c, ++kc) {
+        const int buf = kc & 1;
+        ok = tc::mbar_wait(&accf[buf], (kc >> 1) & 1, abortp, stt);
         ok = __all_sync(0xffffffffu, ok);
         if (!ok) break;
         tc::fence_after_sync();
 #pragma unroll
-        for (int j = 0; j < BN / 32; ++j) {
+        for (int j = 0; j < JG; ++j) {
           float v[32];
-          tc::tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN + j * 32), v);
+          tc::tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN + (cg + j) * 32), v);
           epi.consume(es, c, j, v);
         }
         tc::fence_before_sync();
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&acce[buf]);
       }
-      if (ok) epi.finish(es, b, m0 + row, n0, M, N);
+      if (ok) epi.finish(es, b, m0 + row, n0 + cg * 32, M, N);
     }
     if constexpr (SB > 0) {
       if (lane == 0) tc::bulk_wait_all();
@@ -298,14 +315,15 @@ inline cudaError_t launch_tc_gemm(const CUtensorMap& mA, const CUtensorMap& mB, 
                                   const CUtensorMap& mB2, const Epi& epi, int H, int M, int N, int K, int chunk_k,
                                   DevStatus* stt, cudaStream_t st, int K1 = 0, const CUtensorMap* mA3 = nullptr) {
   using C = TcCfg<BN, MODE>;
-  constexpr int smem = C::SMEM + 4 * EpiStage<Epi>::bytes;
+  constexpr int NE = EpiWarps<Epi>::value;
+  constexpr int smem = C::SMEM + NE * EpiStage<Epi>::bytes;
   static_assert(smem <= 227 * 1024, "stage ring and epilogue staging exceed shared memory");
   auto kern = tc_gemm_kernel<BN, MODE, Epi>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const long long ntiles = (long long)cdiv(N, BN) * cdiv(M, 128) * H;
   const int grid = (int)std::min<long long>(ntiles, tc_gemm_sm_count());
-  kern<<<grid, 192, smem, st>>>(mA, mB, mA2, mB2, mA3 ? *mA3 : mA, epi, H, M, N, K, chunk_k, K1, stt);
+  kern<<<grid, 64 + 32 * NE, smem, st>>>(mA, mB, mA2, mB2, mA3 ? *mA3 : mA, epi, H, M, N, K, chunk_k, K1, stt);
   return cudaGetLastError();
 }
 
@@ -344,16 +362,17 @@ struct TcEpiStore {
 
 // Staged TMA store of one warp's 32 rows x 32 columns at (x, y, b): the rows
 // go into a 128-byte-swizzled staging buffer (conflict-free 16-byte stores)
-// and one lane issues the tiled bulk store.  Two buffers alternate by issued
-// store; before a buffer is rewritten, at most one store (the other
-// buffer's) may still be reading.  Boxes wholly outside [0, N) x [0, M) are
-// skipped (warp-uniform).  v is scaled by alpha.
+// and one lane issues the tiled bulk store.  NBUF buffers of 4 KB rotate by
+// issued store; before a buffer is rewritten, at most NBUF - 1 stores (the
+// other buffers') may still be reading.  Boxes wholly outside [0, N) x [0, M)
+// are skipped (warp-uniform).  v is scaled by alpha.
+template <int NBUF = 2>
 __device__ __forceinline__ void staged_store_32x32(const CUtensorMap* map, uint8_t* stage, int* stores, int x, int y,
                                                    int b, int M, int N, const float* v, float alpha) {
   if (y >= M || x >= N) return;
   const int lane = threadIdx.x & 31;
-  uint8_t* buf = stage + (*stores & 1) * 4096;
-  if (lane == 0) tc::bulk_wait_read<1>();
+  uint8_t* buf = stage + (*stores % NBUF) * 4096;
+  if (lane == 0) tc::bulk_wait_read<NBUF - 1>();
   __syncwarp();
 #pragma unroll
   for (int k = 0; k < 8; ++k)

@@ -7,24 +7,30 @@
 // columns) at a time: every head's partial dot products land in their own
 // TMEM accumulator and the epilogue folds them through the LeakyReLU and the
 // row's head weight w_ia before the next head is added.  The epilogue then
-// writes the tile's row-softmax partials (max, sum of exp) and the I tile.
+// writes the row-softmax partials (max, sum of exp) of each kIndexPartW
+// columns and the I tile.
 #include "kernels.h"
 #include "tc_gemm.cuh"
 
 namespace arckv {
 
-// kTma: the I tile leaves through TMA stores staged in shared memory (32 x 32
-// boxes, two buffers per epilogue warp); else each row writes its 128 values.
-template <bool kTma>
+// Each epilogue thread folds one row of kW columns (kW = 128: four epilogue
+// warps, the whole tile; kW = 64: eight warps, half a tile each) and writes
+// their row-softmax partials, part[b][row][n0 / kW].  kTma: the I tile leaves
+// through TMA stores staged in shared memory (32 x 32 boxes; two buffers per
+// warp with four warps, one with eight); else each row writes its kW values.
+template <bool kTma, int kW_>
 struct TcEpiIndexT {
+  static constexpr int kW = kW_;
+  static constexpr int kEpiWarps = 128 / kW * 4;
+  static constexpr int kStageBytes = kTma ? (kW == 128 ? 2 : 1) * 32 * 128 : 0;
   const float* wts;  // [H][n_pos][H_I]
   float* I;          // [H][n][T]
-  float2* part;      // [H][n][ntiles]
+  float2* part;      // [H][n][ntiles], ntiles = ceil(T / kW)
   int n, T, H_I, G, n_pos, ntiles;
   CUtensorMap map;   // kTma: I as [H][n][T], box {32, 32, 1}, 128-byte swizzle
-  static constexpr int kStageBytes = kTma ? 2 * 32 * 128 : 0;
   struct State {
-    float acc[128];
+    float acc[kW];
     const float* wrow;
     uint8_t* stage;
     int* stores;
@@ -37,7 +43,7 @@ struct TcEpiIndexT {
     s.w = 0.f;
     s.wn = s.row_ok ? s.wrow[0] : 0.f;
 #pragma unroll
-    for (int q = 0; q < 128; ++q) s.acc[q] = 0.f;
+    for (int q = 0; q < kW; ++q) s.acc[q] = 0.f;
   }
   __device__ __forceinline__ void attach(State& s, uint8_t* stage, int* stores) const {
     s.stage = stage;
@@ -53,14 +59,14 @@ struct TcEpiIndexT {
     for (int q = 0; q < 32; ++q) s.acc[j * 32 + q] = fmaf(s.w, fmaxf(v[q], 0.1f * v[q]), s.acc[j * 32 + q]);
   }
   __device__ __forceinline__ void finish(State& s, int b, int row, int n0, int, int N) const {
-    const int nc = min(128, N - n0);
-    if (s.row_ok) {
-      // eight independent max / sum chains over the tile's columns
+    const int nc = min(kW, N - n0);
+    if (s.row_ok && nc > 0) {
+      // eight independent max / sum chains over the half tile's columns
       float m8[8], a8[8];
 #pragma unroll
       for (int k = 0; k < 8; ++k) m8[k] = -INFINITY;
 #pragma unroll
-      for (int q = 0; q < 128; ++q)
+      for (int q = 0; q < kW; ++q)
         if (q < nc) m8[q & 7] = fmaxf(m8[q & 7], s.acc[q]);
       const float mx =
           fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])), fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
@@ -68,26 +74,27 @@ struct TcEpiIndexT {
 #pragma unroll
       for (int k = 0; k < 8; ++k) a8[k] = 0.f;
 #pragma unroll
-      for (int q = 0; q < 128; ++q)
+      for (int q = 0; q < kW; ++q)
         if (q < nc) a8[q & 7] += ex2_approx(fmaf(s.acc[q], kLog2e, -ml));
       const float sm = ((a8[0] + a8[1]) + (a8[2] + a8[3])) + ((a8[4] + a8[5]) + (a8[6] + a8[7]));
-      part[((long long)b * n + row) * ntiles + n0 / 128] = make_float2(mx, sm);
+      part[((long long)b * n + row) * ntiles + n0 / kW] = make_float2(mx, sm);
     }
     if constexpr (kTma) {
       // rows past n and columns past T fall outside the tensor map: not written
       const int y = row & ~31;
 #pragma unroll
-      for (int j = 0; j < 4; ++j) staged_store_32x32(&map, s.stage, s.stores, n0 + 32 * j, y, b, n, T, s.acc + 32 * j, 1.f);
+      for (int j = 0; j < kW / 32; ++j)
+        staged_store_32x32<kW == 128 ? 2 : 1>(&map, s.stage, s.stores, n0 + 32 * j, y, b, n, T, s.acc + 32 * j, 1.f);
     } else {
-      if (!s.row_ok) return;
+      if (!s.row_ok || nc <= 0) return;
       float* dst = I + ((long long)b * n + row) * T + n0;
-      if ((T & 3) == 0 && nc == 128) {
+      if ((T & 3) == 0 && nc == kW) {
 #pragma unroll
-        for (int q = 0; q < 128; q += 4)
+        for (int q = 0; q < kW; q += 4)
           *(float4*)(dst + q) = make_float4(s.acc[q], s.acc[q + 1], s.acc[q + 2], s.acc[q + 3]);
       } else {
 #pragma unroll
-        for (int q = 0; q < 128; ++q)
+        for (int q = 0; q < kW; ++q)
           if (q < nc) dst[q] = s.acc[q];
       }
     }
@@ -102,13 +109,13 @@ int launch_index_logits(const Dims& D, const bf16* qbar_hi, const bf16* qbar_lo,
       !encode_bf16_map_3d(&mB, kbar_hi, D.HD, D.T, D.H, 128) || !encode_bf16_map_3d(&mB2, kbar_lo, D.HD, D.T, D.H, 128))
     return -1;
   if ((D.T & 3) == 0 && ((uintptr_t)I & 15u) == 0) {
-    TcEpiIndexT<true> epi{wts, I, part, D.n, D.T, D.H_I, D.G, D.n_pos, cdiv(D.T, 128), {}};
+    TcEpiIndexT<true, kIndexPartW> epi{wts, I, part, D.n, D.T, D.H_I, D.G, D.n_pos, cdiv(D.T, kIndexPartW), {}};
     if (!encode_f32_map_3d(&epi.map, I, D.T, D.n, D.H, 32, 32, D.T, (uint64_t)D.n * D.T, true)) return -1;
     if (launch_tc_gemm<128, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.n, D.T, D.HD, 128, stt, st) != cudaSuccess)
       return -1;
     return 1;
   }
-  TcEpiIndexT<false> epi{wts, I, part, D.n, D.T, D.H_I, D.G, D.n_pos, cdiv(D.T, 128), {}};
+  TcEpiIndexT<false, kIndexPartW> epi{wts, I, part, D.n, D.T, D.H_I, D.G, D.n_pos, cdiv(D.T, kIndexPartW), {}};
   if (launch_tc_gemm<128, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.n, D.T, D.HD, 128, stt, st) != cudaSuccess) return -1;
   return 1;
 }
