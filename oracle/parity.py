@@ -5,8 +5,11 @@ Tolerances (applied by the tests, stated here once):
     relative error <= 1e-3 on the oracle's top-2t scores;
   * anchor sets: identical, except that positions whose oracle score lies
     within ``band`` (relative to the oracle's t-th largest score) of that
-    threshold may be exchanged for one another (a tie band); with chunked
-    selection the same holds within each chunk at its own t_c-th score;
+    threshold, widened by the GPU scores' own relative errors at the position
+    and at the t-th key, may be exchanged for one another (a tie band: top-t
+    cannot order keys closer than the errors of the scores that rank them);
+    with chunked selection the same holds within each chunk at its own t_c-th
+    score;
   * assignment (an argmax whose exact ties are frequent): where the oracle's
     best and second-best similarities differ by more than ``tau`` the GPU
     must agree; elsewhere the GPU's choice must be within ``tau`` of the best;
@@ -39,21 +42,34 @@ def score_errors(s_gpu: np.ndarray, s: np.ndarray, t: int):
     return rel_inf(s_gpu, s), float(np.max(np.abs(s_gpu[top] - s[top]) / np.abs(s[top])))
 
 
-def anchors_match(S_gpu: np.ndarray, S: np.ndarray, s: np.ndarray, t: int, band: float):
+def anchors_match(S_gpu: np.ndarray, S: np.ndarray, s: np.ndarray, t: int, band: float, s_gpu=None):
     """True if the anchor sets agree up to exchanges inside the tie band.
-    Returns (ok, number of exchanged positions, widest relative gap seen)."""
-    thr = np.sort(s)[::-1][t - 1]
+
+    Top-t keeps the t largest scores; a key can only enter or leave the set
+    through an error of the scores that decided it.  An exchanged position j
+    is accepted when its oracle score lies within ``band`` (relative) of the
+    oracle's t-th score, widened, when the GPU scores ``s_gpu`` are given, by
+    the GPU's own relative errors at j and at the t-th key: the two keys'
+    order is then not fixed by scores carrying those errors.
+    Returns (ok, number of exchanged positions, widest unexplained relative gap)."""
+    order = np.argsort(-s, kind="stable")
+    k_thr = int(order[t - 1])
+    thr = s[k_thr]
     a, b = set(map(int, S_gpu)), set(map(int, S))
     diff = sorted(a ^ b)
     if len(a) != len(b) or len(S_gpu) != t:
         return False, len(diff), float("inf")
     if not diff:
         return True, 0, 0.0
-    gaps = [abs(s[j] - thr) / thr for j in diff]
-    return bool(max(gaps) <= band), len(diff), float(max(gaps))
+
+    def err(j):
+        return 0.0 if s_gpu is None else abs(float(s_gpu[j]) - s[j]) / abs(s[j])
+
+    excess = [abs(s[j] - thr) / thr - err(j) - err(k_thr) for j in diff]
+    return bool(max(excess) <= band), len(diff), float(max(excess))
 
 
-def anchors_match_chunked(S_gpu: np.ndarray, S: np.ndarray, s: np.ndarray, chunks, band: float):
+def anchors_match_chunked(S_gpu: np.ndarray, S: np.ndarray, s: np.ndarray, chunks, band: float, s_gpu=None):
     """anchors_match within every chunk (start, T_c, t_c) of the chunked
     selection of App. A.3, the tie band taken at the chunk's own t_c-th score.
     Returns (ok, exchanged positions, widest relative gap)."""
@@ -62,7 +78,8 @@ def anchors_match_chunked(S_gpu: np.ndarray, S: np.ndarray, s: np.ndarray, chunk
         def part(X):
             X = np.asarray(X)
             return X[(X >= start) & (X < start + Tc)] - start
-        ok, nd, gap = anchors_match(part(S_gpu), part(S), s[start:start + Tc], tc, band)
+        sg = None if s_gpu is None else s_gpu[start:start + Tc]
+        ok, nd, gap = anchors_match(part(S_gpu), part(S), s[start:start + Tc], tc, band, sg)
         if not ok:
             return False, nd, gap
         n_ex += nd

@@ -14,9 +14,9 @@ constexpr size_t kAlign = 256;
 inline size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct Layout {
-  size_t status, kbar_hi, kbar_lo, vq, qpp, q_h, q_m, q_l, av, VT, p_h, p_m, p_l, cctx, qbar_hi, qbar_lo, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
+  size_t status, kbar_hi, kbar_lo, vq, qpp, q_h, q_m, q_l, av, VT, p_h, p_m, p_l, vq3, av3, ukt, qbar_hi, qbar_lo, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
       qcat, wcat, Ut_hi, Ut_lo, S_hi, S_lo, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z,
-      YT_hi, YT_lo, G64, L64, B64, Z64, X64, total;
+      ck3, YT_hi, YT_lo, G64, L64, B64, Z64, X64, total;
 };
 
 Dims dims_of(const arckv_config& c) {
@@ -66,8 +66,8 @@ Layout plan(const arckv_config& c) {
   const size_t ldT = (T + 7) / 8 * 8;
   L.kbar_hi = take(H * T * HD * 2);
   L.kbar_lo = take(H * T * HD * 2);
-  L.vq = take(H * n * 128 * f);
-  L.qpp = take(H * n * 128 * f);
+  L.vq = take(H * n * 128 * f);    // VI selector scratch
+  L.qpp = take(H * n * 128 * f);   // VI selector scratch
   L.q_h = take(H * n * 128 * 2);
   L.q_m = take(H * n * 128 * 2);
   L.q_l = take(H * n * 128 * 2);
@@ -77,8 +77,10 @@ Layout plan(const arckv_config& c) {
   L.p_h = take(ptrip);
   L.p_m = take(ptrip);
   L.p_l = take(ptrip);
-  L.cctx = take(H * n * 128 * f);
   L.qcat = take(H * n * 512 * 2);
+  L.vq3 = take(3 * H * n * 128 * 2);
+  L.av3 = take(3 * H * n * 128 * 2);
+  L.ukt = take(H * 128 * 128 * 2);
   L.wcat = take(H * HD * 512 * 2);
   L.qbar_hi = take(H * n * HD * 2);
   L.qbar_lo = take(H * n * HD * 2);
@@ -113,6 +115,7 @@ Layout plan(const arckv_config& c) {
   L.wsol = take(H * t * f);
   L.R = take(H * t * 128 * f);
   L.Z = take(H * t * 128 * f);
+  L.ck3 = take(3 * H * t * 128 * 2);
   L.YT_hi = take(H * 128 * ldn * 2);
   L.YT_lo = take(H * 128 * ldn * 2);
   // fp64 dual-form scratch, only when t > n
@@ -232,7 +235,7 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
       // p = softmax(l): the same pooling as the index scores, on l's row partials
       nl += launch_index_pool(D, F(L.NT), (const float2*)(w + L.part), cdiv(D.T, 128), F(L.lse), F(L.s), st);
     } else {
-      float* vq = F(L.vq);   // n-sized rows in the (unused) indexer buffers
+      float* vq = F(L.vq);   // VI scratch: n-sized rows here, O^(-a) in L.qpp
       const size_t hn = (size_t)D.H * D.n;
       ViBufs VB{(int*)vq, vq + hn, vq + 2 * hn, vq + 3 * hn, vq + 4 * hn, F(L.qpp), F(L.best), F(L.Ut_hi),
                 B16(L.p_h), B16(L.p_m), B16(L.p_l), B16(L.q_h), B16(L.q_m), B16(L.q_l)};
@@ -248,9 +251,10 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
                                            B16(L.kbar_lo), stt, st);
     if (nlk < 0) return ARCKV_ERR_CUDA;
     nl += nlk;
-    QueryBufs QB{F(L.vq),     F(L.qpp),   F(L.NT),    F(L.rA),    F(L.rB),    F(L.av),
-                 F(L.cctx),   B16(L.q_h), B16(L.q_m), B16(L.q_l), B16(L.p_h), B16(L.p_m),
-                 B16(L.p_l),  (float2*)(w + L.part), B16(L.qcat), B16(L.wcat)};
+    QueryBufs QB{F(L.NT),    F(L.rA),    F(L.rB),    F(L.av),     B16(L.q_h),
+                 B16(L.q_m), B16(L.q_l), B16(L.p_h), B16(L.p_m), B16(L.p_l),
+                 (float2*)(w + L.part),  B16(L.qcat), B16(L.wcat), B16(L.vq3), B16(L.av3),
+                 B16(L.ukt)};
     const int nlq = launch_query_features(D, Qb, (const bf16*)X_ref, Kb, B16(L.VT), (const bf16*)idx->U_q,
                                           (const bf16*)idx->U_k, (const bf16*)idx->U_v, (const bf16*)idx->L_q,
                                           (const bf16*)idx->L_c, (const bf16*)idx->L_x, (const bf16*)idx->b_x, QB,
@@ -299,7 +303,8 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
   FitBufs B{F(L.LC),  F(L.Phi), F(L.Gram), F(L.Linv), F(L.rhs), F(L.wsol), F(L.R), F(L.Z),
             (bf16*)(w + L.S_hi), (bf16*)(w + L.S_lo), (bf16*)(w + L.YT_hi), (bf16*)(w + L.YT_lo),
             (double*)(w + L.G64), (double*)(w + L.L64), (double*)(w + L.B64), (double*)(w + L.Z64),
-            (double*)(w + L.X64), (bf16*)(w + L.Ut_hi)};   // Ut_hi [H][T][ldn] is free after the assignment
+            (double*)(w + L.X64), (bf16*)(w + L.Ut_hi),   // Ut_hi [H][T][ldn] is free after the assignment
+            (bf16*)(w + L.ck3)};
   const int nlf = launch_fits(D, scale, cfg->ridge_w, cfg->ridge_v, cfg->eps_w, cfg->b_min, cfg->b_max, Qb, C_k,
                               F(L.z), F(L.m), F(L.Y), B, beta, C_v, stt, st);
   if (nlf < 0) return ARCKV_ERR_CUDA;

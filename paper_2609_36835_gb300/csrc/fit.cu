@@ -876,11 +876,22 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
                 float b_max, const bf16* Q, const float* C_k, const float* z, const float* m,
                 const float* Y, const FitBufs& B, float* beta, float* C_v, DevStatus* stt, cudaStream_t st) {
   int nl = 0;
-  const long long nd = (long long)D.n * D.d, nt = (long long)D.n * D.t;
-  // logits of the compact keys: scale Q C_k^T
-  launch_gemm(RowK<bf16>{Q, nd, D.d}, RowK<float>{C_k, (long long)D.t * D.d, D.d},
-              EpiStore{B.LC, nt, 0, D.t, scale, false}, D.H, D.n, D.t, D.d, 1, st);
-  ++nl;
+  const long long nt = (long long)D.n * D.t;
+  // logits of the compact keys LC = scale Q C_k^T [n][t]: C_k enters as a bf16
+  // triple, LC^T = C_k Q^T runs on the tensor cores and is stored transposed
+  {
+    const long long htd = (long long)D.H * D.t * D.d;
+    bf16 *ck_h = B.ck3, *ck_m = B.ck3 + htd, *ck_l = B.ck3 + 2 * htd;
+    nl += launch_split3(C_k, ck_h, ck_m, ck_l, htd, st);
+    CUtensorMap mA, mA2, mA3, mB;
+    if (!encode_bf16_map_3d(&mA, ck_h, D.d, D.t, D.H, 128) || !encode_bf16_map_3d(&mA2, ck_m, D.d, D.t, D.H, 128) ||
+        !encode_bf16_map_3d(&mA3, ck_l, D.d, D.t, D.H, 128) || !encode_bf16_map_3d(&mB, Q, D.d, D.n, D.H, 128))
+      return -1;
+    if (launch_tc_gemm<128, kSplit3A>(mA, mB, mA2, mA, TcEpiStoreT{B.LC, nt, D.t, scale}, D.H, D.t, D.n, D.d, D.d,
+                                      stt, st, 0, &mA3) != cudaSuccess)
+      return -1;
+    ++nl;
+  }
   const long long cnt = (long long)D.H * nt;
   phi_kernel<<<min(cdiv(cnt, 256), 152 * 16), 256, 0, st>>>(B.LC, z, B.Phi, D.n, D.t, cnt);
   ++nl;

@@ -7,8 +7,8 @@
 // (Eq. indexer_projection); I_ij = sum_a w_ia LeakyReLU_0.1(q_bar_ia.k_bar_ja / sqrt(d_I))
 // (Eq. pairwise_index_score, in tc_index.cu); pi = row softmax of I and
 // s_j = (mean_i pi_ij^2)^(1/2) (Eq. indexer_pooling).
-#include "gemm.cuh"
 #include "kernels.h"
+#include "tc_gemm.cuh"
 
 namespace arckv {
 
@@ -40,32 +40,59 @@ __global__ void __launch_bounds__(512) index_weights_kernel(const bf16* X, const
   if (lane == 0) wts[((long long)b * n_pos + r) * H_I + a] = acc + to_f32(b_x[b * H_I + a]);
 }
 
+// out = A W^T for the n reference rows of every head, W [H][128][128] bf16
+// (K-major), A either an exact bf16 input (A_m == nullptr: one MMA per
+// product) or a bf16 triple (kSplit3A); the epilogue writes a bf16 triple.
+static int gemm_rows128(const Dims& D, const bf16* A_h, const bf16* A_m, const bf16* A_l, const bf16* W,
+                        const TcEpiSplit3& epi, DevStatus* stt, cudaStream_t st) {
+  CUtensorMap mA, mA2, mA3, mB;
+  if (!encode_bf16_map_3d(&mA, A_h, 128, D.n, D.H, 128) || !encode_bf16_map_3d(&mB, W, 128, 128, D.H, 128)) return -1;
+  if (A_m == nullptr)
+    return launch_tc_gemm<128, kPlain>(mA, mB, mA, mB, epi, D.H, D.n, 128, 128, 128, stt, st) == cudaSuccess ? 1 : -1;
+  if (!encode_bf16_map_3d(&mA2, A_m, 128, D.n, D.H, 128) || !encode_bf16_map_3d(&mA3, A_l, 128, D.n, D.H, 128))
+    return -1;
+  return launch_tc_gemm<128, kSplit3A>(mA, mB, mA2, mA, epi, D.H, D.n, 128, 128, 128, stt, st, 0, &mA3) == cudaSuccess
+             ? 1
+             : -1;
+}
+
 int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf16* K, const bf16* VT,
                           const bf16* U_q, const bf16* U_k, const bf16* U_v, const bf16* L_q, const bf16* L_c,
                           const bf16* L_x, const bf16* b_x, const QueryBufs& B, bf16* qbar_hi, bf16* qbar_lo,
                           float* wts, DevStatus* stt, cudaStream_t st) {
   int nl = 0;
-  const long long nd = (long long)D.n * D.d, nA = (long long)D.n * D.d_A, dd = (long long)D.d_A * D.d;
-  // vq = U_q q;  q'' = U_k^T vq, so that (U_q q_i).(U_k k_j) = q''_i . k_j
-  launch_gemm(RowK<bf16>{Q, nd, D.d}, RowK<bf16>{U_q, dd, D.d}, EpiStore{B.vq, nA, 0, D.d_A, 1.f, false}, D.H, D.n,
-              D.d_A, D.d, 1, st);
-  launch_gemm(RowK<float>{B.vq, nA, D.d_A}, ColK<bf16>{U_k, dd, D.d}, EpiStore{B.qpp, nd, 0, D.d, 1.f, false}, D.H,
-              D.n, D.d, D.d_A, 1, st);
-  nl += 2;
+  const long long hn = (long long)D.H * D.n * 128, nd = (long long)D.n * 128;
+  // vq = U_q q (exact products of bf16 inputs) and q'' = U_k^T vq, so that
+  // (U_q q_i).(U_k k_j) = q''_i . k_j; both leave their GEMM as bf16 triples
+  // (vq for the q'' product, q'' as the A operand of the value logits)
+  Dims Dw = D;
+  Dw.T = 128;
+  nl += launch_transpose_v(Dw, U_k, B.ukt, st);   // U_k^T [H][d][d_A]
+  bf16 *vq_h = B.vq3, *vq_m = B.vq3 + hn, *vq_l = B.vq3 + 2 * hn;
+  int r = gemm_rows128(D, Q, nullptr, nullptr, U_q, TcEpiSplit3{vq_h, vq_m, vq_l, nd, 128}, stt, st);
+  if (r < 0) return -1;
+  nl += r;
+  r = gemm_rows128(D, vq_h, vq_m, vq_l, B.ukt, TcEpiSplit3{B.q_h, B.q_m, B.q_l, nd, 128}, stt, st);
+  if (r < 0) return -1;
+  nl += r;
   // value-attention logits on the tensor cores, unscaled as printed in Eq. value_context
-  int r = launch_value_logits_tc(D, B.qpp, B.q_h, B.q_m, B.q_l, K, B.logits, B.part, stt, st);
+  r = launch_value_logits_tc(D, B.q_h, B.q_m, B.q_l, K, B.logits, B.part, stt, st);
   if (r < 0) return -1;
   nl += r;
   nl += launch_part_stats(D.H, D.n, cdiv(D.T, 128), B.part, B.rshift, B.rmul, nullptr, st);
-  // A^V V on the tensor cores, then c = (A^V V) U_v^T = A^V (U_v V)
+  // A^V V on the tensor cores, then c = (A^V V) U_v^T = A^V (U_v V), written as
+  // the bf16 triple that the q_bar GEMM reads (columns 128.. of its A operand)
   r = launch_probs_v_tc(D, B.logits, B.rshift, B.rmul, B.p_h, B.p_m, B.p_l, VT, B.av, stt, st);
   if (r < 0) return -1;
   nl += r;
-  launch_gemm(RowK<float>{B.av, nd, D.d}, RowK<bf16>{U_v, dd, D.d}, EpiStore{B.cctx, nA, 0, D.d_A, 1.f, false},
-              D.H, D.n, D.d_A, D.d, 1, st);
-  ++nl;
+  bf16 *av_h = B.av3, *av_m = B.av3 + hn, *av_l = B.av3 + 2 * hn;
+  nl += launch_split3(B.av, av_h, av_m, av_l, hn, st);
+  r = gemm_rows128(D, av_h, av_m, av_l, U_v, TcEpiSplit3{B.qcat + 128, B.qcat + 256, B.qcat + 384, nd * 4, 512}, stt,
+                   st);
+  if (r < 0) return -1;
+  nl += r;
   // q_bar = N(L_q q + L_c c) per block, as a split-bf16 pair
-  r = launch_query_proj_tc(D, Q, B.cctx, L_q, L_c, B.qcat, B.wcat, qbar_hi, qbar_lo, stt, st);
+  r = launch_query_proj_tc(D, Q, L_q, L_c, B.qcat, B.wcat, qbar_hi, qbar_lo, stt, st);
   if (r < 0) return -1;
   nl += r;
   index_weights_kernel<<<dim3(D.n_pos, D.H), 32 * D.H_I, 0, st>>>(X, L_x, b_x, wts, D.d_x, D.H_I, D.n_pos);

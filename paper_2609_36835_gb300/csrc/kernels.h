@@ -40,16 +40,18 @@ constexpr int kCholNB = 64;  // Cholesky block size
 // ---- indexer (Sec. 3.3, App. A.1) --------------------------------------
 // k_bar = N(L_k k + L_v v) per d_I block, as a split-bf16 pair (one tcgen05
 // GEMM over [K | V] against [L_k | L_v]).
-int launch_query_proj_tc(const Dims& D, const bf16* Q, const float* cctx, const bf16* L_q, const bf16* L_c,
-                         bf16* qcat, bf16* wcat, bf16* qbar_hi, bf16* qbar_lo, DevStatus* stt, cudaStream_t st);
+int launch_query_proj_tc(const Dims& D, const bf16* Q, const bf16* L_q, const bf16* L_c, bf16* qcat, bf16* wcat,
+                         bf16* qbar_hi, bf16* qbar_lo, DevStatus* stt, cudaStream_t st);
 int launch_key_features_tc(const Dims& D, const bf16* K, const bf16* V, const bf16* L_k, const bf16* L_v,
                            bf16* kbar_hi, bf16* kbar_lo, DevStatus* stt, cudaStream_t st);
 // Scratch of the query-side features.
 struct QueryBufs {
-  float *vq, *qpp, *logits, *rshift, *rmul, *av, *cctx;
+  float *logits, *rshift, *rmul, *av;
   bf16 *q_h, *q_m, *q_l, *p_h, *p_m, *p_l;
-  float2* part;  // per-(row, 128-column tile) softmax partials of the logits
+  float2* part;        // per-(row, 128-column tile) softmax partials of the logits
   bf16 *qcat, *wcat;   // K-concatenated operands of the q_bar GEMM ([n][512], [HD][512])
+  bf16 *vq3, *av3;     // bf16 triples of U_q q and A^V V (parts [H][n][128], one after another)
+  bf16* ukt;           // U_k^T [H][d][d_A]
 };
 // value context c (Eq. value_context), q_bar (Eq. indexer_projection), w.
 // VT is V transposed ([H][d][ldT] bf16, launch_transpose_v).  -1 on a TMA failure.
@@ -59,7 +61,8 @@ int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf1
                           float* wts, DevStatus* stt, cudaStream_t st);
 // softmax products with fp32-grade split-3 operands (tc_attn.cu)
 int launch_transpose_v(const Dims& D, const bf16* V, bf16* VT, cudaStream_t st);
-int launch_value_logits_tc(const Dims& D, const float* qpp, bf16* q_h, bf16* q_m, bf16* q_l, const bf16* K,
+// value logits [H][n][T] from the q'' triple and the bf16 keys, with row partials
+int launch_value_logits_tc(const Dims& D, const bf16* q_h, const bf16* q_m, const bf16* q_l, const bf16* K,
                            float* logits, float2* part, DevStatus* stt, cudaStream_t st);
 // out [H][n][128] = (exp(X - shift) * mul) V over rows of X [H][n][T].
 int launch_probs_v_tc(const Dims& D, const float* X, const float* shift, const float* mul, bf16* p_h, bf16* p_m,
@@ -110,6 +113,7 @@ struct FitBufs {
   bf16 *PT_hi, *PT_lo, *YT_hi, *YT_lo;  // transposed split-bf16 operands ([t][ldn], [d][ldn])
   double *G64, *L64, *B64, *Z64, *X64;   // fp64 dual-form scratch (t > n only): [n][n], blocks, [n][d] x 3
   bf16* PT_mid;                         // middle part of the transposed triple of Phi_C ([t][ldn])
+  bf16* ck3;                            // bf16 triple of C_k (parts [H][t][128], one after another)
 };
 // Returns launches, or -1 when a TMA descriptor cannot be encoded.
 int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float eps_w, float b_min,

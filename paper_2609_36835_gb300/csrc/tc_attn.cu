@@ -66,10 +66,8 @@ static int gemm_split3a(int H, int rows, int N, int K, int ldk, const bf16* h, c
   return 1;
 }
 
-int launch_value_logits_tc(const Dims& D, const float* qpp, bf16* q_h, bf16* q_m, bf16* q_l, const bf16* K,
+int launch_value_logits_tc(const Dims& D, const bf16* q_h, const bf16* q_m, const bf16* q_l, const bf16* K,
                            float* logits, float2* part, DevStatus* stt, cudaStream_t st) {
-  const long long cnt = (long long)D.H * D.n * 128;
-  split3_kernel<<<min(cdiv(cnt, 256), 152 * 8), 256, 0, st>>>(qpp, q_h, q_m, q_l, cnt);
   CUtensorMap mA, mA2, mA3, mB;
   if (!encode_bf16_map_3d(&mA, q_h, 128, D.n, D.H, 128) || !encode_bf16_map_3d(&mA2, q_m, 128, D.n, D.H, 128) ||
       !encode_bf16_map_3d(&mA3, q_l, 128, D.n, D.H, 128) || !encode_bf16_map_3d(&mB, K, 128, D.T, D.H, 128))
@@ -77,7 +75,7 @@ int launch_value_logits_tc(const Dims& D, const float* qpp, bf16* q_h, bf16* q_m
   if (launch_tc_logits_rowpart<kSplit3A>(mA, mB, mA2, mA, &mA3, logits, 1.f, part, D.H, D.n, D.T, 128, stt, st) !=
       cudaSuccess)
     return -1;
-  return 2;
+  return 1;
 }
 
 int launch_split3(const float* x, bf16* h, bf16* m, bf16* l, long long count, cudaStream_t st) {

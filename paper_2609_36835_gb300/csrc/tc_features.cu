@@ -102,13 +102,12 @@ int launch_key_features_tc(const Dims& D, const bf16* K, const bf16* V, const bf
 // are concatenated along K as
 //   A = [q | c_h | c_m | c_l]  [n][4 * 128],   B = [L_q | L_c | L_c | L_c]  [HD][4 * 128]
 // and one plain GEMM gives L_q q + L_c (c_h + c_m + c_l) with exact bf16 products.
-__global__ void __launch_bounds__(256) qcat_kernel(const bf16* Q, const float* C, bf16* A, int n) {
-  const int b = blockIdx.y, i = blockIdx.x * 2 + (threadIdx.x >> 7), k = threadIdx.x & 127;
+// The c triple is written into A by the GEMM that forms c; qcat_kernel adds q.
+__global__ void __launch_bounds__(256) qcat_kernel(const bf16* Q, bf16* A, int n) {
+  const int b = blockIdx.y, i = blockIdx.x * 16 + (threadIdx.x >> 4), k = (threadIdx.x & 15) * 8;
   if (i >= n) return;
   const long long r = (long long)b * n + i;
-  bf16* a = A + r * 512;
-  a[k] = Q[r * 128 + k];
-  split3_bf16(C[r * 128 + k], a[128 + k], a[256 + k], a[384 + k]);
+  *(uint4*)(A + r * 512 + k) = *(const uint4*)(Q + r * 128 + k);
 }
 __global__ void __launch_bounds__(256) wcat_kernel(const bf16* L_q, const bf16* L_c, bf16* W, long long rows) {
   const long long r = blockIdx.x * 2ll + (threadIdx.x >> 7);
@@ -122,9 +121,9 @@ __global__ void __launch_bounds__(256) wcat_kernel(const bf16* L_q, const bf16* 
   w[384 + k] = c;
 }
 
-int launch_query_proj_tc(const Dims& D, const bf16* Q, const float* cctx, const bf16* L_q, const bf16* L_c,
-                         bf16* qcat, bf16* wcat, bf16* qbar_hi, bf16* qbar_lo, DevStatus* stt, cudaStream_t st) {
-  qcat_kernel<<<dim3(cdiv(D.n, 2), D.H), 256, 0, st>>>(Q, cctx, qcat, D.n);
+int launch_query_proj_tc(const Dims& D, const bf16* Q, const bf16* L_q, const bf16* L_c, bf16* qcat, bf16* wcat,
+                         bf16* qbar_hi, bf16* qbar_lo, DevStatus* stt, cudaStream_t st) {
+  qcat_kernel<<<dim3(cdiv(D.n, 16), D.H), 256, 0, st>>>(Q, qcat, D.n);
   const long long wrows = (long long)D.H * D.HD;
   wcat_kernel<<<(unsigned)cdiv(wrows, 2), 256, 0, st>>>(L_q, L_c, wcat, wrows);
   CUtensorMap mA, mB;

@@ -360,6 +360,71 @@ struct TcEpiStore {
   __device__ __forceinline__ void finish(State&, int, int, int, int, int) const {}
 };
 
+// Transposed fp32 store: C[b][col][row] = alpha * acc (column stride ldc).
+// A warp's 32 rows are 32 consecutive addresses of each output row.
+struct TcEpiStoreT {
+  float* C;
+  long long cbs;
+  int ldc;
+  float alpha;
+  struct State {
+    float* base;
+    int ncols;
+    bool ok;
+  };
+  __device__ __forceinline__ void init(State& s, int b, int row, int n0, int M, int N) const {
+    s.ok = row < M;
+    s.ncols = N - n0;
+    s.base = C + (long long)b * cbs + (long long)n0 * ldc + (s.ok ? row : 0);
+  }
+  __device__ __forceinline__ void consume(State& s, int, int j, float (&v)[32]) const {
+    if (!s.ok) return;
+#pragma unroll
+    for (int q = 0; q < 32; ++q)
+      if (j * 32 + q < s.ncols) s.base[(long long)(j * 32 + q) * ldc] = alpha * v[q];
+  }
+  __device__ __forceinline__ void finish(State&, int, int, int, int, int) const {}
+};
+
+// The fp32 result as a bf16 triple (h, m, l) (split3_bf16): element
+// (b, row, col) of each part at b * bs + row * ldc + col, the operand format
+// of a following kSplit3A product.
+struct TcEpiSplit3 {
+  bf16 *h, *m, *l;
+  long long bs;
+  int ldc;
+  struct State {
+    long long off;
+    int ncols;
+    bool ok;
+  };
+  __device__ __forceinline__ void init(State& s, int b, int row, int n0, int M, int N) const {
+    s.ok = row < M;
+    s.ncols = N - n0;
+    s.off = (long long)b * bs + (long long)(s.ok ? row : 0) * ldc + n0;
+  }
+  __device__ __forceinline__ void consume(State& s, int, int j, float (&v)[32]) const {
+    if (!s.ok) return;
+#pragma unroll
+    for (int q = 0; q < 32; q += 8) {
+      const long long o = s.off + j * 32 + q;
+      if (j * 32 + q + 8 <= s.ncols && (o & 7) == 0) {
+        __align__(16) bf16 hh[8], mm[8], ll[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) split3_bf16(v[q + e], hh[e], mm[e], ll[e]);
+        *(uint4*)(h + o) = *(const uint4*)hh;
+        *(uint4*)(m + o) = *(const uint4*)mm;
+        *(uint4*)(l + o) = *(const uint4*)ll;
+      } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+          if (j * 32 + q + e < s.ncols) split3_bf16(v[q + e], h[o + e], m[o + e], l[o + e]);
+      }
+    }
+  }
+  __device__ __forceinline__ void finish(State&, int, int, int, int, int) const {}
+};
+
 // Staged TMA store of one warp's 32 rows x 32 columns at (x, y, b): the rows
 // go into a 128-byte-swizzled staging buffer (conflict-free 16-byte stores)
 // and one lane issues the tiled bulk store.  NBUF buffers of 4 KB rotate by
