@@ -233,7 +233,7 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
     nl += nlr0;
     if (cfg->selector == ARCKV_SELECTOR_HA) {
       // p = softmax(l): the same pooling as the index scores, on l's row partials
-      nl += launch_index_pool(D, F(L.NT), (const float2*)(w + L.part), cdiv(D.T, 128), F(L.lse), F(L.s), st);
+      nl += launch_index_pool(D, F(L.NT), (const float2*)(w + L.part), cdiv(D.T, kRowPartW), F(L.lse), F(L.s), st);
     } else {
       float* vq = F(L.vq);   // VI scratch: n-sized rows here, O^(-a) in L.qpp
       const size_t hn = (size_t)D.H * D.n;
@@ -290,7 +290,7 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
     if (nla < 0) return ARCKV_ERR_CUDA;
     nl += nla;
   } else {
-    const int nlc = launch_col_profiles(D, F(L.NT), F(L.logphi), nullptr, nullptr, st);   // log phi only
+    const int nlc = launch_col_profiles(D, F(L.NT), F(L.logphi), nullptr, nullptr, stt, st);   // log phi only
     if (nlc < 0) return ARCKV_ERR_CUDA;
     nl += nlc;
     cudaMemcpyAsync(kappa, aux->assign_in, sizeof(int) * (size_t)D.H * D.T, cudaMemcpyDeviceToDevice, st);

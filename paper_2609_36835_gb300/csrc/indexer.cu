@@ -79,7 +79,7 @@ int launch_query_features(const Dims& D, const bf16* Q, const bf16* X, const bf1
   r = launch_value_logits_tc(D, B.q_h, B.q_m, B.q_l, K, B.logits, B.part, stt, st);
   if (r < 0) return -1;
   nl += r;
-  nl += launch_part_stats(D.H, D.n, cdiv(D.T, 128), B.part, B.rshift, B.rmul, nullptr, st);
+  nl += launch_part_stats(D.H, D.n, cdiv(D.T, kRowPartW), B.part, B.rshift, B.rmul, nullptr, st);
   // A^V V on the tensor cores, then c = (A^V V) U_v^T = A^V (U_v V), written as
   // the bf16 triple that the q_bar GEMM reads (columns 128.. of its A operand)
   r = launch_probs_v_tc(D, B.logits, B.rshift, B.rmul, B.p_h, B.p_m, B.p_l, VT, B.av, stt, st);

@@ -77,8 +77,11 @@ int launch_index_logits(const Dims& D, const bf16* qbar_hi, const bf16* qbar_lo,
                         const bf16* kbar_lo, const float* wts, float* I, float2* part, DevStatus* stt,
                         cudaStream_t st);
 // row log-sum-exp and pooled s (Eq. indexer_pooling).
-// Index-logit softmax partials cover kIndexPartW columns each ([H][n][ceil(T / kIndexPartW)]).
+// Softmax partials of the index logits cover kIndexPartW columns each
+// ([H][n][ceil(T / kIndexPartW)]); those of the value and reference logits
+// kRowPartW columns each.
 constexpr int kIndexPartW = 128;
+constexpr int kRowPartW = 64;
 int launch_index_pool(const Dims& D, const float* I, const float2* part, int ntiles, float* lse, float* s,
                       cudaStream_t st);
 
@@ -98,7 +101,8 @@ int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* 
                          DevStatus* stt, cudaStream_t st);
 // Column statistics of the reference logits L: log phi [H][T] (mass weights of
 // the merge) and, when Ut_hi is given, the transposed split-bf16 profiles.
-int launch_col_profiles(const Dims& D, const float* L, float* logphi, bf16* Ut_hi, bf16* Ut_lo, cudaStream_t st);
+int launch_col_profiles(const Dims& D, const float* L, float* logphi, bf16* Ut_hi, bf16* Ut_lo, DevStatus* stt,
+                        cudaStream_t st);
 // Assignment on tcgen05: column statistics and transposed split-bf16 profiles
 // (log phi written on the way), anchor rows, argmax GEMM.
 int launch_assign_tc(const Dims& D, const float* L, float* logphi, const int* anchors, bf16* Ut_hi, bf16* Ut_lo,

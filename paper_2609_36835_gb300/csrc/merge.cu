@@ -19,7 +19,7 @@ int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const 
   // l = scale * Q K^T on the tensor cores, with per-tile row softmax partials
   if (launch_ref_logits_tc(D, scale, Q, K, L, part, stt, st) < 0) return -1;
   // z_i = max_j l_ij (z^fit of Eq. mass_fit), m_i = sum_j e^{l_ij - z_i} = (Phi_K 1)_i
-  launch_part_stats(D.H, D.n, cdiv(D.T, 128), part, z, invm, m, st);
+  launch_part_stats(D.H, D.n, cdiv(D.T, kRowPartW), part, z, invm, m, st);
   // Y = softmax(l) V
   const int r = launch_probs_v_tc(D, L, z, invm, p_h, p_m, p_l, VT, Y, stt, st);
   if (r < 0) return -1;

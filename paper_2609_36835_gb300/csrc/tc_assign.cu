@@ -149,8 +149,154 @@ __global__ void __launch_bounds__(512) col_profiles_kernel(const float* L, float
   }
 }
 
-int launch_col_profiles(const Dims& D, const float* L, float* logphi, bf16* Ut_hi, bf16* Ut_lo, cudaStream_t st) {
+// col_profiles_kernel with the n x W strip of l staged in shared memory by
+// TMA (boxes of 256 rows x W columns, one mbarrier), so l crosses HBM once.
+// Thread t owns column t % W and the rows congruent to t / W modulo 512 / W
+// (the row phases are combined in order): pass 1 takes the column maxima,
+// pass 2 overwrites the strip with e^{l - M_j} while summing s1 and s2, pass
+// 3 scales by invN_j and writes the transposed split profiles.
+template <int W>
+__global__ void __launch_bounds__(512) col_profiles_tma_kernel(const __grid_constant__ CUtensorMap mL, float* logphi,
+                                                               bf16* Ut_hi, bf16* Ut_lo, int n, int T, int ldn,
+                                                               int nbox, DevStatus* stt) {
+  constexpr int PH = 512 / W;   // row phases
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t r0 = tc::smem_u32(smem_raw);
+  float* strip = (float*)(smem_raw + (((r0 + 127u) & ~127u) - r0));   // [nbox * 256][W], 128-byte aligned
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  __shared__ float red[3][PH][W];
+  __shared__ float cstat[2][W];
+  __shared__ float tile[64][W + 1];
+  const int b = blockIdx.y, j0 = blockIdx.x * W, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int c = tid % W, ph = tid / W, j = j0 + c;
+  if (tid == 0) {
+    tc::mbar_init(&bar, 1);
+    abort_flag = 0;
+    tc::mbar_fence_init();
+  }
+  __syncthreads();
+  if (tid == 0) {
+    tc::mbar_arrive_expect_tx(&bar, (uint32_t)(nbox * 256 * W * 4));
+    for (int q = 0; q < nbox; ++q) tc::tma_load_3d(strip + q * 256 * W, &mL, j0, q * 256, b, &bar);
+  }
+  const bool ok = tc::mbar_wait(&bar, 0, &abort_flag, stt);
+  if (!__syncthreads_and(ok)) {   // timed out: let the copies land (bounded) before leaving
+    volatile int never = 0;
+    if (tid == 0) tc::mbar_wait(&bar, 0, &never, stt);
+    __syncthreads();
+    return;
+  }
+  // pass 1: column maxima (four independent chains per thread)
+  float m0 = -INFINITY, m1 = -INFINITY, m2 = -INFINITY, m3 = -INFINITY;
+  if (j < T) {
+    int i = ph;
+    for (; i + 3 * PH < n; i += 4 * PH) {
+      m0 = fmaxf(m0, strip[i * W + c]);
+      m1 = fmaxf(m1, strip[(i + PH) * W + c]);
+      m2 = fmaxf(m2, strip[(i + 2 * PH) * W + c]);
+      m3 = fmaxf(m3, strip[(i + 3 * PH) * W + c]);
+    }
+    for (; i < n; i += PH) m0 = fmaxf(m0, strip[i * W + c]);
+  }
+  red[0][ph][c] = fmaxf(fmaxf(m0, m1), fmaxf(m2, m3));
+  __syncthreads();
+  if (tid < W) {
+    float M = -INFINITY;
+#pragma unroll 8
+    for (int q = 0; q < PH; ++q) M = fmaxf(M, red[0][q][tid]);
+    cstat[0][tid] = M;
+  }
+  __syncthreads();
+  // pass 2: e_ij = e^{l_ij - M_j} replaces l in the strip; s1 = sum e, s2 = sum e^2
+  {
+    const float M = cstat[0][c];
+    float a1 = 0.f, b1 = 0.f, a2 = 0.f, b2 = 0.f;
+    if (j < T && M != -INFINITY) {
+      int i = ph;
+      for (; i + PH < n; i += 2 * PH) {
+        const float e0 = ex2_approx((strip[i * W + c] - M) * kLog2e);
+        const float e1 = ex2_approx((strip[(i + PH) * W + c] - M) * kLog2e);
+        strip[i * W + c] = e0;
+        strip[(i + PH) * W + c] = e1;
+        a1 += e0;
+        b1 += e1;
+        a2 = fmaf(e0, e0, a2);
+        b2 = fmaf(e1, e1, b2);
+      }
+      if (i < n) {
+        const float e0 = ex2_approx((strip[i * W + c] - M) * kLog2e);
+        strip[i * W + c] = e0;
+        a1 += e0;
+        a2 = fmaf(e0, e0, a2);
+      }
+    }
+    red[1][ph][c] = a1 + b1;
+    red[2][ph][c] = a2 + b2;
+  }
+  __syncthreads();
+  if (tid < W) {
+    float S1 = 0.f, S2 = 0.f;
+#pragma unroll 8
+    for (int q = 0; q < PH; ++q) {
+      S1 += red[1][q][tid];
+      S2 += red[2][q][tid];
+    }
+    if (j < T) logphi[(long long)b * T + j] = cstat[0][tid] + logf(S1) - logf((float)n);
+    cstat[1][tid] = j < T ? 1.0f / sqrtf(S2) : 0.f;
+  }
+  __syncthreads();
+  if (Ut_hi == nullptr) return;
+  // pass 3: U_ij = e_ij invN_j, transposed through a padded tile 64 rows at a time
+  constexpr int RPT = (64 + PH - 1) / PH;   // tile rows per thread: rows ph + k PH below 64
+  const float inv = cstat[1][c];
+  for (int i0 = 0; i0 < ldn; i0 += 64) {
+#pragma unroll
+    for (int k = 0; k < RPT; ++k) {
+      const int r = ph + k * PH, i = i0 + r;
+      if (r < 64) tile[r][c] = (i < n) ? strip[i * W + c] * inv : 0.f;
+    }
+    __syncthreads();
+    // warp w writes columns w, w + 16, ...: lane l rows i0 + 2l and i0 + 2l + 1 (ldn even)
+    for (int cc = warp; cc < W; cc += 16) {
+      const int jj = j0 + cc, i = i0 + 2 * lane;
+      if (jj < T && i < ldn) {
+        const float x0 = tile[2 * lane][cc], x1 = tile[2 * lane + 1][cc];
+        const __nv_bfloat162 h = __floats2bfloat162_rn(x0, x1);
+        const float2 hf = __bfloat1622float2(h);
+        const long long o = ((long long)b * T + jj) * ldn + i;
+        *(__nv_bfloat162*)(Ut_hi + o) = h;
+        *(__nv_bfloat162*)(Ut_lo + o) = __floats2bfloat162_rn(x0 - hf.x, x1 - hf.y);
+      }
+    }
+    __syncthreads();
+  }
+}
+
+template <int W>
+static int launch_col_profiles_tma(const Dims& D, const float* L, float* logphi, bf16* Ut_hi, bf16* Ut_lo, int ldn,
+                                   int nbox, DevStatus* stt, cudaStream_t st) {
+  CUtensorMap m;
+  if (!encode_f32_map_3d(&m, L, D.T, D.n, D.H, W, 256)) return -1;
+  const int smem = nbox * 256 * W * 4 + 128;
+  if (cudaFuncSetAttribute(col_profiles_tma_kernel<W>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+      cudaSuccess)
+    return -1;
+  col_profiles_tma_kernel<W><<<dim3(cdiv(D.T, W), D.H), 512, smem, st>>>(m, logphi, Ut_hi, Ut_lo, D.n, D.T, ldn, nbox,
+                                                                        stt);
+  return 1;
+}
+
+int launch_col_profiles(const Dims& D, const float* L, float* logphi, bf16* Ut_hi, bf16* Ut_lo, DevStatus* stt,
+                        cudaStream_t st) {
   const int ldn = (D.n + 7) / 8 * 8;
+  // staged strips of at most 64 KB (three CTAs per SM) when l is TMA-tileable
+  const int nbox = cdiv(D.n, 256);
+  if ((D.T & 3) == 0 && ((uintptr_t)L & 15u) == 0 && nbox <= 16) {
+    if (nbox <= 4) return launch_col_profiles_tma<16>(D, L, logphi, Ut_hi, Ut_lo, ldn, nbox, stt, st);
+    if (nbox <= 8) return launch_col_profiles_tma<8>(D, L, logphi, Ut_hi, Ut_lo, ldn, nbox, stt, st);
+    return launch_col_profiles_tma<4>(D, L, logphi, Ut_hi, Ut_lo, ldn, nbox, stt, st);
+  }
   // each CTA re-reads its n x 32 strip from L2: with n > 1024 a shared-memory
   // reservation keeps at most two CTAs per SM so the live strips fit in L2
   const int smem = D.n > 1024 ? 80 * 1024 : 0;
@@ -193,7 +339,7 @@ __global__ void anchor_self_assign_kernel2(const int* anchors, int* kappa, int T
 int launch_assign_tc(const Dims& D, const float* L, float* logphi, const int* anchors, bf16* Ut_hi, bf16* Ut_lo,
                      bf16* S_hi, bf16* S_lo, unsigned long long* best, int* kappa, DevStatus* stt, cudaStream_t st) {
   const int ldn = (D.n + 7) / 8 * 8;
-  if (launch_col_profiles(D, L, logphi, Ut_hi, Ut_lo, st) < 0) return -1;
+  if (launch_col_profiles(D, L, logphi, Ut_hi, Ut_lo, stt, st) < 0) return -1;
   gather_anchor_rows_kernel<<<dim3(D.t, D.H), 128, 0, st>>>(Ut_hi, Ut_lo, anchors, S_hi, S_lo, D.T, D.t, ldn);
   cudaMemsetAsync(best, 0, sizeof(unsigned long long) * (size_t)D.H * D.T, st);
   CUtensorMap mA, mA2, mB, mB2;

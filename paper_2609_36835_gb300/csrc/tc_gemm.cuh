@@ -452,14 +452,15 @@ __device__ __forceinline__ void staged_store_32x32(const CUtensorMap* map, uint8
   ++*stores;
 }
 
-// fp32 store through shared memory and TMA (staged_store_32x32 per chunk):
-// a chunk's store overlaps the next chunk.  C is [H][M][N] with row stride
-// ldc (a multiple of 4) in `map`.
-struct TcEpiStoreTma {
+// fp32 store through shared memory and TMA (staged_store_32x32 per chunk,
+// NBUF staging buffers per warp).  C is [H][M][N] with row stride ldc (a
+// multiple of 4) in `map`.
+template <int NBUF>
+struct TcEpiStoreTmaT {
   CUtensorMap map;   // box {32, 32, 1}, 128-byte swizzle
   float alpha;
   int M, N;
-  static constexpr int kStageBytes = 2 * 32 * 128;
+  static constexpr int kStageBytes = NBUF * 32 * 128;
   struct State {
     uint8_t* stage;
     int* stores;
@@ -475,19 +476,21 @@ struct TcEpiStoreTma {
     s.stores = stores;
   }
   __device__ __forceinline__ void consume(State& s, int, int j, float (&v)[32]) const {
-    staged_store_32x32(&map, s.stage, s.stores, s.n0 + 32 * j, s.y, s.b, M, N, v, alpha);
+    staged_store_32x32<NBUF>(&map, s.stage, s.stores, s.n0 + 32 * j, s.y, s.b, M, N, v, alpha);
   }
   __device__ __forceinline__ void finish(State&, int, int, int, int, int) const {}
 };
 
 // A store epilogue (TcEpiStore or TcEpiStoreTma) that also writes each row's
-// softmax partials over the tile's columns: part[b][row][n0 / BN] =
-// (max, sum exp(x - max)) of alpha * acc (exp as 2^(x log2 e) on the MUFU unit).
+// softmax partials over each kRowPartW = 64 columns: part[b][row][col / 64] =
+// (max, sum exp(x - max)) of alpha * acc (exp as 2^(x log2 e) on the MUFU
+// unit).  Eight epilogue warps, each draining 64 columns of a 128-wide tile.
 template <class Store>
 struct TcEpiRowPartT {
   Store st;
   float2* part;
-  int ntiles, BNt;
+  int ntiles, BNt;   // ntiles = ceil(N / 64), BNt = 64
+  static constexpr int kEpiWarps = 8;
   static constexpr int kStageBytes = EpiStage<Store>::bytes;
   struct State {
     typename Store::State s;
@@ -529,11 +532,12 @@ struct TcEpiRowPartT {
     s.mx = mn;
   }
   __device__ __forceinline__ void finish(State& s, int, int, int, int, int) const {
-    if (s.row_ok) part[s.prow] = make_float2(s.mx, s.sm);
+    // a half tile that starts past the last column has no partial slot
+    if (s.row_ok && s.ncols > 0) part[s.prow] = make_float2(s.mx, s.sm);
   }
 };
 using TcEpiStoreRowPart = TcEpiRowPartT<TcEpiStore>;
-using TcEpiStoreRowPartTma = TcEpiRowPartT<TcEpiStoreTma>;
+using TcEpiStoreRowPartTma = TcEpiRowPartT<TcEpiStoreTmaT<1>>;
 
 // Row-partial logits L = alpha * (A B^T) [H][M][N] (row stride N) through the
 // TMA-store epilogue when N is a multiple of 4 (row pitch on the 16-byte grid),
@@ -543,7 +547,7 @@ inline cudaError_t launch_tc_logits_rowpart(const CUtensorMap& mA, const CUtenso
                                             const CUtensorMap& mB2, const CUtensorMap* mA3, float* L, float alpha,
                                             float2* part, int H, int M, int N, int K, DevStatus* stt,
                                             cudaStream_t st) {
-  const int ntiles = cdiv(N, 128);
+  const int ntiles = cdiv(N, 64);
   if ((N & 3) == 0 && (((uintptr_t)L) & 15u) == 0) {
     TcEpiStoreRowPartTma epi{};
     epi.st.alpha = alpha;
@@ -551,12 +555,12 @@ inline cudaError_t launch_tc_logits_rowpart(const CUtensorMap& mA, const CUtenso
     epi.st.N = N;
     epi.part = part;
     epi.ntiles = ntiles;
-    epi.BNt = 128;
+    epi.BNt = 64;
     if (!encode_f32_map_3d(&epi.st.map, L, N, M, H, 32, 32, N, (uint64_t)M * N, true))
       return cudaErrorInvalidValue;
     return launch_tc_gemm<128, MODE>(mA, mB, mA2, mB2, epi, H, M, N, K, K, stt, st, 0, mA3);
   }
-  TcEpiStoreRowPart epi{{L, (long long)M * N, N, alpha}, part, ntiles, 128};
+  TcEpiStoreRowPart epi{{L, (long long)M * N, N, alpha}, part, ntiles, 64};
   return launch_tc_gemm<128, MODE>(mA, mB, mA2, mB2, epi, H, M, N, K, K, stt, st, 0, mA3);
 }
 

@@ -131,6 +131,12 @@ def test_many_row_tiles_single_k_split():
     check_layer(synth.WORKLOADS["llama8b_layer_T8192"], list(range(8)), [3], T=2048, n_pos=300, t=205)
 
 
+def test_many_reference_rows():
+    """n = 2400 reference rows (n_pos = 600, GQA 4) against a short cache: the
+    column statistics stage the longest row strips it supports."""
+    check_layer(synth.WORKLOADS["llama8b_layer_T8192"], [4], [0], T=1024, n_pos=600, t=100)
+
+
 def test_full_context_layer_retention_2pct():
     w = synth.WORKLOADS["llama8b_T8192_r02"]
     check_layer(w, list(range(8)), [5], layer=17)
