@@ -421,6 +421,12 @@ def run_gpu(args, dist: Dist):
                                "launch_ms_isolated: the same launch with the GPU to itself (median of 5)",
                 "peak_note": "bf16 dense, sustained, of %s (MEASURED_PEAKS.json); achieved counts useful flops, "
                              "issued counts the 3 bf16 MMAs of each split-bf16 product" % peak_src}
+    if args.selector != "indexer":
+        # the index-logit GEMM is not launched by the HA / VI selectors
+        roofline = {"kernel": roofline["kernel"], "bound": "tensor", "achieved": None, "peak": peak,
+                    "unit": "TFLOP/s", "frac": None, "traffic": None,
+                    "note": "not launched under --selector %s; the roofline line belongs to the indexer "
+                            "selector (the default)" % args.selector}
 
     # end to end: pinned host inputs -> device -> compaction -> host outputs, every step
     pinned = [workload.to_device(a, pin=True) for a in host]
