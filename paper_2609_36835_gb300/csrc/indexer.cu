@@ -151,10 +151,66 @@ __global__ void __launch_bounds__(256) pool_kernel(const float* I, const float* 
   }
 }
 
+// pool_kernel on 128 columns per CTA for T % 4 == 0: lane l owns columns
+// 4l..4l+3 (16-byte loads), warp w the rows w, w+8, ... with four rows in
+// flight, and pi^2 = e^{2 (I - lse)} = 2^(2 log2 e (I - lse)) is one MUFU op.
+__global__ void __launch_bounds__(256) pool4_kernel(const float* I, const float* lse, float* s, int n, int T) {
+  const int b = blockIdx.y, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int j = blockIdx.x * 128 + lane * 4;
+  __shared__ float4 red[8][32];
+  const float* Ib = I + (long long)b * n * T + j;
+  const float* lb = lse + (long long)b * n;
+  const float k2 = 2.0f * kLog2e;
+  float4 a = make_float4(0.f, 0.f, 0.f, 0.f), c = a;
+  if (j < T) {   // T % 4 == 0: all four columns are inside
+    int i = warp;
+    for (; i + 24 < n; i += 32) {
+      const float4 x0 = *(const float4*)(Ib + (long long)i * T), x1 = *(const float4*)(Ib + (long long)(i + 8) * T);
+      const float4 x2 = *(const float4*)(Ib + (long long)(i + 16) * T);
+      const float4 x3 = *(const float4*)(Ib + (long long)(i + 24) * T);
+      const float l0 = lb[i], l1 = lb[i + 8], l2 = lb[i + 16], l3 = lb[i + 24];
+      a.x += ex2_approx((x0.x - l0) * k2) + ex2_approx((x2.x - l2) * k2);
+      a.y += ex2_approx((x0.y - l0) * k2) + ex2_approx((x2.y - l2) * k2);
+      a.z += ex2_approx((x0.z - l0) * k2) + ex2_approx((x2.z - l2) * k2);
+      a.w += ex2_approx((x0.w - l0) * k2) + ex2_approx((x2.w - l2) * k2);
+      c.x += ex2_approx((x1.x - l1) * k2) + ex2_approx((x3.x - l3) * k2);
+      c.y += ex2_approx((x1.y - l1) * k2) + ex2_approx((x3.y - l3) * k2);
+      c.z += ex2_approx((x1.z - l1) * k2) + ex2_approx((x3.z - l3) * k2);
+      c.w += ex2_approx((x1.w - l1) * k2) + ex2_approx((x3.w - l3) * k2);
+    }
+    for (; i < n; i += 8) {
+      const float4 x0 = *(const float4*)(Ib + (long long)i * T);
+      const float l0 = lb[i];
+      a.x += ex2_approx((x0.x - l0) * k2);
+      a.y += ex2_approx((x0.y - l0) * k2);
+      a.z += ex2_approx((x0.z - l0) * k2);
+      a.w += ex2_approx((x0.w - l0) * k2);
+    }
+  }
+  red[warp][lane] = make_float4(a.x + c.x, a.y + c.y, a.z + c.z, a.w + c.w);
+  __syncthreads();
+  if (warp == 0 && j < T) {
+    float4 t4 = red[0][lane];
+    for (int w = 1; w < 8; ++w) {
+      const float4 u = red[w][lane];
+      t4.x += u.x;
+      t4.y += u.y;
+      t4.z += u.z;
+      t4.w += u.w;
+    }
+    const float inv = 1.0f / (float)n;
+    *(float4*)(s + (long long)b * T + j) =
+        make_float4(sqrtf(t4.x * inv), sqrtf(t4.y * inv), sqrtf(t4.z * inv), sqrtf(t4.w * inv));
+  }
+}
+
 int launch_index_pool(const Dims& D, const float* I, const float2* part, int ntiles, float* lse, float* s,
                       cudaStream_t st) {
   lse_reduce_kernel<<<dim3(cdiv(D.n, 8), D.H), 256, 0, st>>>(part, lse, D.n, ntiles);
-  pool_kernel<<<dim3(cdiv(D.T, 32), D.H), 256, 0, st>>>(I, lse, s, D.n, D.T);
+  if ((D.T & 3) == 0 && (((uintptr_t)I | (uintptr_t)s) & 15u) == 0)
+    pool4_kernel<<<dim3(cdiv(D.T, 128), D.H), 256, 0, st>>>(I, lse, s, D.n, D.T);
+  else
+    pool_kernel<<<dim3(cdiv(D.T, 32), D.H), 256, 0, st>>>(I, lse, s, D.n, D.T);
   return 2;
 }
 

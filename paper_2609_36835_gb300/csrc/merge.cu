@@ -128,21 +128,22 @@ __global__ void __launch_bounds__(1024) group_sort_kernel(const int* kappa, int 
   }
 }
 
-// One CTA per group r: mu_r = sum_{G_r} w_j k_j / sum_{G_r} w_j with
-// w_j = e^{log phi_j - max_{G_r} log phi} (Eq. mass_centroid).  Warp w sums the
-// members w, w+8, ... (ascending position order inside G_r) over 4 dims per
-// lane; the eight partial sums are added in warp order, so the result does not
-// depend on scheduling.  c_r = k_{s_r} + lambda_m (mu_r - k_{s_r}), which is
-// (1 - lambda_m) k_{s_r} + lambda_m mu_r of Eq. key_merge.
-__global__ void __launch_bounds__(256) group_merge_kernel(const bf16* K, const int* anchors, const int* perm,
-                                                          const int* goff, const float* logphi, float lambda_m,
-                                                          float* C_k, int T, int t) {
+constexpr int kMergeWarpMax = 128;
+
+// Groups of more than kMergeWarpMax members (this launch skips the others),
+// one CTA per group with the member layout of group_merge_kernel in each of
+// its eight warps (32 members in flight); the warps' partial sums are added in
+// warp order, so the result does not depend on scheduling.
+__global__ void __launch_bounds__(256) group_merge_cta_kernel(const bf16* K, const int* anchors, const int* perm,
+                                                              const int* goff, const float* logphi, float lambda_m,
+                                                              float* C_k, int T, int t) {
   const int b = blockIdx.y, r = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int* pb = perm + (long long)b * T;
   const int* gb = goff + (long long)b * (t + 1);
   const float* lp = logphi + (long long)b * T;
   const bf16* Kb = K + (long long)b * T * 128;
   const int beg = gb[r], end = gb[r + 1];
+  if (end - beg <= kMergeWarpMax) return;
   __shared__ float red[8][129];
   __shared__ float gmax_s[8];
   float gm = -INFINITY;
@@ -152,41 +153,128 @@ __global__ void __launch_bounds__(256) group_merge_kernel(const bf16* K, const i
   __syncthreads();
   gm = gmax_s[0];
   for (int w = 1; w < 8; ++w) gm = fmaxf(gm, gmax_s[w]);
-  float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f, ws = 0.f;
-  for (int q = beg + warp; q < end; q += 8) {
+  const int slot = lane >> 3, d0 = (lane & 7) * 16;
+  float acc[16], ws = 0.f;
+#pragma unroll
+  for (int e = 0; e < 16; ++e) acc[e] = 0.f;
+  for (int q = beg + warp * 4 + slot; q < end; q += 32) {
     const int j = pb[q];
-    const float om = expf(lp[j] - gm);
-    const uint2 raw = *(const uint2*)(Kb + (long long)j * 128 + lane * 4);
-    const bf16* h = (const bf16*)&raw;
-    a0 = fmaf(om, to_f32(h[0]), a0);
-    a1 = fmaf(om, to_f32(h[1]), a1);
-    a2 = fmaf(om, to_f32(h[2]), a2);
-    a3 = fmaf(om, to_f32(h[3]), a3);
+    const float om = ex2_approx((lp[j] - gm) * kLog2e);
+    const uint4* src = (const uint4*)(Kb + (long long)j * 128 + d0);
+    const uint4 u0 = src[0], u1 = src[1];
+    const __nv_bfloat162* h0 = (const __nv_bfloat162*)&u0;
+    const __nv_bfloat162* h1 = (const __nv_bfloat162*)&u1;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float2 f0 = __bfloat1622float2(h0[e]), f1 = __bfloat1622float2(h1[e]);
+      acc[2 * e] = fmaf(om, f0.x, acc[2 * e]);
+      acc[2 * e + 1] = fmaf(om, f0.y, acc[2 * e + 1]);
+      acc[8 + 2 * e] = fmaf(om, f1.x, acc[8 + 2 * e]);
+      acc[8 + 2 * e + 1] = fmaf(om, f1.y, acc[8 + 2 * e + 1]);
+    }
     ws += om;
   }
-  red[warp][lane * 4 + 0] = a0;
-  red[warp][lane * 4 + 1] = a1;
-  red[warp][lane * 4 + 2] = a2;
-  red[warp][lane * 4 + 3] = a3;
-  if (lane == 0) red[warp][128] = ws;
+#pragma unroll
+  for (int o = 8; o < 32; o <<= 1) {
+#pragma unroll
+    for (int e = 0; e < 16; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], o);
+    ws += __shfl_xor_sync(0xffffffffu, ws, o);
+  }
+  if (lane < 8) {
+#pragma unroll
+    for (int e = 0; e < 16; ++e) red[warp][d0 + e] = acc[e];
+    if (lane == 0) red[warp][128] = ws;
+  }
   __syncthreads();
   if (threadIdx.x >= 128) return;
   const int dcol = threadIdx.x;
-  float acc = 0.f, wsum = 0.f;
+  float a = 0.f, wsum = 0.f;
   for (int w = 0; w < 8; ++w) {
-    acc += red[w][dcol];
+    a += red[w][dcol];
     wsum += red[w][128];
   }
   const int s = anchors[(long long)b * t + r];
   const float k = to_f32(Kb[(long long)s * 128 + dcol]);
-  C_k[((long long)b * t + r) * 128 + dcol] = fmaf(lambda_m, acc * (1.0f / wsum) - k, k);
+  C_k[((long long)b * t + r) * 128 + dcol] = fmaf(lambda_m, a * (1.0f / wsum) - k, k);
+}
+
+// Groups of up to kMergeWarpMax members, one warp per group r:
+// mu_r = sum_{G_r} w_j k_j / sum_{G_r} w_j with
+// w_j = e^{log phi_j - max_{G_r} log phi} (Eq. mass_centroid).  The members
+// j = perm[goff[r] .. goff[r+1]) are read four at a time (eight lanes per
+// member, sixteen dimensions per lane, two 16-byte loads); each of the four
+// member slots sums its members in ascending order and the slots are combined
+// by a fixed shuffle tree, so the result does not depend on scheduling.
+// c_r = k_{s_r} + lambda_m (mu_r - k_{s_r}), which is (1 - lambda_m) k_{s_r} +
+// lambda_m mu_r of Eq. key_merge.  Groups hold ~10 members, so one warp per
+// group avoids the block barriers and idle warps of a CTA per group.
+__global__ void __launch_bounds__(256) group_merge_kernel(const bf16* K, const int* anchors, const int* perm,
+                                                          const int* goff, const float* logphi, float lambda_m,
+                                                          float* C_k, int T, int t) {
+  const int b = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * 8 + warp;
+  if (r >= t) return;
+  const int* pb = perm + (long long)b * T;
+  const int* gb = goff + (long long)b * (t + 1);
+  const float* lp = logphi + (long long)b * T;
+  const bf16* Kb = K + (long long)b * T * 128;
+  const int beg = gb[r], end = gb[r + 1];
+  if (end - beg > kMergeWarpMax) return;   // group_merge_cta_kernel
+  float gm = -INFINITY;
+  for (int q = beg + lane; q < end; q += 32) gm = fmaxf(gm, lp[pb[q]]);
+  gm = warp_max(gm);
+  const int slot = lane >> 3, d0 = (lane & 7) * 16;
+  float acc[16], ws = 0.f;
+#pragma unroll
+  for (int e = 0; e < 16; ++e) acc[e] = 0.f;
+  for (int q = beg + slot; q < end; q += 4) {
+    const int j = pb[q];
+    const float om = ex2_approx((lp[j] - gm) * kLog2e);
+    const uint4* src = (const uint4*)(Kb + (long long)j * 128 + d0);
+    const uint4 u0 = src[0], u1 = src[1];
+    const __nv_bfloat162* h0 = (const __nv_bfloat162*)&u0;
+    const __nv_bfloat162* h1 = (const __nv_bfloat162*)&u1;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float2 f0 = __bfloat1622float2(h0[e]), f1 = __bfloat1622float2(h1[e]);
+      acc[2 * e] = fmaf(om, f0.x, acc[2 * e]);
+      acc[2 * e + 1] = fmaf(om, f0.y, acc[2 * e + 1]);
+      acc[8 + 2 * e] = fmaf(om, f1.x, acc[8 + 2 * e]);
+      acc[8 + 2 * e + 1] = fmaf(om, f1.y, acc[8 + 2 * e + 1]);
+    }
+    ws += om;
+  }
+#pragma unroll
+  for (int o = 8; o < 32; o <<= 1) {
+#pragma unroll
+    for (int e = 0; e < 16; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], o);
+    ws += __shfl_xor_sync(0xffffffffu, ws, o);
+  }
+  if (lane < 8) {
+    const int s = anchors[(long long)b * t + r];
+    const float inv = 1.0f / ws;
+    const bf16* ks = Kb + (long long)s * 128 + d0;
+    float* dst = C_k + ((long long)b * t + r) * 128 + d0;
+#pragma unroll
+    for (int e = 0; e < 16; e += 4) {
+      float o4[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float k = to_f32(ks[e + u]);
+        o4[u] = fmaf(lambda_m, acc[e + u] * inv - k, k);
+      }
+      *(float4*)(dst + e) = make_float4(o4[0], o4[1], o4[2], o4[3]);
+    }
+  }
 }
 
 int launch_merge(const Dims& D, float lambda_m, const bf16* K, const int* anchors, const int* kappa,
                  const float* logphi, int* perm, int* goff, int* cursor, float* C_k, cudaStream_t st) {
   group_sort_kernel<<<D.H, 1024, 0, st>>>(kappa, D.T, D.t, perm, goff, cursor);
-  group_merge_kernel<<<dim3(D.t, D.H), 256, 0, st>>>(K, anchors, perm, goff, logphi, lambda_m, C_k, D.T, D.t);
-  return 2;
+  group_merge_kernel<<<dim3(cdiv(D.t, 8), D.H), 256, 0, st>>>(K, anchors, perm, goff, logphi, lambda_m, C_k, D.T,
+                                                              D.t);
+  group_merge_cta_kernel<<<dim3(D.t, D.H), 256, 0, st>>>(K, anchors, perm, goff, logphi, lambda_m, C_k, D.T, D.t);
+  return 3;
 }
 
 }  // namespace arckv
