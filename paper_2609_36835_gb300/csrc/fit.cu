@@ -616,6 +616,47 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     rmw_sub(Zb + (long long)(i0 + ry) * ldb + c0 + cx, ldb, NB - ry, nc - cx, acc);   // block i < k is full
     __syncthreads();
   };
+  if (nrhs == 1 && t <= 2 * kTileF<R>) {
+    // one right-hand side: the block steps are 64-long mat-vecs whose cost is
+    // the barrier between them, so rank 0 runs them alone with CTA barriers
+    // (Z in shared memory) and the other CTAs of the cluster leave
+    if (rank == 0) {
+      R* zs = &S3[0][0];   // Z [t] in S3 and S4 (free now: t <= 2 kTileF)
+      R* vs = &S1[0][0];   // Y_k + Z_k [64]
+      R* xs = &S1[1][0];   // X_k [64]
+      for (int e = tid; e < t; e += kCT) zs[e] = R(0);
+      __syncthreads();
+      for (int k = nblk - 1; k >= 0; --k) {
+        const int k0 = k * NB, kb = min(NB, t - k0);
+        if (tid < NB) vs[tid] = tid < kb ? __ldcg(Bb + (long long)(k0 + tid) * ldb) + zs[k0 + tid] : R(0);
+        __syncthreads();
+        {  // X_k[c] = sum_l Linv_k[l][c] v[l]: eight threads per column, l = part, part + 8, ...
+          const int c = tid >> 3, part = tid & 7;
+          const R* Li = Lb + (long long)k * NB * NB;
+          R a = R(0);
+#pragma unroll
+          for (int l = part; l < NB; l += 8) a = fma_r(__ldcg(Li + l * NB + c), vs[l], a);
+          a += __shfl_xor_sync(0xffffffffu, a, 1);
+          a += __shfl_xor_sync(0xffffffffu, a, 2);
+          a += __shfl_xor_sync(0xffffffffu, a, 4);
+          if (part == 0) {
+            xs[c] = c < kb ? a : R(0);
+            if (c < kb) Xb[(long long)(k0 + c) * ldb] = a;
+          }
+        }
+        __syncthreads();
+        // Z_j -= L_kj^T X_k for the columns before block k (one thread per column)
+        for (int cc = tid; cc < k0; cc += kCT) {
+          R a = R(0);
+          for (int l = 0; l < kb; ++l) a = fma_r(__ldcg(Ab + (long long)(k0 + l) * t + cc), xs[l], a);
+          zs[cc] -= a;
+        }
+        __syncthreads();
+      }
+    }
+    if (tid == 0 && bad) set_status(stt, ARCKV_ERR_NOT_SPD);
+    return;
+  }
   if (rank == (nblk - 1) % kCL) form_x(nblk - 1);
   cluster_sync_all();
   for (int k = nblk - 1; k >= 1; --k) {
