@@ -12,6 +12,7 @@
 // fused into the trailing updates, then blocked back substitution, all in one
 // cluster launch per system (chol_cluster_kernel).
 #include <cooperative_groups.h>
+#include <type_traits>
 
 #include "gemm.cuh"
 #include "kernels.h"
@@ -415,6 +416,25 @@ __device__ __forceinline__ void st_acc(R* P, long long ld, int pn, int qn, const
       if (p < pn && q < qn) P[p * ld + q] = acc[p][q];
 }
 
+// Eight fp32 values of operand row r, K elements 8 ch .. 8 ch + 7, as bf16
+// triples at their 128-byte-swizzled K-major positions (row r at r * 128
+// bytes, 16-byte chunk ch at ch ^ (r % 8)) of the three part tiles.
+__device__ __forceinline__ void put_split3_chunk(uint8_t* h, uint8_t* m, uint8_t* l, int r, int ch,
+                                                 const float (&x)[8]) {
+  __align__(16) bf16 hh[8], mm[8], ll[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) split3_bf16(x[e], hh[e], mm[e], ll[e]);
+  const int off = r * 128 + ((ch ^ (r & 7)) << 4);
+  *(uint4*)(h + off) = *(const uint4*)hh;
+  *(uint4*)(m + off) = *(const uint4*)mm;
+  *(uint4*)(l + off) = *(const uint4*)ll;
+}
+
+// Shared memory of the fp32 solver beyond its four tiles: the bf16 triples of
+// the tensor-core update operands (A: 128 x 64, B: 64 x 64), 1024-byte aligned.
+constexpr int kTcStageA = 128 * 128, kTcStageB = 64 * 128;
+constexpr int kTcStageBytes = 3 * (kTcStageA + kTcStageB) + 1024;
+
 template <typename R, int kCL>
 __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     chol_cluster_kernel(R* A, R* Linv, R* B, R* Z, R* X, int t, int nrhs, int ldb, long long bbs, R ridge, R tdiv,
@@ -429,6 +449,10 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
   __shared__ R red[kCT / 32];
   __shared__ int bad, grab;
   __shared__ int ctr[2];   // rank 0's pair deals the tiles of alternate dynamic phases
+  constexpr bool kTc = std::is_same<R, float>::value;   // tensor-core trailing updates (fp32 systems)
+  __shared__ uint64_t mma_bar;
+  __shared__ uint32_t tmem_slot;
+  __shared__ int tc_abort;
   const int head = blockIdx.x / kCL;
   const int rank = (int)cluster_rank();
   const int tid = threadIdx.x;
@@ -441,6 +465,33 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
   const int ry = tile_ry(), cx = tile_cx();
   R acc[kTP][kTQ];
   int* ctr0 = cg::this_cluster().map_shared_rank(ctr, 0);
+  // tensor-core update state: operand triples, a 64-column TMEM accumulator, its mbarrier
+  uint8_t* stg = nullptr;
+  uint32_t tmem = 0, mma_ph = 0;
+  if constexpr (kTc) {
+    const uint32_t s0 = tc::smem_u32(smraw), e0 = s0 + 4u * kTileF<R> * (uint32_t)sizeof(R);
+    stg = smraw + (((e0 + 1023u) & ~1023u) - s0);
+    if (tid == 0) {
+      tc::mbar_init(&mma_bar, 1);
+      tc_abort = 0;
+      tc::mbar_fence_init();
+    }
+    if (tid < 32) tc::tmem_alloc(&tmem_slot, 64);
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    tmem = tmem_slot;
+  }
+  auto tc_release = [&]() {   // every exit of a CTA that allocated TMEM
+    if constexpr (kTc) {
+      tc::fence_before_sync();
+      __syncthreads();
+      if (tid < 32) {
+        tc::fence_after_sync();
+        tc::tmem_dealloc(tmem, 64);
+      }
+    }
+  };
   int ep = 0;   // dynamic phase number; phase ep draws from ctr0[ep & 1]
   // next tile of the current dynamic phase (block-uniform)
   auto next_tile = [&]() -> int {
@@ -546,6 +597,133 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
   };
 
 
+  // Tensor-core trailing update (fp32 systems).  Row i of step k holds the
+  // syrk tiles A_ij -= L_ik L_jk^T (j = k+1 .. i) and then the rhs tiles
+  // B_i -= L_ik Y_k; all share L_ik, so a unit takes two tiles of one row:
+  //   D [128 x 64] = [X_1; X_2] L_ik^T,  X = L_jk (syrk) or Y_k^T (rhs),
+  // D's rows m < 64 being tile 1 transposed and the rest tile 2.  Operands
+  // enter as bf16 triples (hh, hm, mh, hl, lh, mm per 16-wide K step:
+  // fp32-grade products); one thread issues the 24 MMAs into TMEM and every
+  // warp then subtracts a 32-row x 16-column slice of D from its tile.
+  auto tc_units = [&](int m) {   // units of step k with m trailing blocks
+    int u = 0;
+    for (int ii = 0; ii < m; ++ii) u += (ii + 2 + nct) / 2;
+    return u;
+  };
+  auto tc_update_unit = [&](int k, int m, int x) {
+    const int k0 = k * NB;
+    int ii = 0, rem = x;
+    for (; ii < m; ++ii) {
+      const int u = (ii + 2 + nct) / 2;
+      if (rem < u) break;
+      rem -= u;
+    }
+    const int i0 = (k + 1 + ii) * NB, len = ii + 1 + nct, e0 = 2 * rem;
+    uint8_t *Ah = stg, *Am = stg + kTcStageA, *Al = stg + 2 * kTcStageA;
+    uint8_t *Bh = stg + 3 * kTcStageA, *Bm = Bh + kTcStageB, *Bl = Bh + 2 * kTcStageB;
+    // B operand: L_ik, rows i0 + n (zero past t), K = block k (full)
+    for (int task = tid; task < 64 * 8; task += kCT) {
+      const int n = task >> 3, ch = task & 7;
+      float xv[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e)
+        xv[e] = (i0 + n < t) ? (float)__ldcg(Ab + (long long)(i0 + n) * t + k0 + 8 * ch + e) : 0.f;
+      put_split3_chunk(Bh, Bm, Bl, n, ch, xv);
+    }
+    // A operand: rows 64 h + r from tile e0 + h
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int e = e0 + h;
+      if (e < ii + 1) {   // syrk: L_jk rows j0 + r
+        const int j0 = (k + 1 + e) * NB;
+        for (int task = tid; task < 64 * 8; task += kCT) {
+          const int r = task >> 3, ch = task & 7;
+          float xv[8];
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            xv[q] = (j0 + r < t) ? (float)__ldcg(Ab + (long long)(j0 + r) * t + k0 + 8 * ch + q) : 0.f;
+          put_split3_chunk(Ah, Am, Al, 64 * h + r, ch, xv);
+        }
+      } else if (e < len) {   // rhs: Y_k^T, row r = column c0 + r of Y_k (zero past nrhs)
+        const int c0 = (e - ii - 1) * NB;
+        for (int task = tid; task < 64 * 8; task += kCT) {
+          const int r = task & 63, ch = task >> 6;
+          float xv[8];
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            xv[q] = (c0 + r < nrhs) ? (float)__ldcg(Bb + (long long)(k0 + 8 * ch + q) * ldb + c0 + r) : 0.f;
+          put_split3_chunk(Ah, Am, Al, 64 * h + r, ch, xv);
+        }
+      } else {   // no second tile
+        for (int task = tid; task < 64 * 8; task += kCT) {
+          const float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+          put_split3_chunk(Ah, Am, Al, 64 * h + (task >> 3), task & 7, z);
+        }
+      }
+    }
+    tc::fence_proxy_async_smem();
+    __syncthreads();
+    if (tid == 0) {
+      tc::fence_after_sync();
+      constexpr uint32_t idesc = tc::idesc_bf16_f32(64);
+#pragma unroll
+      for (int ks = 0; ks < 4; ++ks) {
+        const uint32_t o = ks * 32;
+        const uint64_t ah = tc::sdesc_k128(tc::smem_u32(Ah) + o), am = tc::sdesc_k128(tc::smem_u32(Am) + o),
+                       al = tc::sdesc_k128(tc::smem_u32(Al) + o);
+        const uint64_t bh = tc::sdesc_k128(tc::smem_u32(Bh) + o), bm = tc::sdesc_k128(tc::smem_u32(Bm) + o),
+                       bl = tc::sdesc_k128(tc::smem_u32(Bl) + o);
+        tc::mma_f16(tmem, ah, bh, idesc, ks > 0 ? 1u : 0u);
+        tc::mma_f16(tmem, ah, bm, idesc, 1u);
+        tc::mma_f16(tmem, am, bh, idesc, 1u);
+        tc::mma_f16(tmem, ah, bl, idesc, 1u);
+        tc::mma_f16(tmem, al, bh, idesc, 1u);
+        tc::mma_f16(tmem, am, bm, idesc, 1u);
+      }
+      tc::mma_commit(&mma_bar);
+    }
+    volatile int* abp = &tc_abort;
+    const bool ok = tc::mbar_wait(&mma_bar, mma_ph, abp, stt);
+    mma_ph ^= 1u;
+    tc::fence_after_sync();
+    // warp w: TMEM lanes 32 (w % 4) .. (rows of D), columns 16 (w / 4) ..
+    const int warp = tid >> 5, lane = tid & 31, q = warp & 3, g = warp >> 2;
+    float v[16];
+    tc::tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(g * 16), v);
+    const int h = q >> 1, r = (q & 1) * 32 + lane, e = e0 + h;
+    if (ok && e < len) {
+      R* dst;
+      long long ld;
+      bool col_ok;
+      if (e < ii + 1) {   // A_ij[n][r] -= D[64 h + r][n]
+        const int j0 = (k + 1 + e) * NB;
+        dst = Ab + (long long)i0 * t + j0 + r;
+        ld = t;
+        col_ok = j0 + r < t;
+      } else {            // B_i[n][c0 + r] -= D[64 h + r][n]
+        const int c0 = (e - ii - 1) * NB;
+        dst = Bb + (long long)i0 * ldb + c0 + r;
+        ld = ldb;
+        col_ok = c0 + r < nrhs;
+      }
+      if (col_ok) {
+        R old[16];
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+          const int n = 16 * g + c;
+          old[c] = (i0 + n < t) ? __ldcg(dst + (long long)n * ld) : R(0);
+        }
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+          const int n = 16 * g + c;
+          if (i0 + n < t) dst[(long long)n * ld] = old[c] - (R)v[c];
+        }
+      }
+    }
+    tc::fence_before_sync();
+    __syncthreads();
+  };
+
   // step k = -1 only factors the first diagonal block (one call site keeps the
   // register-resident factorisation inlined once)
   for (int k = -1; k < nblk; ++k) {
@@ -579,14 +757,28 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     // updates); every CTA then draws the remaining tiles from the counter
     const int ntri = k >= 0 ? m * (m + 1) / 2 : 0, ntot = k >= 0 ? ntri + m * nct : 0;
     if (rank == 0 && tid == 0) ctr[(ep + 1) & 1] = 0;
-    if (rank == (k + 1) % kCL) {
-      if (k >= 0) update_tiles(k, 0, ntot, ntot, ntri);
-      factor_diag(Ab, Lb, t, k + 1, lam, S1, S2, S3, &bad);
-    }
-    for (;;) {   // tiles are drawn two at a time
-      const int x = 1 + 2 * next_tile();
-      if (x >= ntot) break;
-      update_tiles(k, x, x + 1, ntot, ntri);
+    if constexpr (kTc) {
+      // unit 0 holds the diagonal tile (k+1, k+1): its owner updates and factors it first
+      const int nu = k >= 0 ? tc_units(m) : 0;
+      if (rank == (k + 1) % kCL) {
+        if (k >= 0) tc_update_unit(k, m, 0);
+        factor_diag(Ab, Lb, t, k + 1, lam, S1, S2, S3, &bad);
+      }
+      for (;;) {
+        const int x = 1 + next_tile();
+        if (x >= nu) break;
+        tc_update_unit(k, m, x);
+      }
+    } else {
+      if (rank == (k + 1) % kCL) {
+        if (k >= 0) update_tiles(k, 0, ntot, ntot, ntri);
+        factor_diag(Ab, Lb, t, k + 1, lam, S1, S2, S3, &bad);
+      }
+      for (;;) {   // tiles are drawn two at a time
+        const int x = 1 + 2 * next_tile();
+        if (x >= ntot) break;
+        update_tiles(k, x, x + 1, ntot, ntri);
+      }
     }
     ++ep;
     cluster_sync_all();
@@ -655,6 +847,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
       }
     }
     if (tid == 0 && bad) set_status(stt, ARCKV_ERR_NOT_SPD);
+    tc_release();
     return;
   }
   if (rank == (nblk - 1) % kCL) form_x(nblk - 1);
@@ -675,12 +868,13 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     cluster_sync_all();
   }
   if (tid == 0 && bad) set_status(stt, ARCKV_ERR_NOT_SPD);
+  tc_release();
 }
 
 template <typename R>
 static int cholesky_solve(int H, int t, R* Gram, R* Linv, R* B, R* Z, R* X, int ldb, int nrhs, long long bbs,
                           float ridge, DevStatus* stt, cudaStream_t st, int tdiv = 0) {
-  const int smem = 4 * kTileF<R> * (int)sizeof(R);
+  const int smem = 4 * kTileF<R> * (int)sizeof(R) + (std::is_same<R, float>::value ? kTcStageBytes : 0);
   const R td = (R)(tdiv > 0 ? tdiv : t);
   if (cluster_size(t) == 8) {
     cudaFuncSetAttribute(chol_cluster_kernel<R, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
