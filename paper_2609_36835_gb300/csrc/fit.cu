@@ -33,28 +33,29 @@ __global__ void phi_kernel(const float* LC, const float* z, float* Phi, int n, i
 // rhs[b][r] = sum_i Phi[b][i][r] m[b][i]   (Phi_C^T Phi_K 1).  A CTA owns 32
 // columns; warp w sums the rows i = w, w+8, ... (four partial sums) and the
 // eight warp sums are added in warp order.
-__global__ void __launch_bounds__(256) mass_rhs_kernel(const float* Phi, const float* m, float* rhs, int n, int t) {
+__global__ void __launch_bounds__(1024) mass_rhs_kernel(const float* Phi, const float* m, float* rhs, int n, int t) {
+  // 32 columns per CTA, the rows split over 32 warps (four loads in flight each)
   const int b = blockIdx.y, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int r = blockIdx.x * 32 + lane;
-  __shared__ float red[8][33];
+  __shared__ float red[32][33];
   const float* P = Phi + (long long)b * n * t + r;
   const float* mb = m + (long long)b * n;
   float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
   if (r < t) {
     int i = warp;
-    for (; i + 24 < n; i += 32) {
+    for (; i + 96 < n; i += 128) {
       a0 = fmaf(P[(long long)i * t], mb[i], a0);
-      a1 = fmaf(P[(long long)(i + 8) * t], mb[i + 8], a1);
-      a2 = fmaf(P[(long long)(i + 16) * t], mb[i + 16], a2);
-      a3 = fmaf(P[(long long)(i + 24) * t], mb[i + 24], a3);
+      a1 = fmaf(P[(long long)(i + 32) * t], mb[i + 32], a1);
+      a2 = fmaf(P[(long long)(i + 64) * t], mb[i + 64], a2);
+      a3 = fmaf(P[(long long)(i + 96) * t], mb[i + 96], a3);
     }
-    for (; i < n; i += 8) a0 = fmaf(P[(long long)i * t], mb[i], a0);
+    for (; i < n; i += 32) a0 = fmaf(P[(long long)i * t], mb[i], a0);
   }
   red[warp][lane] = (a0 + a1) + (a2 + a3);
   __syncthreads();
   if (warp == 0 && r < t) {
     float a = 0.f;
-    for (int w = 0; w < 8; ++w) a += red[w][lane];
+    for (int w = 0; w < 32; ++w) a += red[w][lane];
     rhs[(long long)b * t + r] = a;
   }
 }
@@ -605,6 +606,111 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
   // enter as bf16 triples (hh, hm, mh, hl, lh, mm per 16-wide K step:
   // fp32-grade products); one thread issues the 24 MMAs into TMEM and every
   // warp then subtracts a 32-row x 16-column slice of D from its tile.
+  // D [128 x 64] = A B^T from the staged triples (24 MMAs by one thread), then
+  // wait for it; false when the wait gave up
+  auto tc_mma = [&]() -> bool {
+    uint8_t *Ah = stg, *Am = stg + kTcStageA, *Al = stg + 2 * kTcStageA;
+    uint8_t *Bh = stg + 3 * kTcStageA, *Bm = Bh + kTcStageB, *Bl = Bh + 2 * kTcStageB;
+    tc::fence_proxy_async_smem();
+    __syncthreads();
+    if (tid == 0) {
+      tc::fence_after_sync();
+      constexpr uint32_t idesc = tc::idesc_bf16_f32(64);
+#pragma unroll
+      for (int ks = 0; ks < 4; ++ks) {
+        const uint32_t o = ks * 32;
+        const uint64_t ah = tc::sdesc_k128(tc::smem_u32(Ah) + o), am = tc::sdesc_k128(tc::smem_u32(Am) + o),
+                       al = tc::sdesc_k128(tc::smem_u32(Al) + o);
+        const uint64_t bh = tc::sdesc_k128(tc::smem_u32(Bh) + o), bm = tc::sdesc_k128(tc::smem_u32(Bm) + o),
+                       bl = tc::sdesc_k128(tc::smem_u32(Bl) + o);
+        tc::mma_f16(tmem, ah, bh, idesc, ks > 0 ? 1u : 0u);
+        tc::mma_f16(tmem, ah, bm, idesc, 1u);
+        tc::mma_f16(tmem, am, bh, idesc, 1u);
+        tc::mma_f16(tmem, ah, bl, idesc, 1u);
+        tc::mma_f16(tmem, al, bh, idesc, 1u);
+        tc::mma_f16(tmem, am, bm, idesc, 1u);
+      }
+      tc::mma_commit(&mma_bar);
+    }
+    volatile int* abp = &tc_abort;
+    const bool ok = tc::mbar_wait(&mma_bar, mma_ph, abp, stt);
+    mma_ph ^= 1u;
+    tc::fence_after_sync();
+    return ok;
+  };
+  // operand rows r < rows of a triple from a column-major source: element
+  // (r, l) = G[l * ld + r] (+ G2[...] when given) for r < rvalid, l < kvalid,
+  // zero elsewhere; consecutive threads take consecutive r (coalesced)
+  auto stage_cols = [&](uint8_t* h, uint8_t* mm, uint8_t* l, int rows, const R* G, const R* G2, long long ld,
+                        int rvalid, int kvalid) {
+    for (int task = tid; task < rows * 8; task += kCT) {
+      const int r = task % rows, ch = task / rows;
+      float xv[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const int kk = 8 * ch + q;
+        float v = 0.f;
+        if (r < rvalid && kk < kvalid) {
+          v = (float)__ldcg(G + (long long)kk * ld + r);
+          if (G2) v += (float)__ldcg(G2 + (long long)kk * ld + r);
+        }
+        xv[q] = v;
+      }
+      put_split3_chunk(h, mm, l, r, ch, xv);
+    }
+  };
+  // D's slice of this warp: rows (TMEM lanes) 32 (w % 4) + lane, columns 16 (w / 4) ..
+  auto tc_slice = [&](float (&v)[16], int& mrow, int& ncol) {
+    const int warp = tid >> 5, lane = tid & 31, q = warp & 3, g = warp >> 2;
+    tc::tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(g * 16), v);
+    mrow = q * 32 + lane;
+    ncol = g * 16;
+  };
+  // back substitution on the tensor cores (nrhs <= 128): rows m of D are the
+  // right-hand-side columns, its columns n the rows of the block
+  //   Z_i -= L_ki^T X_k:     D = X_k^T L_ki,         Z_i[n][m] -= D[m][n]
+  //   X_k = Linv^T (Y + Z):  D = (Y_k + Z_k)^T Linv,  X_k[n][m] = D[m][n]
+  auto tc_z_unit = [&](int k, int i) {
+    const int k0 = k * NB, kb = min(NB, t - k0), i0 = i * NB;
+    uint8_t* Ah = stg;
+    uint8_t* Bh = stg + 3 * kTcStageA;
+    stage_cols(Ah, Ah + kTcStageA, Ah + 2 * kTcStageA, 128, Xb + (long long)k0 * ldb, nullptr, ldb, nrhs, kb);
+    stage_cols(Bh, Bh + kTcStageB, Bh + 2 * kTcStageB, 64, Ab + (long long)k0 * t + i0, nullptr, t, 64, kb);
+    const bool ok = tc_mma();
+    float v[16];
+    int mrow, ncol;
+    tc_slice(v, mrow, ncol);
+    if (ok && mrow < nrhs) {   // block i < k is full
+      R* dst = Zb + (long long)(i0 + ncol) * ldb + mrow;
+      R old[16];
+#pragma unroll
+      for (int c = 0; c < 16; ++c) old[c] = __ldcg(dst + (long long)c * ldb);
+#pragma unroll
+      for (int c = 0; c < 16; ++c) dst[(long long)c * ldb] = old[c] - (R)v[c];
+    }
+    tc::fence_before_sync();
+    __syncthreads();
+  };
+  auto tc_x_unit = [&](int k) {
+    const int k0 = k * NB, kb = min(NB, t - k0);
+    uint8_t* Ah = stg;
+    uint8_t* Bh = stg + 3 * kTcStageA;
+    stage_cols(Ah, Ah + kTcStageA, Ah + 2 * kTcStageA, 128, Bb + (long long)k0 * ldb, Zb + (long long)k0 * ldb, ldb,
+               nrhs, kb);
+    stage_cols(Bh, Bh + kTcStageB, Bh + 2 * kTcStageB, 64, Lb + (long long)k * NB * NB, nullptr, NB, 64, NB);
+    const bool ok = tc_mma();
+    float v[16];
+    int mrow, ncol;
+    tc_slice(v, mrow, ncol);
+    if (ok && mrow < nrhs) {
+      R* dst = Xb + (long long)(k0 + ncol) * ldb + mrow;
+#pragma unroll
+      for (int c = 0; c < 16; ++c)
+        if (ncol + c < kb) dst[(long long)c * ldb] = (R)v[c];
+    }
+    tc::fence_before_sync();
+    __syncthreads();
+  };
   auto tc_units = [&](int m) {   // units of step k with m trailing blocks
     int u = 0;
     for (int ii = 0; ii < m; ++ii) u += (ii + 2 + nct) / 2;
@@ -849,6 +955,29 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     if (tid == 0 && bad) set_status(stt, ARCKV_ERR_NOT_SPD);
     tc_release();
     return;
+  }
+  if constexpr (kTc) {
+    if (nrhs <= 128) {
+      if (rank == (nblk - 1) % kCL) tc_x_unit(nblk - 1);
+      cluster_sync_all();
+      for (int k = nblk - 1; k >= 1; --k) {
+        if (rank == 0 && tid == 0) ctr[(ep + 1) & 1] = 0;
+        if (rank == (k - 1) % kCL) {   // the owner of block k-1 finishes Z_{k-1} and forms X_{k-1}
+          tc_z_unit(k, k - 1);
+          tc_x_unit(k - 1);
+        }
+        for (;;) {
+          const int i = next_tile();
+          if (i >= k - 1) break;
+          tc_z_unit(k, i);
+        }
+        ++ep;
+        cluster_sync_all();
+      }
+      if (tid == 0 && bad) set_status(stt, ARCKV_ERR_NOT_SPD);
+      tc_release();
+      return;
+    }
   }
   if (rank == (nblk - 1) % kCL) form_x(nblk - 1);
   cluster_sync_all();
@@ -1140,7 +1269,7 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
   transpose_split3_kernel<<<tgrid, 256, 0, st>>>(B.Phi, D.n, D.t, B.PT_hi, B.PT_mid, B.PT_lo, ldn);
   if (gram3_tc(D.H, D.t, ldn, B.PT_hi, B.PT_mid, B.PT_lo, B.Gram, stt, st) < 0) return -1;
   nl += 2;
-  mass_rhs_kernel<<<dim3(cdiv(D.t, 32), D.H), 256, 0, st>>>(B.Phi, m, B.rhs, D.n, D.t);
+  mass_rhs_kernel<<<dim3(cdiv(D.t, 32), D.H), 1024, 0, st>>>(B.Phi, m, B.rhs, D.n, D.t);
   ++nl;
   nl += cholesky_solve(D.H, D.t, B.Gram, B.Linv, B.rhs, B.Z, B.wsol, 1, 1, D.t, ridge_w, stt, st);
   const long long ht = (long long)D.H * D.t;
