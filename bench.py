@@ -567,7 +567,7 @@ def run_decode(args, dist: Dist):
         "config": {"workload": "decode step: 64 sequences x 8 KV heads x 4 query rows, head_dim 128, t = 0.2 T",
                    "l2": "inputs larger than L2 at every context; calls back to back"},
         "contexts": rows,
-        "roofline": {"kernel": "attend_split_kernel (split-key decode attention)", "bound": "hbm",
+        "roofline": {"kernel": "attend_bulk_kernel (split-key decode attention, bulk-copy K/V ring)", "bound": "hbm",
                      "achieved": last["compact_gbs"], "peak": hbm_peak, "unit": "GB/s",
                      "frac": last["compact_frac"], "traffic": None,
                      "peak_note": "HBM copy bandwidth, of %s (MEASURED_PEAKS.json)" % peak_src},
