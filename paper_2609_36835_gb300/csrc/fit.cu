@@ -76,6 +76,10 @@ __global__ void __launch_bounds__(1024) mass_rhs_kernel(const float* Phi, const 
 // Z_i -= L_ki^T X_k (i < k).  lam = ridge * trace(Gram) / tdiv is added to the
 // diagonal as each diagonal block is factored (tdiv = t, or the primal size
 // when the dual system is solved).
+// fp32 systems run the trailing updates and (up to 128 right-hand sides) the
+// back substitution as tcgen05 units of bf16-triple products; with one
+// right-hand side rank 0 does the back substitution alone.  fp64 systems use
+// SIMT tile products throughout.
 // CTAs per cluster (one cluster per head): 4 up to 16 blocks (t <= 1024) --
 // half the SMs of 8 at nearly the same latency, which leaves room for the
 // concurrent layers -- and 8 for longer systems, whose tile work dominates.
