@@ -505,6 +505,23 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     __syncthreads();
     return grab;
   };
+  // the same with the grab issued one draw ahead: next_tile_ahead() returns the
+  // index grabbed by the previous call and already issues the following grab,
+  // whose round trip to rank 0 then overlaps the caller's unit (thread 0 keeps
+  // it in a register); start_ahead() issues the first grab of a phase
+  int ahead = 0;
+  auto start_ahead = [&]() {
+    if (tid == 0) ahead = atomicAdd(ctr0 + (ep & 1), 1);
+  };
+  auto next_tile_ahead = [&]() -> int {
+    __syncthreads();
+    if (tid == 0) {
+      grab = ahead;
+      ahead = atomicAdd(ctr0 + (ep & 1), 1);
+    }
+    __syncthreads();
+    return grab;
+  };
 
   // lam = ridge * trace / t (every CTA forms it; the trace precedes all writes)
   R tr = R(0);
@@ -874,8 +891,9 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
         if (k >= 0) tc_update_unit(k, m, 0);
         factor_diag(Ab, Lb, t, k + 1, lam, S1, S2, S3, &bad);
       }
+      start_ahead();
       for (;;) {
-        const int x = 1 + next_tile();
+        const int x = 1 + next_tile_ahead();
         if (x >= nu) break;
         tc_update_unit(k, m, x);
       }
@@ -970,8 +988,9 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
           tc_z_unit(k, k - 1);
           tc_x_unit(k - 1);
         }
+        start_ahead();
         for (;;) {
-          const int i = next_tile();
+          const int i = next_tile_ahead();
           if (i >= k - 1) break;
           tc_z_unit(k, i);
         }
