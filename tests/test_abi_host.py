@@ -46,7 +46,7 @@ def _cfg(**kw):
 
 def test_workspace_bytes_sizes_and_rejections(lib):
     ws = pk.workspace_bytes(_cfg())
-    # the n x T fp32 spill, its split-3 bf16 probabilities, k_bar and the t x t Gram dominate
+    # the n x T fp32 spill, k_bar, the transposed profiles and the t x t Gram dominate
     assert 0.8e9 < ws < 2.0e9
     assert pk.workspace_bytes(_cfg(t=9000)) == 0           # t > T
     assert pk.workspace_bytes(_cfg(t=0)) == 0
@@ -54,6 +54,17 @@ def test_workspace_bytes_sizes_and_rejections(lib):
     assert pk.workspace_bytes(_cfg(chunk_len=4096)) == ws  # T = 8192 <= 10,000: chunking is bypassed
     assert pk.attend_workspace_bytes(8, 1024, 819) > 0
     assert pk.attend_workspace_bytes(8, 1024, 0) == 0
+
+
+def test_probability_triple_only_when_t_not_tileable(lib):
+    """softmax(X) V runs fused (no probability triple in the workspace) when T
+    is a multiple of 4; one key more and the unfused path's three bf16 n x T
+    arrays are allocated."""
+    cfg = _cfg(T=8192)
+    H, n = cfg.H_kv, cfg.n_pos * cfg.G
+    extra = pk.workspace_bytes(_cfg(T=8193)) - pk.workspace_bytes(cfg)
+    triple = 3 * H * n * 8200 * 2   # three bf16 arrays with rows padded to a multiple of 8
+    assert triple <= extra < triple + 64 * 1024 * 1024
 
 
 @pytest.mark.parametrize("kw,code", [
