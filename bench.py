@@ -434,16 +434,42 @@ def run_gpu(args, dist: Dist):
     h2d = sum(t.numel() * t.element_size() for p in pinned for t in p.values())
     d2h = sum(t.numel() * t.element_size() for o in host_out for t in o.values())
 
+    h2d_stream, d2h_stream = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+
     def e2e_step():
+        # the host-to-device copies run ahead on their own stream (one event per
+        # layer), each layer's compaction waits only for its own inputs, and its
+        # outputs go back on a third stream as soon as it finishes; the step
+        # ends when every stream has drained, so the next step's copies never
+        # overwrite inputs still in use
         fork()
-        for i in range(len(layers)):
-            with torch.cuda.stream(streams[i % n_str]):
+        start = torch.cuda.Event()
+        start.record(stream)
+        h2d_stream.wait_event(start)
+        d2h_stream.wait_event(start)
+        ready = []
+        with torch.cuda.stream(h2d_stream):
+            for i in range(len(layers)):
                 for k, t in pinned[i].items():
                     dev_in[i][k].copy_(t, non_blocking=True)
-                compact(i)
+                e = torch.cuda.Event()
+                e.record(h2d_stream)
+                ready.append(e)
+        for i in range(len(layers)):
+            s_i = streams[i % n_str]
+            s_i.wait_event(ready[i])
+            compact(i)
+            done = torch.cuda.Event()
+            done.record(s_i)
+            d2h_stream.wait_event(done)
+            with torch.cuda.stream(d2h_stream):
                 for k, t in outs[i].items():
                     host_out[i][k].copy_(t, non_blocking=True)
         join()
+        for side in (h2d_stream, d2h_stream):
+            e = torch.cuda.Event()
+            e.record(side)
+            stream.wait_event(e)
 
     e2e_step()
     torch.cuda.synchronize()
