@@ -23,8 +23,8 @@ Readings of points the paper leaves open (each is listed in the design doc):
   used exactly as printed (value head unscaled, index head divided by
   sqrt(d_I)), App. A.1.
 * top-t ties go to the lower position; S is returned in ascending order.
-* assignment ties go to the smallest anchor index r (App. A.8 asks only for
-  a fixed deterministic rule).
+* assignment ties go to the smallest anchor index r (App. A.8 leaves the
+  tie rule open beyond being deterministic).
 * both least-squares fits are solved with a ridge lam = ridge * tr(Gram)/t;
   ridge = 0 is the paper's unregularised solve for beta (Eq. mass_fit).
 * eps_w, b_min, b_max (unstated in Eq. mass_fit) default to e^-20, -20, 20.
