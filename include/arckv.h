@@ -278,6 +278,16 @@ arckv_status arckv_attend_static(int32_t H_kv, int32_t n, int32_t t, int32_t d, 
  * non-blocking call; synchronises `stream`. */
 arckv_status arckv_query_status(void* ws, void* stream);
 
+/* Diagnostic of the bounded device waits (the failure detection every
+ * tensor-core kernel relies on): one CTA waits on an mbarrier that nothing
+ * arrives on, with a wall-clock limit of limit_us microseconds (1 .. 10^6)
+ * instead of the kernels' 2 s.  The wait gives up, records ARCKV_ERR_TIMEOUT
+ * in the status word of `ws` (>= 256 bytes, 256-byte aligned) and the CTA
+ * returns, so the call synchronises `stream` and returns ARCKV_ERR_TIMEOUT
+ * with the CUDA context still usable.  ARCKV_ERR_INVALID_ARG for a limit out
+ * of range, ARCKV_ERR_WORKSPACE for a missing or short workspace. */
+arckv_status arckv_wait_probe(void* ws, size_t ws_bytes, uint32_t limit_us, void* stream);
+
 /* Static description of a status code (never NULL). Host-only. */
 const char* arckv_status_string(arckv_status s);
 

@@ -18,6 +18,7 @@ __all__ = [
     "attend_workspace_bytes", "arckv_compact", "arckv_attend", "arckv_query_status", "status_string",
     "compact_layer", "attend", "INDEXER_FIELDS", "attend_joint", "arckv_attend_joint",
     "attend_joint_workspace_bytes", "FLAG_COMPACT_BF16", "truncated_error", "arckv_truncated_error", "SELECTOR_INDEXER", "SELECTOR_HA", "SELECTOR_VI",
+    "arckv_wait_probe",
 ]
 
 _LIB_PATH = Path(__file__).resolve().parent / "libarckv.so"
@@ -127,6 +128,8 @@ def load_library():
     lib.arckv_truncated_error.restype = ctypes.c_int
     lib.arckv_query_status.argtypes = [P, P]
     lib.arckv_query_status.restype = ctypes.c_int
+    lib.arckv_wait_probe.argtypes = [P, ctypes.c_size_t, ctypes.c_uint32, P]
+    lib.arckv_wait_probe.restype = ctypes.c_int
     lib.arckv_status_string.argtypes = [ctypes.c_int]
     lib.arckv_status_string.restype = ctypes.c_char_p
     _lib = lib
@@ -221,6 +224,12 @@ def arckv_truncated_error(H: int, n: int, T: int, t: int, d: int, logit_scale: f
 
 def arckv_query_status(ws, stream=None) -> int:
     return int(load_library().arckv_query_status(_ptr(ws), _stream_handle(stream)))
+
+
+def arckv_wait_probe(ws, ws_bytes: int, limit_us: int, stream=None) -> int:
+    """Direct binding of ``arckv_wait_probe`` (a bounded device wait made to
+    give up); returns the status code."""
+    return int(load_library().arckv_wait_probe(_ptr(ws), int(ws_bytes), int(limit_us), _stream_handle(stream)))
 
 
 # ----------------------------------------------------------- torch helpers

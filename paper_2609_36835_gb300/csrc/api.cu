@@ -4,6 +4,7 @@
 #include <string.h>
 
 #include "kernels.h"
+#include "tc.cuh"
 
 using namespace arckv;
 
@@ -177,6 +178,35 @@ arckv_status arckv_query_status(void* ws, void* stream) {
   if (s == ARCKV_ERR_CUDA) return s;
   if (cudaMemsetAsync(ws, 0, sizeof(unsigned int), st) != cudaSuccess) return ARCKV_ERR_CUDA;
   return s;
+}
+
+// One CTA waits on an mbarrier that nothing arrives on, through the bounded
+// wait of the tensor-core kernels with a limit of limit_ns: the wait gives up
+// and records ARCKV_ERR_TIMEOUT in the status word, and the CTA returns.
+__global__ void wait_probe_kernel(DevStatus* stt, unsigned long long limit_ns) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    tc::mbar_init(&bar, 1);
+    abort_flag = 0;
+    tc::mbar_fence_init();
+  }
+  __syncthreads();
+  volatile int* ab = &abort_flag;
+  if (threadIdx.x == 0) tc::mbar_wait_for(&bar, 0, ab, stt, limit_ns);
+  __syncthreads();
+}
+
+arckv_status arckv_wait_probe(void* ws, size_t ws_bytes, uint32_t limit_us, void* stream) {
+  if (limit_us == 0 || limit_us > 1000000u) return ARCKV_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < sizeof(DevStatus) || ((uintptr_t)ws % kAlign) != 0) return ARCKV_ERR_WORKSPACE;
+  cudaStream_t st = (cudaStream_t)stream;
+  cudaGetLastError();
+  DevStatus* stt = (DevStatus*)ws;
+  if (cudaMemsetAsync(stt, 0, sizeof(DevStatus), st) != cudaSuccess) return ARCKV_ERR_CUDA;
+  wait_probe_kernel<<<1, 32, 0, st>>>(stt, (unsigned long long)limit_us * 1000ull);
+  if (cudaGetLastError() != cudaSuccess) return ARCKV_ERR_CUDA;
+  return read_status(ws, st);
 }
 
 arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V, const void* Q_ref,

@@ -50,22 +50,27 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Wait for `parity` on `bar`; gives up when *abort is raised or after the
-// wall-clock limit (then raises *abort and records ARCKV_ERR_TIMEOUT).
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort, DevStatus* stt) {
+// Wait for `parity` on `bar`; gives up when *abort is raised or after
+// limit_ns of wall-clock time (then raises *abort and records
+// ARCKV_ERR_TIMEOUT).
+__device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity, volatile int* abort, DevStatus* stt,
+                                              unsigned long long limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = globaltimer();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 63u) == 0) {
       if (*abort) return false;
-      if (globaltimer() - t0 > kWaitLimitNs) {
+      if (globaltimer() - t0 > limit_ns) {
         *abort = 1;
         set_status(stt, ARCKV_ERR_TIMEOUT);
         return false;
       }
     }
   }
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort, DevStatus* stt) {
+  return mbar_wait_for(bar, parity, abort, stt, kWaitLimitNs);
 }
 
 // ------------------------------------------------------------------- TMA

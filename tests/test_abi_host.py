@@ -56,6 +56,12 @@ def test_workspace_bytes_sizes_and_rejections(lib):
     assert pk.attend_workspace_bytes(8, 1024, 0) == 0
 
 
+def test_wait_probe_rejects_bad_arguments_on_the_host(lib):
+    assert pk.arckv_wait_probe(None, 256, 1000, stream=0) == 3     # no workspace
+    assert pk.arckv_wait_probe(None, 256, 0, stream=0) == 1        # limit out of range
+    assert pk.arckv_wait_probe(None, 256, 2000000, stream=0) == 1
+
+
 def test_probability_triple_only_when_t_not_tileable(lib):
     """softmax(X) V runs fused (no probability triple in the workspace) when T
     is a multiple of 4; one key more and the unfused path's three bf16 n x T

@@ -265,6 +265,22 @@ def test_nonblocking_then_query_status():
     assert torch.equal(out["C_v"], ref["C_v"])
 
 
+def test_bounded_wait_gives_up_and_context_stays_usable():
+    """Failure detection without a GPU fault: a bounded device wait on an
+    mbarrier that nothing completes gives up after 20 ms and reports
+    ARCKV_ERR_TIMEOUT through the status word; the next compaction on the same
+    context runs normally."""
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    assert pk.arckv_wait_probe(ws, 256, 20000) == 6
+    assert pk.arckv_query_status(ws) == 6   # still recorded; reading it clears it
+    assert pk.arckv_query_status(ws) == 0
+    w = synth.WORKLOADS["single_head_T1024"]
+    arr = workload.layer_inputs_np(w, 0, [0], T=256, n_pos=16)
+    cfg = workload.layer_config(w, 1, T=256, n_pos=16, t=20)
+    out = _run(cfg, workload.to_device(arr, "cuda"))
+    assert out["status"] == 0 and bool(torch.isfinite(out["C_v"]).all())
+
+
 def test_nonfinite_input_is_reported():
     w = synth.WORKLOADS["single_head_T1024"]
     arr = workload.layer_inputs_np(w, 0, [0], T=256, n_pos=16)
