@@ -84,7 +84,7 @@ WORKLOADS: Dict[str, Workload] = {
     "single_head_T1024": Workload("single_head_T1024", 0, 1, 1, 1024, 64, 102),
     # one Llama-3.1-8B layer
     "llama8b_layer_T8192": Workload("llama8b_layer_T8192", 1, 1, 8, 8192, 256, 819),
-    # the full 32-layer Llama-3.1-8B cache at three retentions
+    # the full 32-layer Llama-3.1-8B cache at three retentions (suffix rNN: t / T = NN %)
     "llama8b_T8192_r10": Workload("llama8b_T8192_r10", 2, 32, 8, 8192, 256, 819),
     "llama8b_T8192_r05": Workload("llama8b_T8192_r05", 2, 32, 8, 8192, 256, 409),
     "llama8b_T8192_r02": Workload("llama8b_T8192_r02", 2, 32, 8, 8192, 256, 163),
