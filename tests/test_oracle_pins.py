@@ -296,6 +296,10 @@ def test_assignment_brute_force_cosine_table_and_ties():
     K2 = K.copy(); K2[9] = K2[5]
     kappa2 = oracle.assign_to_anchors(oracle.response_profiles(oracle.attention_logits(Q, K2, SC))[0], S)
     assert not np.any(kappa2[np.setdiff1d(np.arange(40), S)] == 2)
+    # Eq. anchor_assignment fixes kappa(s_r) = r for every anchor, also for the
+    # anchor whose profile equals an earlier anchor's (the argmax alone would
+    # send it to the earlier one)
+    assert list(kappa2[S]) == list(range(len(S)))
 
 
 def test_mass_centroid_closed_form_one_query():
@@ -402,6 +406,50 @@ def test_fit_beta_projection_and_clip():
     assert np.all(fb["w_star"][neg] == 0.0) and np.all(fb["beta"][neg] == -20.0)
     pos = fb["w_tilde"] > np.exp(-20)
     assert np.allclose(fb["beta"][pos], np.clip(np.log(fb["w_tilde"][pos]), -20, 20), rtol=1e-15)
+
+
+def test_fit_beta_negative_weight_closed_form_projection_and_clip():
+    """Two queries along e_1, e_2 at scale 1; cache keys a = 2 e_1 and
+    c = 3 e_2, compact keys a and b = e_1 + e_2.  Each row's shift z_i scales
+    both sides of Phi_C w = Phi_K 1 alike, so w~ solves
+    [(e^2, 1), (e, e)] w = (e^2 + 1, 1 + e^3) (columns phi_a, phi_b):
+    w~_a = -e^2 / (e + 1) < 0 and w~_b = (1 + e^3 - w~_a) / e.  Eq. mass_fit
+    projects w~_a to 0 (beta_a = log eps_w, then clipped to b_min) and clips
+    beta_b = log w~_b ~ 2.14 to b_max when b_max is below it."""
+    e = np.e
+    Q = np.zeros((2, 128)); Q[0, 0] = 1.0; Q[1, 1] = 1.0
+    a = np.zeros(128); a[0] = 2.0
+    c = np.zeros(128); c[1] = 3.0
+    b = np.zeros(128); b[0] = 1.0; b[1] = 1.0
+    wa = -e * e / (e + 1.0)
+    wb = (1.0 + e ** 3 - wa) / e
+    fb = oracle.fit_beta(Q, np.stack([a, c]), np.stack([a, b]), oracle.OracleConfig(t=2, ridge_w=0.0), 1.0)
+    assert np.allclose(fb["w_tilde"], [wa, wb], rtol=1e-12)
+    assert fb["w_star"][0] == 0.0 and fb["w_star"][1] == pytest.approx(wb, rel=1e-12)
+    assert fb["beta"][0] == pytest.approx(-20.0, abs=1e-12)
+    assert fb["beta"][1] == pytest.approx(np.log(wb), rel=1e-12)
+    cfg = oracle.OracleConfig(t=2, ridge_w=0.0, eps_w=float(np.exp(-20.0)), b_min=-5.0, b_max=1.0)
+    fb = oracle.fit_beta(Q, np.stack([a, c]), np.stack([a, b]), cfg, 1.0)
+    assert list(fb["beta"]) == [-5.0, 1.0]
+
+
+def test_fit_values_duplicate_keys_reproduce_exact_values():
+    """Three copies of key k (values v_1..v_3) and one key k2 (value v_4),
+    anchors k and k2 with beta = (log 3, 0): softmax(q C_k^T + beta) equals the
+    full attention's mass on the two groups, so Y = P^ [mean(v_1..v_3); v_4]
+    holds exactly and the unregularised fit of Eq. value_lstsq returns those
+    rows; the compact attention then reproduces the full output."""
+    rng = np.random.default_rng(21)
+    k = rng.normal(size=128); k2 = rng.normal(size=128)
+    K = np.stack([k, k, k, k2])
+    V = rng.normal(size=(4, 128))
+    Q = rng.normal(size=(7, 128))
+    beta = np.array([np.log(3.0), 0.0])
+    fv = oracle.fit_values(Q, K, V, K[[0, 3]], beta, oracle.OracleConfig(t=2, ridge_v=0.0), SC)
+    want = np.stack([V[:3].mean(axis=0), V[3]])
+    assert np.allclose(fv["C_v"], want, rtol=1e-9, atol=1e-11)
+    _, O = oracle.full_attention(Q, K, V, SC)
+    assert np.allclose(oracle.compact_attention(Q, K[[0, 3]], beta, fv["C_v"], SC), O, rtol=1e-9, atol=1e-11)
 
 
 def test_fit_values_single_anchor_closed_form():
@@ -565,3 +613,60 @@ def test_pipeline_anchors_in_matches_scored_pipeline():
     b = oracle.compact_pair(K, V, Q, Xr, W, cfg, anchors_in=a["anchors"])
     for k in ("C_k", "beta", "C_v", "assign"):
         assert np.array_equal(a[k], b[k])
+
+
+def test_pipeline_tiny_brute_force_loops():
+    """Sec. 3.2 stages after selection on a tiny pair, each written here as
+    explicit loops over the definitions: logits, response profiles with the
+    single global shift (Eq. response_profile), the cosine argmax with
+    kappa(s_r) = r (Eq. anchor_assignment), mass weights and the convex merge
+    (Eqs. mass_centroid, key_merge), then both fits by Householder QR of the
+    stacked ridge systems (Eqs. mass_fit, value_lstsq).  Plain Gaussian
+    inputs keep the logits of order one, so the single global shift of the
+    printed profile stays inside fp64's range."""
+    rng = np.random.default_rng(5)
+    K, V, Q = rng.normal(size=(12, 128)), rng.normal(size=(12, 128)), rng.normal(size=(12, 128))
+    S = np.array([1, 6, 10])
+    sc = SC
+    cfg = oracle.OracleConfig(t=3, lambda_m=0.4, ridge_w=1e-3, ridge_v=1e-2, scale=sc)
+    out = oracle.compact_pair(K, V, Q, None, None, cfg, anchors_in=S)
+    n, T, t, d = Q.shape[0], K.shape[0], 3, K.shape[1]
+    l = np.array([[sc * sum(Q[i, c] * K[j, c] for c in range(d)) for j in range(T)] for i in range(n)])
+    zm = max(max(row) for row in l)
+    u = np.zeros((n, T))
+    for j in range(T):
+        col = [np.exp(l[i, j] - zm) for i in range(n)]
+        nrm = np.sqrt(sum(x * x for x in col))
+        for i in range(n):
+            u[i, j] = col[i] / nrm
+    kappa = []
+    for j in range(T):
+        if j in S:
+            kappa.append(list(S).index(j))
+            continue
+        sims = [sum(u[i, j] * u[i, s] for i in range(n)) for s in S]
+        kappa.append(int(np.argmax(sims)))
+    assert list(out["assign"]) == kappa
+    phi = [sum(np.exp(l[i, j] - zm) for i in range(n)) / n for j in range(T)]
+    Ck = np.zeros((t, d))
+    for r in range(t):
+        grp = [j for j in range(T) if kappa[j] == r]
+        mu = sum(phi[j] * K[j] for j in grp) / sum(phi[j] for j in grp)
+        Ck[r] = (1 - cfg.lambda_m) * K[S[r]] + cfg.lambda_m * mu
+    assert np.allclose(out["C_k"], Ck, rtol=1e-12, atol=1e-13)
+    lc = np.array([[sc * sum(Q[i, c] * Ck[r, c] for c in range(d)) for r in range(t)] for i in range(n)])
+    z = [max(l[i]) for i in range(n)]
+    PhiC = np.array([[np.exp(lc[i, r] - z[i]) for r in range(t)] for i in range(n)])
+    mass = np.array([sum(np.exp(l[i, j] - z[i]) for j in range(T)) for i in range(n)])
+    wt = _stacked_qr_solve(PhiC, mass, cfg.ridge_w * np.trace(PhiC.T @ PhiC) / t)
+    beta = np.clip(np.log(np.maximum(np.maximum(wt, 0.0), cfg.eps_w)), cfg.b_min, cfg.b_max)
+    assert np.allclose(out["beta"], beta, rtol=1e-9, atol=1e-11)
+    Ph = np.zeros((n, t))
+    Y = np.zeros((n, d))
+    for i in range(n):
+        a = [np.exp(lc[i, r] + beta[r]) for r in range(t)]
+        Ph[i] = np.array(a) / sum(a)
+        p = [np.exp(l[i, j] - z[i]) for j in range(T)]
+        Y[i] = sum(p[j] * V[j] for j in range(T)) / sum(p)
+    Cv = _stacked_qr_solve(Ph, Y, cfg.ridge_v * np.trace(Ph.T @ Ph) / t)
+    assert np.allclose(out["C_v"], Cv, rtol=1e-9, atol=1e-11)
