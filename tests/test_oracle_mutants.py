@@ -6,7 +6,9 @@ wrong tie rule).  The test plants it in a copy of the oracle's source text,
 loads that copy as a module of its own, points the pin suite
 (``tests/test_oracle_pins.py``) at it and runs the pins until one fails.  A
 case that no pin catches means the pins leave that part of the oracle
-unchecked.  Everything runs on the CPU; the oracle on disk is not touched.
+unchecked.  The comparison helpers of ``oracle/parity.py`` get the same
+treatment against ``tests/test_parity_helpers.py``.  Everything runs on the
+CPU; the files on disk are not touched.
 """
 import importlib.util
 import sys
@@ -18,6 +20,8 @@ import pytest
 ROOT = Path(__file__).resolve().parent.parent
 ORACLE_SRC = ROOT / "oracle" / "arckv_oracle.py"
 PINS_SRC = Path(__file__).resolve().parent / "test_oracle_pins.py"
+PARITY_SRC = ROOT / "oracle" / "parity.py"
+PARITY_PINS_SRC = Path(__file__).resolve().parent / "test_parity_helpers.py"
 
 # (name, exact fragment of the oracle's source, replacement)
 MUTANTS = [
@@ -93,6 +97,35 @@ MUTANTS = [
 ]
 
 
+# slips in the comparison helpers the GPU parity tests rely on
+PARITY_MUTANTS = [
+    ("rel_fro_absolute", "return float(np.linalg.norm(a - b) / (nb if nb > 0 else 1.0))",
+     "return float(np.linalg.norm(a - b))"),
+    ("score_errors_top_t_only", "[: min(len(s), 2 * t)]", "[: min(len(s), t)]"),
+    ("anchors_threshold_off_by_one", "k_thr = int(order[t - 1])", "k_thr = int(order[t])"),
+    ("anchors_errors_narrow_the_band", "excess = [abs(s[j] - thr) / thr - err(j) - err(k_thr) for j in diff]",
+     "excess = [abs(s[j] - thr) / thr + err(j) + err(k_thr) for j in diff]"),
+    ("anchors_errors_ignored", "return 0.0 if s_gpu is None else abs(float(s_gpu[j]) - s[j]) / abs(s[j])",
+     "return 0.0"),
+    ("anchors_no_size_check", "if len(a) != len(b) or len(S_gpu) != t:", "if False:"),
+    ("chunked_scores_not_sliced", "s[start:start + Tc], tc, band, sg)", "s, tc, band, sg)"),
+    ("chunked_positions_not_offset", "return X[(X >= start) & (X < start + Tc)] - start",
+     "return X[(X >= start) & (X < start + Tc)]"),
+    ("assignment_decided_rows_inverted", "    dec = (~is_anchor) & (gap > tau)\n    kappa_ref",
+     "    dec = (~is_anchor) & (gap < tau)\n    kappa_ref"),
+    ("assignment_anchor_rows_unchecked", "return (n_dec_mis == 0 and anchors_ok and worst <= tau)",
+     "return (n_dec_mis == 0 and worst <= tau)"),
+    ("assignment_shortfall_unchecked", "return (n_dec_mis == 0 and anchors_ok and worst <= tau)",
+     "return (n_dec_mis == 0 and anchors_ok)"),
+    ("profiles_form_wrong_block", "kg = kappa_gpu[j0:j0 + rows]", "kg = kappa_gpu[:rows][: sim.shape[0]]"),
+    ("beta_support_everything", "sup = w_star > 1e-6 * wmax", "sup = w_star >= 0.0"),
+    ("beta_rest_unchecked", "rest_ok = bool(np.all(beta_gpu[~sup] <= np.log(max(1e-5 * wmax, 1e-300)) + 1e-6))",
+     "rest_ok = True"),
+    ("mass_weights_in_log_space", "return rel_fro(np.exp(np.asarray(beta_gpu, dtype=np.float64)), "
+     "np.exp(np.asarray(beta, dtype=np.float64)))", "return rel_fro(np.asarray(beta_gpu), np.asarray(beta))"),
+]
+
+
 def _load(name: str, source: str, path: Path) -> types.ModuleType:
     mod = types.ModuleType(name)
     mod.__file__ = str(path)
@@ -105,13 +138,13 @@ def _load(name: str, source: str, path: Path) -> types.ModuleType:
     return mod
 
 
-def _run_pins(oracle_mod: types.ModuleType, stop_at_first: bool):
-    """Run every pin with ``oracle`` bound to ``oracle_mod``.  Returns the
-    names of the pins that raised."""
-    spec = importlib.util.spec_from_file_location("_pins_under_mutation", PINS_SRC)
+def _run_pins(mod: types.ModuleType, stop_at_first: bool, pins_src: Path = PINS_SRC, attr: str = "oracle"):
+    """Run every test of ``pins_src`` with its global ``attr`` bound to
+    ``mod``.  Returns the names of the tests that raised."""
+    spec = importlib.util.spec_from_file_location("_pins_under_mutation", pins_src)
     pins = importlib.util.module_from_spec(spec)
     spec.loader.exec_module(pins)
-    pins.oracle = oracle_mod
+    setattr(pins, attr, mod)
     failed = []
     for name in sorted(n for n in vars(pins) if n.startswith("test_")):
         try:
@@ -123,18 +156,20 @@ def _run_pins(oracle_mod: types.ModuleType, stop_at_first: bool):
     return failed
 
 
-def _mutant_source(old: str, new: str) -> str:
-    src = ORACLE_SRC.read_text()
+def _mutant_source(old: str, new: str, src_path: Path = ORACLE_SRC) -> str:
+    src = src_path.read_text()
     assert src.count(old) == 1, f"fragment occurs {src.count(old)} times: {old!r}"
     return src.replace(old, new)
 
 
-def test_unmodified_copy_passes_every_pin():
-    mod = _load("_oracle_copy", ORACLE_SRC.read_text(), ORACLE_SRC)
+@pytest.mark.parametrize("src,pins,attr", [(ORACLE_SRC, PINS_SRC, "oracle"), (PARITY_SRC, PARITY_PINS_SRC, "parity")],
+                         ids=["oracle", "parity"])
+def test_unmodified_copy_passes_every_pin(src, pins, attr):
+    mod = _load("_copy_" + attr, src.read_text(), src)
     try:
-        assert _run_pins(mod, stop_at_first=False) == []
+        assert _run_pins(mod, False, pins, attr) == []
     finally:
-        del sys.modules["_oracle_copy"]
+        del sys.modules["_copy_" + attr]
 
 
 @pytest.mark.parametrize("name,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
@@ -143,5 +178,15 @@ def test_planted_mistake_fails_a_pin(name, old, new):
     mod = _load(mod_name, _mutant_source(old, new), ORACLE_SRC)
     try:
         assert _run_pins(mod, stop_at_first=True), f"no pin catches {name}"
+    finally:
+        del sys.modules[mod_name]
+
+
+@pytest.mark.parametrize("name,old,new", PARITY_MUTANTS, ids=[m[0] for m in PARITY_MUTANTS])
+def test_planted_mistake_in_parity_helpers_fails_a_check(name, old, new):
+    mod_name = "_parity_mutant_" + name
+    mod = _load(mod_name, _mutant_source(old, new, PARITY_SRC), PARITY_SRC)
+    try:
+        assert _run_pins(mod, True, PARITY_PINS_SRC, "parity"), f"no check catches {name}"
     finally:
         del sys.modules[mod_name]
