@@ -15,7 +15,7 @@ no blocking, fusion or reformulation beyond what the cited equation states.
 Notation: T cache rows, d head dim, n reference-query rows of this KV head
 (row i = r*G + g pairs reference position r with query head g), t budget.
 
-Readings of points the paper leaves open (each is listed in the design doc):
+Readings of points the paper leaves open:
 
 * ``scale``: the paper omits the 1/sqrt(d) factor of attention logits as a
   notational convention (Sec. 3.1).  Every model-attention logit q.k here is

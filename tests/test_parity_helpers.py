@@ -1,5 +1,5 @@
 """The GPU-vs-oracle comparison helpers (``oracle/parity.py``) on constructed
-cases whose verdict is known: a checker that accepts everything would make
+cases whose outcome is known: a checker that accepts everything would make
 every GPU parity test vacuous, one that rejects valid results would hide
 real agreement.  CPU only."""
 import numpy as np
