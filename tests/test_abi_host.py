@@ -41,7 +41,7 @@ def test_status_strings(lib):
 
 def _cfg(**kw):
     w = synth.WORKLOADS["llama8b_layer_T8192"]
-    return workload.layer_config(w, 8, **kw)
+    return workload.layer_config(w, kw.pop("H_kv", 8), **kw)
 
 
 def test_workspace_bytes_sizes_and_rejections(lib):
@@ -78,6 +78,11 @@ def test_probability_triple_only_when_t_not_tileable(lib):
     (dict(chunk_len=-1), 1), (dict(T=1 << 20, chunk_len=8), 2), (dict(selector=3), 1), (dict(selector=-1), 1),
     (dict(selector=2, T=1, t=1), 2), (dict(lambda_m=1.5), 1), (dict(ridge_w=-1.0), 1), (dict(eps_w=0.0), 1),
     (dict(b_min=3.0, b_max=2.0), 1), (dict(flags=0x80), 1),
+    (dict(logit_scale=float("nan")), 1), (dict(logit_scale=float("inf")), 1), (dict(lambda_m=float("nan")), 1),
+    (dict(ridge_v=float("inf")), 1), (dict(b_max=float("inf")), 1), (dict(eps_w=float("nan")), 1),
+    (dict(n_pos=65536), 2),            # n T = 2^31: per-head offsets would leave 32 bits
+    (dict(H_kv=8192), 2),              # H_kv times the K slices exceeds the grid's y limit
+    (dict(t=50000, T=60000), 2),       # t^2 >= 2^31
 ])
 def test_compact_rejects_bad_config_without_gpu(lib, kw, code):
     idx = {f: 1 for f in pk.INDEXER_FIELDS}
