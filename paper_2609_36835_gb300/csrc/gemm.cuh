@@ -53,9 +53,6 @@ struct RowK {
       for (int q = 0; q < 8; ++q) v[q] = (r < R && k + q < kend) ? to_f32(src[q]) : 0.f;
     }
   }
-  __device__ __forceinline__ bool inb(int k0, int kend, int q) const {
-    return (r0 + (int)(threadIdx.x & 127) < R) && (k0 + (int)(threadIdx.x >> 7) * 8 + q < kend);
-  }
   __device__ __forceinline__ int row() const { return r0 + (threadIdx.x & 127); }
   __device__ __forceinline__ void store(float* S, const float (&v)[8]) const {
     const int r = threadIdx.x & 127, kq = (threadIdx.x >> 7) * 8;
@@ -109,7 +106,6 @@ struct ColK {
 };
 
 __device__ __forceinline__ int tile_row(int i) { return (threadIdx.x >> 4) * 4 + (i & 3) + (i >> 2) * 64; }
-__device__ __forceinline__ int tile_col(int j) { return (threadIdx.x & 15) * 4 + (j & 3) + (j >> 2) * 64; }
 
 template <class LA, class LB>
 __device__ __forceinline__ void gemm_mainloop(LA& la, LB& lb, int kb, int ke, float (&acc)[8][8],
