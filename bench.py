@@ -16,6 +16,7 @@ from __future__ import annotations
 
 import argparse
 import ctypes
+import datetime
 import hashlib
 import json
 import os
@@ -60,7 +61,7 @@ def dominant_source_hash() -> str:
 def parse_args(argv=None):
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=("gpu", "reference"), default="gpu")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
@@ -127,10 +128,15 @@ def context_layers(layers: int, rank: int):
 # ------------------------------------------------------------------ clocks
 
 class ClockSampler:
-    """nvidia-smi clock / throttle sampling in the background (-lms 200)."""
-    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    """nvidia-smi clock / throttle sampling in the background (-lms 200).
+
+    Each sample carries nvidia-smi's own query time, so ``stop(window)``
+    keeps the samples taken inside the timed region (host wall-clock
+    seconds), whatever buffering the pipe adds."""
+    Q = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    REASONS = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
 
     def __init__(self, index: int):
         self.index = index
@@ -152,7 +158,44 @@ class ClockSampler:
         for line in self.proc.stdout:
             self.lines.append(line.strip())
 
-    def stop(self):
+    @staticmethod
+    def _when(field: str):
+        """nvidia-smi's 'YYYY/MM/DD HH:MM:SS.mmm' (local time) as epoch seconds, or None."""
+        try:
+            dt = datetime.datetime.strptime(field.strip(), "%Y/%m/%d %H:%M:%S.%f")
+        except ValueError:
+            return None
+        return time.mktime(dt.timetuple()) + dt.microsecond / 1e6
+
+    @classmethod
+    def parse(cls, lines, window=None):
+        """Summary of the sample lines: median SM clock, max clock, active
+        throttle reasons.  With ``window`` = (t0, t1), host wall-clock seconds,
+        only samples queried inside it count; if none were, all samples count
+        and ``in_window`` says so."""
+        rows = []
+        for l in lines:
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 10:
+                continue
+            try:
+                sm, mx = float(f[2]), float(f[3])
+            except ValueError:
+                continue
+            act = {nm for nm, v in zip(cls.REASONS, f[6:10]) if v.lower().startswith("active")}
+            rows.append((cls._when(f[0]), sm, mx, act))
+        if not rows:
+            return None
+        inside = rows
+        if window is not None:
+            t0, t1 = window
+            inside = [r for r in rows if r[0] is not None and t0 <= r[0] <= t1]
+        use = inside if inside else rows
+        return {"sm_mhz": statistics.median(r[1] for r in use), "sm_max_mhz": max(r[2] for r in use),
+                "reasons": sorted(set().union(*(r[3] for r in use))), "samples": len(use),
+                "in_window": bool(inside) if window is not None else None, "samples_total": len(rows)}
+
+    def stop(self, window=None):
         if self.proc is None:
             return None
         self.proc.terminate()
@@ -161,24 +204,7 @@ class ClockSampler:
         except subprocess.TimeoutExpired:
             self.proc.kill()
         self.th.join(timeout=5)
-        sm, mx, reasons = [], [], set()
-        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
-        for l in self.lines:
-            f = [x.strip() for x in l.split(",")]
-            if len(f) < 9:
-                continue
-            try:
-                sm.append(float(f[1]))
-                mx.append(float(f[2]))
-            except ValueError:
-                continue
-            for nm, v in zip(names, f[5:9]):
-                if v.lower().startswith("active"):
-                    reasons.add(nm)
-        if not sm:
-            return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm)}
+        return self.parse(self.lines, window)
 
 
 # ------------------------------------------------------------- helpers
@@ -371,13 +397,15 @@ def run_gpu(args, dist: Dist):
     time.sleep(0.3)
     dist.barrier()
     torch.cuda.synchronize()
+    w0 = time.time()
     t_start.record(stream)
     for s in range(args.steps):
         launches += step(handles[s])
     t_end.record(stream)
     torch.cuda.synchronize()
+    w1 = time.time()
     dist.barrier()
-    clk = clocks.stop()
+    clk = clocks.stop((w0, w1))
     ms_total = t_start.elapsed_time(t_end)
     ms_total = dist.max(ms_total, dev)
     ms_step = ms_total / args.steps

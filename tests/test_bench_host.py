@@ -72,3 +72,46 @@ def test_reference_arm_only_rank0_prints(monkeypatch):
     with redirect_stdout(buf):
         assert bench.main(["--impl", "reference", "--workload", "single_head_T1024"]) == 0
     assert buf.getvalue() == ""
+
+
+_FAKE_SMI = """#!/bin/bash
+# stand-in for nvidia-smi's looped query: one sample every 50 ms, power cap active
+while true; do
+  printf '%s, 0, 2070, 2070, 612.50, 0x0000000000000004, Not Active, Not Active, Not Active, Active\\n' \\
+    "$(date +'%Y/%m/%d %H:%M:%S.%3N')"
+  sleep 0.05
+done
+"""
+
+
+def test_clock_sampler_keeps_the_samples_of_the_timed_region(monkeypatch, tmp_path):
+    import time
+    smi = tmp_path / "nvidia-smi"
+    smi.write_text(_FAKE_SMI)
+    smi.chmod(0o755)
+    monkeypatch.setenv("PATH", str(tmp_path) + os.pathsep + os.environ["PATH"])
+    c = bench.ClockSampler(0)
+    c.start()
+    time.sleep(0.4)
+    t0 = time.time()
+    time.sleep(0.5)
+    t1 = time.time()
+    time.sleep(0.3)
+    clk = c.stop((t0, t1))
+    assert clk["in_window"] and clk["sm_mhz"] == 2070.0 and clk["reasons"] == ["sw_power_cap"]
+    assert 4 <= clk["samples"] <= 12 < clk["samples_total"]
+
+
+def test_clock_summary_parsing_and_fallback():
+    lines = ["2026/01/02 03:04:05.100, 0, 1980, 2070, 900.1, 0x0, Not Active, Not Active, Not Active, Not Active",
+             "2026/01/02 03:04:05.300, 0, 2070, 2070, 950.0, 0x4, Not Active, Active, Not Active, Active",
+             "2026/01/02 03:04:05.500, 0, [N/A], 2070, 950.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+             "garbage"]
+    t = bench.ClockSampler._when("2026/01/02 03:04:05.200")
+    clk = bench.ClockSampler.parse(lines, (t, t + 0.2))
+    assert clk["samples"] == 1 and clk["sm_mhz"] == 2070.0
+    assert clk["reasons"] == ["hw_thermal_slowdown", "sw_power_cap"] and clk["samples_total"] == 2
+    # no sample inside the window: all samples count, flagged
+    clk = bench.ClockSampler.parse(lines, (t + 10, t + 11))
+    assert clk["in_window"] is False and clk["samples"] == 2 and clk["sm_mhz"] == 2025.0
+    assert bench.ClockSampler.parse(["garbage"]) is None
