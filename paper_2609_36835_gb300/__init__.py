@@ -160,7 +160,41 @@ def _ptr(x) -> Optional[int]:
         return None
     if isinstance(x, int):
         return x
+    if not x.is_contiguous():
+        # the C ABI takes dense row-major arrays; a strided view would be read with the wrong layout
+        raise ValueError("arckv: tensor arguments must be contiguous (row-major); got strides %s"
+                         % (tuple(x.stride()),))
     return x.data_ptr()
+
+
+def _expect(name: str, x, dtypes, shape=None):
+    """Check a torch tensor argument of the helpers below: dtype, shape (None
+    entries match any extent) and dense layout.  Raises ValueError."""
+    import torch
+    if not isinstance(x, torch.Tensor):
+        raise ValueError("arckv: %s must be a torch tensor" % name)
+    if x.dtype not in dtypes:
+        raise ValueError("arckv: %s must be %s, got %s" % (name, " or ".join(map(str, dtypes)), x.dtype))
+    if shape is not None and (x.dim() != len(shape) or
+                              any(w is not None and int(g) != int(w) for g, w in zip(x.shape, shape))):
+        raise ValueError("arckv: %s must have shape %s, got %s" % (
+            name, tuple("*" if w is None else w for w in shape), tuple(x.shape)))
+    if not x.is_contiguous():
+        raise ValueError("arckv: %s must be contiguous (row-major)" % name)
+
+
+def _on_one_cuda_device(**tensors):
+    """All given tensors (None entries skipped) on one CUDA device: the
+    kernels read them there and there is no CPU path.  Raises ValueError."""
+    dev = None
+    for name, x in tensors.items():
+        if x is None:
+            continue
+        if x.device.type != "cuda":
+            raise ValueError("arckv: %s must be on a CUDA device, got %s (there is no CPU path)" % (name, x.device))
+        if dev is not None and x.device != dev:
+            raise ValueError("arckv: %s is on %s but the other arguments on %s" % (name, x.device, dev))
+        dev = x.device
 
 
 def _stream_handle(stream) -> Optional[int]:
@@ -246,6 +280,28 @@ def compact_layer(cfg: Config, K, V, Q_ref, X_ref, idx: Dict[str, object], *, ws
     and call ``arckv_compact``.  Returns a dict of tensors plus 'status' and
     'launches'.  Raises ArckvError on a non-OK status when ``check``."""
     import torch
+    bf, i32 = (torch.bfloat16,), (torch.int32,)
+    H, T, d, n = cfg.H_kv, cfg.T, cfg.d, cfg.n_pos * cfg.G
+    _expect("K", K, bf, (H, T, d))
+    _expect("V", V, bf, (H, T, d))
+    _expect("Q_ref", Q_ref, bf)
+    if Q_ref.shape[0] != H or Q_ref.numel() != H * n * d:
+        raise ValueError("arckv: Q_ref must hold [H_kv][n_pos * G][d] = %s, got shape %s"
+                         % ((H, n, d), tuple(Q_ref.shape)))
+    if cfg.selector == SELECTOR_INDEXER and anchors_in is None:
+        _expect("X_ref", X_ref, bf, (cfg.n_pos, cfg.d_x))
+        for f in INDEXER_FIELDS:
+            _expect("indexer." + f, idx.get(f), bf)
+            if idx[f].shape[0] != H:
+                raise ValueError("arckv: indexer.%s must lead with H_kv = %d, got shape %s"
+                                 % (f, H, tuple(idx[f].shape)))
+    if anchors_in is not None:
+        _expect("anchors_in", anchors_in, i32, (H, anchor_count(cfg)))
+    if assign_in is not None:
+        _expect("assign_in", assign_in, i32, (H, T))
+    checked_idx = {} if not (cfg.selector == SELECTOR_INDEXER and anchors_in is None) else \
+        {"X_ref": X_ref, **{"indexer." + f: idx[f] for f in INDEXER_FIELDS}}
+    _on_one_cuda_device(K=K, V=V, Q_ref=Q_ref, anchors_in=anchors_in, assign_in=assign_in, **checked_idx)
     dev = K.device
     f32 = dict(dtype=torch.float32, device=dev)
     need = workspace_bytes(cfg)
@@ -278,8 +334,13 @@ def compact_layer(cfg: Config, K, V, Q_ref, X_ref, idx: Dict[str, object], *, ws
 def attend(Q, C_k, beta, C_v, logit_scale: float = 0.0, *, ws=None, stream=None, check: bool = True):
     """O = softmax(scale Q C_k^T + beta) C_v for Q [H, n, 128] bf16 on the device."""
     import torch
+    _expect("Q", Q, (torch.bfloat16,), (None, None, None))
     H, n, d = Q.shape
+    _expect("C_k", C_k, (torch.float32,), (H, None, d))
     t = C_k.shape[1]
+    _expect("beta", beta, (torch.float32,), (H, t))
+    _expect("C_v", C_v, (torch.float32,), (H, t, d))
+    _on_one_cuda_device(Q=Q, C_k=C_k, beta=beta, C_v=C_v)
     need = attend_workspace_bytes(H, n, t, d)
     if need == 0:
         raise ArckvError(2, "arckv_attend_workspace_bytes")
@@ -297,7 +358,20 @@ def attend_joint(Q, C_k=None, beta=None, C_v=None, K_fixed=None, V_fixed=None, l
     """O = softmax(scale Q [C_k; K_fixed]^T + [beta; 0]) [C_v; V_fixed] (App. A.7) for Q [H, n, 128] bf16.
     C_k / C_v fp32 or bf16 (both the same); either block may be omitted."""
     import torch
+    _expect("Q", Q, (torch.bfloat16,), (None, None, None))
     H, n, d = Q.shape
+    if (C_k is None) != (C_v is None) or (C_k is None) != (beta is None):
+        raise ValueError("arckv: C_k, beta and C_v are given together or not at all")
+    if (K_fixed is None) != (V_fixed is None):
+        raise ValueError("arckv: K_fixed and V_fixed are given together or not at all")
+    if C_k is not None:
+        _expect("C_k", C_k, (torch.float32, torch.bfloat16), (H, None, d))
+        _expect("C_v", C_v, (C_k.dtype,), (H, C_k.shape[1], d))
+        _expect("beta", beta, (torch.float32,), (H, C_k.shape[1]))
+    if K_fixed is not None:
+        _expect("K_fixed", K_fixed, (torch.bfloat16,), (H, None, d))
+        _expect("V_fixed", V_fixed, (torch.bfloat16,), (H, K_fixed.shape[1], d))
+    _on_one_cuda_device(Q=Q, C_k=C_k, beta=beta, C_v=C_v, K_fixed=K_fixed, V_fixed=V_fixed)
     t = 0 if C_k is None else C_k.shape[1]
     F = 0 if K_fixed is None else K_fixed.shape[1]
     need = attend_joint_workspace_bytes(H, n, t, F, d)
@@ -317,8 +391,14 @@ def attend_joint(Q, C_k=None, beta=None, C_v=None, K_fixed=None, V_fixed=None, l
 def truncated_error(Q_eval, K, V, S, logit_scale: float = 0.0, *, stream=None, check: bool = True):
     """E(S) per head (App. B.1) for Q_eval [H, n, 128], K, V [H, T, 128] bf16 and anchors S [H, t] int32."""
     import torch
+    _expect("Q_eval", Q_eval, (torch.bfloat16,), (None, None, None))
     H, n, d = Q_eval.shape
+    _expect("K", K, (torch.bfloat16,), (H, None, d))
     T = K.shape[1]
+    _expect("V", V, (torch.bfloat16,), (H, T, d))
+    if S is not None:
+        _expect("S", S, (torch.int32,), (H, None))
+    _on_one_cuda_device(Q_eval=Q_eval, K=K, V=V, S=S)
     t = 0 if S is None else S.shape[1]
     need = int(load_library().arckv_truncated_error_workspace_bytes(H, n, T, t, d))
     if need == 0:

@@ -150,3 +150,35 @@ def test_attend_joint_rejects_bad_arguments_without_gpu(lib):
     assert call(ws_bytes=need - 1) == 3
     assert call(flags=0x4) == 1
     assert call(logit_scale=-1.0) == 1
+
+
+def test_torch_helpers_validate_arguments_before_the_library():
+    """Wrong dtype, shape or layout, or host tensors, are refused by the
+    binding itself: nothing reaches the library, and there is no CPU path."""
+    import torch
+    cfg = _cfg(T=64, n_pos=4, t=8, H_kv=2)
+    bf = lambda *s: torch.zeros(*s, dtype=torch.bfloat16)
+    K = bf(2, 64, 128)
+    with pytest.raises(ValueError, match="contiguous"):
+        pk._ptr(torch.zeros(4, 4).t())
+    with pytest.raises(ValueError, match="K must be torch.bfloat16"):
+        pk.compact_layer(cfg, K.float(), K, bf(2, 16, 128), bf(4, cfg.d_x), {})
+    with pytest.raises(ValueError, match="K must have shape"):
+        pk.compact_layer(cfg, bf(2, 65, 128), K, bf(2, 16, 128), bf(4, cfg.d_x), {})
+    with pytest.raises(ValueError, match="indexer.L_q must be a torch tensor"):
+        pk.compact_layer(cfg, K, K, bf(2, 16, 128), bf(4, cfg.d_x), {})
+    with pytest.raises(ValueError, match="anchors_in must have shape"):
+        pk.compact_layer(cfg, K, K, bf(2, 16, 128), None, None, anchors_in=torch.zeros(2, 7, dtype=torch.int32))
+    with pytest.raises(ValueError, match="K must be on a CUDA device"):
+        pk.compact_layer(cfg, K, K, bf(2, 16, 128), None, None, anchors_in=torch.zeros(2, 8, dtype=torch.int32))
+    f32 = lambda *s: torch.zeros(*s, dtype=torch.float32)
+    with pytest.raises(ValueError, match="beta must be torch.float32"):
+        pk.attend(bf(2, 4, 128), f32(2, 8, 128), torch.zeros(2, 8, dtype=torch.float64), f32(2, 8, 128))
+    with pytest.raises(ValueError, match="CUDA device"):
+        pk.attend(bf(2, 4, 128), f32(2, 8, 128), f32(2, 8), f32(2, 8, 128))
+    with pytest.raises(ValueError, match="together"):
+        pk.attend_joint(bf(2, 4, 128), f32(2, 8, 128), f32(2, 8), None)
+    with pytest.raises(ValueError, match="C_v must be torch.float32"):
+        pk.attend_joint(bf(2, 4, 128), f32(2, 8, 128), f32(2, 8), bf(2, 8, 128))
+    with pytest.raises(ValueError, match="S must be torch.int32"):
+        pk.truncated_error(bf(2, 4, 128), K, K, torch.zeros(2, 8, dtype=torch.int64))
