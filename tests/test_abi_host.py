@@ -182,3 +182,30 @@ def test_torch_helpers_validate_arguments_before_the_library():
         pk.attend_joint(bf(2, 4, 128), f32(2, 8, 128), f32(2, 8), bf(2, 8, 128))
     with pytest.raises(ValueError, match="S must be torch.int32"):
         pk.truncated_error(bf(2, 4, 128), K, K, torch.zeros(2, 8, dtype=torch.int64))
+
+
+def test_plain_c_program_uses_the_header_and_library(lib, tmp_path):
+    """The boundary is a C ABI: a C99 program (tests/abi_consumer.c) compiles
+    against include/arckv.h with -pedantic, links libarckv.so, and gets the
+    same host-side answers as the Python binding."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no C compiler")
+    root = Path(__file__).resolve().parent.parent
+    pkg = root / "paper_2609_36835_gb300"
+    exe = tmp_path / "abi_consumer"
+    subprocess.run([gcc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", "-I", str(root / "include"),
+                    str(root / "tests" / "abi_consumer.c"), "-L", str(pkg), "-larckv", "-Wl,-rpath," + str(pkg),
+                    "-o", str(exe)], check=True)
+    out = dict(l.split(" ", 1) for l in subprocess.run([str(exe)], check=True, capture_output=True,
+                                                         text=True).stdout.splitlines())
+    assert int(out["workspace_bytes"]) == pk.workspace_bytes(_cfg()) > 0
+    assert int(out["workspace_bytes_bad"]) == 0
+    w32 = synth.WORKLOADS["llama8b_T32768_r05"]
+    assert int(out["anchor_count_chunked"]) == pk.anchor_count(workload.layer_config(w32, 8, chunk_len=8192)) == 1640
+    assert int(out["attend_workspace_bytes"]) == pk.attend_workspace_bytes(2, 16, 8)
+    for code in range(9):
+        assert out["status_%d" % code] == pk.status_string(code)
+    assert int(out["compact_null_config"]) == 1 and int(out["compact_bad_shape"]) == 2
