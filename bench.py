@@ -68,7 +68,8 @@ def parse_args(argv=None):
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--streams", type=int, default=4,
                     help="CUDA streams (each with its own workspace) the layers of a context are spread over")
-    ap.add_argument("--cpu-pairs", type=int, default=4, help="(layer, head) pairs the oracle baseline times")
+    ap.add_argument("--cpu-pairs", type=int, default=12,
+                    help="(layer, head) pairs the oracle baseline times (about 1 s each on 16 cores)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--selector", choices=("indexer", "ha", "vi"), default="indexer",
                     help="anchor scores: the ARC-KV indexer (default) or the HA / VI selectors of App. B.1")
@@ -225,6 +226,23 @@ def blas_threads() -> int:
     except OSError:
         pass
     return len(os.sched_getaffinity(0))
+
+
+def cpu_sample_pairs(layers: int, heads: int, k: int):
+    """k distinct (layer, KV head) pairs spread over the context: layers evenly
+    spaced from the first to the last with heads stepping by 3, topped up in
+    (layer, head) order where those repeat (deterministic)."""
+    k = max(1, min(k, layers * heads))
+    out = []
+    for i in range(k):
+        p = ((i * (layers - 1)) // max(1, k - 1), (3 * i) % heads)
+        if p not in out:
+            out.append(p)
+    for l in range(layers):
+        for h in range(heads):
+            if len(out) < k and (l, h) not in out:
+                out.append((l, h))
+    return out
 
 
 def oracle_pair_seconds(w, pairs, selector="indexer", chunk_len=0):
@@ -530,8 +548,7 @@ def run_gpu(args, dist: Dist):
         "clocks": clk,
     }
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
-        spread = [(0, 0), (w.layers - 1, w.H_kv - 1), (w.layers // 2, 3 % w.H_kv), (w.layers // 4, 5 % w.H_kv)]
-        pairs = spread[:max(1, min(len(spread), args.cpu_pairs))]
+        pairs = cpu_sample_pairs(w.layers, w.H_kv, args.cpu_pairs)
         times = oracle_pair_seconds(w, pairs, args.selector, args.chunk_len)
         per_pair = statistics.mean(times)
         n_pairs = w.layers * w.H_kv

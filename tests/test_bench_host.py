@@ -115,3 +115,11 @@ def test_clock_summary_parsing_and_fallback():
     clk = bench.ClockSampler.parse(lines, (t + 10, t + 11))
     assert clk["in_window"] is False and clk["samples"] == 2 and clk["sm_mhz"] == 2025.0
     assert bench.ClockSampler.parse(["garbage"]) is None
+
+
+@pytest.mark.parametrize("layers,heads,k", [(32, 8, 12), (1, 1, 12), (1, 6, 6), (3, 3, 9), (32, 8, 400)])
+def test_cpu_baseline_sample_pairs_are_distinct_and_spread(layers, heads, k):
+    pairs = bench.cpu_sample_pairs(layers, heads, k)
+    assert len(pairs) == len(set(pairs)) == min(k, layers * heads)
+    assert all(0 <= l < layers and 0 <= h < heads for l, h in pairs)
+    assert pairs[0] == (0, 0) and (k < 2 or layers * heads < 2 or max(l for l, _ in pairs) == layers - 1)
