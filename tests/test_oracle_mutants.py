@@ -90,6 +90,17 @@ MUTANTS = [
     # diagnostics
     ("output_loss_unnormalised", "axis=1) / np.sum(y * y, axis=1))", "axis=1))"),
     ("mass_error_sign", "np.linalg.norm(Phi_C @ w_star - m)", "np.linalg.norm(Phi_C @ w_star + m)"),
+    # axes and groupings
+    ("projection_heads_grouped_wrongly", "qz = (Q @ W[\"L_q\"].T + c @ W[\"L_c\"].T).reshape(Q.shape[0], H_I, d_I)",
+     "qz = (Q @ W[\"L_q\"].T + c @ W[\"L_c\"].T).reshape(Q.shape[0], d_I, H_I).transpose(0, 2, 1)"),
+    ("value_context_softmax_over_queries", "    A = _softmax_rows(logits)\n", "    A = _softmax_rows(logits.T).T\n"),
+    ("pool_softmax_over_queries", "    pi = _softmax_rows(I)\n", "    pi = _softmax_rows(I.T).T\n"),
+    ("merge_not_normalised", "    mu = num / den[:, None]\n", "    mu = num\n"),
+    ("loo_distance_sign", "dist2 = np.maximum(vv - 2.0 * (O @ V.T) + oo, 0.0)", "dist2 = np.maximum(vv + 2.0 * (O @ V.T) + oo, 0.0)"),
+    ("pipeline_default_scale_1_over_d", "scale = cfg.scale if cfg.scale is not None else 1.0 / np.sqrt(d)",
+     "scale = cfg.scale if cfg.scale is not None else 1.0 / d"),
+    ("beta_fit_against_cache_keys", "Phi_C = np.exp(attention_logits(Q, C_k, scale) - z[:, None])",
+     "Phi_C = np.exp(attention_logits(Q, C_k, 1.0) - z[:, None])"),
     # the pipeline of Sec. 3.2
     ("pipeline_merges_values", "C_k, _ = merge_keys(K, kappa, logphi, S, cfg.lambda_m)",
      "C_k, _ = merge_keys(V, kappa, logphi, S, cfg.lambda_m)"),

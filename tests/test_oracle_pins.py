@@ -670,3 +670,18 @@ def test_pipeline_tiny_brute_force_loops():
         Y[i] = sum(p[j] * V[j] for j in range(T)) / sum(p)
     Cv = _stacked_qr_solve(Ph, Y, cfg.ridge_v * np.trace(Ph.T @ Ph) / t)
     assert np.allclose(out["C_v"], Cv, rtol=1e-9, atol=1e-11)
+
+
+def test_pipeline_default_logit_scale_is_inverse_sqrt_d():
+    """Reading of Sec. 3.1: the paper writes attention logits without the
+    1/sqrt(d) factor as a notational convention, so the default model-attention
+    scale is 1/sqrt(d) = 1/sqrt(128): the pipeline with no scale given equals
+    the one with that scale, and differs from scale 1."""
+    w, K, V, Q, Xr, W = small_pair(T=40, n_pos=8)
+    a = oracle.compact_pair(K, V, Q, Xr, W, oracle.OracleConfig(t=6))
+    b = oracle.compact_pair(K, V, Q, Xr, W, oracle.OracleConfig(t=6, scale=128 ** -0.5))
+    c = oracle.compact_pair(K, V, Q, Xr, W, oracle.OracleConfig(t=6, scale=1.0))
+    # 128 ** -0.5 and 1 / sqrt(128) may differ in the last bit: integer decisions equal, values to 1e-12
+    assert all(np.array_equal(a[k], b[k]) for k in ("anchors", "assign"))
+    assert all(np.allclose(a[k], b[k], rtol=1e-12, atol=1e-12) for k in ("C_k", "beta", "C_v"))
+    assert not np.allclose(a["C_v"], c["C_v"])
