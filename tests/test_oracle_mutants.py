@@ -137,6 +137,22 @@ PARITY_MUTANTS = [
 ]
 
 
+# slips in the seeded input generator, against tests/test_synth_recipe.py
+SYNTH_SRC = ROOT / "synth" / "__init__.py"
+SYNTH_PINS_SRC = Path(__file__).resolve().parent / "test_synth_recipe.py"
+SYNTH_MUTANTS = [
+    ("outliers_x4", "k[:, _outlier_channels(w, layer)] *= 8.0", "k[:, _outlier_channels(w, layer)] *= 4.0"),
+    ("no_attention_sink", "    k[0] *= 10.0\n", ""),
+    ("rope_theta_10000", "ROPE_THETA = 500000.0", "ROPE_THETA = 10000.0"),
+    ("rope_interleaved_pairs", "x1, x2 = x[:, :half], x[:, half:]", "x1, x2 = x[:, 0::2], x[:, 1::2]"),
+    ("query_noise_1", "+ 0.5 * g.standard_normal((n, D_HEAD))", "+ 1.0 * g.standard_normal((n, D_HEAD))"),
+    ("bf16_truncates", "u = (u + 0x7FFF + ((u >> 16) & 1)) >> 16", "u = u >> 16"),
+    ("bias_std_1", '"b_x": nrm((s.H_I,), 0.1)', '"b_x": nrm((s.H_I,), 1.0)'),
+    ("outliers_reseeded_everywhere", "layer if w.outliers_per_layer else 0", "layer"),
+    ("values_from_key_stream", "gv = _rng(w.wid, layer, head, _S_VALS)", "gv = _rng(w.wid, layer, head, _S_KEYS)"),
+]
+
+
 def _load(name: str, source: str, path: Path) -> types.ModuleType:
     mod = types.ModuleType(name)
     mod.__file__ = str(path)
@@ -158,8 +174,11 @@ def _run_pins(mod: types.ModuleType, stop_at_first: bool, pins_src: Path = PINS_
     setattr(pins, attr, mod)
     failed = []
     for name in sorted(n for n in vars(pins) if n.startswith("test_")):
+        fn = getattr(pins, name)
+        if fn.__code__.co_argcount:   # parametrized tests need their arguments: not run here
+            continue
         try:
-            getattr(pins, name)()
+            fn()
         except Exception:   # an AssertionError, or an error the slip provokes
             failed.append(name)
             if stop_at_first:
@@ -173,8 +192,9 @@ def _mutant_source(old: str, new: str, src_path: Path = ORACLE_SRC) -> str:
     return src.replace(old, new)
 
 
-@pytest.mark.parametrize("src,pins,attr", [(ORACLE_SRC, PINS_SRC, "oracle"), (PARITY_SRC, PARITY_PINS_SRC, "parity")],
-                         ids=["oracle", "parity"])
+@pytest.mark.parametrize("src,pins,attr", [(ORACLE_SRC, PINS_SRC, "oracle"), (PARITY_SRC, PARITY_PINS_SRC, "parity"),
+                                           (SYNTH_SRC, SYNTH_PINS_SRC, "synth")],
+                         ids=["oracle", "parity", "synth"])
 def test_unmodified_copy_passes_every_pin(src, pins, attr):
     mod = _load("_copy_" + attr, src.read_text(), src)
     try:
@@ -199,5 +219,15 @@ def test_planted_mistake_in_parity_helpers_fails_a_check(name, old, new):
     mod = _load(mod_name, _mutant_source(old, new, PARITY_SRC), PARITY_SRC)
     try:
         assert _run_pins(mod, True, PARITY_PINS_SRC, "parity"), f"no check catches {name}"
+    finally:
+        del sys.modules[mod_name]
+
+
+@pytest.mark.parametrize("name,old,new", SYNTH_MUTANTS, ids=[m[0] for m in SYNTH_MUTANTS])
+def test_planted_mistake_in_input_recipe_fails_a_check(name, old, new):
+    mod_name = "_synth_mutant_" + name
+    mod = _load(mod_name, _mutant_source(old, new, SYNTH_SRC), SYNTH_SRC)
+    try:
+        assert _run_pins(mod, True, SYNTH_PINS_SRC, "synth"), f"no check catches {name}"
     finally:
         del sys.modules[mod_name]

@@ -32,6 +32,10 @@ def test_rope_is_a_rotation_with_relative_position_dot_products():
     # pair 0 turns by exactly the position (inverse frequency theta^0 = 1)
     ang = np.arctan2(r[:, half], r[:, 0]) - np.arctan2(x[:, half], x[:, 0])
     assert np.allclose(np.cos(ang), np.cos(pos), atol=1e-9) and np.allclose(np.sin(ang), np.sin(pos), atol=1e-9)
+    # the last pair turns at theta^(-126/128) per position, theta = 500000
+    e = np.zeros((1, 128)); e[0, 63] = 1.0
+    re = synth._rope(e, np.array([1000]))
+    assert np.isclose(np.arctan2(re[0, 127], re[0, 63]), 1000 * 500000.0 ** (-126 / 128), rtol=1e-12)
     # q(m) . k(n) depends on m - n only
     q, k = rng.standard_normal((1, 128)), rng.standard_normal((1, 128))
     a = synth._rope(q, np.array([10])) @ synth._rope(k, np.array([3])).T
@@ -66,6 +70,10 @@ def test_values_queries_and_activations_follow_their_laws():
     p = synth.make_pair(W, 0, 1, T=1024, n_pos=64)
     v = synth.bf16_to_f64(p["V"])
     assert abs(v.mean()) < 0.02 and abs(v.var() - 1.0) < 0.03
+    # values are drawn independently of the keys: matched channels are uncorrelated
+    kk = synth.bf16_to_f64(p["K"])[1:]
+    corr = [np.corrcoef(kk[:, c], v[1:, c])[0, 1] for c in range(128)]
+    assert np.max(np.abs(corr)) < 0.15
     # each query is a key plus N(0, 0.5^2): its nearest key sits at squared distance ~0.25 per dim
     q, k = synth.bf16_to_f64(p["Q"]), synth.bf16_to_f64(p["K"])
     d2 = ((q[:, None, :] - k[None, :, :]) ** 2).sum(-1).min(1) / 128
