@@ -140,7 +140,8 @@ typedef struct {
  *   assign     out int32 [H_kv][T] group index kappa(j) in [0, t)
  *   anchors_in in  int32 [H_kv][t] strictly ascending positions in [0, T):
  *              replaces indexer scoring and selection (the hard branch of
- *              Sec. 3.5 and stage-isolated testing); `scores` is then not written
+ *              Sec. 3.5 and stage-isolated testing); `scores` is then not written,
+ *              and X_ref and the indexer weights are not read (they may be NULL)
  *   assign_in  in  int32 [H_kv][T] replaces the computed assignment; requires
  *              anchors_in and must satisfy assign_in[s_r] = r
  *   stage_events  cudaEvent_t[ARCKV_NUM_STAGES + 1] created by the caller; when
