@@ -255,19 +255,28 @@ arckv_status arckv_truncated_error(int32_t H, int32_t n, int32_t T, int32_t t, i
  * kernels, arguments (minus the workspace) and errors.
  *
  * Scratch: one fixed array of ARCKV_ATTEND_STATIC_MAX_FLOATS floats (32 MiB)
- * compiled into libarckv.so as a device global.  Every GPU on which the library
- * is loaded holds it until the process exits; the call itself allocates
- * nothing (no cudaMalloc, no allocating library routine).  A problem needs
- * arckv_attend_static_floats(H_kv, n, t, d) floats of it; larger problems are
- * rejected with ARCKV_ERR_WORKSPACE before anything is enqueued.
+ * compiled into libarckv.so as a device global.  Every GPU on which the
+ * library's device code is loaded holds it until the process exits.  A
+ * problem needs arckv_attend_static_floats(H_kv, n, t, d) floats of it;
+ * larger problems are rejected with ARCKV_ERR_WORKSPACE before anything is
+ * enqueued.
  *
- * The first call on a device looks up the array's device address with that
- * device current (cudaGetSymbolAddress) and caches it; make that first call
- * before any stream capture.  All calls share the one array and it keeps the
- * previous call's contents (the call clears what must start at zero): calls
- * whose GPU work overlaps -- on different streams, or from several host
- * threads -- race on it, so serialise them.  The call always synchronises
- * `stream` and returns the device status.
+ * Set-up: the first call on a device (with that device current) looks up the
+ * array's device address with cudaGetSymbolAddress and keeps it.  Under
+ * CUDA's default lazy module loading that lookup is also when the driver
+ * loads the module holding the array and so reserves its 32 MiB; with
+ * CUDA_MODULE_LOADING=EAGER the reservation happens when the library is
+ * loaded.  Make that first call during start-up -- before any stream capture
+ * and before the phase in which nothing may allocate.  Every later call on
+ * that device makes no allocation of any kind (no cudaMalloc, no cudaFree,
+ * no allocating library routine).  If the device's primary context is reset
+ * (cudaDeviceReset), the next call repeats the set-up in the new context.
+ *
+ * All calls share the one array and it keeps the previous call's contents
+ * (each call clears what must start at zero): calls whose GPU work overlaps
+ * -- on different streams, or from several host threads -- race on it, so
+ * serialise them.  The call synchronises `stream` and returns the device
+ * status.
  */
 #define ARCKV_ATTEND_STATIC_MAX_FLOATS (8u << 20)
 size_t arckv_attend_static_floats(int32_t H_kv, int32_t n, int32_t t, int32_t d);

@@ -2,6 +2,8 @@
 // allocation at call time.  Its scratch is one file-scope __device__ array
 // that the CUDA module loader places in every context that loads this
 // library; the array stays resident until the process exits.
+#include <cudaTypedefs.h>
+
 #include <algorithm>
 #include <mutex>
 
@@ -16,19 +18,51 @@ __device__ __align__(256) float g_attend_scratch[kStaticScratchFloats];
 
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
-float* g_scratch_addr[kMaxDevices];  // per device, filled by the first call on that device
+float* g_scratch_addr[kMaxDevices];        // per device, filled by the first call on that device
+unsigned long long g_scratch_ctx[kMaxDevices];   // id of the context the address belongs to
 
-// The symbol's device address, looked up once per device with that device
-// current.  In host code `g_attend_scratch` names a host-side shadow, never
-// the device memory, so kernels only ever receive this looked-up address.
+PFN_cuCtxGetCurrent_v4000 g_ctx_current = nullptr;
+PFN_cuCtxGetId_v12000 g_ctx_id = nullptr;
+std::once_flag g_ctx_once;
+
+// Id of the current CUDA context (unique for the life of the process), or 0
+// when the driver does not report one or no context is current yet (the
+// address is then looked up again on the next call).  A reset of the device's primary
+// context (cudaDeviceReset) makes a new context with a new id, in which the
+// array has to be looked up again.
+unsigned long long current_context_id() {
+  std::call_once(g_ctx_once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &fn, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_ctx_current = (PFN_cuCtxGetCurrent_v4000)fn;
+    fn = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &fn, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_ctx_id = (PFN_cuCtxGetId_v12000)fn;
+  });
+  if (!g_ctx_current || !g_ctx_id) return 0;
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (g_ctx_current(&ctx) != CUDA_SUCCESS || !ctx || g_ctx_id(ctx, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
+
+// The symbol's device address, looked up with the device current the first
+// time a call runs on that device (and again after a reset of its context).
+// In host code `g_attend_scratch` names a host-side shadow, never the device
+// memory, so kernels only ever receive this looked-up address.
 arckv_status scratch_for_current_device(float** out) {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return ARCKV_ERR_CUDA;
+  const unsigned long long ctx = current_context_id();
   std::lock_guard<std::mutex> lock(g_mu);
-  if (!g_scratch_addr[dev]) {
+  if (!g_scratch_addr[dev] || g_scratch_ctx[dev] != ctx) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_attend_scratch) != cudaSuccess || !p) return ARCKV_ERR_CUDA;
     g_scratch_addr[dev] = (float*)p;
+    g_scratch_ctx[dev] = ctx;
   }
   *out = g_scratch_addr[dev];
   return ARCKV_OK;

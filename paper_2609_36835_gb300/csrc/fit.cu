@@ -1280,7 +1280,7 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
     ++nl;
   }
   const long long cnt = (long long)D.H * nt;
-  phi_kernel<<<min(cdiv(cnt, 256), 152 * 16), 256, 0, st>>>(B.LC, z, B.Phi, D.n, D.t, cnt);
+  phi_kernel<<<stride_grid(cnt, 256, 16), 256, 0, st>>>(B.LC, z, B.Phi, D.n, D.t, cnt);
   ++nl;
   if (D.t > D.n) return nl + fits_dual(D, ridge_w, ridge_v, eps_w, b_min, b_max, m, Y, B, beta, C_v, stt, st);
   // beta system: Gram = Phi_C^T Phi_C.  Its condition number reaches ~1e6 on
@@ -1324,7 +1324,7 @@ __global__ void check_finite_kernel(const float* x, long long count, DevStatus* 
 }
 
 int launch_check_finite(const float* x, long long count, DevStatus* stt, cudaStream_t st) {
-  check_finite_kernel<<<min(cdiv(count, 256), 152 * 8), 256, 0, st>>>(x, count, stt);
+  check_finite_kernel<<<stride_grid(count, 256, 8), 256, 0, st>>>(x, count, stt);
   return 1;
 }
 

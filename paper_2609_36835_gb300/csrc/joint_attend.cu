@@ -633,7 +633,7 @@ int launch_truncated_error(int H, int n, int T, int t, float scale, float eps, c
                            cudaStream_t st) {
   cudaMemsetAsync(inS, 0, (size_t)H * T, st);
   if (t > 0)
-    anchor_mask_kernel<<<std::min(cdiv((long long)H * t, 256), 152 * 4), 256, 0, st>>>(S, t, T, H, inS, stt);
+    anchor_mask_kernel<<<stride_grid((long long)H * t, 256, 4), 256, 0, st>>>(S, t, T, H, inS, stt);
   trunc_err_kernel<<<dim3(cdiv(n, kJR), H), kJThreads, 0, st>>>(Q, n, K, V, T, inS, scale, eps, err);
   row_mean_kernel<<<cdiv(H, 128), 128, 0, st>>>(err, n, H, E);
   return 3;
@@ -643,7 +643,7 @@ JointSplit joint_split(int H, int n, int t, int F) {
   JointSplit s;
   const int L = t + F, rb = cdiv(n, kJR);
   const long long ctas = (long long)H * rb;
-  const int want = (int)std::max<long long>(1, (152LL * 8 + ctas - 1) / ctas);   // about 8 CTAs per SM
+  const int want = (int)std::max<long long>(1, ((long long)tc_gemm_sm_count() * 8 + ctas - 1) / ctas);   // about 8 CTAs per SM
   const int ntiles = cdiv(L, kJTile);
   const int nsp = std::min(want, ntiles);
   s.per_split = cdiv(ntiles, nsp) * kJTile;

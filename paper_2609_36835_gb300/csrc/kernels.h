@@ -35,6 +35,16 @@ inline int realized_anchors(int T, int t, int chunk_len) {
 }
 
 constexpr int kSplitK = 8;   // K slices of the skinny (N = 128) long-K products
+
+// Streaming multiprocessors of the current device (queried once per device).
+int tc_gemm_sm_count();
+// Grid of a grid-stride kernel: enough CTAs for `count` elements at `per_cta`
+// each, capped at `per_sm` resident CTAs on every SM of the device.
+inline int stride_grid(long long count, int per_cta, int per_sm) {
+  const long long want = (count + per_cta - 1) / per_cta;
+  const long long cap = (long long)tc_gemm_sm_count() * per_sm;
+  return (int)(want < 1 ? 1 : (want < cap ? want : cap));
+}
 constexpr int kCholNB = 64;  // Cholesky block size
 
 // ---- indexer (Sec. 3.3, App. A.1) --------------------------------------

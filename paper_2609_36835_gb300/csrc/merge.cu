@@ -29,9 +29,9 @@ int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const 
 // Caller-supplied assignment (copied into the workspace): values in [0, t)
 // and kappa(s_r) = r.  A violation is recorded as ARCKV_ERR_INVALID_ARG and
 // out-of-range entries are clamped to [0, t).  Runs after the anchors check,
-// so anchors are already inside [0, T).
-__global__ void check_assign_kernel(int* kappa, const int* anchors, int T, int t, int H, DevStatus* stt) {
-  const long long total = (long long)H * T;
+// so anchors are already inside [0, T).  Two kernels: the anchor rows are
+// read only after every clamp has landed.
+__global__ void check_assign_range_kernel(int* kappa, int t, long long total, DevStatus* stt) {
   for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < total;
        k += (long long)gridDim.x * blockDim.x) {
     const int v = kappa[k];
@@ -40,20 +40,23 @@ __global__ void check_assign_kernel(int* kappa, const int* anchors, int T, int t
       kappa[k] = min(max(v, 0), t - 1);
     }
   }
+}
+
+__global__ void check_assign_anchor_kernel(const int* kappa, const int* anchors, int T, int t, int H, DevStatus* stt) {
   const long long ta = (long long)H * t;
   for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < ta;
        k += (long long)gridDim.x * blockDim.x) {
     const long long b = k / t;
-    const int a = anchors[k];
-    const int v = kappa[b * T + a];
-    if (v != (int)(k - b * t) && (v >= 0 && v < t)) set_status(stt, ARCKV_ERR_INVALID_ARG);
+    if (kappa[b * T + anchors[k]] != (int)(k - b * t)) set_status(stt, ARCKV_ERR_INVALID_ARG);
   }
 }
 
 int launch_check_assign(const Dims& D, int* kappa, const int* anchors, DevStatus* stt, cudaStream_t st) {
-  check_assign_kernel<<<min(cdiv((long long)D.H * D.T, 256), 152 * 8), 256, 0, st>>>(kappa, anchors, D.T, D.t,
-                                                                                      D.H, stt);
-  return 1;
+  const long long total = (long long)D.H * D.T;
+  check_assign_range_kernel<<<stride_grid(total, 256, 8), 256, 0, st>>>(kappa, D.t, total, stt);
+  check_assign_anchor_kernel<<<stride_grid((long long)D.H * D.t, 256, 8), 256, 0, st>>>(kappa, anchors, D.T, D.t,
+                                                                                     D.H, stt);
+  return 2;
 }
 
 __device__ __forceinline__ int block_excl_scan_1024_m(int v, int* sc, int& total) {

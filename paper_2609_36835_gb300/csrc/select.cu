@@ -162,7 +162,7 @@ __global__ void split_reduce_kernel(const float* part, float* out, long long cou
 
 int launch_split_reduce(int H, int M, int N, int splits, const float* part, float* out, cudaStream_t st) {
   const long long count = (long long)H * M * N;
-  split_reduce_kernel<<<min(cdiv(count, 256), 152 * 16), 256, 0, st>>>(part, out, count, splits);
+  split_reduce_kernel<<<stride_grid(count, 256, 16), 256, 0, st>>>(part, out, count, splits);
   return 1;
 }
 

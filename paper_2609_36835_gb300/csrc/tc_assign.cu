@@ -351,7 +351,7 @@ int launch_assign_tc(const Dims& D, const float* L, float* logphi, const int* an
   if (launch_tc_gemm<128, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.T, D.t, ldn, kfull, stt, st) != cudaSuccess)
     return -1;
   const long long cnt = (long long)D.H * D.T;
-  decode_assign_kernel2<<<min(cdiv(cnt, 256), 152 * 8), 256, 0, st>>>(best, kappa, cnt);
+  decode_assign_kernel2<<<stride_grid(cnt, 256, 8), 256, 0, st>>>(best, kappa, cnt);
   anchor_self_assign_kernel2<<<cdiv((long long)D.H * D.t, 256), 256, 0, st>>>(anchors, kappa, D.T, D.t, D.H);
   return 5;
 }

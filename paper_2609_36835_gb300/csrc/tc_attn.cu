@@ -79,7 +79,7 @@ int launch_value_logits_tc(const Dims& D, const bf16* q_h, const bf16* q_m, cons
 }
 
 int launch_split3(const float* x, bf16* h, bf16* m, bf16* l, long long count, cudaStream_t st) {
-  split3_kernel<<<min(cdiv(count, 256), 152 * 8), 256, 0, st>>>(x, h, m, l, count);
+  split3_kernel<<<stride_grid(count, 256, 8), 256, 0, st>>>(x, h, m, l, count);
   return 1;
 }
 

@@ -19,3 +19,24 @@ def lib():
     _build.build()
     import paper_2609_36835_gb300 as pk
     return pk.load_library()
+
+
+# Figures the GPU parity tests record for the end-of-run summary: the widest
+# anchor tie gap each test accepted, and the end-to-end errors of the call a
+# user makes (its own anchors and assignment).
+PARITY_REPORT = []
+
+
+def pytest_terminal_summary(terminalreporter, exitstatus, config):
+    if not PARITY_REPORT:
+        return
+    terminalreporter.write_sep("-", "parity figures (widest accepted anchor gap relative to the t-th score; "
+                                    "end-to-end held-out output error)")
+    widest = max(r["gap"] for r in PARITY_REPORT)
+    worst_o = max(r["o_err"] for r in PARITY_REPORT)
+    for r in PARITY_REPORT:
+        terminalreporter.write_line(
+            "%-58s h=%-2d exch=%-3d gap=%.2e o_e2e=%.2e assign_ties=%d outputs=%s"
+            % (r["test"][:58], r["head"], r["exch"], r["gap"], r["o_err"], r["ties"], r["outputs"]))
+    terminalreporter.write_line("widest accepted anchor gap %.3e (band 1e-5, widening capped at 2e-5); "
+                                "worst end-to-end held-out error %.3e (bound 2e-3)" % (widest, worst_o))

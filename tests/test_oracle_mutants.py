@@ -114,8 +114,9 @@ PARITY_MUTANTS = [
      "return float(np.linalg.norm(a - b))"),
     ("score_errors_top_t_only", "[: min(len(s), 2 * t)]", "[: min(len(s), t)]"),
     ("anchors_threshold_off_by_one", "k_thr = int(order[t - 1])", "k_thr = int(order[t])"),
-    ("anchors_errors_narrow_the_band", "excess = [abs(s[j] - thr) / thr - err(j) - err(k_thr) for j in diff]",
-     "excess = [abs(s[j] - thr) / thr + err(j) + err(k_thr) for j in diff]"),
+    ("anchors_errors_narrow_the_band", "ok = all(g <= band + widen(j) for", "ok = all(g <= band - widen(j) for"),
+    ("anchors_widening_uncapped", "return w if w <= WIDEN_CAP else 0.0", "return w"),
+    ("anchors_widening_from_one_key", "w = err(j) + err(k_thr)", "w = err(j)"),
     ("anchors_errors_ignored", "return 0.0 if s_gpu is None else abs(float(s_gpu[j]) - s[j]) / abs(s[j])",
      "return 0.0"),
     ("anchors_no_size_check", "if len(a) != len(b) or len(S_gpu) != t:", "if False:"),

@@ -49,19 +49,30 @@ def test_anchor_exchange_inside_and_outside_the_band():
 
 def test_anchor_band_widened_by_the_gpu_score_errors():
     thr = 2.0
-    s = np.array([5.0, 4.0, 3.0, thr, thr * (1 - 3e-5), 1.0])
+    s = np.array([5.0, 4.0, 3.0, thr, thr * (1 - 2.5e-5), 1.0])
     S = np.array([0, 1, 2, 3])
     swapped = np.array([0, 1, 2, 4])
-    assert not parity.anchors_match(swapped, S, s, 4, 1e-5)[0]          # 3e-5 > band
+    assert not parity.anchors_match(swapped, S, s, 4, 1e-5)[0]          # 2.5e-5 > band
     g = s.copy()
-    g[4] *= 1 + 2.5e-5   # the GPU's score at key 4 carries a 2.5e-5 error: 3e-5 - 2.5e-5 <= 1e-5
-    assert parity.anchors_match(swapped, S, s, 4, 1e-5, g)[0]
+    g[4] *= 1 + 1.8e-5   # the GPU's score at key 4 carries a 1.8e-5 error: 2.5e-5 - 1.8e-5 <= 1e-5
+    ok, nd, gap = parity.anchors_match(swapped, S, s, 4, 1e-5, g)
+    assert ok and nd == 2 and np.isclose(gap, 2.5e-5, rtol=1e-9)      # the widest accepted gap is reported
     g = s.copy()
-    g[4] *= 1 + 1e-5     # too small an error to explain a 3e-5 gap
+    g[4] *= 1 + 1e-5     # too small an error to explain a 2.5e-5 gap
     assert not parity.anchors_match(swapped, S, s, 4, 1e-5, g)[0]
     g = s.copy()
-    g[3] *= 1 - 2.5e-5   # the error may sit at the t-th key instead
+    g[3] *= 1 - 1.8e-5   # the error may sit at the t-th key instead
     assert parity.anchors_match(swapped, S, s, 4, 1e-5, g)[0]
+    # errors above the cap (2e-5 in total) widen nothing: a GPU whose scores are
+    # that far off cannot excuse an exchange beyond the plain band
+    g = s.copy()
+    g[4] *= 1 + 3e-5
+    assert not parity.anchors_match(swapped, S, s, 4, 1e-5, g)[0]
+    g = s.copy()
+    g[4] *= 1 + 1.2e-5
+    g[3] *= 1 - 1.2e-5   # 2.4e-5 in total: above the cap
+    assert not parity.anchors_match(swapped, S, s, 4, 1e-5, g)[0]
+    assert parity.WIDEN_CAP == 2e-5
 
 
 def test_chunked_anchors_keep_each_chunk_to_its_own_budget():

@@ -43,16 +43,25 @@ def _inputs(H, n, t, seed):
 
 
 def test_static_scratch_attend_matches_workspace_attend(static_fn, lib):
+    """Two calls in a row against arckv_attend (the same kernels, so the same
+    bits); from the second call on, a call changes neither the device's free
+    memory nor torch's allocations: the first call on a device did the set-up."""
     H, n, t = 3, 200, 77
     stream = torch.cuda.current_stream().cuda_stream
     for call in range(2):                       # two calls in a row share the scratch array
         Q, Ck, beta, Cv = _inputs(H, n, t, seed=call)
         ref = pk.attend(Q, Ck, beta, Cv)        # the workspace entry point
         O = torch.full((H, n, 128), float("nan"), device="cuda")
+        torch.cuda.synchronize()
+        free0, alloc0 = torch.cuda.mem_get_info()[0], torch.cuda.memory_allocated()
         st = static_fn(H, n, t, 128, 0.0, Q.data_ptr(), Ck.data_ptr(), beta.data_ptr(), Cv.data_ptr(),
                        O.data_ptr(), stream)
         assert st == 0, pk.status_string(st)
         torch.cuda.synchronize()
+        free1, alloc1 = torch.cuda.mem_get_info()[0], torch.cuda.memory_allocated()
+        if call > 0:
+            assert free1 == free0 and alloc1 == alloc0, (free0, free1, alloc0, alloc1)
+        assert torch.equal(O, ref)
         assert parity.rel_fro(O.cpu().numpy(), ref.cpu().numpy()) <= 2e-3
 
 
