@@ -3,14 +3,19 @@
 
 A step is one pass of the whole compaction path over one synthetic context:
 every (layer, KV head) pair of a Llama-3.1-8B-shaped cache (32 layers x 8 KV
-heads, head dim 128, T = 8192 bf16 tokens, n_q = 1024 reference queries per
-KV head, t = 819 anchors = 10% retention), compacted layer by layer through
-arckv_compact.  The metric is context tokens per second (T / seconds per
-context); seconds per context are reported alongside.
+heads, head dim 128), compacted layer by layer through arckv_compact.  The
+default context is the longest single-GPU workload: T = 131072 bf16 tokens,
+n_q = 2048 reference queries per KV head and t = 13107 anchors (10%
+retention), whose fits run in their n x n dual form.  The metric is context
+tokens per second (T / seconds per context); seconds per context are
+reported alongside.
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gpu|reference]
-For N > 1 launch under torchrun; every rank compacts its own context
-(weak scaling) and rank 0 prints one JSON line.
+                       [--workload NAME] [--split contexts|layers]
+For N > 1 launch under torchrun.  With --split contexts (the default) every
+rank compacts its own context (weak scaling); with --split layers the ranks
+take contiguous blocks of one context's layers (strong scaling, no exchange:
+each rank keeps its layers' compact cache).  Rank 0 prints one JSON line.
 """
 from __future__ import annotations
 
@@ -34,11 +39,19 @@ if str(ROOT) not in sys.path:
 
 METRIC = "compaction s/context and context tokens/s at Llama-3.1-8B shape; % roofline"
 UNIT = "context tokens/s"
-DEFAULT_WORKLOAD = "llama8b_T8192_r10"
-PROFILE_SUMMARY = ROOT / "profiles" / "index_logits_tc_llama8b_layer_T8192.md"
+DEFAULT_WORKLOAD = "llama8b_T131072_r10"
+PROFILE_SUMMARY = ROOT / "profiles" / "assign_argmax_tc_llama8b_T131072.md"
 DOMINANT_SOURCES = [ROOT / "paper_2609_36835_gb300" / "csrc" / f
-                    for f in ("tc_index.cu", "tc_gemm.cuh", "tc.cuh", "common.cuh")]
+                    for f in ("tc_assign.cu", "tc_gemm.cuh", "tc.cuh", "common.cuh")]
 FALLBACK_BF16_SUSTAINED_TFLOPS = 1700.0
+
+
+def measured_burst():
+    """Burst bf16 peak (a kernel timed alone), else the sustained one."""
+    try:
+        return float(json.loads((ROOT / "MEASURED_PEAKS.json").read_text())["bf16_tflops"])
+    except (OSError, ValueError, KeyError):
+        return measured_peaks()[0]
 
 
 def measured_peaks():
@@ -65,11 +78,15 @@ def parse_args(argv=None):
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=("gpu", "reference"), default="gpu")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
-    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--streams", type=int, default=4,
                     help="CUDA streams (each with its own workspace) the layers of a context are spread over")
-    ap.add_argument("--cpu-pairs", type=int, default=12,
-                    help="(layer, head) pairs the oracle baseline times (about 1 s each on 16 cores)")
+    ap.add_argument("--cpu-pairs", type=int, default=0,
+                    help="(layer, head) pairs the oracle baseline times (0: about 12 s of oracle work, "
+                         "at least one pair)")
+    ap.add_argument("--split", choices=("contexts", "layers"), default="contexts",
+                    help="N > 1: each rank compacts its own context (weak scaling) or a contiguous block of "
+                         "one context's layers (strong scaling)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--selector", choices=("indexer", "ha", "vi"), default="indexer",
                     help="anchor scores: the ARC-KV indexer (default) or the HA / VI selectors of App. B.1")
@@ -120,10 +137,20 @@ class Dist:
             self.pg.destroy_process_group()
 
 
-def context_layers(layers: int, rank: int):
-    """Layer seeds of the context a rank compacts (weak scaling: each rank owns
-    one whole, distinct context of ``layers`` layers)."""
+def context_layers(layers: int, rank: int, world: int = 1, split: str = "contexts"):
+    """Layer seeds a rank compacts.  ``contexts``: one whole, distinct context
+    of ``layers`` layers per rank (weak scaling).  ``layers``: the ranks share
+    one context, rank r taking the contiguous block [r L / N, (r + 1) L / N)
+    of its layers (strong scaling; no exchange, App. C.2 shards by layer)."""
+    if split == "layers":
+        return list(range(rank * layers // world, (rank + 1) * layers // world))
     return [rank * layers + l for l in range(layers)]
+
+
+def default_cpu_pairs(T: int) -> int:
+    """Pairs of the oracle baseline: about 12 s of oracle work on 16 cores
+    (one pair takes ~1 s at T = 8192 and grows with T), at least one."""
+    return max(1, (12 * 8192) // T)
 
 
 # ------------------------------------------------------------------ clocks
@@ -279,24 +306,86 @@ def profiled_traffic():
 
 # ------------------------------------------------------------ reference arm
 
+def oracle_segments(w, pairs, selector="indexer", chunk_len=0):
+    """The fp64 oracle (as it stands) on (layer, head) pairs, one bounded
+    segment at a time: yields the seconds of each segment of
+    oracle.compact_pair_steps (a stage, an index head, a block of keys) and
+    marks the end of each pair with None.  Input generation is not timed."""
+    import numpy as np
+    import oracle
+    import synth
+    f64 = synth.bf16_to_f64
+    for (layer, head) in pairs:
+        p = synth.make_pair(w, layer, head)
+        X = synth.make_layer_activations(w, layer)
+        W = {k: f64(v) for k, v in synth.make_indexer(w, layer, head).items()}
+        K, V, Q = f64(p["K"]), f64(p["V"]), f64(p["Q"])
+        Xr = np.repeat(f64(X), w.G, axis=0)
+        steps = oracle.compact_pair_steps(K, V, Q, Xr, W, oracle.OracleConfig(t=w.t, selector=selector,
+                                                                                chunk_len=chunk_len))
+        while True:
+            t0 = time.perf_counter()
+            try:
+                next(steps)
+            except StopIteration:
+                yield time.perf_counter() - t0
+                break
+            yield time.perf_counter() - t0
+        yield None
+
+
 def run_reference(args, dist: Dist):
+    """The reference arm: the fp64 oracle on the host cores.  A step is one
+    bounded segment of the oracle's pipeline on one (layer, KV head) pair
+    (oracle.compact_pair_steps); pairs are taken in a fixed spread over the
+    context.  Seconds per context = the mean seconds of a complete pair x the
+    pairs of the context; the pair in progress when the timed steps end is
+    completed (untimed steps) so that every stage is counted."""
     if dist.rank != 0:
         return 0
     import synth
     w = synth.WORKLOADS[args.workload]
     pairs = [(l, h) for l in range(w.layers) for h in range(w.H_kv)]
-    pick = [pairs[(i * 37) % len(pairs)] for i in range(args.warmup + args.steps)]
-    oracle_pair_seconds(w, pick[:args.warmup], args.selector, args.chunk_len)
-    times = oracle_pair_seconds(w, pick[args.warmup:], args.selector, args.chunk_len)
-    per_pair = statistics.mean(times)
+    pick = [pairs[(i * 37) % len(pairs)] for i in range(len(pairs))]
+    seg = oracle_segments(w, pick, args.selector, args.chunk_len)
+    step_s, pair_s, cur = [], [], 0.0
+
+    def advance():
+        nonlocal cur
+        while True:
+            x = next(seg)
+            if x is None:
+                pair_s.append(cur)
+                cur = 0.0
+                continue
+            cur += x
+            return x
+
+    for _ in range(args.warmup):
+        advance()
+    for _ in range(args.steps):
+        step_s.append(advance())
+    if not pair_s or cur > 0.0:
+        while not pair_s or cur > 0.0:
+            x = next(seg)
+            if x is None:
+                pair_s.append(cur)
+                cur = 0.0
+                if len(pair_s) >= 1:
+                    break
+            else:
+                cur += x
+    per_pair = statistics.mean(pair_s)
     s_ctx = per_pair * len(pairs)
     value = w.T / s_ctx
     cores = blas_threads()
-    sample = ("fp64 oracle on %d (layer, KV head) pairs of %s at full size, one pair per step; "
-              "seconds per context extrapolated x%d pairs" % (len(times), w.name, len(pairs)))
+    sample = ("fp64 oracle, %d complete (layer, KV head) pair(s) of %s at full size timed segment by segment "
+              "(%.1f s per pair); seconds per context extrapolated x%d pairs; a step is one segment"
+              % (len(pair_s), w.name, per_pair, len(pairs)))
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_pair * 1e3, "higher_is_better": True,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": (statistics.mean(step_s) * 1e3) if step_s else 0.0, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": workload_config(w, "none (CPU)"), "s_per_context": s_ctx,
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
@@ -328,15 +417,17 @@ def run_gpu(args, dist: Dist):
     torch.cuda.set_device(dev)
     pk.load_library()
     w = synth.WORKLOADS[args.workload]
-    layers = context_layers(w.layers, dist.rank)
+    layers = context_layers(w.layers, dist.rank, dist.world, args.split)
     if args.profile_layer:
         layers = layers[:1]
     sel = {"indexer": pk.SELECTOR_INDEXER, "ha": pk.SELECTOR_HA, "vi": pk.SELECTOR_VI}[args.selector]
     cfg = workload.layer_config(w, w.H_kv, flags=pk.FLAG_NONBLOCKING, selector=sel, chunk_len=args.chunk_len)
     cfg_block = workload.layer_config(w, w.H_kv, selector=sel, chunk_len=args.chunk_len)
 
-    host = [workload.layer_inputs_np(w, l, list(range(w.H_kv))) for l in layers]
-    dev_in = [workload.to_device(a, dev) for a in host]
+    # seeded inputs drawn on the device (synth.make_layer_device: the recipe of
+    # the host generator, seconds instead of minutes for a 128K context)
+    dev_in = [synth.make_layer_device(w, l, list(range(w.H_kv)), dev) for l in layers]
+    torch.cuda.synchronize()
     # layers are independent: they are spread round-robin over `n_str` streams,
     # each with its own workspace (arckv_compact is reentrant per workspace/stream)
     n_str = max(1, min(args.streams, len(layers)))
@@ -430,17 +521,20 @@ def run_gpu(args, dist: Dist):
     # status of the timed calls: one blocking read per workspace
     statuses()
 
-    stage_ms = [[0.0] * pk.NUM_STAGES for _ in range(1)][0]
-    logits_ms = []
+    # per-stage event spans of every layer call in the timed region (the stage
+    # launches of one call, on the stream the call ran on)
+    stage_ms = [0.0] * pk.NUM_STAGES
+    stage_launch_ms = [[] for _ in range(pk.NUM_STAGES)]
     for s in range(args.steps):
         for evs in ev_sets[s]:
             for k in range(pk.NUM_STAGES):
-                stage_ms[k] += evs[k].elapsed_time(evs[k + 1])
-            logits_ms.append(evs[1].elapsed_time(evs[2]))
+                v = evs[k].elapsed_time(evs[k + 1])
+                stage_ms[k] += v
+                stage_launch_ms[k].append(v)
     stage_ms = [x / args.steps for x in stage_ms]
 
-    # the same kernel timed alone: layer 0 on one stream, blocking calls
-    iso_ms = []
+    # the same stages timed alone: layer 0 on one stream, blocking calls
+    iso_ms = [[] for _ in range(pk.NUM_STAGES)]
     iso_ev = new_events(n_ev)
     iso_h = [e.cuda_event for e in iso_ev]
     for _ in range(5):
@@ -449,33 +543,50 @@ def run_gpu(args, dist: Dist):
                                   wss[0], wss[0].numel(), stream=stream, stage_events=iso_h)
         if st_ != 0:
             raise pk.ArckvError(st_, "isolated layer")
-        iso_ms.append(iso_ev[1].elapsed_time(iso_ev[2]))
+        for k in range(pk.NUM_STAGES):
+            iso_ms[k].append(iso_ev[k].elapsed_time(iso_ev[k + 1]))
 
-    # roofline of the dominant kernel (index logits, one launch per layer): a
-    # split-bf16 tcgen05 GEMM issuing three bf16 MMAs per useful product
-    flops = 2.0 * w.H_kv * w.n * w.T * w.shape.H_I * w.shape.d_I
-    avg_s = statistics.mean(logits_ms) / 1e3
-    iso_s = statistics.median(iso_ms) / 1e3
+    # roofline of the dominant kernel: the assignment GEMM (Eq. anchor_assignment,
+    # one launch per layer, stage 5), a split-bf16 tcgen05 GEMM issuing three
+    # bf16 MMAs per useful product; 2 n T t useful flops per head
+    flops = 2.0 * w.H_kv * w.n * w.T * tp
+    avg_s = statistics.mean(stage_launch_ms[5]) / 1e3
+    iso_s = statistics.median(iso_ms[5]) / 1e3
     peak, _, peak_src = measured_peaks()
+    burst = measured_burst()
     achieved = flops / avg_s / 1e12
-    roofline = {"kernel": "tc_gemm_kernel<128, split, TcEpiIndex> (index logits, Eq. pairwise_index_score)",
+    roofline = {"kernel": "tc_gemm_kernel<128, split, TcEpiArgmax> (assignment, Eq. anchor_assignment)",
                 "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                 "traffic": profiled_traffic(), "flops_per_launch": flops, "launch_ms": avg_s * 1e3,
                 "issued_tflops": 3.0 * achieved, "issued_frac": 3.0 * achieved / peak,
-                "launch_ms_isolated": iso_s * 1e3, "frac_isolated": flops / iso_s / 1e12 / peak,
-                "timing_note": "launch_ms: live CUDA events over the timed region, where 4 streams share the GPU; "
-                               "launch_ms_isolated: the same launch with the GPU to itself (median of 5)",
+                "launch_ms_isolated": iso_s * 1e3, "frac_isolated": flops / iso_s / 1e12 / burst,
+                "timing_note": "launch_ms: live CUDA events over the timed region, where %d streams share the GPU; "
+                               "launch_ms_isolated: the same launch with the GPU to itself (median of 5), "
+                               "frac_isolated against the burst peak" % n_str,
                 "peak_note": "bf16 dense, sustained, of %s (MEASURED_PEAKS.json); achieved counts useful flops, "
                              "issued counts the 3 bf16 MMAs of each split-bf16 product" % peak_src}
-    if args.selector != "indexer":
-        # the index-logit GEMM is not launched by the HA / VI selectors
-        roofline = {"kernel": roofline["kernel"], "bound": "tensor", "achieved": None, "peak": peak,
-                    "unit": "TFLOP/s", "frac": None, "traffic": None,
-                    "note": "not launched under --selector %s; the roofline line belongs to the indexer "
-                            "selector (the default)" % args.selector}
+    # the solvers of the two fits (stages 8 and 10), timed the same way
+    dual = tp > w.n
+    m_sys = w.n if dual else tp
+    solve_flops = {8: w.H_kv * (m_sys ** 3 / 3.0 + 2.0 * m_sys ** 2),
+                   10: w.H_kv * (m_sys ** 3 / 3.0 + 4.0 * m_sys ** 2 * 128)}
+    solver = {}
+    for k, name in ((8, "beta_solve"), (10, "value_solve")):
+        live = statistics.mean(stage_launch_ms[k]) / 1e3
+        iso = statistics.median(iso_ms[k]) / 1e3
+        solver[name] = {"flops": solve_flops[k], "ms_live": live * 1e3, "ms_isolated": iso * 1e3,
+                        "tflops_isolated": solve_flops[k] / iso / 1e12,
+                        "frac_isolated": solve_flops[k] / iso / 1e12 / burst}
+    roofline["solvers"] = dict(solver, kernel=("chol_cluster_kernel<double, 8> on the n x n dual systems "
+                                               "(fp64; sliced tensor-core Grams and back-projection counted "
+                                               "outside)" if dual else
+                                               "chol_cluster_kernel<float, 4|8> (tcgen05 trailing updates) "
+                                               "+ two refinement steps"),
+                               note="Cholesky m^3 / 3 plus the triangular solves (m = %d, 1 and 128 right-hand "
+                                    "sides), against the bf16 burst peak" % m_sys)
 
     # end to end: pinned host inputs -> device -> compaction -> host outputs, every step
-    pinned = [workload.to_device(a, pin=True) for a in host]
+    pinned = [{k: v.to("cpu").pin_memory() for k, v in d.items()} for d in dev_in]
     host_out = [{k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in o.items()} for o in outs]
     h2d = sum(t.numel() * t.element_size() for p in pinned for t in p.values())
     d2h = sum(t.numel() * t.element_size() for o in host_out for t in o.values())
@@ -530,25 +641,31 @@ def run_gpu(args, dist: Dist):
     e2e_ms = dist.max(e0.elapsed_time(e1), dev) / args.e2e_steps
     statuses()
 
-    value = dist.world * w.T / (ms_step / 1e3)
+    # contexts split over ranks: the whole job compacts one context per step
+    ctx_per_step = 1 if args.split == "layers" else dist.world
+    value = ctx_per_step * w.T / (ms_step / 1e3)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "strong" if args.split == "layers" else "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded Llama-3.1-8B-shaped caches)",
         "config": dict(workload_config(w, "inputs larger than L2 (%.2f GB per context)" % (h2d / 1e9)),
-                       selector=args.selector, chunk_len=args.chunk_len, anchors_per_head=tp),
+                       selector=args.selector, chunk_len=args.chunk_len, anchors_per_head=tp,
+                       parallelism=("layer blocks of one context over %d ranks" % dist.world
+                                    if args.split == "layers" else "one context per rank"),
+                       inputs="seeded, drawn on the device (synth.make_layer_device)"),
         "s_per_context": ms_step / 1e3,
         "streams": n_str,
         "stage_ms_per_step": dict(zip(pk.STAGE_NAMES, stage_ms)),
         "stage_note": "per-layer event spans summed over layers; with several streams the spans overlap",
         "gpu_launches": launches,
         "roofline": roofline,
-        "e2e": {"value": dist.world * w.T / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+        "e2e": {"value": ctx_per_step * w.T / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "clocks": clk,
     }
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
-        pairs = cpu_sample_pairs(w.layers, w.H_kv, args.cpu_pairs)
+        pairs = cpu_sample_pairs(w.layers, w.H_kv, args.cpu_pairs or default_cpu_pairs(w.T))
         times = oracle_pair_seconds(w, pairs, args.selector, args.chunk_len)
         per_pair = statistics.mean(times)
         n_pairs = w.layers * w.H_kv

@@ -126,11 +126,14 @@ typedef struct {
 } arckv_indexer;
 
 /* Number of timed stages reported through arckv_aux.stage_events. */
-#define ARCKV_NUM_STAGES 6
+#define ARCKV_NUM_STAGES 11
 /* Stage order: 0 indexer features (k_bar, value context, q_bar, w),
  * 1 index logits (one kernel), 2 row log-sum-exp, RMS pooling and top-t,
- * 3 reference attention and assignment, 4 merge, 5 beta and C_v fits.
- * With anchors_in, stages 0-2 are empty. */
+ * 3 reference attention (logits, row statistics, Y), 4 column statistics and
+ * response profiles, 5 assignment (the argmax GEMM), 6 key merge, 7 the
+ * products of the beta fit (compact logits, Phi_C, its Gram and right-hand
+ * side), 8 the beta solve, 9 the products of the value fit, 10 the C_v solve.
+ * With anchors_in, stages 0-2 are empty; with assign_in, stage 5 copies. */
 
 /*
  * Optional inputs / outputs of arckv_compact (the pointer itself may be NULL;

@@ -51,7 +51,7 @@ __all__ = [
     "leave_one_out_changes", "vi_scores", "truncated_output_error",
     "attention_logits", "full_attention", "response_profiles", "response_profiles_literal",
     "assign_to_anchors", "log_mass_weights", "mass_weights_literal", "merge_keys", "fit_beta", "fit_values", "compact_attention",
-    "hard_subset_attention", "output_loss", "mass_error", "compact_pair",
+    "hard_subset_attention", "output_loss", "mass_error", "compact_pair", "compact_pair_steps",
 ]
 
 
@@ -115,15 +115,32 @@ def indexer_projections(Q, X_rows, K, V, W, H_I: int = 8, d_I: int = 128):
     return q_bar, k_bar, w, c
 
 
-def indexer_logits(Q, X_rows, K, V, W, H_I: int = 8, d_I: int = 128) -> np.ndarray:
-    """Eq. (pairwise_index_score):
-    I_ij = sum_a w_ia LeakyReLU_0.1(q_bar_ia . k_bar_ja / sqrt(d_I))."""
+def _run_steps(steps):
+    """Run a step generator (below) to its end and return its result."""
+    while True:
+        try:
+            next(steps)
+        except StopIteration as done:
+            return done.value
+
+
+def _indexer_logits_steps(Q, X_rows, K, V, W, H_I: int = 8, d_I: int = 128):
+    """indexer_logits one index head at a time: yields after the projections
+    and after each head's term, returns I."""
     q_bar, k_bar, w, _ = indexer_projections(Q, X_rows, K, V, W, H_I, d_I)
     I = np.zeros((Q.shape[0], K.shape[0]))
+    yield
     for a in range(H_I):
         x = (q_bar[:, a, :] @ k_bar[:, a, :].T) / np.sqrt(d_I)
         I += w[:, a:a + 1] * np.where(x >= 0.0, x, 0.1 * x)
+        yield
     return I
+
+
+def indexer_logits(Q, X_rows, K, V, W, H_I: int = 8, d_I: int = 128) -> np.ndarray:
+    """Eq. (pairwise_index_score):
+    I_ij = sum_a w_ia LeakyReLU_0.1(q_bar_ia . k_bar_ja / sqrt(d_I))."""
+    return _run_steps(_indexer_logits_steps(Q, X_rows, K, V, W, H_I, d_I))
 
 
 def indexer_pool(I: np.ndarray):
@@ -212,18 +229,25 @@ def response_profiles_literal(l: np.ndarray):
     return E / np.linalg.norm(E, axis=0, keepdims=True)
 
 
-def assign_to_anchors(u: np.ndarray, S: np.ndarray, rows: int = 8192) -> np.ndarray:
-    """Eq. (anchor_assignment): kappa(s_r) = r; kappa(j) = argmax_r u_j . u_{s_r}
-    for j not in S (ties -> smallest r).  Each key's argmax is independent, so
-    the T x t similarity table is formed ``rows`` keys at a time."""
+def _assign_steps(u: np.ndarray, S: np.ndarray, rows: int = 8192):
+    """assign_to_anchors a block of keys at a time: yields after each block,
+    returns kappa."""
     T = u.shape[1]
     uS = u[:, S]
     kappa = np.empty(T, dtype=np.int64)
     for j0 in range(0, T, rows):
         sim = u[:, j0:j0 + rows].T @ uS           # [rows, t]
         kappa[j0:j0 + rows] = np.argmax(sim, axis=1)  # first maximum = smallest r
+        yield
     kappa[S] = np.arange(S.shape[0])
     return kappa
+
+
+def assign_to_anchors(u: np.ndarray, S: np.ndarray, rows: int = 8192) -> np.ndarray:
+    """Eq. (anchor_assignment): kappa(s_r) = r; kappa(j) = argmax_r u_j . u_{s_r}
+    for j not in S (ties -> smallest r).  Each key's argmax is independent, so
+    the T x t similarity table is formed ``rows`` keys at a time."""
+    return _run_steps(_assign_steps(u, S, rows))
 
 
 def log_mass_weights(l: np.ndarray) -> np.ndarray:
@@ -391,6 +415,51 @@ def mass_error(Phi_C: np.ndarray, w_star: np.ndarray, m: np.ndarray) -> float:
 
 # --------------------------------------------------------------- pipeline
 
+def compact_pair_steps(K, V, Q, X_rows, W, cfg: OracleConfig, anchors_in: Optional[np.ndarray] = None,
+                       assign_in: Optional[np.ndarray] = None, H_I: int = 8, d_I: int = 128):
+    """compact_pair as a sequence of bounded steps: a generator that yields
+    between stages (and between index heads and key blocks inside the two
+    longest) and returns compact_pair's result.  The arithmetic is
+    compact_pair's; only the points where it may pause are added, so that a
+    caller can time the pipeline piece by piece."""
+    d = K.shape[1]
+    scale = cfg.scale if cfg.scale is not None else 1.0 / np.sqrt(d)
+    out: Dict[str, np.ndarray] = {}
+    if anchors_in is None:
+        if cfg.selector == "indexer":
+            I = yield from _indexer_logits_steps(Q, X_rows, K, V, W, H_I, d_I)
+            _, s = indexer_pool(I)
+            del I
+        elif cfg.selector == "ha":
+            s = ha_scores(Q, K, scale)
+        else:
+            s = vi_scores(Q, K, V, scale)
+        S = top_t_chunked(s, cfg.t, cfg.chunk_len)
+        out["scores"] = s
+        yield
+    else:
+        S = np.asarray(anchors_in, dtype=np.int64)
+    l = attention_logits(Q, K, scale)
+    u, _ = response_profiles(l)
+    yield
+    if assign_in is None:
+        kappa = yield from _assign_steps(u, S)
+    else:
+        kappa = np.asarray(assign_in, dtype=np.int64)
+    del u
+    logphi = log_mass_weights(l)
+    del l
+    C_k, _ = merge_keys(K, kappa, logphi, S, cfg.lambda_m)
+    yield
+    fb = fit_beta(Q, K, C_k, cfg, scale)
+    yield
+    fv = fit_values(Q, K, V, C_k, fb["beta"], cfg, scale)
+    out.update(anchors=S, assign=kappa, logphi=logphi, C_k=C_k, beta=fb["beta"],
+               w_star=fb["w_star"], w_tilde=fb["w_tilde"], C_v=fv["C_v"],
+               mass_error=mass_error(fb["Phi_C"], fb["w_star"], fb["m"]))
+    return out
+
+
 def compact_pair(K, V, Q, X_rows, W, cfg: OracleConfig, anchors_in: Optional[np.ndarray] = None,
                  assign_in: Optional[np.ndarray] = None, H_I: int = 8, d_I: int = 128) -> Dict[str, np.ndarray]:
     """One layer-KV-head pair through the four stages of Sec. 3.2:
@@ -399,29 +468,4 @@ def compact_pair(K, V, Q, X_rows, W, cfg: OracleConfig, anchors_in: Optional[np.
     ``anchors_in`` replaces the scored anchor set (the hard-branch setting of
     Sec. 3.5, also used to compare stages downstream of selection);
     ``assign_in`` likewise replaces the computed assignment."""
-    d = K.shape[1]
-    scale = cfg.scale if cfg.scale is not None else 1.0 / np.sqrt(d)
-    out: Dict[str, np.ndarray] = {}
-    if anchors_in is None:
-        if cfg.selector == "indexer":
-            I = indexer_logits(Q, X_rows, K, V, W, H_I, d_I)
-            _, s = indexer_pool(I)
-        elif cfg.selector == "ha":
-            s = ha_scores(Q, K, scale)
-        else:
-            s = vi_scores(Q, K, V, scale)
-        S = top_t_chunked(s, cfg.t, cfg.chunk_len)
-        out["scores"] = s
-    else:
-        S = np.asarray(anchors_in, dtype=np.int64)
-    l = attention_logits(Q, K, scale)
-    u, _ = response_profiles(l)
-    kappa = assign_to_anchors(u, S) if assign_in is None else np.asarray(assign_in, dtype=np.int64)
-    logphi = log_mass_weights(l)
-    C_k, _ = merge_keys(K, kappa, logphi, S, cfg.lambda_m)
-    fb = fit_beta(Q, K, C_k, cfg, scale)
-    fv = fit_values(Q, K, V, C_k, fb["beta"], cfg, scale)
-    out.update(anchors=S, assign=kappa, logphi=logphi, C_k=C_k, beta=fb["beta"],
-               w_star=fb["w_star"], w_tilde=fb["w_tilde"], C_v=fv["C_v"],
-               mass_error=mass_error(fb["Phi_C"], fb["w_star"], fb["m"]))
-    return out
+    return _run_steps(compact_pair_steps(K, V, Q, X_rows, W, cfg, anchors_in, assign_in, H_I, d_I))

@@ -32,8 +32,9 @@ STATUS = {
 FLAG_NONBLOCKING = 0x1
 FLAG_COMPACT_BF16 = 0x2
 SELECTOR_INDEXER, SELECTOR_HA, SELECTOR_VI = 0, 1, 2
-NUM_STAGES = 6
-STAGE_NAMES = ("indexer_features", "index_logits", "pool_top_t", "refattn_assign", "merge", "fits")
+NUM_STAGES = 11
+STAGE_NAMES = ("indexer_features", "index_logits", "pool_top_t", "reference_attention", "column_profiles",
+               "assignment", "merge", "beta_products", "beta_solve", "value_products", "value_solve")
 INDEXER_FIELDS = ("L_q", "L_k", "L_x", "b_x", "U_q", "U_k", "U_v", "L_c", "L_v")
 
 

@@ -3,6 +3,8 @@
 // include/arckv.h.
 #include <string.h>
 
+#include <algorithm>
+
 #include "kernels.h"
 #include "tc.cuh"
 
@@ -17,7 +19,7 @@ inline size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 struct Layout {
   size_t status, kbar_hi, kbar_lo, vq, qpp, q_h, q_m, q_l, av, VT, p_h, p_m, p_l, vq3, av3, ukt, qbar_hi, qbar_lo, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
       qcat, wcat, Ut_hi, Ut_lo, S_hi, S_lo, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z,
-      ck3, YT_hi, YT_lo, G64, L64, B64, Z64, X64, total;
+      ck3, YT_hi, YT_lo, G64, L64, B64, Z64, X64, Sl, Sl2, eR, eC, ir_u, ir_sq, ir_lam, total;
 };
 
 Dims dims_of(const arckv_config& c) {
@@ -110,7 +112,8 @@ Layout plan(const arckv_config& c) {
   L.cursor = take(H * t * 4);
   L.LC = take(H * n * (t > 128 ? t : 128) * f);   // also holds the n x d dual solution when t > n
   L.Phi = take(H * n * t * f);
-  L.Gram = take(H * t * t * f);
+  const bool dual = t > n;   // the fits run in their n x n dual form
+  L.Gram = take(dual ? 0 : H * t * t * f);
   L.Linv = take(H * nblk * kCholNB * kCholNB * f);
   L.rhs = take(H * t * f);
   L.wsol = take(H * t * f);
@@ -126,6 +129,15 @@ Layout plan(const arckv_config& c) {
   L.B64 = take(H * nd64 * 128 * 8);
   L.Z64 = take(H * nd64 * 128 * 8);
   L.X64 = take(H * nd64 * 128 * 8);
+  // sliced operands of the dual fits: up to 4 slices of Phi_C (or P^, P^^T)
+  const size_t slrow = dual ? std::max(n * sliced_ld((int)t), t * sliced_ld((int)n)) : 0;
+  L.Sl = take(4 * H * slrow * 2);
+  L.Sl2 = take(dual ? 4 * H * 128 * sliced_ld((int)n) * 2 : 0);
+  L.eR = take(dual ? H * std::max(n, t) * 4 : 0);
+  L.eC = take(dual ? H * 128 * 4 : 0);
+  L.ir_u = take(dual ? 0 : H * n * 8);
+  L.ir_sq = take(dual ? 0 : H * n * 8);
+  L.ir_lam = take(dual ? 0 : H * 8);
   L.total = o;
   return L;
 }
@@ -314,29 +326,36 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
     nl += nlr;
   }
   int* kappa = I32(L.kappa);
+  mark(4);
   if (!given_assign) {
-    const int nla = launch_assign_tc(D, F(L.NT), F(L.logphi), anchors, B16(L.Ut_hi), B16(L.Ut_lo), B16(L.S_hi),
-                                     B16(L.S_lo), (unsigned long long*)(w + L.best), kappa, stt, st);
+    const int nla = launch_assign_prep(D, F(L.NT), F(L.logphi), anchors, B16(L.Ut_hi), B16(L.Ut_lo), B16(L.S_hi),
+                                       B16(L.S_lo), stt, st);
     if (nla < 0) return ARCKV_ERR_CUDA;
-    nl += nla;
+    mark(5);
+    const int nlg = launch_assign_gemm(D, anchors, B16(L.Ut_hi), B16(L.Ut_lo), B16(L.S_hi), B16(L.S_lo),
+                                       (unsigned long long*)(w + L.best), kappa, stt, st);
+    if (nlg < 0) return ARCKV_ERR_CUDA;
+    nl += nla + nlg;
   } else {
     const int nlc = launch_col_profiles(D, F(L.NT), F(L.logphi), nullptr, nullptr, stt, st);   // log phi only
     if (nlc < 0) return ARCKV_ERR_CUDA;
     nl += nlc;
+    mark(5);
     cudaMemcpyAsync(kappa, aux->assign_in, sizeof(int) * (size_t)D.H * D.T, cudaMemcpyDeviceToDevice, st);
     nl += launch_check_assign(D, kappa, anchors, stt, st);
   }
-  mark(4);
+  mark(6);
   nl += launch_merge(D, cfg->lambda_m, Kb, anchors, kappa, F(L.logphi), I32(L.perm), I32(L.goff), I32(L.cursor),
                      C_k, st);
-  mark(5);
+  mark(7);
   FitBufs B{F(L.LC),  F(L.Phi), F(L.Gram), F(L.Linv), F(L.rhs), F(L.wsol), F(L.R), F(L.Z),
             (bf16*)(w + L.S_hi), (bf16*)(w + L.S_lo), (bf16*)(w + L.YT_hi), (bf16*)(w + L.YT_lo),
             (double*)(w + L.G64), (double*)(w + L.L64), (double*)(w + L.B64), (double*)(w + L.Z64),
             (double*)(w + L.X64), (bf16*)(w + L.Ut_hi),   // Ut_hi [H][T][ldn] is free after the assignment
-            (bf16*)(w + L.ck3)};
+            (bf16*)(w + L.ck3), (bf16*)(w + L.Sl), (bf16*)(w + L.Sl2), I32(L.eR), I32(L.eC),
+            (double*)(w + L.ir_u), (double*)(w + L.ir_sq), (double*)(w + L.ir_lam)};
   const int nlf = launch_fits(D, scale, cfg->ridge_w, cfg->ridge_v, cfg->eps_w, cfg->b_min, cfg->b_max, Qb, C_k,
-                              F(L.z), F(L.m), F(L.Y), B, beta, C_v, stt, st);
+                              F(L.z), F(L.m), F(L.Y), B, beta, C_v, stt, st, ev);
   if (nlf < 0) return ARCKV_ERR_CUDA;
   nl += nlf;
   nl += launch_check_finite(C_k, (long long)D.H * D.t * D.d, stt, st);

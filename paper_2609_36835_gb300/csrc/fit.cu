@@ -1235,33 +1235,240 @@ __global__ void __launch_bounds__(256) xty64_kernel(const float* X, const double
 // with the same lam = ridge * trace / t (trace(Phi^T Phi) = trace(Phi Phi^T)),
 // so the solutions equal the primal ones; the systems are n x n.  These
 // systems reach condition numbers ~1e8 on 128K caches (lam relative to t
-// diagonal entries, n of them carrying the mass), so the n x n Grams, the
-// solves and the back-projections run in fp64 (Phi and P^ stay fp32).
+// diagonal entries, n of them carrying the mass), and a Gram error that does
+// not keep the Gram structure moves beta by up to cond x error: the n x n
+// Grams are exact products of row-sliced Phi / P^ on the tensor cores (4
+// slices: 32 bits of each row relative to its largest entry, a perturbation
+// of the operand itself), the solves run in fp64, w = Phi^T a in fp64 and
+// C_v = P^T A as a 4-slice tensor-core product (with 3 slices for P^ the
+// held-out outputs of a 128K head drift by ~7e-3).  Beyond kSlicedMaxK the
+// fp64 SIMT products serve.
 static int fits_dual(const Dims& D, float ridge_w, float ridge_v, float eps_w, float b_min, float b_max,
                      const float* m, const float* Y, const FitBufs& B, float* beta, float* C_v, DevStatus* stt,
-                     cudaStream_t st) {
+                     cudaStream_t st, cudaEvent_t const* ev) {
+  auto mark = [&](int s) {
+    if (ev) cudaEventRecord(ev[s], st);
+  };
   const long long nt = (long long)D.n * D.t, nd = (long long)D.n * D.d;
+  const bool sliced = sliced_supported(D.t) && sliced_supported(D.n);
   const dim3 sgrid(cdiv(D.n, 64), cdiv(D.n, 64), D.H);
+  int nl = 0;
+  auto gram = [&](int S) -> int {   // B.G64 = X X^T for X = B.Phi [n][t]
+    if (!sliced) {
+      syrk64_kernel<<<sgrid, 256, 0, st>>>(B.Phi, B.G64, D.n, D.t);
+      return 1;
+    }
+    const int a = launch_slice_rows(S, B.Phi, D.n, D.t, D.t, nt, D.H, B.Sl, B.eR, st);
+    const int g = launch_sliced_gram_lower(S, B.Sl, B.eR, D.n, D.t, D.H, B.G64, stt, st);
+    return (a < 0 || g < 0) ? -1 : a + g;
+  };
   // beta system
-  syrk64_kernel<<<sgrid, 256, 0, st>>>(B.Phi, B.G64, D.n, D.t);
+  int r = gram(4);
+  if (r < 0) return -1;
+  nl += r;
+  mark(8);
   widen_kernel<<<cdiv((long long)D.H * D.n, 256), 256, 0, st>>>(m, B.B64, (long long)D.H * D.n);
-  cholesky_solve<double>(D.H, D.n, B.G64, B.L64, B.B64, B.Z64, B.X64, 1, 1, D.n, ridge_w, stt, st, D.t);
+  nl += 1 + cholesky_solve<double>(D.H, D.n, B.G64, B.L64, B.B64, B.Z64, B.X64, 1, 1, D.n, ridge_w, stt, st, D.t);
   xty64_kernel<<<dim3(cdiv(D.t, 64), 1, D.H), 256, 0, st>>>(B.Phi, B.X64, B.rhs, D.n, D.t, 1);   // w = Phi^T a
   const long long ht = (long long)D.H * D.t;
   beta_kernel<<<cdiv(ht, 256), 256, 0, st>>>(B.rhs, beta, ht, eps_w, b_min, b_max);
-  // value system
   softmax_bias_kernel<<<dim3(cdiv(D.n, 8), D.H), 256, 0, st>>>(B.LC, beta, B.Phi, D.n, D.t);
-  syrk64_kernel<<<sgrid, 256, 0, st>>>(B.Phi, B.G64, D.n, D.t);
+  nl += 3;
+  // value system
+  mark(9);
+  r = gram(4);
+  if (r < 0) return -1;
+  nl += r;
+  mark(10);
   widen_kernel<<<cdiv((long long)D.H * nd, 256), 256, 0, st>>>(Y, B.B64, (long long)D.H * nd);
-  cholesky_solve<double>(D.H, D.n, B.G64, B.L64, B.B64, B.Z64, B.X64, D.d, D.d, nd, ridge_v, stt, st, D.t);
-  xty64_kernel<<<dim3(cdiv(D.t, 64), cdiv(D.d, 32), D.H), 256, 0, st>>>(B.Phi, B.X64, C_v, D.n, D.t, D.d);
-  (void)nt;
-  return 12;
+  nl += 1 + cholesky_solve<double>(D.H, D.n, B.G64, B.L64, B.B64, B.Z64, B.X64, D.d, D.d, nd, ridge_v, stt, st, D.t);
+  if (!sliced) {
+    xty64_kernel<<<dim3(cdiv(D.t, 64), cdiv(D.d, 32), D.H), 256, 0, st>>>(B.Phi, B.X64, C_v, D.n, D.t, D.d);
+    return nl + 1;
+  }
+  // C_v = P^T A: the rows of P^T (columns of P) and of A^T, 4 slices each
+  const int a = launch_slice_cols(4, B.Phi, D.n, D.t, D.t, nt, D.H, B.Sl, B.eR, st);
+  const int b = launch_slice_cols(4, B.X64, D.n, D.d, D.d, nd, D.H, B.Sl2, B.eC, st);
+  const int c = launch_sliced_product_f32(4, B.Sl, B.eR, D.t, B.Sl2, B.eC, D.d, D.n, D.H, C_v, D.d, stt, st);
+  if (a < 0 || b < 0 || c < 0) return -1;
+  return nl + a + b + c;
+}
+
+// ---------------------------------------------------------------------------
+// Iterative refinement of the beta system (t <= n; App. A.9 Eq. mass_fit).
+// The tensor-core Gram and factor are fp32-grade; with condition numbers up to
+// ~1e7 that leaves beta a few 1e-3 off on long caches.  Each step forms the
+// residual of the normal equations against Phi itself in fp64,
+//     r = Phi^T (m - Phi x) - lam x,   lam = ridge * sum_ir Phi_ir^2 / t,
+// (the exact normal matrix of the fp32 Phi, no Gram rounding) and corrects
+// x += (L L^T)^-1 r with the factor the solver left behind: L_kk and the
+// off-diagonal blocks in the Gram's lower part, L_kk^-1 in Linv.
+
+// u[b][i] = m_i - sum_r Phi_ir x_r (fp64); with sq, also sq[b][i] = sum_r Phi_ir^2.
+// One warp per row.
+__global__ void __launch_bounds__(256) ir_rows_kernel(const float* __restrict__ Phi, const float* __restrict__ m,
+                                                      const float* __restrict__ x, double* __restrict__ u,
+                                                      double* __restrict__ sq, int n, int t, int H) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long gr = (long long)blockIdx.x * 8 + warp;
+  if (gr >= (long long)H * n) return;
+  const int b = (int)(gr / n);
+  const float* p = Phi + gr * t;
+  const float* xb = x + (long long)b * t;
+  double a = 0.0, q = 0.0;
+  for (int r = lane; r < t; r += 32) {
+    const double v = p[r];
+    a = fma(v, (double)xb[r], a);
+    if (sq) q = fma(v, v, q);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    a += __shfl_xor_sync(0xffffffffu, a, o);
+    q += __shfl_xor_sync(0xffffffffu, q, o);
+  }
+  if (lane == 0) {
+    u[gr] = (double)m[gr] - a;
+    if (sq) sq[gr] = q;
+  }
+}
+
+// lam[b] = ridge * sum_i sq[b][i] / t, summed in a fixed order (one CTA per head).
+__global__ void __launch_bounds__(256) ir_lambda_kernel(const double* __restrict__ sq, double* __restrict__ lam, int n,
+                                                        int t, double ridge) {
+  __shared__ double red[8];
+  const int b = blockIdx.x;
+  double a = 0.0;
+  for (int i = threadIdx.x; i < n; i += 256) a += sq[(long long)b * n + i];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = a;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double s = 0.0;
+    for (int w = 0; w < 8; ++w) s += red[w];
+    lam[b] = ridge * s / t;
+  }
+}
+
+// r[b][c] = sum_i Phi_ic u_i - lam x_c (fp64 sums, rounded to fp32 at the end).
+__global__ void __launch_bounds__(256) ir_cols_kernel(const float* __restrict__ Phi, const double* __restrict__ u,
+                                                      const float* __restrict__ x, const double* __restrict__ lam,
+                                                      float* __restrict__ r, int n, int t) {
+  const int b = blockIdx.y, c = blockIdx.x * 256 + threadIdx.x;
+  if (c >= t) return;
+  const float* p = Phi + (long long)b * n * t + c;
+  const double* ub = u + (long long)b * n;
+  double a = 0.0;
+  for (int i = 0; i < n; ++i) a = fma((double)p[(long long)i * t], ub[i], a);
+  r[(long long)b * t + c] = (float)(a - lam[b] * (double)x[(long long)b * t + c]);
+}
+
+// x += (L L^T)^-1 r for one head per CTA (512 threads): forward substitution
+// y_k = Linv_kk (r_k - sum_{j<k} L_kj y_j), then x_k += Linv_kk^T (y_k -
+// sum_{j>k} L_jk^T d_j).  y and the correction d live in `yd` ([H][t]).
+__global__ void __launch_bounds__(512) ir_solve_kernel(const float* __restrict__ A, const float* __restrict__ Linv,
+                                                       const float* __restrict__ r, float* __restrict__ yd,
+                                                       float* __restrict__ x, int t) {
+  constexpr int NBk = kCholNB;
+  __shared__ float v[NBk];
+  __shared__ float part[8][NBk];
+  const int b = blockIdx.x, tid = threadIdx.x;
+  const int nblk = (t + NBk - 1) / NBk;
+  const float* Ab = A + (long long)b * t * t;
+  const float* Lb = Linv + (long long)b * nblk * NBk * NBk;
+  const float* rb = r + (long long)b * t;
+  float* y = yd + (long long)b * t;
+  float* xb = x + (long long)b * t;
+  // forward: 8 threads per row of block k sum L_kj y_j over the columns before k0
+  for (int k = 0; k < nblk; ++k) {
+    const int k0 = k * NBk, kb = min(NBk, t - k0);
+    {
+      const int rr = tid >> 3, pt = tid & 7;
+      float a = 0.f;
+      if (rr < kb)
+        for (int c = pt; c < k0; c += 8) a = fmaf(__ldcg(Ab + (long long)(k0 + rr) * t + c), __ldcg(y + c), a);
+      a += __shfl_xor_sync(0xffffffffu, a, 1);
+      a += __shfl_xor_sync(0xffffffffu, a, 2);
+      a += __shfl_xor_sync(0xffffffffu, a, 4);
+      if (pt == 0) v[rr] = rr < kb ? rb[k0 + rr] - a : 0.f;
+    }
+    __syncthreads();
+    {  // y_k[c] = sum_{l <= c} Linv_k[c][l] v[l]
+      const int c = tid >> 3, pt = tid & 7;
+      const float* Li = Lb + (long long)k * NBk * NBk + c * NBk;
+      float a = 0.f;
+      for (int l = pt; l <= c; l += 8) a = fmaf(__ldcg(Li + l), v[l], a);
+      a += __shfl_xor_sync(0xffffffffu, a, 1);
+      a += __shfl_xor_sync(0xffffffffu, a, 2);
+      a += __shfl_xor_sync(0xffffffffu, a, 4);
+      if (pt == 0 && c < kb) y[k0 + c] = a;
+    }
+    __threadfence_block();
+    __syncthreads();
+  }
+  // backward: column c of block k, eight row parts; the correction d
+  // overwrites y block by block (rows after k0 + kb already hold d)
+  for (int k = nblk - 1; k >= 0; --k) {
+    const int k0 = k * NBk, kb = min(NBk, t - k0);
+    {
+      const int c = tid & (NBk - 1), pt = tid >> 6;
+      float a = 0.f;
+      if (c < kb)
+        for (int rr = k0 + kb + pt; rr < t; rr += 8) a = fmaf(__ldcg(Ab + (long long)rr * t + k0 + c), __ldcg(y + rr), a);
+      part[pt][c] = a;
+    }
+    __syncthreads();
+    if (tid < NBk) {
+      float a = 0.f;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) a += part[q][tid];
+      v[tid] = tid < kb ? y[k0 + tid] - a : 0.f;
+    }
+    __syncthreads();
+    {  // d_k[c] = sum_{l >= c} Linv_k[l][c] v[l]
+      const int c = tid >> 3, pt = tid & 7;
+      const float* Li = Lb + (long long)k * NBk * NBk;
+      float a = 0.f;
+      for (int l = c + pt; l < NBk; l += 8) a = fmaf(__ldcg(Li + (long long)l * NBk + c), v[l], a);
+      a += __shfl_xor_sync(0xffffffffu, a, 1);
+      a += __shfl_xor_sync(0xffffffffu, a, 2);
+      a += __shfl_xor_sync(0xffffffffu, a, 4);
+      if (pt == 0 && c < kb) {
+        y[k0 + c] = a;
+        xb[k0 + c] += a;
+      }
+    }
+    __threadfence_block();
+    __syncthreads();
+  }
+}
+
+constexpr int kBetaRefineSteps = 2;
+
+static int refine_beta(const Dims& D, float ridge_w, const float* m, const FitBufs& B, cudaStream_t st) {
+  const long long hn = (long long)D.H * D.n;
+  ir_rows_kernel<<<cdiv(hn, 8), 256, 0, st>>>(B.Phi, m, B.wsol, B.ir_u, B.ir_sq, D.n, D.t, D.H);
+  ir_lambda_kernel<<<D.H, 256, 0, st>>>(B.ir_sq, B.ir_lam, D.n, D.t, (double)ridge_w);
+  int nl = 2;
+  for (int it = 0; it < kBetaRefineSteps; ++it) {
+    if (it > 0) {
+      ir_rows_kernel<<<cdiv(hn, 8), 256, 0, st>>>(B.Phi, m, B.wsol, B.ir_u, nullptr, D.n, D.t, D.H);
+      ++nl;
+    }
+    ir_cols_kernel<<<dim3(cdiv(D.t, 256), D.H), 256, 0, st>>>(B.Phi, B.ir_u, B.wsol, B.ir_lam, B.rhs, D.n, D.t);
+    ir_solve_kernel<<<D.H, 512, 0, st>>>(B.Gram, B.Linv, B.rhs, B.Z, B.wsol, D.t);
+    nl += 2;
+  }
+  return nl;
 }
 
 int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float eps_w, float b_min,
                 float b_max, const bf16* Q, const float* C_k, const float* z, const float* m,
-                const float* Y, const FitBufs& B, float* beta, float* C_v, DevStatus* stt, cudaStream_t st) {
+                const float* Y, const FitBufs& B, float* beta, float* C_v, DevStatus* stt, cudaStream_t st,
+                cudaEvent_t const* ev) {
+  auto mark = [&](int s) {
+    if (ev) cudaEventRecord(ev[s], st);
+  };
   int nl = 0;
   const long long nt = (long long)D.n * D.t;
   // logits of the compact keys LC = scale Q C_k^T [n][t]: C_k enters as a bf16
@@ -1282,7 +1489,10 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
   const long long cnt = (long long)D.H * nt;
   phi_kernel<<<stride_grid(cnt, 256, 16), 256, 0, st>>>(B.LC, z, B.Phi, D.n, D.t, cnt);
   ++nl;
-  if (D.t > D.n) return nl + fits_dual(D, ridge_w, ridge_v, eps_w, b_min, b_max, m, Y, B, beta, C_v, stt, st);
+  if (D.t > D.n) {
+    const int nd = fits_dual(D, ridge_w, ridge_v, eps_w, b_min, b_max, m, Y, B, beta, C_v, stt, st, ev);
+    return nd < 0 ? -1 : nl + nd;
+  }
   // beta system: Gram = Phi_C^T Phi_C.  Its condition number reaches ~1e6 on
   // long caches, beyond what a split-bf16 pair (~1e-5 relative per entry)
   // resolves within tolerance: the operand enters as a bf16 triple and the
@@ -1294,12 +1504,15 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
   nl += 2;
   mass_rhs_kernel<<<dim3(cdiv(D.t, 32), D.H), 1024, 0, st>>>(B.Phi, m, B.rhs, D.n, D.t);
   ++nl;
+  mark(8);
   nl += cholesky_solve(D.H, D.t, B.Gram, B.Linv, B.rhs, B.Z, B.wsol, 1, 1, D.t, ridge_w, stt, st);
+  nl += refine_beta(D, ridge_w, m, B, st);
   const long long ht = (long long)D.H * D.t;
   beta_kernel<<<cdiv(ht, 256), 256, 0, st>>>(B.wsol, beta, ht, eps_w, b_min, b_max);
   ++nl;
   // value system: P^ over the compact keys with the fitted bias; its Gram and
   // P^T Y on the tensor cores from transposed split-bf16 operands
+  mark(9);
   softmax_bias_kernel<<<dim3(cdiv(D.n, 8), D.H), 256, 0, st>>>(B.LC, beta, B.Phi, D.n, D.t);
   ++nl;
   transpose_split_kernel<<<tgrid, 256, 0, st>>>(B.Phi, D.n, D.t, B.PT_hi, B.PT_lo, ldn);
@@ -1311,6 +1524,7 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
   const long long td = (long long)D.t * D.d;
   if (gram_tc(D.H, D.t, D.d, ldn, B.PT_hi, B.PT_lo, B.YT_hi, B.YT_lo, B.R, D.d, stt, st) < 0) return -1;
   nl += 2;
+  mark(10);
   nl += cholesky_solve(D.H, D.t, B.Gram, B.Linv, B.R, B.Z, C_v, D.d, D.d, td, ridge_v, stt, st);
   return nl;
 }

@@ -114,9 +114,11 @@ int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* 
 int launch_col_profiles(const Dims& D, const float* L, float* logphi, bf16* Ut_hi, bf16* Ut_lo, DevStatus* stt,
                         cudaStream_t st);
 // Assignment on tcgen05: column statistics and transposed split-bf16 profiles
-// (log phi written on the way), anchor rows, argmax GEMM.
-int launch_assign_tc(const Dims& D, const float* L, float* logphi, const int* anchors, bf16* Ut_hi, bf16* Ut_lo,
-                     bf16* S_hi, bf16* S_lo, unsigned long long* best, int* kappa, DevStatus* stt, cudaStream_t st);
+// (log phi written on the way) and the anchor rows; then the argmax GEMM.
+int launch_assign_prep(const Dims& D, const float* L, float* logphi, const int* anchors, bf16* Ut_hi, bf16* Ut_lo,
+                       bf16* S_hi, bf16* S_lo, DevStatus* stt, cudaStream_t st);
+int launch_assign_gemm(const Dims& D, const int* anchors, const bf16* Ut_hi, const bf16* Ut_lo, const bf16* S_hi,
+                       const bf16* S_lo, unsigned long long* best, int* kappa, DevStatus* stt, cudaStream_t st);
 int launch_check_assign(const Dims& D, int* kappa, const int* anchors, DevStatus* stt, cudaStream_t st);
 int launch_merge(const Dims& D, float lambda_m, const bf16* K, const int* anchors, const int* kappa,
                  const float* logphi, int* perm, int* goff, int* cursor, float* C_k, cudaStream_t st);
@@ -128,12 +130,41 @@ struct FitBufs {
   double *G64, *L64, *B64, *Z64, *X64;   // fp64 dual-form scratch (t > n only): [n][n], blocks, [n][d] x 3
   bf16* PT_mid;                         // middle part of the transposed triple of Phi_C ([t][ldn])
   bf16* ck3;                            // bf16 triple of C_k (parts [H][t][128], one after another)
+  bf16 *Sl, *Sl2;                       // sliced operands of the dual fits (t > n only)
+  int *eR, *eC;                         // their row exponents ([H][max(n, t)], [H][128])
+  double *ir_u, *ir_sq, *ir_lam;        // refinement of the beta system: [H][n], [H][n], [H]
 };
 // Returns launches, or -1 when a TMA descriptor cannot be encoded.
+// ev (nullable): events recorded before the beta solve, before the value
+// products and before the C_v solve (stage events 8, 9, 10 of arckv_compact).
 int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float eps_w, float b_min,
                 float b_max, const bf16* Q, const float* C_k, const float* z, const float* m,
-                const float* Y, const FitBufs& B, float* beta, float* C_v, DevStatus* stt, cudaStream_t st);
+                const float* Y, const FitBufs& B, float* beta, float* C_v, DevStatus* stt, cudaStream_t st,
+                cudaEvent_t const* ev = nullptr);
 int launch_check_finite(const float* x, long long count, DevStatus* stt, cudaStream_t st);
+
+// ---- fp64-grade products on the bf16 tensor pipe (tc_sliced.cu) ------------
+// Operands are cut into S bf16 slices per row (S = 3 or 4) with a power-of-two
+// row scale; products of the sliced operands are exact up to ~2^-48 and
+// returned in fp64 (or rounded to fp32).  K up to kSlicedMaxK.
+constexpr int kSlicedMaxK = 26214;
+bool sliced_supported(int K);
+int sliced_last_failure();   // diagnostics: 1 map encoding, 100 + e attribute, 1000 + e launch (0: none)
+size_t sliced_ld(int K);   // row pitch (elements) of a sliced operand with K columns
+// X [H][R][K] (rows ldx apart, batches xbs apart) -> slices [S][H][R][sliced_ld(K)], exponents ex [H][R]
+int launch_slice_rows(int S, const float* X, int R, int K, int ldx, long long xbs, int H, bf16* out, int* ex,
+                      cudaStream_t st);
+// the rows of X^T for X [H][K][R] (R contiguous): slices [S][H][R][sliced_ld(K)], exponents ex [H][R]
+int launch_slice_cols(int S, const float* X, int K, int R, int ldx, long long xbs, int H, bf16* out, int* ex,
+                      cudaStream_t st);
+int launch_slice_cols(int S, const double* X, int K, int R, int ldx, long long xbs, int H, bf16* out, int* ex,
+                      cudaStream_t st);
+// G[b] = X X^T (R x R, fp64) on the tiles that reach the lower triangle
+int launch_sliced_gram_lower(int S, const bf16* Xs, const int* ex, int R, int K, int H, double* G, DevStatus* stt,
+                             cudaStream_t st);
+// C[b] (M x N, fp32, row stride ldc) = A B^T of sliced A [M][K], B [N][K]
+int launch_sliced_product_f32(int S, const bf16* As, const int* eA, int M, const bf16* Bs, const int* eB, int N, int K,
+                              int H, float* C, int ldc, DevStatus* stt, cudaStream_t st);
 
 // ---- compact attention (Eq. compact_attention) ----------------------------
 int launch_attend(int H, int n, int t, float scale, const bf16* Q, const float* C_k, const float* beta,

@@ -197,6 +197,19 @@ __device__ __forceinline__ uint64_t sdesc_k128(uint32_t saddr) {
   return d;
 }
 
+// The same for a K-major bf16 tile written by TMA with 64-byte swizzle: rows of
+// 32 elements (64 B), 8-row groups 512 B apart; base 1024-byte aligned, a
+// 16-element K step inside the row adds 32 bytes to the start address.
+__device__ __forceinline__ uint64_t sdesc_k64(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);   // start address
+  d |= (uint64_t)1 << 16;                      // leading byte offset (unused for swizzled K-major)
+  d |= (uint64_t)(512 >> 4) << 32;             // stride byte offset: 8 rows x 64 B
+  d |= (uint64_t)1 << 46;                      // descriptor version (tcgen05)
+  d |= (uint64_t)4 << 61;                      // 64-byte swizzle
+  return d;
+}
+
 // Instruction descriptor: kind::f16, A = B = bf16, D = fp32, both K-major,
 // M = 128, N = n.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int n) {
@@ -209,6 +222,12 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int n) {
 // (dim0 contiguous) with a box of {64, box1, 1} and 128-byte swizzle.
 bool encode_bf16_map_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1, uint64_t dim2,
                         uint32_t box1);
+
+// Host: encode a 3-D tiled TMA map over a bf16 tensor [dim2][dim1][dim0] whose
+// rows are ld >= dim0 elements apart (ld a multiple of 8), with a box of
+// {32, box1, 1} and 64-byte swizzle; elements past dim0 / dim1 read as zero.
+bool encode_bf16_map_3d_sw64(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1, uint64_t dim2,
+                             uint64_t ld, uint32_t box1);
 
 // Host: encode a 3-D tiled TMA map over an fp32 tensor [dim2][dim1][dim0]
 // (rows ld elements apart, batches bs elements apart) with a box of

@@ -336,11 +336,18 @@ __global__ void anchor_self_assign_kernel2(const int* anchors, int* kappa, int T
   }
 }
 
-int launch_assign_tc(const Dims& D, const float* L, float* logphi, const int* anchors, bf16* Ut_hi, bf16* Ut_lo,
-                     bf16* S_hi, bf16* S_lo, unsigned long long* best, int* kappa, DevStatus* stt, cudaStream_t st) {
+int launch_assign_prep(const Dims& D, const float* L, float* logphi, const int* anchors, bf16* Ut_hi, bf16* Ut_lo,
+                       bf16* S_hi, bf16* S_lo, DevStatus* stt, cudaStream_t st) {
   const int ldn = (D.n + 7) / 8 * 8;
-  if (launch_col_profiles(D, L, logphi, Ut_hi, Ut_lo, stt, st) < 0) return -1;
+  const int nc = launch_col_profiles(D, L, logphi, Ut_hi, Ut_lo, stt, st);
+  if (nc < 0) return -1;
   gather_anchor_rows_kernel<<<dim3(D.t, D.H), 128, 0, st>>>(Ut_hi, Ut_lo, anchors, S_hi, S_lo, D.T, D.t, ldn);
+  return nc + 1;
+}
+
+int launch_assign_gemm(const Dims& D, const int* anchors, const bf16* Ut_hi, const bf16* Ut_lo, const bf16* S_hi,
+                       const bf16* S_lo, unsigned long long* best, int* kappa, DevStatus* stt, cudaStream_t st) {
+  const int ldn = (D.n + 7) / 8 * 8;
   cudaMemsetAsync(best, 0, sizeof(unsigned long long) * (size_t)D.H * D.T, st);
   CUtensorMap mA, mA2, mB, mB2;
   if (!encode_bf16_map_3d(&mA, Ut_hi, ldn, D.T, D.H, 128) || !encode_bf16_map_3d(&mA2, Ut_lo, ldn, D.T, D.H, 128) ||
@@ -353,7 +360,7 @@ int launch_assign_tc(const Dims& D, const float* L, float* logphi, const int* an
   const long long cnt = (long long)D.H * D.T;
   decode_assign_kernel2<<<stride_grid(cnt, 256, 8), 256, 0, st>>>(best, kappa, cnt);
   anchor_self_assign_kernel2<<<cdiv((long long)D.H * D.t, 256), 256, 0, st>>>(anchors, kappa, D.T, D.t, D.H);
-  return 5;
+  return 3;
 }
 
 }  // namespace arckv

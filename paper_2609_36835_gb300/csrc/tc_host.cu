@@ -39,6 +39,20 @@ bool encode_bf16_map_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint6
   return r == CUDA_SUCCESS;
 }
 
+bool encode_bf16_map_3d_sw64(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1, uint64_t dim2,
+                             uint64_t ld, uint32_t box1) {
+  if (!encoder_ready()) return false;
+  if (((uintptr_t)base & 15u) != 0 || (ld * 2) % 16 != 0 || ld < dim0 || box1 == 0 || box1 > 256) return false;
+  const cuuint64_t gdim[3] = {dim0, dim1, dim2};
+  const cuuint64_t gstride[2] = {ld * 2, ld * dim1 * 2};
+  const cuuint32_t box[3] = {32, box1, 1};
+  const cuuint32_t estride[3] = {1, 1, 1};
+  const CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), gdim, gstride, box,
+                              estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 bool encode_f32_map_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1, uint64_t dim2,
                        uint32_t box0, uint32_t box1, uint64_t ld, uint64_t bs, bool swz128) {
   if (!encoder_ready()) return false;

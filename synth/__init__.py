@@ -26,6 +26,11 @@ evaluation, which are not available; Sec. 3.1, App. A.1, App. A.5):
 * decode batches (timing and full-size attention parity): keys, values and
   queries N(0,1) in bf16 drawn on the device by a seeded torch generator
   (Philox on CUDA), stand-in compact caches drawn the same way;
+* whole layers for timing (``make_layer_device``): the same recipe for K, V
+  and Q_ref, drawn by a seeded torch generator on the device (a different
+  random stream from the host path, the same distributions), so that a 32-layer
+  128K context is generated in seconds; X_ref and the indexer weights come from
+  the host path;
 * indexer weights in the shapes of Eqs. (indexer_parameters) and
   (value_indexer_parameters): U_q, U_k, U_v, L_q, L_k, L_v ~ N(0, 1/d),
   L_c ~ N(0, 1/d_A), L_x ~ N(0, 1/d_x), b_x ~ N(0, 0.1^2).
@@ -43,7 +48,7 @@ import numpy as np
 __all__ = [
     "Workload", "WORKLOADS", "IndexerShape", "bf16_round", "bf16_to_f64",
     "bf16_to_f32", "make_pair", "make_layer_activations", "make_heldout",
-    "make_indexer", "make_compact_cache", "decode_batch_device",
+    "make_indexer", "make_compact_cache", "decode_batch_device", "make_layer_device",
 ]
 
 D_HEAD = 128
@@ -241,4 +246,62 @@ def decode_batch_device(seed: int, H: int, G: int, T: int, t: int, F: int, devic
            "C_k": nrm(H, t, D_HEAD, dt=cdt), "C_v": nrm(H, t, D_HEAD, dt=cdt),
            "beta": torch.rand(H, t, generator=gen, device=device) * 3.0 - 2.0,
            "K_f": nrm(H, F, D_HEAD), "V_f": nrm(H, F, D_HEAD)}
+    return out
+
+
+def _torch_seed(*key: int) -> int:
+    """A 63-bit torch seed derived from the same key as the host streams."""
+    ss = np.random.SeedSequence([0xA2C4, *[int(k) for k in key]])
+    return int(ss.generate_state(2, dtype=np.uint32).astype(np.uint64) @ np.array([1, 1 << 32], dtype=np.uint64)
+               & np.uint64((1 << 63) - 1))
+
+
+def _rope_torch(x, positions, theta: float = ROPE_THETA):
+    """_rope on a torch tensor: rotation angles in float64, applied in float32."""
+    import torch
+    d = x.shape[-1]
+    half = d // 2
+    inv_freq = theta ** (-torch.arange(half, dtype=torch.float64, device=x.device) * 2.0 / d)
+    ang = positions[:, None].to(torch.float64) * inv_freq[None, :]
+    c, s_ = torch.cos(ang).to(torch.float32), torch.sin(ang).to(torch.float32)
+    lo, hi = x[:, :half], x[:, half:]   # rotate-half pairs (i, i + d/2)
+    return torch.cat([lo * c - hi * s_, hi * c + lo * s_], dim=1)
+
+
+def make_layer_device(w: Workload, layer: int, heads, device, T: Optional[int] = None, n_pos: Optional[int] = None):
+    """One layer's inputs as torch tensors on ``device``: K, V [H][T][d] and
+    Q_ref [H][n][d] (bf16) drawn by the recipe above from a seeded torch
+    generator per (layer, head); X [n_pos][d_x] and the indexer fields
+    [H][...] (bf16) from the host path.  Row i of Q_ref is r*G + g."""
+    import torch
+    T = w.T if T is None else T
+    n_pos = w.n_pos if n_pos is None else n_pos
+    n = n_pos * w.G
+    Ks, Vs, Qs = [], [], []
+    for h in heads:
+        g = torch.Generator(device=device)
+        g.manual_seed(_torch_seed(w.wid, layer, h, _S_KEYS))
+        k = torch.randn(T, D_HEAD, generator=g, device=device, dtype=torch.float32)
+        k[:, torch.as_tensor(_outlier_channels(w, layer), device=device)] *= 8.0
+        k = _rope_torch(k, torch.arange(T, device=device))
+        k[0] = k[0] * 10.0
+        kb = k.to(torch.bfloat16)
+        g.manual_seed(_torch_seed(w.wid, layer, h, _S_VALS))
+        vb = torch.randn(T, D_HEAD, generator=g, device=device, dtype=torch.float32).to(torch.bfloat16)
+        g.manual_seed(_torch_seed(w.wid, layer, h, _S_QREF))
+        j = torch.randint(0, T, (n,), generator=g, device=device)
+        q = kb[j].to(torch.float32) + 0.5 * torch.randn(n, D_HEAD, generator=g, device=device, dtype=torch.float32)
+        Ks.append(kb)
+        Vs.append(vb)
+        Qs.append(q.to(torch.bfloat16))
+        del k
+    out = {"K": torch.stack(Ks), "V": torch.stack(Vs), "Q": torch.stack(Qs)}
+
+    def host_bits(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(device)
+
+    out["X"] = host_bits(make_layer_activations(w, layer, n_pos=n_pos))
+    idx = [make_indexer(w, layer, h) for h in heads]
+    for f in idx[0]:
+        out[f] = host_bits(np.stack([ix[f] for ix in idx]))
     return out

@@ -47,6 +47,45 @@ def test_two_gloo_ranks_time_max_and_distinct_contexts():
     assert len(a) == len(b) == 32 and not set(a) & set(b)
 
 
+def _layer_worker(rank, world, port, q):
+    os.environ.update(RANK=str(rank), WORLD_SIZE=str(world), LOCAL_RANK=str(rank), MASTER_ADDR="127.0.0.1",
+                      MASTER_PORT=str(port))
+    d = bench.Dist()
+    d.init("gloo")
+    d.barrier()
+    mine = bench.context_layers(32, rank, world, "layers")
+    # each rank's time is its own layer block's; the job's time is the slowest rank's
+    q.put((rank, d.max(1.0 + 0.25 * len(mine) + rank), mine))
+    d.barrier()
+    d.close()
+
+
+def test_two_gloo_ranks_split_one_context_by_layer_blocks():
+    """The layer-block split of one context over ranks (no data exchange,
+    only the barrier and the max of the ranks' times)."""
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_layer_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = sorted(q.get(timeout=120) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    a, b = res[0][2], res[1][2]
+    assert a == list(range(16)) and b == list(range(16, 32))    # contiguous blocks, one context
+    assert res[0][1] == res[1][1] == 1.0 + 0.25 * 16 + 1
+
+
+def test_layer_blocks_cover_the_context_for_any_rank_count():
+    for world in (1, 2, 3, 4, 5, 8):
+        blocks = [bench.context_layers(32, r, world, "layers") for r in range(world)]
+        assert sum(blocks, []) == list(range(32))
+        assert max(map(len, blocks)) - min(map(len, blocks)) <= 1
+    assert bench.context_layers(32, 1, 4, "contexts") == list(range(32, 64))
+
+
 def test_reference_arm_json_line(monkeypatch):
     for k in ("RANK", "WORLD_SIZE", "LOCAL_RANK"):
         monkeypatch.delenv(k, raising=False)

@@ -97,23 +97,26 @@ def check_layer(w, heads, sample, T=None, n_pos=None, t=None, layer=0, n_hold=64
     O_user = pk.attend(Qh_t, out["C_k"], out["beta"], out["C_v"], cfg.logit_scale)
     for h in sample:
         ref = refs[h]
-        # the call a user makes, end to end (Eq. compact_attention on held-out queries)
+        # the call a user makes, end to end (Eq. compact_attention on held-out
+        # queries).  Its decisions are integers taken at near-ties (anchor
+        # scores within the tie band, assignment rows within TAU, some of them
+        # 1e-13 apart); a tied row decided the other way moves its group's
+        # merged key, and the fits and the held-out output with it, so the
+        # end-to-end bound holds where the decisions agree, and the floating-
+        # point stages are otherwise compared on the oracle's decisions below.
         O_ref = oracle.compact_attention(synth.bf16_to_f64(Qh[h]), ref["C_k"], ref["beta"], ref["C_v"], scale)
         e_user = parity.rel_fro(_np(O_user[h]), O_ref)
-        assert e_user <= 2e-3, ("held-out output of the unassisted call", h, e_user)
         same_S = np.array_equal(_np(out["anchors"][h]), ref["anchors"])
         n_ties = int(np.sum(_np(out["assign"][h]) != ref["assign"])) if same_S else -1
-        compared = "O"
-        if same_S and n_ties == 0 and ref.get("_exch", 0) == 0:
+        compared = "decisions differ on tied keys"
+        if same_S and n_ties == 0:
             # identical decisions: the unassisted outputs themselves
+            assert e_user <= 2e-3, ("held-out output of the unassisted call", h, e_user)
             assert parity.rel_fro(_np(out["C_k"][h]), ref["C_k"]) <= 2e-3, ("unassisted C_k", h)
-            if cfg.selector == pk.SELECTOR_INDEXER:
-                eb, rest_ok = parity.beta_errors(_np(out["beta"][h]), ref["beta"], ref["w_star"])
-                assert eb <= 2e-3 and rest_ok, ("unassisted beta", h, eb, rest_ok)
-                assert parity.rel_fro(_np(out["C_v"][h]), ref["C_v"]) <= 2e-3, ("unassisted C_v", h)
-                compared = "O,C_k,beta,C_v"
-            else:
-                compared = "O,C_k"
+            eb, rest_ok = parity.beta_errors(_np(out["beta"][h]), ref["beta"], ref["w_star"])
+            assert eb <= 2e-3 and rest_ok, ("unassisted beta", h, eb, rest_ok)
+            assert parity.rel_fro(_np(out["C_v"][h]), ref["C_v"]) <= 2e-3, ("unassisted C_v", h)
+            compared = "O,C_k,beta,C_v"
         elif same_S:
             # assignment differs on tied rows only (checked below): the merged
             # keys of the groups both sides formed alike must agree
@@ -121,25 +124,15 @@ def check_layer(w, heads, sample, T=None, n_pos=None, t=None, layer=0, n_hold=64
             moved = np.unique(np.concatenate([kg[kg != kr], kr[kg != kr]]))
             keep = np.setdiff1d(np.arange(len(ref["anchors"])), moved)
             assert parity.rel_fro(_np(out["C_k"][h])[keep], ref["C_k"][keep]) <= 2e-3, ("unassisted C_k rows", h)
-            compared = "O,C_k(%d of %d groups)" % (len(keep), len(ref["anchors"]))
+            compared = "C_k(%d of %d groups)" % (len(keep), len(ref["anchors"]))
         conftest.PARITY_REPORT.append({
             "test": os.environ.get("PYTEST_CURRENT_TEST", "?").split(" ")[0].split("::")[-1], "head": h,
-            "exch": ref.get("_exch", 0), "gap": ref.get("_gap", 0.0), "o_err": e_user, "ties": max(n_ties, 0),
-            "outputs": compared})
+            "exch": ref.get("_exch", 0), "gap": ref.get("_gap", 0.0), "o_err": e_user,
+            "ties": n_ties, "outputs": compared})
         assert parity.rel_fro(_np(out2["C_k"][h]), ref["C_k"]) <= 2e-3
-        if cfg.selector == pk.SELECTOR_INDEXER:
-            eb, rest_ok = parity.beta_errors(_np(out2["beta"][h]), ref["beta"], ref["w_star"])
-            assert eb <= 2e-3 and rest_ok, ("beta", h, eb, rest_ok)
-        else:   # ill-conditioned anchor sets: the mass weights e^beta (see oracle/parity.py)
-            em = parity.mass_weight_error(_np(out2["beta"][h]), ref["beta"])
-            assert em <= 2e-3, ("mass weights", h, em)
-        if cfg.selector == pk.SELECTOR_INDEXER:
-            assert parity.rel_fro(_np(out2["C_v"][h]), ref["C_v"]) <= 2e-3
-        else:   # stage-isolated: the oracle's C_v fit on the GPU's own beta
-            K_, V_, Q_, _, _ = _pair64(arr, h, cfg.G)
-            Cv_ref = oracle.fit_values(Q_, K_, V_, ref["C_k"], _np(out2["beta"][h]).astype(np.float64), _ocfg(cfg),
-                                       scale)["C_v"]
-            assert parity.rel_fro(_np(out2["C_v"][h]), Cv_ref) <= 2e-3
+        eb, rest_ok = parity.beta_errors(_np(out2["beta"][h]), ref["beta"], ref["w_star"])
+        assert eb <= 2e-3 and rest_ok, ("beta", h, eb, rest_ok)
+        assert parity.rel_fro(_np(out2["C_v"][h]), ref["C_v"]) <= 2e-3, ("C_v", h)
         assert parity.rel_fro(_np(O[h]), O_ref) <= 2e-3
         K, V, Q, Xr, W = _pair64(arr, h, cfg.G)
         u, _ = oracle.response_profiles(oracle.attention_logits(Q, K, scale))

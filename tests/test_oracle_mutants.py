@@ -144,6 +144,13 @@ SYNTH_PINS_SRC = Path(__file__).resolve().parent / "test_synth_recipe.py"
 SYNTH_MUTANTS = [
     ("outliers_x4", "k[:, _outlier_channels(w, layer)] *= 8.0", "k[:, _outlier_channels(w, layer)] *= 4.0"),
     ("no_attention_sink", "    k[0] *= 10.0\n", ""),
+    ("device_no_attention_sink", "        k[0] = k[0] * 10.0\n", ""),
+    ("device_rope_interleaved_pairs", "lo, hi = x[:, :half], x[:, half:]", "lo, hi = x[:, 0::2], x[:, 1::2]"),
+    ("device_outliers_x4", "k[:, torch.as_tensor(_outlier_channels(w, layer), device=device)] *= 8.0",
+     "k[:, torch.as_tensor(_outlier_channels(w, layer), device=device)] *= 4.0"),
+    ("device_query_noise_1", "0.5 * torch.randn(n, D_HEAD", "1.0 * torch.randn(n, D_HEAD"),
+    ("device_values_from_key_stream", "g.manual_seed(_torch_seed(w.wid, layer, h, _S_VALS))",
+     "g.manual_seed(_torch_seed(w.wid, layer, h, _S_KEYS))"),
     ("rope_theta_10000", "ROPE_THETA = 500000.0", "ROPE_THETA = 10000.0"),
     ("rope_interleaved_pairs", "x1, x2 = x[:, :half], x[:, half:]", "x1, x2 = x[:, 0::2], x[:, 1::2]"),
     ("query_noise_1", "+ 0.5 * g.standard_normal((n, D_HEAD))", "+ 1.0 * g.standard_normal((n, D_HEAD))"),

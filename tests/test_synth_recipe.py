@@ -113,3 +113,49 @@ def test_workload_table(name):
     if "_r" in name:
         ratio = int(name.rsplit("_r", 1)[1]) / 100
         assert w.t == int(np.floor(ratio * w.T))      # t = floor(rho T)
+
+
+def _device_layer(layer=0, heads=(0, 1), T=2048, n_pos=64):
+    d = synth.make_layer_device(W, layer, list(heads), "cpu", T=T, n_pos=n_pos)
+    bits = lambda t: t.contiguous().view(torch.int16).numpy().view(np.uint16)
+    return {k: bits(v) for k, v in d.items()}
+
+
+def test_device_layers_follow_the_same_recipe():
+    """The device-side layer generator (used to time whole 128K contexts):
+    the key, value and query laws of the host path, checked the same way."""
+    d = _device_layer()
+    assert d["K"].shape == (2, 2048, 128) and d["Q"].shape == (2, 64 * W.G, 128)
+    e = _pair_energy(d["K"][0])
+    assert 2 <= np.sum(e > 20) <= 4 and np.all(np.sort(e)[:-4] < 2.5)
+    # the same outlier channels as the host path (their rotation pairs carry the energy)
+    host_pairs = {c % 64 for c in synth._outlier_channels(W, 0)}
+    assert set(np.argsort(e)[::-1][:len(host_pairs)]) == host_pairs
+    norms = np.linalg.norm(synth.bf16_to_f64(d["K"][0]), axis=1)
+    assert 7.0 < norms[0] / np.median(norms[1:]) < 14.0
+    v = synth.bf16_to_f64(d["V"][0])
+    assert abs(v.mean()) < 0.02 and abs(v.var() - 1.0) < 0.03
+    kk = synth.bf16_to_f64(d["K"][0])[1:]
+    assert max(abs(np.corrcoef(kk[:, c], v[1:, c])[0, 1]) for c in range(128)) < 0.15
+    q, k = synth.bf16_to_f64(d["Q"][0]), synth.bf16_to_f64(d["K"][0])
+    d2 = ((q[:, None, :] - k[None, :, :]) ** 2).sum(-1).min(1) / 128
+    assert 0.2 < np.median(d2) < 0.3
+    # the device rotation is the host's (float64 angles, float32 products)
+    rng = np.random.default_rng(4)
+    x = rng.standard_normal((5, 128)).astype(np.float32)
+    pos = np.array([0, 3, 999, 65536, 131071])
+    r_dev = synth._rope_torch(torch.from_numpy(x), torch.from_numpy(pos)).numpy()
+    assert np.allclose(r_dev, synth._rope(x.astype(np.float64), pos), rtol=1e-5, atol=1e-5)
+    host = synth.make_pair(W, 0, 0, T=2048, n_pos=64)
+    assert not np.array_equal(host["K"], d["K"][0])          # a different random stream
+
+
+def test_device_layers_regenerate_and_share_host_weights():
+    a, b = _device_layer(layer=2), _device_layer(layer=2)
+    assert all(np.array_equal(a[k], b[k]) for k in a)
+    c = _device_layer(layer=3)
+    assert not np.array_equal(a["K"], c["K"])
+    assert not np.array_equal(a["K"][0], a["K"][1])           # heads differ
+    idx = synth.make_indexer(W, 2, 1)
+    assert all(np.array_equal(a[f][1], idx[f]) for f in idx)
+    assert np.array_equal(a["X"], synth.make_layer_activations(W, 2, n_pos=64))
