@@ -19,7 +19,7 @@ inline size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 struct Layout {
   size_t status, kbar_hi, kbar_lo, vq, qpp, q_h, q_m, q_l, av, VT, p_h, p_m, p_l, vq3, av3, ukt, qbar_hi, qbar_lo, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
       qcat, wcat, Ut_hi, Ut_lo, S_hi, S_lo, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z,
-      ck3, YT_hi, YT_lo, G64, L64, B64, Z64, X64, Sl, Sl2, eR, eC, ir_u, ir_sq, ir_lam, total;
+      ck3, YT_hi, YT_lo, G64, L64, B64, Z64, X64, Sl, Sl2, eR, eC, ir_u, ir_sq, ir_lam, Sl3, eC2, cl_lam, total;
 };
 
 Dims dims_of(const arckv_config& c) {
@@ -138,6 +138,10 @@ Layout plan(const arckv_config& c) {
   L.ir_u = take(dual ? 0 : H * n * 8);
   L.ir_sq = take(dual ? 0 : H * n * 8);
   L.ir_lam = take(dual ? 0 : H * 8);
+  // the blocked dual solves: 5-slice right-hand-side columns (up to 128 rows of K <= n)
+  L.Sl3 = take(dual ? 5 * H * 128 * sliced_ld((int)n) * 2 : 0);
+  L.eC2 = take(dual ? H * 128 * 4 : 0);
+  L.cl_lam = take(dual ? H * 8 : 0);
   L.total = o;
   return L;
 }
@@ -353,7 +357,8 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
             (double*)(w + L.G64), (double*)(w + L.L64), (double*)(w + L.B64), (double*)(w + L.Z64),
             (double*)(w + L.X64), (bf16*)(w + L.Ut_hi),   // Ut_hi [H][T][ldn] is free after the assignment
             (bf16*)(w + L.ck3), (bf16*)(w + L.Sl), (bf16*)(w + L.Sl2), I32(L.eR), I32(L.eC),
-            (double*)(w + L.ir_u), (double*)(w + L.ir_sq), (double*)(w + L.ir_lam)};
+            (double*)(w + L.ir_u), (double*)(w + L.ir_sq), (double*)(w + L.ir_lam), (bf16*)(w + L.Sl3),
+            I32(L.eC2), (double*)(w + L.cl_lam)};
   const int nlf = launch_fits(D, scale, cfg->ridge_w, cfg->ridge_v, cfg->eps_w, cfg->b_min, cfg->b_max, Qb, C_k,
                               F(L.z), F(L.m), F(L.Y), B, beta, C_v, stt, st, ev);
   if (nlf < 0) return ARCKV_ERR_CUDA;

@@ -1029,10 +1029,10 @@ static int cholesky_solve(int H, int t, R* Gram, R* Linv, R* B, R* Z, R* X, int 
   const int smem = 4 * kTileF<R> * (int)sizeof(R) + (std::is_same<R, float>::value ? kTcStageBytes : 0);
   const R td = (R)(tdiv > 0 ? tdiv : t);
   if (cluster_size(t) == 8) {
-    cudaFuncSetAttribute(chol_cluster_kernel<R, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    set_dyn_smem((const void*)chol_cluster_kernel<R, 8>, smem);
     chol_cluster_kernel<R, 8><<<8 * H, kCT, smem, st>>>(Gram, Linv, B, Z, X, t, nrhs, ldb, bbs, (R)ridge, td, stt);
   } else {
-    cudaFuncSetAttribute(chol_cluster_kernel<R, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    set_dyn_smem((const void*)chol_cluster_kernel<R, 4>, smem);
     chol_cluster_kernel<R, 4><<<4 * H, kCT, smem, st>>>(Gram, Linv, B, Z, X, t, nrhs, ldb, bbs, (R)ridge, td, stt);
   }
   return 1;
@@ -1228,6 +1228,187 @@ __global__ void __launch_bounds__(256) xty64_kernel(const float* X, const double
   }
 }
 
+// ---------------------------------------------------------------------------
+// Blocked Cholesky solve of the fp64 dual systems, (A + lam I) X = B with
+// lam = ridge * trace(A) / tdiv, A [H][n][n] (lower part read, overwritten
+// by L), B [H][n][nrhs] (overwritten by the forward solution Y = L^-1 B),
+// X [H][n][nrhs].  Right-looking over 64-wide block columns; every block
+// product runs on the tensor pipe as an exact product of 5-slice operands
+// (2^-40 of each row's largest entry per operand, the same backward error as
+// an fp64 factorisation to ~1e-12), and only the 64 x 64 diagonal factors
+// and inverses run in fp64 on the SIMT pipes:
+//   for k:  L_kk = chol(A_kk + lam I), Linv_kk = L_kk^-1        (fp64 SIMT)
+//           L_ik = A_ik Linv_kk^T                        i > k  (sliced)
+//           A_ij -= L_ik L_jk^T                    j <= i, i > k  (sliced, lower tiles)
+//           Y_k = Linv_kk B_k;  B_i -= L_ik Y_k         i > k  (sliced)
+//   for k descending:  Z_k = sum_{i>k} L_ik^T X_i            (sliced)
+//           X_k = Linv_kk^T (Y_k - Z_k)                         (fp64 SIMT)
+
+constexpr int kCholSlices = 5;
+
+__global__ void chol_lambda_kernel(const double* A, int n, double ridge, double tdiv, double* lam, DevStatus* stt) {
+  __shared__ double red[8];
+  const int b = blockIdx.x;
+  const double* Ab = A + (long long)b * n * n;
+  double a = 0.0;
+  for (int r = threadIdx.x; r < n; r += 256) a += Ab[(long long)r * n + r];
+  a = warp_sum_r(a);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = a;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double tr = 0.0;
+    for (int w = 0; w < 8; ++w) tr += red[w];
+    if (!isfinite(tr)) set_status(stt, ARCKV_ERR_NONFINITE);
+    lam[b] = ridge * tr / tdiv;
+  }
+}
+
+// Factor diagonal block k of every head (one CTA per head): L_kk into A,
+// L_kk^-1 into Linv[k]; a non-positive pivot records ARCKV_ERR_NOT_SPD.
+__global__ void __launch_bounds__(kCT, 1) chol_diag_kernel(double* A, double* Linv, int n, int k, const double* lam,
+                                                           DevStatus* stt) {
+  extern __shared__ __align__(16) unsigned char smraw[];
+  double* sm = (double*)smraw;
+  Tile<double> S1 = (Tile<double>)sm;
+  Tile<double> S2 = (Tile<double>)(sm + kTileF<double>);
+  Tile<double> S3 = (Tile<double>)(sm + 2 * kTileF<double>);
+  __shared__ int bad;
+  const int b = blockIdx.x, nblk = (n + NB - 1) / NB;
+  if (threadIdx.x == 0) bad = 0;
+  __syncthreads();
+  factor_diag<double>(A + (long long)b * n * n, Linv + (long long)b * nblk * NB * NB, n, k, lam[b], S1, S2, S3, &bad);
+  if (threadIdx.x == 0 && bad) set_status(stt, ARCKV_ERR_NOT_SPD);
+}
+
+// X_k = Linv_kk^T (Y_k - Z_k) for block k of every head, 32 right-hand sides
+// per CTA (grid: head x column group): V = Y_k - Z_k and Linv_kk go through
+// shared memory, X[k0 + c][j] = sum_{l >= c} Linv_k[l][c] V[l][j].
+__global__ void __launch_bounds__(256) chol_back_block_kernel(const double* Linv, const double* Y, const double* Z,
+                                                              double* X, int n, int k, int nrhs, int useZ) {
+  __shared__ double Ls[NB][NB + 1];
+  __shared__ double Vs[NB][33];
+  const int b = blockIdx.x, j0 = blockIdx.y * 32, nblk = (n + NB - 1) / NB, k0 = k * NB, kb = min(NB, n - k0);
+  const int nj = min(32, nrhs - j0);
+  const double* Li = Linv + ((long long)b * nblk + k) * NB * NB;
+  const double* Yb = Y + ((long long)b * n + k0) * nrhs + j0;
+  const double* Zb = Z + (long long)b * NB * nrhs + j0;
+  double* Xb = X + ((long long)b * n + k0) * nrhs + j0;
+  for (int e = threadIdx.x; e < NB * NB; e += 256) Ls[e / NB][e % NB] = Li[e];
+  for (int e = threadIdx.x; e < NB * 32; e += 256) {
+    const int l = e >> 5, j = e & 31;
+    Vs[l][j] = (l < kb && j < nj) ? Yb[(long long)l * nrhs + j] - (useZ ? Zb[(long long)l * nrhs + j] : 0.0) : 0.0;
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < kb * 32; e += 256) {
+    const int c = e >> 5, j = e & 31;
+    double a = 0.0;
+    for (int l = c; l < kb; ++l) a = fma(Ls[l][c], Vs[l][j], a);
+    if (j < nj) Xb[(long long)c * nrhs + j] = a;
+  }
+}
+
+// w[b][r] = sum_i Phi[b][i][r] a[b][i] in fp64 (Phi fp32 [n][t]): one thread
+// per column r, the rows of the column read coalesced across the warp.
+__global__ void __launch_bounds__(256) phi_t_vec_kernel(const float* __restrict__ Phi, const double* __restrict__ a,
+                                                        float* __restrict__ w, int n, int t) {
+  const int b = blockIdx.y, r = blockIdx.x * 256 + threadIdx.x;
+  if (r >= t) return;
+  const float* p = Phi + (long long)b * n * t + r;
+  const double* ab = a + (long long)b * n;
+  double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
+  int i = 0;
+  for (; i + 4 <= n; i += 4) {
+    s0 = fma((double)p[(long long)i * t], ab[i], s0);
+    s1 = fma((double)p[(long long)(i + 1) * t], ab[i + 1], s1);
+    s2 = fma((double)p[(long long)(i + 2) * t], ab[i + 2], s2);
+    s3 = fma((double)p[(long long)(i + 3) * t], ab[i + 3], s3);
+  }
+  for (; i < n; ++i) s0 = fma((double)p[(long long)i * t], ab[i], s0);
+  w[(long long)b * t + r] = (float)((s0 + s1) + (s2 + s3));
+}
+
+template <typename R>
+__global__ void __launch_bounds__(512) tri_solve_kernel(const R* __restrict__ A, const R* __restrict__ Linv,
+                                                        const R* __restrict__ r, R* __restrict__ yd,
+                                                        R* __restrict__ x, int t);
+
+struct CholSlicedBufs {
+  bf16 *sA, *sB, *sC;   // 5-slice operands: panel rows / columns, Linv_kk rows, right-hand-side columns
+  int *eA, *eB, *eC;
+  double *lam, *Z;      // [H], [H][64][nrhs]
+};
+
+static int chol_solve_sliced(int H, int n, double* A, double* Linv, double* B, double* X, int nrhs, double ridge,
+                             double tdiv, const CholSlicedBufs& W, DevStatus* stt, cudaStream_t st) {
+  constexpr int S = kCholSlices;
+  const int nblk = (n + NB - 1) / NB;
+  const long long nn = (long long)n * n, nr = (long long)n * nrhs, lb = (long long)nblk * NB * NB;
+  const int dsm = 3 * kTileF<double> * (int)sizeof(double);
+  if (set_dyn_smem((const void*)chol_diag_kernel, dsm) != cudaSuccess)
+    return -1;
+  int nl = 0;
+  auto ok = [&](int r) {
+    if (r < 0) return false;
+    nl += r;
+    return true;
+  };
+  chol_lambda_kernel<<<H, 256, 0, st>>>(A, n, ridge, tdiv, W.lam, stt);
+  ++nl;
+  for (int k = 0; k < nblk; ++k) {
+    const int k0 = k * NB, kb = std::min(NB, n - k0), m = n - k0 - kb;
+    chol_diag_kernel<<<H, kCT, dsm, st>>>(A, Linv, n, k, W.lam, stt);
+    ++nl;
+    // Linv_kk rows (K = kb)
+    if (!ok(launch_slice_rows(S, Linv + (long long)k * NB * NB, kb, kb, NB, lb, H, W.sB, W.eB, st))) return -1;
+    double* panel = A + (long long)(k0 + kb) * n + k0;
+    if (m > 0) {
+      // L_ik = A_ik Linv_kk^T, written over A_ik
+      if (!ok(launch_slice_rows(S, panel, m, kb, n, nn, H, W.sA, W.eA, st))) return -1;
+      if (!ok(launch_sliced_f64(S, W.sA, W.eA, m, W.sB, W.eB, kb, kb, H, panel, nn, n, false, false, stt, st)))
+        return -1;
+      // A_ij -= L_ik L_jk^T on the trailing lower triangle
+      if (!ok(launch_slice_rows(S, panel, m, kb, n, nn, H, W.sA, W.eA, st))) return -1;
+      if (!ok(launch_sliced_f64(S, W.sA, W.eA, m, W.sA, W.eA, m, kb, H, A + (long long)(k0 + kb) * n + k0 + kb, nn,
+                                n, true, true, stt, st)))
+        return -1;
+    }
+    if (nrhs == 1) continue;   // one right-hand side: substituted after the factorisation (below)
+    // Y_k = Linv_kk B_k over B_k; B_i -= L_ik Y_k
+    double* Bk = B + (long long)k0 * nrhs;
+    if (!ok(launch_slice_cols(S, Bk, kb, nrhs, nrhs, nr, H, W.sC, W.eC, st))) return -1;
+    if (!ok(launch_sliced_f64(S, W.sB, W.eB, kb, W.sC, W.eC, nrhs, kb, H, Bk, nr, nrhs, false, false, stt, st)))
+      return -1;
+    if (m > 0) {
+      if (!ok(launch_slice_cols(S, Bk, kb, nrhs, nrhs, nr, H, W.sC, W.eC, st))) return -1;
+      if (!ok(launch_sliced_f64(S, W.sA, W.eA, m, W.sC, W.eC, nrhs, kb, H, Bk + (long long)kb * nrhs, nr, nrhs, false,
+                                true, stt, st)))
+        return -1;
+    }
+  }
+  if (nrhs == 1) {
+    // one right-hand side: both substitutions by one CTA per head (fp64 SIMT,
+    // n^2 multiply-adds), the forward result left in W.Z
+    cudaMemsetAsync(X, 0, sizeof(double) * (size_t)H * n, st);
+    tri_solve_kernel<double><<<H, 512, 0, st>>>(A, Linv, B, W.Z, X, n);
+    return nl + 1;
+  }
+  for (int k = nblk - 1; k >= 0; --k) {
+    const int k0 = k * NB, kb = std::min(NB, n - k0), m = n - k0 - kb;
+    if (m > 0) {
+      // Z_k = sum_{i>k} L_ik^T X_i: the columns of the panel against the columns of X below block k
+      const double* panel = A + (long long)(k0 + kb) * n + k0;
+      if (!ok(launch_slice_cols(S, panel, m, kb, n, nn, H, W.sA, W.eA, st))) return -1;
+      if (!ok(launch_slice_cols(S, X + (long long)(k0 + kb) * nrhs, m, nrhs, nrhs, nr, H, W.sC, W.eC, st))) return -1;
+      if (!ok(launch_sliced_f64(S, W.sA, W.eA, kb, W.sC, W.eC, nrhs, m, H, W.Z, (long long)NB * nrhs, nrhs, false,
+                                false, stt, st)))
+        return -1;
+    }
+    chol_back_block_kernel<<<dim3(H, cdiv(nrhs, 32)), 256, 0, st>>>(Linv, B, W.Z, X, n, k, nrhs, m > 0 ? 1 : 0);
+    ++nl;
+  }
+  return nl;
+}
+
 // Dual (push-through) form of both ridge fits for t > n, where the primal
 // t x t normal matrices have rank <= n:
 //   (Phi^T Phi + lam I) w = Phi^T m   <=>   w = Phi^T a,  (Phi Phi^T + lam I) a = m
@@ -1266,10 +1447,17 @@ static int fits_dual(const Dims& D, float ridge_w, float ridge_v, float eps_w, f
   int r = gram(4);
   if (r < 0) return -1;
   nl += r;
+  const CholSlicedBufs CW{B.Sl, B.Sl2, B.Sl3, B.eR, B.eC, B.eC2, B.cl_lam, B.Z64};
+  auto solve = [&](int nrhs, long long nrow, float ridge) -> int {
+    if (sliced) return chol_solve_sliced(D.H, D.n, B.G64, B.L64, B.B64, B.X64, nrhs, ridge, D.t, CW, stt, st);
+    return cholesky_solve<double>(D.H, D.n, B.G64, B.L64, B.B64, B.Z64, B.X64, nrhs, nrhs, nrow, ridge, stt, st, D.t);
+  };
   mark(8);
   widen_kernel<<<cdiv((long long)D.H * D.n, 256), 256, 0, st>>>(m, B.B64, (long long)D.H * D.n);
-  nl += 1 + cholesky_solve<double>(D.H, D.n, B.G64, B.L64, B.B64, B.Z64, B.X64, 1, 1, D.n, ridge_w, stt, st, D.t);
-  xty64_kernel<<<dim3(cdiv(D.t, 64), 1, D.H), 256, 0, st>>>(B.Phi, B.X64, B.rhs, D.n, D.t, 1);   // w = Phi^T a
+  r = solve(1, D.n, ridge_w);
+  if (r < 0) return -1;
+  nl += 1 + r;
+  phi_t_vec_kernel<<<dim3(cdiv(D.t, 256), D.H), 256, 0, st>>>(B.Phi, B.X64, B.rhs, D.n, D.t);   // w = Phi^T a
   const long long ht = (long long)D.H * D.t;
   beta_kernel<<<cdiv(ht, 256), 256, 0, st>>>(B.rhs, beta, ht, eps_w, b_min, b_max);
   softmax_bias_kernel<<<dim3(cdiv(D.n, 8), D.H), 256, 0, st>>>(B.LC, beta, B.Phi, D.n, D.t);
@@ -1281,7 +1469,9 @@ static int fits_dual(const Dims& D, float ridge_w, float ridge_v, float eps_w, f
   nl += r;
   mark(10);
   widen_kernel<<<cdiv((long long)D.H * nd, 256), 256, 0, st>>>(Y, B.B64, (long long)D.H * nd);
-  nl += 1 + cholesky_solve<double>(D.H, D.n, B.G64, B.L64, B.B64, B.Z64, B.X64, D.d, D.d, nd, ridge_v, stt, st, D.t);
+  r = solve(D.d, nd, ridge_v);
+  if (r < 0) return -1;
+  nl += 1 + r;
   if (!sliced) {
     xty64_kernel<<<dim3(cdiv(D.t, 64), cdiv(D.d, 32), D.H), 256, 0, st>>>(B.Phi, B.X64, C_v, D.n, D.t, D.d);
     return nl + 1;
@@ -1366,38 +1556,48 @@ __global__ void __launch_bounds__(256) ir_cols_kernel(const float* __restrict__ 
 // x += (L L^T)^-1 r for one head per CTA (512 threads): forward substitution
 // y_k = Linv_kk (r_k - sum_{j<k} L_kj y_j), then x_k += Linv_kk^T (y_k -
 // sum_{j>k} L_jk^T d_j).  y and the correction d live in `yd` ([H][t]).
-__global__ void __launch_bounds__(512) ir_solve_kernel(const float* __restrict__ A, const float* __restrict__ Linv,
-                                                       const float* __restrict__ r, float* __restrict__ yd,
-                                                       float* __restrict__ x, int t) {
+// Also the single-right-hand-side solve of the fp64 dual beta system (x = 0).
+template <typename R>
+__global__ void __launch_bounds__(512) tri_solve_kernel(const R* __restrict__ A, const R* __restrict__ Linv,
+                                                        const R* __restrict__ r, R* __restrict__ yd,
+                                                        R* __restrict__ x, int t) {
   constexpr int NBk = kCholNB;
-  __shared__ float v[NBk];
-  __shared__ float part[8][NBk];
+  __shared__ R v[NBk];
+  __shared__ R part[8][NBk];
   const int b = blockIdx.x, tid = threadIdx.x;
   const int nblk = (t + NBk - 1) / NBk;
-  const float* Ab = A + (long long)b * t * t;
-  const float* Lb = Linv + (long long)b * nblk * NBk * NBk;
-  const float* rb = r + (long long)b * t;
-  float* y = yd + (long long)b * t;
-  float* xb = x + (long long)b * t;
+  const R* Ab = A + (long long)b * t * t;
+  const R* Lb = Linv + (long long)b * nblk * NBk * NBk;
+  const R* rb = r + (long long)b * t;
+  R* y = yd + (long long)b * t;
+  R* xb = x + (long long)b * t;
   // forward: 8 threads per row of block k sum L_kj y_j over the columns before k0
   for (int k = 0; k < nblk; ++k) {
     const int k0 = k * NBk, kb = min(NBk, t - k0);
     {
       const int rr = tid >> 3, pt = tid & 7;
-      float a = 0.f;
-      if (rr < kb)
-        for (int c = pt; c < k0; c += 8) a = fmaf(__ldcg(Ab + (long long)(k0 + rr) * t + c), __ldcg(y + c), a);
+      R a = R(0), a2 = R(0);
+      if (rr < kb) {
+        const R* row = Ab + (long long)(k0 + rr) * t;
+        int c = pt;
+        for (; c + 8 < k0; c += 16) {   // two independent chains: loads in flight together
+          a = fma_r(__ldcg(row + c), __ldcg(y + c), a);
+          a2 = fma_r(__ldcg(row + c + 8), __ldcg(y + c + 8), a2);
+        }
+        if (c < k0) a = fma_r(__ldcg(row + c), __ldcg(y + c), a);
+      }
+      a += a2;
       a += __shfl_xor_sync(0xffffffffu, a, 1);
       a += __shfl_xor_sync(0xffffffffu, a, 2);
       a += __shfl_xor_sync(0xffffffffu, a, 4);
-      if (pt == 0) v[rr] = rr < kb ? rb[k0 + rr] - a : 0.f;
+      if (pt == 0) v[rr] = rr < kb ? rb[k0 + rr] - a : R(0);
     }
     __syncthreads();
     {  // y_k[c] = sum_{l <= c} Linv_k[c][l] v[l]
       const int c = tid >> 3, pt = tid & 7;
-      const float* Li = Lb + (long long)k * NBk * NBk + c * NBk;
-      float a = 0.f;
-      for (int l = pt; l <= c; l += 8) a = fmaf(__ldcg(Li + l), v[l], a);
+      const R* Li = Lb + (long long)k * NBk * NBk + c * NBk;
+      R a = R(0);
+      for (int l = pt; l <= c; l += 8) a = fma_r(__ldcg(Li + l), v[l], a);
       a += __shfl_xor_sync(0xffffffffu, a, 1);
       a += __shfl_xor_sync(0xffffffffu, a, 2);
       a += __shfl_xor_sync(0xffffffffu, a, 4);
@@ -1412,24 +1612,30 @@ __global__ void __launch_bounds__(512) ir_solve_kernel(const float* __restrict__
     const int k0 = k * NBk, kb = min(NBk, t - k0);
     {
       const int c = tid & (NBk - 1), pt = tid >> 6;
-      float a = 0.f;
-      if (c < kb)
-        for (int rr = k0 + kb + pt; rr < t; rr += 8) a = fmaf(__ldcg(Ab + (long long)rr * t + k0 + c), __ldcg(y + rr), a);
-      part[pt][c] = a;
+      R a = R(0), a2 = R(0);
+      if (c < kb) {
+        int rr = k0 + kb + pt;
+        for (; rr + 8 < t; rr += 16) {
+          a = fma_r(__ldcg(Ab + (long long)rr * t + k0 + c), __ldcg(y + rr), a);
+          a2 = fma_r(__ldcg(Ab + (long long)(rr + 8) * t + k0 + c), __ldcg(y + rr + 8), a2);
+        }
+        if (rr < t) a = fma_r(__ldcg(Ab + (long long)rr * t + k0 + c), __ldcg(y + rr), a);
+      }
+      part[pt][c] = a + a2;
     }
     __syncthreads();
     if (tid < NBk) {
-      float a = 0.f;
+      R a = R(0);
 #pragma unroll
       for (int q = 0; q < 8; ++q) a += part[q][tid];
-      v[tid] = tid < kb ? y[k0 + tid] - a : 0.f;
+      v[tid] = tid < kb ? y[k0 + tid] - a : R(0);
     }
     __syncthreads();
     {  // d_k[c] = sum_{l >= c} Linv_k[l][c] v[l]
       const int c = tid >> 3, pt = tid & 7;
-      const float* Li = Lb + (long long)k * NBk * NBk;
-      float a = 0.f;
-      for (int l = c + pt; l < NBk; l += 8) a = fmaf(__ldcg(Li + (long long)l * NBk + c), v[l], a);
+      const R* Li = Lb + (long long)k * NBk * NBk;
+      R a = R(0);
+      for (int l = c + pt; l < NBk; l += 8) a = fma_r(__ldcg(Li + (long long)l * NBk + c), v[l], a);
       a += __shfl_xor_sync(0xffffffffu, a, 1);
       a += __shfl_xor_sync(0xffffffffu, a, 2);
       a += __shfl_xor_sync(0xffffffffu, a, 4);
@@ -1456,7 +1662,7 @@ static int refine_beta(const Dims& D, float ridge_w, const float* m, const FitBu
       ++nl;
     }
     ir_cols_kernel<<<dim3(cdiv(D.t, 256), D.H), 256, 0, st>>>(B.Phi, B.ir_u, B.wsol, B.ir_lam, B.rhs, D.n, D.t);
-    ir_solve_kernel<<<D.H, 512, 0, st>>>(B.Gram, B.Linv, B.rhs, B.Z, B.wsol, D.t);
+    tri_solve_kernel<float><<<D.H, 512, 0, st>>>(B.Gram, B.Linv, B.rhs, B.Z, B.wsol, D.t);
     nl += 2;
   }
   return nl;

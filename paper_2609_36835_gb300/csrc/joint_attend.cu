@@ -658,7 +658,7 @@ int launch_attend_joint(int H, int n, int t, int F, float scale, const bf16* Q, 
   const dim3 grid(s.nsplit, cdiv(n, kJR), H);
   if (compact_bf16 || t == 0) {
     const int smem = 2 * kBStages * kBTileBytes;
-    cudaFuncSetAttribute(attend_bulk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    set_dyn_smem((const void*)attend_bulk_kernel, smem);
     attend_bulk_kernel<<<grid, kJThreads, smem, st>>>(Q, n, (const bf16*)Ck, beta, (const bf16*)Cv, t, Kf, Vf, F,
                                                       scale, s.per_split, s.nsplit, Opart, ml, stt);
   } else

@@ -38,6 +38,9 @@ constexpr int kSplitK = 8;   // K slices of the skinny (N = 128) long-K products
 
 // Streaming multiprocessors of the current device (queried once per device).
 int tc_gemm_sm_count();
+// cudaFuncSetAttribute(kern, MaxDynamicSharedMemorySize, bytes), issued once
+// per kernel and device (later calls with no larger size return at once).
+cudaError_t set_dyn_smem(const void* kern, int bytes);
 // Grid of a grid-stride kernel: enough CTAs for `count` elements at `per_cta`
 // each, capped at `per_sm` resident CTAs on every SM of the device.
 inline int stride_grid(long long count, int per_cta, int per_sm) {
@@ -133,6 +136,9 @@ struct FitBufs {
   bf16 *Sl, *Sl2;                       // sliced operands of the dual fits (t > n only)
   int *eR, *eC;                         // their row exponents ([H][max(n, t)], [H][128])
   double *ir_u, *ir_sq, *ir_lam;        // refinement of the beta system: [H][n], [H][n], [H]
+  bf16* Sl3;                            // right-hand-side slices of the dual solves (t > n only)
+  int* eC2;
+  double* cl_lam;                       // [H]
 };
 // Returns launches, or -1 when a TMA descriptor cannot be encoded.
 // ev (nullable): events recorded before the beta solve, before the value
@@ -144,7 +150,7 @@ int launch_fits(const Dims& D, float scale, float ridge_w, float ridge_v, float 
 int launch_check_finite(const float* x, long long count, DevStatus* stt, cudaStream_t st);
 
 // ---- fp64-grade products on the bf16 tensor pipe (tc_sliced.cu) ------------
-// Operands are cut into S bf16 slices per row (S = 3 or 4) with a power-of-two
+// Operands are cut into S bf16 slices per row (S = 3, 4 or 5) with a power-of-two
 // row scale; products of the sliced operands are exact up to ~2^-48 and
 // returned in fp64 (or rounded to fp32).  K up to kSlicedMaxK.
 constexpr int kSlicedMaxK = 26214;
@@ -154,11 +160,17 @@ size_t sliced_ld(int K);   // row pitch (elements) of a sliced operand with K co
 // X [H][R][K] (rows ldx apart, batches xbs apart) -> slices [S][H][R][sliced_ld(K)], exponents ex [H][R]
 int launch_slice_rows(int S, const float* X, int R, int K, int ldx, long long xbs, int H, bf16* out, int* ex,
                       cudaStream_t st);
+int launch_slice_rows(int S, const double* X, int R, int K, int ldx, long long xbs, int H, bf16* out, int* ex,
+                      cudaStream_t st);
 // the rows of X^T for X [H][K][R] (R contiguous): slices [S][H][R][sliced_ld(K)], exponents ex [H][R]
 int launch_slice_cols(int S, const float* X, int K, int R, int ldx, long long xbs, int H, bf16* out, int* ex,
                       cudaStream_t st);
 int launch_slice_cols(int S, const double* X, int K, int R, int ldx, long long xbs, int H, bf16* out, int* ex,
                       cudaStream_t st);
+// C[b] (M x N, fp64, rows ldc apart, batches cbs apart) = A B^T, or C -= A B^T
+// with `sub`; with `lower` only the tiles that reach C's lower triangle (M = N)
+int launch_sliced_f64(int S, const bf16* As, const int* eA, int M, const bf16* Bs, const int* eB, int N, int K, int H,
+                      double* C, long long cbs, int ldc, bool lower, bool sub, DevStatus* stt, cudaStream_t st);
 // G[b] = X X^T (R x R, fp64) on the tiles that reach the lower triangle
 int launch_sliced_gram_lower(int S, const bf16* Xs, const int* ex, int R, int K, int H, double* G, DevStatus* stt,
                              cudaStream_t st);

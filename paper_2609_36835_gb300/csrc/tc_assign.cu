@@ -279,7 +279,7 @@ static int launch_col_profiles_tma(const Dims& D, const float* L, float* logphi,
   CUtensorMap m;
   if (!encode_f32_map_3d(&m, L, D.T, D.n, D.H, W, 256)) return -1;
   const int smem = nbox * 256 * W * 4 + 128;
-  if (cudaFuncSetAttribute(col_profiles_tma_kernel<W>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+  if (set_dyn_smem((const void*)col_profiles_tma_kernel<W>, smem) !=
       cudaSuccess)
     return -1;
   col_profiles_tma_kernel<W><<<dim3(cdiv(D.T, W), D.H), 512, smem, st>>>(m, logphi, Ut_hi, Ut_lo, D.n, D.T, ldn, nbox,
@@ -300,7 +300,7 @@ int launch_col_profiles(const Dims& D, const float* L, float* logphi, bf16* Ut_h
   // each CTA re-reads its n x 32 strip from L2: with n > 1024 a shared-memory
   // reservation keeps at most two CTAs per SM so the live strips fit in L2
   const int smem = D.n > 1024 ? 80 * 1024 : 0;
-  if (smem > 0 && cudaFuncSetAttribute(col_profiles_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+  if (smem > 0 && set_dyn_smem((const void*)col_profiles_kernel, smem) !=
                       cudaSuccess)
     return -1;
   col_profiles_kernel<<<dim3(cdiv(D.T, 32), D.H), 512, smem, st>>>(L, logphi, Ut_hi, Ut_lo, D.n, D.T, ldn);

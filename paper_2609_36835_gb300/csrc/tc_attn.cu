@@ -309,7 +309,7 @@ static int launch_probs_v_fused(const Dims& D, const float* X, const float* shif
   const int tiles = D.H * cdiv(D.n, 128), nk = cdiv(D.T, 64);
   const int splits = (2 * tiles <= tc_gemm_sm_count() && nk >= 2) ? 2 : 1;
   auto kern = skip ? probs_v_kernel<true> : probs_v_kernel<false>;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kPvSmem) != cudaSuccess) return -1;
+  if (set_dyn_smem((const void*)kern, kPvSmem) != cudaSuccess) return -1;
   if (splits > 1 && cudaMemsetAsync(out, 0, sizeof(float) * (size_t)D.H * D.n * 128, st) != cudaSuccess) return -1;
   kern<<<tiles * splits, kPvThreads, kPvSmem, st>>>(mX, mVT, shift, mul, skip, out, D.n, D.T, splits, stt);
   return cudaGetLastError() == cudaSuccess ? 1 : -1;

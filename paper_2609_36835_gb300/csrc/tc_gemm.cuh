@@ -307,6 +307,7 @@ __global__ void __launch_bounds__(64 + 32 * EpiWarps<Epi>::value, 1)
 // Resident CTAs of the persistent GEMM: one per SM (the stage ring takes most
 // of the shared memory), looked up once per device.
 int tc_gemm_sm_count();
+cudaError_t set_dyn_smem(const void* kern, int bytes);
 
 // Host: launch over H batches; maps are built by the caller (encode_bf16_map_3d,
 // box rows 128 for A and BN for B).
@@ -319,7 +320,7 @@ inline cudaError_t launch_tc_gemm(const CUtensorMap& mA, const CUtensorMap& mB, 
   constexpr int smem = C::SMEM + NE * EpiStage<Epi>::bytes;
   static_assert(smem <= 227 * 1024, "stage ring and epilogue staging exceed shared memory");
   auto kern = tc_gemm_kernel<BN, MODE, Epi>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e = set_dyn_smem((const void*)kern, smem);
   if (e != cudaSuccess) return e;
   const long long ntiles = (long long)cdiv(N, BN) * cdiv(M, 128) * H;
   const int grid = (int)std::min<long long>(ntiles, tc_gemm_sm_count());

@@ -1,7 +1,9 @@
 // Host side of the tensor-core kernels: TMA tensor-map encoding through the
 // driver entry point (no link-time dependency on libcuda).
 #include <cudaTypedefs.h>
+#include <map>
 #include <mutex>
+#include <utility>
 
 #include "tc.cuh"
 
@@ -70,6 +72,19 @@ bool encode_f32_map_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint64
                               swz128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+cudaError_t set_dyn_smem(const void* kern, int bytes) {
+  static std::mutex mu;
+  static std::map<std::pair<const void*, int>, int> done;   // (kernel, device) -> bytes already allowed
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) dev = -1;
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = done.find({kern, dev});
+  if (it != done.end() && it->second >= bytes) return cudaSuccess;
+  const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) done[{kern, dev}] = bytes;
+  return e;
 }
 
 int tc_gemm_sm_count() {

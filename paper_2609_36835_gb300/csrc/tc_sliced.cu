@@ -57,6 +57,7 @@ struct SlOutF64 {
   double* C;
   long long cbs;
   int ldc;
+  int sub;   // 0: C = A B^T; 1: C -= A B^T
   template <class F>
   __device__ __forceinline__ void put(int b, int row, int c0, int M, int N, F&& val) const {
     if (row >= M) return;
@@ -65,12 +66,17 @@ struct SlOutF64 {
 #pragma unroll
       for (int q = 0; q < 16; q += 2) {
         const double x0 = val(q), x1 = val(q + 1);
-        *(double2*)(d + q) = make_double2(x0, x1);
+        if (sub) {
+          const double2 o = *(const double2*)(d + q);
+          *(double2*)(d + q) = make_double2(o.x - x0, o.y - x1);
+        } else {
+          *(double2*)(d + q) = make_double2(x0, x1);
+        }
       }
     } else {
 #pragma unroll
       for (int q = 0; q < 16; ++q)
-        if (c0 + q < N) d[q] = val(q);
+        if (c0 + q < N) d[q] = sub ? d[q] - val(q) : val(q);
     }
   }
 };
@@ -313,8 +319,8 @@ __global__ void __launch_bounds__(kSlThreads, 1)
           const double t = (double)acc[p2 * 16 + e] * 0x1p-32 + (double)v5[p2][e];   // |acc| < 2^53: exact
           // 2^(er + ec) built from its bits (row and column exponents of finite
           // fp32 / fp64 data stay well inside the normal range)
-          const long long ex2 = 1023 + er + ecol[c0 + e];   // only evaluated for columns below N
-          return t * __longlong_as_double(ex2 << 52);
+          const int ex = er + ecol[c0 + e];   // only evaluated for columns below N
+          return (ex > -1023 && ex < 1024) ? t * __longlong_as_double((long long)(1023 + ex) << 52) : ldexp(t, ex);
         });
       }
     }
@@ -384,15 +390,24 @@ __global__ void __launch_bounds__(256) slice_rows_kernel(const T* __restrict__ X
 }
 
 // Column maxima exponents of X [H][K][R] (R contiguous, rows ldx apart): ex [H][R].
+// A CTA takes 32 columns (lane = column, coalesced rows); its 8 warps split
+// the rows and meet in shared memory.
 template <typename T>
 __global__ void __launch_bounds__(256) col_exp_kernel(const T* __restrict__ X, int K, int R, int ldx, long long xbs,
                                                       int* __restrict__ ex) {
-  const int b = blockIdx.y, r = blockIdx.x * 256 + threadIdx.x;
-  if (r >= R) return;
+  __shared__ T part[8][32];
+  const int b = blockIdx.y, lane = threadIdx.x & 31, warp = threadIdx.x >> 5, r = blockIdx.x * 32 + lane;
   const T* x = X + (long long)b * xbs + r;
   T mx = T(0);
-  for (int k = 0; k < K; ++k) mx = fmax(mx, fabs(x[(long long)k * ldx]));
-  ex[(long long)b * R + r] = bound_exp(mx);
+  if (r < R)
+    for (int k = warp; k < K; k += 8) mx = fmax(mx, fabs(x[(long long)k * ldx]));
+  part[warp][lane] = mx;
+  __syncthreads();
+  if (warp == 0 && r < R) {
+#pragma unroll
+    for (int w = 1; w < 8; ++w) mx = fmax(mx, part[w][lane]);
+    ex[(long long)b * R + r] = bound_exp(mx);
+  }
 }
 
 // Column-sliced operand (the rows of X^T): X [H][K][R] -> slices
@@ -437,7 +452,7 @@ int launch_sliced(const bf16* As, const int* eA, int M, const bf16* Bs, const in
   }
   using C = SlCfg<S>;
   auto kern = sliced_gemm_kernel<S, Out>;
-  const cudaError_t ea = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  const cudaError_t ea = set_dyn_smem((const void*)kern, C::SMEM);
   if (ea != cudaSuccess) {
     g_sliced_fail = 100 + (int)ea;
     return -1;
@@ -464,28 +479,43 @@ int sliced_last_failure() { return g_sliced_fail; }
 
 bool sliced_supported(int K) { return K >= 1 && K <= kSlicedMaxK; }
 
-int launch_slice_rows(int S, const float* X, int R, int K, int ldx, long long xbs, int H, bf16* out, int* ex,
-                      cudaStream_t st) {
+template <typename T>
+static int slice_rows_t(int S, const T* X, int R, int K, int ldx, long long xbs, int H, bf16* out, int* ex,
+                        cudaStream_t st) {
   const int grid = cdiv((long long)H * R, 8), ldo = (int)sliced_ld(K);
   if (S == 3)
-    slice_rows_kernel<3, float><<<grid, 256, 0, st>>>(X, R, K, ldx, xbs, H, out, ldo, ex);
+    slice_rows_kernel<3, T><<<grid, 256, 0, st>>>(X, R, K, ldx, xbs, H, out, ldo, ex);
   else if (S == 4)
-    slice_rows_kernel<4, float><<<grid, 256, 0, st>>>(X, R, K, ldx, xbs, H, out, ldo, ex);
+    slice_rows_kernel<4, T><<<grid, 256, 0, st>>>(X, R, K, ldx, xbs, H, out, ldo, ex);
+  else if (S == 5)
+    slice_rows_kernel<5, T><<<grid, 256, 0, st>>>(X, R, K, ldx, xbs, H, out, ldo, ex);
   else
     return -1;
   return 1;
+}
+
+int launch_slice_rows(int S, const float* X, int R, int K, int ldx, long long xbs, int H, bf16* out, int* ex,
+                      cudaStream_t st) {
+  return slice_rows_t<float>(S, X, R, K, ldx, xbs, H, out, ex, st);
+}
+
+int launch_slice_rows(int S, const double* X, int R, int K, int ldx, long long xbs, int H, bf16* out, int* ex,
+                      cudaStream_t st) {
+  return slice_rows_t<double>(S, X, R, K, ldx, xbs, H, out, ex, st);
 }
 
 template <typename T>
 static int slice_cols_t(int S, const T* X, int K, int R, int ldx, long long xbs, int H, bf16* out, int* ex,
                         cudaStream_t st) {
   const int ldo = (int)sliced_ld(K);
-  col_exp_kernel<T><<<dim3(cdiv(R, 256), H), 256, 0, st>>>(X, K, R, ldx, xbs, ex);
+  col_exp_kernel<T><<<dim3(cdiv(R, 32), H), 256, 0, st>>>(X, K, R, ldx, xbs, ex);
   const dim3 grid(cdiv(R, 32), cdiv(K, 32), H);
   if (S == 3)
     slice_cols_kernel<3, T><<<grid, 256, 0, st>>>(X, K, R, ldx, xbs, H, ex, out, ldo);
   else if (S == 4)
     slice_cols_kernel<4, T><<<grid, 256, 0, st>>>(X, K, R, ldx, xbs, H, ex, out, ldo);
+  else if (S == 5)
+    slice_cols_kernel<5, T><<<grid, 256, 0, st>>>(X, K, R, ldx, xbs, H, ex, out, ldo);
   else
     return -1;
   return 2;
@@ -503,10 +533,16 @@ int launch_slice_cols(int S, const double* X, int K, int R, int ldx, long long x
 
 int launch_sliced_gram_lower(int S, const bf16* Xs, const int* ex, int R, int K, int H, double* G, DevStatus* stt,
                              cudaStream_t st) {
+  return launch_sliced_f64(S, Xs, ex, R, Xs, ex, R, K, H, G, (long long)R * R, R, true, false, stt, st);
+}
+
+int launch_sliced_f64(int S, const bf16* As, const int* eA, int M, const bf16* Bs, const int* eB, int N, int K, int H,
+                      double* C, long long cbs, int ldc, bool lower, bool sub, DevStatus* stt, cudaStream_t st) {
   const int ldk = (int)sliced_ld(K);
-  const SlOutF64 out{G, (long long)R * R, R};
-  if (S == 3) return launch_sliced<3>(Xs, ex, R, Xs, ex, R, K, ldk, H, true, out, stt, st);
-  if (S == 4) return launch_sliced<4>(Xs, ex, R, Xs, ex, R, K, ldk, H, true, out, stt, st);
+  const SlOutF64 out{C, cbs, ldc, sub ? 1 : 0};
+  if (S == 3) return launch_sliced<3>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st);
+  if (S == 4) return launch_sliced<4>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st);
+  if (S == 5) return launch_sliced<5>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st);
   return -1;
 }
 
