@@ -5,6 +5,8 @@
 
 #include <algorithm>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "kernels.h"
 #include "tc.cuh"
 
@@ -252,9 +254,27 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
   const bf16* Vb = (const bf16*)V;
   const bf16* Qb = (const bf16*)Q_ref;
   cudaEvent_t const* ev = (aux && aux->stage_events) ? (cudaEvent_t const*)aux->stage_events : nullptr;
+  // stage boundaries: the caller's CUDA events, and one NVTX range per stage
+  // (host-side enqueue spans, visible to Nsight; no cost without a tool attached)
+  // (stages 7-10, whose boundaries lie inside launch_fits, share one range)
+  static const char* const kStageNames[8] = {
+      "arckv.indexer_features", "arckv.index_logits", "arckv.pool_top_t", "arckv.reference_attention",
+      "arckv.column_profiles", "arckv.assignment", "arckv.merge", "arckv.fits"};
+  int open_stage = -1;
   auto mark = [&](int s) {
     if (ev) cudaEventRecord(ev[s], st);
+    if (open_stage >= 0) nvtxRangePop();
+    open_stage = s < 8 ? s : -1;
+    if (open_stage >= 0) nvtxRangePushA(kStageNames[s]);
   };
+  nvtxRangePushA("arckv_compact");
+  struct RangeGuard {
+    int* open;
+    ~RangeGuard() {
+      if (*open >= 0) nvtxRangePop();
+      nvtxRangePop();
+    }
+  } guard{&open_stage};
   int nl = 0;
 
   cudaGetLastError();  // clear a stale error from earlier, unrelated work
@@ -383,9 +403,9 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
 
 size_t arckv_attend_workspace_bytes(int32_t H_kv, int32_t n, int32_t t, int32_t d) {
   if (H_kv < 1 || n < 1 || t < 1 || d != 128) return 0;
-  if ((long long)n * t >= (1LL << 31) || (long long)H_kv * kSplitK > 65535) return 0;
-  const size_t H = H_kv;
-  return up(sizeof(DevStatus)) + up(H * n * t * 4) + up((size_t)kSplitK * H * n * 128 * 4);
+  if ((long long)n * t >= (1LL << 31) || (long long)H_kv * n >= (1LL << 31) || (long long)H_kv * t * 128 >= (1LL << 31))
+    return 0;
+  return attend_layout(H_kv, n, t).total;
 }
 
 arckv_status arckv_attend(int32_t H_kv, int32_t n, int32_t t, int32_t d, float logit_scale, const void* Q,
@@ -401,12 +421,10 @@ arckv_status arckv_attend(int32_t H_kv, int32_t n, int32_t t, int32_t d, float l
   cudaStream_t st = (cudaStream_t)stream;
   char* w = (char*)ws;
   DevStatus* stt = (DevStatus*)w;
-  float* LC = (float*)(w + up(sizeof(DevStatus)));
-  float* split = (float*)(w + up(sizeof(DevStatus)) + up((size_t)H_kv * n * t * 4));
   const float scale = logit_scale > 0.f ? logit_scale : 1.0f / sqrtf((float)d);
   cudaGetLastError();
   if (cudaMemsetAsync(stt, 0, sizeof(DevStatus), st) != cudaSuccess) return ARCKV_ERR_CUDA;
-  launch_attend(H_kv, n, t, scale, (const bf16*)Q, C_k, beta, C_v, O, LC, split, st);
+  if (launch_attend(H_kv, n, t, scale, (const bf16*)Q, C_k, beta, C_v, O, w, stt, st) < 0) return ARCKV_ERR_CUDA;
   launch_check_finite(O, (long long)H_kv * n * d, stt, st);
   if (cudaGetLastError() != cudaSuccess) return ARCKV_ERR_CUDA;
   if (flags & ARCKV_FLAG_NONBLOCKING) return ARCKV_OK;

@@ -11,7 +11,8 @@
 
 namespace {
 
-// status word (256 bytes) + compact logits + split-K partials, in floats
+// the scratch layout of arckv_attend (attend_layout: status word, logits,
+// operand triples, partial outputs), in floats
 constexpr size_t kStaticScratchFloats = ARCKV_ATTEND_STATIC_MAX_FLOATS;
 
 __device__ __align__(256) float g_attend_scratch[kStaticScratchFloats];
@@ -74,8 +75,8 @@ extern "C" {
 
 size_t arckv_attend_static_floats(int32_t H_kv, int32_t n, int32_t t, int32_t d) {
   if (H_kv < 1 || n < 1 || t < 1 || d != 128) return 0;
-  const size_t splits = (size_t)std::max(1, std::min(arckv::kSplitK, (t + 127) / 128));
-  return 64 + ((size_t)H_kv * n * t + 63) / 64 * 64 + splits * H_kv * n * 128;
+  const size_t bytes = arckv_attend_workspace_bytes(H_kv, n, t, d);   // the workspace layout of arckv_attend
+  return bytes == 0 ? 0 : (bytes + 3) / 4;
 }
 
 arckv_status arckv_attend_static(int32_t H_kv, int32_t n, int32_t t, int32_t d, float logit_scale, const void* Q,
@@ -91,13 +92,13 @@ arckv_status arckv_attend_static(int32_t H_kv, int32_t n, int32_t t, int32_t d, 
   if (s != ARCKV_OK) return s;
   cudaStream_t st = (cudaStream_t)stream;
   arckv::DevStatus* stt = (arckv::DevStatus*)base;
-  float* LC = base + 64;
-  float* split = LC + ((size_t)H_kv * n * t + 63) / 64 * 64;
   const float scale = logit_scale > 0.f ? logit_scale : 1.0f / sqrtf((float)d);
   cudaGetLastError();
-  // the array keeps the previous call's contents: the status word must start at zero
+  // the array keeps the previous call's contents: the status word must start at
+  // zero (every other scratch region is written before it is read)
   if (cudaMemsetAsync(stt, 0, sizeof(arckv::DevStatus), st) != cudaSuccess) return ARCKV_ERR_CUDA;
-  arckv::launch_attend(H_kv, n, t, scale, (const arckv::bf16*)Q, C_k, beta, C_v, O, LC, split, st);
+  if (arckv::launch_attend(H_kv, n, t, scale, (const arckv::bf16*)Q, C_k, beta, C_v, O, (char*)base, stt, st) < 0)
+    return ARCKV_ERR_CUDA;
   arckv::launch_check_finite(O, (long long)H_kv * n * d, stt, st);
   if (cudaGetLastError() != cudaSuccess) return ARCKV_ERR_CUDA;
   unsigned int code = 0;

@@ -14,7 +14,6 @@
 #include <cooperative_groups.h>
 #include <type_traits>
 
-#include "gemm.cuh"
 #include "kernels.h"
 #include "tc_gemm.cuh"
 
@@ -1748,18 +1747,104 @@ int launch_check_finite(const float* x, long long count, DevStatus* stt, cudaStr
   return 1;
 }
 
+// ---------------------------------------------------------------------------
+// Compact attention (Sec. 3.1 Eq. compact_attention) on the tensor pipe:
+//   X = scale Q C_k^T + 1 beta^T   (C_k as a bf16 triple against the exact bf16
+//                                   queries; transposed store; beta added with
+//                                   the row statistics)
+//   O = softmax(X) C_v = sum_p softmax(X) C_v,p over the bf16 triple
+//       (h, m, l) of C_v: three fused softmax-V products (fp32-grade
+//       probabilities formed on the fly), added in a fixed order.
+
+// x += beta over each row, then shift = max, mul = 1 / sum exp(x - shift); one
+// warp per row of X [H][n][t].
+__global__ void __launch_bounds__(256) bias_rowstats_kernel(float* X, const float* beta, float* shift, float* mul,
+                                                            int n, int t) {
+  const int b = blockIdx.y, row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= n) return;
+  float* x = X + ((long long)b * n + row) * t;
+  const float* be = beta + (long long)b * t;
+  float mx = -INFINITY;
+  for (int c = lane; c < t; c += 32) {
+    const float v = x[c] + be[c];
+    x[c] = v;
+    mx = fmaxf(mx, v);
+  }
+  mx = warp_max(mx);
+  float sm = 0.f;
+  for (int c = lane; c < t; c += 32) sm += expf(x[c] - mx);
+  sm = warp_sum(sm);
+  if (lane == 0) {
+    shift[(long long)b * n + row] = mx;
+    mul[(long long)b * n + row] = 1.0f / sm;
+  }
+}
+
+// O[e] = P0[e] + P1[e] + P2[e]
+__global__ void sum3_kernel(const float* P, float* O, long long count) {
+  for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < count;
+       k += (long long)gridDim.x * blockDim.x)
+    O[k] = (P[k] + P[count + k]) + P[2 * count + k];
+}
+
+AttendLayout attend_layout(int H, int n, int t) {
+  AttendLayout L{};
+  const size_t h = H, ldt = (size_t)(t + 7) / 8 * 8;
+  size_t o = 0;
+  auto take = [&](size_t bytes) { const size_t r = o; o += (bytes + 255) / 256 * 256; return r; };
+  L.status = take(256);
+  L.X = take(h * n * t * 4);
+  L.shift = take(h * n * 4);
+  L.mul = take(h * n * 4);
+  L.ck3 = take(3 * h * t * 128 * 2);
+  L.vt3 = take(3 * h * 128 * ldt * 2);
+  L.parts = take(3 * h * n * 128 * 4);
+  L.p3 = take(probs_fused(t) ? 0 : 3 * h * n * ldt * 2);
+  L.total = o;
+  return L;
+}
+
 int launch_attend(int H, int n, int t, float scale, const bf16* Q, const float* C_k, const float* beta,
-                  const float* C_v, float* O, float* LC, float* split, cudaStream_t st) {
-  const int d = 128;
-  const long long nd = (long long)n * d, nt = (long long)n * t, td = (long long)t * d;
-  launch_gemm(RowK<bf16>{Q, nd, d}, RowK<float>{C_k, td, d}, EpiStore{LC, nt, 0, t, scale, false}, H, n, t, d, 1,
-              st);
-  softmax_bias_kernel<<<dim3(cdiv(n, 8), H), 256, 0, st>>>(LC, beta, LC, n, t);
-  const int splits = max(1, min(kSplitK, cdiv(t, 128)));
-  launch_gemm(RowK<float>{LC, nt, t}, ColK<float>{C_v, td, d}, EpiStore{split, nd, (long long)H * nd, d, 1.f, false},
-              H, n, d, t, splits, st);
-  launch_split_reduce(H, n, d, splits, split, O, st);
-  return 4;
+                  const float* C_v, float* O, char* ws, DevStatus* stt, cudaStream_t st) {
+  const AttendLayout L = attend_layout(H, n, t);
+  const long long htd = (long long)H * t * 128, ldt = (t + 7) / 8 * 8;
+  float* X = (float*)(ws + L.X);
+  float* shift = (float*)(ws + L.shift);
+  float* mul = (float*)(ws + L.mul);
+  bf16* ck = (bf16*)(ws + L.ck3);
+  bf16* vt = (bf16*)(ws + L.vt3);
+  float* parts = (float*)(ws + L.parts);
+  bf16* p3 = (bf16*)(ws + L.p3);
+  int nl = launch_split3(C_k, ck, ck + htd, ck + 2 * htd, htd, st);
+  {  // X^T = C_k Q^T, stored transposed as X [H][n][t] and scaled
+    CUtensorMap mA, mA2, mA3, mB;
+    if (!encode_bf16_map_3d(&mA, ck, 128, t, H, 128) || !encode_bf16_map_3d(&mA2, ck + htd, 128, t, H, 128) ||
+        !encode_bf16_map_3d(&mA3, ck + 2 * htd, 128, t, H, 128) || !encode_bf16_map_3d(&mB, Q, 128, n, H, 128))
+      return -1;
+    if (launch_tc_gemm<128, kSplit3A>(mA, mB, mA2, mA, TcEpiStoreT{X, (long long)n * t, t, scale}, H, t, n, 128, 128,
+                                      stt, st, 0, &mA3) != cudaSuccess)
+      return -1;
+    ++nl;
+  }
+  bias_rowstats_kernel<<<dim3(cdiv(n, 8), H), 256, 0, st>>>(X, beta, shift, mul, n, t);
+  // C_v^T as a bf16 triple [H][128][ldt] (zero pad)
+  transpose_split3_kernel<<<dim3(cdiv(128, 32), cdiv(ldt, 32), H), 256, 0, st>>>(
+      C_v, t, 128, vt, vt + (long long)H * 128 * ldt, vt + 2LL * H * 128 * ldt, (int)ldt);
+  nl += 2;
+  Dims D{};
+  D.H = H;
+  D.n = n;
+  D.T = t;
+  D.d = 128;
+  const long long hnd = (long long)H * n * 128, pl = (long long)H * n * ldt;
+  for (int p = 0; p < 3; ++p) {
+    const int r = launch_probs_v_tc(D, X, shift, mul, p3, p3 + pl, p3 + 2 * pl, vt + p * (long long)H * 128 * ldt,
+                                    parts + p * hnd, stt, st);
+    if (r < 0) return -1;
+    nl += r;
+  }
+  sum3_kernel<<<stride_grid(hnd, 256, 8), 256, 0, st>>>(parts, O, hnd);
+  return nl + 1;
 }
 
 }  // namespace arckv

@@ -34,7 +34,7 @@ inline int realized_anchors(int T, int t, int chunk_len) {
   return total;
 }
 
-constexpr int kSplitK = 8;   // K slices of the skinny (N = 128) long-K products
+constexpr int kSplitK = 8;   // grid slices per head some launches take (heads x slices ride in one grid dimension)
 
 // Streaming multiprocessors of the current device (queried once per device).
 int tc_gemm_sm_count();
@@ -179,8 +179,16 @@ int launch_sliced_product_f32(int S, const bf16* As, const int* eA, int M, const
                               int H, float* C, int ldc, DevStatus* stt, cudaStream_t st);
 
 // ---- compact attention (Eq. compact_attention) ----------------------------
+// Scratch of launch_attend: byte offsets from one 256-byte aligned base (the
+// first 256 bytes are the status word) and the total size.
+struct AttendLayout {
+  size_t status, X, shift, mul, ck3, vt3, parts, p3, total;
+};
+AttendLayout attend_layout(int H, int n, int t);
+// O [H][n][128] = softmax(scale Q C_k^T + beta) C_v on the tensor pipe; `ws` is
+// the scratch base of attend_layout.  Returns launches or -1.
 int launch_attend(int H, int n, int t, float scale, const bf16* Q, const float* C_k, const float* beta,
-                  const float* C_v, float* O, float* LC, float* split, cudaStream_t st);
+                  const float* C_v, float* O, char* ws, DevStatus* stt, cudaStream_t st);
 
 // ---- HA / VI anchor scores (App. B.1) ----------------------------------
 // E[h] = mean_i ||O_i - O~_i(S)|| / (||O_i|| + eps) (Eq. background_truncated_error);
@@ -216,6 +224,5 @@ int launch_attend_joint(int H, int n, int t, int F, float scale, const bf16* Q, 
 // Shared small kernels.
 int launch_part_stats(int H, int rows, int ntiles, const float2* part, float* shift, float* mul, float* sum,
                       cudaStream_t st);
-int launch_split_reduce(int H, int M, int N, int splits, const float* part, float* out, cudaStream_t st);
 
 }  // namespace arckv

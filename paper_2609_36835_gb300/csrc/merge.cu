@@ -8,7 +8,6 @@
 // which keeps every column representable in fp32 when the logit range
 // exceeds the fp32 exponent range (column statistics and profiles: the
 // col_profiles kernel of the assignment stage).
-#include "gemm.cuh"
 #include "kernels.h"
 
 namespace arckv {

@@ -150,20 +150,5 @@ int launch_part_stats(int H, int rows, int ntiles, const float2* part, float* sh
   return 1;
 }
 
-// out[i] = sum over slices (in slice order) of part[slice][i].
-__global__ void split_reduce_kernel(const float* part, float* out, long long count, int splits) {
-  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < count;
-       i += (long long)gridDim.x * blockDim.x) {
-    float a = 0.f;
-    for (int s = 0; s < splits; ++s) a += part[(long long)s * count + i];
-    out[i] = a;
-  }
-}
-
-int launch_split_reduce(int H, int M, int N, int splits, const float* part, float* out, cudaStream_t st) {
-  const long long count = (long long)H * M * N;
-  split_reduce_kernel<<<stride_grid(count, 256, 16), 256, 0, st>>>(part, out, count, splits);
-  return 1;
-}
 
 }  // namespace arckv

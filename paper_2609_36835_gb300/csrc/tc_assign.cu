@@ -6,6 +6,8 @@
 //     U^T [T x n] against the anchor rows U_S^T [t x n] whose epilogue keeps
 //     the row maximum (lowest r on ties) and merges it across column tiles
 //     with a 64-bit atomicMax; the T x t similarity is never stored.
+#include <algorithm>
+
 #include "kernels.h"
 #include "tc_gemm.cuh"
 
@@ -355,7 +357,13 @@ int launch_assign_gemm(const Dims& D, const int* anchors, const bf16* Ut_hi, con
     return -1;
   TcEpiArgmax epi{best, D.T};
   const int kfull = (ldn + 63) / 64 * 64;
-  if (launch_tc_gemm<128, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.T, D.t, ldn, kfull, stt, st) != cudaSuccess)
+  // anchor tiles in groups whose split profiles (128 rows x ldn x 4 bytes per
+  // tile) take about 40 MB, so each group stays in L2 while the key profiles
+  // stream past it (one pass over them per group instead of one per wave)
+  const long long tile_bytes = 128LL * ldn * 4;
+  const int group = (int)std::max<long long>(1, (40LL << 20) / tile_bytes);
+  if (launch_tc_gemm<128, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.T, D.t, ldn, kfull, stt, st, 0, nullptr, group) !=
+      cudaSuccess)
     return -1;
   const long long cnt = (long long)D.H * D.T;
   decode_assign_kernel2<<<stride_grid(cnt, 256, 8), 256, 0, st>>>(best, kappa, cnt);

@@ -3,7 +3,10 @@
 //   D[b](m, n) = sum_k A[b](m, k) B[b](n, k)      (A, B bf16, K-major, D fp32 in TMEM)
 //
 // Persistent: one CTA per SM walks the 128 x BN output tiles (b, row tile,
-// column tile; columns fastest) in a grid-stride loop.  Warp 0 streams 64-wide K slabs of A and B
+// column tile; columns fastest) in a grid-stride loop.  With col_group > 0
+// the column tiles are taken col_group at a time (b, column group, row tile,
+// column tile in the group), so that the B operand of one group stays in L2
+// while the A rows stream past it once per group.  Warp 0 streams 64-wide K slabs of A and B
 // into a STAGES-deep ring of 128-byte-swizzled shared tiles with TMA; warp 1
 // issues tcgen05.mma (M = 128, N = BN, K = 16) into one of two TMEM
 // accumulators; warps 2..5 drain the accumulator with tcgen05.ld, one TMEM
@@ -96,7 +99,7 @@ __global__ void __launch_bounds__(64 + 32 * EpiWarps<Epi>::value, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
                    const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mB2,
                    const __grid_constant__ CUtensorMap mA3, const __grid_constant__ Epi epi, int H, int M, int N, int K,
-                   int chunk_k, int K1, DevStatus* stt) {
+                   int chunk_k, int K1, DevStatus* stt, int col_group) {
   using C = TcCfg<BN, MODE>;
   constexpr int SB = EpiStage<Epi>::bytes;
   constexpr int NE = EpiWarps<Epi>::value;   // epilogue warps: 4 or 8
@@ -117,11 +120,15 @@ __global__ void __launch_bounds__(64 + 32 * EpiWarps<Epi>::value, 1)
   // persistent: CTA c takes tiles c, c + grid, ...; tile = (b, row tile, column tile), columns fastest
   const int Mt = (M + 127) / 128, Nt = (N + BN - 1) / BN;
   const int ntiles = H * Mt * Nt;
+  const int Gc = col_group > 0 ? min(col_group, Nt) : Nt;   // column tiles per group
   auto tile_coords = [&](int tl, int& b, int& m0, int& n0) {
     b = tl / (Mt * Nt);
-    const int r = tl - b * (Mt * Nt);
-    m0 = (r / Nt) * 128;
-    n0 = (r % Nt) * BN;
+    int r = tl - b * (Mt * Nt);
+    const int g = r / (Mt * Gc);                 // full groups of Mt x Gc tiles come first
+    const int gw = min(Gc, Nt - g * Gc);         // the last group may be narrower
+    r -= g * (Mt * Gc);
+    m0 = (r / gw) * 128;
+    n0 = (g * Gc + r % gw) * BN;
   };
 
   if (threadIdx.x == 0) {
@@ -314,7 +321,8 @@ cudaError_t set_dyn_smem(const void* kern, int bytes);
 template <int BN, int MODE, class Epi>
 inline cudaError_t launch_tc_gemm(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mA2,
                                   const CUtensorMap& mB2, const Epi& epi, int H, int M, int N, int K, int chunk_k,
-                                  DevStatus* stt, cudaStream_t st, int K1 = 0, const CUtensorMap* mA3 = nullptr) {
+                                  DevStatus* stt, cudaStream_t st, int K1 = 0, const CUtensorMap* mA3 = nullptr,
+                                  int col_group = 0) {
   using C = TcCfg<BN, MODE>;
   constexpr int NE = EpiWarps<Epi>::value;
   constexpr int smem = C::SMEM + NE * EpiStage<Epi>::bytes;
@@ -324,7 +332,8 @@ inline cudaError_t launch_tc_gemm(const CUtensorMap& mA, const CUtensorMap& mB, 
   if (e != cudaSuccess) return e;
   const long long ntiles = (long long)cdiv(N, BN) * cdiv(M, 128) * H;
   const int grid = (int)std::min<long long>(ntiles, tc_gemm_sm_count());
-  kern<<<grid, 64 + 32 * NE, smem, st>>>(mA, mB, mA2, mB2, mA3 ? *mA3 : mA, epi, H, M, N, K, chunk_k, K1, stt);
+  kern<<<grid, 64 + 32 * NE, smem, st>>>(mA, mB, mA2, mB2, mA3 ? *mA3 : mA, epi, H, M, N, K, chunk_k, K1, stt,
+                                         col_group);
   return cudaGetLastError();
 }
 
