@@ -79,8 +79,9 @@ def parse_args(argv=None):
     ap.add_argument("--impl", choices=("gpu", "reference"), default="gpu")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--e2e-steps", type=int, default=2)
-    ap.add_argument("--streams", type=int, default=4,
-                    help="CUDA streams (each with its own workspace) the layers of a context are spread over")
+    ap.add_argument("--streams", type=int, default=0,
+                    help="CUDA streams (each with its own workspace) the layers of a context are spread over "
+                         "(0: 3 for caches of 64K tokens and more, else 4)")
     ap.add_argument("--cpu-pairs", type=int, default=0,
                     help="(layer, head) pairs the oracle baseline times (0: about 12 s of oracle work, "
                          "at least one pair)")
@@ -430,7 +431,7 @@ def run_gpu(args, dist: Dist):
     torch.cuda.synchronize()
     # layers are independent: they are spread round-robin over `n_str` streams,
     # each with its own workspace (arckv_compact is reentrant per workspace/stream)
-    n_str = max(1, min(args.streams, len(layers)))
+    n_str = max(1, min(args.streams or (3 if w.T >= 65536 else 4), len(layers)))
     wss = [torch.empty(pk.workspace_bytes(cfg), dtype=torch.uint8, device=dev) for _ in range(n_str)]
     f32 = dict(dtype=torch.float32, device=dev)
     tp = pk.anchor_count(cfg)   # = w.t without chunking

@@ -44,6 +44,12 @@ struct TcEpiArgmax {
   }
 };
 
+// The same with eight epilogue warps, two per TMEM lane quarter, for 256-wide
+// tiles (each warp takes 128 columns).
+struct TcEpiArgmax8 : TcEpiArgmax {
+  static constexpr int kEpiWarps = 8;
+};
+
 int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* K, float* L, float2* part,
                          DevStatus* stt, cudaStream_t st) {
   CUtensorMap mA, mB;
@@ -351,18 +357,23 @@ int launch_assign_gemm(const Dims& D, const int* anchors, const bf16* Ut_hi, con
                        const bf16* S_lo, unsigned long long* best, int* kappa, DevStatus* stt, cudaStream_t st) {
   const int ldn = (D.n + 7) / 8 * 8;
   cudaMemsetAsync(best, 0, sizeof(unsigned long long) * (size_t)D.H * D.T, st);
+  // 128 keys x 256 anchors per tile (M = 128, N = 256 MMAs): half the key-side
+  // operand bytes per flop of a 128-wide tile
+  constexpr int BN = 256;
   CUtensorMap mA, mA2, mB, mB2;
   if (!encode_bf16_map_3d(&mA, Ut_hi, ldn, D.T, D.H, 128) || !encode_bf16_map_3d(&mA2, Ut_lo, ldn, D.T, D.H, 128) ||
-      !encode_bf16_map_3d(&mB, S_hi, ldn, D.t, D.H, 128) || !encode_bf16_map_3d(&mB2, S_lo, ldn, D.t, D.H, 128))
+      !encode_bf16_map_3d(&mB, S_hi, ldn, D.t, D.H, BN) || !encode_bf16_map_3d(&mB2, S_lo, ldn, D.t, D.H, BN))
     return -1;
-  TcEpiArgmax epi{best, D.T};
+  TcEpiArgmax8 epi;
+  epi.best = best;
+  epi.bbs = D.T;
   const int kfull = (ldn + 63) / 64 * 64;
-  // anchor tiles in groups whose split profiles (128 rows x ldn x 4 bytes per
+  // anchor tiles in groups whose split profiles (BN rows x ldn x 4 bytes per
   // tile) take about 40 MB, so each group stays in L2 while the key profiles
   // stream past it (one pass over them per group instead of one per wave)
-  const long long tile_bytes = 128LL * ldn * 4;
+  const long long tile_bytes = (long long)BN * ldn * 4;
   const int group = (int)std::max<long long>(1, (40LL << 20) / tile_bytes);
-  if (launch_tc_gemm<128, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.T, D.t, ldn, kfull, stt, st, 0, nullptr, group) !=
+  if (launch_tc_gemm<BN, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.T, D.t, ldn, kfull, stt, st, 0, nullptr, group) !=
       cudaSuccess)
     return -1;
   const long long cnt = (long long)D.H * D.T;

@@ -89,7 +89,9 @@ struct TcCfg {
                                : MODE == kSplit3A ? 3 * TILE_A + TILE_B
                                : MODE == kSplit3S ? 3 * (TILE_A + TILE_B)
                                                   : TILE_A + TILE_B;
-  static constexpr int STAGES = MODE == kSplit3S ? 2 : (MODE == kSplit || MODE == kSplit3A) ? 3 : 4;
+  static constexpr int STAGES_WANT = MODE == kSplit3S ? 2 : (MODE == kSplit || MODE == kSplit3A) ? 3 : 4;
+  // as many of those as fit beside the epilogue staging (wide tiles take fewer)
+  static constexpr int STAGES = STAGES_WANT * STAGE <= 200 * 1024 ? STAGES_WANT : (200 * 1024) / STAGE;
   static constexpr int SMEM = STAGES * STAGE + 1024;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
 };
