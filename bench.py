@@ -100,6 +100,9 @@ def parse_args(argv=None):
     ap.add_argument("--decode-iters", type=int, default=50)
     ap.add_argument("--profile-layer", action="store_true",
                     help="compact layer 0 twice and exit (a small case for ncu captures)")
+    ap.add_argument("--layer-shape", default="",
+                    help="with --profile-layer: T,n_pos,t overriding the workload's sizes (same distributions), "
+                         "e.g. 16384,64,2048 for a small case of the dual-form fits (t > n)")
     return ap.parse_args(argv)
 
 
@@ -422,12 +425,17 @@ def run_gpu(args, dist: Dist):
     if args.profile_layer:
         layers = layers[:1]
     sel = {"indexer": pk.SELECTOR_INDEXER, "ha": pk.SELECTOR_HA, "vi": pk.SELECTOR_VI}[args.selector]
-    cfg = workload.layer_config(w, w.H_kv, flags=pk.FLAG_NONBLOCKING, selector=sel, chunk_len=args.chunk_len)
-    cfg_block = workload.layer_config(w, w.H_kv, selector=sel, chunk_len=args.chunk_len)
+    shape = {}
+    if args.profile_layer and args.layer_shape:
+        T_, np_, t_ = (int(x) for x in args.layer_shape.split(","))
+        shape = dict(T=T_, n_pos=np_, t=t_)
+    cfg = workload.layer_config(w, w.H_kv, flags=pk.FLAG_NONBLOCKING, selector=sel, chunk_len=args.chunk_len, **shape)
+    cfg_block = workload.layer_config(w, w.H_kv, selector=sel, chunk_len=args.chunk_len, **shape)
 
     # seeded inputs drawn on the device (synth.make_layer_device: the recipe of
     # the host generator, seconds instead of minutes for a 128K context)
-    dev_in = [synth.make_layer_device(w, l, list(range(w.H_kv)), dev) for l in layers]
+    dev_in = [synth.make_layer_device(w, l, list(range(w.H_kv)), dev, T=shape.get("T"), n_pos=shape.get("n_pos"))
+              for l in layers]
     torch.cuda.synchronize()
     # layers are independent: they are spread round-robin over `n_str` streams,
     # each with its own workspace (arckv_compact is reentrant per workspace/stream)
@@ -556,7 +564,7 @@ def run_gpu(args, dist: Dist):
     peak, _, peak_src = measured_peaks()
     burst = measured_burst()
     achieved = flops / avg_s / 1e12
-    roofline = {"kernel": "tc_gemm_kernel<128, split, TcEpiArgmax> (assignment, Eq. anchor_assignment)",
+    roofline = {"kernel": "tc_gemm_kernel<256, kSplit, TcEpiArgmax8> (assignment, Eq. anchor_assignment)",
                 "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                 "traffic": profiled_traffic(), "flops_per_launch": flops, "launch_ms": avg_s * 1e3,
                 "issued_tflops": 3.0 * achieved, "issued_frac": 3.0 * achieved / peak,
@@ -578,9 +586,10 @@ def run_gpu(args, dist: Dist):
         solver[name] = {"flops": solve_flops[k], "ms_live": live * 1e3, "ms_isolated": iso * 1e3,
                         "tflops_isolated": solve_flops[k] / iso / 1e12,
                         "frac_isolated": solve_flops[k] / iso / 1e12 / burst}
-    roofline["solvers"] = dict(solver, kernel=("chol_cluster_kernel<double, 8> on the n x n dual systems "
-                                               "(fp64; sliced tensor-core Grams and back-projection counted "
-                                               "outside)" if dual else
+    roofline["solvers"] = dict(solver, kernel=("blocked Cholesky of the n x n dual systems: fp64 64 x 64 "
+                                               "diagonal factors, 5-slice tensor-core block products "
+                                               "(sliced_gemm_kernel<5>); the 4-slice Grams and back-projection "
+                                               "are counted outside" if dual else
                                                "chol_cluster_kernel<float, 4|8> (tcgen05 trailing updates) "
                                                "+ two refinement steps"),
                                note="Cholesky m^3 / 3 plus the triangular solves (m = %d, 1 and 128 right-hand "

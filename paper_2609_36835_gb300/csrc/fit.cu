@@ -1540,16 +1540,35 @@ __global__ void __launch_bounds__(256) ir_lambda_kernel(const double* __restrict
 }
 
 // r[b][c] = sum_i Phi_ic u_i - lam x_c (fp64 sums, rounded to fp32 at the end).
+// A CTA takes 32 columns (lane = column, coalesced rows) and its 8 warps
+// split the rows, each with four independent partial sums; the warps' sums
+// are added in warp order.
 __global__ void __launch_bounds__(256) ir_cols_kernel(const float* __restrict__ Phi, const double* __restrict__ u,
                                                       const float* __restrict__ x, const double* __restrict__ lam,
                                                       float* __restrict__ r, int n, int t) {
-  const int b = blockIdx.y, c = blockIdx.x * 256 + threadIdx.x;
-  if (c >= t) return;
+  __shared__ double part[8][32];
+  const int b = blockIdx.y, lane = threadIdx.x & 31, warp = threadIdx.x >> 5, c = blockIdx.x * 32 + lane;
   const float* p = Phi + (long long)b * n * t + c;
   const double* ub = u + (long long)b * n;
-  double a = 0.0;
-  for (int i = 0; i < n; ++i) a = fma((double)p[(long long)i * t], ub[i], a);
-  r[(long long)b * t + c] = (float)(a - lam[b] * (double)x[(long long)b * t + c]);
+  double a0 = 0.0, a1 = 0.0, a2 = 0.0, a3 = 0.0;
+  if (c < t) {
+    int i = warp;
+    for (; i + 24 < n; i += 32) {
+      a0 = fma((double)p[(long long)i * t], ub[i], a0);
+      a1 = fma((double)p[(long long)(i + 8) * t], ub[i + 8], a1);
+      a2 = fma((double)p[(long long)(i + 16) * t], ub[i + 16], a2);
+      a3 = fma((double)p[(long long)(i + 24) * t], ub[i + 24], a3);
+    }
+    for (; i < n; i += 8) a0 = fma((double)p[(long long)i * t], ub[i], a0);
+  }
+  part[warp][lane] = (a0 + a1) + (a2 + a3);
+  __syncthreads();
+  if (warp == 0 && c < t) {
+    double a = part[0][lane];
+#pragma unroll
+    for (int w = 1; w < 8; ++w) a += part[w][lane];
+    r[(long long)b * t + c] = (float)(a - lam[b] * (double)x[(long long)b * t + c]);
+  }
 }
 
 // x += (L L^T)^-1 r for one head per CTA (512 threads): forward substitution
@@ -1575,17 +1594,21 @@ __global__ void __launch_bounds__(512) tri_solve_kernel(const R* __restrict__ A,
     const int k0 = k * NBk, kb = min(NBk, t - k0);
     {
       const int rr = tid >> 3, pt = tid & 7;
-      R a = R(0), a2 = R(0);
+      R a = R(0), a2 = R(0), a3 = R(0), a4 = R(0);
       if (rr < kb) {
         const R* row = Ab + (long long)(k0 + rr) * t;
         int c = pt;
-        for (; c + 8 < k0; c += 16) {   // two independent chains: loads in flight together
-          a = fma_r(__ldcg(row + c), __ldcg(y + c), a);
-          a2 = fma_r(__ldcg(row + c + 8), __ldcg(y + c + 8), a2);
+        for (; c + 24 < k0; c += 32) {   // four independent chains: eight loads in flight together
+          const R l0 = __ldcg(row + c), l1 = __ldcg(row + c + 8), l2 = __ldcg(row + c + 16), l3 = __ldcg(row + c + 24);
+          const R y0 = __ldcg(y + c), y1 = __ldcg(y + c + 8), y2 = __ldcg(y + c + 16), y3 = __ldcg(y + c + 24);
+          a = fma_r(l0, y0, a);
+          a2 = fma_r(l1, y1, a2);
+          a3 = fma_r(l2, y2, a3);
+          a4 = fma_r(l3, y3, a4);
         }
-        if (c < k0) a = fma_r(__ldcg(row + c), __ldcg(y + c), a);
+        for (; c < k0; c += 8) a = fma_r(__ldcg(row + c), __ldcg(y + c), a);
       }
-      a += a2;
+      a = (a + a2) + (a3 + a4);
       a += __shfl_xor_sync(0xffffffffu, a, 1);
       a += __shfl_xor_sync(0xffffffffu, a, 2);
       a += __shfl_xor_sync(0xffffffffu, a, 4);
@@ -1611,16 +1634,22 @@ __global__ void __launch_bounds__(512) tri_solve_kernel(const R* __restrict__ A,
     const int k0 = k * NBk, kb = min(NBk, t - k0);
     {
       const int c = tid & (NBk - 1), pt = tid >> 6;
-      R a = R(0), a2 = R(0);
+      R a = R(0), a2 = R(0), a3 = R(0), a4 = R(0);
       if (c < kb) {
+        const R* col = Ab + k0 + c;
         int rr = k0 + kb + pt;
-        for (; rr + 8 < t; rr += 16) {
-          a = fma_r(__ldcg(Ab + (long long)rr * t + k0 + c), __ldcg(y + rr), a);
-          a2 = fma_r(__ldcg(Ab + (long long)(rr + 8) * t + k0 + c), __ldcg(y + rr + 8), a2);
+        for (; rr + 24 < t; rr += 32) {
+          const R l0 = __ldcg(col + (long long)rr * t), l1 = __ldcg(col + (long long)(rr + 8) * t);
+          const R l2 = __ldcg(col + (long long)(rr + 16) * t), l3 = __ldcg(col + (long long)(rr + 24) * t);
+          const R y0 = __ldcg(y + rr), y1 = __ldcg(y + rr + 8), y2 = __ldcg(y + rr + 16), y3 = __ldcg(y + rr + 24);
+          a = fma_r(l0, y0, a);
+          a2 = fma_r(l1, y1, a2);
+          a3 = fma_r(l2, y2, a3);
+          a4 = fma_r(l3, y3, a4);
         }
-        if (rr < t) a = fma_r(__ldcg(Ab + (long long)rr * t + k0 + c), __ldcg(y + rr), a);
+        for (; rr < t; rr += 8) a = fma_r(__ldcg(col + (long long)rr * t), __ldcg(y + rr), a);
       }
-      part[pt][c] = a + a2;
+      part[pt][c] = (a + a2) + (a3 + a4);
     }
     __syncthreads();
     if (tid < NBk) {
@@ -1660,7 +1689,7 @@ static int refine_beta(const Dims& D, float ridge_w, const float* m, const FitBu
       ir_rows_kernel<<<cdiv(hn, 8), 256, 0, st>>>(B.Phi, m, B.wsol, B.ir_u, nullptr, D.n, D.t, D.H);
       ++nl;
     }
-    ir_cols_kernel<<<dim3(cdiv(D.t, 256), D.H), 256, 0, st>>>(B.Phi, B.ir_u, B.wsol, B.ir_lam, B.rhs, D.n, D.t);
+    ir_cols_kernel<<<dim3(cdiv(D.t, 32), D.H), 256, 0, st>>>(B.Phi, B.ir_u, B.wsol, B.ir_lam, B.rhs, D.n, D.t);
     tri_solve_kernel<float><<<D.H, 512, 0, st>>>(B.Gram, B.Linv, B.rhs, B.Z, B.wsol, D.t);
     nl += 2;
   }

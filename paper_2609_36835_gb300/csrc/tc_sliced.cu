@@ -390,22 +390,31 @@ __global__ void __launch_bounds__(256) slice_rows_kernel(const T* __restrict__ X
 }
 
 // Column maxima exponents of X [H][K][R] (R contiguous, rows ldx apart): ex [H][R].
-// A CTA takes 32 columns (lane = column, coalesced rows); its 8 warps split
-// the rows and meet in shared memory.
+// A CTA takes 32 columns (lane = column, coalesced rows); its 32 warps split
+// the rows (four loads in flight each) and meet in shared memory.
 template <typename T>
-__global__ void __launch_bounds__(256) col_exp_kernel(const T* __restrict__ X, int K, int R, int ldx, long long xbs,
-                                                      int* __restrict__ ex) {
-  __shared__ T part[8][32];
+__global__ void __launch_bounds__(1024) col_exp_kernel(const T* __restrict__ X, int K, int R, int ldx, long long xbs,
+                                                       int* __restrict__ ex) {
+  __shared__ T part[32][33];
   const int b = blockIdx.y, lane = threadIdx.x & 31, warp = threadIdx.x >> 5, r = blockIdx.x * 32 + lane;
   const T* x = X + (long long)b * xbs + r;
-  T mx = T(0);
-  if (r < R)
-    for (int k = warp; k < K; k += 8) mx = fmax(mx, fabs(x[(long long)k * ldx]));
-  part[warp][lane] = mx;
+  T m0 = T(0), m1 = T(0), m2 = T(0), m3 = T(0);
+  if (r < R) {
+    int k = warp;
+    for (; k + 96 < K; k += 128) {
+      m0 = fmax(m0, fabs(x[(long long)k * ldx]));
+      m1 = fmax(m1, fabs(x[(long long)(k + 32) * ldx]));
+      m2 = fmax(m2, fabs(x[(long long)(k + 64) * ldx]));
+      m3 = fmax(m3, fabs(x[(long long)(k + 96) * ldx]));
+    }
+    for (; k < K; k += 32) m0 = fmax(m0, fabs(x[(long long)k * ldx]));
+  }
+  part[warp][lane] = fmax(fmax(m0, m1), fmax(m2, m3));
   __syncthreads();
   if (warp == 0 && r < R) {
+    T mx = part[0][lane];
 #pragma unroll
-    for (int w = 1; w < 8; ++w) mx = fmax(mx, part[w][lane]);
+    for (int w = 1; w < 32; ++w) mx = fmax(mx, part[w][lane]);
     ex[(long long)b * R + r] = bound_exp(mx);
   }
 }
@@ -508,7 +517,7 @@ template <typename T>
 static int slice_cols_t(int S, const T* X, int K, int R, int ldx, long long xbs, int H, bf16* out, int* ex,
                         cudaStream_t st) {
   const int ldo = (int)sliced_ld(K);
-  col_exp_kernel<T><<<dim3(cdiv(R, 32), H), 256, 0, st>>>(X, K, R, ldx, xbs, ex);
+  col_exp_kernel<T><<<dim3(cdiv(R, 32), H), 1024, 0, st>>>(X, K, R, ldx, xbs, ex);
   const dim3 grid(cdiv(R, 32), cdiv(K, 32), H);
   if (S == 3)
     slice_cols_kernel<3, T><<<grid, 256, 0, st>>>(X, K, R, ldx, xbs, H, ex, out, ldo);
