@@ -97,6 +97,75 @@ __device__ __forceinline__ float fma_r(float a, float b, float c) { return fmaf(
 __device__ __forceinline__ double fma_r(double a, double b, double c) { return fma(a, b, c); }
 __device__ __forceinline__ float rcp_r(float x) { return __frcp_rn(x); }
 __device__ __forceinline__ double rcp_r(double x) { return __drcp_rn(x); }
+
+// Double-float arithmetic: a value hi + lo of two fp32 numbers (|lo| <= ulp(hi) / 2),
+// ~48 significant bits.  The GB300's fp64 pipe issues at a small fraction of its
+// fp32 rate, so the fp64 64 x 64 diagonal blocks of the dual Cholesky are
+// factored in this arithmetic (each operation a short chain of fp32 operations:
+// the error-free sum and product transformations of Dekker and Knuth, and one
+// Newton step for the reciprocal and the square root), with the block read
+// from and written back to fp64 storage.
+struct df64 {
+  float hi, lo;
+  df64() = default;
+  __device__ __forceinline__ df64(float h, float l) : hi(h), lo(l) {}
+  __device__ __forceinline__ explicit df64(int v) : hi((float)v), lo(0.f) {}
+};
+__device__ __forceinline__ df64 df_fast2(float a, float b) {   // |a| >= |b| (or a = 0)
+  const float s = a + b;
+  return df64(s, b - (s - a));
+}
+__device__ __forceinline__ df64 df_two(float a, float b) {
+  const float s = a + b, bb = s - a;
+  return df64(s, (a - (s - bb)) + (b - bb));
+}
+__device__ __forceinline__ df64 operator+(df64 x, df64 y) {
+  df64 s = df_two(x.hi, y.hi);
+  const df64 t = df_two(x.lo, y.lo);
+  s.lo += t.hi;
+  s = df_fast2(s.hi, s.lo);
+  s.lo += t.lo;
+  return df_fast2(s.hi, s.lo);
+}
+__device__ __forceinline__ df64 operator-(df64 x) { return df64(-x.hi, -x.lo); }
+__device__ __forceinline__ df64 operator-(df64 x, df64 y) { return x + (-y); }
+__device__ __forceinline__ df64 operator*(df64 x, df64 y) {
+  const float p = x.hi * y.hi;
+  float e = fmaf(x.hi, y.hi, -p);
+  e = fmaf(x.hi, y.lo, e);
+  e = fmaf(x.lo, y.hi, e);
+  return df_fast2(p, e);
+}
+__device__ __forceinline__ df64& operator*=(df64& x, df64 y) { return x = x * y; }
+__device__ __forceinline__ bool operator>(df64 x, df64 y) { return x.hi > y.hi || (x.hi == y.hi && x.lo > y.lo); }
+__device__ __forceinline__ bool finite_r(float x) { return isfinite(x); }
+__device__ __forceinline__ bool finite_r(double x) { return isfinite(x); }
+__device__ __forceinline__ bool finite_r(df64 x) { return isfinite(x.hi); }
+__device__ __forceinline__ df64 fma_r(df64 a, df64 b, df64 c) { return a * b + c; }
+__device__ __forceinline__ df64 rcp_r(df64 x) {   // r + r (1 - x r)
+  const df64 r(__frcp_rn(x.hi), 0.f);
+  return r + r * (df64(1) - x * r);
+}
+__device__ __forceinline__ float sqrt_r(float x) { return sqrtf(x); }
+__device__ __forceinline__ double sqrt_r(double x) { return ::sqrt(x); }
+__device__ __forceinline__ df64 sqrt_r(df64 x) {    // s + (x - s^2) / (2 s)
+  if (!(x.hi > 0.f)) return df64(sqrtf(x.hi), 0.f);
+  const float s = sqrtf(x.hi);
+  const df64 r = x - df64(s, 0.f) * df64(s, 0.f);
+  return df_fast2(s, r.hi * (0.5f / s));
+}
+// storage conversions (the block lives in fp64 in global memory)
+template <typename R, typename G>
+__device__ __forceinline__ R to_reg(G v) { return v; }
+template <>
+__device__ __forceinline__ df64 to_reg<df64, double>(double v) {
+  const float h = __double2float_rn(v);
+  return df64(h, __double2float_rn(v - (double)h));
+}
+template <typename G, typename R>
+__device__ __forceinline__ G to_mem(R v) { return v; }
+template <>
+__device__ __forceinline__ double to_mem<double, df64>(df64 v) { return (double)v.hi + (double)v.lo; }
 template <typename R>
 __device__ __forceinline__ R warp_sum_r(R v) {
 #pragma unroll
@@ -241,14 +310,14 @@ __device__ __forceinline__ void mm64(Tile<R> XT, Tile<R> Y, R (&acc)[kTP][kTQ]) 
 
 // Load the lower part of A_kk + lam I into the tile L (identity beyond the
 // matrix when kb < NB; zero above the diagonal).
-template <typename R>
-__device__ __forceinline__ void load_diag(Tile<R> L, const R* Ab, int t, int k0, int kb, R lam) {
+template <typename R, typename G>
+__device__ __forceinline__ void load_diag(Tile<R> L, const G* Ab, int t, int k0, int kb, G lam) {
   constexpr int NE = NB * NB / kCT;
   R v[NE];
 #pragma unroll
   for (int q = 0; q < NE; ++q) {
     const int e = threadIdx.x + q * kCT, r = e / NB, c = e % NB;
-    v[q] = (r < kb && c <= r) ? __ldcg(Ab + (long long)(k0 + r) * t + k0 + c) + (r == c ? lam : R(0))
+    v[q] = (r < kb && c <= r) ? to_reg<R>(__ldcg(Ab + (long long)(k0 + r) * t + k0 + c) + (r == c ? lam : G(0)))
                               : (r == c ? R(1) : R(0));
   }
 #pragma unroll
@@ -259,14 +328,14 @@ __device__ __forceinline__ void load_diag(Tile<R> L, const R* Ab, int t, int k0,
 }
 
 // Write L_kk (lower part, rows < kb) into A and the full tile Li into Linv[k].
-template <typename R>
-__device__ __forceinline__ void store_diag(Tile<R> L, Tile<R> Li, R* Ab, R* Lb, int t, int k, int kb) {
-  R* Lo = Lb + (long long)k * NB * NB;
+template <typename R, typename G>
+__device__ __forceinline__ void store_diag(Tile<R> L, Tile<R> Li, G* Ab, G* Lb, int t, int k, int kb) {
+  G* Lo = Lb + (long long)k * NB * NB;
   const int k0 = k * NB;
   for (int e = threadIdx.x; e < NB * NB; e += kCT) {
     const int rr = e / NB, cc = e % NB;
-    Lo[e] = Li[rr][cc];
-    if (rr < kb && cc <= rr) Ab[(long long)(k0 + rr) * t + k0 + cc] = L[rr][cc];
+    Lo[e] = cc <= rr ? to_mem<G>(Li[rr][cc]) : G(0);   // the inverse is lower triangular
+    if (rr < kb && cc <= rr) Ab[(long long)(k0 + rr) * t + k0 + cc] = to_mem<G>(L[rr][cc]);
   }
 }
 
@@ -282,8 +351,8 @@ __device__ __forceinline__ void store_diag(Tile<R> L, Tile<R> Li, R* Ab, R* Lb, 
 //            level by level (i - j = 1, 2, 3).
 // Tiles: L (the block; pad column NB holds 1 / l_cc), Li (the inverse), T
 // (scratch).  Pad rows beyond the matrix (kb < NB) are the identity.
-template <typename R>
-__device__ void factor_diag(R* Ab, R* Lb, int t, int k, R lam, Tile<R> L, Tile<R> Li, Tile<R> T, int* bad) {
+template <typename R, typename G = R>
+__device__ void factor_diag(G* Ab, G* Lb, int t, int k, G lam, Tile<R> L, Tile<R> Li, Tile<R> T, int* bad) {
   static_assert(kCT == 512 && NB == 64, "thread map of the 16-wide panels");
   const int tid = threadIdx.x, k0 = k * NB, kb = min(NB, t - k0);
   load_diag(L, Ab, t, k0, kb, lam);
@@ -296,7 +365,7 @@ __device__ void factor_diag(R* Ab, R* Lb, int t, int k, R lam, Tile<R> L, Tile<R
     for (int j = 0; j < 15; ++j) {   // factor the diagonal block
       if (blk && ec > j && er >= ec) {
         R piv = L[c0 + j][c0 + j];
-        if (!(piv > R(0)) || !isfinite(piv)) piv = R(1);
+        if (!(piv > R(0)) || !finite_r(piv)) piv = R(1);
         L[c0 + er][c0 + ec] = fma_r(-L[c0 + er][c0 + j] * rcp_r(piv), L[c0 + ec][c0 + j], L[c0 + er][c0 + ec]);
       }
       __syncthreads();
@@ -304,11 +373,11 @@ __device__ void factor_diag(R* Ab, R* Lb, int t, int k, R lam, Tile<R> L, Tile<R
     R v = R(0);
     if (blk && er >= ec) {   // column scaling
       R pc = L[c0 + ec][c0 + ec];
-      if (!(pc > R(0)) || !isfinite(pc)) {
+      if (!(pc > R(0)) || !finite_r(pc)) {
         if (er == ec && c0 + ec < kb) *bad = 1;
         pc = R(1);
       }
-      const R d = sqrt(pc);
+      const R d = sqrt_r(pc);
       v = (er == ec) ? d : L[c0 + er][c0 + ec] * rcp_r(d);
     }
     __syncthreads();
@@ -1262,20 +1331,22 @@ __global__ void chol_lambda_kernel(const double* A, int n, double ridge, double 
   }
 }
 
-// Factor diagonal block k of every head (one CTA per head): L_kk into A,
-// L_kk^-1 into Linv[k]; a non-positive pivot records ARCKV_ERR_NOT_SPD.
+// Factor diagonal block k of every head (one CTA per head) in double-float
+// arithmetic: L_kk into A, L_kk^-1 into Linv[k] (fp64 storage); a
+// non-positive pivot records ARCKV_ERR_NOT_SPD.
 __global__ void __launch_bounds__(kCT, 1) chol_diag_kernel(double* A, double* Linv, int n, int k, const double* lam,
                                                            DevStatus* stt) {
   extern __shared__ __align__(16) unsigned char smraw[];
-  double* sm = (double*)smraw;
-  Tile<double> S1 = (Tile<double>)sm;
-  Tile<double> S2 = (Tile<double>)(sm + kTileF<double>);
-  Tile<double> S3 = (Tile<double>)(sm + 2 * kTileF<double>);
+  df64* sm = (df64*)smraw;
+  Tile<df64> S1 = (Tile<df64>)sm;
+  Tile<df64> S2 = (Tile<df64>)(sm + kTileF<df64>);
+  Tile<df64> S3 = (Tile<df64>)(sm + 2 * kTileF<df64>);
   __shared__ int bad;
   const int b = blockIdx.x, nblk = (n + NB - 1) / NB;
   if (threadIdx.x == 0) bad = 0;
   __syncthreads();
-  factor_diag<double>(A + (long long)b * n * n, Linv + (long long)b * nblk * NB * NB, n, k, lam[b], S1, S2, S3, &bad);
+  factor_diag<df64, double>(A + (long long)b * n * n, Linv + (long long)b * nblk * NB * NB, n, k, lam[b], S1, S2, S3,
+                            &bad);
   if (threadIdx.x == 0 && bad) set_status(stt, ARCKV_ERR_NOT_SPD);
 }
 
@@ -1342,7 +1413,7 @@ static int chol_solve_sliced(int H, int n, double* A, double* Linv, double* B, d
   constexpr int S = kCholSlices;
   const int nblk = (n + NB - 1) / NB;
   const long long nn = (long long)n * n, nr = (long long)n * nrhs, lb = (long long)nblk * NB * NB;
-  const int dsm = 3 * kTileF<double> * (int)sizeof(double);
+  const int dsm = 3 * kTileF<df64> * (int)sizeof(df64);
   if (set_dyn_smem((const void*)chol_diag_kernel, dsm) != cudaSuccess)
     return -1;
   int nl = 0;

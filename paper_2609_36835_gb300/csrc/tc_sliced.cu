@@ -5,10 +5,15 @@
 // Slices.  Row r of an operand X (fp32 or fp64) is scaled by 2^-e_r, where
 // 2^e_r bounds the row's largest magnitude, and cut into S bf16 slices
 //     X[r][k] = 2^e_r (x_1 + x_2 + ... + x_S) + residual,
-//     x_i = I_i 2^(-8 i),  I_1 in [-256, 256],  I_i in [-128, 128] (i > 1),
-// each x_i the rounding of what the earlier slices left to the next 8 bits, so
+//     x_i = I_i 2^(-8 i),  I_1 in [-256, 256],  I_i in [-128, 127] (i > 1):
+// the balanced base-256 digits of Z = round(X[r][k] 2^(8 S - e_r)), so
 // |residual| <= 2^(-8 S - 1) 2^e_r.  Every slice is an integer of at most 8
-// significant bits times a power of two: exact in bf16.
+// significant bits times a power of two: exact in bf16.  The GB300's fp64
+// pipe runs at a small fraction of its integer and fp32 rates, so the
+// exponents, the rounding to Z and the digits are taken with integer
+// operations on the operand's bits, and each fp64 result is one rounding
+// conversion of a 64-bit integer sum with its power of two added to the
+// exponent field (plus the subtraction of the `sub` mode).
 //
 // Products.  C = A B^T is the sum over all S^2 slice pairs (i, j).  A pair's
 // products are integers times 2^(-8(i + j)), so the pairs of one level
@@ -18,17 +23,20 @@
 // per 128-wide K chunk, and the epilogue converts each chunk's sums to
 // integers and adds them up exactly (in 64-bit, for K <= 26214); the levels
 // above 4 weigh at most 2^-24 of the total and accumulate in one fp32
-// accumulator over the whole K.  The result, assembled in fp64 and scaled by
-// 2^(e_m + f_n), is the exact product of the sliced operands up to the fp32
-// rounding of the levels above 4 (~2^-48 relative): the fp32 arithmetic of the
-// tensor pipe never meets a rounding that matters.
+// accumulator over the whole K.  The result (the exact levels in units of
+// 2^-32 shifted to units of 2^-44, plus the fp32 levels rounded to that unit,
+// in one 64-bit integer), rounded once to fp64 and scaled by 2^(e_m + f_n), is
+// the exact product of the sliced operands up to ~2^-44 relative: the fp32
+// arithmetic of the tensor pipe never meets a rounding that matters.
 //
 // Kernel layout (persistent, one CTA per SM): warp 0 streams 32-wide K slabs
 // of the S slices of a 128-row A tile and a 64-row B tile with TMA (64-byte
 // swizzle) into a shared ring; warp 1 issues the S^2 tcgen05 MMAs (M = 128,
-// N = 64, K = 16) of every K step into the level accumulators; warps 2..9
-// drain the exact levels after every chunk (two warps per TMEM lane quarter,
-// 32 columns each) and assemble the tile.
+// N = 64, K = 16) of every K step into the level accumulators (the exact
+// levels of two alternating chunks, the higher levels of two alternating
+// tiles: 512 TMEM columns); warps 2..9 drain the exact levels after every
+// chunk (two warps per TMEM lane quarter, 32 columns each) and assemble the
+// tile while the MMAs of the next tile run.
 #include <algorithm>
 
 #include "kernels.h"
@@ -44,63 +52,120 @@ constexpr int kSlEpiWarps = 8;
 constexpr int kSlThreads = 64 + 32 * kSlEpiWarps;
 constexpr int kSlTileA = kSlBM * kSlBK * 2, kSlTileB = kSlBN * kSlBK * 2;   // 8 KB, 4 KB
 
+// Each epilogue warp stages its 32 rows x 16 columns of results (rows padded
+// to 17 elements) in shared memory and writes them back row-contiguously, so
+// that the stores (and the loads of the `sub` mode) are coalesced.
+constexpr int kSlStageLd = 17;
+constexpr int kSlStageBytes = 32 * kSlStageLd * 8;
+
 template <int S>
 struct SlCfg {
   static constexpr int STAGE = S * (kSlTileA + kSlTileB);
-  static constexpr int STAGES = std::min(6, (200 * 1024) / STAGE);
-  static constexpr int SMEM = STAGES * STAGE + 1024;
+  // the ring takes what the staging tiles, the 1 KB alignment slack and 1 KB
+  // of static barriers leave of the 227 KB a CTA may hold
+  static constexpr int RING = 227 * 1024 - 2048 - kSlEpiWarps * kSlStageBytes;
+  static constexpr int STAGES = std::min(6, RING / STAGE);
+  static constexpr int SMEM = STAGES * STAGE + 1024 + kSlEpiWarps * kSlStageBytes;
+  static_assert(STAGES >= 2, "two ring stages at least");
 };
 
-// Epilogue outputs: 16 consecutive columns c0.. of one row, value e given by
-// val(e) (evaluated once per element, in order, so no array of them is held).
+// Marks an element whose sum met a non-finite operand (kept as NaN).
+constexpr int kSlNaN = -0x40000000;
+
+// T 2^ex rounded once to fp64: the conversion of T rounds (to nearest even),
+// the scaling by 2^ex is an exact exponent adjustment; ldexp only outside the
+// normal range (never for finite operands).
+__device__ __forceinline__ double compose_f64(long long T, int ex) {
+  if (ex == kSlNaN) return __longlong_as_double(0x7FF8000000000000ll);
+  const double d = __ll2double_rn(T);
+  const long long bits = __double_as_longlong(d);
+  const int E = (int)((bits >> 52) & 0x7FF);
+  if (E == 0) return d;   // zero (|T| >= 1 otherwise)
+  const int E2 = E + ex;
+  if (E2 <= 0 || E2 >= 2047) return ldexp(d, ex);
+  return __longlong_as_double(bits + ((long long)ex << 52));
+}
+
+// T 2^ex rounded once to fp32.
+__device__ __forceinline__ float compose_f32(long long T, int ex) {
+  if (ex == kSlNaN) return __uint_as_float(0x7FC00000u);
+  const float f = __ll2float_rn(T);           // the one rounding; the scaling below is exact
+  const unsigned int b = __float_as_uint(f);
+  const int E = (int)((b >> 23) & 0xFFu);
+  if (E == 0) return f;                       // zero (T below 2^24 never rounds to a subnormal)
+  const int E2 = E + ex;
+  if (E2 <= 0 || E2 >= 255) return ldexpf(f, ex);
+  return __uint_as_float((b & 0x807FFFFFu) | ((unsigned int)E2 << 23));
+}
+
+// A tile element: the integer T of its sum (units 2^-44 of the scaled
+// operands) and the power of two that scales it back.
+struct SlVal {
+  long long T;
+  int ex;
+};
+
+// Epilogue outputs: make() turns a tile element into the stored type; store()
+// writes one element (row < M, col < N).
 struct SlOutF64 {
+  using Elem = double;
   double* C;
   long long cbs;
   int ldc;
   int sub;   // 0: C = A B^T; 1: C -= A B^T
-  template <class F>
-  __device__ __forceinline__ void put(int b, int row, int c0, int M, int N, F&& val) const {
-    if (row >= M) return;
-    double* d = C + (long long)b * cbs + (long long)row * ldc + c0;
-    if (((((uintptr_t)d) & 15) == 0) && c0 + 16 <= N) {
-#pragma unroll
-      for (int q = 0; q < 16; q += 2) {
-        const double x0 = val(q), x1 = val(q + 1);
-        if (sub) {
-          const double2 o = *(const double2*)(d + q);
-          *(double2*)(d + q) = make_double2(o.x - x0, o.y - x1);
-        } else {
-          *(double2*)(d + q) = make_double2(x0, x1);
-        }
-      }
-    } else {
-#pragma unroll
-      for (int q = 0; q < 16; ++q)
-        if (c0 + q < N) d[q] = sub ? d[q] - val(q) : val(q);
-    }
+  // `sub`: bring the 32 values this thread's row will update into L2 while
+  // the tile's products run
+  __device__ __forceinline__ void prefetch(int b, int row, int c0, int M, int N) const {
+    if (!sub || row >= M) return;
+    const double* d = C + (long long)b * cbs + (long long)row * ldc + c0;
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(d));
+    if (c0 + 16 < N) asm volatile("prefetch.global.L2 [%0];" ::"l"(d + 16));
   }
+  __device__ __forceinline__ double make(SlVal v) const { return compose_f64(v.T, v.ex); }
+  __device__ __forceinline__ double* at(int b, int row, int col) const {
+    return C + (long long)b * cbs + (long long)row * ldc + col;
+  }
+  __device__ __forceinline__ double old(const double* d) const { return sub ? __ldcg(d) : 0.0; }
+  __device__ __forceinline__ void put(double* d, double old, double v) const { *d = sub ? old - v : v; }
 };
 struct SlOutF32 {
+  using Elem = float;
   float* C;
   long long cbs;
   int ldc;
-  template <class F>
-  __device__ __forceinline__ void put(int b, int row, int c0, int M, int N, F&& val) const {
-    if (row >= M) return;
-    float* d = C + (long long)b * cbs + (long long)row * ldc + c0;
-    if (((((uintptr_t)d) & 15) == 0) && c0 + 16 <= N) {
-#pragma unroll
-      for (int q = 0; q < 16; q += 4) {
-        const float x0 = (float)val(q), x1 = (float)val(q + 1), x2 = (float)val(q + 2), x3 = (float)val(q + 3);
-        *(float4*)(d + q) = make_float4(x0, x1, x2, x3);
-      }
-    } else {
-#pragma unroll
-      for (int q = 0; q < 16; ++q)
-        if (c0 + q < N) d[q] = (float)val(q);
-    }
+  __device__ __forceinline__ void prefetch(int, int, int, int, int) const {}
+  __device__ __forceinline__ float make(SlVal v) const { return compose_f32(v.T, v.ex); }
+  __device__ __forceinline__ float* at(int b, int row, int col) const {
+    return C + (long long)b * cbs + (long long)row * ldc + col;
   }
+  __device__ __forceinline__ float old(const float*) const { return 0.f; }
+  __device__ __forceinline__ void put(float* d, float, float v) const { *d = v; }
 };
+
+// One warp's 32 rows (y0 + lane) x 16 columns (c0..) of results: each lane
+// makes its row's values into the staging tile, then the warp writes the tile
+// two rows per instruction (16 lanes per row: consecutive columns).
+template <class Out, class F>
+__device__ __forceinline__ void sl_store_rows(const Out& out, typename Out::Elem* stg, int lane, int b, int y0, int c0,
+                                              int M, int N, F&& val) {
+  using E = typename Out::Elem;
+#pragma unroll
+  for (int e = 0; e < 16; ++e) stg[lane * kSlStageLd + e] = out.make(val(e));
+  __syncwarp();
+  const int rr = lane >> 4, cc = lane & 15, col = c0 + cc;
+  E* dst[16];
+  E old[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {   // all loads of the `sub` mode in flight before the stores
+    const int row = y0 + 2 * i + rr;
+    dst[i] = (row < M && col < N) ? out.at(b, row, col) : nullptr;
+    old[i] = dst[i] ? out.old(dst[i]) : E(0);
+  }
+#pragma unroll
+  for (int i = 0; i < 16; ++i)
+    if (dst[i]) out.put(dst[i], old[i], stg[(2 * i + rr) * kSlStageLd + cc]);
+  __syncwarp();
+}
 
 // Tiles of one batch: all (row tile, column tile) pairs, or with `lower` only
 // those that reach the lower triangle (column tile start <= row tile end) of a
@@ -133,7 +198,7 @@ __global__ void __launch_bounds__(kSlThreads, 1)
   using C = SlCfg<S>;
   constexpr int STAGES = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
-  __shared__ uint64_t full[STAGES], empty[STAGES], accf[2], acce[2], l5f, l5e, drain;
+  __shared__ uint64_t full[STAGES], empty[STAGES], accf[2], acce[2], l5f[2], l5e[2], drain;
   __shared__ uint32_t tmem_slot;
   __shared__ int abort_flag;
   const uint32_t raw = tc::smem_u32(smem_raw);
@@ -158,15 +223,15 @@ __global__ void __launch_bounds__(kSlThreads, 1)
     for (int i = 0; i < 2; ++i) {
       tc::mbar_init(&accf[i], 1);
       tc::mbar_init(&acce[i], kSlEpiWarps);
+      tc::mbar_init(&l5f[i], 1);
+      tc::mbar_init(&l5e[i], kSlEpiWarps);
     }
-    tc::mbar_init(&l5f, 1);
-    tc::mbar_init(&l5e, kSlEpiWarps);
     tc::mbar_init(&drain, 1);
     abort_flag = 0;
     tc::mbar_fence_init();
   }
   // TMEM: exact levels 2..4 of two alternating chunks at columns (buf * 3 + lvl) * 64,
-  // the levels above 4 at column 384
+  // the levels above 4 of two alternating tiles at columns 384 + 64 (tile & 1)
   if (warp == 1) tc::tmem_alloc(&tmem_slot, 512);
   tc::fence_before_sync();
   __syncthreads();
@@ -209,12 +274,14 @@ __global__ void __launch_bounds__(kSlThreads, 1)
       bool ok = true;
       int g = 0, cg = 0, tcount = 0;
       for (int tl = blockIdx.x; tl < ntiles && ok; tl += gridDim.x, ++tcount) {
-        // the level-5+ accumulator of the previous tile must have been read
-        if (tcount >= 1 && !tc::mbar_wait(&l5e, (tcount - 1) & 1, abortp, stt)) {
+        // the level-5+ accumulator of this parity must have been read (two tiles ago)
+        const int b5 = tcount & 1;
+        if (tcount >= 2 && !tc::mbar_wait(&l5e[b5], ((tcount >> 1) - 1) & 1, abortp, stt)) {
           ok = false;
           break;
         }
         tc::fence_after_sync();
+        const uint32_t t5 = tmem + 384u + (uint32_t)(b5 * 64);
         bool started5 = false;
         for (int c = 0; c < nchunks && ok; ++c, ++cg) {
           const int buf = cg & 1;
@@ -246,7 +313,7 @@ __global__ void __launch_bounds__(kSlThreads, 1)
                     tc::mma_f16(tmem + (uint32_t)((buf * 3 + lvl) * 64), ad, bd, idesc, started[lvl] ? 1u : 0u);
                     started[lvl] = true;
                   } else {
-                    tc::mma_f16(tmem + 384u, ad, bd, idesc, started5 ? 1u : 0u);
+                    tc::mma_f16(t5, ad, bd, idesc, started5 ? 1u : 0u);
                     started5 = true;
                   }
                 }
@@ -256,7 +323,7 @@ __global__ void __launch_bounds__(kSlThreads, 1)
           }
           if (ok) tc::mma_commit(&accf[buf]);
         }
-        if (ok) tc::mma_commit(&l5f);
+        if (ok) tc::mma_commit(&l5f[b5]);
       }
       tc::mma_commit(&drain);
       volatile int never = 0;
@@ -273,6 +340,7 @@ __global__ void __launch_bounds__(kSlThreads, 1)
       sl_tile(tl, Mt, Nt, lower != 0, b, mt, nt);
       // exact running sum of levels 2..4 in units of 2^-32: level l contributes
       // its integer chunk sums shifted left by 8 (4 - l) bits (|sum| < 2^47)
+      out.prefetch(b, mt * kSlBM + row_in, nt * kSlBN + half * 32, M, N);
       long long acc[32];
 #pragma unroll
       for (int e = 0; e < 32; ++e) acc[e] = 0;
@@ -300,27 +368,45 @@ __global__ void __launch_bounds__(kSlThreads, 1)
         if (lane == 0) tc::mbar_arrive(&acce[buf]);
       }
       if (!ok) break;
-      ok = __all_sync(0xffffffffu, tc::mbar_wait(&l5f, tcount & 1, abortp, stt));
+      const int b5 = tcount & 1;
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(&l5f[b5], (tcount >> 1) & 1, abortp, stt));
       if (!ok) break;
       tc::fence_after_sync();
       float v5[2][16];
-      tc::tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + 384u + (uint32_t)(half * 32), v5[0]);
-      tc::tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + 384u + (uint32_t)(half * 32 + 16), v5[1]);
+      const uint32_t t5 = tmem + ((uint32_t)(q * 32) << 16) + 384u + (uint32_t)(b5 * 64 + half * 32);
+      tc::tmem_ld16(t5, v5[0]);
+      tc::tmem_ld16(t5 + 16u, v5[1]);
       tc::fence_before_sync();
       __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&l5e);
+      if (lane == 0) tc::mbar_arrive(&l5e[b5]);
       const int row = mt * kSlBM + row_in;
       const int er = row < M ? eA[(long long)b * M + row] : 0;
+      typename Out::Elem* stg =
+          (typename Out::Elem*)(base + C::STAGES * C::STAGE + (warp - 2) * kSlStageBytes);
       const int* ecol = eB + (long long)b * N;
+      // the sum in units of 2^-44: the exact levels (|acc| < 2^47 in units
+      // of 2^-32) and the levels above 4 (|v5| < 2^-8) rounded to the unit,
+      // taken as two fp32 halves of 22 bits (no 64-bit conversion)
+      // (a non-finite operand leaves NaN in the levels above 4: every slice of
+      // its row or column is NaN; such elements are marked in nanmask)
+      unsigned nanmask = 0;
+#pragma unroll
+      for (int e = 0; e < 32; ++e) {
+        const float h = v5[e >> 4][e & 15] * 0x1p22f;   // exact
+        if (h != h) nanmask |= 1u << e;
+        const int hi = __float2int_rn(h);
+        const int lo = __float2int_rn((h - (float)hi) * 0x1p22f);   // both steps exact
+        acc[e] = acc[e] * 4096ll + (long long)hi * 4194304ll + lo;
+      }
 #pragma unroll
       for (int p2 = 0; p2 < 2; ++p2) {
         const int c0 = nt * kSlBN + half * 32 + p2 * 16;
-        out.put(b, row, c0, M, N, [&](int e) -> double {
-          const double t = (double)acc[p2 * 16 + e] * 0x1p-32 + (double)v5[p2][e];   // |acc| < 2^53: exact
-          // 2^(er + ec) built from its bits (row and column exponents of finite
-          // fp32 / fp64 data stay well inside the normal range)
-          const int ex = er + ecol[c0 + e];   // only evaluated for columns below N
-          return (ex > -1023 && ex < 1024) ? t * __longlong_as_double((long long)(1023 + ex) << 52) : ldexp(t, ex);
+        int ec[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) ec[e] = c0 + e < N ? ecol[c0 + e] : 0;
+        sl_store_rows(out, stg, lane, b, mt * kSlBM + q * 32, c0, M, N, [&](int e) -> SlVal {
+          if ((nanmask >> (p2 * 16 + e)) & 1u) return SlVal{0, kSlNaN};
+          return SlVal{acc[p2 * 16 + e], er + ec[e] - 44};
         });
       }
     }
@@ -335,31 +421,83 @@ __global__ void __launch_bounds__(kSlThreads, 1)
 
 // --------------------------------------------------------------- slicing
 
-// Exponent e with |x| <= 2^e for every x of magnitude <= mx (0 for mx = 0).
+// Bits of |x|: for non-negative floats the bit patterns order like the values,
+// so maxima of magnitudes are integer maxima.
+__device__ __forceinline__ unsigned long long mag_bits(double x) {
+  return (unsigned long long)__double_as_longlong(x) & 0x7FFFFFFFFFFFFFFFull;
+}
+__device__ __forceinline__ unsigned long long mag_bits(float x) { return __float_as_uint(x) & 0x7FFFFFFFu; }
+__device__ __forceinline__ unsigned long long raw_bits(double x) { return (unsigned long long)__double_as_longlong(x); }
+__device__ __forceinline__ unsigned long long raw_bits(float x) { return __float_as_uint(x); }
+
 template <typename T>
-__device__ __forceinline__ int bound_exp(T mx) {
-  int e = 0;
-  if (mx > T(0)) frexp((double)mx, &e);
-  return e;
+struct FBits;
+template <>
+struct FBits<double> {
+  static constexpr int kMant = 52, kBias = 1023, kExpMask = 0x7FF;
+};
+template <>
+struct FBits<float> {
+  static constexpr int kMant = 23, kBias = 127, kExpMask = 0xFF;
+};
+
+// Exponent of a row or column holding a non-finite value: its slices are NaN.
+constexpr int kSlNonFinite = 0x40000000;
+
+// Exponent e with |x| < 2^e for every |x| <= the magnitude whose bits are mb
+// (frexp's exponent; 0 for 0, kSlNonFinite for a non-finite maximum).
+template <typename T>
+__device__ __forceinline__ int bound_exp_bits(unsigned long long mb) {
+  using F = FBits<T>;
+  if (mb == 0) return 0;
+  const int E = (int)(mb >> F::kMant);
+  if (E == F::kExpMask) return kSlNonFinite;
+  if (E == 0) {   // subnormal: position of the leading mantissa bit
+    const int lead = 63 - __clzll((long long)mb);
+    return lead - F::kMant - F::kBias + 2;
+  }
+  return E - F::kBias + 1;
 }
 
-// x 2^p, exact (the scale 2^p alone may not be representable: a row of tiny
-// fp32 values has p > 127).
-__device__ __forceinline__ float scale2(float x, int p) { return ldexpf(x, p); }
-__device__ __forceinline__ double scale2(double x, int p) { return ldexp(x, p); }
-
-// Slices of value x (already scaled by 2^-e into [-1, 1]): x_i = I_i 2^(-8 i).
+// Z = round(x 2^(8 S - e)) from the bits of x (|x| < 2^e): |Z| <= 2^(8 S).
 template <int S, typename T>
-__device__ __forceinline__ void make_slices(T y, bf16 (&o)[S]) {
-  T r = y;
-  T sc = T(256);
+__device__ __forceinline__ long long fixed_digits(T x, int e) {
+  using F = FBits<T>;
+  const unsigned long long mb = mag_bits(x);
+  const int E = (int)(mb >> F::kMant);
+  const unsigned long long m = (mb & ((1ull << F::kMant) - 1)) | (E ? (1ull << F::kMant) : 0ull);
+  const int Ee = E ? E : 1;
+  // x = m 2^(Ee - bias - mant); Z = m 2^-sh
+  const int sh = F::kBias + F::kMant + e - 8 * S - Ee;
+  long long Z;
+  if (sh <= 0)
+    Z = (long long)(m << (-sh));   // -sh <= 8 S - mant: no overflow
+  else if (sh >= 63)
+    Z = 0;
+  else
+    Z = (long long)((m + (1ull << (sh - 1))) >> sh);
+  return (mag_bits(x) != raw_bits(x)) ? -Z : Z;   // sign bit set
+}
+
+// The S bf16 slices x_i = I_i 2^(-8 i) of Z 2^(-8 S): balanced base-256
+// digits, I_S..I_2 in [-128, 127], I_1 = what remains (|I_1| <= 256).
+// e = kSlNonFinite gives NaN slices.
+template <int S, typename T>
+__device__ __forceinline__ void digit_slices(T x, int e, bf16 (&o)[S]) {
+  static_assert(S <= 5, "slice scales are built as normal fp32 powers of two");
+  if (e == kSlNonFinite) {
 #pragma unroll
-  for (int i = 0; i < S; ++i) {
-    const T a = rint(r * sc) / sc;   // exact: power-of-two scaling and rounding to an integer
-    o[i] = __float2bfloat16_rn((float)a);
-    r = r - a;                       // exact: the bits of y below slice i
-    sc *= T(256);
+    for (int i = 0; i < S; ++i) o[i] = __ushort_as_bfloat16((unsigned short)0x7FC0);
+    return;
   }
+  long long Z = fixed_digits<S>(x, e);
+#pragma unroll
+  for (int i = S - 1; i >= 1; --i) {
+    const int d = (int)((Z + 128) & 255) - 128;
+    Z = (Z - d) >> 8;
+    o[i] = __float2bfloat16_rn((float)d * __uint_as_float((unsigned)(127 - 8 * (i + 1)) << 23));
+  }
+  o[0] = __float2bfloat16_rn((float)Z * 0x1p-8f);
 }
 
 // Row-sliced operand: X [H][R][K] (rows ldx apart, batches xbs apart) ->
@@ -373,17 +511,17 @@ __global__ void __launch_bounds__(256) slice_rows_kernel(const T* __restrict__ X
   if (gr >= (long long)H * R) return;
   const int b = (int)(gr / R), r = (int)(gr - (long long)b * R);
   const T* x = X + (long long)b * xbs + (long long)r * ldx;
-  T mx = T(0);
-  for (int k = lane; k < K; k += 32) mx = fmax(mx, fabs(x[k]));
+  unsigned long long mb = 0;
+  for (int k = lane; k < K; k += 32) mb = max(mb, mag_bits(x[k]));
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) mx = fmax(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-  const int e = bound_exp(mx);
+  for (int o = 16; o > 0; o >>= 1) mb = max(mb, __shfl_xor_sync(0xffffffffu, mb, o));
+  const int e = bound_exp_bits<T>(mb);
   if (lane == 0) ex[gr] = e;
   const long long slice = (long long)H * R * ldo;
   bf16* o = out + gr * ldo;
   for (int k = lane; k < K; k += 32) {
     bf16 s[S];
-    make_slices<S>(scale2(x[k], -e), s);
+    digit_slices<S>(x[k], e, s);
 #pragma unroll
     for (int i = 0; i < S; ++i) o[i * slice + k] = s[i];
   }
@@ -395,27 +533,27 @@ __global__ void __launch_bounds__(256) slice_rows_kernel(const T* __restrict__ X
 template <typename T>
 __global__ void __launch_bounds__(1024) col_exp_kernel(const T* __restrict__ X, int K, int R, int ldx, long long xbs,
                                                        int* __restrict__ ex) {
-  __shared__ T part[32][33];
+  __shared__ unsigned long long part[32][33];
   const int b = blockIdx.y, lane = threadIdx.x & 31, warp = threadIdx.x >> 5, r = blockIdx.x * 32 + lane;
   const T* x = X + (long long)b * xbs + r;
-  T m0 = T(0), m1 = T(0), m2 = T(0), m3 = T(0);
+  unsigned long long m0 = 0, m1 = 0, m2 = 0, m3 = 0;
   if (r < R) {
     int k = warp;
     for (; k + 96 < K; k += 128) {
-      m0 = fmax(m0, fabs(x[(long long)k * ldx]));
-      m1 = fmax(m1, fabs(x[(long long)(k + 32) * ldx]));
-      m2 = fmax(m2, fabs(x[(long long)(k + 64) * ldx]));
-      m3 = fmax(m3, fabs(x[(long long)(k + 96) * ldx]));
+      m0 = max(m0, mag_bits(x[(long long)k * ldx]));
+      m1 = max(m1, mag_bits(x[(long long)(k + 32) * ldx]));
+      m2 = max(m2, mag_bits(x[(long long)(k + 64) * ldx]));
+      m3 = max(m3, mag_bits(x[(long long)(k + 96) * ldx]));
     }
-    for (; k < K; k += 32) m0 = fmax(m0, fabs(x[(long long)k * ldx]));
+    for (; k < K; k += 32) m0 = max(m0, mag_bits(x[(long long)k * ldx]));
   }
-  part[warp][lane] = fmax(fmax(m0, m1), fmax(m2, m3));
+  part[warp][lane] = max(max(m0, m1), max(m2, m3));
   __syncthreads();
   if (warp == 0 && r < R) {
-    T mx = part[0][lane];
+    unsigned long long mb = part[0][lane];
 #pragma unroll
-    for (int w = 1; w < 32; ++w) mx = fmax(mx, part[w][lane]);
-    ex[(long long)b * R + r] = bound_exp(mx);
+    for (int w = 1; w < 32; ++w) mb = max(mb, part[w][lane]);
+    ex[(long long)b * R + r] = bound_exp_bits<T>(mb);
   }
 }
 
@@ -440,7 +578,7 @@ __global__ void __launch_bounds__(256) slice_cols_kernel(const T* __restrict__ X
     const int r = r0 + q, k = k0 + tx;
     if (r < R && k < K) {
       bf16 s[S];
-      make_slices<S>(scale2(tile[tx][q], -ex[(long long)b * R + r]), s);
+      digit_slices<S>(tile[tx][q], ex[(long long)b * R + r], s);
       const long long o = ((long long)b * R + r) * ldo + k;
 #pragma unroll
       for (int i = 0; i < S; ++i) out[i * slice + o] = s[i];
