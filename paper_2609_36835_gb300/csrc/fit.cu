@@ -1377,30 +1377,148 @@ __global__ void __launch_bounds__(256) chol_back_block_kernel(const double* Linv
   }
 }
 
-// w[b][r] = sum_i Phi[b][i][r] a[b][i] in fp64 (Phi fp32 [n][t]): one thread
-// per column r, the rows of the column read coalesced across the warp.
+// w[b][r] = sum_i Phi[b][i][r] a[b][i] (Phi fp32 [n][t], a fp64): one thread
+// per column r, the rows of the column read coalesced across the warp.  The
+// terms cancel heavily (|a| |Phi| exceeds |w| by ~1e4 on 128K caches), so the
+// sum runs in double-float arithmetic: each product Phi a_hi + Phi a_lo is
+// formed exactly up to the lo part's rounding and added with an error-free
+// sum; a is split into fp32 (hi, lo) pairs in shared memory, 1024 rows at a time.
 __global__ void __launch_bounds__(256) phi_t_vec_kernel(const float* __restrict__ Phi, const double* __restrict__ a,
                                                         float* __restrict__ w, int n, int t) {
+  __shared__ float ah[1024], al[1024];
   const int b = blockIdx.y, r = blockIdx.x * 256 + threadIdx.x;
-  if (r >= t) return;
-  const float* p = Phi + (long long)b * n * t + r;
+  const float* p = Phi + (long long)b * n * t + min(r, t - 1);
   const double* ab = a + (long long)b * n;
-  double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
-  int i = 0;
-  for (; i + 4 <= n; i += 4) {
-    s0 = fma((double)p[(long long)i * t], ab[i], s0);
-    s1 = fma((double)p[(long long)(i + 1) * t], ab[i + 1], s1);
-    s2 = fma((double)p[(long long)(i + 2) * t], ab[i + 2], s2);
-    s3 = fma((double)p[(long long)(i + 3) * t], ab[i + 3], s3);
+  df64 sum(0.f, 0.f);
+  for (int i0 = 0; i0 < n; i0 += 1024) {
+    const int cnt = min(1024, n - i0);
+    __syncthreads();
+    for (int i = threadIdx.x; i < cnt; i += 256) {
+      const double v = ab[i0 + i];
+      const float h = __double2float_rn(v);
+      ah[i] = h;
+      al[i] = __double2float_rn(v - (double)h);
+    }
+    __syncthreads();
+    if (r < t) {
+      for (int i = 0; i < cnt; ++i) {
+        const float x = p[(long long)(i0 + i) * t];
+        const float ph = x * ah[i];
+        const float pl = fmaf(x, al[i], fmaf(x, ah[i], -ph));
+        df64 s2 = df_two(sum.hi, ph);
+        s2.lo += sum.lo + pl;
+        sum = df_fast2(s2.hi, s2.lo);
+      }
+    }
   }
-  for (; i < n; ++i) s0 = fma((double)p[(long long)i * t], ab[i], s0);
-  w[(long long)b * t + r] = (float)((s0 + s1) + (s2 + s3));
+  if (r < t) w[(long long)b * t + r] = sum.hi + sum.lo;
 }
 
 template <typename R>
 __global__ void __launch_bounds__(512) tri_solve_kernel(const R* __restrict__ A, const R* __restrict__ Linv,
                                                         const R* __restrict__ r, R* __restrict__ yd,
                                                         R* __restrict__ x, int t);
+
+// Both substitutions of the single-right-hand-side dual beta system
+// L L^T x = r (the fp64 factor in A's lower triangle, Linv the inverses of its
+// 64 x 64 diagonal blocks) by a cluster of kTsCL CTAs per head: in each block
+// step every rank sums its share of the off-diagonal blocks (block index
+// j = rank mod kTsCL) into rank 0's shared memory, and rank 0 applies the
+// diagonal block's inverse and publishes the block of the solution.  The fp64
+// multiply-adds (n^2 per head) are spread over the cluster's SMs.  Every rank
+// runs the same fixed trip counts, so every cluster barrier is reached by all.
+constexpr int kTsCL = 8;
+__global__ void __cluster_dims__(kTsCL, 1, 1) __launch_bounds__(256, 1)
+    tri_solve_cluster_kernel(const double* __restrict__ A, const double* __restrict__ Linv,
+                             const double* __restrict__ r, double* __restrict__ yd, double* __restrict__ x, int n) {
+  namespace cg = cooperative_groups;
+  __shared__ double red[kTsCL][NB];   // rank 0: the ranks' partial sums
+  __shared__ double part[4][NB];
+  __shared__ double v[NB];
+  const int head = blockIdx.x / kTsCL, rank = (int)cluster_rank(), tid = threadIdx.x;
+  const int nblk = (n + NB - 1) / NB;
+  const double* Ab = A + (long long)head * n * n;
+  const double* Lb = Linv + (long long)head * nblk * NB * NB;
+  const double* rb = r + (long long)head * n;
+  double* y = yd + (long long)head * n;
+  double* xb = x + (long long)head * n;
+  double* red0 = cg::this_cluster().map_shared_rank(&red[0][0], 0);
+  // forward: y_k = Linv_kk (r_k - sum_{j<k} L_kj y_j)
+  for (int k = 0; k < nblk; ++k) {
+    const int k0 = k * NB, kb = min(NB, n - k0);
+    {  // four threads per row of block k
+      const int rr = tid >> 2, pt = tid & 3;
+      double a0 = 0.0, a1 = 0.0;
+      if (rr < kb) {
+        const double* row = Ab + (long long)(k0 + rr) * n;
+        for (int j = rank; j < k; j += kTsCL)
+          for (int c = j * NB + pt; c < j * NB + NB; c += 8) {
+            a0 = fma(__ldcg(row + c), __ldcg(y + c), a0);
+            a1 = fma(__ldcg(row + c + 4), __ldcg(y + c + 4), a1);
+          }
+      }
+      double a = a0 + a1;
+      a += __shfl_xor_sync(0xffffffffu, a, 1);
+      a += __shfl_xor_sync(0xffffffffu, a, 2);
+      if (pt == 0) red0[rank * NB + rr] = a;
+    }
+    cluster_sync_all();
+    if (rank == 0) {
+      if (tid < NB) {
+        double sum = 0.0;
+#pragma unroll
+        for (int q = 0; q < kTsCL; ++q) sum += red[q][tid];
+        v[tid] = tid < kb ? rb[k0 + tid] - sum : 0.0;
+      }
+      __syncthreads();
+      const int c = tid >> 2, pt = tid & 3;   // y_k[c] = sum_{l <= c} Linv_k[c][l] v[l]
+      const double* Li = Lb + (long long)k * NB * NB + c * NB;
+      double a = 0.0;
+      for (int l = pt; l <= c; l += 4) a = fma(__ldcg(Li + l), v[l], a);
+      a += __shfl_xor_sync(0xffffffffu, a, 1);
+      a += __shfl_xor_sync(0xffffffffu, a, 2);
+      if (pt == 0 && c < kb) y[k0 + c] = a;
+    }
+    cluster_sync_all();
+  }
+  // backward: x_k = Linv_kk^T (y_k - sum_{j>k} L_jk^T x_j)
+  for (int k = nblk - 1; k >= 0; --k) {
+    const int k0 = k * NB, kb = min(NB, n - k0);
+    {  // column c of block k, four row groups
+      const int c = tid & (NB - 1), pt = tid >> 6;
+      double a0 = 0.0, a1 = 0.0;
+      if (c < kb)
+        for (int j = k + 1 + rank; j < nblk; j += kTsCL) {
+          const int i1 = min(n, j * NB + NB);
+          for (int i = j * NB + pt; i < i1; i += 8) {
+            a0 = fma(__ldcg(Ab + (long long)i * n + k0 + c), __ldcg(xb + i), a0);
+            if (i + 4 < i1) a1 = fma(__ldcg(Ab + (long long)(i + 4) * n + k0 + c), __ldcg(xb + i + 4), a1);
+          }
+        }
+      part[pt][c] = a0 + a1;
+    }
+    __syncthreads();
+    if (tid < NB) red0[rank * NB + tid] = (part[0][tid] + part[1][tid]) + (part[2][tid] + part[3][tid]);
+    cluster_sync_all();
+    if (rank == 0) {
+      if (tid < NB) {
+        double sum = 0.0;
+#pragma unroll
+        for (int q = 0; q < kTsCL; ++q) sum += red[q][tid];
+        v[tid] = tid < kb ? y[k0 + tid] - sum : 0.0;
+      }
+      __syncthreads();
+      const int c = tid >> 2, pt = tid & 3;   // x_k[c] = sum_{l >= c} Linv_k[l][c] v[l]
+      const double* Li = Lb + (long long)k * NB * NB;
+      double a = 0.0;
+      for (int l = c + pt; l < NB; l += 4) a = fma(__ldcg(Li + (long long)l * NB + c), v[l], a);
+      a += __shfl_xor_sync(0xffffffffu, a, 1);
+      a += __shfl_xor_sync(0xffffffffu, a, 2);
+      if (pt == 0 && c < kb) xb[k0 + c] = a;
+    }
+    cluster_sync_all();
+  }
+}
 
 struct CholSlicedBufs {
   bf16 *sA, *sB, *sC;   // 5-slice operands: panel rows / columns, Linv_kk rows, right-hand-side columns
@@ -1456,10 +1574,9 @@ static int chol_solve_sliced(int H, int n, double* A, double* Linv, double* B, d
     }
   }
   if (nrhs == 1) {
-    // one right-hand side: both substitutions by one CTA per head (fp64 SIMT,
-    // n^2 multiply-adds), the forward result left in W.Z
-    cudaMemsetAsync(X, 0, sizeof(double) * (size_t)H * n, st);
-    tri_solve_kernel<double><<<H, 512, 0, st>>>(A, Linv, B, W.Z, X, n);
+    // one right-hand side: both substitutions by a cluster per head (fp64,
+    // n^2 multiply-adds spread over its SMs), the forward result left in W.Z
+    tri_solve_cluster_kernel<<<H * kTsCL, 256, 0, st>>>(A, Linv, B, W.Z, X, n);
     return nl + 1;
   }
   for (int k = nblk - 1; k >= 0; --k) {

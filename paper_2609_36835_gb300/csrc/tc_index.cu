@@ -14,16 +14,18 @@
 
 namespace arckv {
 
-// Each epilogue thread folds one row of kW columns (kW = 128: four epilogue
-// warps, the whole tile; kW = 64: eight warps, half a tile each) and writes
-// their row-softmax partials, part[b][row][n0 / kW].  kTma: the I tile leaves
-// through TMA stores staged in shared memory (32 x 32 boxes; two buffers per
-// warp with four warps, one with eight); else each row writes its kW values.
-template <bool kTma, int kW_>
+// Each epilogue thread folds one row of kW columns of a kBN-wide tile (kBN / kW
+// warps per TMEM lane quarter: four epilogue warps for 128-wide tiles, eight
+// for 256-wide ones) and writes their row-softmax partials,
+// part[b][row][n0 / kW].  kTma: the I tile leaves through TMA stores staged in
+// shared memory (32 x 32 boxes; two buffers per warp with four warps, one
+// with eight); else each row writes its kW values.
+template <bool kTma, int kW_, int kBN = 128>
 struct TcEpiIndexT {
   static constexpr int kW = kW_;
-  static constexpr int kEpiWarps = 128 / kW * 4;
-  static constexpr int kStageBytes = kTma ? (kW == 128 ? 2 : 1) * 32 * 128 : 0;
+  static constexpr int kEpiWarps = kBN / kW * 4;
+  static constexpr int kNBuf = kEpiWarps == 4 ? 2 : 1;
+  static constexpr int kStageBytes = kTma ? kNBuf * 32 * 128 : 0;
   const float* wts;  // [H][n_pos][H_I]
   float* I;          // [H][n][T]
   float2* part;      // [H][n][ntiles], ntiles = ceil(T / kW)
@@ -84,7 +86,7 @@ struct TcEpiIndexT {
       const int y = row & ~31;
 #pragma unroll
       for (int j = 0; j < kW / 32; ++j)
-        staged_store_32x32<kW == 128 ? 2 : 1>(&map, s.stage, s.stores, n0 + 32 * j, y, b, n, T, s.acc + 32 * j, 1.f);
+        staged_store_32x32<kNBuf>(&map, s.stage, s.stores, n0 + 32 * j, y, b, n, T, s.acc + 32 * j, 1.f);
     } else {
       if (!s.row_ok || nc <= 0) return;
       float* dst = I + ((long long)b * n + row) * T + n0;
@@ -105,13 +107,30 @@ int launch_index_logits(const Dims& D, const bf16* qbar_hi, const bf16* qbar_lo,
                         const bf16* kbar_lo, const float* wts, float* I, float2* part, DevStatus* stt,
                         cudaStream_t st) {
   CUtensorMap mA, mA2, mB, mB2;
+  // 128 x 256 tiles (M = 128, N = 256 MMAs: a quarter fewer operand bytes per
+  // flop than 128 x 128) where T fills them; the key operand's box is 256 rows
+  const bool wide = D.T >= 256;
+  const int bB = wide ? 256 : 128;
   if (!encode_bf16_map_3d(&mA, qbar_hi, D.HD, D.n, D.H, 128) || !encode_bf16_map_3d(&mA2, qbar_lo, D.HD, D.n, D.H, 128) ||
-      !encode_bf16_map_3d(&mB, kbar_hi, D.HD, D.T, D.H, 128) || !encode_bf16_map_3d(&mB2, kbar_lo, D.HD, D.T, D.H, 128))
+      !encode_bf16_map_3d(&mB, kbar_hi, D.HD, D.T, D.H, bB) || !encode_bf16_map_3d(&mB2, kbar_lo, D.HD, D.T, D.H, bB))
     return -1;
   if ((D.T & 3) == 0 && ((uintptr_t)I & 15u) == 0) {
+    if (wide) {
+      TcEpiIndexT<true, kIndexPartW, 256> epi{wts, I, part, D.n, D.T, D.H_I, D.G, D.n_pos, cdiv(D.T, kIndexPartW), {}};
+      if (!encode_f32_map_3d(&epi.map, I, D.T, D.n, D.H, 32, 32, D.T, (uint64_t)D.n * D.T, true)) return -1;
+      if (launch_tc_gemm<256, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.n, D.T, D.HD, 128, stt, st) != cudaSuccess)
+        return -1;
+      return 1;
+    }
     TcEpiIndexT<true, kIndexPartW> epi{wts, I, part, D.n, D.T, D.H_I, D.G, D.n_pos, cdiv(D.T, kIndexPartW), {}};
     if (!encode_f32_map_3d(&epi.map, I, D.T, D.n, D.H, 32, 32, D.T, (uint64_t)D.n * D.T, true)) return -1;
     if (launch_tc_gemm<128, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.n, D.T, D.HD, 128, stt, st) != cudaSuccess)
+      return -1;
+    return 1;
+  }
+  if (wide) {
+    TcEpiIndexT<false, kIndexPartW, 256> epi{wts, I, part, D.n, D.T, D.H_I, D.G, D.n_pos, cdiv(D.T, kIndexPartW), {}};
+    if (launch_tc_gemm<256, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.n, D.T, D.HD, 128, stt, st) != cudaSuccess)
       return -1;
     return 1;
   }
