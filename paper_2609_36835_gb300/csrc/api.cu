@@ -111,7 +111,7 @@ Layout plan(const arckv_config& c) {
   L.kappa = take(H * T * 4);
   L.perm = take(H * T * 4);
   L.goff = take(H * (t + 1) * 4);
-  L.cursor = take(H * t * 4);
+  L.cursor = take((size_t)sort_scratch_ints((int)H, (int)T, (int)t) * 4);
   L.LC = take(H * n * (t > 128 ? t : 128) * f);   // also holds the n x d dual solution when t > n
   L.Phi = take(H * n * t * f);
   const bool dual = t > n;   // the fits run in their n x n dual form

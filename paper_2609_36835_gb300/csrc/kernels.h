@@ -123,6 +123,16 @@ int launch_assign_prep(const Dims& D, const float* L, float* logphi, const int* 
 int launch_assign_gemm(const Dims& D, const int* anchors, const bf16* Ut_hi, const bf16* Ut_lo, const bf16* S_hi,
                        const bf16* S_lo, unsigned long long* best, int* kappa, DevStatus* stt, cudaStream_t st);
 int launch_check_assign(const Dims& D, int* kappa, const int* anchors, DevStatus* stt, cudaStream_t st);
+// The counting sort of the merge runs over chunks of kSortChunk positions
+// when a group histogram fits shared memory; its scratch (`cursor`) then
+// holds sort_scratch_ints(H, T, t) ints.
+constexpr int kSortChunk = 2048;
+constexpr int kSortMaxT = 40 * 1024;
+inline bool sort_chunked(int T, int t) { return t <= kSortMaxT && T > kSortChunk; }
+inline long long sort_scratch_ints(int H, int T, int t) {
+  const long long C = (T + kSortChunk - 1) / kSortChunk;
+  return sort_chunked(T, t) ? (long long)H * t * (C + 1) : (long long)H * t;
+}
 int launch_merge(const Dims& D, float lambda_m, const bf16* K, const int* anchors, const int* kappa,
                  const float* logphi, int* perm, int* goff, int* cursor, float* C_k, cudaStream_t st);
 

@@ -130,6 +130,102 @@ __global__ void __launch_bounds__(1024) group_sort_kernel(const int* kappa, int 
   }
 }
 
+// The same stable counting sort over many CTAs: the positions are cut into
+// chunks of kSortChunk; each chunk counts its members per group (a
+// shared-memory histogram), the counts give every (group, chunk) its first
+// slot in group-major, chunk-minor order, and each chunk then scatters its
+// positions in ascending order from those slots.  perm and goff come out
+// identical to group_sort_kernel's.  cnt is [H][t][C], C = ceil(T / kSortChunk).
+__global__ void __launch_bounds__(1024) sort_hist_kernel(const int* __restrict__ kappa, int T, int t, int C,
+                                                         int* __restrict__ cnt) {
+  extern __shared__ int hist[];
+  const int c = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
+  for (int g = tid; g < t; g += 1024) hist[g] = 0;
+  __syncthreads();
+  const int* kb = kappa + (long long)b * T;
+  const int j1 = min(T, (c + 1) * kSortChunk);
+  // (assignments are in [0, t) by construction and by launch_check_assign;
+  // the clamp keeps the shared-memory index in bounds regardless)
+  for (int j = c * kSortChunk + tid; j < j1; j += 1024) atomicAdd(&hist[min(max(kb[j], 0), t - 1)], 1);
+  __syncthreads();
+  int* cb = cnt + (long long)b * t * C + c;
+  for (int g = tid; g < t; g += 1024) cb[(long long)g * C] = hist[g];
+}
+
+// tot[b][g] = sum over chunks of cnt[b][g][.]
+__global__ void __launch_bounds__(256) sort_totals_kernel(const int* __restrict__ cnt, int t, int C, int H,
+                                                          int* __restrict__ tot) {
+  const long long gi = (long long)blockIdx.x * 256 + threadIdx.x;
+  if (gi >= (long long)H * t) return;
+  const int* row = cnt + gi * C;
+  int a = 0;
+  for (int c = 0; c < C; ++c) a += row[c];
+  tot[gi] = a;
+}
+
+// goff[b] = exclusive scan of tot[b] (one CTA per head); goff[b][t] = T
+__global__ void __launch_bounds__(1024) sort_scan_kernel(const int* __restrict__ tot, int t, int* __restrict__ goff) {
+  __shared__ int sc[32];
+  const int b = blockIdx.x, tid = threadIdx.x;
+  const int* tb = tot + (long long)b * t;
+  int* gb = goff + (long long)b * (t + 1);
+  int base = 0;
+  for (int r0 = 0; r0 < t; r0 += 1024) {
+    const int r = r0 + tid;
+    int total;
+    const int ex = block_excl_scan_1024_m(r < t ? tb[r] : 0, sc, total) + base;
+    if (r < t) gb[r] = ex;
+    base += total;
+  }
+  if (tid == 0) gb[t] = base;
+}
+
+// cnt[b][g][c] <- the first slot of chunk c's members of group g
+__global__ void __launch_bounds__(256) sort_slots_kernel(int* __restrict__ cnt, const int* __restrict__ goff, int t,
+                                                         int C, int H) {
+  const long long gi = (long long)blockIdx.x * 256 + threadIdx.x;
+  if (gi >= (long long)H * t) return;
+  const int b = (int)(gi / t), g = (int)(gi - (long long)b * t);
+  int* row = cnt + gi * C;
+  int run = goff[(long long)b * (t + 1) + g];
+  for (int c = 0; c < C; ++c) {
+    const int k = row[c];
+    row[c] = run;
+    run += k;
+  }
+}
+
+// each chunk's positions, ascending, to their groups' slots
+__global__ void __launch_bounds__(1024) sort_scatter_kernel(const int* __restrict__ kappa, int T, int t, int C,
+                                                            const int* __restrict__ cnt, int* __restrict__ perm) {
+  extern __shared__ int cur[];
+  const int c = blockIdx.x, b = blockIdx.y, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int* cb = cnt + (long long)b * t * C + c;
+  for (int g = tid; g < t; g += 1024) cur[g] = cb[(long long)g * C];
+  __syncthreads();
+  const int* kb = kappa + (long long)b * T;
+  int* pb = perm + (long long)b * T;
+  const unsigned int lt = (1u << lane) - 1u;
+  const int j1 = min(T, (c + 1) * kSortChunk);
+  for (int j0 = c * kSortChunk; j0 < j1; j0 += 1024) {
+    const int j = j0 + tid;
+    const int key = (j < j1) ? min(max(kb[j], 0), t - 1) : -1;
+    const unsigned int peers = __match_any_sync(0xffffffffu, key);
+    const int rank = __popc(peers & lt);
+    const bool leader = (__ffs(peers) - 1) == lane;
+    int pos = 0;
+    for (int w = 0; w < 32; ++w) {   // warps in order: ascending positions within the chunk
+      if (warp == w) {
+        if (key >= 0) pos = cur[key] + rank;
+        __syncwarp();
+        if (key >= 0 && leader) cur[key] += __popc(peers);
+      }
+      __syncthreads();
+    }
+    if (key >= 0) pb[pos] = j;
+  }
+}
+
 constexpr int kMergeWarpMax = 128;
 
 // Groups of more than kMergeWarpMax members (this launch skips the others),
@@ -272,11 +368,27 @@ __global__ void __launch_bounds__(256) group_merge_kernel(const bf16* K, const i
 
 int launch_merge(const Dims& D, float lambda_m, const bf16* K, const int* anchors, const int* kappa,
                  const float* logphi, int* perm, int* goff, int* cursor, float* C_k, cudaStream_t st) {
-  group_sort_kernel<<<D.H, 1024, 0, st>>>(kappa, D.T, D.t, perm, goff, cursor);
+  int nl = 2;
+  const int C = cdiv(D.T, kSortChunk), hb = (int)cdiv((long long)D.H * D.t, 256);
+  const int hsm = D.t * (int)sizeof(int);
+  if (sort_chunked(D.T, D.t) && set_dyn_smem((const void*)sort_hist_kernel, hsm) == cudaSuccess &&
+      set_dyn_smem((const void*)sort_scatter_kernel, hsm) == cudaSuccess) {
+    // cursor: the chunk counts [H][t][C], then the group totals [H][t]
+    int* tot = cursor + (long long)D.H * D.t * C;
+    sort_hist_kernel<<<dim3(C, D.H), 1024, hsm, st>>>(kappa, D.T, D.t, C, cursor);
+    sort_totals_kernel<<<hb, 256, 0, st>>>(cursor, D.t, C, D.H, tot);
+    sort_scan_kernel<<<D.H, 1024, 0, st>>>(tot, D.t, goff);
+    sort_slots_kernel<<<hb, 256, 0, st>>>(cursor, goff, D.t, C, D.H);
+    sort_scatter_kernel<<<dim3(C, D.H), 1024, hsm, st>>>(kappa, D.T, D.t, C, cursor, perm);
+    nl += 5;
+  } else {
+    group_sort_kernel<<<D.H, 1024, 0, st>>>(kappa, D.T, D.t, perm, goff, cursor);
+    ++nl;
+  }
   group_merge_kernel<<<dim3(cdiv(D.t, 8), D.H), 256, 0, st>>>(K, anchors, perm, goff, logphi, lambda_m, C_k, D.T,
                                                               D.t);
   group_merge_cta_kernel<<<dim3(D.t, D.H), 256, 0, st>>>(K, anchors, perm, goff, logphi, lambda_m, C_k, D.T, D.t);
-  return 3;
+  return nl;
 }
 
 }  // namespace arckv

@@ -37,6 +37,8 @@ __device__ __forceinline__ int block_excl_scan_1024(int v, int* sc, int& total) 
 // score, plus the lowest-position ones among those equal to the threshold
 // (ties -> lower position), written in ascending position order after the
 // anchors of the chunks before it.  L = 0: one chunk, the whole cache, t_c = t.
+constexpr int kSelE = 8;   // consecutive scores per thread per round
+
 __global__ void __launch_bounds__(1024) top_t_kernel(const float* s, int Tall, int tb, int L, int tp, int* anchors,
                                                      DevStatus* stt) {
   const int b = blockIdx.y, c = blockIdx.x, tid = threadIdx.x;
@@ -59,11 +61,17 @@ __global__ void __launch_bounds__(1024) top_t_kernel(const float* s, int Tall, i
     const int shift = 24 - 8 * pass;
     if (tid < 256) hist[tid] = 0;
     __syncthreads();
-    for (int j = tid; j < T; j += 1024) {
-      const float v = sb[j];
-      if (pass == 0 && !isfinite(v)) set_status(stt, ARCKV_ERR_NONFINITE);
-      const unsigned int key = f32_ordered(v);
-      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1);
+    for (int j0 = tid * kSelE; j0 < T; j0 += 1024 * kSelE) {   // kSelE consecutive scores per thread
+      float v[kSelE];
+#pragma unroll
+      for (int q = 0; q < kSelE; ++q) v[q] = j0 + q < T ? sb[j0 + q] : 0.f;
+#pragma unroll
+      for (int q = 0; q < kSelE; ++q) {
+        if (j0 + q >= T) break;
+        if (pass == 0 && !isfinite(v[q])) set_status(stt, ARCKV_ERR_NONFINITE);
+        const unsigned int key = f32_ordered(v[q]);
+        if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1);
+      }
     }
     __syncthreads();
     if (tid == 0) {
@@ -80,16 +88,34 @@ __global__ void __launch_bounds__(1024) top_t_kernel(const float* s, int Tall, i
     rem = sh_rem;
     mask |= 0xffu << shift;
   }
+  // compaction, kSelE consecutive positions per thread per round: threads in
+  // order, each thread's positions in order, so the output stays ascending
   int base = 0, eqseen = 0;
-  for (int j0 = 0; j0 < T; j0 += 1024) {
-    const int j = j0 + tid;
-    const unsigned int key = (j < T) ? f32_ordered(sb[j]) : 0u;
-    const int eq = (j < T && key == prefix) ? 1 : 0;
+  for (int r0 = 0; r0 < T; r0 += 1024 * kSelE) {
+    const int jb = r0 + tid * kSelE;
+    unsigned int key[kSelE];
+    int neq = 0;
+#pragma unroll
+    for (int q = 0; q < kSelE; ++q) {
+      key[q] = jb + q < T ? f32_ordered(sb[jb + q]) : 0u;
+      neq += (jb + q < T && key[q] == prefix) ? 1 : 0;
+    }
     int eqtot, tot;
-    const int eqrank = block_excl_scan_1024(eq, sc, eqtot) + eqseen;
-    const int take = (j < T && (key > prefix || (eq && eqrank < rem))) ? 1 : 0;
-    const int pos = block_excl_scan_1024(take, sc, tot) + base;
-    if (take && pos < t) out[pos] = cstart + j;
+    int eqrank = block_excl_scan_1024(neq, sc, eqtot) + eqseen;
+    unsigned int take = 0u;
+#pragma unroll
+    for (int q = 0; q < kSelE; ++q) {
+      const bool in = jb + q < T, eq = in && key[q] == prefix;
+      if (in && (key[q] > prefix || (eq && eqrank < rem))) take |= 1u << q;
+      eqrank += eq ? 1 : 0;
+    }
+    int pos = block_excl_scan_1024(__popc(take), sc, tot) + base;
+#pragma unroll
+    for (int q = 0; q < kSelE; ++q)
+      if ((take >> q) & 1u) {
+        if (pos < t) out[pos] = cstart + jb + q;
+        ++pos;
+      }
     base += tot;
     eqseen += eqtot;
   }
