@@ -30,13 +30,14 @@
 // arithmetic of the tensor pipe never meets a rounding that matters.
 //
 // Kernel layout (persistent, one CTA per SM): warp 0 streams 32-wide K slabs
-// of the S slices of a 128-row A tile and a 64-row B tile with TMA (64-byte
+// of the S slices of a 128-row A tile and a BN-row B tile with TMA (64-byte
 // swizzle) into a shared ring; warp 1 issues the S^2 tcgen05 MMAs (M = 128,
-// N = 64, K = 16) of every K step into the level accumulators (the exact
-// levels of two alternating chunks, the higher levels of two alternating
-// tiles: 512 TMEM columns); warps 2..9 drain the exact levels after every
-// chunk (two warps per TMEM lane quarter, 32 columns each) and assemble the
-// tile while the MMAs of the next tile run.
+// N = BN, K = 16) of every K step into the level accumulators; the epilogue
+// warps (32 columns each) drain the exact levels after every chunk and
+// assemble the tile.  With BN = 64 the accumulators are double-buffered (the
+// exact levels of two alternating chunks, the higher levels of two
+// alternating tiles: 512 TMEM columns), so a tile is assembled while the next
+// one's MMAs run; with BN = 128 they fill the 512 columns once (SlShape).
 #include <algorithm>
 
 #include "kernels.h"
@@ -46,11 +47,9 @@ namespace arckv {
 
 namespace {
 
-constexpr int kSlBM = 128, kSlBN = 64, kSlBK = 32;   // tile rows, columns, K slab
+constexpr int kSlBM = 128, kSlBK = 32;   // tile rows, K slab
 constexpr int kSlChunkSlabs = 4;                      // 128 K per exact chunk
-constexpr int kSlEpiWarps = 8;
-constexpr int kSlThreads = 64 + 32 * kSlEpiWarps;
-constexpr int kSlTileA = kSlBM * kSlBK * 2, kSlTileB = kSlBN * kSlBK * 2;   // 8 KB, 4 KB
+constexpr int kSlTileA = kSlBM * kSlBK * 2;   // 8 KB
 
 // Each epilogue warp stages its 32 rows x 16 columns of results (rows padded
 // to 17 elements) in shared memory and writes them back row-contiguously, so
@@ -58,14 +57,38 @@ constexpr int kSlTileA = kSlBM * kSlBK * 2, kSlTileB = kSlBN * kSlBK * 2;   // 8
 constexpr int kSlStageLd = 17;
 constexpr int kSlStageBytes = 32 * kSlStageLd * 8;
 
-template <int S>
+// Tile shapes.  BN = 64: eight epilogue warps, the exact-level and the
+// high-level accumulators double-buffered in TMEM (6 x 64 + 2 x 64 columns), the
+// results staged per warp for coalesced stores; for the short-K block
+// products of the Cholesky, where each tile's epilogue overlaps the next
+// tile's MMAs.  BN = 128: each MMA reads as many operand bytes as its tensor
+// time allows (an N = 64 MMA reads more per cycle than shared memory
+// delivers), sixteen epilogue warps (32 columns each), single-buffered
+// accumulators (3 x 128 + 128 columns) and plain stores; for the long-K Grams
+// and back-projections, whose epilogue runs once per tile.
+template <int BN_>
+struct SlShape {
+  static constexpr int BN = BN_;
+  static constexpr int EW = BN == 64 ? 8 : 16;              // epilogue warps
+  static constexpr int THREADS = 64 + 32 * EW;
+  static constexpr int NBUF = BN == 64 ? 2 : 1;             // accumulator buffers
+  static constexpr bool STAGED = BN == 64;
+  static constexpr int TILE_B = BN * kSlBK * 2;
+  static constexpr int COLT = kSlBM / BN;                   // column tiles per row tile (lower mode)
+  static_assert(BN == 64 || BN == 128, "tile widths");
+  static_assert(3 * NBUF * BN + NBUF * BN <= 512, "TMEM columns");
+};
+
+template <int S, int BN>
 struct SlCfg {
-  static constexpr int STAGE = S * (kSlTileA + kSlTileB);
+  using Sh = SlShape<BN>;
+  static constexpr int STAGE_BYTES = Sh::STAGED ? Sh::EW * kSlStageBytes : 0;
+  static constexpr int STAGE = S * (kSlTileA + Sh::TILE_B);
   // the ring takes what the staging tiles, the 1 KB alignment slack and 1 KB
   // of static barriers leave of the 227 KB a CTA may hold
-  static constexpr int RING = 227 * 1024 - 2048 - kSlEpiWarps * kSlStageBytes;
+  static constexpr int RING = 227 * 1024 - 2048 - STAGE_BYTES;
   static constexpr int STAGES = std::min(6, RING / STAGE);
-  static constexpr int SMEM = STAGES * STAGE + 1024 + kSlEpiWarps * kSlStageBytes;
+  static constexpr int SMEM = STAGES * STAGE + 1024 + STAGE_BYTES;
   static_assert(STAGES >= 2, "two ring stages at least");
 };
 
@@ -167,10 +190,22 @@ __device__ __forceinline__ void sl_store_rows(const Out& out, typename Out::Elem
   __syncwarp();
 }
 
+// The same 16 values of one row (row < M), written by their own thread.
+template <class Out, class F>
+__device__ __forceinline__ void sl_store_direct(const Out& out, int b, int row, int c0, int M, int N, F&& val) {
+  if (row >= M) return;
+#pragma unroll
+  for (int e = 0; e < 16; ++e)
+    if (c0 + e < N) {
+      auto* d = out.at(b, row, c0 + e);
+      out.put(d, out.old(d), out.make(val(e)));
+    }
+}
+
 // Tiles of one batch: all (row tile, column tile) pairs, or with `lower` only
 // those that reach the lower triangle (column tile start <= row tile end) of a
-// square product; column tiles fastest.
-__device__ __forceinline__ void sl_tile(int tl, int Mt, int Nt, bool lower, int& b, int& mt, int& nt) {
+// square product (ct column tiles per row tile); column tiles fastest.
+__device__ __forceinline__ void sl_tile(int tl, int Mt, int Nt, bool lower, int ct, int& b, int& mt, int& nt) {
   if (!lower) {
     b = tl / (Mt * Nt);
     const int r = tl - b * (Mt * Nt);
@@ -179,24 +214,25 @@ __device__ __forceinline__ void sl_tile(int tl, int Mt, int Nt, bool lower, int&
     return;
   }
   int per = 0;
-  for (int i = 0; i < Mt; ++i) per += min(Nt, 2 * (i + 1));
+  for (int i = 0; i < Mt; ++i) per += min(Nt, ct * (i + 1));
   b = tl / per;
   int r = tl - b * per;
   mt = 0;
-  while (r >= min(Nt, 2 * (mt + 1))) {
-    r -= min(Nt, 2 * (mt + 1));
+  while (r >= min(Nt, ct * (mt + 1))) {
+    r -= min(Nt, ct * (mt + 1));
     ++mt;
   }
   nt = r;
 }
 
-template <int S, class Out>
-__global__ void __launch_bounds__(kSlThreads, 1)
+template <int S, class Out, int BN>
+__global__ void __launch_bounds__(SlShape<BN>::THREADS, 1)
     sliced_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB, const Out out,
                        const int* __restrict__ eA, const int* __restrict__ eB, int H, int M, int N, int K, int lower,
                        DevStatus* stt) {
-  using C = SlCfg<S>;
-  constexpr int STAGES = C::STAGES;
+  using C = SlCfg<S, BN>;
+  using Sh = SlShape<BN>;
+  constexpr int STAGES = C::STAGES, EW = Sh::EW, NBUF = Sh::NBUF, TILE_B = Sh::TILE_B;
   extern __shared__ uint8_t smem_raw[];
   __shared__ uint64_t full[STAGES], empty[STAGES], accf[2], acce[2], l5f[2], l5e[2], drain;
   __shared__ uint32_t tmem_slot;
@@ -206,10 +242,10 @@ __global__ void __launch_bounds__(kSlThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nk = (K + kSlBK - 1) / kSlBK;
   const int nchunks = (nk + kSlChunkSlabs - 1) / kSlChunkSlabs;
-  const int Mt = (M + kSlBM - 1) / kSlBM, Nt = (N + kSlBN - 1) / kSlBN;
+  const int Mt = (M + kSlBM - 1) / kSlBM, Nt = (N + BN - 1) / BN;
   int per = 0;
   if (lower) {
-    for (int i = 0; i < Mt; ++i) per += min(Nt, 2 * (i + 1));
+    for (int i = 0; i < Mt; ++i) per += min(Nt, Sh::COLT * (i + 1));
   } else {
     per = Mt * Nt;
   }
@@ -222,9 +258,9 @@ __global__ void __launch_bounds__(kSlThreads, 1)
     }
     for (int i = 0; i < 2; ++i) {
       tc::mbar_init(&accf[i], 1);
-      tc::mbar_init(&acce[i], kSlEpiWarps);
+      tc::mbar_init(&acce[i], EW);
       tc::mbar_init(&l5f[i], 1);
-      tc::mbar_init(&l5e[i], kSlEpiWarps);
+      tc::mbar_init(&l5e[i], EW);
     }
     tc::mbar_init(&drain, 1);
     abort_flag = 0;
@@ -247,7 +283,7 @@ __global__ void __launch_bounds__(kSlThreads, 1)
       bool ok = true;
       for (int tl = blockIdx.x; tl < ntiles && ok; tl += gridDim.x) {
         int b, mt, nt;
-        sl_tile(tl, Mt, Nt, lower != 0, b, mt, nt);
+        sl_tile(tl, Mt, Nt, lower != 0, Sh::COLT, b, mt, nt);
         for (int kb = 0; kb < nk; ++kb) {
           const int s = g % STAGES;
           if (g >= STAGES && !tc::mbar_wait(&empty[s], ((g / STAGES) - 1) & 1, abortp, stt)) {
@@ -259,7 +295,7 @@ __global__ void __launch_bounds__(kSlThreads, 1)
 #pragma unroll
           for (int i = 0; i < S; ++i) {
             tc::tma_load_3d(st + i * kSlTileA, &mA, kb * kSlBK, mt * kSlBM, i * H + b, &full[s]);
-            tc::tma_load_3d(st + S * kSlTileA + i * kSlTileB, &mB, kb * kSlBK, nt * kSlBN, i * H + b, &full[s]);
+            tc::tma_load_3d(st + S * kSlTileA + i * TILE_B, &mB, kb * kSlBK, nt * BN, i * H + b, &full[s]);
           }
           ++g;
         }
@@ -270,22 +306,22 @@ __global__ void __launch_bounds__(kSlThreads, 1)
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      constexpr uint32_t idesc = tc::idesc_bf16_f32(kSlBN);
+      constexpr uint32_t idesc = tc::idesc_bf16_f32(BN);
       bool ok = true;
       int g = 0, cg = 0, tcount = 0;
       for (int tl = blockIdx.x; tl < ntiles && ok; tl += gridDim.x, ++tcount) {
-        // the level-5+ accumulator of this parity must have been read (two tiles ago)
-        const int b5 = tcount & 1;
-        if (tcount >= 2 && !tc::mbar_wait(&l5e[b5], ((tcount >> 1) - 1) & 1, abortp, stt)) {
+        // the level-5+ accumulator of this buffer must have been read (NBUF tiles ago)
+        const int b5 = tcount % NBUF, u5 = tcount / NBUF;
+        if (u5 >= 1 && !tc::mbar_wait(&l5e[b5], (u5 - 1) & 1, abortp, stt)) {
           ok = false;
           break;
         }
         tc::fence_after_sync();
-        const uint32_t t5 = tmem + 384u + (uint32_t)(b5 * 64);
+        const uint32_t t5 = tmem + (uint32_t)((3 * NBUF + b5) * BN);
         bool started5 = false;
         for (int c = 0; c < nchunks && ok; ++c, ++cg) {
-          const int buf = cg & 1;
-          if (cg >= 2 && !tc::mbar_wait(&acce[buf], ((cg >> 1) - 1) & 1, abortp, stt)) {
+          const int buf = cg % NBUF, ub = cg / NBUF;
+          if (ub >= 1 && !tc::mbar_wait(&acce[buf], (ub - 1) & 1, abortp, stt)) {
             ok = false;
             break;
           }
@@ -307,10 +343,10 @@ __global__ void __launch_bounds__(kSlThreads, 1)
                 const uint64_t ad = tc::sdesc_k64(a + i * kSlTileA + ks * 32);
 #pragma unroll
                 for (int j = 0; j < S; ++j) {
-                  const uint64_t bd = tc::sdesc_k64(bb + j * kSlTileB + ks * 32);
+                  const uint64_t bd = tc::sdesc_k64(bb + j * TILE_B + ks * 32);
                   const int lvl = i + j;   // 0-based: level l = lvl + 2
                   if (lvl <= 2) {
-                    tc::mma_f16(tmem + (uint32_t)((buf * 3 + lvl) * 64), ad, bd, idesc, started[lvl] ? 1u : 0u);
+                    tc::mma_f16(tmem + (uint32_t)((buf * 3 + lvl) * BN), ad, bd, idesc, started[lvl] ? 1u : 0u);
                     started[lvl] = true;
                   } else {
                     tc::mma_f16(t5, ad, bd, idesc, started5 ? 1u : 0u);
@@ -331,22 +367,22 @@ __global__ void __launch_bounds__(kSlThreads, 1)
     }
   } else {
     const int q = warp & 3;                 // TMEM lane quarter
-    const int half = (warp - 2) >> 2;       // 32-column half of the 64-wide tile
+    const int part = (warp - 2) >> 2;       // 32-column part of the tile
     const int row_in = q * 32 + lane;
     bool ok = true;
     int kc = 0, tcount = 0;
     for (int tl = blockIdx.x; tl < ntiles && ok; tl += gridDim.x, ++tcount) {
       int b, mt, nt;
-      sl_tile(tl, Mt, Nt, lower != 0, b, mt, nt);
+      sl_tile(tl, Mt, Nt, lower != 0, Sh::COLT, b, mt, nt);
       // exact running sum of levels 2..4 in units of 2^-32: level l contributes
       // its integer chunk sums shifted left by 8 (4 - l) bits (|sum| < 2^47)
-      out.prefetch(b, mt * kSlBM + row_in, nt * kSlBN + half * 32, M, N);
+      out.prefetch(b, mt * kSlBM + row_in, nt * BN + part * 32, M, N);
       long long acc[32];
 #pragma unroll
       for (int e = 0; e < 32; ++e) acc[e] = 0;
       for (int c = 0; c < nchunks; ++c, ++kc) {
-        const int buf = kc & 1;
-        ok = tc::mbar_wait(&accf[buf], (kc >> 1) & 1, abortp, stt);
+        const int buf = kc % NBUF;
+        ok = tc::mbar_wait(&accf[buf], (kc / NBUF) & 1, abortp, stt);
         ok = __all_sync(0xffffffffu, ok);
         if (!ok) break;
         tc::fence_after_sync();
@@ -358,7 +394,7 @@ __global__ void __launch_bounds__(kSlThreads, 1)
 #pragma unroll
           for (int p2 = 0; p2 < 2; ++p2) {
             float v[16];
-            tc::tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)((buf * 3 + l) * 64 + half * 32 + p2 * 16), v);
+            tc::tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)((buf * 3 + l) * BN + part * 32 + p2 * 16), v);
 #pragma unroll
             for (int e = 0; e < 16; ++e) acc[p2 * 16 + e] += (long long)__float2int_rn(v[e] * sc) << sh;
           }
@@ -368,12 +404,12 @@ __global__ void __launch_bounds__(kSlThreads, 1)
         if (lane == 0) tc::mbar_arrive(&acce[buf]);
       }
       if (!ok) break;
-      const int b5 = tcount & 1;
-      ok = __all_sync(0xffffffffu, tc::mbar_wait(&l5f[b5], (tcount >> 1) & 1, abortp, stt));
+      const int b5 = tcount % NBUF;
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(&l5f[b5], (tcount / NBUF) & 1, abortp, stt));
       if (!ok) break;
       tc::fence_after_sync();
       float v5[2][16];
-      const uint32_t t5 = tmem + ((uint32_t)(q * 32) << 16) + 384u + (uint32_t)(b5 * 64 + half * 32);
+      const uint32_t t5 = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)((3 * NBUF + b5) * BN + part * 32);
       tc::tmem_ld16(t5, v5[0]);
       tc::tmem_ld16(t5 + 16u, v5[1]);
       tc::fence_before_sync();
@@ -382,7 +418,7 @@ __global__ void __launch_bounds__(kSlThreads, 1)
       const int row = mt * kSlBM + row_in;
       const int er = row < M ? eA[(long long)b * M + row] : 0;
       typename Out::Elem* stg =
-          (typename Out::Elem*)(base + C::STAGES * C::STAGE + (warp - 2) * kSlStageBytes);
+          Sh::STAGED ? (typename Out::Elem*)(base + C::STAGES * C::STAGE + (warp - 2) * kSlStageBytes) : nullptr;
       const int* ecol = eB + (long long)b * N;
       // the sum in units of 2^-44: the exact levels (|acc| < 2^47 in units
       // of 2^-32) and the levels above 4 (|v5| < 2^-8) rounded to the unit,
@@ -400,14 +436,18 @@ __global__ void __launch_bounds__(kSlThreads, 1)
       }
 #pragma unroll
       for (int p2 = 0; p2 < 2; ++p2) {
-        const int c0 = nt * kSlBN + half * 32 + p2 * 16;
+        const int c0 = nt * BN + part * 32 + p2 * 16;
         int ec[16];
 #pragma unroll
         for (int e = 0; e < 16; ++e) ec[e] = c0 + e < N ? ecol[c0 + e] : 0;
-        sl_store_rows(out, stg, lane, b, mt * kSlBM + q * 32, c0, M, N, [&](int e) -> SlVal {
+        auto val = [&](int e) -> SlVal {
           if ((nanmask >> (p2 * 16 + e)) & 1u) return SlVal{0, kSlNaN};
           return SlVal{acc[p2 * 16 + e], er + ec[e] - 44};
-        });
+        };
+        if constexpr (Sh::STAGED)
+          sl_store_rows(out, stg, lane, b, mt * kSlBM + q * 32, c0, M, N, val);
+        else
+          sl_store_direct(out, b, row, c0, M, N, val);
       }
     }
   }
@@ -588,31 +628,32 @@ __global__ void __launch_bounds__(256) slice_cols_kernel(const T* __restrict__ X
 
 int g_sliced_fail = 0;   // which step of the last failed launch_sliced gave up (diagnostics)
 
-template <int S, class Out>
+template <int S, int BN, class Out>
 int launch_sliced(const bf16* As, const int* eA, int M, const bf16* Bs, const int* eB, int N, int K, int ldk, int H,
                   bool lower, const Out& out, DevStatus* stt, cudaStream_t st) {
   CUtensorMap mA, mB;
   if (!encode_bf16_map_3d_sw64(&mA, As, K, M, (uint64_t)S * H, ldk, kSlBM) ||
-      !encode_bf16_map_3d_sw64(&mB, Bs, K, N, (uint64_t)S * H, ldk, kSlBN)) {
+      !encode_bf16_map_3d_sw64(&mB, Bs, K, N, (uint64_t)S * H, ldk, BN)) {
     g_sliced_fail = 1;
     return -1;
   }
-  using C = SlCfg<S>;
-  auto kern = sliced_gemm_kernel<S, Out>;
+  using C = SlCfg<S, BN>;
+  using Sh = SlShape<BN>;
+  auto kern = sliced_gemm_kernel<S, Out, BN>;
   const cudaError_t ea = set_dyn_smem((const void*)kern, C::SMEM);
   if (ea != cudaSuccess) {
     g_sliced_fail = 100 + (int)ea;
     return -1;
   }
-  const int Mt = cdiv(M, kSlBM), Nt = cdiv(N, kSlBN);
+  const int Mt = cdiv(M, kSlBM), Nt = cdiv(N, BN);
   long long per = 0;
   if (lower) {
-    for (int i = 0; i < Mt; ++i) per += std::min(Nt, 2 * (i + 1));
+    for (int i = 0; i < Mt; ++i) per += std::min(Nt, Sh::COLT * (i + 1));
   } else {
     per = (long long)Mt * Nt;
   }
   const int grid = (int)std::min<long long>(per * H, tc_gemm_sm_count());
-  kern<<<grid, kSlThreads, C::SMEM, st>>>(mA, mB, out, eA, eB, H, M, N, K, lower ? 1 : 0, stt);
+  kern<<<grid, Sh::THREADS, C::SMEM, st>>>(mA, mB, out, eA, eB, H, M, N, K, lower ? 1 : 0, stt);
   const cudaError_t el = cudaGetLastError();
   if (el != cudaSuccess) g_sliced_fail = 1000 + (int)el;
   return el == cudaSuccess ? 1 : -1;
@@ -683,13 +724,23 @@ int launch_sliced_gram_lower(int S, const bf16* Xs, const int* ex, int R, int K,
   return launch_sliced_f64(S, Xs, ex, R, Xs, ex, R, K, H, G, (long long)R * R, R, true, false, stt, st);
 }
 
+// 128-wide tiles for the long-K products of up to four slices (the Grams and
+// back-projections: the epilogue runs once per many chunks), 64-wide ones for
+// the short-K block products of the Cholesky.
+static bool sliced_wide(int S, int K) { return S <= 4 && K >= 256; }
+
 int launch_sliced_f64(int S, const bf16* As, const int* eA, int M, const bf16* Bs, const int* eB, int N, int K, int H,
                       double* C, long long cbs, int ldc, bool lower, bool sub, DevStatus* stt, cudaStream_t st) {
   const int ldk = (int)sliced_ld(K);
   const SlOutF64 out{C, cbs, ldc, sub ? 1 : 0};
-  if (S == 3) return launch_sliced<3>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st);
-  if (S == 4) return launch_sliced<4>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st);
-  if (S == 5) return launch_sliced<5>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st);
+  const bool w = sliced_wide(S, K);
+  if (S == 3)
+    return w ? launch_sliced<3, 128>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st)
+             : launch_sliced<3, 64>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st);
+  if (S == 4)
+    return w ? launch_sliced<4, 128>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st)
+             : launch_sliced<4, 64>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st);
+  if (S == 5) return launch_sliced<5, 64>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st);
   return -1;
 }
 
@@ -697,8 +748,13 @@ int launch_sliced_product_f32(int S, const bf16* As, const int* eA, int M, const
                               int H, float* C, int ldc, DevStatus* stt, cudaStream_t st) {
   const int ldk = (int)sliced_ld(K);
   const SlOutF32 out{C, (long long)M * ldc, ldc};
-  if (S == 3) return launch_sliced<3>(As, eA, M, Bs, eB, N, K, ldk, H, false, out, stt, st);
-  if (S == 4) return launch_sliced<4>(As, eA, M, Bs, eB, N, K, ldk, H, false, out, stt, st);
+  const bool w = sliced_wide(S, K);
+  if (S == 3)
+    return w ? launch_sliced<3, 128>(As, eA, M, Bs, eB, N, K, ldk, H, false, out, stt, st)
+             : launch_sliced<3, 64>(As, eA, M, Bs, eB, N, K, ldk, H, false, out, stt, st);
+  if (S == 4)
+    return w ? launch_sliced<4, 128>(As, eA, M, Bs, eB, N, K, ldk, H, false, out, stt, st)
+             : launch_sliced<4, 64>(As, eA, M, Bs, eB, N, K, ldk, H, false, out, stt, st);
   return -1;
 }
 
