@@ -20,7 +20,7 @@ inline size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct Layout {
   size_t status, kbar_hi, kbar_lo, vq, qpp, q_h, q_m, q_l, av, VT, p_h, p_m, p_l, vq3, av3, ukt, qbar_hi, qbar_lo, wts, NT, rA, rB, part, lse, s, anchors, z, m, invm, Y, logphi,
-      qcat, wcat, Ut_hi, Ut_lo, S_hi, S_lo, best, kappa, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z,
+      qcat, wcat, Ut_hi, Ut_lo, S_hi, S_lo, best, kappa, kmap, perm, goff, cursor, LC, Phi, Gram, Linv, rhs, wsol, R, Z,
       ck3, YT_hi, YT_lo, G64, L64, B64, Z64, X64, Sl, Sl2, eR, eC, ir_u, ir_sq, ir_lam, Sl3, eC2, cl_lam, total;
 };
 
@@ -109,6 +109,7 @@ Layout plan(const arckv_config& c) {
   L.S_lo = take(H * t * ldn * 2);
   L.best = take(H * T * 8);
   L.kappa = take(H * T * 4);
+  L.kmap = take(H * T * 4);
   L.perm = take(H * T * 4);
   L.goff = take(H * (t + 1) * 4);
   L.cursor = take((size_t)sort_scratch_ints((int)H, (int)T, (int)t) * 4);
@@ -353,15 +354,15 @@ arckv_status arckv_compact(const arckv_config* cfg, const void* K, const void* V
   mark(4);
   if (!given_assign) {
     const int nla = launch_assign_prep(D, F(L.NT), F(L.logphi), anchors, B16(L.Ut_hi), B16(L.Ut_lo), B16(L.S_hi),
-                                       B16(L.S_lo), stt, st);
+                                       B16(L.S_lo), I32(L.kmap), stt, st);
     if (nla < 0) return ARCKV_ERR_CUDA;
     mark(5);
     const int nlg = launch_assign_gemm(D, anchors, B16(L.Ut_hi), B16(L.Ut_lo), B16(L.S_hi), B16(L.S_lo),
-                                       (unsigned long long*)(w + L.best), kappa, stt, st);
+                                       I32(L.kmap), (unsigned long long*)(w + L.best), kappa, stt, st);
     if (nlg < 0) return ARCKV_ERR_CUDA;
     nl += nla + nlg;
   } else {
-    const int nlc = launch_col_profiles(D, F(L.NT), F(L.logphi), nullptr, nullptr, stt, st);   // log phi only
+    const int nlc = launch_col_profiles(D, F(L.NT), F(L.logphi), stt, st);   // log phi only
     if (nlc < 0) return ARCKV_ERR_CUDA;
     nl += nlc;
     mark(5);

@@ -113,15 +113,18 @@ int launch_reference_attention(const Dims& D, float scale, const bf16* Q, const 
 int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* K, float* L, float2* part,
                          DevStatus* stt, cudaStream_t st);
 // Column statistics of the reference logits L: log phi [H][T] (mass weights of
-// the merge) and, when Ut_hi is given, the transposed split-bf16 profiles.
-int launch_col_profiles(const Dims& D, const float* L, float* logphi, bf16* Ut_hi, bf16* Ut_lo, DevStatus* stt,
-                        cudaStream_t st);
-// Assignment on tcgen05: column statistics and transposed split-bf16 profiles
-// (log phi written on the way) and the anchor rows; then the argmax GEMM.
+// the merge) alone.
+int launch_col_profiles(const Dims& D, const float* L, float* logphi, DevStatus* stt, cudaStream_t st);
+// Assignment on tcgen05: column statistics (log phi written on the way) and
+// the transposed split-bf16 profiles, the anchors' into the anchor rows S and
+// the other keys' compacted into the first T - t rows of Ut (kmap: row -> key);
+// then the argmax GEMM over the compacted rows (the anchors' own kappa(s_r) = r
+// is set directly).
 int launch_assign_prep(const Dims& D, const float* L, float* logphi, const int* anchors, bf16* Ut_hi, bf16* Ut_lo,
-                       bf16* S_hi, bf16* S_lo, DevStatus* stt, cudaStream_t st);
+                       bf16* S_hi, bf16* S_lo, int* kmap, DevStatus* stt, cudaStream_t st);
 int launch_assign_gemm(const Dims& D, const int* anchors, const bf16* Ut_hi, const bf16* Ut_lo, const bf16* S_hi,
-                       const bf16* S_lo, unsigned long long* best, int* kappa, DevStatus* stt, cudaStream_t st);
+                       const bf16* S_lo, const int* kmap, unsigned long long* best, int* kappa, DevStatus* stt,
+                       cudaStream_t st);
 int launch_check_assign(const Dims& D, int* kappa, const int* anchors, DevStatus* stt, cudaStream_t st);
 // The counting sort of the merge runs over chunks of kSortChunk positions
 // when a group histogram fits shared memory; its scratch (`cursor`) then

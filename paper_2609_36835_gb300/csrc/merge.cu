@@ -97,7 +97,7 @@ __global__ void __launch_bounds__(1024) group_sort_kernel(const int* kappa, int 
   __shared__ int sc[32];
   for (int r = tid; r < t; r += 1024) cb[r] = 0;
   __syncthreads();
-  for (int j = tid; j < T; j += 1024) atomicAdd(&cb[kb[j]], 1);
+  for (int j = tid; j < T; j += 1024) atomicAdd(&cb[min(max(kb[j], 0), t - 1)], 1);   // (in range by construction)
   __syncthreads();
   int base = 0;
   for (int r0 = 0; r0 < t; r0 += 1024) {
@@ -113,7 +113,7 @@ __global__ void __launch_bounds__(1024) group_sort_kernel(const int* kappa, int 
   const unsigned int lt = (1u << lane) - 1u;
   for (int j0 = 0; j0 < T; j0 += 1024) {
     const int j = j0 + tid;
-    const int key = (j < T) ? kb[j] : -1;
+    const int key = (j < T) ? min(max(kb[j], 0), t - 1) : -1;
     const unsigned int peers = __match_any_sync(0xffffffffu, key);
     const int rank = __popc(peers & lt);
     const bool leader = (__ffs(peers) - 1) == lane;

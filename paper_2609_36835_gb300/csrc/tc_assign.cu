@@ -60,6 +60,38 @@ int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* 
   return 1;
 }
 
+// Where key j's profile row goes.  An anchor's (anchors[r] == j) to row r of
+// the anchor rows U_S^T; every other key to row j - #{anchors < j} of the
+// compacted key rows, the T - t rows the assignment GEMM takes as M: the
+// anchors' own assignment is fixed, kappa(s_r) = r, so their GEMM rows would
+// only be discarded.  ab: the head's anchors, ascending (checked upstream).
+// The element offset of that row (an anchor row as -1 - offset), or
+// kNoRow when invalid anchors (a caller's, already flagged
+// ARCKV_ERR_INVALID_ARG) leave no valid row.
+constexpr long long kNoRow = -(1ll << 62);
+__device__ __forceinline__ long long profile_row(const int* ab, int t, int T, int b, int j, int ldn, int* kmap) {
+  int lo = 0, hi = t;   // first index with ab[index] >= j
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (ab[mid] < j) lo = mid + 1;
+    else hi = mid;
+  }
+  if (lo < t && ab[lo] == j) return -1 - ((long long)b * t + lo) * ldn;
+  const int r = j - lo;
+  if (r < 0 || r >= T - t) return kNoRow;
+  kmap[(long long)b * T + r] = j;
+  return ((long long)b * T + r) * ldn;
+}
+
+// Output rows of the profiles: key rows (Ut, compacted) or anchor rows (S),
+// and the compacted row -> key map.
+struct ProfileOut {
+  bf16 *Ut_hi, *Ut_lo, *S_hi, *S_lo;
+  int* kmap;           // [H][T]: key of compacted row c (c < T - t)
+  const int* anchors;  // [H][t]
+  int t;
+};
+
 // Column statistics of the reference logits and the transposed response
 // profiles (Sec. 3.4, Eq. response_profile), one CTA per (32 columns, head):
 //   pass 1: per column the online (M_j, s1, s2) over the n rows, the 16 row
@@ -72,13 +104,14 @@ int launch_ref_logits_tc(const Dims& D, float scale, const bf16* Q, const bf16* 
 //     transposed, Ut[b][j][i] (row stride ldn >= n, a multiple of 8; the pad
 //     columns n..ldn-1 are written as zeros).
 // e^x is taken as 2^(x log2 e) after the subtraction.
-__global__ void __launch_bounds__(512) col_profiles_kernel(const float* L, float* logphi, bf16* Ut_hi, bf16* Ut_lo,
-                                                           int n, int T, int ldn) {
+__global__ void __launch_bounds__(512) col_profiles_kernel(const float* L, float* logphi, ProfileOut po, int n, int T,
+                                                           int ldn) {
   const int b = blockIdx.y, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int j0 = blockIdx.x * 32, j = j0 + lane;
   __shared__ float red[3][16][32];
   __shared__ float cstat[2][32];
   __shared__ float tile[64][33];
+  __shared__ long long orow[32];   // element offset of each column's output row
   const float* Lb = L + (long long)b * n * T + j;
   float mx = -INFINITY, s1 = 0.f, s2 = 0.f;
   if (j < T) {
@@ -131,7 +164,8 @@ __global__ void __launch_bounds__(512) col_profiles_kernel(const float* L, float
     cstat[1][lane] = j < T ? 1.0f / sqrtf(S2) : 0.f;
   }
   __syncthreads();
-  if (Ut_hi == nullptr) return;
+  if (po.Ut_hi == nullptr) return;
+  if (w == 0 && j < T) orow[lane] = profile_row(po.anchors + (long long)b * po.t, po.t, T, b, j, ldn, po.kmap);
   const float cm = cstat[0][lane], ci = cstat[1][lane];
   for (int i0 = 0; i0 < ldn; i0 += 64) {
 #pragma unroll
@@ -144,13 +178,15 @@ __global__ void __launch_bounds__(512) col_profiles_kernel(const float* L, float
 #pragma unroll
     for (int c = 2 * w; c < 2 * w + 2; ++c) {
       const int jj = j0 + c, i = i0 + 2 * lane;
-      if (jj < T && i < ldn) {
+      if (jj < T && i < ldn && orow[c] != kNoRow) {
         bf16 h0, l0, h1, l1;
         split_bf16(tile[2 * lane][c], h0, l0);
         split_bf16(tile[2 * lane + 1][c], h1, l1);
-        const long long o = ((long long)b * T + jj) * ldn + i;
-        *(__nv_bfloat162*)(Ut_hi + o) = __halves2bfloat162(h0, h1);
-        *(__nv_bfloat162*)(Ut_lo + o) = __halves2bfloat162(l0, l1);
+        const long long ro = orow[c];
+        bf16* dh = ro >= 0 ? po.Ut_hi + ro : po.S_hi + (-1 - ro);
+        bf16* dl = ro >= 0 ? po.Ut_lo + ro : po.S_lo + (-1 - ro);
+        *(__nv_bfloat162*)(dh + i) = __halves2bfloat162(h0, h1);
+        *(__nv_bfloat162*)(dl + i) = __halves2bfloat162(l0, l1);
       }
     }
     __syncthreads();
@@ -165,8 +201,8 @@ __global__ void __launch_bounds__(512) col_profiles_kernel(const float* L, float
 // 3 scales by invN_j and writes the transposed split profiles.
 template <int W>
 __global__ void __launch_bounds__(512) col_profiles_tma_kernel(const __grid_constant__ CUtensorMap mL, float* logphi,
-                                                               bf16* Ut_hi, bf16* Ut_lo, int n, int T, int ldn,
-                                                               int nbox, DevStatus* stt) {
+                                                               ProfileOut po, int n, int T, int ldn, int nbox,
+                                                               DevStatus* stt) {
   constexpr int PH = 512 / W;   // row phases
   extern __shared__ uint8_t smem_raw[];
   const uint32_t r0 = tc::smem_u32(smem_raw);
@@ -176,6 +212,7 @@ __global__ void __launch_bounds__(512) col_profiles_tma_kernel(const __grid_cons
   __shared__ float red[3][PH][W];
   __shared__ float cstat[2][W];
   __shared__ float tile[64][W + 1];
+  __shared__ long long orow[W];   // element offset of each column's output row (anchor rows: -1 - offset)
   const int b = blockIdx.y, j0 = blockIdx.x * W, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int c = tid % W, ph = tid / W, j = j0 + c;
   if (tid == 0) {
@@ -252,9 +289,11 @@ __global__ void __launch_bounds__(512) col_profiles_tma_kernel(const __grid_cons
     }
     if (j < T) logphi[(long long)b * T + j] = cstat[0][tid] + logf(S1) - logf((float)n);
     cstat[1][tid] = j < T ? 1.0f / sqrtf(S2) : 0.f;
+    if (po.Ut_hi != nullptr && j < T)
+      orow[tid] = profile_row(po.anchors + (long long)b * po.t, po.t, T, b, j, ldn, po.kmap);
   }
   __syncthreads();
-  if (Ut_hi == nullptr) return;
+  if (po.Ut_hi == nullptr) return;
   // pass 3: U_ij = e_ij invN_j, transposed through a padded tile 64 rows at a time
   constexpr int RPT = (64 + PH - 1) / PH;   // tile rows per thread: rows ph + k PH below 64
   const float inv = cstat[1][c];
@@ -268,13 +307,15 @@ __global__ void __launch_bounds__(512) col_profiles_tma_kernel(const __grid_cons
     // warp w writes columns w, w + 16, ...: lane l rows i0 + 2l and i0 + 2l + 1 (ldn even)
     for (int cc = warp; cc < W; cc += 16) {
       const int jj = j0 + cc, i = i0 + 2 * lane;
-      if (jj < T && i < ldn) {
+      if (jj < T && i < ldn && orow[cc] != kNoRow) {
         const float x0 = tile[2 * lane][cc], x1 = tile[2 * lane + 1][cc];
         const __nv_bfloat162 h = __floats2bfloat162_rn(x0, x1);
         const float2 hf = __bfloat1622float2(h);
-        const long long o = ((long long)b * T + jj) * ldn + i;
-        *(__nv_bfloat162*)(Ut_hi + o) = h;
-        *(__nv_bfloat162*)(Ut_lo + o) = __floats2bfloat162_rn(x0 - hf.x, x1 - hf.y);
+        const long long ro = orow[cc];
+        bf16* dh = ro >= 0 ? po.Ut_hi + ro : po.S_hi + (-1 - ro);
+        bf16* dl = ro >= 0 ? po.Ut_lo + ro : po.S_lo + (-1 - ro);
+        *(__nv_bfloat162*)(dh + i) = h;
+        *(__nv_bfloat162*)(dl + i) = __floats2bfloat162_rn(x0 - hf.x, x1 - hf.y);
       }
     }
     __syncthreads();
@@ -282,7 +323,7 @@ __global__ void __launch_bounds__(512) col_profiles_tma_kernel(const __grid_cons
 }
 
 template <int W>
-static int launch_col_profiles_tma(const Dims& D, const float* L, float* logphi, bf16* Ut_hi, bf16* Ut_lo, int ldn,
+static int launch_col_profiles_tma(const Dims& D, const float* L, float* logphi, const ProfileOut& po, int ldn,
                                    int nbox, DevStatus* stt, cudaStream_t st) {
   CUtensorMap m;
   if (!encode_f32_map_3d(&m, L, D.T, D.n, D.H, W, 256)) return -1;
@@ -290,20 +331,19 @@ static int launch_col_profiles_tma(const Dims& D, const float* L, float* logphi,
   if (set_dyn_smem((const void*)col_profiles_tma_kernel<W>, smem) !=
       cudaSuccess)
     return -1;
-  col_profiles_tma_kernel<W><<<dim3(cdiv(D.T, W), D.H), 512, smem, st>>>(m, logphi, Ut_hi, Ut_lo, D.n, D.T, ldn, nbox,
-                                                                        stt);
+  col_profiles_tma_kernel<W><<<dim3(cdiv(D.T, W), D.H), 512, smem, st>>>(m, logphi, po, D.n, D.T, ldn, nbox, stt);
   return 1;
 }
 
-int launch_col_profiles(const Dims& D, const float* L, float* logphi, bf16* Ut_hi, bf16* Ut_lo, DevStatus* stt,
+static int col_profiles(const Dims& D, const float* L, float* logphi, const ProfileOut& po, DevStatus* stt,
                         cudaStream_t st) {
   const int ldn = (D.n + 7) / 8 * 8;
   // staged strips of at most 64 KB (three CTAs per SM) when l is TMA-tileable
   const int nbox = cdiv(D.n, 256);
   if ((D.T & 3) == 0 && ((uintptr_t)L & 15u) == 0 && nbox <= 16) {
-    if (nbox <= 4) return launch_col_profiles_tma<16>(D, L, logphi, Ut_hi, Ut_lo, ldn, nbox, stt, st);
-    if (nbox <= 8) return launch_col_profiles_tma<8>(D, L, logphi, Ut_hi, Ut_lo, ldn, nbox, stt, st);
-    return launch_col_profiles_tma<4>(D, L, logphi, Ut_hi, Ut_lo, ldn, nbox, stt, st);
+    if (nbox <= 4) return launch_col_profiles_tma<16>(D, L, logphi, po, ldn, nbox, stt, st);
+    if (nbox <= 8) return launch_col_profiles_tma<8>(D, L, logphi, po, ldn, nbox, stt, st);
+    return launch_col_profiles_tma<4>(D, L, logphi, po, ldn, nbox, stt, st);
   }
   // each CTA re-reads its n x 32 strip from L2: with n > 1024 a shared-memory
   // reservation keeps at most two CTAs per SM so the live strips fit in L2
@@ -311,27 +351,24 @@ int launch_col_profiles(const Dims& D, const float* L, float* logphi, bf16* Ut_h
   if (smem > 0 && set_dyn_smem((const void*)col_profiles_kernel, smem) !=
                       cudaSuccess)
     return -1;
-  col_profiles_kernel<<<dim3(cdiv(D.T, 32), D.H), 512, smem, st>>>(L, logphi, Ut_hi, Ut_lo, D.n, D.T, ldn);
+  col_profiles_kernel<<<dim3(cdiv(D.T, 32), D.H), 512, smem, st>>>(L, logphi, po, D.n, D.T, ldn);
   return 1;
 }
 
-// UtS[b][r] = Ut[b][S_r] (hi and lo rows).
-__global__ void gather_anchor_rows_kernel(const bf16* Ut_hi, const bf16* Ut_lo, const int* anchors, bf16* S_hi,
-                                          bf16* S_lo, int T, int t, int ldn) {
-  const int b = blockIdx.y, r = blockIdx.x;
-  const int j = anchors[(long long)b * t + r];
-  const long long src = ((long long)b * T + j) * ldn, dst = ((long long)b * t + r) * ldn;
-  for (int i = threadIdx.x; i < ldn; i += blockDim.x) {
-    S_hi[dst + i] = Ut_hi[src + i];
-    S_lo[dst + i] = Ut_lo[src + i];
-  }
+int launch_col_profiles(const Dims& D, const float* L, float* logphi, DevStatus* stt, cudaStream_t st) {
+  return col_profiles(D, L, logphi, ProfileOut{nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, D.t}, stt, st);
 }
 
-__global__ void decode_assign_kernel2(const unsigned long long* best, int* kappa, long long count) {
+// kappa of the non-anchor keys from the argmax of their compacted rows
+// (rows c < T - t of head b; kmap gives the key)
+__global__ void decode_assign_kernel2(const unsigned long long* best, const int* kmap, int* kappa, int T, int Tm,
+                                      long long count) {
   for (long long k = blockIdx.x * (long long)blockDim.x + threadIdx.x; k < count;
        k += (long long)gridDim.x * blockDim.x) {
-    const unsigned long long v = best[k];
-    kappa[k] = v ? (int)(0xffffffffu - (unsigned int)(v & 0xffffffffull)) : 0;
+    const long long b = k / Tm, o = b * T + (k - b * Tm);
+    const unsigned long long v = best[o];
+    const int j = kmap[o];
+    if ((unsigned)j < (unsigned)T) kappa[b * T + j] = v ? (int)(0xffffffffu - (unsigned int)(v & 0xffffffffull)) : 0;
   }
 }
 
@@ -345,41 +382,47 @@ __global__ void anchor_self_assign_kernel2(const int* anchors, int* kappa, int T
 }
 
 int launch_assign_prep(const Dims& D, const float* L, float* logphi, const int* anchors, bf16* Ut_hi, bf16* Ut_lo,
-                       bf16* S_hi, bf16* S_lo, DevStatus* stt, cudaStream_t st) {
-  const int ldn = (D.n + 7) / 8 * 8;
-  const int nc = launch_col_profiles(D, L, logphi, Ut_hi, Ut_lo, stt, st);
-  if (nc < 0) return -1;
-  gather_anchor_rows_kernel<<<dim3(D.t, D.H), 128, 0, st>>>(Ut_hi, Ut_lo, anchors, S_hi, S_lo, D.T, D.t, ldn);
-  return nc + 1;
+                       bf16* S_hi, bf16* S_lo, int* kmap, DevStatus* stt, cudaStream_t st) {
+  return col_profiles(D, L, logphi, ProfileOut{Ut_hi, Ut_lo, S_hi, S_lo, kmap, anchors, D.t}, stt, st);
 }
 
 int launch_assign_gemm(const Dims& D, const int* anchors, const bf16* Ut_hi, const bf16* Ut_lo, const bf16* S_hi,
-                       const bf16* S_lo, unsigned long long* best, int* kappa, DevStatus* stt, cudaStream_t st) {
+                       const bf16* S_lo, const int* kmap, unsigned long long* best, int* kappa, DevStatus* stt,
+                       cudaStream_t st) {
   const int ldn = (D.n + 7) / 8 * 8;
-  cudaMemsetAsync(best, 0, sizeof(unsigned long long) * (size_t)D.H * D.T, st);
-  // 128 keys x 256 anchors per tile (M = 128, N = 256 MMAs): half the key-side
-  // operand bytes per flop of a 128-wide tile
-  constexpr int BN = 256;
-  CUtensorMap mA, mA2, mB, mB2;
-  if (!encode_bf16_map_3d(&mA, Ut_hi, ldn, D.T, D.H, 128) || !encode_bf16_map_3d(&mA2, Ut_lo, ldn, D.T, D.H, 128) ||
-      !encode_bf16_map_3d(&mB, S_hi, ldn, D.t, D.H, BN) || !encode_bf16_map_3d(&mB2, S_lo, ldn, D.t, D.H, BN))
-    return -1;
-  TcEpiArgmax8 epi;
-  epi.best = best;
-  epi.bbs = D.T;
-  const int kfull = (ldn + 63) / 64 * 64;
-  // anchor tiles in groups whose split profiles (BN rows x ldn x 4 bytes per
-  // tile) take about 40 MB, so each group stays in L2 while the key profiles
-  // stream past it (one pass over them per group instead of one per wave)
-  const long long tile_bytes = (long long)BN * ldn * 4;
-  const int group = (int)std::max<long long>(1, (40LL << 20) / tile_bytes);
-  if (launch_tc_gemm<BN, kSplit>(mA, mB, mA2, mB2, epi, D.H, D.T, D.t, ldn, kfull, stt, st, 0, nullptr, group) !=
-      cudaSuccess)
-    return -1;
-  const long long cnt = (long long)D.H * D.T;
-  decode_assign_kernel2<<<stride_grid(cnt, 256, 8), 256, 0, st>>>(best, kappa, cnt);
+  const int Tm = D.T - D.t;   // the non-anchor keys, compacted (none when t = T)
+  int nl = 1;
+  // every key gets an assignment in [0, t) even when invalid caller anchors
+  // (flagged upstream) leave some compacted rows without a key
+  cudaMemsetAsync(kappa, 0, sizeof(int) * (size_t)D.H * D.T, st);
+  if (Tm > 0) {
+    cudaMemsetAsync(best, 0, sizeof(unsigned long long) * (size_t)D.H * D.T, st);
+    // 128 keys x 256 anchors per tile (M = 128, N = 256 MMAs): half the key-side
+    // operand bytes per flop of a 128-wide tile.  The key map spans all T rows
+    // of a head (its plane stride); the GEMM takes the first Tm.
+    constexpr int BN = 256;
+    CUtensorMap mA, mA2, mB, mB2;
+    if (!encode_bf16_map_3d(&mA, Ut_hi, ldn, D.T, D.H, 128) || !encode_bf16_map_3d(&mA2, Ut_lo, ldn, D.T, D.H, 128) ||
+        !encode_bf16_map_3d(&mB, S_hi, ldn, D.t, D.H, BN) || !encode_bf16_map_3d(&mB2, S_lo, ldn, D.t, D.H, BN))
+      return -1;
+    TcEpiArgmax8 epi;
+    epi.best = best;
+    epi.bbs = D.T;
+    const int kfull = (ldn + 63) / 64 * 64;
+    // anchor tiles in groups whose split profiles (BN rows x ldn x 4 bytes per
+    // tile) take about 40 MB, so each group stays in L2 while the key profiles
+    // stream past it (one pass over them per group instead of one per wave)
+    const long long tile_bytes = (long long)BN * ldn * 4;
+    const int group = (int)std::max<long long>(1, (40LL << 20) / tile_bytes);
+    if (launch_tc_gemm<BN, kSplit>(mA, mB, mA2, mB2, epi, D.H, Tm, D.t, ldn, kfull, stt, st, 0, nullptr, group) !=
+        cudaSuccess)
+      return -1;
+    const long long cnt = (long long)D.H * Tm;
+    decode_assign_kernel2<<<stride_grid(cnt, 256, 8), 256, 0, st>>>(best, kmap, kappa, D.T, Tm, cnt);
+    nl += 2;
+  }
   anchor_self_assign_kernel2<<<cdiv((long long)D.H * D.t, 256), 256, 0, st>>>(anchors, kappa, D.T, D.t, D.H);
-  return 3;
+  return nl;
 }
 
 }  // namespace arckv
