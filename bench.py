@@ -557,9 +557,9 @@ def run_gpu(args, dist: Dist):
 
     # roofline of the dominant kernel: the assignment GEMM (Eq. anchor_assignment,
     # one launch per layer, stage 5), a split-bf16 tcgen05 GEMM issuing three
-    # bf16 MMAs per useful product; 2 n T t useful flops per head
-    # (the anchors' own assignment is fixed, kappa(s_r) = r: the launch scores
-    # the T - t other keys against the t anchors)
+    # bf16 MMAs per useful product; 2 n (T - t) t useful flops per head (the
+    # anchors' own assignment is fixed, kappa(s_r) = r: the launch scores the
+    # T - t other keys against the t anchors)
     flops = 2.0 * w.H_kv * w.n * (w.T - tp) * tp
     avg_s = statistics.mean(stage_launch_ms[5]) / 1e3
     iso_s = statistics.median(iso_ms[5]) / 1e3
