@@ -134,9 +134,10 @@ Layout plan(const arckv_config& c) {
   L.X64 = take(H * nd64 * 128 * 8);
   // sliced operands of the dual fits: up to 4 slices of Phi_C (or P^, P^^T)
   const size_t slrow = dual ? std::max(n * sliced_ld((int)t), t * sliced_ld((int)n)) : 0;
-  L.Sl = take(4 * H * slrow * 2);
-  L.Sl2 = take(dual ? 4 * H * 128 * sliced_ld((int)n) * 2 : 0);
-  L.eR = take(dual ? H * std::max(n, t) * 4 : 0);
+  // (the blocked dual Cholesky takes two 5-slice 64-column panel sets from it)
+  L.Sl = take(std::max(4 * H * slrow, dual ? 2 * 5 * H * n * kCholNB : 0) * 2);
+  L.Sl2 = take(dual ? std::max(4 * H * 128 * sliced_ld((int)n), 2 * 5 * H * kCholNB * kCholNB) * 2 : 0);
+  L.eR = take(dual ? H * std::max(2 * n, t) * 4 : 0);
   L.eC = take(dual ? H * 128 * 4 : 0);
   L.ir_u = take(dual ? 0 : H * n * 8);
   L.ir_sq = take(dual ? 0 : H * n * 8);

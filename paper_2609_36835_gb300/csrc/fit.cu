@@ -12,6 +12,8 @@
 // fused into the trailing updates, then blocked back substitution, all in one
 // cluster launch per system (chol_cluster_kernel).
 #include <cooperative_groups.h>
+#include <map>
+#include <mutex>
 #include <type_traits>
 
 #include "kernels.h"
@@ -1526,6 +1528,47 @@ struct CholSlicedBufs {
   double *lam, *Z;      // [H], [H][64][nrhs]
 };
 
+// A second stream per calling stream (created on first use, kept for the
+// process) and two events, for the look-ahead of the blocked dual Cholesky.
+struct SideStream {
+  cudaStream_t s;
+  cudaEvent_t fork, join;
+};
+static bool side_stream(cudaStream_t main, SideStream& out) {
+  static std::mutex mu;
+  static std::map<std::pair<int, cudaStream_t>, SideStream> cache;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  std::lock_guard<std::mutex> g(mu);
+  auto it = cache.find({dev, main});
+  if (it != cache.end()) {
+    out = it->second;
+    return true;
+  }
+  SideStream ss{};
+  if (cudaStreamCreateWithFlags(&ss.s, cudaStreamNonBlocking) != cudaSuccess) return false;
+  if (cudaEventCreateWithFlags(&ss.fork, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&ss.join, cudaEventDisableTiming) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  cache[{dev, main}] = ss;
+  out = ss;
+  return true;
+}
+
+// Blocked right-looking Cholesky of the n x n systems with a look-ahead of
+// one block: after step k's panel the trailing matrix is updated in two
+// launches, first its leading 64-column block (block k + 1, all rows), then
+// the rest of its lower triangle; the second runs on the calling stream
+// while a side stream factors block k + 1, slices its inverse and forms and
+// slices the panel below it, so the diagonal factor and the panel leave the
+// critical path: the second update leaves kAheadSMs SMs free (its
+// persistent grid is capped) and the side stream's panel product takes at
+// most that many CTAs.  Slices of consecutive steps alternate between two
+// buffers.
+// The operations and their order per element are those of the plain blocked
+// algorithm.
 static int chol_solve_sliced(int H, int n, double* A, double* Linv, double* B, double* X, int nrhs, double ridge,
                              double tdiv, const CholSlicedBufs& W, DevStatus* stt, cudaStream_t st) {
   constexpr int S = kCholSlices;
@@ -1540,37 +1583,68 @@ static int chol_solve_sliced(int H, int n, double* A, double* Linv, double* B, d
     nl += r;
     return true;
   };
+  SideStream ss{};
+  const bool ahead = nblk > 1 && side_stream(st, ss);
+  constexpr int kAheadSMs = 16;
+  const int main_ctas = ahead ? std::max(1, tc_gemm_sm_count() - kAheadSMs) : 0, side_ctas = ahead ? kAheadSMs : 0;
+  const cudaStream_t sd = ahead ? ss.s : st;
+  const long long sa_stride = (long long)S * H * n * NB, sb_stride = (long long)S * H * NB * NB;
+  auto SA = [&](int k) { return W.sA + (k & 1) * sa_stride; };
+  auto EA = [&](int k) { return W.eA + (k & 1) * (long long)H * n; };
+  auto SB = [&](int k) { return W.sB + (k & 1) * sb_stride; };
+  auto EB = [&](int k) { return W.eB + (k & 1) * (long long)H * NB; };
+  // block k: its diagonal factor and inverse, the inverse's slices, the panel
+  // L_ik = A_ik Linv_kk^T below it and the panel's slices (on stream s)
+  auto diag_panel = [&](int k, cudaStream_t s) -> bool {
+    const int k0 = k * NB, kb = std::min(NB, n - k0), m = n - k0 - kb;
+    chol_diag_kernel<<<H, kCT, dsm, s>>>(A, Linv, n, k, W.lam, stt);
+    ++nl;
+    if (!ok(launch_slice_rows(S, Linv + (long long)k * NB * NB, kb, kb, NB, lb, H, SB(k), EB(k), s))) return false;
+    if (m > 0) {
+      double* panel = A + (long long)(k0 + kb) * n + k0;
+      if (!ok(launch_slice_rows(S, panel, m, kb, n, nn, H, SA(k), EA(k), s))) return false;
+      if (!ok(launch_sliced_f64(S, SA(k), EA(k), m, SB(k), EB(k), kb, kb, H, panel, nn, n, false, false, stt, s, 0,
+                                1 << 30, s == st ? 0 : side_ctas)))
+        return false;
+      if (!ok(launch_slice_rows(S, panel, m, kb, n, nn, H, SA(k), EA(k), s))) return false;
+    }
+    return true;
+  };
   chol_lambda_kernel<<<H, 256, 0, st>>>(A, n, ridge, tdiv, W.lam, stt);
   ++nl;
+  if (!diag_panel(0, st)) return -1;
   for (int k = 0; k < nblk; ++k) {
     const int k0 = k * NB, kb = std::min(NB, n - k0), m = n - k0 - kb;
-    chol_diag_kernel<<<H, kCT, dsm, st>>>(A, Linv, n, k, W.lam, stt);
-    ++nl;
-    // Linv_kk rows (K = kb)
-    if (!ok(launch_slice_rows(S, Linv + (long long)k * NB * NB, kb, kb, NB, lb, H, W.sB, W.eB, st))) return -1;
-    double* panel = A + (long long)(k0 + kb) * n + k0;
     if (m > 0) {
-      // L_ik = A_ik Linv_kk^T, written over A_ik
-      if (!ok(launch_slice_rows(S, panel, m, kb, n, nn, H, W.sA, W.eA, st))) return -1;
-      if (!ok(launch_sliced_f64(S, W.sA, W.eA, m, W.sB, W.eB, kb, kb, H, panel, nn, n, false, false, stt, st)))
+      // A_ij -= L_ik L_jk^T on the trailing lower triangle: block k + 1 first
+      double* trail = A + (long long)(k0 + kb) * n + k0 + kb;
+      if (!ok(launch_sliced_f64(S, SA(k), EA(k), m, SA(k), EA(k), m, kb, H, trail, nn, n, true, true, stt, st, 0, 1)))
         return -1;
-      // A_ij -= L_ik L_jk^T on the trailing lower triangle
-      if (!ok(launch_slice_rows(S, panel, m, kb, n, nn, H, W.sA, W.eA, st))) return -1;
-      if (!ok(launch_sliced_f64(S, W.sA, W.eA, m, W.sA, W.eA, m, kb, H, A + (long long)(k0 + kb) * n + k0 + kb, nn,
-                                n, true, true, stt, st)))
+      if (ahead) {
+        cudaEventRecord(ss.fork, st);
+        cudaStreamWaitEvent(sd, ss.fork, 0);
+      }
+      if (!diag_panel(k + 1, sd)) return -1;
+      if (!ok(launch_sliced_f64(S, SA(k), EA(k), m, SA(k), EA(k), m, kb, H, trail, nn, n, true, true, stt, st, 1,
+                                1 << 30, main_ctas)))
         return -1;
     }
-    if (nrhs == 1) continue;   // one right-hand side: substituted after the factorisation (below)
-    // Y_k = Linv_kk B_k over B_k; B_i -= L_ik Y_k
-    double* Bk = B + (long long)k0 * nrhs;
-    if (!ok(launch_slice_cols(S, Bk, kb, nrhs, nrhs, nr, H, W.sC, W.eC, st))) return -1;
-    if (!ok(launch_sliced_f64(S, W.sB, W.eB, kb, W.sC, W.eC, nrhs, kb, H, Bk, nr, nrhs, false, false, stt, st)))
-      return -1;
-    if (m > 0) {
+    if (nrhs > 1) {
+      // Y_k = Linv_kk B_k over B_k; B_i -= L_ik Y_k
+      double* Bk = B + (long long)k0 * nrhs;
       if (!ok(launch_slice_cols(S, Bk, kb, nrhs, nrhs, nr, H, W.sC, W.eC, st))) return -1;
-      if (!ok(launch_sliced_f64(S, W.sA, W.eA, m, W.sC, W.eC, nrhs, kb, H, Bk + (long long)kb * nrhs, nr, nrhs, false,
-                                true, stt, st)))
+      if (!ok(launch_sliced_f64(S, SB(k), EB(k), kb, W.sC, W.eC, nrhs, kb, H, Bk, nr, nrhs, false, false, stt, st)))
         return -1;
+      if (m > 0) {
+        if (!ok(launch_slice_cols(S, Bk, kb, nrhs, nrhs, nr, H, W.sC, W.eC, st))) return -1;
+        if (!ok(launch_sliced_f64(S, SA(k), EA(k), m, W.sC, W.eC, nrhs, kb, H, Bk + (long long)kb * nrhs, nr, nrhs,
+                                  false, true, stt, st)))
+          return -1;
+      }
+    }
+    if (ahead && m > 0) {
+      cudaEventRecord(ss.join, sd);
+      cudaStreamWaitEvent(st, ss.join, 0);
     }
   }
   if (nrhs == 1) {

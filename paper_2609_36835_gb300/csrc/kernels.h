@@ -182,8 +182,11 @@ int launch_slice_cols(int S, const double* X, int K, int R, int ldx, long long x
                       cudaStream_t st);
 // C[b] (M x N, fp64, rows ldc apart, batches cbs apart) = A B^T, or C -= A B^T
 // with `sub`; with `lower` only the tiles that reach C's lower triangle (M = N)
+// (with 5 slices: nt0, nt1 select the 64-wide column tiles [nt0, nt1);
+// max_ctas > 0 caps the persistent grid, leaving SMs to a concurrent stream)
 int launch_sliced_f64(int S, const bf16* As, const int* eA, int M, const bf16* Bs, const int* eB, int N, int K, int H,
-                      double* C, long long cbs, int ldc, bool lower, bool sub, DevStatus* stt, cudaStream_t st);
+                      double* C, long long cbs, int ldc, bool lower, bool sub, DevStatus* stt, cudaStream_t st,
+                      int nt0 = 0, int nt1 = 1 << 30, int max_ctas = 0);
 // G[b] = X X^T (R x R, fp64) on the tiles that reach the lower triangle
 int launch_sliced_gram_lower(int S, const bf16* Xs, const int* ex, int R, int K, int H, double* G, DevStatus* stt,
                              cudaStream_t st);

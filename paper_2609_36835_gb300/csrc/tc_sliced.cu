@@ -202,34 +202,36 @@ __device__ __forceinline__ void sl_store_direct(const Out& out, int b, int row, 
     }
 }
 
-// Tiles of one batch: all (row tile, column tile) pairs, or with `lower` only
-// those that reach the lower triangle (column tile start <= row tile end) of a
-// square product (ct column tiles per row tile); column tiles fastest.
-__device__ __forceinline__ void sl_tile(int tl, int Mt, int Nt, bool lower, int ct, int& b, int& mt, int& nt) {
-  if (!lower) {
-    b = tl / (Mt * Nt);
-    const int r = tl - b * (Mt * Nt);
-    mt = r / Nt;
-    nt = r - mt * Nt;
-    return;
-  }
-  int per = 0;
-  for (int i = 0; i < Mt; ++i) per += min(Nt, ct * (i + 1));
+// Column tiles [nt0, row end) of row tile i: all of [nt0, nt1), or with
+// `lower` only those that reach the lower triangle (column tile start <= row
+// tile end) of a square product (ct column tiles per row tile).
+__host__ __device__ __forceinline__ int sl_row_tiles(int i, int nt0, int nt1, bool lower, int ct) {
+  const int e = lower ? (nt1 < ct * (i + 1) ? nt1 : ct * (i + 1)) : nt1;
+  return e > nt0 ? e - nt0 : 0;
+}
+// Tile tl of the batch-major enumeration, column tiles fastest.
+__device__ __forceinline__ void sl_tile(int tl, int Mt, int nt0, int nt1, bool lower, int ct, int per, int& b, int& mt,
+                                        int& nt) {
   b = tl / per;
   int r = tl - b * per;
+  if (!lower) {
+    mt = r / (nt1 - nt0);
+    nt = nt0 + (r - mt * (nt1 - nt0));
+    return;
+  }
   mt = 0;
-  while (r >= min(Nt, ct * (mt + 1))) {
-    r -= min(Nt, ct * (mt + 1));
+  while (r >= sl_row_tiles(mt, nt0, nt1, true, ct)) {
+    r -= sl_row_tiles(mt, nt0, nt1, true, ct);
     ++mt;
   }
-  nt = r;
+  nt = nt0 + r;
 }
 
 template <int S, class Out, int BN>
 __global__ void __launch_bounds__(SlShape<BN>::THREADS, 1)
     sliced_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB, const Out out,
                        const int* __restrict__ eA, const int* __restrict__ eB, int H, int M, int N, int K, int lower,
-                       DevStatus* stt) {
+                       int nt0, int nt1, DevStatus* stt) {
   using C = SlCfg<S, BN>;
   using Sh = SlShape<BN>;
   constexpr int STAGES = C::STAGES, EW = Sh::EW, NBUF = Sh::NBUF, TILE_B = Sh::TILE_B;
@@ -242,13 +244,9 @@ __global__ void __launch_bounds__(SlShape<BN>::THREADS, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nk = (K + kSlBK - 1) / kSlBK;
   const int nchunks = (nk + kSlChunkSlabs - 1) / kSlChunkSlabs;
-  const int Mt = (M + kSlBM - 1) / kSlBM, Nt = (N + BN - 1) / BN;
+  const int Mt = (M + kSlBM - 1) / kSlBM;
   int per = 0;
-  if (lower) {
-    for (int i = 0; i < Mt; ++i) per += min(Nt, Sh::COLT * (i + 1));
-  } else {
-    per = Mt * Nt;
-  }
+  for (int i = 0; i < Mt; ++i) per += sl_row_tiles(i, nt0, nt1, lower != 0, Sh::COLT);
   const int ntiles = H * per;
 
   if (threadIdx.x == 0) {
@@ -283,7 +281,7 @@ __global__ void __launch_bounds__(SlShape<BN>::THREADS, 1)
       bool ok = true;
       for (int tl = blockIdx.x; tl < ntiles && ok; tl += gridDim.x) {
         int b, mt, nt;
-        sl_tile(tl, Mt, Nt, lower != 0, Sh::COLT, b, mt, nt);
+        sl_tile(tl, Mt, nt0, nt1, lower != 0, Sh::COLT, per, b, mt, nt);
         for (int kb = 0; kb < nk; ++kb) {
           const int s = g % STAGES;
           if (g >= STAGES && !tc::mbar_wait(&empty[s], ((g / STAGES) - 1) & 1, abortp, stt)) {
@@ -373,7 +371,7 @@ __global__ void __launch_bounds__(SlShape<BN>::THREADS, 1)
     int kc = 0, tcount = 0;
     for (int tl = blockIdx.x; tl < ntiles && ok; tl += gridDim.x, ++tcount) {
       int b, mt, nt;
-      sl_tile(tl, Mt, Nt, lower != 0, Sh::COLT, b, mt, nt);
+      sl_tile(tl, Mt, nt0, nt1, lower != 0, Sh::COLT, per, b, mt, nt);
       // exact running sum of levels 2..4 in units of 2^-32: level l contributes
       // its integer chunk sums shifted left by 8 (4 - l) bits (|sum| < 2^47)
       out.prefetch(b, mt * kSlBM + row_in, nt * BN + part * 32, M, N);
@@ -630,7 +628,8 @@ int g_sliced_fail = 0;   // which step of the last failed launch_sliced gave up 
 
 template <int S, int BN, class Out>
 int launch_sliced(const bf16* As, const int* eA, int M, const bf16* Bs, const int* eB, int N, int K, int ldk, int H,
-                  bool lower, const Out& out, DevStatus* stt, cudaStream_t st) {
+                  bool lower, const Out& out, DevStatus* stt, cudaStream_t st, int nt0 = 0, int nt1 = 1 << 30,
+                  int max_ctas = 0) {
   CUtensorMap mA, mB;
   if (!encode_bf16_map_3d_sw64(&mA, As, K, M, (uint64_t)S * H, ldk, kSlBM) ||
       !encode_bf16_map_3d_sw64(&mB, Bs, K, N, (uint64_t)S * H, ldk, BN)) {
@@ -646,14 +645,14 @@ int launch_sliced(const bf16* As, const int* eA, int M, const bf16* Bs, const in
     return -1;
   }
   const int Mt = cdiv(M, kSlBM), Nt = cdiv(N, BN);
+  nt1 = std::min(nt1, Nt);
+  nt0 = std::max(nt0, 0);
   long long per = 0;
-  if (lower) {
-    for (int i = 0; i < Mt; ++i) per += std::min(Nt, Sh::COLT * (i + 1));
-  } else {
-    per = (long long)Mt * Nt;
-  }
-  const int grid = (int)std::min<long long>(per * H, tc_gemm_sm_count());
-  kern<<<grid, Sh::THREADS, C::SMEM, st>>>(mA, mB, out, eA, eB, H, M, N, K, lower ? 1 : 0, stt);
+  for (int i = 0; i < Mt; ++i) per += sl_row_tiles(i, nt0, nt1, lower, Sh::COLT);
+  if (per == 0) return 0;   // no tile in the column range
+  int grid = (int)std::min<long long>(per * H, tc_gemm_sm_count());
+  if (max_ctas > 0) grid = std::min(grid, max_ctas);
+  kern<<<grid, Sh::THREADS, C::SMEM, st>>>(mA, mB, out, eA, eB, H, M, N, K, lower ? 1 : 0, nt0, nt1, stt);
   const cudaError_t el = cudaGetLastError();
   if (el != cudaSuccess) g_sliced_fail = 1000 + (int)el;
   return el == cudaSuccess ? 1 : -1;
@@ -730,7 +729,8 @@ int launch_sliced_gram_lower(int S, const bf16* Xs, const int* ex, int R, int K,
 static bool sliced_wide(int S, int K) { return S <= 4 && K >= 256; }
 
 int launch_sliced_f64(int S, const bf16* As, const int* eA, int M, const bf16* Bs, const int* eB, int N, int K, int H,
-                      double* C, long long cbs, int ldc, bool lower, bool sub, DevStatus* stt, cudaStream_t st) {
+                      double* C, long long cbs, int ldc, bool lower, bool sub, DevStatus* stt, cudaStream_t st,
+                      int nt0, int nt1, int max_ctas) {
   const int ldk = (int)sliced_ld(K);
   const SlOutF64 out{C, cbs, ldc, sub ? 1 : 0};
   const bool w = sliced_wide(S, K);
@@ -740,7 +740,7 @@ int launch_sliced_f64(int S, const bf16* As, const int* eA, int M, const bf16* B
   if (S == 4)
     return w ? launch_sliced<4, 128>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st)
              : launch_sliced<4, 64>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st);
-  if (S == 5) return launch_sliced<5, 64>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st);
+  if (S == 5) return launch_sliced<5, 64>(As, eA, M, Bs, eB, N, K, ldk, H, lower, out, stt, st, nt0, nt1, max_ctas);
   return -1;
 }
 
