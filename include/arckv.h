@@ -29,7 +29,14 @@
  * - Arguments are checked on the host before anything is enqueued; a bad
  *   argument returns ARCKV_ERR_INVALID_ARG / ARCKV_ERR_SHAPE /
  *   ARCKV_ERR_WORKSPACE / ARCKV_ERR_UNSUPPORTED and enqueues nothing.
- * - All kernels are enqueued on `stream` in order.  Errors found on the
+ * - All kernels are enqueued on `stream` in order, with one exception:
+ *   arckv_compact's dual-form solves (t > n) run part of their kernels on a
+ *   second stream that the library creates for each calling stream on its
+ *   first such call (a non-blocking stream and two events, kept for the
+ *   life of the process), forked from `stream` and joined back to it with
+ *   events, so the call's work still begins after the work enqueued on
+ *   `stream` before it and ends before the work enqueued after it.  These
+ *   are the only resources the library creates itself.  Errors found on the
  *   device (a non-positive Cholesky pivot, a non-finite output) are recorded
  *   in a status word inside the workspace.  Without ARCKV_FLAG_NONBLOCKING
  *   the call synchronises `stream` and returns that status; with it the call
