@@ -112,6 +112,8 @@ __global__ void __launch_bounds__(512) col_profiles_kernel(const float* L, float
   __shared__ float cstat[2][32];
   __shared__ float tile[64][33];
   __shared__ long long orow[32];   // element offset of each column's output row
+  if (po.Ut_hi != nullptr && w == 0 && j < T)
+    orow[lane] = profile_row(po.anchors + (long long)b * po.t, po.t, T, b, j, ldn, po.kmap);
   const float* Lb = L + (long long)b * n * T + j;
   float mx = -INFINITY, s1 = 0.f, s2 = 0.f;
   if (j < T) {
@@ -165,7 +167,6 @@ __global__ void __launch_bounds__(512) col_profiles_kernel(const float* L, float
   }
   __syncthreads();
   if (po.Ut_hi == nullptr) return;
-  if (w == 0 && j < T) orow[lane] = profile_row(po.anchors + (long long)b * po.t, po.t, T, b, j, ldn, po.kmap);
   const float cm = cstat[0][lane], ci = cstat[1][lane];
   for (int i0 = 0; i0 < ldn; i0 += 64) {
 #pragma unroll
@@ -225,6 +226,10 @@ __global__ void __launch_bounds__(512) col_profiles_tma_kernel(const __grid_cons
     tc::mbar_arrive_expect_tx(&bar, (uint32_t)(nbox * 256 * W * 4));
     for (int q = 0; q < nbox; ++q) tc::tma_load_3d(strip + q * 256 * W, &mL, j0, q * 256, b, &bar);
   }
+  // the output rows of the CTA's keys (a binary search over the anchors)
+  // while the strip is in flight
+  if (po.Ut_hi != nullptr && tid >= 32 && tid < 32 + W && j0 + tid - 32 < T)
+    orow[tid - 32] = profile_row(po.anchors + (long long)b * po.t, po.t, T, b, j0 + tid - 32, ldn, po.kmap);
   const bool ok = tc::mbar_wait(&bar, 0, &abort_flag, stt);
   if (!__syncthreads_and(ok)) {   // timed out: let the copies land (bounded) before leaving
     volatile int never = 0;
@@ -289,8 +294,6 @@ __global__ void __launch_bounds__(512) col_profiles_tma_kernel(const __grid_cons
     }
     if (j < T) logphi[(long long)b * T + j] = cstat[0][tid] + logf(S1) - logf((float)n);
     cstat[1][tid] = j < T ? 1.0f / sqrtf(S2) : 0.f;
-    if (po.Ut_hi != nullptr && j < T)
-      orow[tid] = profile_row(po.anchors + (long long)b * po.t, po.t, T, b, j, ldn, po.kmap);
   }
   __syncthreads();
   if (po.Ut_hi == nullptr) return;
