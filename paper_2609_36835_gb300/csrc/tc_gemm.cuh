@@ -80,6 +80,17 @@ struct EpiStage<E, std::void_t<decltype(E::kStageBytes)>> {
   static constexpr int bytes = E::kStageBytes;
 };
 
+// An epilogue that declares kHalfLoads = true is fed 16 columns at a time
+// through consume16(State&, int chunk, int j, int half, float (&v)[16]).
+template <class E, class = void>
+struct EpiHalfLoads {
+  static constexpr bool value = false;
+};
+template <class E>
+struct EpiHalfLoads<E, std::void_t<decltype(E::kHalfLoads)>> {
+  static constexpr bool value = E::kHalfLoads;
+};
+
 template <int BN, int MODE>
 struct TcCfg {
   static constexpr bool SPLIT = MODE == kSplit;
@@ -290,9 +301,18 @@ __global__ void __launch_bounds__(64 + 32 * EpiWarps<Epi>::value, 1)
         tc::fence_after_sync();
 #pragma unroll
         for (int j = 0; j < JG; ++j) {
-          float v[32];
-          tc::tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN + (cg + j) * 32), v);
-          epi.consume(es, c, j, v);
+          if constexpr (EpiHalfLoads<Epi>::value) {   // 16 columns at a time (fewer live registers)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              float v[16];
+              tc::tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN + (cg + j) * 32 + h * 16), v);
+              epi.consume16(es, c, j, h, v);
+            }
+          } else {
+            float v[32];
+            tc::tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN + (cg + j) * 32), v);
+            epi.consume(es, c, j, v);
+          }
         }
         tc::fence_before_sync();
         __syncwarp();

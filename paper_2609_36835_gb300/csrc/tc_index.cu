@@ -60,6 +60,18 @@ struct TcEpiIndexT {
 #pragma unroll
     for (int q = 0; q < 32; ++q) s.acc[j * 32 + q] = fmaf(s.w, fmaxf(v[q], 0.1f * v[q]), s.acc[j * 32 + q]);
   }
+  // the 256-wide tiles take their columns 16 at a time: with 128 running sums
+  // per thread a 32-column load left the eight-warp epilogue spilling
+  static constexpr bool kHalfLoads = kBN == 256;
+  __device__ __forceinline__ void consume16(State& s, int chunk, int j, int h, float (&v)[16]) const {
+    if (j == 0 && h == 0) {
+      s.w = s.wn * 0.08838834764831845f;
+      s.wn = (s.row_ok && chunk + 1 < H_I) ? s.wrow[chunk + 1] : 0.f;
+    }
+#pragma unroll
+    for (int q = 0; q < 16; ++q)
+      s.acc[j * 32 + h * 16 + q] = fmaf(s.w, fmaxf(v[q], 0.1f * v[q]), s.acc[j * 32 + h * 16 + q]);
+  }
   __device__ __forceinline__ void finish(State& s, int b, int row, int n0, int, int N) const {
     const int nc = min(kW, N - n0);
     if (s.row_ok && nc > 0) {
