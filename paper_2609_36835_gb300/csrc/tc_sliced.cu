@@ -539,7 +539,10 @@ __device__ __forceinline__ void digit_slices(T x, int e, bf16 (&o)[S]) {
 }
 
 // Row-sliced operand: X [H][R][K] (rows ldx apart, batches xbs apart) ->
-// slices [S][H][R][ldo] bf16 and exponents [H][R].  One warp per row.
+// slices [S][H][R][ldo] bf16 and exponents [H][R].  One warp per row, four
+// consecutive elements per lane and round, each plane's four slices written
+// as one 8-byte store (ldo is a multiple of 8, so every plane row is 16-byte
+// aligned).
 template <int S, typename T>
 __global__ void __launch_bounds__(256) slice_rows_kernel(const T* __restrict__ X, int R, int K, int ldx, long long xbs,
                                                          int H, bf16* __restrict__ out, int ldo,
@@ -550,18 +553,42 @@ __global__ void __launch_bounds__(256) slice_rows_kernel(const T* __restrict__ X
   const int b = (int)(gr / R), r = (int)(gr - (long long)b * R);
   const T* x = X + (long long)b * xbs + (long long)r * ldx;
   unsigned long long mb = 0;
-  for (int k = lane; k < K; k += 32) mb = max(mb, mag_bits(x[k]));
+  for (int k = 4 * lane; k < K; k += 128) {
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      if (k + u < K) mb = max(mb, mag_bits(x[k + u]));
+  }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) mb = max(mb, __shfl_xor_sync(0xffffffffu, mb, o));
   const int e = bound_exp_bits<T>(mb);
   if (lane == 0) ex[gr] = e;
   const long long slice = (long long)H * R * ldo;
   bf16* o = out + gr * ldo;
-  for (int k = lane; k < K; k += 32) {
-    bf16 s[S];
-    digit_slices<S>(x[k], e, s);
+  for (int k = 4 * lane; k < K; k += 128) {
+    bf16 s[4][S];
 #pragma unroll
-    for (int i = 0; i < S; ++i) o[i * slice + k] = s[i];
+    for (int u = 0; u < 4; ++u) digit_slices<S>(k + u < K ? x[k + u] : T(0), e, s[u]);
+    if (k + 4 <= K) {
+#pragma unroll
+      for (int i = 0; i < S; ++i) {
+        __nv_bfloat162 lo2, hi2;
+        lo2.x = s[0][i];
+        lo2.y = s[1][i];
+        hi2.x = s[2][i];
+        hi2.y = s[3][i];
+        uint2 w;
+        w.x = *reinterpret_cast<const unsigned int*>(&lo2);
+        w.y = *reinterpret_cast<const unsigned int*>(&hi2);
+        *reinterpret_cast<uint2*>(o + i * slice + k) = w;
+      }
+    } else {
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (k + u < K) {
+#pragma unroll
+          for (int i = 0; i < S; ++i) o[i * slice + k + u] = s[u][i];
+        }
+    }
   }
 }
 
