@@ -1306,13 +1306,15 @@ __global__ void __launch_bounds__(256) xty64_kernel(const float* X, const double
 // product runs on the tensor pipe as an exact product of 5-slice operands
 // (2^-40 of each row's largest entry per operand, the same backward error as
 // an fp64 factorisation to ~1e-12), and only the 64 x 64 diagonal factors
-// and inverses run in fp64 on the SIMT pipes:
-//   for k:  L_kk = chol(A_kk + lam I), Linv_kk = L_kk^-1        (fp64 SIMT)
+// and inverses (double-float, ~48 bits, from fp64 storage) and the block
+// back substitution run on the SIMT pipes:
+//   for k:  L_kk = chol(A_kk + lam I), Linv_kk = L_kk^-1        (double-float)
 //           L_ik = A_ik Linv_kk^T                        i > k  (sliced)
 //           A_ij -= L_ik L_jk^T                    j <= i, i > k  (sliced, lower tiles)
 //           Y_k = Linv_kk B_k;  B_i -= L_ik Y_k         i > k  (sliced)
 //   for k descending:  Z_k = sum_{i>k} L_ik^T X_i            (sliced)
 //           X_k = Linv_kk^T (Y_k - Z_k)                         (fp64 SIMT)
+// With one right-hand side both substitutions run in tri_solve_cluster_kernel.
 
 constexpr int kCholSlices = 5;
 
@@ -1681,10 +1683,10 @@ static int chol_solve_sliced(int H, int n, double* A, double* Linv, double* B, d
 // not keep the Gram structure moves beta by up to cond x error: the n x n
 // Grams are exact products of row-sliced Phi / P^ on the tensor cores (4
 // slices: 32 bits of each row relative to its largest entry, a perturbation
-// of the operand itself), the solves run in fp64, w = Phi^T a in fp64 and
-// C_v = P^T A as a 4-slice tensor-core product (with 3 slices for P^ the
-// held-out outputs of a 128K head drift by ~7e-3).  Beyond kSlicedMaxK the
-// fp64 SIMT products serve.
+// of the operand itself), the solves are fp64-grade (chol_solve_sliced),
+// w = Phi^T a is summed in double-float and C_v = P^T A is a 4-slice
+// tensor-core product (with 3 slices for P^ the held-out outputs of a 128K
+// head drift by ~7e-3).  Beyond kSlicedMaxK the fp64 SIMT products serve.
 static int fits_dual(const Dims& D, float ridge_w, float ridge_v, float eps_w, float b_min, float b_max,
                      const float* m, const float* Y, const FitBufs& B, float* beta, float* C_v, DevStatus* stt,
                      cudaStream_t st, cudaEvent_t const* ev) {
