@@ -74,7 +74,9 @@ def dominant_source_hash() -> str:
 def parse_args(argv=None):
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=0,
+                    help="timed steps (default: 20, or 14 for contexts of 64K tokens and more, so that the "
+                         "timed region stays near a minute)")
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=("gpu", "reference"), default="gpu")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
@@ -103,7 +105,12 @@ def parse_args(argv=None):
     ap.add_argument("--layer-shape", default="",
                     help="with --profile-layer: T,n_pos,t overriding the workload's sizes (same distributions), "
                          "e.g. 16384,64,2048 for a small case of the dual-form fits (t > n)")
-    return ap.parse_args(argv)
+    args = ap.parse_args(argv)
+    if args.steps <= 0:
+        import synth
+        w = synth.WORKLOADS.get(args.workload)
+        args.steps = 14 if (w is not None and w.T >= 65536 and args.impl == "gpu") else 20
+    return args
 
 
 # ------------------------------------------------------------ distributed
