@@ -56,6 +56,18 @@ def test_workspace_bytes_sizes_and_rejections(lib):
     assert pk.attend_workspace_bytes(8, 1024, 0) == 0
 
 
+def test_long_context_workspaces_fit_the_bench(lib):
+    """The dual-form workspace of a 128K layer call (8 heads) and the 32K one:
+    the bench holds three 128K workspaces beside a 17.8 GB context in HBM."""
+    w128 = synth.WORKLOADS["llama8b_T131072_r10"]
+    ws128 = pk.workspace_bytes(workload.layer_config(w128, w128.H_kv))
+    assert 20e9 < ws128 < 30e9
+    w32 = synth.WORKLOADS["llama8b_T32768_r05"]
+    ws32 = pk.workspace_bytes(workload.layer_config(w32, w32.H_kv))
+    assert 4e9 < ws32 < 8e9
+    assert 3 * ws128 + 17.8e9 < 200e9
+
+
 def test_wait_probe_rejects_bad_arguments_on_the_host(lib):
     assert pk.arckv_wait_probe(None, 256, 1000, stream=0) == 3     # no workspace
     assert pk.arckv_wait_probe(None, 256, 0, stream=0) == 1        # limit out of range

@@ -162,3 +162,13 @@ def test_cpu_baseline_sample_pairs_are_distinct_and_spread(layers, heads, k):
     assert len(pairs) == len(set(pairs)) == min(k, layers * heads)
     assert all(0 <= l < layers and 0 <= h < heads for l, h in pairs)
     assert pairs[0] == (0, 0) and (k < 2 or layers * heads < 2 or max(l for l, _ in pairs) == layers - 1)
+
+
+def test_default_timed_steps_follow_the_context_length():
+    """About a minute of timed work at 128K (14 steps of ~4.4 s), 20 steps at
+    shorter contexts and for the reference arm (whose steps are segments)."""
+    assert bench.parse_args([]).steps == 14
+    assert bench.parse_args(["--workload", "llama8b_T8192_r10"]).steps == 20
+    assert bench.parse_args(["--impl", "reference"]).steps == 20
+    assert bench.parse_args(["--steps", "5"]).steps == 5
+    assert bench.parse_args([]).warmup >= 3
