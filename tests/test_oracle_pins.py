@@ -96,6 +96,53 @@ def test_index_weights_use_activation_of_the_rows_position():
     assert np.allclose(I2, 3.0 * I1, rtol=1e-12, atol=1e-14)
 
 
+def test_indexer_projections_block_normalised_and_weights_closed_form():
+    """Eq. (indexer_projection), App. A.1: each of the H_I blocks of q_bar and
+    k_bar is the raw block scaled to mean square 1 (up to the 1e-6 guard);
+    with L_q = L_c = 0 and L_k = 0, L_v = I on the first block the key block
+    is N(v); with X = 0 the weights are b_x."""
+    w, K, V, Q, Xr, W = small_pair(T=24, n_pos=8)
+    H_I, d_I, d = 8, 128, K.shape[1]
+    q_bar, k_bar, wts, c = oracle.indexer_projections(Q, Xr, K, V, W, H_I, d_I)
+    assert q_bar.shape == (Q.shape[0], H_I, d_I) and k_bar.shape == (K.shape[0], H_I, d_I)
+    for z in (q_bar, k_bar):
+        ms = np.mean(z * z, axis=-1)
+        assert np.all(np.abs(ms - 1.0) < 1e-4)
+    # a block keeps the direction of its raw projection: q_bar block 3 is parallel to rows 384..511 of L_q q + L_c c
+    raw = Q @ W["L_q"][3 * d_I:4 * d_I].T + c @ W["L_c"][3 * d_I:4 * d_I].T
+    cos = np.sum(raw * q_bar[:, 3], axis=1) / (np.linalg.norm(raw, axis=1) * np.linalg.norm(q_bar[:, 3], axis=1))
+    assert np.allclose(cos, 1.0, atol=1e-12)
+    L_v = np.zeros((H_I * d_I, d))
+    L_v[:d_I] = np.eye(d_I, d)
+    W2 = dict(W, L_k=np.zeros_like(W["L_k"]), L_v=L_v)
+    _, k2, _, _ = oracle.indexer_projections(Q, Xr, K, V, W2, H_I, d_I)
+    expect = V / np.sqrt(np.sum(V * V, axis=1, keepdims=True) / d_I + 1e-6)
+    assert np.allclose(k2[:, 0], expect, rtol=1e-12, atol=1e-12)
+    _, _, w0, _ = oracle.indexer_projections(Q, np.zeros_like(Xr), K, V, W, H_I, d_I)
+    assert np.array_equal(w0, np.broadcast_to(W["b_x"], w0.shape))
+
+
+def test_compact_pair_steps_pauses_and_returns_the_pipeline_result():
+    """compact_pair_steps pauses between stages (after the projections, each
+    index head, the selection, the profiles, each key block, the merge and the
+    beta fit) and returns compact_pair's result unchanged."""
+    w, K, V, Q, Xr, W = small_pair(T=40, n_pos=10)
+    cfg = oracle.OracleConfig(t=8)
+    gen = oracle.compact_pair_steps(K, V, Q, Xr, W, cfg)
+    pauses = 0
+    while True:
+        try:
+            next(gen)
+            pauses += 1
+        except StopIteration as done:
+            res = done.value
+            break
+    assert pauses == 1 + 8 + 1 + 1 + 1 + 1 + 1   # projections, 8 heads, top-t, profiles, 1 key block, merge, beta
+    ref = oracle.compact_pair(K, V, Q, Xr, W, cfg)
+    for k in ("anchors", "assign", "C_k", "beta", "C_v"):
+        assert np.array_equal(res[k], ref[k])
+
+
 def test_indexer_is_value_independent_with_zero_value_path():
     """App. A.1: with L_c = L_v = 0 the logits reproduce a query-key-only scorer."""
     w, K, V, Q, Xr, W = small_pair(zero_value_path=True)
