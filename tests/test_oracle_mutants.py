@@ -33,6 +33,9 @@ MUTANTS = [
     ("value_context_keys_for_values", "c = A @ (V @ U_v.T)", "c = A @ (K @ U_v.T)"),
     ("projection_drops_value_context", "Q @ W[\"L_q\"].T + c @ W[\"L_c\"].T", "Q @ W[\"L_q\"].T"),
     ("projection_drops_value_key_path", "K @ W[\"L_k\"].T + V @ W[\"L_v\"].T", "K @ W[\"L_k\"].T"),
+    ("key_blocks_not_normalised", "k_bar = rms_normalize(kz, d_I)", "k_bar = kz"),
+    ("query_blocks_normalised_over_heads", "q_bar = rms_normalize(qz, d_I)",
+     "q_bar = rms_normalize(qz.reshape(qz.shape[0], -1), d_I * qz.shape[1]).reshape(qz.shape)"),
     ("weights_drop_bias", "w = X_rows @ W[\"L_x\"].T + W[\"b_x\"][None, :]", "w = X_rows @ W[\"L_x\"].T"),
     ("leaky_slope_0_01", "x, 0.1 * x)", "x, 0.01 * x)"),
     ("leaky_sign_flipped", "np.where(x >= 0.0, x,", "np.where(x <= 0.0, x,"),
