@@ -1418,11 +1418,6 @@ __global__ void __launch_bounds__(256) phi_t_vec_kernel(const float* __restrict_
   if (r < t) w[(long long)b * t + r] = sum.hi + sum.lo;
 }
 
-template <typename R>
-__global__ void __launch_bounds__(512) tri_solve_kernel(const R* __restrict__ A, const R* __restrict__ Linv,
-                                                        const R* __restrict__ r, R* __restrict__ yd,
-                                                        R* __restrict__ x, int t);
-
 // Both substitutions of the single-right-hand-side dual beta system
 // L L^T x = r (the fp64 factor in A's lower triangle, Linv the inverses of its
 // 64 x 64 diagonal blocks) by a cluster of kTsCL CTAs per head: in each block
@@ -1838,7 +1833,7 @@ __global__ void __launch_bounds__(256) ir_cols_kernel(const float* __restrict__ 
 // x += (L L^T)^-1 r for one head per CTA (512 threads): forward substitution
 // y_k = Linv_kk (r_k - sum_{j<k} L_kj y_j), then x_k += Linv_kk^T (y_k -
 // sum_{j>k} L_jk^T d_j).  y and the correction d live in `yd` ([H][t]).
-// Also the single-right-hand-side solve of the fp64 dual beta system (x = 0).
+// Used by the refinement steps of the primal beta solve.
 template <typename R>
 __global__ void __launch_bounds__(512) tri_solve_kernel(const R* __restrict__ A, const R* __restrict__ Linv,
                                                         const R* __restrict__ r, R* __restrict__ yd,
