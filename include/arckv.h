@@ -23,7 +23,9 @@
  * ---------------------------------------
  * - Pointers named in the signatures are DEVICE pointers on the current CUDA
  *   device, owned by the caller; the library allocates no device or host
- *   memory.  Scratch space is the caller's workspace `ws` of at least the
+ *   memory (apart from the fixed array inside libarckv.so that
+ *   arckv_attend_static uses, described there).  Scratch space is the
+ *   caller's workspace `ws` of at least the
  *   size returned by the matching *_workspace_bytes function, aligned to
  *   256 bytes.
  * - Arguments are checked on the host before anything is enqueued; a bad
