@@ -302,6 +302,40 @@ def oracle_pair_seconds(w, pairs, selector="indexer", chunk_len=0):
     return times
 
 
+def gemm_rates(dev, reps: int = 5):
+    """Library GEMM rates of this GPU in the precisions the peak file does not
+    carry, timed like its bf16 figure (torch.matmul, best of `reps` after two
+    warm-up calls, CUDA events): fp64, fp32 on the SIMT pipes (tf32 off) and
+    tf32.  Measured outside every timed region; the denominators for the
+    fp64-grade solvers and for SIMT work."""
+    import torch
+    out = {}
+    prev = torch.backends.cuda.matmul.allow_tf32
+    try:
+        for name, dtype, size, tf32 in (("fp64", torch.float64, 4096, False), ("fp32_simt", torch.float32, 8192, False),
+                                        ("tf32", torch.float32, 8192, True)):
+            torch.backends.cuda.matmul.allow_tf32 = tf32
+            g = torch.Generator(device=dev).manual_seed(7)
+            a = torch.randn(size, size, device=dev, dtype=dtype, generator=g)
+            b = torch.randn(size, size, device=dev, dtype=dtype, generator=g)
+            best = float("inf")
+            for i in range(reps + 2):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                torch.matmul(a, b)
+                e1.record()
+                e1.synchronize()
+                if i >= 2:
+                    best = min(best, e0.elapsed_time(e1) / 1e3)
+            out[name] = 2.0 * size ** 3 / best / 1e12
+            del a, b
+    finally:
+        torch.backends.cuda.matmul.allow_tf32 = prev
+    out["how"] = ("torch.matmul (cuBLAS), 4096^3 fp64, 8192^3 fp32 with tf32 off and on; best of %d after 2 "
+                  "warm-up calls, CUDA events" % reps)
+    return out
+
+
 def profiled_traffic():
     """dram bytes per launch of the dominant kernel from the committed ncu
     summary, if it was taken on the current source of that kernel."""
@@ -588,13 +622,15 @@ def run_gpu(args, dist: Dist):
     m_sys = w.n if dual else tp
     solve_flops = {8: w.H_kv * (m_sys ** 3 / 3.0 + 2.0 * m_sys ** 2),
                    10: w.H_kv * (m_sys ** 3 / 3.0 + 4.0 * m_sys ** 2 * 128)}
+    rates = gemm_rates(dev)
     solver = {}
     for k, name in ((8, "beta_solve"), (10, "value_solve")):
         live = statistics.mean(stage_launch_ms[k]) / 1e3
         iso = statistics.median(iso_ms[k]) / 1e3
         solver[name] = {"flops": solve_flops[k], "ms_live": live * 1e3, "ms_isolated": iso * 1e3,
                         "tflops_isolated": solve_flops[k] / iso / 1e12,
-                        "frac_isolated": solve_flops[k] / iso / 1e12 / burst}
+                        "frac_isolated": solve_flops[k] / iso / 1e12 / burst,
+                        "vs_fp64_gemm": solve_flops[k] / iso / 1e12 / rates["fp64"]}
     roofline["solvers"] = dict(solver, kernel=("blocked Cholesky of the n x n dual systems: fp64 64 x 64 "
                                                "diagonal factors, 5-slice tensor-core block products "
                                                "(sliced_gemm_kernel<5>); the 4-slice Grams and back-projection "
@@ -602,7 +638,9 @@ def run_gpu(args, dist: Dist):
                                                "chol_cluster_kernel<float, 4|8> (tcgen05 trailing updates) "
                                                "+ two refinement steps"),
                                note="Cholesky m^3 / 3 plus the triangular solves (m = %d, 1 and 128 right-hand "
-                                    "sides), against the bf16 burst peak" % m_sys)
+                                    "sides), against the bf16 burst peak; vs_fp64_gemm against this GPU's own "
+                                    "fp64 GEMM rate (gemm_rates)" % m_sys)
+    roofline["gemm_rates"] = rates
 
     # end to end: pinned host inputs -> device -> compaction -> host outputs, every step
     pinned = [{k: v.to("cpu").pin_memory() for k, v in d.items()} for d in dev_in]
